@@ -1,0 +1,16 @@
+"""CPU oracle for ShallowStream query-time evidence retrieval.
+
+TEST INFRASTRUCTURE. Only tests/, __graft_entry__.smoke() and bench.py's CPU
+baseline (the cpu_baseline leg and the reference arm) may import or run anything in
+this package. The product path (the CUDA library and its Python binding) never
+imports it and shares no code with it.
+
+Plain, slow, fp64 numpy written from the paper's definitions:
+  retrieval.py  Eq. 3 (unit descriptor), Eq. 4 (recent/history split), Sec. 4.2
+                scored Q-K attention, Eq. 11 (per-layer top-M), unit votes, the
+                vote-ranked pool, max-min diversity, Eq. 12 (temporal expansion)
+  kmeans.py     token-level k-means compression of 20-frame windows and retrieval
+                over the centroids with member expansion (the cluster-compressed
+                index variant; closest paper text Sec. 4.1 Eq. 5-7 and Eq. 13)
+"""
+from . import retrieval, kmeans  # noqa: F401
