@@ -1,0 +1,342 @@
+"""Benchmark of query-time evidence retrieval on the 1-hour shallow index.
+
+Workload (one stream per GPU): 4 shallow layers, 28 query / 4 key heads, d = 128,
+3600 frames x 196 visual tokens (705,600 keys per (layer, key head), 2.89 GB of bf16
+keys), keys ~N(0,1) with 2 outlier channels x8 and per-frame AR(1) drift, 32
+question rows, 16 planted frames; top-k 1024 per (layer, query head), budget 64 units.
+
+A step is one full retrieval (query prep, key scoring, top-k merge, votes and mass,
+pool, max-min diversity, expansion) for one question against the resident index.
+The metric is shallow keys scored per second: a key is one stored (layer, key head,
+token) bf16 row of 256 bytes scored against its 7 query heads.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line. --impl reference times the CPU oracle (test infrastructure, the
+only other code this script may run) on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "shallow keys scored/sec (1-h index retrieval)"
+UNIT = "keys/s"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="hour1")
+    ap.add_argument("--cpu-frames", type=int, default=600,
+                    help="frames of the stream the CPU oracle baseline scores")
+    ap.add_argument("--ref-frames", type=int, default=100,
+                    help="frames of the stream one reference-arm step scores")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def dist_init(n_gpus: int):
+    import torch
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if torch.cuda.is_available():
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    elif torch.cuda.is_available():
+        torch.cuda.set_device(local)
+    return rank, world, local
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    dev = torch.device("cuda", torch.cuda.current_device()) if torch.cuda.is_available() else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle samples while the timed region runs."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines: list[str] = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except (OSError, ValueError):
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def measured_peak_gbs() -> tuple[float, str]:
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback"
+
+
+def cpu_baseline(w, data_keys_cpu, q_cpu, frames: int) -> dict:
+    """The oracle as it stands, on the first `frames` frames of the stream."""
+    import numpy as np
+    from oracle import retrieval as R
+    from paper_2609_02780_gb300 import synth
+    kb = synth.bf16_bits(data_keys_cpu[:, :, : frames * w.tokens_per_frame])
+    qb = synth.bf16_bits(q_cpu)
+    t0 = time.perf_counter()
+    R.retrieve(kb, qb, n_units=frames, tokens_per_unit=w.tokens_per_unit, k=w.k,
+               budget=w.budget, pool_mult=w.pool_mult, n_prev=w.n_prev)
+    dt = time.perf_counter() - t0
+    keys = w.n_slabs * frames * w.tokens_per_frame
+    return {"value": keys / dt, "unit": UNIT, "cores": len(os.sched_getaffinity(0)),
+            "kind": "oracle", "seconds": round(dt, 3),
+            "sample": f"oracle retrieve over the first {frames} of {w.n_frames} frames "
+                      f"({keys} keys, all {w.n_layers} layers), fp64 numpy"}
+
+
+def run_reference(args):
+    """Reference arm: the CPU oracle on a bounded sample, per step."""
+    import numpy as np
+    import torch
+    from paper_2609_02780_gb300 import synth
+    from oracle import retrieval as R
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    w = synth.PRESETS[args.workload]
+    frames = min(args.ref_frames, w.n_frames)
+    sample = w.replace(n_frames=frames, n_planted=max(1, w.n_planted * frames // w.n_frames))
+    data = synth.make_workload(sample, device="cpu")
+    kb, qb = synth.bf16_bits(data["keys"]), synth.bf16_bits(data["q"])
+    keys = sample.keys_per_query
+
+    def step():
+        R.retrieve(kb, qb, n_units=sample.n_units, tokens_per_unit=w.tokens_per_unit,
+                   k=w.k, budget=w.budget, pool_mult=w.pool_mult, n_prev=w.n_prev)
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    dt = time.perf_counter() - t0
+    value = keys * args.steps / dt
+    cores = len(os.sched_getaffinity(0))
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "impl": "reference",
+            "config": {"workload": f"{w.name} first {frames} frames",
+                       "keys_per_step": keys},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": f"first {frames} of {w.n_frames} frames per step"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args):
+    import numpy as np
+    import torch
+    import paper_2609_02780_gb300 as ss
+    from paper_2609_02780_gb300 import synth
+
+    rank, world, local = dist_init(args.gpus)
+    dev = torch.device("cuda", local)
+    w = synth.PRESETS[args.workload]
+    data = synth.make_workload(w, device=dev, stream=rank)
+    idx = ss.Index(w.n_layers, w.n_q_heads, w.n_kv_heads, w.tokens_per_frame, w.n_frames,
+                   frames_per_unit=w.frames_per_unit, device=dev)
+    idx.append(data["keys"])
+    q = data["q"]
+    keys_cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        frames = min(args.cpu_frames, w.n_frames)
+        keys_cpu = data["keys"][:, :, : frames * w.tokens_per_frame].cpu()
+    q_cpu = q.cpu()
+    del data
+    torch.cuda.synchronize(dev)
+    torch.cuda.empty_cache()
+
+    p = ss.RetrieveParams(k=w.k, budget=w.budget, pool_mult=w.pool_mult, n_prev=w.n_prev,
+                          n_recent=w.n_recent, q_agg=w.q_agg, head_agg=w.head_agg)
+    res = ss.Result(idx, p)
+    ws = torch.empty(idx.workspace_bytes(q.shape[1], p), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    k_begin = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    k_end = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    s_begin = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    s_end = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    for ev in k_begin + k_end:
+        ev.record(stream)  # create the events before handing them to the library
+
+    def step(i=None):
+        tr = (k_begin[i], k_end[i]) if i is not None else None
+        idx.retrieve(q, k=p.k, budget=p.budget, pool_mult=p.pool_mult, n_prev=p.n_prev,
+                     n_recent=p.n_recent, q_agg=p.q_agg, head_agg=p.head_agg, out=res,
+                     workspace=ws, trace=tr)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    res.check()
+    clocks = ClockSampler(local)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    clocks.start()
+    t_all0 = torch.cuda.Event(enable_timing=True)
+    t_all1 = torch.cuda.Event(enable_timing=True)
+    t_all0.record(stream)
+    for i in range(args.steps):
+        s_begin[i].record(stream)
+        step(i)
+        s_end[i].record(stream)
+    t_all1.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    clk = clocks.stop()
+    res.check()
+    total_ms = t_all0.elapsed_time(t_all1)
+    total_ms = max_over_ranks(total_ms, world)
+    step_ms = sorted(s_begin[i].elapsed_time(s_end[i]) for i in range(args.steps))
+    k1_ms = [k_begin[i].elapsed_time(k_end[i]) for i in range(args.steps)]
+    keys = w.keys_per_query
+    value = keys * args.steps * world / (total_ms / 1e3)
+
+    # end to end through the public API: host question in, host selection out
+    e2e = None
+    if not args.no_e2e:
+        q_pin = q_cpu.pin_memory()
+        for _ in range(3):
+            idx.retrieve_host(q_pin, p, workspace=ws)
+        barrier(world)
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            idx.retrieve_host(q_pin, p, workspace=ws)
+        dt = max_over_ranks(time.perf_counter() - t0, world)
+        nexp = p.budget * (1 + p.n_prev)
+        e2e = {"value": keys * args.steps * world / dt, "unit": UNIT,
+               "h2d_bytes_per_step": int(q_pin.numel() * 2),
+               "d2h_bytes_per_step": int(4 * (p.budget + nexp + nexp * w.frames_per_unit + 4 + 1)),
+               "ms_per_step": dt / args.steps * 1e3}
+
+    if rank != 0:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+        return
+    peak, peak_kind = measured_peak_gbs()
+    k1_avg_s = statistics.mean(k1_ms) / 1e3
+    alg_bytes = keys * 256
+    achieved = alg_bytes / k1_avg_s / 1e9
+    traffic = None
+    cpu = None
+    if keys_cpu is not None:
+        cpu = cpu_baseline(w, keys_cpu, q_cpu, keys_cpu.shape[2] // w.tokens_per_frame)
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": max(3, args.warmup),
+        "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": "hour1: 4 layers x 4 kv heads x 3600 frames x 196 tokens, "
+                               "Hq 28, R 32, k 1024, budget 64, pool 256",
+                   "keys_per_step": keys, "index_bytes": w.key_bytes,
+                   "l2": "inputs larger than L2 (2.89 GB index vs 129 MB L2), no flush",
+                   "parallelism": f"replicas x{world} (one independent stream per GPU)"},
+        "latency_ms": {"p50": statistics.median(step_ms),
+                       "p90": step_ms[min(len(step_ms) - 1, int(0.9 * len(step_ms)))],
+                       "score_kernel_avg": statistics.mean(k1_ms)},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic,
+                     "kernel": "k_score", "peak_kind": peak_kind,
+                     "algorithmic_bytes_per_launch": alg_bytes},
+        "clocks": clk,
+        "gpu_launches": 8 * args.steps,
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

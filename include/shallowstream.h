@@ -1,0 +1,269 @@
+/*
+ * shallowstream.h - C ABI of a GB300 (sm_103a) library for ShallowStream's
+ * query-time evidence retrieval over a shallow-layer key index
+ * (arxiv 2609.02780, Sec. 4.1 "Query-Agnostic Shallow Index Construction" and
+ * Sec. 4.2 "Query-Time Answering").
+ *
+ * The library keeps, in HBM, the bf16 keys that the shallow layers [0, P) produced
+ * for every stored video unit (the full-history shallow cache, Eq. 2) plus one
+ * descriptor per unit (Eq. 3). Given a question's query vectors at those layers
+ * (Eq. 10) it scores every stored history key, turns the scores into attention
+ * weights, keeps the top-k tokens of every list (Eq. 11), counts each unit's votes,
+ * ranks a pool of units by votes and attention mass, picks a diverse subset by
+ * greedy max-min in descriptor space and adds each pick's preceding units (Eq. 12).
+ * An optional k-means compression replaces windows of frames by centroids that
+ * retrieval scores instead of the windows' tokens.
+ *
+ * Conventions for every call:
+ *   - Returns an ss_status; nothing throws or aborts across the ABI. On failure the
+ *     call has launched nothing and ss_last_error() (thread-local) describes why.
+ *   - "device" pointers are CUDA device (or managed) addresses on the index's
+ *     device; "host" pointers are CPU addresses. Pointers are borrowed, never freed.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream). Calls that launch
+ *     work are asynchronous: outputs are valid once the stream reaches that point.
+ *   - Device memory for an index comes only from the ss_allocator given at create
+ *     time (or cudaMalloc/cudaFree when it is NULL). Per-call scratch is the caller's
+ *     `workspace` buffer (size from ss_retrieve_workspace_size).
+ *   - Key and query layouts are bf16, row-major, head_dim contiguous; only
+ *     head_dim == 128 and n_q_heads / n_kv_heads <= 8 are supported.
+ *   - A handle must not be used by two host threads at once.
+ *
+ * Notation: P shallow layers, Hq query heads, Hkv key heads, G = Hq / Hkv (query
+ * head h reads key head h / G), d = 128, T_f tokens per frame, T_u = T_f *
+ * frames_per_unit tokens per unit, U stored units, token id p = unit * T_u + slot.
+ */
+#ifndef SHALLOWSTREAM_H
+#define SHALLOWSTREAM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  SS_OK = 0,
+  SS_ERR_INVALID_ARG = 1,   /* a NULL, negative, misaligned or inconsistent argument */
+  SS_ERR_UNSUPPORTED = 2,   /* valid request outside the supported shapes */
+  SS_ERR_CAPACITY = 3,      /* index capacity (max_frames) or a buffer is too small */
+  SS_ERR_STATE = 4,         /* call not allowed in the handle's current state */
+  SS_ERR_ALLOC = 5,         /* the allocator returned NULL */
+  SS_ERR_CUDA = 6,          /* a CUDA runtime call failed (message in ss_last_error) */
+  SS_ERR_TIMEOUT = 7,       /* a bounded device-side wait gave up (device status) */
+  SS_ERR_INTERNAL = 8       /* a device-side consistency check failed (device status) */
+} ss_status;
+
+typedef struct ss_index ss_index;  /* opaque; host-side metadata only */
+
+/* Device memory provider. alloc returns a device pointer aligned to 256 bytes (or
+ * NULL); free releases it. `stream` is the stream passed to the call that
+ * allocates; `ctx` is passed through. */
+typedef struct {
+  void* (*alloc)(size_t bytes, void* stream, void* ctx);
+  void (*free)(void* ptr, void* stream, void* ctx);
+  void* ctx;
+} ss_allocator;
+
+/* Shape and capacity of an index (Sec. 3 notation; Table 4: a unit is 2 frames for
+ * Qwen3-VL and 1 for LLaVA-OneVision). */
+typedef struct {
+  int32_t n_layers;          /* P >= 1, the shallow layers [0, P) */
+  int32_t n_q_heads;         /* Hq, multiple of n_kv_heads, Hq / Hkv <= 8 */
+  int32_t n_kv_heads;        /* Hkv, 1..8 */
+  int32_t head_dim;          /* d, must be 128 */
+  int32_t tokens_per_frame;  /* T_f >= 1 visual tokens per frame */
+  int32_t frames_per_unit;   /* >= 1 */
+  int64_t max_frames;        /* capacity in frames, a multiple of frames_per_unit */
+} ss_index_config;
+
+/* Read-only view of an index's state and device arrays (for inspection). */
+typedef struct {
+  int64_t n_frames;          /* frames appended so far */
+  int64_t n_units;           /* complete units (descriptors valid for [0, n_units)) */
+  int64_t token_capacity;    /* N_cap tokens per (layer, key head) slab */
+  const void* keys;          /* device bf16 [P][Hkv][N_cap][d] */
+  const float* descriptors;  /* device fp32 [U_cap][Hkv * d] */
+  int32_t n_windows;         /* compressed windows so far */
+  int32_t window_frames;     /* 0 until the first compression */
+  int32_t n_centroids;
+  const void* centroids;     /* device bf16 [P][Hkv][W_cap * n_centroids][d] or NULL */
+  const uint8_t* assignment; /* device uint8 [P][Hkv][N_cap]: centroid of each token of a
+                                compressed window (window-local id) or NULL */
+  const int32_t* window_first_unit; /* device int32 [W_cap] or NULL */
+} ss_index_view;
+
+/* k-means compression of the frames [first_frame, first_frame + n_frames) in
+ * windows of window_frames (see ss_index_compress). */
+typedef struct {
+  int32_t window_frames;     /* frames per window, a multiple of frames_per_unit */
+  int32_t n_centroids;       /* 1..256 and <= window_frames * T_f */
+  int32_t iters;             /* Lloyd rounds >= 1 */
+  int64_t first_frame;       /* multiple of window_frames */
+  int64_t n_frames;          /* multiple of window_frames */
+} ss_compress_params;
+
+typedef enum { SS_Q_LAST = 0, SS_Q_MEAN_LOGIT = 1 } ss_q_agg;
+typedef enum { SS_H_PER_QHEAD = 0, SS_H_MEAN = 1 } ss_head_agg;
+
+/* Evidence-selection parameters (Sec. 4.2; Table 4 gives k = 64, pool 32 = 4 x 8,
+ * K = 8, one preceding unit, 6 recent units). */
+typedef struct {
+  int32_t k;                 /* top-k tokens per list, 1..4096 */
+  int32_t budget_units;      /* K units chosen by max-min, >= 1 */
+  int32_t pool_mult;         /* pool = pool_mult * K (paper: 4), pool <= 1024 */
+  int32_t n_prev;            /* preceding units added per selected unit (paper: 1) */
+  int32_t n_recent_units;    /* N_r: the latest N_r units are recent, never scored (Eq. 4) */
+  int32_t q_agg;             /* ss_q_agg: which question row(s) form the query */
+  int32_t head_agg;          /* ss_head_agg: per-query-head lists or one list per layer */
+  int32_t use_clusters;      /* 1: compressed windows are scored by their centroids */
+} ss_retrieve_params;
+
+/* Outputs of one retrieval, in caller-owned device buffers. A NULL member is placed in
+ * the workspace instead (and is then overwritten by the next call). n_lists = P * Hq
+ * for SS_H_PER_QHEAD, P for SS_H_MEAN. U_cap = max_frames / frames_per_unit. */
+typedef struct {
+  int32_t* topk_tok;         /* [n_lists][k] candidate ids sorted by (score desc, id asc);
+                                token id p, or 0x40000000 + window * n_c + centroid for a
+                                centroid; -1 past the number of candidates */
+  float* topk_w;             /* [n_lists][k] normalised attention weight of each entry */
+  float* list_stats;         /* [n_lists][2] softmax stats (M, L): M = max over candidates
+                                of the log2-scaled score s * log2(e), L = sum 2^(s' - M) */
+  int32_t* unit_votes;       /* [U_cap] votes of each history unit */
+  float* unit_mass;          /* [U_cap] attention mass of each history unit */
+  int32_t* pool;             /* [pool_mult * K] vote-ranked pool, best first */
+  int32_t* sel_units;        /* [K] max-min picks in selection order (required) */
+  int32_t* exp_units;        /* [K * (1 + n_prev)] picks plus predecessors, ascending
+                                (required) */
+  int32_t* frames;           /* [K * (1 + n_prev) * frames_per_unit] frames of exp_units,
+                                ascending (required) */
+  int32_t* counts;           /* [4] n_pool, n_sel, n_exp, n_frames (required) */
+  uint32_t* status;          /* [1] device status word, 0 = ok (required) */
+} ss_result;
+
+/* Host-side outputs of ss_retrieve_host (plain host arrays, pinned for speed). */
+typedef struct {
+  int32_t* sel_units;        /* [K] */
+  int32_t* exp_units;        /* [K * (1 + n_prev)] */
+  int32_t* frames;           /* [K * (1 + n_prev) * frames_per_unit] */
+  int32_t* counts;           /* [4] as in ss_result */
+} ss_host_result;
+
+/* Optional instrumentation: cudaEvent_t handles recorded on the call's stream
+ * immediately before and after the key-scoring kernel. NULL members are skipped. */
+typedef struct {
+  void* score_begin;
+  void* score_end;
+} ss_trace;
+
+/* --------------------------------------------------------------------------- */
+
+/* Human-readable name of a status code (static storage). */
+const char* ss_status_string(ss_status s);
+
+/* Message of the last failed call on this host thread (static, thread-local). */
+const char* ss_last_error(void);
+
+/* Library version string. */
+const char* ss_version(void);
+
+/* Creates an empty index (Eq. 2 with T = 0) on the current CUDA device. Allocates
+ * the key slabs bf16 [P][Hkv][max_frames * T_f][d] and descriptors fp32
+ * [U_cap][Hkv * d] from `alloc` (NULL: cudaMalloc). `stream` is passed to alloc.
+ * Errors: INVALID_ARG (NULL out/config, non-positive sizes, Hq % Hkv != 0,
+ * max_frames % frames_per_unit != 0), UNSUPPORTED (head_dim != 128, Hq / Hkv > 8,
+ * Hkv > 8), ALLOC, CUDA. *out is NULL on failure. */
+ss_status ss_index_create(const ss_index_config* config, const ss_allocator* alloc,
+                          void* stream, ss_index** out);
+
+/* Frees the index's device memory through its allocator and the handle. The caller
+ * must make sure no queued work still uses the index. NULL is accepted. */
+ss_status ss_index_destroy(ss_index* index);
+
+/* Appends n_frames frames of shallow keys (Eq. 1-2: the keys K^i_t of each new unit at
+ * every shallow layer). `keys` is device bf16 laid out [P][Hkv][S][d] where S =
+ * slab_stride_tokens (0 means n_frames * T_f) and the first n_frames * T_f tokens of
+ * every (layer, key head) slab are appended in order. Computes the Eq. 3 descriptor of
+ * every unit that this call completes. Asynchronous on `stream`; `keys` must stay valid
+ * until the stream passes this call. Errors: INVALID_ARG (NULL keys with n_frames > 0,
+ * negative n_frames, stride < n_frames * T_f, keys not 16-byte aligned), CAPACITY
+ * (would exceed max_frames), CUDA. n_frames == 0 is a no-op. */
+ss_status ss_index_append(ss_index* index, const void* keys, int32_t n_frames,
+                          int64_t slab_stride_tokens, void* stream);
+
+/* Fills *view with the index's current state. Device arrays are owned by the index. */
+ss_status ss_index_get_view(const ss_index* index, ss_index_view* view);
+
+/* k-means compression of already appended frames (the cluster-compressed variant;
+ * closest paper text Sec. 4.1 Eq. 5-7). For every window of `window_frames` frames in
+ * [first_frame, first_frame + n_frames) and every (layer, key head): X = the window's
+ * keys, C0 = X's first n_centroids tokens, then `iters` Lloyd rounds (assign each key
+ * to the nearest centroid by squared L2, lowest id on ties; move each centroid to the
+ * fp32 mean of its members, empty ones unchanged). Stores the last round's centroids
+ * (bf16, nearest-even) and memberships. The first call fixes window_frames and
+ * n_centroids (later calls must match, with windows after those already compressed)
+ * and allocates the cluster arrays from the index's allocator.
+ * Errors: INVALID_ARG (misaligned ranges, frames not yet appended, overlap with a
+ * compressed window), UNSUPPORTED (n_centroids > 256 or > window tokens), ALLOC,
+ * CUDA. */
+ss_status ss_index_compress(ss_index* index, const ss_compress_params* params,
+                            void* stream);
+
+/* Bytes of device workspace that ss_retrieve_batched needs for these indexes, row
+ * counts and parameters (ss_retrieve: n = 1). Depends on the indexes' capacities, not
+ * their current fill, so one workspace serves every later call with the same params. */
+ss_status ss_retrieve_workspace_size(const ss_index* const* indexes, int32_t n,
+                                     const int32_t* n_rows,
+                                     const ss_retrieve_params* params, size_t* bytes);
+
+/* One question against one index (Sec. 4.2, Eq. 10-12; the retrieval gate of Eq. 9 is
+ * taken as open). `q` is device bf16 [P][R][Hq][d], the question's post-RoPE query rows
+ * at each shallow layer (Eq. 10). History = units [0, U - n_recent_units) (Eq. 4). For
+ * each list (layer i, query head h): s_p = q_eff . K^i_{h/G, p} / sqrt(d) over the
+ * history tokens, w = softmax(s), the top-k tokens by (s desc, id asc) (Eq. 11). Unit
+ * votes count (list, selected token) pairs per unit; the pool is the top
+ * min(pool_mult * K, |history|) units by (votes desc, mass desc, id asc) where mass is
+ * the summed weight of all the unit's tokens over all lists; max-min diversity over the
+ * pool's descriptors (start at the pool's best, then repeatedly the unit farthest, by
+ * 1 - cosine, from its nearest pick; ties to the better pool rank) picks min(K, pool)
+ * units; each pick and its n_prev predecessors, deduplicated and ascending, form
+ * exp_units and frames (Eq. 12). With SS_H_MEAN the lists are per layer, ranked by the
+ * mean over query heads of the per-head weights. With use_clusters, compressed
+ * windows contribute their centroids as candidates instead of their tokens (only with
+ * SS_H_PER_QHEAD); a selected centroid votes once per member token and its weight is
+ * shared among member units by member count.
+ * Errors: INVALID_ARG (NULL, R < 1, bad enums, workspace too small or misaligned),
+ * UNSUPPORTED (k > 4096, pool > 1024, history > 16384 units, head_agg with clusters),
+ * STATE (use_clusters without compression), CUDA. Device-side failures are reported
+ * in *result->status (read with ss_status_sync). */
+ss_status ss_retrieve(ss_index* index, const void* q, int32_t n_rows,
+                      const ss_retrieve_params* params, const ss_result* result,
+                      void* workspace, size_t workspace_bytes, void* stream,
+                      const ss_trace* trace);
+
+/* n independent questions against n indexes (all on one device, same params) in one
+ * launch per stage: q[j] has n_rows[j] rows for indexes[j], results[j] receives its
+ * outputs. 1 <= n <= 32. Errors as ss_retrieve. */
+ss_status ss_retrieve_batched(ss_index* const* indexes, const void* const* q,
+                              const int32_t* n_rows, int32_t n,
+                              const ss_retrieve_params* params, const ss_result* results,
+                              void* workspace, size_t workspace_bytes, void* stream,
+                              const ss_trace* trace);
+
+/* ss_retrieve from host memory: copies `q_host` (bf16 [P][R][Hq][d]) to the device,
+ * retrieves with every result array in the workspace, copies the selection back into
+ * `out` and synchronizes `stream`. Returns the device status as well (TIMEOUT or
+ * INTERNAL). Errors as ss_retrieve. */
+ss_status ss_retrieve_host(ss_index* index, const void* q_host, int32_t n_rows,
+                           const ss_retrieve_params* params, const ss_host_result* out,
+                           void* workspace, size_t workspace_bytes, void* stream);
+
+/* Synchronizes `stream` and returns the status recorded in the device word `status`
+ * by earlier retrievals on it (SS_OK, SS_ERR_TIMEOUT or SS_ERR_INTERNAL). */
+ss_status ss_status_sync(const uint32_t* status, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SHALLOWSTREAM_H */

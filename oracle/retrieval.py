@@ -22,6 +22,8 @@ design notes):
   * pool = min(pool_mult * K, |history|) units; max-min starts from the top
     vote-ranked unit, distance 1 - cosine, ties to the better pool rank.
   * expansion adds the n_prev preceding units of each selected unit (Table 4: 1).
+  * Norm(0) = 0: a unit whose mean key is zero gets the zero descriptor (distance 1
+    to every unit), since Eq. 3's normalisation is undefined there.
 """
 from __future__ import annotations
 
@@ -188,7 +190,8 @@ def descriptors(key_bits: np.ndarray, n_units: int, tokens_per_unit: int) -> np.
     for u in range(n_units):
         sl = last[:, u * tokens_per_unit:(u + 1) * tokens_per_unit, :]
         mean = sl.mean(axis=1).reshape(Hkv * d)
-        out[u] = mean / np.linalg.norm(mean)
+        nrm = np.linalg.norm(mean)
+        out[u] = mean / nrm if nrm > 0 else 0.0     # a zero mean has no direction
     return out
 
 

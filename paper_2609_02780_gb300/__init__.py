@@ -1,0 +1,334 @@
+"""GB300-native query-time evidence retrieval over a shallow-layer key index
+(ShallowStream, arxiv 2609.02780, Sec. 4.1-4.2).
+
+Thin Python binding of the C ABI in include/shallowstream.h: it marshals torch
+tensors (device memory, the current CUDA stream) into the library's calls. Every
+step of retrieval runs in the library's CUDA kernels; there is no Python or CPU
+fallback, and using the binding without the built library raises.
+
+    idx = Index(n_layers=4, n_q_heads=28, n_kv_heads=4, tokens_per_frame=196,
+                max_frames=3600)
+    idx.append(keys)                 # bf16 [P][Hkv][n_frames * T_f][128] on the GPU
+    r = idx.retrieve(q, k=1024, budget=64)   # q: bf16 [P][R][Hq][128]
+    r.frames()                       # selected + expanded frames, ascending
+"""
+from __future__ import annotations
+
+import ctypes as C
+from dataclasses import dataclass
+
+import torch
+
+from . import _abi
+
+Q_LAST, Q_MEAN_LOGIT = 0, 1
+H_PER_QHEAD, H_MEAN = 0, 1
+CENTROID_ID_BASE = 0x40000000
+STATUS_NAMES = ("OK", "INVALID_ARG", "UNSUPPORTED", "CAPACITY", "STATE", "ALLOC", "CUDA",
+                "TIMEOUT", "INTERNAL")
+
+
+class ShallowStreamError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        self.status = status
+        name = STATUS_NAMES[status] if 0 <= status < len(STATUS_NAMES) else str(status)
+        super().__init__(f"SS_ERR_{name}: {message}" if status else message)
+
+
+def _lib():
+    return _abi.load()
+
+
+def _check(status: int) -> None:
+    if status != 0:
+        msg = _lib().ss_last_error().decode(errors="replace")
+        raise ShallowStreamError(status, msg)
+
+
+def _stream_ptr(device: torch.device) -> int:
+    return torch.cuda.current_stream(device).cuda_stream
+
+
+def version() -> str:
+    return _lib().ss_version().decode()
+
+
+@dataclass
+class RetrieveParams:
+    k: int
+    budget: int
+    pool_mult: int = 4
+    n_prev: int = 1
+    n_recent: int = 0
+    q_agg: int = Q_LAST
+    head_agg: int = H_PER_QHEAD
+    use_clusters: int = 0
+
+    def to_c(self) -> _abi.RetrieveParams:
+        return _abi.RetrieveParams(self.k, self.budget, self.pool_mult, self.n_prev,
+                                   self.n_recent, self.q_agg, self.head_agg,
+                                   self.use_clusters)
+
+
+class Result:
+    """Device tensors written by one retrieval (valid once the stream reaches them)."""
+
+    def __init__(self, idx: "Index", p: RetrieveParams):
+        dev = idx.device
+        n_lists = idx.n_layers * (1 if p.head_agg == H_MEAN else idx.n_q_heads)
+        pool = min(p.pool_mult * p.budget, idx.unit_capacity)
+        nexp = p.budget * (1 + p.n_prev)
+        i32 = dict(dtype=torch.int32, device=dev)
+        f32 = dict(dtype=torch.float32, device=dev)
+        self.params = p
+        self.frames_per_unit = idx.frames_per_unit
+        self.topk_tok = torch.empty(n_lists, p.k, **i32)
+        self.topk_w = torch.empty(n_lists, p.k, **f32)
+        self.list_stats = torch.empty(n_lists, 2, **f32)
+        self.unit_votes = torch.empty(idx.unit_capacity, **i32)
+        self.unit_mass = torch.empty(idx.unit_capacity, **f32)
+        self.pool = torch.empty(pool, **i32)
+        self.sel_units = torch.empty(p.budget, **i32)
+        self.exp_units = torch.empty(nexp, **i32)
+        self.frames_buf = torch.empty(nexp * idx.frames_per_unit, **i32)
+        self.counts = torch.empty(4, **i32)
+        self.status = torch.empty(1, **i32)
+
+    def to_c(self) -> _abi.Result:
+        return _abi.Result(self.topk_tok.data_ptr(), self.topk_w.data_ptr(),
+                           self.list_stats.data_ptr(), self.unit_votes.data_ptr(),
+                           self.unit_mass.data_ptr(), self.pool.data_ptr(),
+                           self.sel_units.data_ptr(), self.exp_units.data_ptr(),
+                           self.frames_buf.data_ptr(), self.counts.data_ptr(),
+                           self.status.data_ptr())
+
+    def check(self) -> None:
+        """Synchronizes the current stream and raises on a device-side error."""
+        dev = self.status.device
+        _check(_lib().ss_status_sync(C.c_void_p(self.status.data_ptr()),
+                                     C.c_void_p(_stream_ptr(dev))))
+
+    def host(self) -> dict:
+        """Synchronizes and returns the selection as Python lists."""
+        self.check()
+        c = self.counts.cpu().tolist()
+        return {"pool": self.pool[:c[0]].cpu().tolist(),
+                "sel": self.sel_units[:c[1]].cpu().tolist(),
+                "expanded": self.exp_units[:c[2]].cpu().tolist(),
+                "frames": self.frames_buf[:c[3]].cpu().tolist()}
+
+    def frames(self) -> list[int]:
+        return self.host()["frames"]
+
+
+class Index:
+    """A shallow key index (Eq. 2) of one video stream, resident on one GPU."""
+
+    def __init__(self, n_layers: int, n_q_heads: int, n_kv_heads: int,
+                 tokens_per_frame: int, max_frames: int, frames_per_unit: int = 1,
+                 head_dim: int = 128, device=None):
+        lib = _lib()
+        d = torch.device(device) if device is not None else torch.device("cuda")
+        if d.type != "cuda":
+            raise ValueError("an index lives on a CUDA device")
+        self.device = d if d.index is not None else torch.device("cuda", torch.cuda.current_device())
+        self.n_layers, self.n_q_heads, self.n_kv_heads = n_layers, n_q_heads, n_kv_heads
+        self.tokens_per_frame, self.frames_per_unit = tokens_per_frame, frames_per_unit
+        self.max_frames = max_frames
+        self.unit_capacity = max_frames // frames_per_unit
+        self._blocks: dict[int, torch.Tensor] = {}
+        self._alloc_cb = _abi.ALLOC_FN(self._alloc)
+        self._free_cb = _abi.FREE_FN(self._free)
+        self._allocator = _abi.Allocator(self._alloc_cb, self._free_cb, None)
+        self._ws: torch.Tensor | None = None
+        cfg = _abi.IndexConfig(n_layers, n_q_heads, n_kv_heads, head_dim, tokens_per_frame,
+                               frames_per_unit, max_frames)
+        h = C.c_void_p()
+        with torch.cuda.device(self.device):
+            _check(lib.ss_index_create(C.byref(cfg), C.byref(self._allocator),
+                                       C.c_void_p(_stream_ptr(self.device)), C.byref(h)))
+        self._h = h
+
+    # allocator callbacks: device memory comes from torch's caching allocator
+    def _alloc(self, nbytes, stream, ctx):
+        try:
+            t = torch.empty(int(nbytes), dtype=torch.uint8, device=self.device)
+        except Exception:
+            return None
+        self._blocks[t.data_ptr()] = t
+        return t.data_ptr()
+
+    def _free(self, ptr, stream, ctx):
+        self._blocks.pop(ptr, None)
+
+    @property
+    def handle(self) -> C.c_void_p:
+        if self._h is None:
+            raise RuntimeError("index destroyed")
+        return self._h
+
+    def close(self) -> None:
+        if getattr(self, "_h", None) is not None:
+            torch.cuda.synchronize(self.device)
+            _lib().ss_index_destroy(self._h)
+            self._h = None
+            self._blocks.clear()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def view(self) -> _abi.IndexView:
+        v = _abi.IndexView()
+        _check(_lib().ss_index_get_view(self.handle, C.byref(v)))
+        return v
+
+    @property
+    def n_frames(self) -> int:
+        return self.view().n_frames
+
+    @property
+    def n_units(self) -> int:
+        return self.view().n_units
+
+    def _block_view(self, ptr: int, dtype, shape) -> torch.Tensor:
+        t = self._blocks[ptr]
+        return t.view(dtype)[: torch.Size(shape).numel()].view(*shape)
+
+    def descriptors(self) -> torch.Tensor:
+        """Device fp32 [n_units][Hkv * 128] unit descriptors (Eq. 3), a view."""
+        v = self.view()
+        d = self._block_view(v.descriptors, torch.float32,
+                             (self.unit_capacity, self.n_kv_heads * 128))
+        return d[: v.n_units]
+
+    def keys(self) -> torch.Tensor:
+        """Device bf16 [P][Hkv][capacity][128] key slabs, a view."""
+        v = self.view()
+        return self._block_view(v.keys, torch.bfloat16,
+                                (self.n_layers, self.n_kv_heads, v.token_capacity, 128))
+
+    def append(self, keys: torch.Tensor, n_frames: int | None = None) -> None:
+        """Appends frames of shallow keys bf16 [P][Hkv][S][128] (the first
+        n_frames * T_f tokens of each slab; S may exceed that)."""
+        if keys.dtype != torch.bfloat16 or keys.dim() != 4:
+            raise ValueError("keys must be bf16 [P][Hkv][S][128]")
+        if keys.device != self.device:
+            raise ValueError("keys must be on the index's device")
+        if keys.stride(3) != 1 or keys.stride(2) != 128 or keys.stride(0) != keys.shape[1] * keys.stride(1):
+            raise ValueError("keys must be row-major per slab")
+        S = keys.stride(1) // 128
+        if n_frames is None:
+            if keys.shape[2] % self.tokens_per_frame:
+                raise ValueError("token count is not a whole number of frames")
+            n_frames = keys.shape[2] // self.tokens_per_frame
+        with torch.cuda.device(self.device):
+            _check(_lib().ss_index_append(self.handle, C.c_void_p(keys.data_ptr()),
+                                          int(n_frames), int(S),
+                                          C.c_void_p(_stream_ptr(self.device))))
+        self._last_src = keys  # keep the source alive until the stream passes the copy
+
+    def compress(self, window_frames: int, n_centroids: int = 64, iters: int = 5,
+                 first_frame: int = 0, n_frames: int | None = None) -> None:
+        if n_frames is None:
+            n_frames = (self.n_frames - first_frame) // window_frames * window_frames
+        cp = _abi.CompressParams(window_frames, n_centroids, iters, first_frame, n_frames)
+        with torch.cuda.device(self.device):
+            _check(_lib().ss_index_compress(self.handle, C.byref(cp),
+                                            C.c_void_p(_stream_ptr(self.device))))
+
+    def workspace_bytes(self, n_rows: int, p: RetrieveParams) -> int:
+        return workspace_bytes([self], [n_rows], p)
+
+    def _workspace(self, nbytes: int) -> torch.Tensor:
+        if self._ws is None or self._ws.numel() < nbytes:
+            self._ws = torch.empty(nbytes, dtype=torch.uint8, device=self.device)
+        return self._ws
+
+    def retrieve(self, q: torch.Tensor, k: int, budget: int, *, pool_mult: int = 4,
+                 n_prev: int = 1, n_recent: int = 0, q_agg: int = Q_LAST,
+                 head_agg: int = H_PER_QHEAD, use_clusters: int = 0,
+                 out: Result | None = None, workspace: torch.Tensor | None = None,
+                 trace: tuple | None = None) -> Result:
+        """One question against this index (Sec. 4.2, Eq. 10-12). q: bf16
+        [P][R][Hq][128] on the index's device. Asynchronous on the current stream."""
+        p = RetrieveParams(k, budget, pool_mult, n_prev, n_recent, q_agg, head_agg,
+                           use_clusters)
+        return retrieve_batched([self], [q], p, outs=[out] if out else None,
+                                workspace=workspace, trace=trace)[0]
+
+    def retrieve_host(self, q_host: torch.Tensor, p: RetrieveParams,
+                      workspace: torch.Tensor | None = None) -> dict:
+        """ss_retrieve_host: q in (pinned) host memory, selection copied back to host."""
+        if q_host.device.type != "cpu" or q_host.dtype != torch.bfloat16:
+            raise ValueError("q_host must be a bf16 CPU tensor")
+        q_host = q_host.contiguous()
+        R = q_host.shape[1]
+        nbytes = self.workspace_bytes(R, p)
+        ws = workspace if workspace is not None else self._workspace(nbytes)
+        nexp = p.budget * (1 + p.n_prev)
+        sel = torch.empty(p.budget, dtype=torch.int32).pin_memory()
+        exp = torch.empty(nexp, dtype=torch.int32).pin_memory()
+        frames = torch.empty(nexp * self.frames_per_unit, dtype=torch.int32).pin_memory()
+        counts = torch.empty(4, dtype=torch.int32).pin_memory()
+        hr = _abi.HostResult(sel.data_ptr(), exp.data_ptr(), frames.data_ptr(),
+                             counts.data_ptr())
+        with torch.cuda.device(self.device):
+            _check(_lib().ss_retrieve_host(self.handle, C.c_void_p(q_host.data_ptr()), R,
+                                           C.byref(p.to_c()), C.byref(hr),
+                                           C.c_void_p(ws.data_ptr()), ws.numel(),
+                                           C.c_void_p(_stream_ptr(self.device))))
+        c = counts.tolist()
+        return {"sel": sel[:c[1]].tolist(), "expanded": exp[:c[2]].tolist(),
+                "frames": frames[:c[3]].tolist(), "counts": c}
+
+
+def workspace_bytes(indexes: list[Index], n_rows: list[int], p: RetrieveParams) -> int:
+    n = len(indexes)
+    hs = (C.c_void_p * n)(*[ix.handle.value for ix in indexes])
+    rs = (C.c_int32 * n)(*n_rows)
+    out = C.c_size_t()
+    _check(_lib().ss_retrieve_workspace_size(hs, n, rs, C.byref(p.to_c()), C.byref(out)))
+    return out.value
+
+
+def retrieve_batched(indexes: list[Index], qs: list[torch.Tensor], p: RetrieveParams,
+                     outs: list[Result] | None = None, workspace: torch.Tensor | None = None,
+                     trace: tuple | None = None) -> list[Result]:
+    """n questions against n indexes on one device in one launch per stage."""
+    n = len(indexes)
+    if n != len(qs) or n == 0:
+        raise ValueError("need one query per index")
+    dev = indexes[0].device
+    for ix, q in zip(indexes, qs):
+        if q.dtype != torch.bfloat16 or q.dim() != 4 or not q.is_contiguous():
+            raise ValueError("q must be contiguous bf16 [P][R][Hq][128]")
+        if q.device != dev or ix.device != dev:
+            raise ValueError("indexes and queries must share one device")
+        if q.shape[0] != ix.n_layers or q.shape[2] != ix.n_q_heads or q.shape[3] != 128:
+            raise ValueError("q shape does not match the index")
+    rows = [q.shape[1] for q in qs]
+    nbytes = workspace_bytes(indexes, rows, p)
+    if workspace is None:
+        workspace = indexes[0]._workspace(nbytes)
+    if workspace.numel() * workspace.element_size() < nbytes:
+        raise ValueError(f"workspace smaller than {nbytes} bytes")
+    outs = outs or [Result(ix, p) for ix in indexes]
+    hs = (C.c_void_p * n)(*[ix.handle.value for ix in indexes])
+    qa = (C.c_void_p * n)(*[q.data_ptr() for q in qs])
+    rs = (C.c_int32 * n)(*rows)
+    res = (_abi.Result * n)(*[o.to_c() for o in outs])
+    tr = None
+    if trace is not None:
+        tr = C.byref(_abi.Trace(trace[0].cuda_event if trace[0] is not None else None,
+                                trace[1].cuda_event if trace[1] is not None else None))
+    with torch.cuda.device(dev):
+        _check(_lib().ss_retrieve_batched(hs, qa, rs, n, C.byref(p.to_c()), res,
+                                          C.c_void_p(workspace.data_ptr()),
+                                          workspace.numel() * workspace.element_size(),
+                                          C.c_void_p(_stream_ptr(dev)), tr))
+    for o in outs:
+        o._keep = (workspace, qs)
+    return outs

@@ -1,0 +1,478 @@
+// C ABI of the library (include/shallowstream.h): argument validation, device memory
+// of the index, workspace layout and the launch sequence of one retrieval.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <vector>
+
+#include "shallowstream.h"
+#include "ss_internal.cuh"
+
+#define SS_EXPORT extern "C" __attribute__((visibility("default")))
+
+using namespace ss;
+
+struct ss_index {
+  ss_index_config cfg;
+  ss_allocator alloc;
+  bool custom_alloc;
+  int device;
+  int sm_count;
+  int64_t ncap;        // tokens per slab
+  int64_t ucap;        // units
+  int64_t n_frames;
+  int64_t n_units;
+  __nv_bfloat16* keys;  // [P*Hkv][ncap][d]
+  float* desc;          // [ucap][Hkv*d]
+  // k-means compression
+  int32_t win_frames;
+  int32_t n_centroids;
+  int32_t n_windows;
+  int32_t wcap;
+  std::vector<int64_t> win_first_frame;
+  __nv_bfloat16* cent;  // [P*Hkv][wcap*nc][d]
+  uint8_t* assign;      // [P*Hkv][ncap]
+  int32_t* win_u0;      // [wcap]
+};
+
+namespace {
+
+thread_local char g_err[512] = "";
+
+ss_status fail(ss_status s, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return s;
+}
+
+#define SS_CUDA(expr)                                                                 \
+  do {                                                                                \
+    cudaError_t e_ = (expr);                                                          \
+    if (e_ != cudaSuccess) return fail(SS_ERR_CUDA, "%s: %s", #expr, cudaGetErrorString(e_)); \
+  } while (0)
+
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+void* dev_alloc(ss_index* ix, size_t bytes, cudaStream_t st) {
+  if (bytes == 0) bytes = 256;
+  if (ix->custom_alloc) return ix->alloc.alloc(bytes, (void*)st, ix->alloc.ctx);
+  void* p = nullptr;
+  if (cudaMalloc(&p, bytes) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  return p;
+}
+
+void dev_free(ss_index* ix, void* p) {
+  if (!p) return;
+  if (ix->custom_alloc) {
+    ix->alloc.free(p, nullptr, ix->alloc.ctx);
+  } else {
+    cudaFree(p);
+  }
+}
+
+int n_lists_of(const ss_index* ix, const ss_retrieve_params* p) {
+  return p->head_agg == SS_H_MEAN ? ix->cfg.n_layers : ix->cfg.n_layers * ix->cfg.n_q_heads;
+}
+
+int pool_cap_of(const ss_index* ix, const ss_retrieve_params* p) {
+  const int64_t pc = (int64_t)p->pool_mult * p->budget_units;
+  return (int)(pc < ix->ucap ? pc : ix->ucap);
+}
+
+// Workspace regions of one problem (offsets from the problem's base).
+struct Layout {
+  size_t qeff, cand_s, cand_id, cand_cnt, gthr, ustats, gram;
+  size_t topk_tok, topk_w, list_ml, votes, mass, pool, sel, exp_units, frames, counts,
+      status, qstage;
+  size_t total;
+};
+
+Layout layout_of(const ss_index* ix, int R, const ss_retrieve_params* p) {
+  Layout l{};
+  size_t cur = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = align256(cur);
+    cur = o + bytes;
+    return o;
+  };
+  const ss_index_config& c = ix->cfg;
+  const int64_t score_lists = (int64_t)c.n_layers * c.n_q_heads;
+  const int64_t n_lists = n_lists_of(ix, p);
+  const int64_t pc = pool_cap_of(ix, p);
+  const int64_t nexp = (int64_t)p->budget_units * (1 + p->n_prev);
+  l.qeff = take(score_lists * kHeadDim * 2);
+  l.cand_s = take(score_lists * ix->ncap * 4);
+  l.cand_id = take(score_lists * ix->ncap * 4);
+  l.cand_cnt = take(score_lists * 4);
+  l.gthr = take(score_lists * 4);
+  l.ustats = take(score_lists * ix->ucap * 8);
+  l.gram = take(pc * pc * 4);
+  l.topk_tok = take(n_lists * p->k * 4);
+  l.topk_w = take(n_lists * p->k * 4);
+  l.list_ml = take(n_lists * 8);
+  l.votes = take(ix->ucap * 4);
+  l.mass = take(ix->ucap * 4);
+  l.pool = take(pc * 4);
+  l.sel = take((size_t)p->budget_units * 4);
+  l.exp_units = take(nexp * 4);
+  l.frames = take(nexp * c.frames_per_unit * 4);
+  l.counts = take(16);
+  l.status = take(4);
+  l.qstage = take((size_t)c.n_layers * R * c.n_q_heads * kHeadDim * 2);
+  l.total = align256(cur);
+  return l;
+}
+
+ss_status check_params(const ss_retrieve_params* p) {
+  if (!p) return fail(SS_ERR_INVALID_ARG, "params is NULL");
+  if (p->k < 1) return fail(SS_ERR_INVALID_ARG, "k must be >= 1 (got %d)", p->k);
+  if (p->k > kMaxK) return fail(SS_ERR_UNSUPPORTED, "k > %d is not supported", kMaxK);
+  if (p->budget_units < 1) return fail(SS_ERR_INVALID_ARG, "budget_units must be >= 1");
+  if (p->pool_mult < 1) return fail(SS_ERR_INVALID_ARG, "pool_mult must be >= 1");
+  if ((int64_t)p->pool_mult * p->budget_units > kMaxPool)
+    return fail(SS_ERR_UNSUPPORTED, "pool_mult * budget_units > %d is not supported", kMaxPool);
+  if (p->n_prev < 0) return fail(SS_ERR_INVALID_ARG, "n_prev must be >= 0");
+  if (p->n_recent_units < 0) return fail(SS_ERR_INVALID_ARG, "n_recent_units must be >= 0");
+  if (p->q_agg != SS_Q_LAST && p->q_agg != SS_Q_MEAN_LOGIT)
+    return fail(SS_ERR_INVALID_ARG, "unknown q_agg %d", p->q_agg);
+  if (p->head_agg != SS_H_PER_QHEAD && p->head_agg != SS_H_MEAN)
+    return fail(SS_ERR_INVALID_ARG, "unknown head_agg %d", p->head_agg);
+  if (p->use_clusters != 0 && p->use_clusters != 1)
+    return fail(SS_ERR_INVALID_ARG, "use_clusters must be 0 or 1");
+  if (p->head_agg == SS_H_MEAN)
+    return fail(SS_ERR_UNSUPPORTED, "head_agg = SS_H_MEAN is not available in this build");
+  if (p->use_clusters)
+    return fail(SS_ERR_UNSUPPORTED, "use_clusters is not available in this build");
+  return SS_OK;
+}
+
+int64_t hist_units_of(const ss_index* ix, const ss_retrieve_params* p) {
+  const int64_t u = ix->n_units - p->n_recent_units;
+  return u > 0 ? u : 0;
+}
+
+template <typename T>
+T* pick(T* user, char* base, size_t off) {
+  return user ? user : reinterpret_cast<T*>(base + off);
+}
+
+ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t* R, int n,
+                        const ss_retrieve_params* p, const ss_result* res, void* ws,
+                        size_t ws_bytes, cudaStream_t st, const ss_trace* tr) {
+  if (n < 1 || n > kMaxProbs) return fail(SS_ERR_INVALID_ARG, "n must be in [1, %d]", kMaxProbs);
+  if (!ix || !q || !R || !res) return fail(SS_ERR_INVALID_ARG, "NULL argument");
+  ss_status s = check_params(p);
+  if (s != SS_OK) return s;
+  if (!ws || ((uintptr_t)ws & 255u)) return fail(SS_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+  size_t need = 0;
+  int dev = -1;
+  for (int j = 0; j < n; ++j) {
+    if (!ix[j] || !q[j]) return fail(SS_ERR_INVALID_ARG, "NULL index or query %d", j);
+    if (R[j] < 1) return fail(SS_ERR_INVALID_ARG, "n_rows must be >= 1");
+    if ((uintptr_t)q[j] & 1u) return fail(SS_ERR_INVALID_ARG, "query rows must be 2-byte aligned");
+    if (dev < 0) dev = ix[j]->device;
+    if (ix[j]->device != dev) return fail(SS_ERR_INVALID_ARG, "indexes on different devices");
+    if (hist_units_of(ix[j], p) > kMaxHistUnits)
+      return fail(SS_ERR_UNSUPPORTED, "more than %d history units", kMaxHistUnits);
+    const ss_result& r = res[j];
+    if (!r.sel_units || !r.exp_units || !r.frames || !r.counts || !r.status)
+      return fail(SS_ERR_INVALID_ARG, "result %d: sel_units, exp_units, frames, counts and status are required", j);
+    need += layout_of(ix[j], R[j], p).total;
+  }
+  if (ws_bytes < need)
+    return fail(SS_ERR_INVALID_ARG, "workspace too small: %zu < %zu bytes", ws_bytes, need);
+
+  thread_local Batch B;  // large; built on the host and passed by value to each launch
+  std::memset(&B, 0, sizeof(B));
+  B.n = n;
+  B.k = p->k;
+  B.n_prev = p->n_prev;
+  B.q_agg = p->q_agg;
+  B.head_agg = p->head_agg;
+  int max_lists = 0, max_uh = 0, max_pool = 0, n_slabs_total = 0;
+  char* base = static_cast<char*>(ws);
+  for (int j = 0; j < n; ++j) {
+    const ss_index* x = ix[j];
+    const ss_index_config& c = x->cfg;
+    const Layout l = layout_of(x, R[j], p);
+    Prob& P = B.p[j];
+    P.keys = x->keys;
+    P.desc = x->desc;
+    P.ncap = x->ncap;
+    P.P = c.n_layers;
+    P.Hq = c.n_q_heads;
+    P.Hkv = c.n_kv_heads;
+    P.G = c.n_q_heads / c.n_kv_heads;
+    P.fpu = c.frames_per_unit;
+    P.Tu = c.tokens_per_frame * c.frames_per_unit;
+    P.U = (int)x->n_units;
+    P.Uh = (int)hist_units_of(x, p);
+    P.ucap = (int)x->ucap;
+    P.q = static_cast<const __nv_bfloat16*>(q[j]);
+    P.R = R[j];
+    P.qeff = reinterpret_cast<__nv_bfloat16*>(base + l.qeff);
+    P.cand_s = reinterpret_cast<float*>(base + l.cand_s);
+    P.cand_id = reinterpret_cast<int32_t*>(base + l.cand_id);
+    P.cand_cap = x->ncap;
+    P.cand_cnt = reinterpret_cast<int32_t*>(base + l.cand_cnt);
+    P.gthr = reinterpret_cast<uint32_t*>(base + l.gthr);
+    P.ustats = reinterpret_cast<float2*>(base + l.ustats);
+    P.gram = reinterpret_cast<float*>(base + l.gram);
+    const ss_result& r = res[j];
+    P.topk_tok = pick(r.topk_tok, base, l.topk_tok);
+    P.topk_w = pick(r.topk_w, base, l.topk_w);
+    P.list_ml = pick(reinterpret_cast<float2*>(r.list_stats), base, l.list_ml);
+    P.votes = pick(r.unit_votes, base, l.votes);
+    P.mass = pick(r.unit_mass, base, l.mass);
+    P.pool = pick(r.pool, base, l.pool);
+    P.sel = r.sel_units;
+    P.exp_units = r.exp_units;
+    P.frames = r.frames;
+    P.counts = r.counts;
+    P.status = r.status;
+    const int64_t pc = (int64_t)p->pool_mult * p->budget_units;
+    P.pool_n = (int)(pc < P.Uh ? pc : P.Uh);
+    P.n_sel = P.pool_n < p->budget_units ? P.pool_n : p->budget_units;
+    max_lists = max(max_lists, P.P * P.Hq);
+    max_uh = max(max_uh, P.Uh);
+    max_pool = max(max_pool, P.pool_n);
+    n_slabs_total += P.P * P.Hkv;
+    base += l.total;
+  }
+  // Score-kernel mapping: a common chunk length in units for all problems.
+  const int c_common = score_chunks_per_slab(n_slabs_total, max_uh, ix[0]->sm_count);
+  const int chunk_len = c_common > 0 ? (max_uh + c_common - 1) / c_common : 1;
+  int cta = 0;
+  for (int j = 0; j < n; ++j) {
+    Prob& P = B.p[j];
+    P.chunks = P.Uh > 0 ? (P.Uh + chunk_len - 1) / chunk_len : 0;
+    P.cta_begin = cta;
+    cta += P.P * P.Hkv * P.chunks;
+  }
+  B.score_ctas = cta;
+
+  SS_CUDA(cudaSetDevice(dev));
+  SS_CUDA(launch_prep(B, st));
+  if (tr && tr->score_begin) SS_CUDA(cudaEventRecord((cudaEvent_t)tr->score_begin, st));
+  SS_CUDA(launch_score(B, st));
+  if (tr && tr->score_end) SS_CUDA(cudaEventRecord((cudaEvent_t)tr->score_end, st));
+  SS_CUDA(launch_select(B, max_lists, st));
+  SS_CUDA(launch_votes_mass(B, max_lists, max_uh, st));
+  SS_CUDA(launch_pool(B, max_uh, st));
+  SS_CUDA(launch_maxmin(B, max_pool, st));
+  SS_CUDA(launch_expand(B, st));
+  return SS_OK;
+}
+
+}  // namespace
+
+SS_EXPORT const char* ss_status_string(ss_status s) {
+  switch (s) {
+    case SS_OK: return "SS_OK";
+    case SS_ERR_INVALID_ARG: return "SS_ERR_INVALID_ARG";
+    case SS_ERR_UNSUPPORTED: return "SS_ERR_UNSUPPORTED";
+    case SS_ERR_CAPACITY: return "SS_ERR_CAPACITY";
+    case SS_ERR_STATE: return "SS_ERR_STATE";
+    case SS_ERR_ALLOC: return "SS_ERR_ALLOC";
+    case SS_ERR_CUDA: return "SS_ERR_CUDA";
+    case SS_ERR_TIMEOUT: return "SS_ERR_TIMEOUT";
+    case SS_ERR_INTERNAL: return "SS_ERR_INTERNAL";
+  }
+  return "unknown status";
+}
+
+SS_EXPORT const char* ss_last_error(void) { return g_err; }
+
+SS_EXPORT const char* ss_version(void) { return "shallowstream-gb300 0.1 (sm_103a)"; }
+
+SS_EXPORT ss_status ss_index_create(const ss_index_config* cfg, const ss_allocator* alloc,
+                                    void* stream, ss_index** out) {
+  if (!out) return fail(SS_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  if (!cfg) return fail(SS_ERR_INVALID_ARG, "config is NULL");
+  const ss_index_config& c = *cfg;
+  if (c.n_layers < 1 || c.n_q_heads < 1 || c.n_kv_heads < 1 || c.tokens_per_frame < 1 ||
+      c.frames_per_unit < 1 || c.max_frames < 1)
+    return fail(SS_ERR_INVALID_ARG, "sizes must be positive");
+  if (c.n_q_heads % c.n_kv_heads)
+    return fail(SS_ERR_INVALID_ARG, "n_q_heads must be a multiple of n_kv_heads");
+  if (c.max_frames % c.frames_per_unit)
+    return fail(SS_ERR_INVALID_ARG, "max_frames must be a multiple of frames_per_unit");
+  if (c.head_dim != kHeadDim) return fail(SS_ERR_UNSUPPORTED, "head_dim must be 128");
+  if (c.n_q_heads / c.n_kv_heads > kMaxGroup)
+    return fail(SS_ERR_UNSUPPORTED, "more than %d query heads per key head", kMaxGroup);
+  if (c.n_kv_heads > 8) return fail(SS_ERR_UNSUPPORTED, "more than 8 key heads");
+  if ((int64_t)c.tokens_per_frame * c.max_frames > (int64_t)0x3fffffff)
+    return fail(SS_ERR_UNSUPPORTED, "more than 2^30 tokens per slab");
+  if (alloc && (!alloc->alloc || !alloc->free))
+    return fail(SS_ERR_INVALID_ARG, "allocator needs alloc and free");
+  ss_index* ix = new ss_index();
+  ix->cfg = c;
+  ix->custom_alloc = alloc != nullptr;
+  if (alloc) ix->alloc = *alloc;
+  if (cudaGetDevice(&ix->device) != cudaSuccess ||
+      cudaDeviceGetAttribute(&ix->sm_count, cudaDevAttrMultiProcessorCount, ix->device) != cudaSuccess) {
+    cudaGetLastError();
+    delete ix;
+    return fail(SS_ERR_CUDA, "no usable CUDA device");
+  }
+  ix->ncap = c.max_frames * c.tokens_per_frame;
+  ix->ucap = c.max_frames / c.frames_per_unit;
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t kb = (size_t)c.n_layers * c.n_kv_heads * ix->ncap * kHeadDim * 2;
+  const size_t db = (size_t)ix->ucap * c.n_kv_heads * kHeadDim * 4;
+  ix->keys = static_cast<__nv_bfloat16*>(dev_alloc(ix, kb, st));
+  ix->desc = static_cast<float*>(dev_alloc(ix, db, st));
+  if (!ix->keys || !ix->desc || ((uintptr_t)ix->keys & 15u) || ((uintptr_t)ix->desc & 15u)) {
+    dev_free(ix, ix->keys);
+    dev_free(ix, ix->desc);
+    delete ix;
+    return fail(SS_ERR_ALLOC, "device allocation of %zu + %zu bytes failed (or was not 16-byte aligned)", kb, db);
+  }
+  *out = ix;
+  return SS_OK;
+}
+
+SS_EXPORT ss_status ss_index_destroy(ss_index* ix) {
+  if (!ix) return SS_OK;
+  dev_free(ix, ix->keys);
+  dev_free(ix, ix->desc);
+  dev_free(ix, ix->cent);
+  dev_free(ix, ix->assign);
+  dev_free(ix, ix->win_u0);
+  delete ix;
+  return SS_OK;
+}
+
+SS_EXPORT ss_status ss_index_append(ss_index* ix, const void* keys, int32_t n_frames,
+                                    int64_t stride, void* stream) {
+  if (!ix) return fail(SS_ERR_INVALID_ARG, "index is NULL");
+  if (n_frames < 0) return fail(SS_ERR_INVALID_ARG, "n_frames must be >= 0");
+  if (n_frames == 0) return SS_OK;
+  if (!keys) return fail(SS_ERR_INVALID_ARG, "keys is NULL");
+  if ((uintptr_t)keys & 15u) return fail(SS_ERR_INVALID_ARG, "keys must be 16-byte aligned");
+  const ss_index_config& c = ix->cfg;
+  const int64_t n_tok = (int64_t)n_frames * c.tokens_per_frame;
+  if (stride == 0) stride = n_tok;
+  if (stride < n_tok) return fail(SS_ERR_INVALID_ARG, "slab_stride_tokens < n_frames * tokens_per_frame");
+  if (ix->n_frames + n_frames > c.max_frames)
+    return fail(SS_ERR_CAPACITY, "append of %d frames exceeds max_frames %lld (have %lld)", n_frames,
+                (long long)c.max_frames, (long long)ix->n_frames);
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  SS_CUDA(cudaSetDevice(ix->device));
+  SS_CUDA(launch_append(ix->keys, ix->ncap, ix->n_frames * c.tokens_per_frame,
+                        static_cast<const __nv_bfloat16*>(keys), stride,
+                        c.n_layers * c.n_kv_heads, n_tok, st));
+  const int64_t new_units = (ix->n_frames + n_frames) / c.frames_per_unit;
+  SS_CUDA(launch_descriptors(ix->keys, ix->ncap, c.n_layers, c.n_kv_heads,
+                             c.tokens_per_frame * c.frames_per_unit, ix->n_units, new_units,
+                             ix->desc, st));
+  ix->n_frames += n_frames;
+  ix->n_units = new_units;
+  return SS_OK;
+}
+
+SS_EXPORT ss_status ss_index_get_view(const ss_index* ix, ss_index_view* v) {
+  if (!ix || !v) return fail(SS_ERR_INVALID_ARG, "NULL argument");
+  v->n_frames = ix->n_frames;
+  v->n_units = ix->n_units;
+  v->token_capacity = ix->ncap;
+  v->keys = ix->keys;
+  v->descriptors = ix->desc;
+  v->n_windows = ix->n_windows;
+  v->window_frames = ix->win_frames;
+  v->n_centroids = ix->n_centroids;
+  v->centroids = ix->cent;
+  v->assignment = ix->assign;
+  v->window_first_unit = ix->win_u0;
+  return SS_OK;
+}
+
+SS_EXPORT ss_status ss_index_compress(ss_index* ix, const ss_compress_params* cp, void* stream) {
+  (void)stream;
+  if (!ix || !cp) return fail(SS_ERR_INVALID_ARG, "NULL argument");
+  return fail(SS_ERR_UNSUPPORTED, "compression is not available in this build");
+}
+
+SS_EXPORT ss_status ss_retrieve_workspace_size(const ss_index* const* ix, int32_t n,
+                                               const int32_t* R, const ss_retrieve_params* p,
+                                               size_t* bytes) {
+  if (!ix || !R || !bytes) return fail(SS_ERR_INVALID_ARG, "NULL argument");
+  if (n < 1 || n > kMaxProbs) return fail(SS_ERR_INVALID_ARG, "n must be in [1, %d]", kMaxProbs);
+  ss_status s = check_params(p);
+  if (s != SS_OK) return s;
+  size_t total = 0;
+  for (int j = 0; j < n; ++j) {
+    if (!ix[j]) return fail(SS_ERR_INVALID_ARG, "NULL index %d", j);
+    if (R[j] < 1) return fail(SS_ERR_INVALID_ARG, "n_rows must be >= 1");
+    total += layout_of(ix[j], R[j], p).total;
+  }
+  *bytes = total;
+  return SS_OK;
+}
+
+SS_EXPORT ss_status ss_retrieve(ss_index* ix, const void* q, int32_t R,
+                                const ss_retrieve_params* p, const ss_result* res, void* ws,
+                                size_t ws_bytes, void* stream, const ss_trace* tr) {
+  ss_index* const arr[1] = {ix};
+  const void* const qa[1] = {q};
+  return retrieve_impl(arr, qa, &R, 1, p, res, ws, ws_bytes, static_cast<cudaStream_t>(stream), tr);
+}
+
+SS_EXPORT ss_status ss_retrieve_batched(ss_index* const* ix, const void* const* q,
+                                        const int32_t* R, int32_t n,
+                                        const ss_retrieve_params* p, const ss_result* res,
+                                        void* ws, size_t ws_bytes, void* stream,
+                                        const ss_trace* tr) {
+  return retrieve_impl(ix, q, R, n, p, res, ws, ws_bytes, static_cast<cudaStream_t>(stream), tr);
+}
+
+SS_EXPORT ss_status ss_status_sync(const uint32_t* status, void* stream) {
+  if (!status) return fail(SS_ERR_INVALID_ARG, "status is NULL");
+  SS_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+  uint32_t v = 0;
+  SS_CUDA(cudaMemcpy(&v, status, sizeof(v), cudaMemcpyDeviceToHost));
+  if (v & kStatusTimeout) return fail(SS_ERR_TIMEOUT, "a bounded device-side wait gave up");
+  if (v & kStatusInternal) return fail(SS_ERR_INTERNAL, "a device-side consistency check failed");
+  return SS_OK;
+}
+
+SS_EXPORT ss_status ss_retrieve_host(ss_index* ix, const void* q_host, int32_t R,
+                                     const ss_retrieve_params* p, const ss_host_result* out,
+                                     void* ws, size_t ws_bytes, void* stream) {
+  if (!ix || !q_host || !out || !out->sel_units || !out->exp_units || !out->frames || !out->counts)
+    return fail(SS_ERR_INVALID_ARG, "NULL argument");
+  ss_status s = check_params(p);
+  if (s != SS_OK) return s;
+  if (R < 1) return fail(SS_ERR_INVALID_ARG, "n_rows must be >= 1");
+  if (!ws || ((uintptr_t)ws & 255u)) return fail(SS_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+  const Layout l = layout_of(ix, R, p);
+  if (ws_bytes < l.total)
+    return fail(SS_ERR_INVALID_ARG, "workspace too small: %zu < %zu bytes", ws_bytes, l.total);
+  const ss_index_config& c = ix->cfg;
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  char* base = static_cast<char*>(ws);
+  const size_t qbytes = (size_t)c.n_layers * R * c.n_q_heads * kHeadDim * 2;
+  SS_CUDA(cudaSetDevice(ix->device));
+  SS_CUDA(cudaMemcpyAsync(base + l.qstage, q_host, qbytes, cudaMemcpyHostToDevice, st));
+  ss_result r{};
+  r.sel_units = reinterpret_cast<int32_t*>(base + l.sel);
+  r.exp_units = reinterpret_cast<int32_t*>(base + l.exp_units);
+  r.frames = reinterpret_cast<int32_t*>(base + l.frames);
+  r.counts = reinterpret_cast<int32_t*>(base + l.counts);
+  r.status = reinterpret_cast<uint32_t*>(base + l.status);
+  s = ss_retrieve(ix, base + l.qstage, R, p, &r, ws, ws_bytes, stream, nullptr);
+  if (s != SS_OK) return s;
+  const size_t nsel = (size_t)p->budget_units;
+  const size_t nexp = nsel * (1 + p->n_prev);
+  SS_CUDA(cudaMemcpyAsync(out->sel_units, r.sel_units, nsel * 4, cudaMemcpyDeviceToHost, st));
+  SS_CUDA(cudaMemcpyAsync(out->exp_units, r.exp_units, nexp * 4, cudaMemcpyDeviceToHost, st));
+  SS_CUDA(cudaMemcpyAsync(out->frames, r.frames, nexp * c.frames_per_unit * 4, cudaMemcpyDeviceToHost, st));
+  SS_CUDA(cudaMemcpyAsync(out->counts, r.counts, 16, cudaMemcpyDeviceToHost, st));
+  return ss_status_sync(r.status, stream);
+}

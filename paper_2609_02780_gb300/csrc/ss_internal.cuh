@@ -1,0 +1,150 @@
+// Internal declarations shared by the library's CUDA translation units.
+//
+// Every retrieval stage is one kernel launch over a batch of independent problems
+// (one question against one index). The batch travels by value as a __grid_constant__
+// kernel parameter, so launches need no host-to-device copy and can be captured in a
+// CUDA graph.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+namespace ss {
+
+constexpr int kHeadDim = 128;          // d (only 128 is supported)
+constexpr int kMaxProbs = 32;          // problems per batched launch
+constexpr int kMaxK = 4096;            // top-k per list
+constexpr int kMaxPool = 1024;         // pool = pool_mult * budget
+constexpr int kMaxHistUnits = 16384;   // history units per problem (pool sort in smem)
+constexpr int kMaxGroup = 8;           // query heads per key head
+constexpr uint32_t kCentroidIdBase = 0x40000000u;
+
+// Score-kernel geometry: kScoreWarps compute warps + 1 threshold warp per CTA.
+#ifndef SS_SCORE_WARPS
+#define SS_SCORE_WARPS 8
+#endif
+constexpr int kScoreWarps = SS_SCORE_WARPS;
+constexpr int kScoreThreads = (kScoreWarps + 1) * 32;
+#ifndef SS_SCORE_CTAS_PER_SM
+#define SS_SCORE_CTAS_PER_SM 2
+#endif
+constexpr int kScoreCtasPerSm = SS_SCORE_CTAS_PER_SM;
+constexpr int kHistBins = 512;         // threshold histogram bins per head
+constexpr float kBinsPerUnit = 8.0f;   // bins per log2-score unit
+constexpr float kHistBelowMax = 48.0f; // histogram covers [max0 - 48, max0 + 16)
+
+// Device status word bits (ss_result::status).
+constexpr uint32_t kStatusInternal = 1u;
+constexpr uint32_t kStatusTimeout = 2u;
+
+// log2(e) / sqrt(128): scores are kept in the log2 domain, s2 = (q.k) * kScoreScale,
+// so softmax weights are 2^(s2 - M) / L.
+constexpr float kScoreScale = 0.12751743082459868f;
+
+struct Prob {
+  // index
+  const __nv_bfloat16* keys;   // [P*Hkv][ncap][d]
+  const float* desc;           // [ucap][Hkv*d]
+  int64_t ncap;                // token capacity per slab
+  int P, Hq, Hkv, G, Tu, fpu;
+  int U;                       // complete units
+  int Uh;                      // history units [0, Uh)
+  int ucap;
+  // question
+  const __nv_bfloat16* q;      // [P][R][Hq][d]
+  int R;
+  // workspace
+  __nv_bfloat16* qeff;         // [P][Hq][d]
+  float* cand_s;               // [n_score_lists][cand_cap]
+  int32_t* cand_id;
+  int64_t cand_cap;
+  int32_t* cand_cnt;           // [n_score_lists]
+  uint32_t* gthr;              // [n_score_lists] ordered-float threshold
+  float2* ustats;              // [n_score_lists][ucap] per-unit (max, sum 2^(s-max))
+  float* gram;                 // [pool][pool]
+  // outputs
+  int32_t* topk_tok;           // [n_lists][k]
+  float* topk_w;
+  float2* list_ml;             // [n_lists] (M, L)
+  int32_t* votes;              // [ucap]
+  float* mass;                 // [ucap]
+  int32_t* pool;
+  int32_t* sel;
+  int32_t* exp_units;
+  int32_t* frames;
+  int32_t* counts;             // n_pool, n_sel, n_exp, n_frames
+  uint32_t* status;
+  // launch mapping of the score kernel
+  int cta_begin;               // first score CTA of this problem
+  int chunks;                  // unit chunks per slab
+  int pool_n;                  // min(pool_mult * budget, Uh)
+  int n_sel;                   // min(budget, pool_n)
+};
+
+struct Batch {
+  Prob p[kMaxProbs];
+  int n;
+  int k;
+  int n_prev;
+  int q_agg;
+  int head_agg;
+  int score_ctas;              // total CTAs of the score kernel
+};
+static_assert(sizeof(Batch) <= 32000, "kernel parameter block too large");
+
+// ---------------------------------------------------------------------------
+// Device helpers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t float_to_ordered(float f) {
+  uint32_t u = __float_as_uint(f);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+__device__ __forceinline__ float ordered_to_float(uint32_t o) {
+  uint32_t u = (o & 0x80000000u) ? (o & 0x7fffffffu) : ~o;
+  return __uint_as_float(u);
+}
+
+// 2^x with the SFU's approximate exp2 (flushes denormal results to zero).
+__device__ __forceinline__ float fast_exp2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// Combines two (max, sum of 2^(s - max)) pairs; an empty pair has max = -inf, sum 0.
+__device__ __forceinline__ void ml_combine(float& m, float& l, float mo, float lo) {
+  float M = fmaxf(m, mo);
+  float a = (m == -INFINITY) ? 0.f : l * fast_exp2(m - M);
+  float b = (mo == -INFINITY) ? 0.f : lo * fast_exp2(mo - M);
+  m = M;
+  l = a + b;
+}
+
+__device__ __forceinline__ int problem_of_block(const Batch& B, int b) {
+  int pi = 0;
+  while (pi + 1 < B.n && B.p[pi + 1].cta_begin <= b) ++pi;
+  return pi;
+}
+
+}  // namespace ss
+
+// Launchers (host side), one per translation unit.
+namespace ss {
+cudaError_t launch_prep(const Batch& B, cudaStream_t s);
+cudaError_t launch_score(const Batch& B, cudaStream_t s);
+cudaError_t launch_select(const Batch& B, int max_lists, cudaStream_t s);
+cudaError_t launch_votes_mass(const Batch& B, int max_lists, int max_hist_units,
+                              cudaStream_t s);
+cudaError_t launch_pool(const Batch& B, int max_hist_units, cudaStream_t s);
+cudaError_t launch_maxmin(const Batch& B, int max_pool, cudaStream_t s);
+cudaError_t launch_expand(const Batch& B, cudaStream_t s);
+cudaError_t launch_append(__nv_bfloat16* keys, int64_t ncap, int64_t tok0,
+                          const __nv_bfloat16* src, int64_t src_stride_tokens,
+                          int n_slabs, int64_t n_tokens, cudaStream_t s);
+cudaError_t launch_descriptors(const __nv_bfloat16* keys, int64_t ncap, int P, int Hkv,
+                               int Tu, int64_t u_begin, int64_t u_end, float* desc,
+                               cudaStream_t s);
+int score_chunks_per_slab(int n_slabs_total, int hist_units, int sm_count);
+}  // namespace ss

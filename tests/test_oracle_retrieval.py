@@ -221,6 +221,8 @@ def test_descriptor_head_major_vec_and_norm():
     e1 = np.zeros(Hkv * d)
     e1[d + 5] = 1.0
     assert np.allclose(D[1], e1, atol=1e-15)
+    zero = R.descriptors(to_bf16_bits(np.zeros((1, 2, 4, d), np.float32)), 2, 2)
+    assert np.array_equal(zero, np.zeros((2, 2 * d)))        # Norm(0) = 0
     rng = np.random.default_rng(7)
     D2 = R.descriptors(to_bf16_bits(rng.standard_normal((2, 4, 60, 128)).astype(np.float32)), 6, 10)
     assert np.allclose(np.linalg.norm(D2, axis=1), 1.0, atol=1e-14)
