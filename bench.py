@@ -44,6 +44,8 @@ def parse():
                     help="frames of the stream the CPU oracle baseline scores")
     ap.add_argument("--ref-frames", type=int, default=100,
                     help="frames of the stream one reference-arm step scores")
+    ap.add_argument("--frames", type=int, default=0,
+                    help="truncate the stream to this many frames (small profiling case)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args()
@@ -214,6 +216,9 @@ def run_ours(args):
     rank, world, local = dist_init(args.gpus)
     dev = torch.device("cuda", local)
     w = synth.PRESETS[args.workload]
+    if args.frames:
+        w = w.replace(n_frames=args.frames,
+                      n_planted=max(1, w.n_planted * args.frames // w.n_frames))
     data = synth.make_workload(w, device=dev, stream=rank)
     idx = ss.Index(w.n_layers, w.n_q_heads, w.n_kv_heads, w.tokens_per_frame, w.n_frames,
                    frames_per_unit=w.frames_per_unit, device=dev)
@@ -307,10 +312,13 @@ def run_ours(args):
         "steps": args.steps, "warmup": max(3, args.warmup),
         "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": "hour1: 4 layers x 4 kv heads x 3600 frames x 196 tokens, "
-                               "Hq 28, R 32, k 1024, budget 64, pool 256",
+        "config": {"workload": f"{w.name}: {w.n_layers} layers x {w.n_kv_heads} kv heads x "
+                               f"{w.n_frames} frames x {w.tokens_per_frame} tokens, "
+                               f"Hq {w.n_q_heads}, R {w.n_rows}, k {w.k}, budget {w.budget}, "
+                               f"pool {w.pool_mult * w.budget}",
                    "keys_per_step": keys, "index_bytes": w.key_bytes,
-                   "l2": "inputs larger than L2 (2.89 GB index vs 129 MB L2), no flush",
+                   "l2": f"inputs larger than L2 ({w.key_bytes / 1e9:.2f} GB index vs "
+                         f"129 MB L2), no flush",
                    "parallelism": f"replicas x{world} (one independent stream per GPU)"},
         "latency_ms": {"p50": statistics.median(step_ms),
                        "p90": step_ms[min(len(step_ms) - 1, int(0.9 * len(step_ms)))],

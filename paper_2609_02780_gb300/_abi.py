@@ -97,7 +97,7 @@ def load(path: str | None = None) -> C.CDLL:
     global _LIB
     if _LIB is not None and path is None:
         return _LIB
-    p = path or _build.LIB
+    p = path or os.environ.get("SHALLOWSTREAM_LIB") or _build.LIB
     if not os.path.exists(p):
         raise RuntimeError(f"CUDA library not built ({p} missing): run "
                            "paper_2609_02780_gb300.build.build() or __graft_entry__.build()")

@@ -84,9 +84,15 @@ int pool_cap_of(const ss_index* ix, const ss_retrieve_params* p) {
   return (int)(pc < ix->ucap ? pc : ix->ucap);
 }
 
+// Candidate slots per list: every token once, plus the unused tails of the slot
+// blocks that score warps reserve.
+int64_t cand_cap_of(const ss_index* ix) {
+  return ix->ncap + (int64_t)kMaxChunksPerSlab * kScoreWarps * kReserve;
+}
+
 // Workspace regions of one problem (offsets from the problem's base).
 struct Layout {
-  size_t qeff, cand_s, cand_id, cand_cnt, gthr, ustats, gram;
+  size_t qeff, cand_s, cand_id, cand_cnt, gthr, ladder, anchor, ustats, gram;
   size_t topk_tok, topk_w, list_ml, votes, mass, pool, sel, exp_units, frames, counts,
       status, qstage;
   size_t total;
@@ -106,10 +112,12 @@ Layout layout_of(const ss_index* ix, int R, const ss_retrieve_params* p) {
   const int64_t pc = pool_cap_of(ix, p);
   const int64_t nexp = (int64_t)p->budget_units * (1 + p->n_prev);
   l.qeff = take(score_lists * kHeadDim * 2);
-  l.cand_s = take(score_lists * ix->ncap * 4);
-  l.cand_id = take(score_lists * ix->ncap * 4);
+  l.cand_s = take(score_lists * cand_cap_of(ix) * 4);
+  l.cand_id = take(score_lists * cand_cap_of(ix) * 4);
   l.cand_cnt = take(score_lists * 4);
   l.gthr = take(score_lists * 4);
+  l.ladder = take(score_lists * kLadderLevels * 4);
+  l.anchor = take(score_lists * 4);
   l.ustats = take(score_lists * ix->ucap * 8);
   l.gram = take(pc * pc * 4);
   l.topk_tok = take(n_lists * p->k * 4);
@@ -218,9 +226,11 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
     P.qeff = reinterpret_cast<__nv_bfloat16*>(base + l.qeff);
     P.cand_s = reinterpret_cast<float*>(base + l.cand_s);
     P.cand_id = reinterpret_cast<int32_t*>(base + l.cand_id);
-    P.cand_cap = x->ncap;
+    P.cand_cap = cand_cap_of(x);
     P.cand_cnt = reinterpret_cast<int32_t*>(base + l.cand_cnt);
     P.gthr = reinterpret_cast<uint32_t*>(base + l.gthr);
+    P.ladder = reinterpret_cast<int32_t*>(base + l.ladder);
+    P.anchor = reinterpret_cast<float*>(base + l.anchor);
     P.ustats = reinterpret_cast<float2*>(base + l.ustats);
     P.gram = reinterpret_cast<float*>(base + l.gram);
     const ss_result& r = res[j];
@@ -245,7 +255,11 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
     base += l.total;
   }
   // Score-kernel mapping: a common chunk length in units for all problems.
+#ifdef SS_FORCE_CHUNKS
+  const int c_common = max_uh > 0 ? min(SS_FORCE_CHUNKS, max_uh) : 0;
+#else
   const int c_common = score_chunks_per_slab(n_slabs_total, max_uh, ix[0]->sm_count);
+#endif
   const int chunk_len = c_common > 0 ? (max_uh + c_common - 1) / c_common : 1;
   int cta = 0;
   for (int j = 0; j < n; ++j) {

@@ -30,9 +30,23 @@ constexpr int kScoreThreads = (kScoreWarps + 1) * 32;
 #define SS_SCORE_CTAS_PER_SM 2
 #endif
 constexpr int kScoreCtasPerSm = SS_SCORE_CTAS_PER_SM;
-constexpr int kHistBins = 512;         // threshold histogram bins per head
-constexpr float kBinsPerUnit = 8.0f;   // bins per log2-score unit
-constexpr float kHistBelowMax = 48.0f; // histogram covers [max0 - 48, max0 + 16)
+#ifndef SS_SCORE_STAGES
+#define SS_SCORE_STAGES 3
+#endif
+constexpr int kScoreStages = SS_SCORE_STAGES;  // bulk-copy stages per compute warp
+constexpr int kTileRows = 16;                  // key rows per stage (one MMA tile)
+constexpr int kTileBytes = kTileRows * kHeadDim * 2;
+// Threshold ladder of each list: level i counts appended scores in
+// [A + (i - kLadderZero) / kLadderPerUnit, + 1 / kLadderPerUnit) where A is the list's
+// anchor (largest score of a small key sample); the top level also takes everything
+// above. kLadderLevels levels span [A - 12, A + 4) log2 units.
+constexpr int kLadderLevels = 256;
+constexpr int kLadderZero = 192;
+constexpr float kLadderPerUnit = 16.0f;
+constexpr int kSampleUnits = 4;        // units scored for the anchor
+// Candidate slots a warp reserves per list at a time (no atomic per append).
+constexpr int kReserve = 64;
+constexpr int kMaxChunksPerSlab = 128;
 
 // Device status word bits (ss_result::status).
 constexpr uint32_t kStatusInternal = 1u;
@@ -61,6 +75,8 @@ struct Prob {
   int64_t cand_cap;
   int32_t* cand_cnt;           // [n_score_lists]
   uint32_t* gthr;              // [n_score_lists] ordered-float threshold
+  int32_t* ladder;             // [n_score_lists][kLadderLevels] appended-score counts
+  float* anchor;               // [n_score_lists] ladder anchor A (log2 units)
   float2* ustats;              // [n_score_lists][ucap] per-unit (max, sum 2^(s-max))
   float* gram;                 // [pool][pool]
   // outputs

@@ -21,6 +21,8 @@ namespace ss {
 // the rows' mean (fp32 sum in row order, divided by R, rounded to bf16 nearest-even).
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kHeadDim) k_prep(const __grid_constant__ Batch B) {
+  __shared__ float qs[kHeadDim];
+  __shared__ float red[kHeadDim / 32];
   const int pi = blockIdx.y;
   if (pi >= B.n) return;
   const Prob& P = B.p[pi];
@@ -39,14 +41,52 @@ __global__ void __launch_bounds__(kHeadDim) k_prep(const __grid_constant__ Batch
     for (int r = 0; r < P.R; ++r) acc = __fadd_rn(acc, __bfloat162float(q0[(int64_t)r * row_stride]));
     v = __fdiv_rn(acc, (float)P.R);
   }
-  P.qeff[(int64_t)L * kHeadDim + d] = __float2bfloat16_rn(v);
+  const __nv_bfloat16 qe = __float2bfloat16_rn(v);
+  P.qeff[(int64_t)L * kHeadDim + d] = qe;
+  qs[d] = __bfloat162float(qe);
   if (d == 0) {
     P.cand_cnt[L] = 0;
     P.gthr[L] = float_to_ordered(-INFINITY);
   }
+  for (int x = d; x < kLadderLevels; x += kHeadDim) P.ladder[(int64_t)L * kLadderLevels + x] = 0;
   for (int u = L * kHeadDim + d; u < P.ucap; u += n_lists * kHeadDim) P.votes[u] = 0;
   if (L == 0 && d < 4) P.counts[d] = 0;
   if (L == 0 && d == 0) *P.status = 0u;
+  __syncthreads();
+
+  // Ladder anchor: the largest score over a few history units spread over the stream.
+  float mx = -INFINITY;
+  if (P.Uh > 0) {
+    const int ns = min(kSampleUnits, P.Uh);
+    const int64_t slab = (int64_t)i * P.Hkv + h / P.G;
+    const __nv_bfloat16* sk = P.keys + slab * P.ncap * kHeadDim;
+    for (int x = d; x < ns * P.Tu; x += kHeadDim) {
+      const int su = x / P.Tu, r = x - su * P.Tu;
+      const int64_t u = ((int64_t)su * P.Uh) / ns;
+      const uint4* row = reinterpret_cast<const uint4*>(sk + (u * P.Tu + r) * kHeadDim);
+      float dot = 0.f;
+#pragma unroll 4
+      for (int c = 0; c < kHeadDim / 8; ++c) {
+        const uint4 w = row[c];
+        const __nv_bfloat162* e = reinterpret_cast<const __nv_bfloat162*>(&w);
+#pragma unroll
+        for (int z = 0; z < 4; ++z) {
+          const float2 f = __bfloat1622float2(e[z]);
+          dot = fmaf(qs[8 * c + 2 * z], f.x, dot);
+          dot = fmaf(qs[8 * c + 2 * z + 1], f.y, dot);
+        }
+      }
+      mx = fmaxf(mx, dot * kScoreScale);
+    }
+  }
+  for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+  if ((d & 31) == 0) red[d >> 5] = mx;
+  __syncthreads();
+  if (d == 0) {
+    float a = red[0];
+    for (int w = 1; w < kHeadDim / 32; ++w) a = fmaxf(a, red[w]);
+    P.anchor[L] = (a == -INFINITY || a != a) ? 0.f : a;
+  }
 }
 
 cudaError_t launch_prep(const Batch& B, cudaStream_t s) {
@@ -64,21 +104,23 @@ cudaError_t launch_prep(const Batch& B, cudaStream_t s) {
 // Block: kScoreWarps compute warps + 1 threshold warp.
 //
 // Compute warps take the chunk's units round-robin and walk each unit in tiles of 16
-// tokens. A tile's scores for the G query heads of the group come from 8
-// m16n8k16 bf16 MMAs: A = 16 keys x 16 dims, B = 16 dims x 8 heads (G used).
-// The contraction order over d is free, so lane (row g, column group t) loads the
-// 64 contiguous bytes {32 v + 8 t .. 32 v + 8 t + 7 : v = 0..3} of rows g and g + 8 with
-// 16-byte loads straight from HBM into the A-fragment registers, and the query
-// fragments use the same permutation. The accumulator gives lane (g, t) the scores
-// of keys g and g + 8 for heads 2t and 2t + 1.
+// tokens. Each warp streams its tiles through its own ring of kScoreStages shared
+// memory buffers with TMA bulk copies (cp.async.bulk + mbarrier transaction counts),
+// so the data in flight costs no registers. A tile's scores for the G query heads
+// of the group come from 8 m16n8k16 bf16 MMAs: A = 16 keys x 16 dims, B = 16 dims x 8
+// heads (G used). The contraction order over d is free, so lane (row g, column
+// group t) reads the 16-byte chunks {4 v + t : v = 0..3} of rows g and g + 8, and the
+// query fragments use the same permutation. The accumulator gives lane (g, t) the
+// scores of keys g and g + 8 for heads 2t and 2t + 1.
 //
 // Candidate filter: a token is appended to its list when s >= thr[h], where thr[h] is
 // always a lower bound of the list's k-th best score, so every top-k token is
-// appended. The threshold warp maintains thr from a per-head histogram of the
-// appended scores (bins of 1/8 log2 unit anchored at the first units' maximum: the
-// lower edge of the bin below the one where the count from the top reaches k is a
-// valid bound whatever the rounding of the bin computation) and
-// shares it with the other CTAs of the list through a global atomicMax.
+// appended. Every appended score also counts in the list's global histogram (bins
+// = top 14 bits of the order-preserving image of s). The threshold warp of each CTA
+// scans its lists' histograms from the highest non-empty bin down: the lower edge of
+// the bin where the count reaches k bounds the k-th best score from below, because
+// at least k appended tokens (of any CTA) score that much. The bound therefore
+// tracks the k-th best of everything scored so far by the whole grid.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ void mma_16816(float (&d)[4], uint32_t a0, uint32_t a1,
                                           uint32_t a2, uint32_t a3, uint32_t b0,
@@ -99,14 +141,61 @@ __device__ __forceinline__ uint4 ld_stream(const void* p) {
 }
 
 struct ScoreShared {
-  int hist[kMaxGroup][kHistBins];
+  int lad[kMaxGroup][kLadderLevels];  // this CTA's appended-score counts not yet merged
   float thr[kMaxGroup];
-  float base[kMaxGroup];
-  uint32_t max0[kMaxGroup];
-  int first_done;
+  float anchor[kMaxGroup];
   int all_done;
-  int base_valid;
+  unsigned long long bar[kScoreWarps][kScoreStages];  // one mbarrier per warp stage
 };
+
+// ---- TMA bulk copies and mbarriers (inline PTX) ----
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Global -> shared bulk copy of `bytes` (multiple of 16, 16-byte aligned ends) that
+// completes the transaction count of `bar`.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes,
+                                          uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+      ::"r"(dst), "l"(src), "r"(bytes), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Bounded wait for a stage's bulk copy: gives up after ~1 s (or 2^26 polls).
+__device__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (uint32_t i = 1; i < (1u << 26); ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 1023u) == 0u && global_ns() - t0 > 1000000000ull) break;
+  }
+  return false;
+}
 
 // One column (query head) of a tile: online (max, sum 2^(s - max)) over valid rows.
 __device__ __forceinline__ void stats_update(float& m, float& l, float x0, bool v0,
@@ -121,89 +210,81 @@ __device__ __forceinline__ void stats_update(float& m, float& l, float x0, bool 
   }
 }
 
-__device__ __forceinline__ void hist_add(ScoreShared& S, int c, float s, float base,
-                                         bool base_ok) {
-  if (!base_ok) return;
-  const int bin = __float2int_rd((s - base) * kBinsPerUnit);
-  if (bin >= 0) atomicAdd(&S.hist[c][min(bin, kHistBins - 1)], 1);
+// Appended score: count it at its ladder level in this CTA's shared counts.
+__device__ __forceinline__ void ladder_add(ScoreShared& S, int c, float s, float a) {
+  const int lv = __float2int_rd((s - a) * kLadderPerUnit) + kLadderZero;
+  if (lv >= 0) atomicAdd(&S.lad[c][min(lv, kLadderLevels - 1)], 1);
 }
 
+// The threshold warp merges this CTA's ladder counts into the lists' global counts and
+// derives from those the lower bound thr of each list's k-th best score: if the
+// levels >= i hold at least k appended tokens (of any CTA), the k-th best score is at
+// least level i's lower edge. One level of margin covers the rounding of the level
+// computation.
 __device__ void threshold_warp(ScoreShared& S, const Prob& P, int list0, int k) {
+  constexpr int per = kLadderLevels / 32;  // levels per lane; lane 0 holds the top ones
   const int lane = threadIdx.x & 31;
   const int G = P.G;
-  bool base_ok = false;
-  volatile int* vfirst = &S.first_done;
   volatile int* vdone = &S.all_done;
   volatile float* vthr = S.thr;
   for (int iter = 0; iter < (1 << 21); ++iter) {
     const int done = *vdone;
-    if (!base_ok) {
-      if (*vfirst >= kScoreWarps) {
-        __threadfence_block();
-        if (lane < G) {
-          const float mx = ordered_to_float(((volatile uint32_t*)S.max0)[lane]);
-          S.base[lane] = (mx == -INFINITY) ? 0.f : mx - kHistBelowMax;
-        }
-        __syncwarp();
-        __threadfence_block();
-        if (lane == 0) *(volatile int*)&S.base_valid = 1;
-        base_ok = true;
-      }
-    } else {
-      for (int c = 0; c < G; ++c) {
-        const volatile int* hc = S.hist[c];
-        int cnts[16];
-        int sum = 0;
+    for (int c = 0; c < G; ++c) {
+      int* gl = P.ladder + (int64_t)(list0 + c) * kLadderLevels;
 #pragma unroll
-        for (int q = 0; q < 16; ++q) {
-          cnts[q] = hc[kHistBins - 1 - (16 * lane + q)];
-          sum += cnts[q];
-        }
-        int cum = sum;
-#pragma unroll
-        for (int off = 1; off < 32; off <<= 1) {
-          const int y = __shfl_up_sync(0xffffffffu, cum, off);
-          if (lane >= off) cum += y;
-        }
-        const unsigned hit = __ballot_sync(0xffffffffu, cum >= k);
-        float t_new = -INFINITY;
-        if (hit) {
-          const int f = __ffs(hit) - 1;
-          if (lane == f) {
-            int run = cum - sum;
-            int q = 0;
-            for (; q < 15; ++q) {
-              run += cnts[q];
-              if (run >= k) break;
-            }
-            // One bin of margin: a score counted in bin b satisfies s >= base + b / 8
-            // only up to the rounding of (s - base), far below a bin width.
-            const int bin = kHistBins - 1 - (16 * lane + q);
-            t_new = S.base[c] + (float)(bin - 1) / kBinsPerUnit;
-          }
-          t_new = __shfl_sync(0xffffffffu, t_new, f);
-        }
-        if (lane == 0) {
-          float t;
-          if (hit) {
-            const uint32_t old = atomicMax(P.gthr + list0 + c, float_to_ordered(t_new));
-            t = fmaxf(t_new, ordered_to_float(old));
-          } else {
-            t = ordered_to_float(*(volatile uint32_t*)(P.gthr + list0 + c));
-          }
-          if (t > vthr[c]) vthr[c] = t;
-        }
-        __syncwarp();
+      for (int q = 0; q < per; ++q) {
+        const int lv = kLadderLevels - 1 - (per * lane + q);
+        const int dv = atomicExch(&S.lad[c][lv], 0);
+        if (dv) atomicAdd(gl + lv, dv);
       }
     }
+    for (int c = 0; c < G; ++c) {
+      const volatile int* gl = P.ladder + (int64_t)(list0 + c) * kLadderLevels;
+      int cnt[per];
+      int sum = 0;
+#pragma unroll
+      for (int q = 0; q < per; ++q) {
+        cnt[q] = gl[kLadderLevels - 1 - (per * lane + q)];
+        sum += cnt[q];
+      }
+      int cum = sum;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, cum, off);
+        if (lane >= off) cum += y;
+      }
+      const unsigned hit = __ballot_sync(0xffffffffu, cum >= k);
+      if (hit) {
+        const int f = __ffs(hit) - 1;
+        float t = -INFINITY;
+        if (lane == f) {
+          int run = cum - sum, qf = per - 1;
+#pragma unroll
+          for (int q = 0; q < per; ++q) {
+            run += cnt[q];
+            if (run >= k && qf == per - 1 && q < per - 1) qf = q;
+          }
+          const int lv = kLadderLevels - 1 - (per * lane + qf);
+          t = S.anchor[c] + (float)(lv - kLadderZero - 1) / kLadderPerUnit;
+          const uint32_t old = atomicMax(P.gthr + list0 + c, float_to_ordered(t));
+          t = fmaxf(t, ordered_to_float(old));
+          if (t > vthr[c]) vthr[c] = t;
+        }
+      } else if (lane == 0) {
+        const float t = ordered_to_float(*(volatile uint32_t*)(P.gthr + list0 + c));
+        if (t > vthr[c]) vthr[c] = t;
+      }
+    }
+    __syncwarp();
     if (done >= kScoreWarps) break;
-    __nanosleep(400);
+    __nanosleep(256);
   }
 }
 
 __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
     k_score(const __grid_constant__ Batch B) {
   __shared__ ScoreShared S;
+  extern __shared__ __align__(128) unsigned char tiles[];  // [warp][stage][kTileBytes]
   const int b = blockIdx.x;
   const int pi = problem_of_block(B, b);
   const Prob& P = B.p[pi];
@@ -215,24 +296,22 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
   const int u0 = (int)(((int64_t)P.Uh * chunk) / P.chunks);
   const int u1 = (int)(((int64_t)P.Uh * (chunk + 1)) / P.chunks);
 
-  for (int x = threadIdx.x; x < kMaxGroup * kHistBins; x += blockDim.x)
-    (&S.hist[0][0])[x] = 0;
-  if (threadIdx.x < kMaxGroup) {
-    S.thr[threadIdx.x] = -INFINITY;
-    S.base[threadIdx.x] = 0.f;
-    S.max0[threadIdx.x] = float_to_ordered(-INFINITY);
-  }
-  if (threadIdx.x == 0) {
-    S.first_done = 0;
-    S.all_done = 0;
-    S.base_valid = 0;
-  }
-  __syncthreads();
-
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int i = slab / P.Hkv, kvh = slab - i * P.Hkv;
   const int G = P.G;
   const int list0 = i * P.Hq + kvh * G;
+  for (int x = threadIdx.x; x < kMaxGroup * kLadderLevels; x += blockDim.x)
+    (&S.lad[0][0])[x] = 0;
+  if (threadIdx.x < kMaxGroup) {
+    S.thr[threadIdx.x] = -INFINITY;
+    S.anchor[threadIdx.x] = threadIdx.x < G ? P.anchor[list0 + threadIdx.x] : 0.f;
+  }
+  if (threadIdx.x == 0) S.all_done = 0;
+  if (threadIdx.x < kScoreWarps * kScoreStages)
+    mbar_init(smem_u32(&S.bar[0][0] + threadIdx.x), 1u);
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  __syncthreads();
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int k = B.k;
   if (warp == kScoreWarps) {
     threshold_warp(S, P, list0, k);
@@ -240,7 +319,7 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
   }
 
   const int g = lane >> 2, t4 = lane & 3;
-  // Query fragments (B operand), permuted like the key loads.
+  // Query fragments (B operand), permuted like the key fragment reads below.
   uint32_t qf[8][2];
   {
     const uint32_t* qw = reinterpret_cast<const uint32_t*>(P.qeff);
@@ -261,73 +340,97 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
   const bool hv0 = c0 < G, hv1 = c1 < G;
   const int L0 = list0 + c0, L1 = list0 + c1;
   const int Tu = P.Tu;
-  const int tpu = (Tu + 15) >> 4;
+  const int tpu = (Tu + kTileRows - 1) / kTileRows;
   const int n_chunk_units = u1 - u0;
   const int n_my = n_chunk_units > warp
                        ? (n_chunk_units - warp + kScoreWarps - 1) / kScoreWarps
                        : 0;
   const int ntiles = n_my * tpu;
   const __nv_bfloat16* slab_keys = P.keys + (int64_t)slab * P.ncap * kHeadDim;
-  float* cs0 = P.cand_s + (int64_t)(hv0 ? L0 : list0) * P.cand_cap;
-  int32_t* ci0 = P.cand_id + (int64_t)(hv0 ? L0 : list0) * P.cand_cap;
-  float* cs1 = P.cand_s + (int64_t)(hv1 ? L1 : list0) * P.cand_cap;
-  int32_t* ci1 = P.cand_id + (int64_t)(hv1 ? L1 : list0) * P.cand_cap;
-  float2* us0 = P.ustats + (int64_t)(hv0 ? L0 : list0) * P.ucap;
-  float2* us1 = P.ustats + (int64_t)(hv1 ? L1 : list0) * P.ucap;
+  const int64_t cbase0 = (int64_t)(hv0 ? L0 : list0) * P.cand_cap;
+  const int64_t cbase1 = (int64_t)(hv1 ? L1 : list0) * P.cand_cap;
   const unsigned gmask = 0x11111111u << t4;
   const unsigned lt_mask = (1u << lane) - 1u;
+  unsigned char* my_tiles = tiles + (size_t)warp * kScoreStages * kTileBytes;
+  const uint32_t my_tiles_s = smem_u32(my_tiles);
+  const uint32_t my_bars = smem_u32(&S.bar[warp][0]);
+  const volatile float* vthr = S.thr;
+  const float an0 = S.anchor[c0 < kMaxGroup ? c0 : 0], an1 = S.anchor[c1 < kMaxGroup ? c1 : 0];
+  // Candidate slots reserved for this lane group's two lists (identical in its 8 lanes).
+  int rp0 = 0, rl0 = 0, rp1 = 0, rl1 = 0;
 
-  float m0 = -INFINITY, l0 = 0.f, m1 = -INFINITY, l1 = 0.f;
-  float thr0 = INFINITY, thr1 = INFINITY, bs0 = 0.f, bs1 = 0.f;
-  bool base_ok = false, first_unit = true;
-
-  auto tile_pos = [&](int t, int& u, int& j) {
-    const int m = t / tpu;
-    j = t - m * tpu;
-    u = u0 + warp + m * kScoreWarps;
-  };
-  auto load_tile = [&](uint4 (&buf)[8], int t) {
-    int u, j;
-    tile_pos(t, u, j);
-    const int r0 = 16 * j + g;
-    const __nv_bfloat16* p0 = slab_keys + ((int64_t)u * Tu + r0) * kHeadDim + 8 * t4;
-    const bool ok0 = r0 < Tu, ok1 = r0 + 8 < Tu;
-#pragma unroll
-    for (int v = 0; v < 4; ++v) {
-      buf[v] = ok0 ? ld_stream(p0 + 32 * v) : make_uint4(0u, 0u, 0u, 0u);
-      buf[4 + v] = ok1 ? ld_stream(p0 + 8 * kHeadDim + 32 * v) : make_uint4(0u, 0u, 0u, 0u);
+  // Lane 0 starts the bulk copy of tile t (unit uu, tile jj of the unit) into its
+  // stage once the warp's reads of that stage are ordered before the async write.
+  auto issue = [&](int t, int uu, int jj) {
+    if (t >= ntiles) return;
+    const int r0 = kTileRows * jj;
+    const int nrows = min(kTileRows, Tu - r0);
+    const int st = t % kScoreStages;
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      const uint32_t bar = my_bars + 8u * st;
+      const uint32_t bytes = (uint32_t)nrows * kHeadDim * 2u;
+      mbar_expect_tx(bar, bytes);
+      bulk_load(my_tiles_s + (uint32_t)st * kTileBytes,
+                slab_keys + ((int64_t)uu * Tu + r0) * kHeadDim, bytes, bar);
     }
   };
-  auto process = [&](const uint4 (&buf)[8], int t) {
-    int u, j;
-    tile_pos(t, u, j);
+
+  // tile cursors: the tile being consumed and the tile being issued
+  int cu = u0 + warp, cj = 0;          // consume position
+  int iu = u0 + warp, ij = 0;          // issue position
+  auto advance = [&](int& uu, int& jj) {
+    if (++jj == tpu) {
+      jj = 0;
+      uu += kScoreWarps;
+    }
+  };
+  for (int t = 0; t < kScoreStages; ++t) {
+    issue(t, iu, ij);
+    advance(iu, ij);
+  }
+
+  float m0 = -INFINITY, l0 = 0.f, m1 = -INFINITY, l1 = 0.f;
+  int t = 0;
+  bool aborted = false;
+  for (; t < ntiles; ++t) {
+    const int st = t % kScoreStages;
+    const bool ok = mbar_wait_bounded(my_bars + 8u * st, (uint32_t)((t / kScoreStages) & 1));
+    if (!__all_sync(0xffffffffu, ok)) {
+      aborted = true;
+      break;
+    }
+    const unsigned char* tb = my_tiles + (size_t)st * kTileBytes;
+    // A fragments: lane (g, t4) takes the 16-byte chunks 4v + t4 of rows g and g + 8.
+    uint4 ra[4], rb[4];
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {
+      ra[v] = *reinterpret_cast<const uint4*>(tb + g * 256 + 16 * (4 * v + t4));
+      rb[v] = *reinterpret_cast<const uint4*>(tb + (g + 8) * 256 + 16 * (4 * v + t4));
+    }
+    // two accumulators halve the dependent MMA chain
+    float acc[4] = {0.f, 0.f, 0.f, 0.f}, acd[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {
+      mma_16816(acc, ra[v].x, rb[v].x, ra[v].y, rb[v].y, qf[2 * v][0], qf[2 * v][1]);
+      mma_16816(acd, ra[v].z, rb[v].z, ra[v].w, rb[v].w, qf[2 * v + 1][0], qf[2 * v + 1][1]);
+    }
+    const int u = cu, j = cj;
+    advance(cu, cj);
+    issue(t + kScoreStages, iu, ij);   // the stage's data now sits in registers
+    advance(iu, ij);
+
     if (j == 0) {
-      const volatile float* vthr = S.thr;
-      thr0 = hv0 ? vthr[c0] : INFINITY;
-      thr1 = hv1 ? vthr[c1] : INFINITY;
-      base_ok = *(volatile int*)&S.base_valid != 0;
-      if (base_ok) {
-        const volatile float* vbase = S.base;
-        bs0 = vbase[c0];
-        bs1 = vbase[c1];
-      }
       m0 = m1 = -INFINITY;
       l0 = l1 = 0.f;
     }
-    float acc[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-    for (int jj = 0; jj < 8; ++jj) {
-      const int v = jj >> 1;
-      const uint32_t a0 = (jj & 1) ? buf[v].z : buf[v].x;
-      const uint32_t a1 = (jj & 1) ? buf[4 + v].z : buf[4 + v].x;
-      const uint32_t a2 = (jj & 1) ? buf[v].w : buf[v].y;
-      const uint32_t a3 = (jj & 1) ? buf[4 + v].w : buf[4 + v].y;
-      mma_16816(acc, a0, a1, a2, a3, qf[jj][0], qf[jj][1]);
-    }
-    const int r0 = 16 * j + g;
+    const float thr0 = hv0 ? vthr[c0] : INFINITY;
+    const float thr1 = hv1 ? vthr[c1] : INFINITY;
+    const int r0 = kTileRows * j + g;
     const bool v0 = r0 < Tu, v1 = r0 + 8 < Tu;
-    const float s00 = acc[0] * kScoreScale, s01 = acc[1] * kScoreScale;
-    const float s10 = acc[2] * kScoreScale, s11 = acc[3] * kScoreScale;
+    const float s00 = (acc[0] + acd[0]) * kScoreScale, s01 = (acc[1] + acd[1]) * kScoreScale;
+    const float s10 = (acc[2] + acd[2]) * kScoreScale, s11 = (acc[3] + acd[3]) * kScoreScale;
     stats_update(m0, l0, s00, v0, s10, v1);
     stats_update(m1, l1, s01, v0, s11, v1);
 
@@ -339,41 +442,53 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
       const unsigned b10 = __ballot_sync(0xffffffffu, p10) & gmask;
       const unsigned b01 = __ballot_sync(0xffffffffu, p01) & gmask;
       const unsigned b11 = __ballot_sync(0xffffffffu, p11) & gmask;
-      {
-        const int n = __popc(b00) + __popc(b10);
-        int base = 0;
-        if (g == 0 && n > 0) base = atomicAdd(P.cand_cnt + L0, n);
-        base = __shfl_sync(0xffffffffu, base, t4);
-        if (p00) {
-          const int pos = base + __popc(b00 & lt_mask);
-          cs0[pos] = s00;
-          ci0[pos] = tok0;
-          hist_add(S, c0, s00, bs0, base_ok);
-        }
-        if (p10) {
-          const int pos = base + __popc(b00) + __popc(b10 & lt_mask);
-          cs0[pos] = s10;
-          ci0[pos] = tok1;
-          hist_add(S, c0, s10, bs0, base_ok);
-        }
+      const int n0 = __popc(b00) + __popc(b10), n1 = __popc(b01) + __popc(b11);
+      // slots: continue the reserved block, reserve a new one when it runs out
+      const bool need0 = n0 > rl0, need1 = n1 > rl1;
+      int nb0 = 0, nb1 = 0;
+      if (g == 0 && need0) nb0 = atomicAdd(P.cand_cnt + L0, kReserve);
+      if (g == 0 && need1) nb1 = atomicAdd(P.cand_cnt + L1, kReserve);
+      nb0 = __shfl_sync(0xffffffffu, nb0, t4);
+      nb1 = __shfl_sync(0xffffffffu, nb1, t4);
+      auto slot0 = [&](int r) { return cbase0 + (r < rl0 ? rp0 + r : nb0 + (r - rl0)); };
+      auto slot1 = [&](int r) { return cbase1 + (r < rl1 ? rp1 + r : nb1 + (r - rl1)); };
+      if (p00) {
+        const int64_t pos = slot0(__popc(b00 & lt_mask));
+        P.cand_s[pos] = s00;
+        P.cand_id[pos] = tok0;
+        ladder_add(S, c0, s00, an0);
       }
-      {
-        const int n = __popc(b01) + __popc(b11);
-        int base = 0;
-        if (g == 0 && n > 0) base = atomicAdd(P.cand_cnt + L1, n);
-        base = __shfl_sync(0xffffffffu, base, t4);
-        if (p01) {
-          const int pos = base + __popc(b01 & lt_mask);
-          cs1[pos] = s01;
-          ci1[pos] = tok0;
-          hist_add(S, c1, s01, bs1, base_ok);
-        }
-        if (p11) {
-          const int pos = base + __popc(b01) + __popc(b11 & lt_mask);
-          cs1[pos] = s11;
-          ci1[pos] = tok1;
-          hist_add(S, c1, s11, bs1, base_ok);
-        }
+      if (p10) {
+        const int64_t pos = slot0(__popc(b00) + __popc(b10 & lt_mask));
+        P.cand_s[pos] = s10;
+        P.cand_id[pos] = tok1;
+        ladder_add(S, c0, s10, an0);
+      }
+      if (p01) {
+        const int64_t pos = slot1(__popc(b01 & lt_mask));
+        P.cand_s[pos] = s01;
+        P.cand_id[pos] = tok0;
+        ladder_add(S, c1, s01, an1);
+      }
+      if (p11) {
+        const int64_t pos = slot1(__popc(b01) + __popc(b11 & lt_mask));
+        P.cand_s[pos] = s11;
+        P.cand_id[pos] = tok1;
+        ladder_add(S, c1, s11, an1);
+      }
+      if (need0) {
+        rp0 = nb0 + (n0 - rl0);
+        rl0 = kReserve - (n0 - rl0);
+      } else {
+        rp0 += n0;
+        rl0 -= n0;
+      }
+      if (need1) {
+        rp1 = nb1 + (n1 - rl1);
+        rl1 = kReserve - (n1 - rl1);
+      } else {
+        rp1 += n1;
+        rl1 -= n1;
       }
     }
     if (j == tpu - 1) {
@@ -387,37 +502,21 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
         ml_combine(m1, l1, mo1, lo1);
       }
       if (g == 0) {
-        if (hv0) us0[u] = make_float2(m0, l0);
-        if (hv1) us1[u] = make_float2(m1, l1);
-        if (first_unit) {
-          if (hv0) atomicMax(&S.max0[c0], float_to_ordered(m0));
-          if (hv1) atomicMax(&S.max0[c1], float_to_ordered(m1));
-        }
-      }
-      if (first_unit) {
-        __syncwarp();
-        __threadfence_block();
-        if (lane == 0) atomicAdd(&S.first_done, 1);
-        first_unit = false;
+        if (hv0) P.ustats[(int64_t)L0 * P.ucap + u] = make_float2(m0, l0);
+        if (hv1) P.ustats[(int64_t)L1 * P.ucap + u] = make_float2(m1, l1);
       }
     }
-  };
-
-  uint4 bufA[8], bufB[8];
-  if (ntiles > 0) load_tile(bufA, 0);
-  if (ntiles > 1) load_tile(bufB, 1);
-  for (int t = 0; t < ntiles; t += 2) {
-    process(bufA, t);
-    if (t + 2 < ntiles) load_tile(bufA, t + 2);
-    if (t + 1 < ntiles) {
-      process(bufB, t + 1);
-      if (t + 3 < ntiles) load_tile(bufB, t + 3);
-    }
   }
-  if (lane == 0) {
-    if (first_unit) atomicAdd(&S.first_done, 1);
-    atomicAdd(&S.all_done, 1);
+  // unused reserved slots are marked empty (score -inf)
+  for (int x = g; x < rl0; x += 8) P.cand_s[cbase0 + rp0 + x] = -INFINITY;
+  for (int x = g; x < rl1; x += 8) P.cand_s[cbase1 + rp1 + x] = -INFINITY;
+  if (aborted) {
+    // report, then let the copies already in flight land before the CTA exits
+    if (lane == 0) atomicOr(P.status, kStatusTimeout);
+    for (int r = t; r < min(ntiles, t + kScoreStages); ++r)
+      mbar_wait_bounded(my_bars + 8u * (r % kScoreStages), (uint32_t)((r / kScoreStages) & 1));
   }
+  if (lane == 0) atomicAdd(&S.all_done, 1);
 }
 
 int score_chunks_per_slab(int n_slabs_total, int hist_units, int sm_count) {
@@ -427,7 +526,7 @@ int score_chunks_per_slab(int n_slabs_total, int hist_units, int sm_count) {
   const int64_t slots = (int64_t)sm_count * kScoreCtasPerSm;
   int best_c = 1;
   int64_t best_cost = INT64_MAX;
-  for (int c = 1; c <= hist_units && c <= 4096; ++c) {
+  for (int c = 1; c <= hist_units && c <= kMaxChunksPerSlab; ++c) {
     const int64_t ctas = (int64_t)n_slabs_total * c;
     const int64_t waves = (ctas + slots - 1) / slots;
     const int64_t len = (hist_units + c - 1) / c;
@@ -442,7 +541,10 @@ int score_chunks_per_slab(int n_slabs_total, int hist_units, int sm_count) {
 
 cudaError_t launch_score(const Batch& B, cudaStream_t s) {
   if (B.score_ctas <= 0) return cudaSuccess;
-  k_score<<<B.score_ctas, kScoreThreads, 0, s>>>(B);
+  const int smem = kScoreWarps * kScoreStages * kTileBytes;
+  cudaError_t e = cudaFuncSetAttribute(k_score, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  k_score<<<B.score_ctas, kScoreThreads, smem, s>>>(B);
   return cudaGetLastError();
 }
 

@@ -146,8 +146,13 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
   const int32_t* ci = P.cand_id + (int64_t)L * P.cand_cap;
   float lo = ordered_to_float(P.gthr[L]);
   if (lo == -INFINITY) {
+    // no threshold was established: start from the smallest real candidate (unused
+    // reserved slots hold -inf and are never candidates)
     float mn = INFINITY;
-    for (int x = tid; x < cnt; x += blockDim.x) mn = fminf(mn, cs[x]);
+    for (int x = tid; x < cnt; x += blockDim.x) {
+      const float s = cs[x];
+      if (s > -INFINITY) mn = fminf(mn, s);
+    }
     lo = block_min(mn, s_m);
   }
   const float hi = M;
