@@ -87,7 +87,8 @@ int pool_cap_of(const ss_index* ix, const ss_retrieve_params* p) {
 // Candidate slots per list: every token once, plus the unused tails of the slot
 // blocks that score warps reserve.
 int64_t cand_cap_of(const ss_index* ix) {
-  return ix->ncap + (int64_t)kMaxChunksPerSlab * kScoreWarps * kReserve;
+  const int64_t c = ix->ncap + (int64_t)kMaxChunksPerSlab * kScoreWarps * kReserve;
+  return (c + 63) & ~(int64_t)63;  // keeps every list's slots 256-byte aligned
 }
 
 // Workspace regions of one problem (offsets from the problem's base).
@@ -117,9 +118,9 @@ Layout layout_of(const ss_index* ix, int R, const ss_retrieve_params* p) {
   l.cand_cnt = take(score_lists * 4);
   l.gthr = take(score_lists * 4);
   l.ladder = take(score_lists * kLadderLevels * 4);
-  l.anchor = take(score_lists * 4);
+  l.anchor = take(score_lists * kSampleUnits * 4);
   l.ustats = take(score_lists * ix->ucap * 8);
-  l.gram = take(pc * pc * 4);
+  l.gram = take(pc * (pc + 1) / 2 * 4);
   l.topk_tok = take(n_lists * p->k * 4);
   l.topk_w = take(n_lists * p->k * 4);
   l.list_ml = take(n_lists * 8);
@@ -276,10 +277,9 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
   SS_CUDA(launch_score(B, st));
   if (tr && tr->score_end) SS_CUDA(cudaEventRecord((cudaEvent_t)tr->score_end, st));
   SS_CUDA(launch_select(B, max_lists, st));
-  SS_CUDA(launch_votes_mass(B, max_lists, max_uh, st));
+  SS_CUDA(launch_mass(B, max_uh, st));
   SS_CUDA(launch_pool(B, max_uh, st));
   SS_CUDA(launch_maxmin(B, max_pool, st));
-  SS_CUDA(launch_expand(B, st));
   return SS_OK;
 }
 

@@ -76,9 +76,9 @@ struct Prob {
   int32_t* cand_cnt;           // [n_score_lists]
   uint32_t* gthr;              // [n_score_lists] ordered-float threshold
   int32_t* ladder;             // [n_score_lists][kLadderLevels] appended-score counts
-  float* anchor;               // [n_score_lists] ladder anchor A (log2 units)
+  float* anchor;               // [n_score_lists][kSampleUnits] sample maxima (log2 units)
   float2* ustats;              // [n_score_lists][ucap] per-unit (max, sum 2^(s-max))
-  float* gram;                 // [pool][pool]
+  float* gram;                 // packed upper triangle of the pool's Gram matrix
   // outputs
   int32_t* topk_tok;           // [n_lists][k]
   float* topk_w;
@@ -138,6 +138,14 @@ __device__ __forceinline__ void ml_combine(float& m, float& l, float mo, float l
   l = a + b;
 }
 
+// Ladder anchor A of list L: the largest score over the sampled units (0 if none).
+__device__ __forceinline__ float list_anchor(const Prob& P, int L) {
+  float a = -INFINITY;
+#pragma unroll
+  for (int z = 0; z < kSampleUnits; ++z) a = fmaxf(a, P.anchor[L * kSampleUnits + z]);
+  return (a == -INFINITY || a != a) ? 0.f : a;
+}
+
 __device__ __forceinline__ int problem_of_block(const Batch& B, int b) {
   int pi = 0;
   while (pi + 1 < B.n && B.p[pi + 1].cta_begin <= b) ++pi;
@@ -151,11 +159,9 @@ namespace ss {
 cudaError_t launch_prep(const Batch& B, cudaStream_t s);
 cudaError_t launch_score(const Batch& B, cudaStream_t s);
 cudaError_t launch_select(const Batch& B, int max_lists, cudaStream_t s);
-cudaError_t launch_votes_mass(const Batch& B, int max_lists, int max_hist_units,
-                              cudaStream_t s);
+cudaError_t launch_mass(const Batch& B, int max_hist_units, cudaStream_t s);
 cudaError_t launch_pool(const Batch& B, int max_hist_units, cudaStream_t s);
 cudaError_t launch_maxmin(const Batch& B, int max_pool, cudaStream_t s);
-cudaError_t launch_expand(const Batch& B, cudaStream_t s);
 cudaError_t launch_append(__nv_bfloat16* keys, int64_t ncap, int64_t tok0,
                           const __nv_bfloat16* src, int64_t src_stride_tokens,
                           int n_slabs, int64_t n_tokens, cudaStream_t s);

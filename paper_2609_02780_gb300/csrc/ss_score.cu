@@ -20,6 +20,9 @@ namespace ss {
 // q_eff[i][h] is the last question row ("final prompt token", Sec. 4.2 / Table 4) or
 // the rows' mean (fp32 sum in row order, divided by R, rounded to bf16 nearest-even).
 // ---------------------------------------------------------------------------
+// Grid (list, problem, sample unit z). Block z = 0 also writes q_eff and resets the
+// per-call state; every block scores the history unit z * Uh / n_sample against its
+// list's query and records the largest score, the anchor of the threshold ladder.
 __global__ void __launch_bounds__(kHeadDim) k_prep(const __grid_constant__ Batch B) {
   __shared__ float qs[kHeadDim];
   __shared__ float red[kHeadDim / 32];
@@ -27,7 +30,7 @@ __global__ void __launch_bounds__(kHeadDim) k_prep(const __grid_constant__ Batch
   if (pi >= B.n) return;
   const Prob& P = B.p[pi];
   const int n_lists = P.P * P.Hq;
-  const int L = blockIdx.x;
+  const int L = blockIdx.x, z = blockIdx.z;
   if (L >= n_lists) return;
   const int i = L / P.Hq, h = L % P.Hq;
   const int d = threadIdx.x;
@@ -42,38 +45,40 @@ __global__ void __launch_bounds__(kHeadDim) k_prep(const __grid_constant__ Batch
     v = __fdiv_rn(acc, (float)P.R);
   }
   const __nv_bfloat16 qe = __float2bfloat16_rn(v);
-  P.qeff[(int64_t)L * kHeadDim + d] = qe;
   qs[d] = __bfloat162float(qe);
-  if (d == 0) {
-    P.cand_cnt[L] = 0;
-    P.gthr[L] = float_to_ordered(-INFINITY);
+  if (z == 0) {
+    P.qeff[(int64_t)L * kHeadDim + d] = qe;
+    if (d == 0) {
+      P.cand_cnt[L] = 0;
+      P.gthr[L] = float_to_ordered(-INFINITY);
+    }
+    for (int x = d; x < kLadderLevels; x += kHeadDim) P.ladder[(int64_t)L * kLadderLevels + x] = 0;
+    for (int u = L * kHeadDim + d; u < P.ucap; u += n_lists * kHeadDim) P.votes[u] = 0;
+    if (L == 0 && d < 4) P.counts[d] = 0;
+    if (L == 0 && d == 0) *P.status = 0u;
   }
-  for (int x = d; x < kLadderLevels; x += kHeadDim) P.ladder[(int64_t)L * kLadderLevels + x] = 0;
-  for (int u = L * kHeadDim + d; u < P.ucap; u += n_lists * kHeadDim) P.votes[u] = 0;
-  if (L == 0 && d < 4) P.counts[d] = 0;
-  if (L == 0 && d == 0) *P.status = 0u;
   __syncthreads();
 
-  // Ladder anchor: the largest score over a few history units spread over the stream.
   float mx = -INFINITY;
-  if (P.Uh > 0) {
-    const int ns = min(kSampleUnits, P.Uh);
+  const int ns = min(kSampleUnits, P.Uh);
+  if (z < ns) {
+    const int64_t u = ((int64_t)z * P.Uh) / ns;
     const int64_t slab = (int64_t)i * P.Hkv + h / P.G;
-    const __nv_bfloat16* sk = P.keys + slab * P.ncap * kHeadDim;
-    for (int x = d; x < ns * P.Tu; x += kHeadDim) {
-      const int su = x / P.Tu, r = x - su * P.Tu;
-      const int64_t u = ((int64_t)su * P.Uh) / ns;
-      const uint4* row = reinterpret_cast<const uint4*>(sk + (u * P.Tu + r) * kHeadDim);
-      float dot = 0.f;
-#pragma unroll 4
-      for (int c = 0; c < kHeadDim / 8; ++c) {
-        const uint4 w = row[c];
-        const __nv_bfloat162* e = reinterpret_cast<const __nv_bfloat162*>(&w);
+    const __nv_bfloat16* sk = P.keys + (slab * P.ncap + u * P.Tu) * kHeadDim;
+    for (int r = d; r < P.Tu; r += kHeadDim) {
+      const uint4* row = reinterpret_cast<const uint4*>(sk + (int64_t)r * kHeadDim);
+      uint4 w[kHeadDim / 8];
 #pragma unroll
-        for (int z = 0; z < 4; ++z) {
-          const float2 f = __bfloat1622float2(e[z]);
-          dot = fmaf(qs[8 * c + 2 * z], f.x, dot);
-          dot = fmaf(qs[8 * c + 2 * z + 1], f.y, dot);
+      for (int c = 0; c < kHeadDim / 8; ++c) w[c] = row[c];
+      float dot = 0.f;
+#pragma unroll
+      for (int c = 0; c < kHeadDim / 8; ++c) {
+        const __nv_bfloat162* e = reinterpret_cast<const __nv_bfloat162*>(&w[c]);
+#pragma unroll
+        for (int zz = 0; zz < 4; ++zz) {
+          const float2 f = __bfloat1622float2(e[zz]);
+          dot = fmaf(qs[8 * c + 2 * zz], f.x, dot);
+          dot = fmaf(qs[8 * c + 2 * zz + 1], f.y, dot);
         }
       }
       mx = fmaxf(mx, dot * kScoreScale);
@@ -85,14 +90,14 @@ __global__ void __launch_bounds__(kHeadDim) k_prep(const __grid_constant__ Batch
   if (d == 0) {
     float a = red[0];
     for (int w = 1; w < kHeadDim / 32; ++w) a = fmaxf(a, red[w]);
-    P.anchor[L] = (a == -INFINITY || a != a) ? 0.f : a;
+    P.anchor[L * kSampleUnits + z] = a;
   }
 }
 
 cudaError_t launch_prep(const Batch& B, cudaStream_t s) {
   int max_lists = 0;
   for (int j = 0; j < B.n; ++j) max_lists = max(max_lists, B.p[j].P * B.p[j].Hq);
-  dim3 grid(max_lists, B.n);
+  dim3 grid(max_lists, B.n, kSampleUnits);
   k_prep<<<grid, kHeadDim, 0, s>>>(B);
   return cudaGetLastError();
 }
@@ -238,46 +243,57 @@ __device__ void threshold_warp(ScoreShared& S, const Prob& P, int list0, int k) 
         if (dv) atomicAdd(gl + lv, dv);
       }
     }
-    for (int c = 0; c < G; ++c) {
-      const volatile int* gl = P.ladder + (int64_t)(list0 + c) * kLadderLevels;
-      int cnt[per];
-      int sum = 0;
+    // the global counts of 4 lists per round trip
 #pragma unroll
-      for (int q = 0; q < per; ++q) {
-        cnt[q] = gl[kLadderLevels - 1 - (per * lane + q)];
-        sum += cnt[q];
+    for (int c0 = 0; c0 < kMaxGroup; c0 += 4) {
+      if (c0 >= G) break;
+      int cnt[4][per];
+#pragma unroll
+      for (int cc = 0; cc < 4; ++cc) {
+        const int c = c0 + cc;
+        const volatile int* gl = P.ladder + (int64_t)(list0 + (c < G ? c : 0)) * kLadderLevels;
+#pragma unroll
+        for (int q = 0; q < per; ++q)
+          cnt[cc][q] = c < G ? gl[kLadderLevels - 1 - (per * lane + q)] : 0;
       }
-      int cum = sum;
 #pragma unroll
-      for (int off = 1; off < 32; off <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, cum, off);
-        if (lane >= off) cum += y;
-      }
-      const unsigned hit = __ballot_sync(0xffffffffu, cum >= k);
-      if (hit) {
-        const int f = __ffs(hit) - 1;
-        float t = -INFINITY;
-        if (lane == f) {
-          int run = cum - sum, qf = per - 1;
+      for (int cc = 0; cc < 4; ++cc) {
+        const int c = c0 + cc;
+        if (c >= G) break;
+        int sum = 0;
 #pragma unroll
-          for (int q = 0; q < per; ++q) {
-            run += cnt[q];
-            if (run >= k && qf == per - 1 && q < per - 1) qf = q;
+        for (int q = 0; q < per; ++q) sum += cnt[cc][q];
+        int cum = sum;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+          const int y = __shfl_up_sync(0xffffffffu, cum, off);
+          if (lane >= off) cum += y;
+        }
+        const unsigned hit = __ballot_sync(0xffffffffu, cum >= k);
+        if (hit) {
+          const int f = __ffs(hit) - 1;
+          if (lane == f) {
+            int run = cum - sum, qf = per - 1;
+#pragma unroll
+            for (int q = 0; q < per; ++q) {
+              run += cnt[cc][q];
+              if (run >= k && qf == per - 1 && q < per - 1) qf = q;
+            }
+            const int lv = kLadderLevels - 1 - (per * lane + qf);
+            float t = S.anchor[c] + (float)(lv - kLadderZero - 1) / kLadderPerUnit;
+            const uint32_t old = atomicMax(P.gthr + list0 + c, float_to_ordered(t));
+            t = fmaxf(t, ordered_to_float(old));
+            if (t > vthr[c]) vthr[c] = t;
           }
-          const int lv = kLadderLevels - 1 - (per * lane + qf);
-          t = S.anchor[c] + (float)(lv - kLadderZero - 1) / kLadderPerUnit;
-          const uint32_t old = atomicMax(P.gthr + list0 + c, float_to_ordered(t));
-          t = fmaxf(t, ordered_to_float(old));
+        } else if (lane == 0) {
+          const float t = ordered_to_float(*(volatile uint32_t*)(P.gthr + list0 + c));
           if (t > vthr[c]) vthr[c] = t;
         }
-      } else if (lane == 0) {
-        const float t = ordered_to_float(*(volatile uint32_t*)(P.gthr + list0 + c));
-        if (t > vthr[c]) vthr[c] = t;
       }
     }
     __syncwarp();
     if (done >= kScoreWarps) break;
-    __nanosleep(256);
+    __nanosleep(128);
   }
 }
 
@@ -303,7 +319,7 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
     (&S.lad[0][0])[x] = 0;
   if (threadIdx.x < kMaxGroup) {
     S.thr[threadIdx.x] = -INFINITY;
-    S.anchor[threadIdx.x] = threadIdx.x < G ? P.anchor[list0 + threadIdx.x] : 0.f;
+    S.anchor[threadIdx.x] = threadIdx.x < G ? list_anchor(P, list0 + threadIdx.x) : 0.f;
   }
   if (threadIdx.x == 0) S.all_done = 0;
   if (threadIdx.x < kScoreWarps * kScoreStages)

@@ -1,12 +1,12 @@
 // Evidence selection after key scoring (Sec. 4.2, Eq. 11-12):
-//   k_select    exact top-k of every list from its candidate array, softmax
-//               statistics from the per-unit (max, sum) pairs, normalised weights
-//   k_votes_mass unit votes (one per (list, selected token) in the unit) and the
-//               attention mass of every history unit (summed weights of all tokens)
-//   k_pool      the vote-ranked pool: top min(pool_mult * K, |H|) units by
-//               (votes desc, mass desc, unit id asc)
-//   k_gram / k_maxmin  greedy max-min diversity over the pool's descriptors
-//   k_expand    each pick plus its preceding units, deduplicated, ascending (Eq. 12)
+//   k_select   exact top-k of every list from its candidate array, softmax statistics
+//              from the per-unit (max, sum) pairs, normalised weights, unit votes
+//              (one per (list, selected token) in the unit, integer atomics)
+//   k_mass     attention mass of every history unit (summed weights of all tokens)
+//   k_pool     the vote-ranked pool: top min(pool_mult * K, |H|) units by
+//              (votes desc, mass desc, unit id asc)
+//   k_gram / k_maxmin  greedy max-min diversity over the pool's descriptors, then each
+//              pick plus its preceding units, deduplicated, ascending (Eq. 12)
 // No floating-point atomics: every float reduction has a fixed order, so results are
 // bit-identical from run to run.
 #include "ss_internal.cuh"
@@ -39,6 +39,71 @@ __device__ void bitonic_desc(unsigned long long* a, int n2) {
       __syncthreads();
     }
   }
+}
+
+// Descending bitonic sort of a[0, n2) for 64 <= n2 <= 2 * blockDim.x (n2 a power of two)
+// with the compare-exchanges of stride < 64 done in registers: thread (warp w, lane l)
+// holds elements 64 w + l and 64 w + 32 + l; strides 1..16 pair lanes (shuffles),
+// stride 32 pairs a thread's two registers, longer strides go through shared memory.
+__device__ __forceinline__ unsigned long long bitonic_keep(unsigned long long mine,
+                                                           unsigned long long other,
+                                                           bool lower, bool desc) {
+  // the lower element of a pair keeps the larger key in a descending block
+  const bool take_max = (lower == desc);
+  return take_max ? (mine > other ? mine : other) : (mine < other ? mine : other);
+}
+
+__device__ void bitonic_desc_hybrid(unsigned long long* a, int n2) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const bool active = 64 * warp < n2;
+  const int i0 = 64 * warp + lane, i1 = i0 + 32;
+  unsigned long long r0 = active ? a[i0] : 0ull, r1 = active ? a[i1] : 0ull;
+  auto reg_stages = [&](int size, int top) {
+    for (int stride = top; stride > 0; stride >>= 1) {
+      if (stride == 32) {
+        const bool desc = (i0 & size) == 0;
+        const unsigned long long x0 = r0, x1 = r1;
+        r0 = bitonic_keep(x0, x1, true, desc);
+        r1 = bitonic_keep(x1, x0, false, desc);
+      } else {
+        const unsigned long long o0 = __shfl_xor_sync(0xffffffffu, r0, stride);
+        const unsigned long long o1 = __shfl_xor_sync(0xffffffffu, r1, stride);
+        const bool lower = (lane & stride) == 0;
+        r0 = bitonic_keep(r0, o0, lower, (i0 & size) == 0);
+        r1 = bitonic_keep(r1, o1, lower, (i1 & size) == 0);
+      }
+    }
+  };
+  for (int size = 2; size <= min(n2, 64); size <<= 1) reg_stages(size, size >> 1);
+  for (int size = 128; size <= n2; size <<= 1) {
+    if (active) {
+      a[i0] = r0;
+      a[i1] = r1;
+    }
+    __syncthreads();
+    for (int stride = size >> 1; stride >= 64; stride >>= 1) {
+      for (int t = threadIdx.x; t < (n2 >> 1); t += blockDim.x) {
+        const int i = 2 * t - (t & (stride - 1));
+        const int j = i + stride;
+        const bool desc = (i & size) == 0;
+        const unsigned long long x = a[i], y = a[j];
+        if ((x < y) == desc) {
+          a[i] = y;
+          a[j] = x;
+        }
+      }
+      __syncthreads();
+    }
+    r0 = active ? a[i0] : 0ull;
+    r1 = active ? a[i1] : 0ull;
+    reg_stages(size, 32);
+  }
+  __syncthreads();
+  if (active) {
+    a[i0] = r0;
+    a[i1] = r1;
+  }
+  __syncthreads();
 }
 
 __device__ __forceinline__ int next_pow2(int x) {
@@ -145,9 +210,47 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
   const float* cs = P.cand_s + (int64_t)L * P.cand_cap;
   const int32_t* ci = P.cand_id + (int64_t)L * P.cand_cap;
   float lo = ordered_to_float(P.gthr[L]);
+  // A tighter bound from the list's completed ladder of appended-score counts: if the
+  // levels >= i hold n tokens, the n-th best score is at least level i's lower edge
+  // (one level of margin for the rounding of the level computation).
+  if (tid < 32) {
+    constexpr int per = kLadderLevels / 32;
+    const int* lad = P.ladder + (int64_t)L * kLadderLevels;
+    int cntl[per];
+    int sum = 0;
+#pragma unroll
+    for (int q = 0; q < per; ++q) {
+      cntl[q] = lad[kLadderLevels - 1 - (per * lane + q)];
+      sum += cntl[q];
+    }
+    int cum = sum;
+    for (int off = 1; off < 32; off <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, cum, off);
+      if (lane >= off) cum += y;
+    }
+    const unsigned hit = __ballot_sync(0xffffffffu, cum >= n);
+    if (lane == 0) s_m[0] = -INFINITY;
+    __syncwarp();
+    if (hit) {
+      const int f = __ffs(hit) - 1;
+      if (lane == f) {
+        int run = cum - sum, qf = per - 1;
+#pragma unroll
+        for (int q = 0; q < per; ++q) {
+          run += cntl[q];
+          if (run >= n && qf == per - 1 && q < per - 1) qf = q;
+        }
+        const int lv = kLadderLevels - 1 - (per * lane + qf);
+        s_m[0] = list_anchor(P, L) + (float)(lv - kLadderZero - 1) / kLadderPerUnit;
+      }
+    }
+  }
+  __syncthreads();
+  lo = fmaxf(lo, s_m[0]);
+  __syncthreads();
   if (lo == -INFINITY) {
-    // no threshold was established: start from the smallest real candidate (unused
-    // reserved slots hold -inf and are never candidates)
+    // no bound: start from the smallest real candidate (unused reserved slots hold
+    // -inf and are never candidates)
     float mn = INFINITY;
     for (int x = tid; x < cnt; x += blockDim.x) {
       const float s = cs[x];
@@ -155,63 +258,95 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
     }
     lo = block_min(mn, s_m);
   }
-  const float hi = M;
-  const float scale = (hi > lo) ? (float)kFineBins / (hi - lo) : 0.f;
-  auto fbin = [&](float s) -> int {
-    const int b = (int)((s - lo) * scale);
-    return min(max(b, 0), kFineBins - 1);
-  };
-
-  for (int x = tid; x < kFineBins; x += blockDim.x) s_hist[x] = 0;
+  // collect the candidates at or above the bound (warp-aggregated slot counter)
+  if (tid == 0) s_n = 0;
   __syncthreads();
-  for (int x = tid; x < cnt; x += blockDim.x) {
-    const float s = cs[x];
-    if (s >= lo) atomicAdd(&s_hist[fbin(s)], 1);
-  }
-  __syncthreads();
-  if (tid < 32) {
-    // lane 0 holds the top 64 bins, lane 31 the bottom 64
-    constexpr int per = kFineBins / 32;
-    int sum = 0;
-    for (int q = 0; q < per; ++q) sum += s_hist[kFineBins - 1 - (per * lane + q)];
-    int cum = sum;
-    for (int off = 1; off < 32; off <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, cum, off);
-      if (lane >= off) cum += y;
-    }
-    const unsigned hit = __ballot_sync(0xffffffffu, cum >= n);
-    if (hit == 0u) {
-      if (lane == 0) s_bstar = -1;
-    } else {
-      const int f = __ffs(hit) - 1;
-      if (lane == f) {
-        int run = cum - sum;
-        int q = 0;
-        for (; q < per - 1; ++q) {
-          run += s_hist[kFineBins - 1 - (per * lane + q)];
-          if (run >= n) break;
+  {
+    // each thread scans 4 consecutive slots per step (one 16-byte load; the list's slots
+    // start 256-byte aligned), with the next step's load issued before this one's work
+    const float4* cs4 = reinterpret_cast<const float4*>(cs);
+    const int n4 = (cnt + 3) >> 2;
+    const int step = blockDim.x;
+    float4 nxt = tid < n4 ? cs4[tid] : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+    for (int b0 = 0; b0 < n4; b0 += step) {
+      const int x4 = b0 + tid;
+      const float4 cur = nxt;
+      const int y4 = x4 + step;
+      nxt = y4 < n4 ? cs4[y4] : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+      const float v[4] = {cur.x, cur.y, cur.z, cur.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int x = 4 * x4 + e;
+        const bool keep = x < cnt && v[e] >= lo;
+        const unsigned m = __ballot_sync(0xffffffffu, keep);
+        int base = 0;
+        if (lane == 0 && m) base = atomicAdd(&s_n, __popc(m));
+        base = __shfl_sync(0xffffffffu, base, 0);
+        if (keep) {
+          const int pos = base + __popc(m & ((1u << lane) - 1u));
+          if (pos < kSelCap) skeys[pos] = cand_key(v[e], ci[x]);
         }
-        s_bstar = kFineBins - 1 - (per * lane + q);
       }
-    }
-    if (lane == 0) s_n = 0;
-  }
-  __syncthreads();
-  const int bstar = s_bstar;
-  if (bstar < 0) {
-    // fewer candidates than n: the lower bound was not one (must not happen)
-    if (tid == 0) atomicOr(P.status, kStatusInternal);
-  }
-  const int bmin = max(bstar, 0);
-  for (int x = tid; x < cnt; x += blockDim.x) {
-    const float s = cs[x];
-    if (s >= lo && fbin(s) >= bmin) {
-      const int pos = atomicAdd(&s_n, 1);
-      if (pos < kSelCap) skeys[pos] = cand_key(s, ci[x]);
     }
   }
   __syncthreads();
   int ns = s_n;
+  if (ns > kSelCap) {
+    // Too many: a 2048-bin histogram of the candidates over [lo, max] locates the bin
+    // of the n-th best; keep the candidates from that bin up.
+    const float hi = M;
+    const float scale = (hi > lo) ? (float)kFineBins / (hi - lo) : 0.f;
+    auto fbin = [&](float s) -> int {
+      const int b = (int)((s - lo) * scale);
+      return min(max(b, 0), kFineBins - 1);
+    };
+    for (int x = tid; x < kFineBins; x += blockDim.x) s_hist[x] = 0;
+    __syncthreads();
+    for (int x = tid; x < cnt; x += blockDim.x) {
+      const float s = cs[x];
+      if (s >= lo) atomicAdd(&s_hist[fbin(s)], 1);
+    }
+    __syncthreads();
+    if (tid < 32) {
+      constexpr int per = kFineBins / 32;  // lane 0 holds the top bins
+      int sum = 0;
+      for (int q = 0; q < per; ++q) sum += s_hist[kFineBins - 1 - (per * lane + q)];
+      int cum = sum;
+      for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, cum, off);
+        if (lane >= off) cum += y;
+      }
+      const unsigned hit = __ballot_sync(0xffffffffu, cum >= n);
+      if (hit == 0u) {
+        if (lane == 0) s_bstar = -1;
+      } else {
+        const int f = __ffs(hit) - 1;
+        if (lane == f) {
+          int run = cum - sum;
+          int q = 0;
+          for (; q < per - 1; ++q) {
+            run += s_hist[kFineBins - 1 - (per * lane + q)];
+            if (run >= n) break;
+          }
+          s_bstar = kFineBins - 1 - (per * lane + q);
+        }
+      }
+      if (lane == 0) s_n = 0;
+    }
+    __syncthreads();
+    const int bstar = s_bstar;
+    if (bstar < 0 && tid == 0) atomicOr(P.status, kStatusInternal);
+    const int bmin = max(bstar, 0);
+    for (int x = tid; x < cnt; x += blockDim.x) {
+      const float s = cs[x];
+      if (s >= lo && fbin(s) >= bmin) {
+        const int pos = atomicAdd(&s_n, 1);
+        if (pos < kSelCap) skeys[pos] = cand_key(s, ci[x]);
+      }
+    }
+    __syncthreads();
+    ns = s_n;
+  }
   if (ns > kSelCap) {
     // Radix select of the n-th largest key, 8 bits at a time from the top.
     if (tid == 0) {
@@ -263,17 +398,24 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
     if (tid == 0) atomicOr(P.status, kStatusInternal);
     n = ns;
   }
-  const int n2 = next_pow2(max(ns, 1));
+  const int n2 = max(64, next_pow2(max(ns, 1)));
   for (int x = ns + tid; x < n2; x += blockDim.x) skeys[x] = 0ull;
   __syncthreads();
-  bitonic_desc(skeys, n2);
+  if (n2 <= 2 * kSelThreads) {
+    bitonic_desc_hybrid(skeys, n2);
+  } else {
+    bitonic_desc(skeys, n2);
+  }
   const float inv_l = 1.0f / Ls;
   for (int r = tid; r < k; r += blockDim.x) {
     if (r < n) {
       const unsigned long long key = skeys[r];
       const float s = ordered_to_float((uint32_t)(key >> 32));
-      tok_out[r] = (int32_t)(~(uint32_t)key);
+      const int32_t id = (int32_t)(~(uint32_t)key);
+      tok_out[r] = id;
       w_out[r] = fast_exp2(s - M) * inv_l;
+      // one vote for the token's unit (integer atomics: exact)
+      if (id >= 0 && id / P.Tu < P.Uh) atomicAdd(&P.votes[id / P.Tu], 1);
     } else {
       tok_out[r] = -1;
       w_out[r] = 0.f;
@@ -292,220 +434,52 @@ cudaError_t launch_select(const Batch& B, int max_lists, cudaStream_t s) {
 }
 
 // ---------------------------------------------------------------------------
-// Unit votes (v_t of Sec. 4.2) and attention mass. Integer atomics only (exact);
-// the mass of unit u sums, over lists in order, 2^(m_u - M) l_u / L, i.e. the
-// normalised weights of all the unit's tokens.
+// Attention mass of every history unit: over lists in a fixed order, the sum of
+// 2^(m_u - M) l_u / L, i.e. the normalised weights of all the unit's tokens. A block
+// covers 32 units; warp w sums lists w, w + 8, ..., then the 8 partial sums are added
+// in warp order (deterministic).
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) k_votes_mass(const __grid_constant__ Batch B,
-                                                    int vote_blocks) {
+constexpr int kMassWarps = 8;
+
+__global__ void __launch_bounds__(kMassWarps * 32) k_mass(const __grid_constant__ Batch B) {
+  __shared__ float part[kMassWarps][32];
   const int pi = blockIdx.y;
   if (pi >= B.n) return;
   const Prob& P = B.p[pi];
   const int n_lists = P.P * P.Hq;
-  if ((int)blockIdx.x < vote_blocks) {
-    const int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (e < (int64_t)n_lists * B.k) {
-      const int32_t tok = P.topk_tok[e];
-      if (tok >= 0 && tok / P.Tu < P.Uh) atomicAdd(&P.votes[tok / P.Tu], 1);
-    }
-    return;
-  }
-  const int u = (blockIdx.x - vote_blocks) * blockDim.x + threadIdx.x;
-  if (u >= P.Uh) return;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int u = blockIdx.x * 32 + lane;
+  if (blockIdx.x * 32 >= P.Uh) return;
   float acc = 0.f;
-  for (int L = 0; L < n_lists; ++L) {
-    const float2 st = P.ustats[(int64_t)L * P.ucap + u];
-    const float2 ml = P.list_ml[L];
-    if (st.x != -INFINITY) acc += st.y * fast_exp2(st.x - ml.x) / ml.y;
+  if (u < P.Uh) {
+#pragma unroll 4
+    for (int L = warp; L < n_lists; L += kMassWarps) {
+      const float2 st = P.ustats[(int64_t)L * P.ucap + u];
+      const float2 ml = P.list_ml[L];
+      if (st.x != -INFINITY) acc += st.y * fast_exp2(st.x - ml.x) / ml.y;
+    }
   }
-  P.mass[u] = acc;
+  part[warp][lane] = acc;
+  __syncthreads();
+  if (warp == 0 && u < P.Uh) {
+    float m = 0.f;
+#pragma unroll
+    for (int w = 0; w < kMassWarps; ++w) m += part[w][lane];
+    P.mass[u] = m;
+  }
 }
 
-cudaError_t launch_votes_mass(const Batch& B, int max_lists, int max_hist_units,
-                              cudaStream_t s) {
-  const int vote_blocks = (int)(((int64_t)max_lists * B.k + 255) / 256);
-  const int mass_blocks = (max_hist_units + 255) / 256;
-  if (vote_blocks + mass_blocks == 0) return cudaSuccess;
-  dim3 grid(vote_blocks + mass_blocks, B.n);
-  k_votes_mass<<<grid, 256, 0, s>>>(B, vote_blocks);
+cudaError_t launch_mass(const Batch& B, int max_hist_units, cudaStream_t s) {
+  const int blocks = (max_hist_units + 31) / 32;
+  if (blocks == 0) return cudaSuccess;
+  dim3 grid(blocks, B.n);
+  k_mass<<<grid, kMassWarps * 32, 0, s>>>(B);
   return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------------------
 // Vote-ranked pool: all history units sorted in shared memory by
 // (votes desc, mass desc, id asc); the first pool_n are the pool.
-// ---------------------------------------------------------------------------
-__device__ __forceinline__ bool unit_before(unsigned long long ka, int ia,
-                                            unsigned long long kb, int ib) {
-  return ka > kb || (ka == kb && ia < ib);
-}
-
-__global__ void __launch_bounds__(1024) k_pool(const __grid_constant__ Batch B) {
-  extern __shared__ unsigned char smem_raw[];
-  const Prob& P = B.p[blockIdx.x];
-  const int Uh = P.Uh;
-  const int n2 = next_pow2(max(Uh, 1));
-  unsigned long long* keys = reinterpret_cast<unsigned long long*>(smem_raw);
-  int* ids = reinterpret_cast<int*>(keys + n2);
-  for (int x = threadIdx.x; x < n2; x += blockDim.x) {
-    if (x < Uh) {
-      keys[x] = ((unsigned long long)(uint32_t)P.votes[x] << 32) | __float_as_uint(P.mass[x]);
-      ids[x] = x;
-    } else {
-      keys[x] = 0ull;
-      ids[x] = 0x7fffffff;
-    }
-  }
-  __syncthreads();
-  for (int size = 2; size <= n2; size <<= 1) {
-    for (int stride = size >> 1; stride > 0; stride >>= 1) {
-      for (int t = threadIdx.x; t < (n2 >> 1); t += blockDim.x) {
-        const int i = 2 * t - (t & (stride - 1));
-        const int j = i + stride;
-        const bool first_half = (i & size) == 0;
-        const unsigned long long ki = keys[i], kj = keys[j];
-        const int ii = ids[i], ij = ids[j];
-        // first_half: entry i must come before j in the final order
-        const bool swap = first_half ? unit_before(kj, ij, ki, ii) : unit_before(ki, ii, kj, ij);
-        if (swap) {
-          keys[i] = kj;
-          keys[j] = ki;
-          ids[i] = ij;
-          ids[j] = ii;
-        }
-      }
-      __syncthreads();
-    }
-  }
-  for (int r = threadIdx.x; r < P.pool_n; r += blockDim.x) P.pool[r] = ids[r];
-  if (threadIdx.x == 0) P.counts[0] = P.pool_n;
-}
-
-cudaError_t launch_pool(const Batch& B, int max_hist_units, cudaStream_t s) {
-  int n2 = 1;
-  while (n2 < max_hist_units) n2 <<= 1;
-  const int smem = n2 * (int)(sizeof(unsigned long long) + sizeof(int));
-  cudaError_t e = cudaFuncSetAttribute(k_pool, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  if (e != cudaSuccess) return e;
-  k_pool<<<B.n, 1024, smem, s>>>(B);
-  return cudaGetLastError();
-}
-
-// ---------------------------------------------------------------------------
-// Max-min diversity (DivTopK): Gram matrix of the pool's descriptors, then the
-// greedy rule. Start from the pool's best unit; each step adds the unselected unit
-// whose smallest distance 1 - k_c . k_s to the picks is largest, ties to the better
-// pool rank.
-// ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) k_gram(const __grid_constant__ Batch B) {
-  const Prob& P = B.p[blockIdx.z];
-  const int pn = P.pool_n;
-  const int dim = P.Hkv * kHeadDim;
-  const int a0 = blockIdx.y * 32, b0 = blockIdx.x * 32;
-  if (a0 >= pn || b0 >= pn) return;
-  __shared__ float As[32][33], Bs[32][33];
-  __shared__ int pa[32], pb[32];
-  const int tx = threadIdx.x, ty = threadIdx.y;
-  if (ty == 0) {
-    pa[tx] = (a0 + tx < pn) ? P.pool[a0 + tx] : -1;
-    pb[tx] = (b0 + tx < pn) ? P.pool[b0 + tx] : -1;
-  }
-  __syncthreads();
-  float acc[4] = {0.f, 0.f, 0.f, 0.f};
-  for (int d0 = 0; d0 < dim; d0 += 32) {
-    for (int r = ty; r < 32; r += 8) {
-      As[r][tx] = pa[r] >= 0 ? P.desc[(int64_t)pa[r] * dim + d0 + tx] : 0.f;
-      Bs[r][tx] = pb[r] >= 0 ? P.desc[(int64_t)pb[r] * dim + d0 + tx] : 0.f;
-    }
-    __syncthreads();
-#pragma unroll 8
-    for (int dd = 0; dd < 32; ++dd) {
-      const float bv = Bs[tx][dd];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) acc[q] = fmaf(As[ty + 8 * q][dd], bv, acc[q]);
-    }
-    __syncthreads();
-  }
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const int a = a0 + ty + 8 * q, bcol = b0 + tx;
-    if (a < pn && bcol < pn) P.gram[(int64_t)a * pn + bcol] = acc[q];
-  }
-}
-
-__global__ void __launch_bounds__(1024) k_maxmin(const __grid_constant__ Batch B) {
-  __shared__ float wv[32];
-  __shared__ int wi[32];
-  __shared__ int s_best;
-  const Prob& P = B.p[blockIdx.x];
-  const int pn = P.pool_n, ns = P.n_sel;
-  const int r = threadIdx.x, lane = r & 31, warp = r >> 5;
-  const int nw = blockDim.x >> 5;
-  const bool act = r < pn;
-  float mind = act ? 1.0f - P.gram[r] : -INFINITY;
-  bool taken = (r == 0);
-  if (r == 0 && ns > 0) P.sel[0] = P.pool[0];
-  for (int step = 1; step < ns; ++step) {
-    float v = -INFINITY;
-    int idx = 0x7fffffff;
-    if (act && !taken) {
-      v = (mind == mind) ? mind : -3.0e38f;  // NaN descriptors rank last
-      idx = r;
-    }
-    for (int off = 16; off > 0; off >>= 1) {
-      const float vo = __shfl_down_sync(0xffffffffu, v, off);
-      const int io = __shfl_down_sync(0xffffffffu, idx, off);
-      if (vo > v || (vo == v && io < idx)) {
-        v = vo;
-        idx = io;
-      }
-    }
-    if (lane == 0) {
-      wv[warp] = v;
-      wi[warp] = idx;
-    }
-    __syncthreads();
-    if (warp == 0) {
-      v = lane < nw ? wv[lane] : -INFINITY;
-      idx = lane < nw ? wi[lane] : 0x7fffffff;
-      for (int off = 16; off > 0; off >>= 1) {
-        const float vo = __shfl_down_sync(0xffffffffu, v, off);
-        const int io = __shfl_down_sync(0xffffffffu, idx, off);
-        if (vo > v || (vo == v && io < idx)) {
-          v = vo;
-          idx = io;
-        }
-      }
-      if (lane == 0) s_best = idx;
-    }
-    __syncthreads();
-    const int best = s_best;
-    if (best < 0 || best >= pn) {
-      if (r == 0) atomicOr(P.status, kStatusInternal);
-      break;
-    }
-    if (r == best) taken = true;
-    if (r == 0) P.sel[step] = P.pool[best];
-    if (act) mind = fminf(mind, 1.0f - P.gram[(int64_t)best * pn + r]);
-  }
-}
-
-cudaError_t launch_maxmin(const Batch& B, int max_pool, cudaStream_t s) {
-  if (max_pool > 0) {
-    const int tiles = (max_pool + 31) / 32;
-    dim3 grid(tiles, tiles, B.n);
-    k_gram<<<grid, dim3(32, 8), 0, s>>>(B);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-  }
-  k_maxmin<<<B.n, 1024, 0, s>>>(B);
-  return cudaGetLastError();
-}
-
-// ---------------------------------------------------------------------------
-// Temporal expansion (Nbr of Eq. 12) with deduplication and temporal ordering: a
-// bitmap over history units marks every pick and its n_prev predecessors; an ordered
-// compaction lists the marked units ascending and their frames.
 // ---------------------------------------------------------------------------
 __device__ int block_excl_scan(int v, int* sw) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -530,24 +504,278 @@ __device__ int block_excl_scan(int v, int* sw) {
   return prefix + x - v;
 }
 
-__global__ void __launch_bounds__(1024) k_expand(const __grid_constant__ Batch B) {
+__device__ __forceinline__ bool unit_before(unsigned long long ka, int ia,
+                                            unsigned long long kb, int ib) {
+  return ka > kb || (ka == kb && ia < ib);
+}
+
+constexpr int kVoteBins = 4096;
+constexpr int kRankMax = 1024;   // candidates ranked by pairwise comparison
+
+__global__ void __launch_bounds__(1024) k_pool(const __grid_constant__ Batch B) {
+  extern __shared__ unsigned char smem_raw[];
+  __shared__ int vh[kVoteBins];
+  __shared__ int sw[32];
+  __shared__ int s_v, s_c;
+  const Prob& P = B.p[blockIdx.x];
+  const int Uh = P.Uh, pn = P.pool_n;
+  const int tid = threadIdx.x;
+  if (tid == 0) P.counts[0] = pn;
+  if (pn == 0) return;
+  // (1) histogram of votes (clipped): the pool's smallest vote level V is the highest
+  //     level whose units and all better ones number at least pool_n
+  for (int x = tid; x < kVoteBins; x += blockDim.x) vh[x] = 0;
+  if (tid == 0) s_c = 0;
+  __syncthreads();
+  for (int u = tid; u < Uh; u += blockDim.x) atomicAdd(&vh[min(P.votes[u], kVoteBins - 1)], 1);
+  __syncthreads();
+  {
+    constexpr int per = kVoteBins / 1024;   // 4 levels per thread, thread 0 the top ones
+    int c = 0;
+    for (int q = 0; q < per; ++q) c += vh[kVoteBins - 1 - (per * tid + q)];
+    const int incl = block_excl_scan(c, sw) + c;
+    if (incl >= pn && incl - c < pn) {
+      int run = incl - c, q = 0;
+      for (; q < per - 1; ++q) {
+        run += vh[kVoteBins - 1 - (per * tid + q)];
+        if (run >= pn) break;
+      }
+      s_v = kVoteBins - 1 - (per * tid + q);
+    }
+  }
+  __syncthreads();
+  const int V = s_v;
+  // (2) the units at or above level V, ranked by (votes desc, mass desc, id asc)
+  unsigned long long* ck = reinterpret_cast<unsigned long long*>(smem_raw);
+  int* ci = reinterpret_cast<int*>(ck + kRankMax);
+  for (int u = tid; u < Uh; u += blockDim.x) {
+    if (min(P.votes[u], kVoteBins - 1) >= V) {
+      const int pos = atomicAdd(&s_c, 1);
+      if (pos < kRankMax) {
+        ck[pos] = ((unsigned long long)(uint32_t)P.votes[u] << 32) | __float_as_uint(P.mass[u]);
+        ci[pos] = u;
+      }
+    }
+  }
+  __syncthreads();
+  const int C = s_c;
+  if (C <= kRankMax) {
+    if (tid < C) {
+      const unsigned long long mk = ck[tid];
+      const int mi = ci[tid];
+      int rank = 0;
+      for (int o = 0; o < C; ++o) rank += unit_before(ck[o], ci[o], mk, mi) ? 1 : 0;
+      if (rank < pn) P.pool[rank] = mi;
+    }
+    return;
+  }
+  // (3) too many ties at level V: sort every history unit
+  const int n2 = next_pow2(max(Uh, 1));
+  unsigned long long* keys = reinterpret_cast<unsigned long long*>(smem_raw);
+  int* ids = reinterpret_cast<int*>(keys + n2);
+  __syncthreads();
+  for (int x = tid; x < n2; x += blockDim.x) {
+    if (x < Uh) {
+      keys[x] = ((unsigned long long)(uint32_t)P.votes[x] << 32) | __float_as_uint(P.mass[x]);
+      ids[x] = x;
+    } else {
+      keys[x] = 0ull;
+      ids[x] = 0x7fffffff;
+    }
+  }
+  __syncthreads();
+  for (int size = 2; size <= n2; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int t = tid; t < (n2 >> 1); t += blockDim.x) {
+        const int i = 2 * t - (t & (stride - 1));
+        const int j = i + stride;
+        const bool first_half = (i & size) == 0;
+        const unsigned long long ki = keys[i], kj = keys[j];
+        const int ii = ids[i], ij = ids[j];
+        const bool swap = first_half ? unit_before(kj, ij, ki, ii) : unit_before(ki, ii, kj, ij);
+        if (swap) {
+          keys[i] = kj;
+          keys[j] = ki;
+          ids[i] = ij;
+          ids[j] = ii;
+        }
+      }
+      __syncthreads();
+    }
+  }
+  for (int r = tid; r < pn; r += blockDim.x) P.pool[r] = ids[r];
+}
+
+cudaError_t launch_pool(const Batch& B, int max_hist_units, cudaStream_t s) {
+  int n2 = 1;
+  while (n2 < max_hist_units) n2 <<= 1;
+  const int smem = max(n2, kRankMax) * (int)(sizeof(unsigned long long) + sizeof(int));
+  cudaError_t e = cudaFuncSetAttribute(k_pool, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  k_pool<<<B.n, 1024, smem, s>>>(B);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Max-min diversity (DivTopK): Gram matrix of the pool's descriptors, then the
+// greedy rule. Start from the pool's best unit; each step adds the unselected unit
+// whose smallest distance 1 - k_c . k_s to the picks is largest, ties to the better
+// pool rank.
+// ---------------------------------------------------------------------------
+// Gram matrix of the pool's descriptors, stored as its packed upper triangle
+// (row a holds G[a][a..pool)). One 16 x 16 tile of the upper triangle per CTA, rows
+// staged in shared memory with a one-float pad per row.
+constexpr int kGramTile = 16;
+
+__device__ __forceinline__ int tri_off(int a, int pn) { return a * pn - (a * (a - 1)) / 2; }
+
+__global__ void __launch_bounds__(256) k_gram(const __grid_constant__ Batch B) {
+  extern __shared__ float gsm[];
+  const Prob& P = B.p[blockIdx.y];
+  const int pn = P.pool_n;
+  const int dim = P.Hkv * kHeadDim;
+  const int T = (pn + kGramTile - 1) / kGramTile;
+  int ta = 0, rem = blockIdx.x;  // blockIdx.x -> tile (ta, tb), ta <= tb
+  while (ta < T && rem >= T - ta) {
+    rem -= T - ta;
+    ++ta;
+  }
+  if (ta >= T) return;
+  const int tb = ta + rem;
+  const int ld = dim + 1;
+  float* A = gsm;
+  float* Bm = gsm + kGramTile * ld;
+  __shared__ int ua[kGramTile], ub[kGramTile];
+  if (threadIdx.x < kGramTile) {
+    const int a = ta * kGramTile + threadIdx.x, b = tb * kGramTile + threadIdx.x;
+    ua[threadIdx.x] = a < pn ? P.pool[a] : -1;
+    ub[threadIdx.x] = b < pn ? P.pool[b] : -1;
+  }
+  __syncthreads();
+  const int d4 = dim / 4;
+  for (int x = threadIdx.x; x < kGramTile * d4; x += blockDim.x) {
+    const int r = x / d4, e = 4 * (x - r * d4);
+    const float4 va = ua[r] >= 0 ? *reinterpret_cast<const float4*>(P.desc + (int64_t)ua[r] * dim + e)
+                                 : make_float4(0.f, 0.f, 0.f, 0.f);
+    const float4 vb = ub[r] >= 0 ? *reinterpret_cast<const float4*>(P.desc + (int64_t)ub[r] * dim + e)
+                                 : make_float4(0.f, 0.f, 0.f, 0.f);
+    float* pa = A + r * ld + e;
+    float* pb = Bm + r * ld + e;
+    pa[0] = va.x; pa[1] = va.y; pa[2] = va.z; pa[3] = va.w;
+    pb[0] = vb.x; pb[1] = vb.y; pb[2] = vb.z; pb[3] = vb.w;
+  }
+  __syncthreads();
+  const int r = threadIdx.x / kGramTile, c = threadIdx.x % kGramTile;
+  float acc = 0.f;
+  for (int d = 0; d < dim; ++d) acc = fmaf(A[r * ld + d], Bm[c * ld + d], acc);
+  const int a = ta * kGramTile + r, b = tb * kGramTile + c;
+  if (a < pn && b < pn && a <= b) P.gram[tri_off(a, pn) + (b - a)] = acc;
+}
+
+// Greedy max-min (DivTopK) by one warp over the packed Gram triangle (in shared memory
+// when it fits), then the expansion (Nbr of Eq. 12) by the whole block. Lane l owns
+// the pool ranks l, l + 32, ...; kPer = ranks per lane.
+constexpr int kMaxMinSmemPool = 320;   // packed triangle of 320 ranks = 201 KB
+constexpr int kMaxMinThreads = kMaxHistUnits / 32;  // one bitmap word per thread
+
+template <int kPer>
+__device__ void greedy_maxmin(const Prob& P, const float* pk, const int* pool, int* sel,
+                              int pn, int ns) {
+  const int lane = threadIdx.x & 31;
+  float mind[kPer];
+  int toff[kPer];  // start of candidate c's row in the packed triangle
+#pragma unroll
+  for (int q = 0; q < kPer; ++q) {
+    const int c = lane + 32 * q;
+    toff[q] = tri_off(c, pn);
+    mind[q] = c < pn ? 1.0f - pk[c] : -INFINITY;  // row 0 of the triangle is G[0][*]
+  }
+  uint32_t taken = lane == 0 ? 1u : 0u;  // bit q: rank lane + 32 q is picked
+  if (lane == 0) sel[0] = pool[0];
+  for (int step = 1; step < ns; ++step) {
+    // best distance over the unpicked ranks, then the smallest rank holding it; distances
+    // are >= 0 (or NaN, which ranks last), so their bit patterns order as unsigned ints
+    uint32_t bv = 0u;
+    int bi = 0x7fffffff;
+#pragma unroll
+    for (int q = 0; q < kPer; ++q) {
+      const int c = lane + 32 * q;
+      if (c < pn && !((taken >> q) & 1u)) {
+        const float m = mind[q];
+        const uint32_t v = (m == m) ? __float_as_uint(fmaxf(m, 0.0f)) + 1u : 0u;
+        if (v > bv) {  // ranks ascend with q: ties keep the smaller rank
+          bv = v;
+          bi = c;
+        }
+      }
+    }
+    const uint32_t best_v = __reduce_max_sync(0xffffffffu, bv);
+    const int best = (int)__reduce_min_sync(0xffffffffu, bv == best_v ? (uint32_t)bi : 0x7fffffffu);
+    if (best < 0 || best >= pn) {
+      if (lane == 0) atomicOr(P.status, kStatusInternal);
+      return;
+    }
+    if ((best & 31) == lane) taken |= 1u << (best >> 5);
+    if (lane == 0) sel[step] = pool[best];
+    // row best of the triangle: ranks >= best are contiguous, ranks < best sit in
+    // column best of their own rows
+    const int rowoff = tri_off(best, pn) - best;
+#pragma unroll
+    for (int q = 0; q < kPer; ++q) {
+      const int c = lane + 32 * q;
+      if (c < pn) {
+        const float g = c >= best ? pk[rowoff + c] : pk[toff[q] + best - c];
+        mind[q] = fminf(mind[q], 1.0f - g);
+      }
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kMaxMinThreads) k_maxmin(const __grid_constant__ Batch B) {
+  extern __shared__ float4 pks4[];
   __shared__ uint32_t bits[kMaxHistUnits / 32];
   __shared__ int sw[32];
+  __shared__ int spool[kMaxPool];
+  __shared__ int ssel[kMaxPool];
   const Prob& P = B.p[blockIdx.x];
+  const int pn = P.pool_n, ns = P.n_sel;
+  const int tid = threadIdx.x, warp = tid >> 5;
+  const bool in_smem = pn <= kMaxMinSmemPool;
+  const float* pk = P.gram;
+  for (int x = tid; x < pn; x += blockDim.x) spool[x] = P.pool[x];
+  if (in_smem) {
+    const int total4 = (tri_off(pn, pn) + 3) / 4;
+    const float4* g4 = reinterpret_cast<const float4*>(P.gram);
+    for (int x = tid; x < total4; x += blockDim.x) pks4[x] = g4[x];
+    pk = reinterpret_cast<const float*>(pks4);
+  }
+  __syncthreads();
+  if (warp == 0 && ns > 0) {
+    const int per = (pn + 31) / 32;
+    if (per <= 1) greedy_maxmin<1>(P, pk, spool, ssel, pn, ns);
+    else if (per <= 2) greedy_maxmin<2>(P, pk, spool, ssel, pn, ns);
+    else if (per <= 4) greedy_maxmin<4>(P, pk, spool, ssel, pn, ns);
+    else if (per <= 8) greedy_maxmin<8>(P, pk, spool, ssel, pn, ns);
+    else if (per <= 16) greedy_maxmin<16>(P, pk, spool, ssel, pn, ns);
+    else greedy_maxmin<32>(P, pk, spool, ssel, pn, ns);
+  }
+  __syncthreads();
+  for (int r = tid; r < ns; r += blockDim.x) P.sel[r] = ssel[r];
+
+  // expansion: each pick and its n_prev predecessors, deduplicated, ascending
   const int Uh = P.Uh;
   const int nwords = (Uh + 31) >> 5;
-  for (int x = threadIdx.x; x < nwords; x += blockDim.x) bits[x] = 0u;
+  for (int x = tid; x < nwords; x += blockDim.x) bits[x] = 0u;
   __syncthreads();
-  for (int r = threadIdx.x; r < P.n_sel; r += blockDim.x) {
-    const int u = P.sel[r];
+  for (int r = tid; r < ns; r += blockDim.x) {
+    const int u = ssel[r];
     for (int j = 0; j <= B.n_prev; ++j) {
       const int v = u - j;
       if (v >= 0 && v < Uh) atomicOr(&bits[v >> 5], 1u << (v & 31));
     }
   }
   __syncthreads();
-  const int w = threadIdx.x;
-  const uint32_t word = (w < nwords) ? bits[w] : 0u;
+  const uint32_t word = (tid < nwords) ? bits[tid] : 0u;
   const int c = __popc(word);
   const int off = block_excl_scan(c, sw);
   uint32_t rest = word;
@@ -555,21 +783,37 @@ __global__ void __launch_bounds__(1024) k_expand(const __grid_constant__ Batch B
   while (rest) {
     const int bpos = __ffs(rest) - 1;
     rest &= rest - 1u;
-    const int u = w * 32 + bpos;
+    const int u = tid * 32 + bpos;
     P.exp_units[q] = u;
     for (int f = 0; f < P.fpu; ++f) P.frames[q * P.fpu + f] = u * P.fpu + f;
     ++q;
   }
-  if (threadIdx.x == blockDim.x - 1) {
+  if (tid == blockDim.x - 1) {
     const int total = off + c;
-    P.counts[1] = P.n_sel;
+    P.counts[1] = ns;
     P.counts[2] = total;
     P.counts[3] = total * P.fpu;
   }
 }
 
-cudaError_t launch_expand(const Batch& B, cudaStream_t s) {
-  k_expand<<<B.n, 1024, 0, s>>>(B);
+cudaError_t launch_maxmin(const Batch& B, int max_pool, cudaStream_t s) {
+  int max_dim = 0;
+  for (int j = 0; j < B.n; ++j) max_dim = max(max_dim, B.p[j].Hkv * kHeadDim);
+  if (max_pool > 0) {
+    const int T = (max_pool + kGramTile - 1) / kGramTile;
+    const int smem = 2 * kGramTile * (max_dim + 1) * (int)sizeof(float);
+    cudaError_t e = cudaFuncSetAttribute(k_gram, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    dim3 grid(T * (T + 1) / 2, B.n);
+    k_gram<<<grid, kGramTile * kGramTile, smem, s>>>(B);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  const int pk_n = max_pool <= kMaxMinSmemPool ? max_pool * (max_pool + 1) / 2 : 0;
+  const int smem = ((max(pk_n, 1) + 3) / 4) * (int)sizeof(float4);
+  cudaError_t e = cudaFuncSetAttribute(k_maxmin, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  k_maxmin<<<B.n, kMaxMinThreads, smem, s>>>(B);
   return cudaGetLastError();
 }
 
