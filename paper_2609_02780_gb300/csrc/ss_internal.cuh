@@ -30,6 +30,12 @@ constexpr int kScoreThreads = (kScoreWarps + 1) * 32;
 #define SS_SCORE_CTAS_PER_SM 2
 #endif
 constexpr int kScoreCtasPerSm = SS_SCORE_CTAS_PER_SM;
+// registers per thread that still fit kScoreCtasPerSm CTAs per SM (64K registers,
+// allocated per warp in multiples of 8 per thread)
+constexpr int kScoreMaxRegs =
+    (65536 / (kScoreCtasPerSm * (kScoreWarps + 1) * 32)) / 8 * 8 > 255
+        ? 255
+        : (65536 / (kScoreCtasPerSm * (kScoreWarps + 1) * 32)) / 8 * 8;
 #ifndef SS_SCORE_STAGES
 #define SS_SCORE_STAGES 3
 #endif

@@ -145,6 +145,8 @@ __device__ __forceinline__ uint4 ld_stream(const void* p) {
   return r;
 }
 
+constexpr int kDefer = 4;  // warm-up tiles per warp whose appends wait for a threshold
+
 struct ScoreShared {
   int lad[kMaxGroup][kLadderLevels];  // this CTA's appended-score counts not yet merged
   float thr[kMaxGroup];
@@ -293,11 +295,11 @@ __device__ void threshold_warp(ScoreShared& S, const Prob& P, int list0, int k) 
     }
     __syncwarp();
     if (done >= kScoreWarps) break;
-    __nanosleep(128);
+    __nanosleep(iter < 32 ? 128 : 1024);
   }
 }
 
-__global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
+__global__ void __maxnreg__(kScoreMaxRegs)
     k_score(const __grid_constant__ Batch B) {
   __shared__ ScoreShared S;
   extern __shared__ __align__(128) unsigned char tiles[];  // [warp][stage][kTileBytes]
@@ -375,6 +377,84 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
   // Candidate slots reserved for this lane group's two lists (identical in its 8 lanes).
   int rp0 = 0, rl0 = 0, rp1 = 0, rl1 = 0;
 
+  // Appends the scores of keys tok0 (row g) and tok0 + 8 (row g + 8) that reach the
+  // current thresholds, counting them in the ladder when `count` (a warm-up score was
+  // counted when it was scored).
+  auto append = [&](float s00, float s01, float s10, float s11, int tok0, bool v0, bool v1,
+                    bool count) {
+    const float thr0 = hv0 ? vthr[c0] : INFINITY;
+    const float thr1 = hv1 ? vthr[c1] : INFINITY;
+    const bool p00 = hv0 && v0 && s00 >= thr0, p10 = hv0 && v1 && s10 >= thr0;
+    const bool p01 = hv1 && v0 && s01 >= thr1, p11 = hv1 && v1 && s11 >= thr1;
+    if (!__any_sync(0xffffffffu, p00 | p01 | p10 | p11)) return;
+    const int tok1 = tok0 + 8;
+    const unsigned b00 = __ballot_sync(0xffffffffu, p00) & gmask;
+    const unsigned b10 = __ballot_sync(0xffffffffu, p10) & gmask;
+    const unsigned b01 = __ballot_sync(0xffffffffu, p01) & gmask;
+    const unsigned b11 = __ballot_sync(0xffffffffu, p11) & gmask;
+    const int n0 = __popc(b00) + __popc(b10), n1 = __popc(b01) + __popc(b11);
+    // slots: continue the reserved block, reserve a new one when it runs out
+    const bool need0 = n0 > rl0, need1 = n1 > rl1;
+    int nb0 = 0, nb1 = 0;
+    if (g == 0 && need0) nb0 = atomicAdd(P.cand_cnt + L0, kReserve);
+    if (g == 0 && need1) nb1 = atomicAdd(P.cand_cnt + L1, kReserve);
+    nb0 = __shfl_sync(0xffffffffu, nb0, t4);
+    nb1 = __shfl_sync(0xffffffffu, nb1, t4);
+    auto slot0 = [&](int r) { return cbase0 + (r < rl0 ? rp0 + r : nb0 + (r - rl0)); };
+    auto slot1 = [&](int r) { return cbase1 + (r < rl1 ? rp1 + r : nb1 + (r - rl1)); };
+    if (p00) {
+      const int64_t pos = slot0(__popc(b00 & lt_mask));
+      P.cand_s[pos] = s00;
+      P.cand_id[pos] = tok0;
+      if (count) ladder_add(S, c0, s00, an0);
+    }
+    if (p10) {
+      const int64_t pos = slot0(__popc(b00) + __popc(b10 & lt_mask));
+      P.cand_s[pos] = s10;
+      P.cand_id[pos] = tok1;
+      if (count) ladder_add(S, c0, s10, an0);
+    }
+    if (p01) {
+      const int64_t pos = slot1(__popc(b01 & lt_mask));
+      P.cand_s[pos] = s01;
+      P.cand_id[pos] = tok0;
+      if (count) ladder_add(S, c1, s01, an1);
+    }
+    if (p11) {
+      const int64_t pos = slot1(__popc(b01) + __popc(b11 & lt_mask));
+      P.cand_s[pos] = s11;
+      P.cand_id[pos] = tok1;
+      if (count) ladder_add(S, c1, s11, an1);
+    }
+    if (need0) {
+      rp0 = nb0 + (n0 - rl0);
+      rl0 = kReserve - (n0 - rl0);
+    } else {
+      rp0 += n0;
+      rl0 -= n0;
+    }
+    if (need1) {
+      rp1 = nb1 + (n1 - rl1);
+      rl1 = kReserve - (n1 - rl1);
+    } else {
+      rp1 += n1;
+      rl1 -= n1;
+    }
+  };
+
+  // The first kDefer tiles of the warp are scored before any threshold exists; their
+  // scores wait in registers and are appended once the ladder has had time to fill.
+  float ds[kDefer][4];
+  int dtok[kDefer];  // bit 0 / 1: rows g / g + 8 valid; token of row g in bits 2..
+  auto flush_deferred = [&](int nd) {
+#pragma unroll
+    for (int q = 0; q < kDefer; ++q) {
+      if (q < nd)
+        append(ds[q][0], ds[q][1], ds[q][2], ds[q][3], dtok[q] >> 2, (dtok[q] & 1) != 0,
+               (dtok[q] & 2) != 0, false);
+    }
+  };
+
   // Lane 0 starts the bulk copy of tile t (unit uu, tile jj of the unit) into its
   // stage once the warp's reads of that stage are ordered before the async write.
   auto issue = [&](int t, int uu, int jj) {
@@ -441,71 +521,29 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
       m0 = m1 = -INFINITY;
       l0 = l1 = 0.f;
     }
-    const float thr0 = hv0 ? vthr[c0] : INFINITY;
-    const float thr1 = hv1 ? vthr[c1] : INFINITY;
     const int r0 = kTileRows * j + g;
     const bool v0 = r0 < Tu, v1 = r0 + 8 < Tu;
     const float s00 = (acc[0] + acd[0]) * kScoreScale, s01 = (acc[1] + acd[1]) * kScoreScale;
     const float s10 = (acc[2] + acd[2]) * kScoreScale, s11 = (acc[3] + acd[3]) * kScoreScale;
     stats_update(m0, l0, s00, v0, s10, v1);
     stats_update(m1, l1, s01, v0, s11, v1);
-
-    const bool p00 = hv0 && v0 && s00 >= thr0, p10 = hv0 && v1 && s10 >= thr0;
-    const bool p01 = hv1 && v0 && s01 >= thr1, p11 = hv1 && v1 && s11 >= thr1;
-    if (__any_sync(0xffffffffu, p00 | p01 | p10 | p11)) {
-      const int tok0 = u * Tu + r0, tok1 = tok0 + 8;
-      const unsigned b00 = __ballot_sync(0xffffffffu, p00) & gmask;
-      const unsigned b10 = __ballot_sync(0xffffffffu, p10) & gmask;
-      const unsigned b01 = __ballot_sync(0xffffffffu, p01) & gmask;
-      const unsigned b11 = __ballot_sync(0xffffffffu, p11) & gmask;
-      const int n0 = __popc(b00) + __popc(b10), n1 = __popc(b01) + __popc(b11);
-      // slots: continue the reserved block, reserve a new one when it runs out
-      const bool need0 = n0 > rl0, need1 = n1 > rl1;
-      int nb0 = 0, nb1 = 0;
-      if (g == 0 && need0) nb0 = atomicAdd(P.cand_cnt + L0, kReserve);
-      if (g == 0 && need1) nb1 = atomicAdd(P.cand_cnt + L1, kReserve);
-      nb0 = __shfl_sync(0xffffffffu, nb0, t4);
-      nb1 = __shfl_sync(0xffffffffu, nb1, t4);
-      auto slot0 = [&](int r) { return cbase0 + (r < rl0 ? rp0 + r : nb0 + (r - rl0)); };
-      auto slot1 = [&](int r) { return cbase1 + (r < rl1 ? rp1 + r : nb1 + (r - rl1)); };
-      if (p00) {
-        const int64_t pos = slot0(__popc(b00 & lt_mask));
-        P.cand_s[pos] = s00;
-        P.cand_id[pos] = tok0;
-        ladder_add(S, c0, s00, an0);
+    const int tok0 = u * Tu + r0;
+    if (t < kDefer) {
+      // warm-up: count every score in the ladder now, decide the appends later
+      if (hv0 && v0) ladder_add(S, c0, s00, an0);
+      if (hv0 && v1) ladder_add(S, c0, s10, an0);
+      if (hv1 && v0) ladder_add(S, c1, s01, an1);
+      if (hv1 && v1) ladder_add(S, c1, s11, an1);
+#pragma unroll
+      for (int q = 0; q < kDefer; ++q) {
+        if (q == t) {
+          ds[q][0] = s00; ds[q][1] = s01; ds[q][2] = s10; ds[q][3] = s11;
+          dtok[q] = (v0 ? 1 : 0) | (v1 ? 2 : 0) | (tok0 << 2);
+        }
       }
-      if (p10) {
-        const int64_t pos = slot0(__popc(b00) + __popc(b10 & lt_mask));
-        P.cand_s[pos] = s10;
-        P.cand_id[pos] = tok1;
-        ladder_add(S, c0, s10, an0);
-      }
-      if (p01) {
-        const int64_t pos = slot1(__popc(b01 & lt_mask));
-        P.cand_s[pos] = s01;
-        P.cand_id[pos] = tok0;
-        ladder_add(S, c1, s01, an1);
-      }
-      if (p11) {
-        const int64_t pos = slot1(__popc(b01) + __popc(b11 & lt_mask));
-        P.cand_s[pos] = s11;
-        P.cand_id[pos] = tok1;
-        ladder_add(S, c1, s11, an1);
-      }
-      if (need0) {
-        rp0 = nb0 + (n0 - rl0);
-        rl0 = kReserve - (n0 - rl0);
-      } else {
-        rp0 += n0;
-        rl0 -= n0;
-      }
-      if (need1) {
-        rp1 = nb1 + (n1 - rl1);
-        rl1 = kReserve - (n1 - rl1);
-      } else {
-        rp1 += n1;
-        rl1 -= n1;
-      }
+      if (t == kDefer - 1) flush_deferred(kDefer);
+    } else {
+      append(s00, s01, s10, s11, tok0, v0, v1, true);
     }
     if (j == tpu - 1) {
 #pragma unroll
@@ -523,6 +561,7 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
       }
     }
   }
+  if (!aborted && ntiles < kDefer) flush_deferred(ntiles);
   // unused reserved slots are marked empty (score -inf)
   for (int x = g; x < rl0; x += 8) P.cand_s[cbase0 + rp0 + x] = -INFINITY;
   for (int x = g; x < rl1; x += 8) P.cand_s[cbase1 + rp1 + x] = -INFINITY;

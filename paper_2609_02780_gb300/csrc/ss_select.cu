@@ -695,22 +695,32 @@ __device__ void greedy_maxmin(const Prob& P, const float* pk, const int* pool, i
   for (int step = 1; step < ns; ++step) {
     // best distance over the unpicked ranks, then the smallest rank holding it; distances
     // are >= 0 (or NaN, which ranks last), so their bit patterns order as unsigned ints
-    uint32_t bv = 0u;
-    int bi = 0x7fffffff;
+    uint32_t vv[kPer];
+    int ii[kPer];
 #pragma unroll
     for (int q = 0; q < kPer; ++q) {
       const int c = lane + 32 * q;
-      if (c < pn && !((taken >> q) & 1u)) {
-        const float m = mind[q];
-        const uint32_t v = (m == m) ? __float_as_uint(fmaxf(m, 0.0f)) + 1u : 0u;
-        if (v > bv) {  // ranks ascend with q: ties keep the smaller rank
-          bv = v;
-          bi = c;
+      const float m = mind[q];
+      vv[q] = (c < pn && !((taken >> q) & 1u) && m == m)  // NaN ranks last
+                  ? __float_as_uint(fmaxf(m, 0.0f)) + 1u
+                  : 0u;
+      ii[q] = c;
+    }
+    // pairwise (tree) reduction; the lower half keeps ties, i.e. the smaller rank
+#pragma unroll
+    for (int w = 1; w < kPer; w <<= 1) {
+#pragma unroll
+      for (int q = 0; q + w < kPer; q += 2 * w) {
+        if (vv[q + w] > vv[q]) {
+          vv[q] = vv[q + w];
+          ii[q] = ii[q + w];
         }
       }
     }
+    const uint32_t bv = vv[0];
+    const int bi = bv ? ii[0] : 0x7fffffff;
     const uint32_t best_v = __reduce_max_sync(0xffffffffu, bv);
-    const int best = (int)__reduce_min_sync(0xffffffffu, bv == best_v ? (uint32_t)bi : 0x7fffffffu);
+    const int best = (int)__reduce_min_sync(0xffffffffu, (bv == best_v && bv) ? (uint32_t)bi : 0x7fffffffu);
     if (best < 0 || best >= pn) {
       if (lane == 0) atomicOr(P.status, kStatusInternal);
       return;
@@ -734,65 +744,79 @@ __device__ void greedy_maxmin(const Prob& P, const float* pk, const int* pool, i
 __global__ void __launch_bounds__(kMaxMinThreads) k_maxmin(const __grid_constant__ Batch B) {
   extern __shared__ float4 pks4[];
   __shared__ uint32_t bits[kMaxHistUnits / 32];
-  __shared__ int sw[32];
   __shared__ int spool[kMaxPool];
   __shared__ int ssel[kMaxPool];
   const Prob& P = B.p[blockIdx.x];
   const int pn = P.pool_n, ns = P.n_sel;
   const int tid = threadIdx.x, warp = tid >> 5;
   const bool in_smem = pn <= kMaxMinSmemPool;
-  const float* pk = P.gram;
   for (int x = tid; x < pn; x += blockDim.x) spool[x] = P.pool[x];
   if (in_smem) {
     const int total4 = (tri_off(pn, pn) + 3) / 4;
     const float4* g4 = reinterpret_cast<const float4*>(P.gram);
     for (int x = tid; x < total4; x += blockDim.x) pks4[x] = g4[x];
-    pk = reinterpret_cast<const float*>(pks4);
   }
   __syncthreads();
-  if (warp == 0 && ns > 0) {
+  // One warp does the rest: warps parked at a barrier would slow its serial greedy.
+  if (warp != 0) return;
+  const int lane = tid;
+  if (ns > 0) {
+    // separate call sites keep the triangle's address space (shared or global) known
+    // to the compiler, so the greedy's reads are plain shared-memory loads when staged
     const int per = (pn + 31) / 32;
-    if (per <= 1) greedy_maxmin<1>(P, pk, spool, ssel, pn, ns);
-    else if (per <= 2) greedy_maxmin<2>(P, pk, spool, ssel, pn, ns);
-    else if (per <= 4) greedy_maxmin<4>(P, pk, spool, ssel, pn, ns);
-    else if (per <= 8) greedy_maxmin<8>(P, pk, spool, ssel, pn, ns);
-    else if (per <= 16) greedy_maxmin<16>(P, pk, spool, ssel, pn, ns);
-    else greedy_maxmin<32>(P, pk, spool, ssel, pn, ns);
+    if (in_smem) {
+      const float* sk = reinterpret_cast<const float*>(pks4);
+      if (per <= 1) greedy_maxmin<1>(P, sk, spool, ssel, pn, ns);
+      else if (per <= 2) greedy_maxmin<2>(P, sk, spool, ssel, pn, ns);
+      else if (per <= 4) greedy_maxmin<4>(P, sk, spool, ssel, pn, ns);
+      else if (per <= 8) greedy_maxmin<8>(P, sk, spool, ssel, pn, ns);
+      else greedy_maxmin<16>(P, sk, spool, ssel, pn, ns);   // pool <= 320 here
+    } else {
+      if (per <= 16) greedy_maxmin<16>(P, P.gram, spool, ssel, pn, ns);
+      else greedy_maxmin<32>(P, P.gram, spool, ssel, pn, ns);
+    }
   }
-  __syncthreads();
-  for (int r = tid; r < ns; r += blockDim.x) P.sel[r] = ssel[r];
+  __syncwarp();
+  for (int r = lane; r < ns; r += 32) P.sel[r] = ssel[r];
 
   // expansion: each pick and its n_prev predecessors, deduplicated, ascending
   const int Uh = P.Uh;
   const int nwords = (Uh + 31) >> 5;
-  for (int x = tid; x < nwords; x += blockDim.x) bits[x] = 0u;
-  __syncthreads();
-  for (int r = tid; r < ns; r += blockDim.x) {
+  for (int x = lane; x < nwords; x += 32) bits[x] = 0u;
+  __syncwarp();
+  for (int r = lane; r < ns; r += 32) {
     const int u = ssel[r];
     for (int j = 0; j <= B.n_prev; ++j) {
       const int v = u - j;
       if (v >= 0 && v < Uh) atomicOr(&bits[v >> 5], 1u << (v & 31));
     }
   }
-  __syncthreads();
-  const uint32_t word = (tid < nwords) ? bits[tid] : 0u;
-  const int c = __popc(word);
-  const int off = block_excl_scan(c, sw);
-  uint32_t rest = word;
-  int q = off;
-  while (rest) {
-    const int bpos = __ffs(rest) - 1;
-    rest &= rest - 1u;
-    const int u = tid * 32 + bpos;
-    P.exp_units[q] = u;
-    for (int f = 0; f < P.fpu; ++f) P.frames[q * P.fpu + f] = u * P.fpu + f;
-    ++q;
+  __syncwarp();
+  // lane l compacts the words [l * wpl, (l + 1) * wpl) in order
+  const int wpl = (nwords + 31) / 32;
+  int c = 0;
+  for (int x = lane * wpl; x < min(nwords, (lane + 1) * wpl); ++x) c += __popc(bits[x]);
+  int incl = c;
+  for (int off = 1; off < 32; off <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += y;
   }
-  if (tid == blockDim.x - 1) {
-    const int total = off + c;
+  int q = incl - c;
+  for (int x = lane * wpl; x < min(nwords, (lane + 1) * wpl); ++x) {
+    uint32_t rest = bits[x];
+    while (rest) {
+      const int bpos = __ffs(rest) - 1;
+      rest &= rest - 1u;
+      const int u = x * 32 + bpos;
+      P.exp_units[q] = u;
+      for (int f = 0; f < P.fpu; ++f) P.frames[q * P.fpu + f] = u * P.fpu + f;
+      ++q;
+    }
+  }
+  if (lane == 31) {
     P.counts[1] = ns;
-    P.counts[2] = total;
-    P.counts[3] = total * P.fpu;
+    P.counts[2] = incl;
+    P.counts[3] = incl * P.fpu;
   }
 }
 
