@@ -93,7 +93,7 @@ int64_t cand_cap_of(const ss_index* ix) {
 
 // Workspace regions of one problem (offsets from the problem's base).
 struct Layout {
-  size_t qeff, cand_s, cand_id, cand_cnt, gthr, ladder, anchor, ustats, gram;
+  size_t qeff, cand_s, cand_id, cand_cnt, gthr, ladder, samp_max, ustats, cstats, gram;
   size_t topk_tok, topk_w, list_ml, votes, mass, pool, sel, exp_units, frames, counts,
       status, qstage;
   size_t total;
@@ -118,8 +118,9 @@ Layout layout_of(const ss_index* ix, int R, const ss_retrieve_params* p) {
   l.cand_cnt = take(score_lists * 4);
   l.gthr = take(score_lists * 4);
   l.ladder = take(score_lists * kLadderLevels * 4);
-  l.anchor = take(score_lists * kSampleUnits * 4);
+  l.samp_max = take(score_lists * kSampleUnits * 4);
   l.ustats = take(score_lists * ix->ucap * 8);
+  l.cstats = take(score_lists * kMaxChunksPerSlab * 8);
   l.gram = take(pc * (pc + 1) / 2 * 4);
   l.topk_tok = take(n_lists * p->k * 4);
   l.topk_w = take(n_lists * p->k * 4);
@@ -231,8 +232,9 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
     P.cand_cnt = reinterpret_cast<int32_t*>(base + l.cand_cnt);
     P.gthr = reinterpret_cast<uint32_t*>(base + l.gthr);
     P.ladder = reinterpret_cast<int32_t*>(base + l.ladder);
-    P.anchor = reinterpret_cast<float*>(base + l.anchor);
+    P.samp_max = reinterpret_cast<float*>(base + l.samp_max);
     P.ustats = reinterpret_cast<float2*>(base + l.ustats);
+    P.cstats = reinterpret_cast<float2*>(base + l.cstats);
     P.gram = reinterpret_cast<float*>(base + l.gram);
     const ss_result& r = res[j];
     P.topk_tok = pick(r.topk_tok, base, l.topk_tok);
@@ -248,6 +250,7 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
     P.status = r.status;
     const int64_t pc = (int64_t)p->pool_mult * p->budget_units;
     P.pool_n = (int)(pc < P.Uh ? pc : P.Uh);
+    P.n_sample = sample_units(p->k, P.Tu, P.Uh);
     P.n_sel = P.pool_n < p->budget_units ? P.pool_n : p->budget_units;
     max_lists = max(max_lists, P.P * P.Hq);
     max_uh = max(max_uh, P.Uh);
@@ -276,8 +279,7 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
   if (tr && tr->score_begin) SS_CUDA(cudaEventRecord((cudaEvent_t)tr->score_begin, st));
   SS_CUDA(launch_score(B, st));
   if (tr && tr->score_end) SS_CUDA(cudaEventRecord((cudaEvent_t)tr->score_end, st));
-  SS_CUDA(launch_select(B, max_lists, st));
-  SS_CUDA(launch_mass(B, max_uh, st));
+  SS_CUDA(launch_select(B, max_lists, max_uh, st));
   SS_CUDA(launch_pool(B, max_uh, st));
   SS_CUDA(launch_maxmin(B, max_pool, st));
   return SS_OK;
@@ -321,6 +323,8 @@ SS_EXPORT ss_status ss_index_create(const ss_index_config* cfg, const ss_allocat
   if (c.n_q_heads / c.n_kv_heads > kMaxGroup)
     return fail(SS_ERR_UNSUPPORTED, "more than %d query heads per key head", kMaxGroup);
   if (c.n_kv_heads > 8) return fail(SS_ERR_UNSUPPORTED, "more than 8 key heads");
+  if ((int64_t)c.n_layers * c.n_q_heads > 1024)
+    return fail(SS_ERR_UNSUPPORTED, "more than 1024 (layer, query head) lists");
   if ((int64_t)c.tokens_per_frame * c.max_frames > (int64_t)0x3fffffff)
     return fail(SS_ERR_UNSUPPORTED, "more than 2^30 tokens per slab");
   if (alloc && (!alloc->alloc || !alloc->free))

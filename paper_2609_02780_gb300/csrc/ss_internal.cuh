@@ -49,7 +49,7 @@ constexpr int kTileBytes = kTileRows * kHeadDim * 2;
 constexpr int kLadderLevels = 256;
 constexpr int kLadderZero = 192;
 constexpr float kLadderPerUnit = 16.0f;
-constexpr int kSampleUnits = 4;        // units scored for the anchor
+constexpr int kSampleUnits = 4;        // history units scored for the ladder anchor
 // Candidate slots a warp reserves per list at a time (no atomic per append).
 constexpr int kReserve = 64;
 constexpr int kMaxChunksPerSlab = 128;
@@ -82,8 +82,10 @@ struct Prob {
   int32_t* cand_cnt;           // [n_score_lists]
   uint32_t* gthr;              // [n_score_lists] ordered-float threshold
   int32_t* ladder;             // [n_score_lists][kLadderLevels] appended-score counts
-  float* anchor;               // [n_score_lists][kSampleUnits] sample maxima (log2 units)
+  float* samp_max;             // [n_score_lists][kSampleUnits] maxima of the sampled units
+  int n_sample;                // sampled units Z (0..kSampleUnits)
   float2* ustats;              // [n_score_lists][ucap] per-unit (max, sum 2^(s-max))
+  float2* cstats;              // [n_score_lists][kMaxChunksPerSlab] per-chunk (max, sum)
   float* gram;                 // packed upper triangle of the pool's Gram matrix
   // outputs
   int32_t* topk_tok;           // [n_lists][k]
@@ -144,11 +146,21 @@ __device__ __forceinline__ void ml_combine(float& m, float& l, float mo, float l
   l = a + b;
 }
 
-// Ladder anchor A of list L: the largest score over the sampled units (0 if none).
+// Softmax statistics (M, L) of list L from its chunks' (max, sum 2^(s - max)) pairs,
+// combined in chunk order (every caller gets bit-identical values).
+__device__ __forceinline__ float2 list_stats_of(const Prob& P, int L) {
+  float m = -INFINITY, l = 0.f;
+  for (int c = 0; c < P.chunks; ++c) {
+    const float2 v = P.cstats[(int64_t)L * kMaxChunksPerSlab + c];
+    ml_combine(m, l, v.x, v.y);
+  }
+  return make_float2(m, l);
+}
+
+// Ladder anchor A of list L: the largest sampled score (0 if nothing was sampled).
 __device__ __forceinline__ float list_anchor(const Prob& P, int L) {
   float a = -INFINITY;
-#pragma unroll
-  for (int z = 0; z < kSampleUnits; ++z) a = fmaxf(a, P.anchor[L * kSampleUnits + z]);
+  for (int z = 0; z < P.n_sample; ++z) a = fmaxf(a, P.samp_max[L * kSampleUnits + z]);
   return (a == -INFINITY || a != a) ? 0.f : a;
 }
 
@@ -163,9 +175,10 @@ __device__ __forceinline__ int problem_of_block(const Batch& B, int b) {
 // Launchers (host side), one per translation unit.
 namespace ss {
 cudaError_t launch_prep(const Batch& B, cudaStream_t s);
+int sample_units(int k, int tokens_per_unit, int hist_units);
 cudaError_t launch_score(const Batch& B, cudaStream_t s);
-cudaError_t launch_select(const Batch& B, int max_lists, cudaStream_t s);
-cudaError_t launch_mass(const Batch& B, int max_hist_units, cudaStream_t s);
+cudaError_t launch_select(const Batch& B, int max_lists, int max_hist_units, cudaStream_t s);
+
 cudaError_t launch_pool(const Batch& B, int max_hist_units, cudaStream_t s);
 cudaError_t launch_maxmin(const Batch& B, int max_pool, cudaStream_t s);
 cudaError_t launch_append(__nv_bfloat16* keys, int64_t ncap, int64_t tok0,

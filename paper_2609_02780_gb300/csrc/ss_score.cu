@@ -20,85 +20,146 @@ namespace ss {
 // q_eff[i][h] is the last question row ("final prompt token", Sec. 4.2 / Table 4) or
 // the rows' mean (fp32 sum in row order, divided by R, rounded to bf16 nearest-even).
 // ---------------------------------------------------------------------------
-// Grid (list, problem, sample unit z). Block z = 0 also writes q_eff and resets the
-// per-call state; every block scores the history unit z * Uh / n_sample against its
-// list's query and records the largest score, the anchor of the threshold ladder.
-__global__ void __launch_bounds__(kHeadDim) k_prep(const __grid_constant__ Batch B) {
-  __shared__ float qs[kHeadDim];
-  __shared__ float red[kHeadDim / 32];
+// k_sample: grid (slab, problem, sample z), 256 threads. Computes q_eff of the slab's G
+// query heads (block z = 0 stores it and resets the per-call state), then scores the G
+// heads against every token of the history unit z * Uh / Z on the tensor cores (keys
+// staged in shared memory, the scoring kernel's fragment layout). The largest sampled
+// score of each list anchors its threshold ladder.
+constexpr int kSampleRows = 128;  // key rows staged per pass of k_sample (8 MMA tiles)
+
+int sample_units(int k, int tokens_per_unit, int hist_units) {
+  (void)k;
+  (void)tokens_per_unit;
+  return hist_units < kSampleUnits ? hist_units : kSampleUnits;
+}
+
+__device__ __forceinline__ void mma_16816(float (&d)[4], uint32_t a0, uint32_t a1,
+                                          uint32_t a2, uint32_t a3, uint32_t b0,
+                                          uint32_t b1);
+
+__global__ void __launch_bounds__(256) k_sample(const __grid_constant__ Batch B) {
+  __shared__ __align__(16) __nv_bfloat16 qsb[kMaxGroup][kHeadDim];
+  __shared__ float wmax[8][kMaxGroup];
+  __shared__ __align__(16) unsigned char kt[kSampleRows * kHeadDim * 2];
   const int pi = blockIdx.y;
   if (pi >= B.n) return;
   const Prob& P = B.p[pi];
-  const int n_lists = P.P * P.Hq;
-  const int L = blockIdx.x, z = blockIdx.z;
-  if (L >= n_lists) return;
-  const int i = L / P.Hq, h = L % P.Hq;
-  const int d = threadIdx.x;
+  const int slab = blockIdx.x, z = blockIdx.z;
+  const int n_slabs = P.P * P.Hkv;
+  if (slab >= n_slabs) return;
+  const int i = slab / P.Hkv, gk = slab - i * P.Hkv, G = P.G;
+  const int list0 = i * P.Hq + gk * G;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t row_stride = (int64_t)P.Hq * kHeadDim;
-  const __nv_bfloat16* q0 = P.q + (int64_t)i * P.R * row_stride + (int64_t)h * kHeadDim + d;
-  float v;
-  if (B.q_agg == 0) {
-    v = __bfloat162float(q0[(int64_t)(P.R - 1) * row_stride]);
-  } else {
-    float acc = 0.f;
-    for (int r = 0; r < P.R; ++r) acc = __fadd_rn(acc, __bfloat162float(q0[(int64_t)r * row_stride]));
-    v = __fdiv_rn(acc, (float)P.R);
-  }
-  const __nv_bfloat16 qe = __float2bfloat16_rn(v);
-  qs[d] = __bfloat162float(qe);
-  if (z == 0) {
-    P.qeff[(int64_t)L * kHeadDim + d] = qe;
-    if (d == 0) {
-      P.cand_cnt[L] = 0;
-      P.gthr[L] = float_to_ordered(-INFINITY);
-    }
-    for (int x = d; x < kLadderLevels; x += kHeadDim) P.ladder[(int64_t)L * kLadderLevels + x] = 0;
-    for (int u = L * kHeadDim + d; u < P.ucap; u += n_lists * kHeadDim) P.votes[u] = 0;
-    if (L == 0 && d < 4) P.counts[d] = 0;
-    if (L == 0 && d == 0) *P.status = 0u;
-  }
-  __syncthreads();
-
-  float mx = -INFINITY;
-  const int ns = min(kSampleUnits, P.Uh);
-  if (z < ns) {
-    const int64_t u = ((int64_t)z * P.Uh) / ns;
-    const int64_t slab = (int64_t)i * P.Hkv + h / P.G;
-    const __nv_bfloat16* sk = P.keys + (slab * P.ncap + u * P.Tu) * kHeadDim;
-    for (int r = d; r < P.Tu; r += kHeadDim) {
-      const uint4* row = reinterpret_cast<const uint4*>(sk + (int64_t)r * kHeadDim);
-      uint4 w[kHeadDim / 8];
-#pragma unroll
-      for (int c = 0; c < kHeadDim / 8; ++c) w[c] = row[c];
-      float dot = 0.f;
-#pragma unroll
-      for (int c = 0; c < kHeadDim / 8; ++c) {
-        const __nv_bfloat162* e = reinterpret_cast<const __nv_bfloat162*>(&w[c]);
-#pragma unroll
-        for (int zz = 0; zz < 4; ++zz) {
-          const float2 f = __bfloat1622float2(e[zz]);
-          dot = fmaf(qs[8 * c + 2 * zz], f.x, dot);
-          dot = fmaf(qs[8 * c + 2 * zz + 1], f.y, dot);
-        }
+  for (int x = tid; x < kMaxGroup * kHeadDim; x += blockDim.x) {
+    const int hh = x / kHeadDim, d = x - hh * kHeadDim;
+    __nv_bfloat16 qe = __float2bfloat16_rn(0.f);
+    if (hh < G) {
+      const __nv_bfloat16* q0 = P.q + (int64_t)i * P.R * row_stride + (int64_t)(gk * G + hh) * kHeadDim + d;
+      float v;
+      if (B.q_agg == 0) {
+        v = __bfloat162float(q0[(int64_t)(P.R - 1) * row_stride]);
+      } else {
+        float acc = 0.f;
+        for (int r = 0; r < P.R; ++r) acc = __fadd_rn(acc, __bfloat162float(q0[(int64_t)r * row_stride]));
+        v = __fdiv_rn(acc, (float)P.R);
       }
-      mx = fmaxf(mx, dot * kScoreScale);
+      qe = __float2bfloat16_rn(v);
+      if (z == 0) P.qeff[(int64_t)(list0 + hh) * kHeadDim + d] = qe;
+    }
+    qsb[hh][d] = qe;
+  }
+  if (z == 0) {
+    if (tid < G) {
+      P.cand_cnt[list0 + tid] = 0;
+      P.gthr[list0 + tid] = float_to_ordered(-INFINITY);
+    }
+    for (int x = tid; x < G * kLadderLevels; x += blockDim.x)
+      P.ladder[(int64_t)list0 * kLadderLevels + x] = 0;
+    for (int u = slab * blockDim.x + tid; u < P.ucap; u += n_slabs * blockDim.x) P.votes[u] = 0;
+    if (slab == 0 && tid < 4) P.counts[tid] = 0;
+    if (slab == 0 && tid == 0) *P.status = 0u;
+  }
+  __syncthreads();
+  if (z >= P.n_sample) return;
+  const int64_t u = ((int64_t)z * P.Uh) / P.n_sample;
+  const __nv_bfloat16* sk = P.keys + ((int64_t)slab * P.ncap + u * P.Tu) * kHeadDim;
+  // query fragments, permuted like the key fragments (as in the scoring kernel)
+  const int g = lane >> 2, t4 = lane & 3;
+  uint32_t qf[8][2];
+  {
+    const uint32_t* qw = reinterpret_cast<const uint32_t*>(&qsb[g][0]);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int e = 8 * (4 * (j >> 1) + t4) + 4 * (j & 1);
+      qf[j][0] = qw[e >> 1];
+      qf[j][1] = qw[(e >> 1) + 1];
     }
   }
-  for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-  if ((d & 31) == 0) red[d >> 5] = mx;
+  const int c0 = 2 * t4, c1 = c0 + 1;
+  const bool hv0 = c0 < G, hv1 = c1 < G;
+  float mx0 = -INFINITY, mx1 = -INFINITY;
+  for (int rb = 0; rb < P.Tu; rb += kSampleRows) {
+    const int nr = min(kSampleRows, P.Tu - rb);
+    __syncthreads();
+    const uint4* src = reinterpret_cast<const uint4*>(sk + (int64_t)rb * kHeadDim);
+    uint4* dst = reinterpret_cast<uint4*>(kt);
+    for (int x = tid; x < nr * (kHeadDim / 8); x += blockDim.x) dst[x] = src[x];
+    __syncthreads();
+    // warp w scores rows [16 w, 16 w + 16) of this pass
+    const int tr = kTileRows * warp;
+    if (tr < nr) {
+      const unsigned char* tb = kt + (size_t)tr * kHeadDim * 2;
+      uint4 ra[4], rbv[4];
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        ra[v] = *reinterpret_cast<const uint4*>(tb + g * 256 + 16 * (4 * v + t4));
+        rbv[v] = *reinterpret_cast<const uint4*>(tb + (g + 8) * 256 + 16 * (4 * v + t4));
+      }
+      float acc[4] = {0.f, 0.f, 0.f, 0.f}, acd[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        mma_16816(acc, ra[v].x, rbv[v].x, ra[v].y, rbv[v].y, qf[2 * v][0], qf[2 * v][1]);
+        mma_16816(acd, ra[v].z, rbv[v].z, ra[v].w, rbv[v].w, qf[2 * v + 1][0], qf[2 * v + 1][1]);
+      }
+      const int r0 = tr + g;
+      const bool v0 = r0 < nr, v1 = r0 + 8 < nr;
+      const float s00 = (acc[0] + acd[0]) * kScoreScale, s01 = (acc[1] + acd[1]) * kScoreScale;
+      const float s10 = (acc[2] + acd[2]) * kScoreScale, s11 = (acc[3] + acd[3]) * kScoreScale;
+      if (hv0) {
+        if (v0) mx0 = fmaxf(mx0, s00);
+        if (v1) mx0 = fmaxf(mx0, s10);
+      }
+      if (hv1) {
+        if (v0) mx1 = fmaxf(mx1, s01);
+        if (v1) mx1 = fmaxf(mx1, s11);
+      }
+    }
+  }
+#pragma unroll
+  for (int off = 4; off < 32; off <<= 1) {
+    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, off));
+    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, off));
+  }
+  if (g == 0) {
+    wmax[warp][c0] = mx0;
+    if (c1 < kMaxGroup) wmax[warp][c1] = mx1;
+  }
   __syncthreads();
-  if (d == 0) {
-    float a = red[0];
-    for (int w = 1; w < kHeadDim / 32; ++w) a = fmaxf(a, red[w]);
-    P.anchor[L * kSampleUnits + z] = a;
+  if (tid < G) {
+    float m = -INFINITY;
+    for (int w = 0; w < 8; ++w) m = fmaxf(m, wmax[w][tid]);
+    P.samp_max[(list0 + tid) * kSampleUnits + z] = m;
   }
 }
 
 cudaError_t launch_prep(const Batch& B, cudaStream_t s) {
-  int max_lists = 0;
-  for (int j = 0; j < B.n; ++j) max_lists = max(max_lists, B.p[j].P * B.p[j].Hq);
-  dim3 grid(max_lists, B.n, kSampleUnits);
-  k_prep<<<grid, kHeadDim, 0, s>>>(B);
+  int max_slabs = 0, max_z = 1;
+  for (int j = 0; j < B.n; ++j) {
+    max_slabs = max(max_slabs, B.p[j].P * B.p[j].Hkv);
+    max_z = max(max_z, B.p[j].n_sample);
+  }
+  k_sample<<<dim3(max_slabs, B.n, max_z), 256, 0, s>>>(B);
   return cudaGetLastError();
 }
 
@@ -145,14 +206,13 @@ __device__ __forceinline__ uint4 ld_stream(const void* p) {
   return r;
 }
 
-constexpr int kDefer = 4;  // warm-up tiles per warp whose appends wait for a threshold
-
 struct ScoreShared {
   int lad[kMaxGroup][kLadderLevels];  // this CTA's appended-score counts not yet merged
   float thr[kMaxGroup];
   float anchor[kMaxGroup];
   int all_done;
   unsigned long long bar[kScoreWarps][kScoreStages];  // one mbarrier per warp stage
+  float2 wstat[kScoreWarps][kMaxGroup];  // per warp: its units' (max, sum) per list
 };
 
 // ---- TMA bulk copies and mbarriers (inline PTX) ----
@@ -324,6 +384,8 @@ __global__ void __maxnreg__(kScoreMaxRegs)
     S.anchor[threadIdx.x] = threadIdx.x < G ? list_anchor(P, list0 + threadIdx.x) : 0.f;
   }
   if (threadIdx.x == 0) S.all_done = 0;
+  if (threadIdx.x < kScoreWarps * kMaxGroup)
+    (&S.wstat[0][0])[threadIdx.x] = make_float2(-INFINITY, 0.f);
   if (threadIdx.x < kScoreWarps * kScoreStages)
     mbar_init(smem_u32(&S.bar[0][0] + threadIdx.x), 1u);
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -367,26 +429,22 @@ __global__ void __maxnreg__(kScoreMaxRegs)
   const __nv_bfloat16* slab_keys = P.keys + (int64_t)slab * P.ncap * kHeadDim;
   const int64_t cbase0 = (int64_t)(hv0 ? L0 : list0) * P.cand_cap;
   const int64_t cbase1 = (int64_t)(hv1 ? L1 : list0) * P.cand_cap;
-  const unsigned gmask = 0x11111111u << t4;
-  const unsigned lt_mask = (1u << lane) - 1u;
   unsigned char* my_tiles = tiles + (size_t)warp * kScoreStages * kTileBytes;
   const uint32_t my_tiles_s = smem_u32(my_tiles);
   const uint32_t my_bars = smem_u32(&S.bar[warp][0]);
   const volatile float* vthr = S.thr;
-  const float an0 = S.anchor[c0 < kMaxGroup ? c0 : 0], an1 = S.anchor[c1 < kMaxGroup ? c1 : 0];
+  const unsigned gmask = 0x11111111u << t4;
+  const unsigned lt_mask = (1u << lane) - 1u;
+  const float an0 = S.anchor[c0], an1 = S.anchor[c1 < kMaxGroup ? c1 : 0];
   // Candidate slots reserved for this lane group's two lists (identical in its 8 lanes).
   int rp0 = 0, rl0 = 0, rp1 = 0, rl1 = 0;
 
   // Appends the scores of keys tok0 (row g) and tok0 + 8 (row g + 8) that reach the
-  // current thresholds, counting them in the ladder when `count` (a warm-up score was
-  // counted when it was scored).
+  // current thresholds, and counts them in the CTA's ladder.
   auto append = [&](float s00, float s01, float s10, float s11, int tok0, bool v0, bool v1,
-                    bool count) {
-    const float thr0 = hv0 ? vthr[c0] : INFINITY;
-    const float thr1 = hv1 ? vthr[c1] : INFINITY;
+                    float thr0, float thr1) {
     const bool p00 = hv0 && v0 && s00 >= thr0, p10 = hv0 && v1 && s10 >= thr0;
     const bool p01 = hv1 && v0 && s01 >= thr1, p11 = hv1 && v1 && s11 >= thr1;
-    if (!__any_sync(0xffffffffu, p00 | p01 | p10 | p11)) return;
     const int tok1 = tok0 + 8;
     const unsigned b00 = __ballot_sync(0xffffffffu, p00) & gmask;
     const unsigned b10 = __ballot_sync(0xffffffffu, p10) & gmask;
@@ -406,25 +464,25 @@ __global__ void __maxnreg__(kScoreMaxRegs)
       const int64_t pos = slot0(__popc(b00 & lt_mask));
       P.cand_s[pos] = s00;
       P.cand_id[pos] = tok0;
-      if (count) ladder_add(S, c0, s00, an0);
+      ladder_add(S, c0, s00, an0);
     }
     if (p10) {
       const int64_t pos = slot0(__popc(b00) + __popc(b10 & lt_mask));
       P.cand_s[pos] = s10;
       P.cand_id[pos] = tok1;
-      if (count) ladder_add(S, c0, s10, an0);
+      ladder_add(S, c0, s10, an0);
     }
     if (p01) {
       const int64_t pos = slot1(__popc(b01 & lt_mask));
       P.cand_s[pos] = s01;
       P.cand_id[pos] = tok0;
-      if (count) ladder_add(S, c1, s01, an1);
+      ladder_add(S, c1, s01, an1);
     }
     if (p11) {
       const int64_t pos = slot1(__popc(b01) + __popc(b11 & lt_mask));
       P.cand_s[pos] = s11;
       P.cand_id[pos] = tok1;
-      if (count) ladder_add(S, c1, s11, an1);
+      ladder_add(S, c1, s11, an1);
     }
     if (need0) {
       rp0 = nb0 + (n0 - rl0);
@@ -439,19 +497,6 @@ __global__ void __maxnreg__(kScoreMaxRegs)
     } else {
       rp1 += n1;
       rl1 -= n1;
-    }
-  };
-
-  // The first kDefer tiles of the warp are scored before any threshold exists; their
-  // scores wait in registers and are appended once the ladder has had time to fill.
-  float ds[kDefer][4];
-  int dtok[kDefer];  // bit 0 / 1: rows g / g + 8 valid; token of row g in bits 2..
-  auto flush_deferred = [&](int nd) {
-#pragma unroll
-    for (int q = 0; q < kDefer; ++q) {
-      if (q < nd)
-        append(ds[q][0], ds[q][1], ds[q][2], ds[q][3], dtok[q] >> 2, (dtok[q] & 1) != 0,
-               (dtok[q] & 2) != 0, false);
     }
   };
 
@@ -488,6 +533,7 @@ __global__ void __maxnreg__(kScoreMaxRegs)
   }
 
   float m0 = -INFINITY, l0 = 0.f, m1 = -INFINITY, l1 = 0.f;
+  float wm0 = -INFINITY, wl0 = 0.f, wm1 = -INFINITY, wl1 = 0.f;  // this warp's units so far
   int t = 0;
   bool aborted = false;
   for (; t < ntiles; ++t) {
@@ -527,24 +573,11 @@ __global__ void __maxnreg__(kScoreMaxRegs)
     const float s10 = (acc[2] + acd[2]) * kScoreScale, s11 = (acc[3] + acd[3]) * kScoreScale;
     stats_update(m0, l0, s00, v0, s10, v1);
     stats_update(m1, l1, s01, v0, s11, v1);
-    const int tok0 = u * Tu + r0;
-    if (t < kDefer) {
-      // warm-up: count every score in the ladder now, decide the appends later
-      if (hv0 && v0) ladder_add(S, c0, s00, an0);
-      if (hv0 && v1) ladder_add(S, c0, s10, an0);
-      if (hv1 && v0) ladder_add(S, c1, s01, an1);
-      if (hv1 && v1) ladder_add(S, c1, s11, an1);
-#pragma unroll
-      for (int q = 0; q < kDefer; ++q) {
-        if (q == t) {
-          ds[q][0] = s00; ds[q][1] = s01; ds[q][2] = s10; ds[q][3] = s11;
-          dtok[q] = (v0 ? 1 : 0) | (v1 ? 2 : 0) | (tok0 << 2);
-        }
-      }
-      if (t == kDefer - 1) flush_deferred(kDefer);
-    } else {
-      append(s00, s01, s10, s11, tok0, v0, v1, true);
-    }
+    const float thr0 = hv0 ? vthr[c0] : INFINITY;
+    const float thr1 = hv1 ? vthr[c1] : INFINITY;
+    const bool pass = (hv0 && ((v0 && s00 >= thr0) || (v1 && s10 >= thr0))) ||
+                      (hv1 && ((v0 && s01 >= thr1) || (v1 && s11 >= thr1)));
+    if (__any_sync(0xffffffffu, pass)) append(s00, s01, s10, s11, u * Tu + r0, v0, v1, thr0, thr1);
     if (j == tpu - 1) {
 #pragma unroll
       for (int off = 4; off < 32; off <<= 1) {
@@ -558,10 +591,11 @@ __global__ void __maxnreg__(kScoreMaxRegs)
       if (g == 0) {
         if (hv0) P.ustats[(int64_t)L0 * P.ucap + u] = make_float2(m0, l0);
         if (hv1) P.ustats[(int64_t)L1 * P.ucap + u] = make_float2(m1, l1);
+        ml_combine(wm0, wl0, m0, l0);
+        ml_combine(wm1, wl1, m1, l1);
       }
     }
   }
-  if (!aborted && ntiles < kDefer) flush_deferred(ntiles);
   // unused reserved slots are marked empty (score -inf)
   for (int x = g; x < rl0; x += 8) P.cand_s[cbase0 + rp0 + x] = -INFINITY;
   for (int x = g; x < rl1; x += 8) P.cand_s[cbase1 + rp1 + x] = -INFINITY;
@@ -571,7 +605,29 @@ __global__ void __maxnreg__(kScoreMaxRegs)
     for (int r = t; r < min(ntiles, t + kScoreStages); ++r)
       mbar_wait_bounded(my_bars + 8u * (r % kScoreStages), (uint32_t)((r / kScoreStages) & 1));
   }
-  if (lane == 0) atomicAdd(&S.all_done, 1);
+  // The chunk's (max, sum) per list: the warps' partials (each over its units in
+  // order) combined in warp order by the last warp to finish.
+  if (g == 0) {
+    if (hv0) S.wstat[warp][c0] = make_float2(wm0, wl0);
+    if (hv1) S.wstat[warp][c1] = make_float2(wm1, wl1);
+  }
+  __threadfence_block();
+  __syncwarp();
+  int order = 0;
+  if (lane == 0) order = atomicAdd(&S.all_done, 1);
+  order = __shfl_sync(0xffffffffu, order, 0);
+  if (order == kScoreWarps - 1) {
+    __threadfence_block();
+    if (lane < G) {
+      float m = -INFINITY, l = 0.f;
+      const volatile float2* ws = &S.wstat[0][0];
+      for (int w = 0; w < kScoreWarps; ++w) {
+        const float mw = ws[w * kMaxGroup + lane].x, lw = ws[w * kMaxGroup + lane].y;
+        ml_combine(m, l, mw, lw);
+      }
+      P.cstats[(int64_t)(list0 + lane) * kMaxChunksPerSlab + chunk] = make_float2(m, l);
+    }
+  }
 }
 
 int score_chunks_per_slab(int n_slabs_total, int hist_units, int sm_count) {
