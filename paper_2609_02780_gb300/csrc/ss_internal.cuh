@@ -10,6 +10,8 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 
+#include <utility>
+
 namespace ss {
 
 constexpr int kHeadDim = 128;          // d (only 128 is supported)
@@ -30,12 +32,6 @@ constexpr int kScoreThreads = (kScoreWarps + 1) * 32;
 #define SS_SCORE_CTAS_PER_SM 2
 #endif
 constexpr int kScoreCtasPerSm = SS_SCORE_CTAS_PER_SM;
-// registers per thread that still fit kScoreCtasPerSm CTAs per SM (64K registers,
-// allocated per warp in multiples of 8 per thread)
-constexpr int kScoreMaxRegs =
-    (65536 / (kScoreCtasPerSm * (kScoreWarps + 1) * 32)) / 8 * 8 > 255
-        ? 255
-        : (65536 / (kScoreCtasPerSm * (kScoreWarps + 1) * 32)) / 8 * 8;
 #ifndef SS_SCORE_STAGES
 #define SS_SCORE_STAGES 3
 #endif
@@ -164,6 +160,14 @@ __device__ __forceinline__ float list_anchor(const Prob& P, int L) {
   return (a == -INFINITY || a != a) ? 0.f : a;
 }
 
+// Programmatic dependent launch: every retrieval kernel may start while its predecessor
+// in the stream drains. pdl_wait() blocks until the predecessor grid has completed and
+// its writes are visible; pdl_release() lets the successor start launching.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_release() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 __device__ __forceinline__ int problem_of_block(const Batch& B, int b) {
   int pi = 0;
   while (pi + 1 < B.n && B.p[pi + 1].cta_begin <= b) ++pi;
@@ -174,6 +178,22 @@ __device__ __forceinline__ int problem_of_block(const Batch& B, int b) {
 
 // Launchers (host side), one per translation unit.
 namespace ss {
+// Launches `kernel` with programmatic stream serialization (see pdl_wait).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t s, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 cudaError_t launch_prep(const Batch& B, cudaStream_t s);
 int sample_units(int k, int tokens_per_unit, int hist_units);
 cudaError_t launch_score(const Batch& B, cudaStream_t s);

@@ -41,6 +41,8 @@ __global__ void __launch_bounds__(256) k_sample(const __grid_constant__ Batch B)
   __shared__ __align__(16) __nv_bfloat16 qsb[kMaxGroup][kHeadDim];
   __shared__ float wmax[8][kMaxGroup];
   __shared__ __align__(16) unsigned char kt[kSampleRows * kHeadDim * 2];
+  pdl_wait();     // keys, queries and the previous call's use of the workspace
+  pdl_release();
   const int pi = blockIdx.y;
   if (pi >= B.n) return;
   const Prob& P = B.p[pi];
@@ -159,8 +161,7 @@ cudaError_t launch_prep(const Batch& B, cudaStream_t s) {
     max_slabs = max(max_slabs, B.p[j].P * B.p[j].Hkv);
     max_z = max(max_z, B.p[j].n_sample);
   }
-  k_sample<<<dim3(max_slabs, B.n, max_z), 256, 0, s>>>(B);
-  return cudaGetLastError();
+  return launch_pdl(k_sample, dim3(max_slabs, B.n, max_z), dim3(256), 0, s, B);
 }
 
 // ---------------------------------------------------------------------------
@@ -359,7 +360,7 @@ __device__ void threshold_warp(ScoreShared& S, const Prob& P, int list0, int k) 
   }
 }
 
-__global__ void __maxnreg__(kScoreMaxRegs)
+__global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
     k_score(const __grid_constant__ Batch B) {
   __shared__ ScoreShared S;
   extern __shared__ __align__(128) unsigned char tiles[];  // [warp][stage][kTileBytes]
@@ -377,6 +378,8 @@ __global__ void __maxnreg__(kScoreMaxRegs)
   const int i = slab / P.Hkv, kvh = slab - i * P.Hkv;
   const int G = P.G;
   const int list0 = i * P.Hq + kvh * G;
+  pdl_wait();     // q_eff, anchors and resets of the prep kernel
+  pdl_release();
   for (int x = threadIdx.x; x < kMaxGroup * kLadderLevels; x += blockDim.x)
     (&S.lad[0][0])[x] = 0;
   if (threadIdx.x < kMaxGroup) {
@@ -567,14 +570,14 @@ __global__ void __maxnreg__(kScoreMaxRegs)
       m0 = m1 = -INFINITY;
       l0 = l1 = 0.f;
     }
+    const float thr0 = hv0 ? vthr[c0] : INFINITY;
+    const float thr1 = hv1 ? vthr[c1] : INFINITY;
     const int r0 = kTileRows * j + g;
     const bool v0 = r0 < Tu, v1 = r0 + 8 < Tu;
     const float s00 = (acc[0] + acd[0]) * kScoreScale, s01 = (acc[1] + acd[1]) * kScoreScale;
     const float s10 = (acc[2] + acd[2]) * kScoreScale, s11 = (acc[3] + acd[3]) * kScoreScale;
     stats_update(m0, l0, s00, v0, s10, v1);
     stats_update(m1, l1, s01, v0, s11, v1);
-    const float thr0 = hv0 ? vthr[c0] : INFINITY;
-    const float thr1 = hv1 ? vthr[c1] : INFINITY;
     const bool pass = (hv0 && ((v0 && s00 >= thr0) || (v1 && s10 >= thr0))) ||
                       (hv1 && ((v0 && s01 >= thr1) || (v1 && s11 >= thr1)));
     if (__any_sync(0xffffffffu, pass)) append(s00, s01, s10, s11, u * Tu + r0, v0, v1, thr0, thr1);
@@ -655,8 +658,7 @@ cudaError_t launch_score(const Batch& B, cudaStream_t s) {
   const int smem = kScoreWarps * kScoreStages * kTileBytes;
   cudaError_t e = cudaFuncSetAttribute(k_score, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  k_score<<<B.score_ctas, kScoreThreads, smem, s>>>(B);
-  return cudaGetLastError();
+  return launch_pdl(k_score, dim3(B.score_ctas), dim3(kScoreThreads), (size_t)smem, s, B);
 }
 
 }  // namespace ss

@@ -149,6 +149,8 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
   __shared__ int s_n, s_bstar, s_rem;
   __shared__ unsigned long long s_prefix;
 
+  pdl_wait();
+  pdl_release();
   const int pi = blockIdx.y;
   if (pi >= B.n) return;
   const Prob& P = B.p[pi];
@@ -401,8 +403,7 @@ cudaError_t launch_select(const Batch& B, int max_lists, int max_hist_units, cud
   if (e != cudaSuccess) return e;
   const int mass_blocks = (max_hist_units + kMassUnits - 1) / kMassUnits;
   dim3 grid(max_lists + mass_blocks, B.n);
-  k_select<<<grid, kSelThreads, smem, s>>>(B, max_lists);
-  return cudaGetLastError();
+  return launch_pdl(k_select, grid, dim3(kSelThreads), (size_t)smem, s, B, max_lists);
 }
 
 // ---------------------------------------------------------------------------
@@ -479,6 +480,8 @@ __global__ void __launch_bounds__(1024) k_pool(const __grid_constant__ Batch B) 
   __shared__ int vh[kVoteBins];
   __shared__ int sw[32];
   __shared__ int s_v, s_c;
+  pdl_wait();
+  pdl_release();
   const Prob& P = B.p[blockIdx.x];
   const int Uh = P.Uh, pn = P.pool_n;
   const int tid = threadIdx.x;
@@ -579,8 +582,7 @@ cudaError_t launch_pool(const Batch& B, int max_hist_units, cudaStream_t s) {
   const int smem = max(n2, kRankMax) * (int)(sizeof(unsigned long long) + sizeof(int));
   cudaError_t e = cudaFuncSetAttribute(k_pool, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  k_pool<<<B.n, 1024, smem, s>>>(B);
-  return cudaGetLastError();
+  return launch_pdl(k_pool, dim3(B.n), dim3(1024), (size_t)smem, s, B);
 }
 
 // ---------------------------------------------------------------------------
@@ -598,6 +600,8 @@ __device__ __forceinline__ int tri_off(int a, int pn) { return a * pn - (a * (a 
 
 __global__ void __launch_bounds__(256) k_gram(const __grid_constant__ Batch B) {
   extern __shared__ float gsm[];
+  pdl_wait();
+  pdl_release();
   const Prob& P = B.p[blockIdx.y];
   const int pn = P.pool_n;
   const int dim = P.Hkv * kHeadDim;
@@ -713,6 +717,8 @@ __global__ void __launch_bounds__(kMaxMinThreads) k_maxmin(const __grid_constant
   __shared__ uint32_t bits[kMaxHistUnits / 32];
   __shared__ int spool[kMaxPool];
   __shared__ int ssel[kMaxPool];
+  pdl_wait();
+  pdl_release();
   const Prob& P = B.p[blockIdx.x];
   const int pn = P.pool_n, ns = P.n_sel;
   const int tid = threadIdx.x, warp = tid >> 5;
@@ -796,16 +802,14 @@ cudaError_t launch_maxmin(const Batch& B, int max_pool, cudaStream_t s) {
     cudaError_t e = cudaFuncSetAttribute(k_gram, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     dim3 grid(T * (T + 1) / 2, B.n);
-    k_gram<<<grid, kGramTile * kGramTile, smem, s>>>(B);
-    e = cudaGetLastError();
+    e = launch_pdl(k_gram, grid, dim3(kGramTile * kGramTile), (size_t)smem, s, B);
     if (e != cudaSuccess) return e;
   }
   const int pk_n = max_pool <= kMaxMinSmemPool ? max_pool * (max_pool + 1) / 2 : 0;
   const int smem = ((max(pk_n, 1) + 3) / 4) * (int)sizeof(float4);
   cudaError_t e = cudaFuncSetAttribute(k_maxmin, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  k_maxmin<<<B.n, kMaxMinThreads, smem, s>>>(B);
-  return cudaGetLastError();
+  return launch_pdl(k_maxmin, dim3(B.n), dim3(kMaxMinThreads), (size_t)smem, s, B);
 }
 
 }  // namespace ss
