@@ -93,7 +93,7 @@ int64_t cand_cap_of(const ss_index* ix) {
 
 // Workspace regions of one problem (offsets from the problem's base).
 struct Layout {
-  size_t qeff, cand_s, cand_id, cand_cnt, gthr, ladder, samp_max, ustats, cstats, gram;
+  size_t qeff, cand_s, cand_id, cand_cnt, gthr, ladder, samp_max, ustats, next_unit, gram;
   size_t topk_tok, topk_w, list_ml, votes, mass, pool, sel, exp_units, frames, counts,
       status, qstage;
   size_t total;
@@ -120,7 +120,7 @@ Layout layout_of(const ss_index* ix, int R, const ss_retrieve_params* p) {
   l.ladder = take(score_lists * kLadderLevels * 4);
   l.samp_max = take(score_lists * kSampleUnits * 4);
   l.ustats = take(score_lists * ix->ucap * 8);
-  l.cstats = take(score_lists * kMaxChunksPerSlab * 8);
+  l.next_unit = take((int64_t)c.n_layers * c.n_kv_heads * 4);
   l.gram = take(pc * (pc + 1) / 2 * 4);
   l.topk_tok = take(n_lists * p->k * 4);
   l.topk_w = take(n_lists * p->k * 4);
@@ -234,7 +234,7 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
     P.ladder = reinterpret_cast<int32_t*>(base + l.ladder);
     P.samp_max = reinterpret_cast<float*>(base + l.samp_max);
     P.ustats = reinterpret_cast<float2*>(base + l.ustats);
-    P.cstats = reinterpret_cast<float2*>(base + l.cstats);
+    P.next_unit = reinterpret_cast<int32_t*>(base + l.next_unit);
     P.gram = reinterpret_cast<float*>(base + l.gram);
     const ss_result& r = res[j];
     P.topk_tok = pick(r.topk_tok, base, l.topk_tok);
@@ -258,12 +258,9 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
     n_slabs_total += P.P * P.Hkv;
     base += l.total;
   }
-  // Score-kernel mapping: a common chunk length in units for all problems.
-#ifdef SS_FORCE_CHUNKS
-  const int c_common = max_uh > 0 ? min(SS_FORCE_CHUNKS, max_uh) : 0;
-#else
+  // Score-kernel mapping: CTAs per slab, sized with a common units-per-CTA length for
+  // all problems (the CTAs of a slab share its units dynamically).
   const int c_common = score_chunks_per_slab(n_slabs_total, max_uh, ix[0]->sm_count);
-#endif
   const int chunk_len = c_common > 0 ? (max_uh + c_common - 1) / c_common : 1;
   int cta = 0;
   for (int j = 0; j < n; ++j) {
@@ -279,7 +276,8 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
   if (tr && tr->score_begin) SS_CUDA(cudaEventRecord((cudaEvent_t)tr->score_begin, st));
   SS_CUDA(launch_score(B, st));
   if (tr && tr->score_end) SS_CUDA(cudaEventRecord((cudaEvent_t)tr->score_end, st));
-  SS_CUDA(launch_select(B, max_lists, max_uh, st));
+  SS_CUDA(launch_select(B, max_lists, st));
+  SS_CUDA(launch_mass(B, max_uh, st));
   SS_CUDA(launch_pool(B, max_uh, st));
   SS_CUDA(launch_maxmin(B, max_pool, st));
   return SS_OK;

@@ -81,7 +81,7 @@ struct Prob {
   float* samp_max;             // [n_score_lists][kSampleUnits] maxima of the sampled units
   int n_sample;                // sampled units Z (0..kSampleUnits)
   float2* ustats;              // [n_score_lists][ucap] per-unit (max, sum 2^(s-max))
-  float2* cstats;              // [n_score_lists][kMaxChunksPerSlab] per-chunk (max, sum)
+  int32_t* next_unit;          // [P*Hkv] next history unit to score in each slab
   float* gram;                 // packed upper triangle of the pool's Gram matrix
   // outputs
   int32_t* topk_tok;           // [n_lists][k]
@@ -97,7 +97,7 @@ struct Prob {
   uint32_t* status;
   // launch mapping of the score kernel
   int cta_begin;               // first score CTA of this problem
-  int chunks;                  // unit chunks per slab
+  int chunks;                  // score CTAs per slab (they share the slab's units)
   int pool_n;                  // min(pool_mult * budget, Uh)
   int n_sel;                   // min(budget, pool_n)
 };
@@ -140,17 +140,6 @@ __device__ __forceinline__ void ml_combine(float& m, float& l, float mo, float l
   float b = (mo == -INFINITY) ? 0.f : lo * fast_exp2(mo - M);
   m = M;
   l = a + b;
-}
-
-// Softmax statistics (M, L) of list L from its chunks' (max, sum 2^(s - max)) pairs,
-// combined in chunk order (every caller gets bit-identical values).
-__device__ __forceinline__ float2 list_stats_of(const Prob& P, int L) {
-  float m = -INFINITY, l = 0.f;
-  for (int c = 0; c < P.chunks; ++c) {
-    const float2 v = P.cstats[(int64_t)L * kMaxChunksPerSlab + c];
-    ml_combine(m, l, v.x, v.y);
-  }
-  return make_float2(m, l);
 }
 
 // Ladder anchor A of list L: the largest sampled score (0 if nothing was sampled).
@@ -197,7 +186,8 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
 cudaError_t launch_prep(const Batch& B, cudaStream_t s);
 int sample_units(int k, int tokens_per_unit, int hist_units);
 cudaError_t launch_score(const Batch& B, cudaStream_t s);
-cudaError_t launch_select(const Batch& B, int max_lists, int max_hist_units, cudaStream_t s);
+cudaError_t launch_select(const Batch& B, int max_lists, cudaStream_t s);
+cudaError_t launch_mass(const Batch& B, int max_hist_units, cudaStream_t s);
 
 cudaError_t launch_pool(const Batch& B, int max_hist_units, cudaStream_t s);
 cudaError_t launch_maxmin(const Batch& B, int max_pool, cudaStream_t s);

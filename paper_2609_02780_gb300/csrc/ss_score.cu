@@ -78,6 +78,7 @@ __global__ void __launch_bounds__(256) k_sample(const __grid_constant__ Batch B)
     }
     for (int x = tid; x < G * kLadderLevels; x += blockDim.x)
       P.ladder[(int64_t)list0 * kLadderLevels + x] = 0;
+    if (tid == 0) P.next_unit[slab] = 0;
     for (int u = slab * blockDim.x + tid; u < P.ucap; u += n_slabs * blockDim.x) P.votes[u] = 0;
     if (slab == 0 && tid < 4) P.counts[tid] = 0;
     if (slab == 0 && tid == 0) *P.status = 0u;
@@ -167,10 +168,11 @@ cudaError_t launch_prep(const Batch& B, cudaStream_t s) {
 // ---------------------------------------------------------------------------
 // Scoring kernel.
 //
-// Grid: one CTA per (problem, slab = (layer i, key head g), chunk of history units).
+// Grid: P.chunks CTAs per (problem, slab = (layer i, key head g)), one wave.
 // Block: kScoreWarps compute warps + 1 threshold warp.
 //
-// Compute warps take the chunk's units round-robin and walk each unit in tiles of 16
+// All compute warps of a slab's CTAs take history units from the slab's shared unit
+// counter, so SMs that run faster score more units, and walk each unit in tiles of 16
 // tokens. Each warp streams its tiles through its own ring of kScoreStages shared
 // memory buffers with TMA bulk copies (cp.async.bulk + mbarrier transaction counts),
 // so the data in flight costs no registers. A tile's scores for the G query heads
@@ -182,12 +184,14 @@ cudaError_t launch_prep(const Batch& B, cudaStream_t s) {
 //
 // Candidate filter: a token is appended to its list when s >= thr[h], where thr[h] is
 // always a lower bound of the list's k-th best score, so every top-k token is
-// appended. Every appended score also counts in the list's global histogram (bins
-// = top 14 bits of the order-preserving image of s). The threshold warp of each CTA
-// scans its lists' histograms from the highest non-empty bin down: the lower edge of
-// the bin where the count reaches k bounds the k-th best score from below, because
-// at least k appended tokens (of any CTA) score that much. The bound therefore
-// tracks the k-th best of everything scored so far by the whole grid.
+// appended. Every appended score also counts in the CTA's ladder for its list (256
+// levels 1/16 apart in log2 units, anchored at the list's best sampled unit); the
+// threshold warp merges the CTA's counts into the list's global ladder and scans it
+// from the top: the level where the count first reaches k bounds the k-th best score
+// from below, because at least k appended tokens (of any CTA) score that much. The
+// bound, shared through gthr, tracks the k-th best of everything scored so far.
+// Each unit's softmax statistics (max, sum 2^(s - max)) are written per list; the
+// list totals are combined later in unit order, whichever warp scored a unit.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ void mma_16816(float (&d)[4], uint32_t a0, uint32_t a1,
                                           uint32_t a2, uint32_t a3, uint32_t b0,
@@ -207,13 +211,15 @@ __device__ __forceinline__ uint4 ld_stream(const void* p) {
   return r;
 }
 
+constexpr int kUnitQueue = 8;  // > units a warp's issue cursor can run ahead
+
 struct ScoreShared {
   int lad[kMaxGroup][kLadderLevels];  // this CTA's appended-score counts not yet merged
   float thr[kMaxGroup];
   float anchor[kMaxGroup];
   int all_done;
   unsigned long long bar[kScoreWarps][kScoreStages];  // one mbarrier per warp stage
-  float2 wstat[kScoreWarps][kMaxGroup];  // per warp: its units' (max, sum) per list
+  int uq[kScoreWarps][kUnitQueue];      // per warp: units taken, in order
 };
 
 // ---- TMA bulk copies and mbarriers (inline PTX) ----
@@ -370,10 +376,8 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
   const int local = b - P.cta_begin;
   const int n_slabs = P.P * P.Hkv;
   if (P.chunks <= 0) return;
-  const int slab = local / P.chunks, chunk = local - slab * P.chunks;
+  const int slab = local / P.chunks;
   if (slab >= n_slabs) return;
-  const int u0 = (int)(((int64_t)P.Uh * chunk) / P.chunks);
-  const int u1 = (int)(((int64_t)P.Uh * (chunk + 1)) / P.chunks);
 
   const int i = slab / P.Hkv, kvh = slab - i * P.Hkv;
   const int G = P.G;
@@ -383,12 +387,11 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
   for (int x = threadIdx.x; x < kMaxGroup * kLadderLevels; x += blockDim.x)
     (&S.lad[0][0])[x] = 0;
   if (threadIdx.x < kMaxGroup) {
-    S.thr[threadIdx.x] = -INFINITY;
+    // a CTA that starts late begins with the bound published by the earlier ones
+    S.thr[threadIdx.x] = threadIdx.x < G ? ordered_to_float(P.gthr[list0 + threadIdx.x]) : -INFINITY;
     S.anchor[threadIdx.x] = threadIdx.x < G ? list_anchor(P, list0 + threadIdx.x) : 0.f;
   }
   if (threadIdx.x == 0) S.all_done = 0;
-  if (threadIdx.x < kScoreWarps * kMaxGroup)
-    (&S.wstat[0][0])[threadIdx.x] = make_float2(-INFINITY, 0.f);
   if (threadIdx.x < kScoreWarps * kScoreStages)
     mbar_init(smem_u32(&S.bar[0][0] + threadIdx.x), 1u);
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -424,11 +427,8 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
   const int L0 = list0 + c0, L1 = list0 + c1;
   const int Tu = P.Tu;
   const int tpu = (Tu + kTileRows - 1) / kTileRows;
-  const int n_chunk_units = u1 - u0;
-  const int n_my = n_chunk_units > warp
-                       ? (n_chunk_units - warp + kScoreWarps - 1) / kScoreWarps
-                       : 0;
-  const int ntiles = n_my * tpu;
+  const int Uh = P.Uh;
+  int* next_unit = P.next_unit + slab;
   const __nv_bfloat16* slab_keys = P.keys + (int64_t)slab * P.ncap * kHeadDim;
   const int64_t cbase0 = (int64_t)(hv0 ? L0 : list0) * P.cand_cap;
   const int64_t cbase1 = (int64_t)(hv1 ? L1 : list0) * P.cand_cap;
@@ -506,7 +506,7 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
   // Lane 0 starts the bulk copy of tile t (unit uu, tile jj of the unit) into its
   // stage once the warp's reads of that stage are ordered before the async write.
   auto issue = [&](int t, int uu, int jj) {
-    if (t >= ntiles) return;
+    if (uu >= Uh) return;
     const int r0 = kTileRows * jj;
     const int nrows = min(kTileRows, Tu - r0);
     const int st = t % kScoreStages;
@@ -521,25 +521,40 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
     }
   };
 
-  // tile cursors: the tile being consumed and the tile being issued
-  int cu = u0 + warp, cj = 0;          // consume position
-  int iu = u0 + warp, ij = 0;          // issue position
-  auto advance = [&](int& uu, int& jj) {
-    if (++jj == tpu) {
-      jj = 0;
-      uu += kScoreWarps;
+  // Units come from the slab's shared counter: every warp of the slab's CTAs takes the
+  // next unit when it needs one, so faster SMs score more units. Lane 0 takes its next
+  // unit one unit ahead (the atomic's latency hides behind a unit of work); the units a
+  // warp takes are queued in shared memory for its consume cursor.
+  int* uq = S.uq[warp];
+  int pre = lane == 0 ? atomicAdd(next_unit, 1) : 0;
+  auto take = [&]() {
+    const int u = __shfl_sync(0xffffffffu, pre, 0);
+    if (lane == 0) pre = u < Uh ? atomicAdd(next_unit, 1) : Uh;
+    return min(u, Uh);
+  };
+  int iu = take(), ij = 0, nq = 0;     // issue position, units queued
+  if (lane == 0) uq[0] = iu;
+  nq = 1;
+  __syncwarp();
+  int cu = iu, cj = 0, qh = 0;         // consume position, queue head
+  auto advance_issue = [&]() {
+    if (++ij == tpu) {
+      ij = 0;
+      iu = iu < Uh ? take() : Uh;
+      if (lane == 0) uq[nq % kUnitQueue] = iu;
+      ++nq;
+      __syncwarp();
     }
   };
   for (int t = 0; t < kScoreStages; ++t) {
     issue(t, iu, ij);
-    advance(iu, ij);
+    advance_issue();
   }
 
   float m0 = -INFINITY, l0 = 0.f, m1 = -INFINITY, l1 = 0.f;
-  float wm0 = -INFINITY, wl0 = 0.f, wm1 = -INFINITY, wl1 = 0.f;  // this warp's units so far
   int t = 0;
   bool aborted = false;
-  for (; t < ntiles; ++t) {
+  for (; cu < Uh; ++t) {
     const int st = t % kScoreStages;
     const bool ok = mbar_wait_bounded(my_bars + 8u * st, (uint32_t)((t / kScoreStages) & 1));
     if (!__all_sync(0xffffffffu, ok)) {
@@ -562,9 +577,13 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
       mma_16816(acd, ra[v].z, rb[v].z, ra[v].w, rb[v].w, qf[2 * v + 1][0], qf[2 * v + 1][1]);
     }
     const int u = cu, j = cj;
-    advance(cu, cj);
+    if (++cj == tpu) {
+      cj = 0;
+      ++qh;
+      cu = uq[qh % kUnitQueue];
+    }
     issue(t + kScoreStages, iu, ij);   // the stage's data now sits in registers
-    advance(iu, ij);
+    advance_issue();
 
     if (j == 0) {
       m0 = m1 = -INFINITY;
@@ -594,8 +613,6 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
       if (g == 0) {
         if (hv0) P.ustats[(int64_t)L0 * P.ucap + u] = make_float2(m0, l0);
         if (hv1) P.ustats[(int64_t)L1 * P.ucap + u] = make_float2(m1, l1);
-        ml_combine(wm0, wl0, m0, l0);
-        ml_combine(wm1, wl1, m1, l1);
       }
     }
   }
@@ -605,32 +622,19 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
   if (aborted) {
     // report, then let the copies already in flight land before the CTA exits
     if (lane == 0) atomicOr(P.status, kStatusTimeout);
-    for (int r = t; r < min(ntiles, t + kScoreStages); ++r)
+    // stages of tiles t .. t + kScoreStages - 1 that were issued (units < Uh)
+    int ru = cu, rj = cj, rq = qh;
+    for (int r = t; r < t + kScoreStages && ru < Uh; ++r) {
       mbar_wait_bounded(my_bars + 8u * (r % kScoreStages), (uint32_t)((r / kScoreStages) & 1));
-  }
-  // The chunk's (max, sum) per list: the warps' partials (each over its units in
-  // order) combined in warp order by the last warp to finish.
-  if (g == 0) {
-    if (hv0) S.wstat[warp][c0] = make_float2(wm0, wl0);
-    if (hv1) S.wstat[warp][c1] = make_float2(wm1, wl1);
-  }
-  __threadfence_block();
-  __syncwarp();
-  int order = 0;
-  if (lane == 0) order = atomicAdd(&S.all_done, 1);
-  order = __shfl_sync(0xffffffffu, order, 0);
-  if (order == kScoreWarps - 1) {
-    __threadfence_block();
-    if (lane < G) {
-      float m = -INFINITY, l = 0.f;
-      const volatile float2* ws = &S.wstat[0][0];
-      for (int w = 0; w < kScoreWarps; ++w) {
-        const float mw = ws[w * kMaxGroup + lane].x, lw = ws[w * kMaxGroup + lane].y;
-        ml_combine(m, l, mw, lw);
+      if (++rj == tpu) {
+        rj = 0;
+        ++rq;
+        ru = rq < nq ? uq[rq % kUnitQueue] : Uh;
       }
-      P.cstats[(int64_t)(list0 + lane) * kMaxChunksPerSlab + chunk] = make_float2(m, l);
     }
   }
+  __threadfence_block();
+  if (lane == 0) atomicAdd(&S.all_done, 1);
 }
 
 int score_chunks_per_slab(int n_slabs_total, int hist_units, int sm_count) {

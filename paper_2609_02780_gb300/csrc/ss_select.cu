@@ -15,7 +15,6 @@ namespace ss {
 
 constexpr int kSelThreads = 1024;
 constexpr int kMassUnits = 32;     // history units per mass block
-constexpr int kMaxLists = 1024;    // P * Hq per problem
 constexpr int kSelCap = 16384;   // survivors sorted in shared memory
 constexpr int kFineBins = 2048;  // second-level score histogram of k_select
 
@@ -114,6 +113,39 @@ __device__ __forceinline__ int next_pow2(int x) {
   return p;
 }
 
+// Block reduction of (max, sum 2^(s - max)) pairs in a fixed order; result to all.
+__device__ void block_ml(float& m, float& l, float* sm, float* sl) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nw = blockDim.x >> 5;
+  for (int off = 16; off > 0; off >>= 1) {
+    const float mo = __shfl_down_sync(0xffffffffu, m, off);
+    const float lo = __shfl_down_sync(0xffffffffu, l, off);
+    ml_combine(m, l, mo, lo);
+  }
+  if (lane == 0) {
+    sm[warp] = m;
+    sl[warp] = l;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    m = lane < nw ? sm[lane] : -INFINITY;
+    l = lane < nw ? sl[lane] : 0.f;
+    for (int off = 16; off > 0; off >>= 1) {
+      const float mo = __shfl_down_sync(0xffffffffu, m, off);
+      const float lo = __shfl_down_sync(0xffffffffu, l, off);
+      ml_combine(m, l, mo, lo);
+    }
+    if (lane == 0) {
+      sm[0] = m;
+      sl[0] = l;
+    }
+  }
+  __syncthreads();
+  m = sm[0];
+  l = sl[0];
+  __syncthreads();
+}
+
 __device__ float block_min(float v, float* sm) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int nw = blockDim.x >> 5;
@@ -139,13 +171,10 @@ __device__ float block_min(float v, float* sm) {
 // If they do not fit (massive ties), an 8-pass radix select on the 64-bit keys over
 // the candidate array finds the n-th key exactly.
 // ---------------------------------------------------------------------------
-__device__ void unit_mass_block(const Prob& P, int blk);
-
-__global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ Batch B,
-                                                        int select_blocks) {
+__global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ Batch B) {
   extern __shared__ unsigned long long skeys[];
   __shared__ int s_hist[kFineBins];
-  __shared__ float s_m[32];
+  __shared__ float s_m[32], s_l[32];
   __shared__ int s_n, s_bstar, s_rem;
   __shared__ unsigned long long s_prefix;
 
@@ -155,18 +184,23 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
   if (pi >= B.n) return;
   const Prob& P = B.p[pi];
   const int n_lists = P.P * P.Hq;
-  if ((int)blockIdx.x >= select_blocks) {
-    unit_mass_block(P, blockIdx.x - select_blocks);
-    return;
-  }
   const int L = blockIdx.x;
   if (L >= n_lists) return;
   const int tid = threadIdx.x, lane = tid & 31;
   const int k = B.k;
 
-  const float2 mlv = list_stats_of(P, L);
-  const float M = mlv.x, Ls = mlv.y;
-  if (tid == 0) P.list_ml[L] = mlv;
+  // softmax statistics from the per-unit pairs in a fixed order (thread t takes units
+  // t, t + 1024, ...; then a fixed tree), whichever warps scored the units
+  float M = -INFINITY, Ls = 0.f;
+  {
+    const float2* us = P.ustats + (int64_t)L * P.ucap;
+    for (int u = tid; u < P.Uh; u += blockDim.x) {
+      const float2 v = us[u];
+      ml_combine(M, Ls, v.x, v.y);
+    }
+    block_ml(M, Ls, s_m, s_l);
+  }
+  if (tid == 0) P.list_ml[L] = make_float2(M, Ls);
 
   int32_t* tok_out = P.topk_tok + (int64_t)L * k;
   float* w_out = P.topk_w + (int64_t)L * k;
@@ -397,36 +431,36 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
   (void)lane;
 }
 
-cudaError_t launch_select(const Batch& B, int max_lists, int max_hist_units, cudaStream_t s) {
+cudaError_t launch_select(const Batch& B, int max_lists, cudaStream_t s) {
   const int smem = kSelCap * (int)sizeof(unsigned long long);
   cudaError_t e = cudaFuncSetAttribute(k_select, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  const int mass_blocks = (max_hist_units + kMassUnits - 1) / kMassUnits;
-  dim3 grid(max_lists + mass_blocks, B.n);
-  return launch_pdl(k_select, grid, dim3(kSelThreads), (size_t)smem, s, B, max_lists);
+  return launch_pdl(k_select, dim3(max_lists, B.n), dim3(kSelThreads), (size_t)smem, s, B);
 }
 
 // ---------------------------------------------------------------------------
-// Attention mass of every history unit (blocks of k_select past the lists): over lists
-// in a fixed order, the sum of 2^(m_u - M) l_u / L, i.e. the normalised weights of all
-// the unit's tokens. A block covers kMassUnits units with 32 warps: warp w sums lists
-// w, w + 32, ... for 32 units, then the 32 partial sums are added in warp order.
+// Attention mass of every history unit: over lists in a fixed order, the sum of
+// 2^(m_u - M) l_u / L, i.e. the normalised weights of all the unit's tokens. A block
+// covers 32 units with 32 warps: warp w sums lists w, w + 32, ..., then the 32 partial
+// sums are added in warp order (deterministic).
 // ---------------------------------------------------------------------------
-__device__ void unit_mass_block(const Prob& P, int blk) {
+__global__ void __launch_bounds__(1024) k_mass(const __grid_constant__ Batch B) {
   __shared__ float part[32][33];
-  __shared__ float2 ml[kMaxLists];
+  pdl_wait();
+  pdl_release();
+  const int pi = blockIdx.y;
+  if (pi >= B.n) return;
+  const Prob& P = B.p[pi];
   const int n_lists = P.P * P.Hq;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  if (blk * kMassUnits >= P.Uh) return;
-  for (int L = threadIdx.x; L < n_lists; L += blockDim.x) ml[L] = list_stats_of(P, L);
-  __syncthreads();
-  const int u = blk * kMassUnits + lane;
+  if ((int)blockIdx.x * kMassUnits >= P.Uh) return;
+  const int u = blockIdx.x * kMassUnits + lane;
   float acc = 0.f;
   if (u < P.Uh) {
 #pragma unroll 4
     for (int L = warp; L < n_lists; L += 32) {
       const float2 st = P.ustats[(int64_t)L * P.ucap + u];
-      const float2 m = ml[L];
+      const float2 m = P.list_ml[L];
       if (st.x != -INFINITY) acc += st.y * fast_exp2(st.x - m.x) / m.y;
     }
   }
@@ -438,6 +472,12 @@ __device__ void unit_mass_block(const Prob& P, int blk) {
     for (int w = 0; w < 32; ++w) mm += part[w][lane];
     P.mass[u] = mm;
   }
+}
+
+cudaError_t launch_mass(const Batch& B, int max_hist_units, cudaStream_t s) {
+  const int blocks = (max_hist_units + kMassUnits - 1) / kMassUnits;
+  if (blocks == 0) return cudaSuccess;
+  return launch_pdl(k_mass, dim3(blocks, B.n), dim3(1024), 0, s, B);
 }
 
 // ---------------------------------------------------------------------------
