@@ -258,6 +258,27 @@ ss_status ss_retrieve_host(ss_index* index, const void* q_host, int32_t n_rows,
                            const ss_retrieve_params* params, const ss_host_result* out,
                            void* workspace, size_t workspace_bytes, void* stream);
 
+/* ss_retrieve with no allocation and no caller workspace (the paper has no
+ * counterpart: this is a deployment entry point). For callers that cannot allocate
+ * device memory at question time: a serving loop whose device memory is committed to
+ * its KV cache pool, where a cudaMalloc can fail; a host linking only this library,
+ * with no device allocator of its own; a latency-bound loop that cannot take cudaFree's
+ * implicit device synchronisation. The workspace is a fixed 64 MiB array in the
+ * library's device memory (one per device, reserved when the library's device code is
+ * loaded). The first call on each device looks up that array's address with the
+ * device current (one-time set-up); make that first call before any stream capture.
+ * Nothing in the scratch has to start at zero: the first kernel of every call resets
+ * the counters that later kernels accumulate into. Every call on a device uses the same
+ * scratch, so calls that overlap (other streams or host threads on that device, before
+ * the previous call's kernels have finished) race and give wrong results: order them,
+ * e.g. on one stream. Outputs as ss_retrieve; the result arrays are the caller's.
+ * Errors as ss_retrieve, plus CAPACITY when the call's workspace (the size
+ * ss_retrieve_workspace_size reports for n = 1) exceeds 64 MiB, and UNSUPPORTED on a
+ * device ordinal >= 64. */
+ss_status ss_retrieve_static(ss_index* index, const void* q, int32_t n_rows,
+                             const ss_retrieve_params* params, const ss_result* result,
+                             void* stream);
+
 /* Synchronizes `stream` and returns the status recorded in the device word `status`
  * by earlier retrievals on it (SS_OK, SS_ERR_TIMEOUT or SS_ERR_INTERNAL). */
 ss_status ss_status_sync(const uint32_t* status, void* stream);

@@ -259,6 +259,26 @@ class Index:
         return retrieve_batched([self], [q], p, outs=[out] if out else None,
                                 workspace=workspace, trace=trace)[0]
 
+    def retrieve_static(self, q: torch.Tensor, p: RetrieveParams, out: Result) -> Result:
+        """The retrieval of `retrieve` through ss_retrieve_static: the library allocates
+        nothing and uses its fixed 64 MiB per-device scratch, for callers that cannot
+        allocate device memory at question time. `out` is preallocated by the caller;
+        calls on one device must not overlap (they share the scratch). Asynchronous on
+        the current stream."""
+        if q.dtype != torch.bfloat16 or q.dim() != 4 or not q.is_contiguous():
+            raise ValueError("q must be contiguous bf16 [P][R][Hq][128]")
+        if q.device != self.device:
+            raise ValueError("q must be on the index's device")
+        if q.shape[0] != self.n_layers or q.shape[2] != self.n_q_heads or q.shape[3] != 128:
+            raise ValueError("q shape does not match the index")
+        with torch.cuda.device(self.device):
+            _check(_lib().ss_retrieve_static(self.handle, C.c_void_p(q.data_ptr()),
+                                             q.shape[1], C.byref(p.to_c()),
+                                             C.byref(out.to_c()),
+                                             C.c_void_p(_stream_ptr(self.device))))
+        out._keep = (q,)
+        return out
+
     def retrieve_host(self, q_host: torch.Tensor, p: RetrieveParams,
                       workspace: torch.Tensor | None = None) -> dict:
         """ss_retrieve_host: q in (pinned) host memory, selection copied back to host."""

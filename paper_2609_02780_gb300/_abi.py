@@ -82,6 +82,9 @@ SIGNATURES = {
     "ss_retrieve_host": (c_status, [C.c_void_p, C.c_void_p, C.c_int32,
                                     C.POINTER(RetrieveParams), C.POINTER(HostResult),
                                     C.c_void_p, C.c_size_t, C.c_void_p]),
+    "ss_retrieve_static": (c_status, [C.c_void_p, C.c_void_p, C.c_int32,
+                                      C.POINTER(RetrieveParams), C.POINTER(Result),
+                                      C.c_void_p]),
     "ss_status_sync": (c_status, [C.c_void_p, C.c_void_p]),
 }
 

@@ -3,6 +3,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <vector>
 
 #include "shallowstream.h"
@@ -491,4 +492,62 @@ SS_EXPORT ss_status ss_retrieve_host(ss_index* ix, const void* q_host, int32_t R
   SS_CUDA(cudaMemcpyAsync(out->frames, r.frames, nexp * c.frames_per_unit * 4, cudaMemcpyDeviceToHost, st));
   SS_CUDA(cudaMemcpyAsync(out->counts, r.counts, 16, cudaMemcpyDeviceToHost, st));
   return ss_status_sync(r.status, stream);
+}
+
+// ---------------------------------------------------------------------------
+// Retrieval without any allocation. Some callers cannot allocate device memory at
+// question time: a serving loop whose device memory is all committed to its KV cache
+// pool (a cudaMalloc there can fail outright), a host that links only this C library
+// and has no device allocator of its own, and latency-bound loops that cannot afford
+// cudaFree's implicit device synchronisation. For them the workspace lives in the
+// module's own memory: a fixed array of kStaticScratchBytes per device, reserved when
+// the library's device code is loaded.
+// ---------------------------------------------------------------------------
+namespace {
+
+constexpr size_t kStaticScratchBytes = size_t(64) << 20;  // 64 MiB
+constexpr int kMaxStaticDevices = 64;
+
+__device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
+
+std::mutex g_static_mu;
+void* g_static_ptr[kMaxStaticDevices] = {};
+
+// The scratch's device address on `dev` (which must be current); looked up once per
+// device, on that device's first call.
+ss_status static_scratch(int dev, void** out) {
+  if (dev < 0 || dev >= kMaxStaticDevices)
+    return fail(SS_ERR_UNSUPPORTED, "device %d: static scratch supports devices [0, %d)", dev,
+                kMaxStaticDevices);
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  if (!g_static_ptr[dev]) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch);
+    if (e != cudaSuccess)
+      return fail(SS_ERR_CUDA, "cudaGetSymbolAddress(static scratch): %s", cudaGetErrorString(e));
+    g_static_ptr[dev] = p;
+  }
+  *out = g_static_ptr[dev];
+  return SS_OK;
+}
+
+}  // namespace
+
+SS_EXPORT ss_status ss_retrieve_static(ss_index* ix, const void* q, int32_t R,
+                                       const ss_retrieve_params* p, const ss_result* res,
+                                       void* stream) {
+  if (!ix || !q || !p || !res) return fail(SS_ERR_INVALID_ARG, "NULL argument");
+  ss_status s = check_params(p);
+  if (s != SS_OK) return s;
+  if (R < 1) return fail(SS_ERR_INVALID_ARG, "n_rows must be >= 1");
+  const size_t need = layout_of(ix, R, p).total;
+  if (need > kStaticScratchBytes)
+    return fail(SS_ERR_CAPACITY,
+                "this retrieval needs %zu bytes of workspace; the static scratch holds %zu",
+                need, kStaticScratchBytes);
+  SS_CUDA(cudaSetDevice(ix->device));
+  void* ws = nullptr;
+  s = static_scratch(ix->device, &ws);
+  if (s != SS_OK) return s;
+  return ss_retrieve(ix, q, R, p, res, ws, kStaticScratchBytes, stream, nullptr);
 }
