@@ -91,13 +91,16 @@ typedef struct {
   const uint8_t* assignment; /* device uint8 [P][Hkv][N_cap]: centroid of each token of a
                                 compressed window (window-local id) or NULL */
   const int32_t* window_first_unit; /* device int32 [W_cap] or NULL */
+  const int32_t* member_counts; /* device int32 [P][Hkv][W_cap][n_centroids][window units]:
+                                   members of each centroid in each unit of its window */
+  const int32_t* member_sizes;  /* device int32 [P][Hkv][W_cap][n_centroids] */
 } ss_index_view;
 
 /* k-means compression of the frames [first_frame, first_frame + n_frames) in
  * windows of window_frames (see ss_index_compress). */
 typedef struct {
   int32_t window_frames;     /* frames per window, a multiple of frames_per_unit */
-  int32_t n_centroids;       /* 1..256 and <= window_frames * T_f */
+  int32_t n_centroids;       /* 1..128 and <= window_frames * T_f (<= 65536 tokens) */
   int32_t iters;             /* Lloyd rounds >= 1 */
   int64_t first_frame;       /* multiple of window_frames */
   int64_t n_frames;          /* multiple of window_frames */
@@ -200,11 +203,16 @@ ss_status ss_index_get_view(const ss_index* index, ss_index_view* view);
  * keys, C0 = X's first n_centroids tokens, then `iters` Lloyd rounds (assign each key
  * to the nearest centroid by squared L2, lowest id on ties; move each centroid to the
  * fp32 mean of its members, empty ones unchanged). Stores the last round's centroids
- * (bf16, nearest-even) and memberships. The first call fixes window_frames and
+ * (bf16, nearest-even) and memberships. Distances are compared as ||c||^2 - 2 x . c in
+ * fp32 (x . c on the tensor cores with c split into two bf16 parts), so a key whose two
+ * nearest centroids are within that rounding of each other may take either; the sums
+ * of the update run in token order (results repeat bit for bit). The first call fixes
+ * window_frames and
  * n_centroids (later calls must match, with windows after those already compressed)
  * and allocates the cluster arrays from the index's allocator.
  * Errors: INVALID_ARG (misaligned ranges, frames not yet appended, overlap with a
- * compressed window), UNSUPPORTED (n_centroids > 256 or > window tokens), ALLOC,
+ * compressed window), UNSUPPORTED (n_centroids > 128 or > window tokens, windows of more
+ * than 65536 tokens), ALLOC,
  * CUDA. */
 ss_status ss_index_compress(ss_index* index, const ss_compress_params* params,
                             void* stream);

@@ -210,6 +210,28 @@ class Index:
         return self._block_view(v.keys, torch.bfloat16,
                                 (self.n_layers, self.n_kv_heads, v.token_capacity, 128))
 
+    def clusters(self) -> dict:
+        """Views of the compressed windows' device arrays (after compress()):
+        centroids bf16 [P][Hkv][n_windows][n_c][128], assignment uint8 [P][Hkv][capacity],
+        member_counts int32 [P][Hkv][n_windows][n_c][units per window], member_sizes
+        int32 [P][Hkv][n_windows][n_c], window_first_unit int32 [n_windows]."""
+        v = self.view()
+        if v.window_frames == 0:
+            raise ValueError("the index has no compressed windows")
+        P, H, nc = self.n_layers, self.n_kv_heads, v.n_centroids
+        wcap = self.unit_capacity * self.frames_per_unit // v.window_frames
+        wu = v.window_frames // self.frames_per_unit
+        nw = v.n_windows
+        cent = self._block_view(v.centroids, torch.bfloat16, (P, H, wcap, nc, 128))
+        asg = self._block_view(v.assignment, torch.uint8, (P, H, v.token_capacity))
+        mc = self._block_view(v.member_counts, torch.int32, (P, H, wcap, nc, wu))
+        ms = self._block_view(v.member_sizes, torch.int32, (P, H, wcap, nc))
+        wf = self._block_view(v.window_first_unit, torch.int32, (wcap,))
+        return {"centroids": cent[:, :, :nw], "assignment": asg,
+                "member_counts": mc[:, :, :nw], "member_sizes": ms[:, :, :nw],
+                "window_first_unit": wf[:nw], "window_frames": v.window_frames,
+                "n_centroids": nc}
+
     def append(self, keys: torch.Tensor, n_frames: int | None = None) -> None:
         """Appends frames of shallow keys bf16 [P][Hkv][S][128] (the first
         n_frames * T_f tokens of each slab; S may exceed that)."""

@@ -28,7 +28,8 @@ class IndexView(C.Structure):
                 ("keys", C.c_void_p), ("descriptors", C.c_void_p), ("n_windows", C.c_int32),
                 ("window_frames", C.c_int32), ("n_centroids", C.c_int32),
                 ("centroids", C.c_void_p), ("assignment", C.c_void_p),
-                ("window_first_unit", C.c_void_p)]
+                ("window_first_unit", C.c_void_p), ("member_counts", C.c_void_p),
+                ("member_sizes", C.c_void_p)]
 
 
 class CompressParams(C.Structure):

@@ -34,6 +34,9 @@ struct ss_index {
   __nv_bfloat16* cent;  // [P*Hkv][wcap*nc][d]
   uint8_t* assign;      // [P*Hkv][ncap]
   int32_t* win_u0;      // [wcap]
+  int32_t* win_slot;    // [ucap / units per window]: window of each window slot, or -1
+  int32_t* mcnt;        // [P*Hkv][wcap][nc][units per window] members per (centroid, unit)
+  int32_t* msize;       // [P*Hkv][wcap][nc] members per centroid
 };
 
 namespace {
@@ -362,6 +365,9 @@ SS_EXPORT ss_status ss_index_destroy(ss_index* ix) {
   dev_free(ix, ix->cent);
   dev_free(ix, ix->assign);
   dev_free(ix, ix->win_u0);
+  dev_free(ix, ix->win_slot);
+  dev_free(ix, ix->mcnt);
+  dev_free(ix, ix->msize);
   delete ix;
   return SS_OK;
 }
@@ -407,13 +413,82 @@ SS_EXPORT ss_status ss_index_get_view(const ss_index* ix, ss_index_view* v) {
   v->centroids = ix->cent;
   v->assignment = ix->assign;
   v->window_first_unit = ix->win_u0;
+  v->member_counts = ix->mcnt;
+  v->member_sizes = ix->msize;
   return SS_OK;
 }
 
 SS_EXPORT ss_status ss_index_compress(ss_index* ix, const ss_compress_params* cp, void* stream) {
-  (void)stream;
   if (!ix || !cp) return fail(SS_ERR_INVALID_ARG, "NULL argument");
-  return fail(SS_ERR_UNSUPPORTED, "compression is not available in this build");
+  const ss_index_config& c = ix->cfg;
+  const ss_compress_params& q = *cp;
+  if (q.window_frames < 1 || q.window_frames % c.frames_per_unit)
+    return fail(SS_ERR_INVALID_ARG, "window_frames must be a positive multiple of frames_per_unit");
+  if (q.iters < 1) return fail(SS_ERR_INVALID_ARG, "iters must be >= 1");
+  if (q.first_frame < 0 || q.n_frames < 0 || q.first_frame % q.window_frames ||
+      q.n_frames % q.window_frames)
+    return fail(SS_ERR_INVALID_ARG, "first_frame and n_frames must be multiples of window_frames");
+  if (q.first_frame + q.n_frames > ix->n_frames)
+    return fail(SS_ERR_INVALID_ARG, "frames [%lld, %lld) are not all appended (have %lld)",
+                (long long)q.first_frame, (long long)(q.first_frame + q.n_frames),
+                (long long)ix->n_frames);
+  const int64_t wt = (int64_t)q.window_frames * c.tokens_per_frame;
+  if (q.n_centroids < 1 || q.n_centroids > kMaxCentroids)
+    return fail(SS_ERR_UNSUPPORTED, "n_centroids must be in [1, %d]", kMaxCentroids);
+  if (q.n_centroids > wt) return fail(SS_ERR_UNSUPPORTED, "n_centroids > tokens per window");
+  if (wt > kMaxWindowTokens)
+    return fail(SS_ERR_UNSUPPORTED, "more than %d tokens per window", kMaxWindowTokens);
+  if (ix->win_frames) {
+    if (q.window_frames != ix->win_frames || q.n_centroids != ix->n_centroids)
+      return fail(SS_ERR_INVALID_ARG, "window_frames / n_centroids differ from the first compression");
+    const int64_t end = ix->win_first_frame.back() + ix->win_frames;
+    if (q.first_frame < end)
+      return fail(SS_ERR_INVALID_ARG, "frames before %lld are already compressed", (long long)end);
+  }
+  if (q.n_frames == 0) return SS_OK;
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  SS_CUDA(cudaSetDevice(ix->device));
+  const int n_slabs = c.n_layers * c.n_kv_heads;
+  const int wu = q.window_frames / c.frames_per_unit;
+  if (!ix->win_frames) {
+    const int64_t wcap = c.max_frames / q.window_frames;
+    const int64_t n_slots = (ix->ucap + wu - 1) / wu;
+    const size_t cb = (size_t)n_slabs * wcap * q.n_centroids * kHeadDim * 2;
+    const size_t ab = (size_t)n_slabs * ix->ncap;
+    const size_t mb = (size_t)n_slabs * wcap * q.n_centroids * wu * 4;
+    const size_t sb = (size_t)n_slabs * wcap * q.n_centroids * 4;
+    ix->cent = static_cast<__nv_bfloat16*>(dev_alloc(ix, cb, st));
+    ix->assign = static_cast<uint8_t*>(dev_alloc(ix, ab, st));
+    ix->mcnt = static_cast<int32_t*>(dev_alloc(ix, mb, st));
+    ix->msize = static_cast<int32_t*>(dev_alloc(ix, sb, st));
+    ix->win_u0 = static_cast<int32_t*>(dev_alloc(ix, (size_t)wcap * 4, st));
+    ix->win_slot = static_cast<int32_t*>(dev_alloc(ix, (size_t)n_slots * 4, st));
+    if (!ix->cent || !ix->assign || !ix->mcnt || !ix->msize || !ix->win_u0 || !ix->win_slot) {
+      dev_free(ix, ix->cent);
+      dev_free(ix, ix->assign);
+      dev_free(ix, ix->mcnt);
+      dev_free(ix, ix->msize);
+      dev_free(ix, ix->win_u0);
+      dev_free(ix, ix->win_slot);
+      ix->cent = nullptr;
+      ix->assign = nullptr;
+      ix->mcnt = ix->msize = ix->win_u0 = ix->win_slot = nullptr;
+      return fail(SS_ERR_ALLOC, "device allocation of the cluster arrays failed");
+    }
+    SS_CUDA(cudaMemsetAsync(ix->win_slot, 0xff, (size_t)n_slots * 4, st));
+    ix->wcap = (int32_t)wcap;
+    ix->win_frames = q.window_frames;
+    ix->n_centroids = q.n_centroids;
+  }
+  const int n_new = (int)(q.n_frames / q.window_frames);
+  SS_CUDA(launch_kmeans(ix->keys, ix->ncap, n_slabs, ix->cent, ix->assign, ix->mcnt, ix->msize,
+                        ix->win_u0, ix->win_slot, ix->wcap, ix->n_windows, n_new, q.first_frame,
+                        q.window_frames, c.tokens_per_frame, c.frames_per_unit, q.n_centroids,
+                        q.iters, st));
+  for (int j = 0; j < n_new; ++j)
+    ix->win_first_frame.push_back(q.first_frame + (int64_t)j * q.window_frames);
+  ix->n_windows += n_new;
+  return SS_OK;
 }
 
 SS_EXPORT ss_status ss_retrieve_workspace_size(const ss_index* const* ix, int32_t n,

@@ -21,6 +21,8 @@ constexpr int kMaxPool = 1024;         // pool = pool_mult * budget
 constexpr int kMaxHistUnits = 16384;   // history units per problem (pool sort in smem)
 constexpr int kMaxGroup = 8;           // query heads per key head
 constexpr uint32_t kCentroidIdBase = 0x40000000u;
+constexpr int kMaxCentroids = 128;     // per window (k-means compression)
+constexpr int kMaxWindowTokens = 65536;
 
 // Score-kernel geometry: kScoreWarps compute warps + 1 threshold warp per CTA.
 #ifndef SS_SCORE_WARPS
@@ -194,6 +196,12 @@ cudaError_t launch_maxmin(const Batch& B, int max_pool, cudaStream_t s);
 cudaError_t launch_append(__nv_bfloat16* keys, int64_t ncap, int64_t tok0,
                           const __nv_bfloat16* src, int64_t src_stride_tokens,
                           int n_slabs, int64_t n_tokens, cudaStream_t s);
+size_t kmeans_smem_bytes(int n_c, int window_tokens);
+cudaError_t launch_kmeans(const __nv_bfloat16* keys, int64_t ncap, int n_slabs,
+                          __nv_bfloat16* cent, uint8_t* assign, int32_t* mcnt, int32_t* msize,
+                          int32_t* win_u0, int32_t* win_slot, int wcap, int w_begin, int n_new,
+                          int64_t first_frame, int window_frames, int tokens_per_frame,
+                          int frames_per_unit, int n_c, int iters, cudaStream_t s);
 cudaError_t launch_descriptors(const __nv_bfloat16* keys, int64_t ncap, int P, int Hkv,
                                int Tu, int64_t u_begin, int64_t u_end, float* desc,
                                cudaStream_t s);

@@ -12,6 +12,7 @@
 //     running lower bound of the list's k-th best score is appended to the list's
 //     candidate array.
 #include "ss_internal.cuh"
+#include "ss_device.cuh"
 
 namespace ss {
 
@@ -32,10 +33,6 @@ int sample_units(int k, int tokens_per_unit, int hist_units) {
   (void)tokens_per_unit;
   return hist_units < kSampleUnits ? hist_units : kSampleUnits;
 }
-
-__device__ __forceinline__ void mma_16816(float (&d)[4], uint32_t a0, uint32_t a1,
-                                          uint32_t a2, uint32_t a3, uint32_t b0,
-                                          uint32_t b1);
 
 __global__ void __launch_bounds__(256) k_sample(const __grid_constant__ Batch B) {
   __shared__ __align__(16) __nv_bfloat16 qsb[kMaxGroup][kHeadDim];
@@ -193,24 +190,6 @@ cudaError_t launch_prep(const Batch& B, cudaStream_t s) {
 // Each unit's softmax statistics (max, sum 2^(s - max)) are written per list; the
 // list totals are combined later in unit order, whichever warp scored a unit.
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ void mma_16816(float (&d)[4], uint32_t a0, uint32_t a1,
-                                          uint32_t a2, uint32_t a3, uint32_t b0,
-                                          uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
-      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
-}
-
-__device__ __forceinline__ uint4 ld_stream(const void* p) {
-  uint4 r;
-  asm("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
-      : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
-      : "l"(p));
-  return r;
-}
-
 constexpr int kUnitQueue = 8;  // > units a warp's issue cursor can run ahead
 
 struct ScoreShared {
@@ -221,55 +200,6 @@ struct ScoreShared {
   unsigned long long bar[kScoreWarps][kScoreStages];  // one mbarrier per warp stage
   int uq[kScoreWarps][kUnitQueue];      // per warp: units taken, in order
 };
-
-// ---- TMA bulk copies and mbarriers (inline PTX) ----
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return (uint32_t)__cvta_generic_to_shared(p);
-}
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared.b64 p, [%1], %2;\n"
-      " selp.u32 %0, 1, 0, p;\n}\n"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-// Global -> shared bulk copy of `bytes` (multiple of 16, 16-byte aligned ends) that
-// completes the transaction count of `bar`.
-__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes,
-                                          uint32_t bar) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
-      ::"r"(dst), "l"(src), "r"(bytes), "r"(bar)
-      : "memory");
-}
-__device__ __forceinline__ void fence_proxy_async_smem() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-__device__ __forceinline__ uint64_t global_ns() {
-  uint64_t t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-// Bounded wait for a stage's bulk copy: gives up after ~1 s (or 2^26 polls).
-__device__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = global_ns();
-  for (uint32_t i = 1; i < (1u << 26); ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 1023u) == 0u && global_ns() - t0 > 1000000000ull) break;
-  }
-  return false;
-}
 
 // One column (query head) of a tile: online (max, sum 2^(s - max)) over valid rows.
 __device__ __forceinline__ void stats_update(float& m, float& l, float x0, bool v0,
