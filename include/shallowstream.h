@@ -129,9 +129,11 @@ typedef struct {
   int32_t* topk_tok;         /* [n_lists][k] candidate ids sorted by (score desc, id asc);
                                 token id p, or 0x40000000 + window * n_c + centroid for a
                                 centroid; -1 past the number of candidates */
-  float* topk_w;             /* [n_lists][k] normalised attention weight of each entry */
+  float* topk_w;             /* [n_lists][k] normalised attention weight of each entry
+                                (SS_H_MEAN: the head-averaged weight alpha) */
   float* list_stats;         /* [n_lists][2] softmax stats (M, L): M = max over candidates
-                                of the log2-scaled score s * log2(e), L = sum 2^(s' - M) */
+                                of the log2-scaled score s * log2(e), L = sum 2^(s' - M)
+                                (SS_H_MEAN: M = max alpha, L = sum alpha = 1) */
   int32_t* unit_votes;       /* [U_cap] votes of each history unit */
   float* unit_mass;          /* [U_cap] attention mass of each history unit */
   int32_t* pool;             /* [pool_mult * K] vote-ranked pool, best first */
@@ -239,7 +241,9 @@ ss_status ss_retrieve_workspace_size(const ss_index* const* indexes, int32_t n,
  * mean over query heads of the per-head weights. With use_clusters, compressed
  * windows contribute their centroids as candidates instead of their tokens (only with
  * SS_H_PER_QHEAD); a selected centroid votes once per member token and its weight is
- * shared among member units by member count.
+ * shared among member units by member count. These two modes keep every candidate's
+ * score in the workspace (P * Hq rows of N_cap floats) and rank dense rows; the
+ * default mode keeps only a running superset of each list's top k.
  * Errors: INVALID_ARG (NULL, R < 1, bad enums, workspace too small or misaligned),
  * UNSUPPORTED (k > 4096, pool > 1024, history > 16384 units, head_agg with clusters),
  * STATE (use_clusters without compression), CUDA. Device-side failures are reported

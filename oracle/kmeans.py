@@ -90,6 +90,39 @@ def compress(key_bits: np.ndarray, *, tokens_per_frame: int, first_frame: int,
             "first_frame": first_frame, "window_frames": window_frames}
 
 
+def _member_units(A, i, g, w, c, f0, WF, tokens_per_frame, tokens_per_unit):
+    """Units of the member tokens of centroid c of window w at (layer i, key head g)."""
+    m = np.nonzero(A[i, g, w] == c)[0]
+    t = (f0 + w * WF) * tokens_per_frame + m
+    return t // tokens_per_unit
+
+
+def compressed_votes(tok: np.ndarray, A: np.ndarray, *, n_q_heads: int, n_kv_heads: int,
+                     n_centroids: int, first_frame: int, window_frames: int,
+                     tokens_per_frame: int, tokens_per_unit: int,
+                     n_hist_units: int) -> np.ndarray:
+    """Unit votes of per-(layer, query head) lists that mix token ids and centroid ids:
+    a token votes for its unit, a centroid once for the unit of each member token
+    (history units only). A: assignments [P][Hkv][n_w][W * T_f]."""
+    G = n_q_heads // n_kv_heads
+    votes = np.zeros(n_hist_units, dtype=np.int64)
+    for li in range(tok.shape[0]):
+        i, g = li // n_q_heads, (li % n_q_heads) // G
+        for cand in tok[li]:
+            cand = int(cand)
+            if cand < 0:
+                continue
+            if cand < CID_BASE:
+                votes[cand // tokens_per_unit] += 1
+                continue
+            w, c = divmod(cand - CID_BASE, n_centroids)
+            for u in _member_units(A, i, g, w, c, first_frame, window_frames,
+                                   tokens_per_frame, tokens_per_unit):
+                if u < n_hist_units:
+                    votes[u] += 1
+    return votes
+
+
 def retrieve_compressed(key_bits: np.ndarray, q_bits: np.ndarray, comp: dict, *,
                         n_units: int, tokens_per_unit: int, frames_per_unit: int,
                         tokens_per_frame: int, k: int, budget: int, pool_mult: int = 4,
@@ -155,23 +188,12 @@ def retrieve_compressed(key_bits: np.ndarray, q_bits: np.ndarray, comp: dict, *,
     tw = np.take_along_axis(w_all, pos, axis=1)
 
     def member_units(i, g, w, c):
-        m = np.nonzero(A[i, g, w] == c)[0]
-        t = (f0 + w * WF) * tokens_per_frame + m
-        return t // tokens_per_unit
+        return _member_units(A, i, g, w, c, f0, WF, tokens_per_frame, tokens_per_unit)
 
-    # votes: a raw token votes for its unit, a centroid once per member token
-    votes = np.zeros(U_h, dtype=np.int64)
-    for li in range(n_lists):
-        i, g = li // Hq, (li % Hq) // G
-        for cand in tok[li]:
-            cand = int(cand)
-            if cand < CID_BASE:
-                votes[cand // tokens_per_unit] += 1
-                continue
-            w, c = divmod(cand - CID_BASE, n_c)
-            for u in member_units(i, g, w, c):
-                if u < U_h:
-                    votes[u] += 1
+    votes = compressed_votes(tok, A, n_q_heads=Hq, n_kv_heads=Hkv, n_centroids=n_c,
+                             first_frame=f0, window_frames=WF,
+                             tokens_per_frame=tokens_per_frame,
+                             tokens_per_unit=tokens_per_unit, n_hist_units=U_h)
     # mass: raw weights to their unit, centroid weights by member share
     mass = np.zeros(U_h, dtype=np.float64)
     n_raw = len(raw_tok)

@@ -98,6 +98,7 @@ int64_t cand_cap_of(const ss_index* ix) {
 // Workspace regions of one problem (offsets from the problem's base).
 struct Layout {
   size_t qeff, cand_s, cand_id, cand_cnt, gthr, ladder, samp_max, ustats, next_unit, gram;
+  size_t raw_units, raw_rank, head_ml, aval, aid;  // general path only
   size_t topk_tok, topk_w, list_ml, votes, mass, pool, sel, exp_units, frames, counts,
       status, qstage;
   size_t total;
@@ -138,6 +139,15 @@ Layout layout_of(const ss_index* ix, int R, const ss_retrieve_params* p) {
   l.counts = take(16);
   l.status = take(4);
   l.qstage = take((size_t)c.n_layers * R * c.n_q_heads * kHeadDim * 2);
+  if (p->use_clusters) {
+    l.raw_units = take(ix->ucap * 4);
+    l.raw_rank = take(ix->ucap * 4);
+  }
+  if (p->head_agg == SS_H_MEAN) {
+    l.head_ml = take(score_lists * 8);
+    l.aval = take((size_t)c.n_layers * cand_cap_of(ix) * 4);
+    l.aid = take((size_t)c.n_layers * cand_cap_of(ix) * 4);
+  }
   l.total = align256(cur);
   return l;
 }
@@ -158,10 +168,8 @@ ss_status check_params(const ss_retrieve_params* p) {
     return fail(SS_ERR_INVALID_ARG, "unknown head_agg %d", p->head_agg);
   if (p->use_clusters != 0 && p->use_clusters != 1)
     return fail(SS_ERR_INVALID_ARG, "use_clusters must be 0 or 1");
-  if (p->head_agg == SS_H_MEAN)
-    return fail(SS_ERR_UNSUPPORTED, "head_agg = SS_H_MEAN is not available in this build");
-  if (p->use_clusters)
-    return fail(SS_ERR_UNSUPPORTED, "use_clusters is not available in this build");
+  if (p->head_agg == SS_H_MEAN && p->use_clusters)
+    return fail(SS_ERR_UNSUPPORTED, "use_clusters needs per-query-head lists");
   return SS_OK;
 }
 
@@ -193,6 +201,8 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
     if (ix[j]->device != dev) return fail(SS_ERR_INVALID_ARG, "indexes on different devices");
     if (hist_units_of(ix[j], p) > kMaxHistUnits)
       return fail(SS_ERR_UNSUPPORTED, "more than %d history units", kMaxHistUnits);
+    if (p->use_clusters && ix[j]->n_windows == 0)
+      return fail(SS_ERR_STATE, "index %d has no compressed windows", j);
     const ss_result& r = res[j];
     if (!r.sel_units || !r.exp_units || !r.frames || !r.counts || !r.status)
       return fail(SS_ERR_INVALID_ARG, "result %d: sel_units, exp_units, frames, counts and status are required", j);
@@ -208,7 +218,10 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
   B.n_prev = p->n_prev;
   B.q_agg = p->q_agg;
   B.head_agg = p->head_agg;
+  B.use_clusters = p->use_clusters;
+  const bool general = p->head_agg == SS_H_MEAN || p->use_clusters;
   int max_lists = 0, max_uh = 0, max_pool = 0, n_slabs_total = 0;
+  int max_cand = 0, max_slabs = 0, max_score_lists = 0;
   char* base = static_cast<char*>(ws);
   for (int j = 0; j < n; ++j) {
     const ss_index* x = ix[j];
@@ -256,7 +269,42 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
     P.pool_n = (int)(pc < P.Uh ? pc : P.Uh);
     P.n_sample = sample_units(p->k, P.Tu, P.Uh);
     P.n_sel = P.pool_n < p->budget_units ? P.pool_n : p->budget_units;
-    max_lists = max(max_lists, P.P * P.Hq);
+    if (general) {
+      // candidates: raw tokens of the history units no window covers, then the
+      // centroids of the windows that start in the history (a prefix of the windows)
+      int64_t covered = 0, n_live = 0;
+      if (p->use_clusters) {
+        const int fpu = c.frames_per_unit;
+        const int64_t wu = x->win_frames / fpu;
+        for (int64_t f : x->win_first_frame) {
+          const int64_t u0 = f / fpu;
+          if (u0 >= P.Uh) break;
+          ++n_live;
+          covered += (u0 + wu < P.Uh ? u0 + wu : P.Uh) - u0;
+        }
+        P.n_c = x->n_centroids;
+        P.wu = (int)wu;
+        P.wcap = x->wcap;
+        P.cent = x->cent;
+        P.mcnt = x->mcnt;
+        P.msize = x->msize;
+        P.win_slot = x->win_slot;
+        P.win_u0 = x->win_u0;
+        P.raw_units = reinterpret_cast<int32_t*>(base + l.raw_units);
+        P.raw_rank = reinterpret_cast<int32_t*>(base + l.raw_rank);
+      }
+      P.n_raw_tok = (int)((P.Uh - covered) * P.Tu);
+      P.n_cand = (int)(P.n_raw_tok + n_live * P.n_c);
+      if (p->head_agg == SS_H_MEAN) {
+        P.head_ml = reinterpret_cast<float2*>(base + l.head_ml);
+        P.aval = reinterpret_cast<float*>(base + l.aval);
+        P.aid = reinterpret_cast<int32_t*>(base + l.aid);
+      }
+      max_cand = max(max_cand, P.n_cand);
+      max_slabs = max(max_slabs, P.P * P.Hkv);
+      max_score_lists = max(max_score_lists, P.P * P.Hq);
+    }
+    max_lists = max(max_lists, p->head_agg == SS_H_MEAN ? P.P : P.P * P.Hq);
     max_uh = max(max_uh, P.Uh);
     max_pool = max(max_pool, P.pool_n);
     n_slabs_total += P.P * P.Hkv;
@@ -278,10 +326,19 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
   SS_CUDA(cudaSetDevice(dev));
   SS_CUDA(launch_prep(B, st));
   if (tr && tr->score_begin) SS_CUDA(cudaEventRecord((cudaEvent_t)tr->score_begin, st));
-  SS_CUDA(launch_score(B, st));
+  if (general) {
+    SS_CUDA(launch_general_score(B, max_cand, max_slabs, max_score_lists, st));
+  } else {
+    SS_CUDA(launch_score(B, st));
+  }
   if (tr && tr->score_end) SS_CUDA(cudaEventRecord((cudaEvent_t)tr->score_end, st));
-  SS_CUDA(launch_select(B, max_lists, st));
-  SS_CUDA(launch_mass(B, max_uh, st));
+  if (general) {
+    SS_CUDA(launch_select_general(B, max_lists, st));
+    SS_CUDA(launch_mass_general(B, max_uh, st));
+  } else {
+    SS_CUDA(launch_select(B, max_lists, st));
+    SS_CUDA(launch_mass(B, max_uh, st));
+  }
   SS_CUDA(launch_pool(B, max_uh, st));
   SS_CUDA(launch_maxmin(B, max_pool, st));
   return SS_OK;

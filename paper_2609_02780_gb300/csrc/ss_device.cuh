@@ -76,4 +76,98 @@ static __device__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity) {
   return false;
 }
 
+// ---- fixed-order block reductions (deterministic) ----
+// Block reduction of (max, sum 2^(s - max)) pairs in a fixed order; result to all.
+static __device__ void block_ml(float& m, float& l, float* sm, float* sl) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nw = blockDim.x >> 5;
+  for (int off = 16; off > 0; off >>= 1) {
+    const float mo = __shfl_down_sync(0xffffffffu, m, off);
+    const float lo = __shfl_down_sync(0xffffffffu, l, off);
+    ml_combine(m, l, mo, lo);
+  }
+  if (lane == 0) {
+    sm[warp] = m;
+    sl[warp] = l;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    m = lane < nw ? sm[lane] : -INFINITY;
+    l = lane < nw ? sl[lane] : 0.f;
+    for (int off = 16; off > 0; off >>= 1) {
+      const float mo = __shfl_down_sync(0xffffffffu, m, off);
+      const float lo = __shfl_down_sync(0xffffffffu, l, off);
+      ml_combine(m, l, mo, lo);
+    }
+    if (lane == 0) {
+      sm[0] = m;
+      sl[0] = l;
+    }
+  }
+  __syncthreads();
+  m = sm[0];
+  l = sl[0];
+  __syncthreads();
+}
+
+// Fixed-order block sum; result to all threads.
+static __device__ float block_sum(float v, float* sm) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nw = blockDim.x >> 5;
+  for (int off = 16; off > 0; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
+  if (lane == 0) sm[warp] = v;
+  __syncthreads();
+  if (warp == 0) {
+    v = lane < nw ? sm[lane] : 0.f;
+    for (int off = 16; off > 0; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
+    if (lane == 0) sm[0] = v;
+  }
+  __syncthreads();
+  v = sm[0];
+  __syncthreads();
+  return v;
+}
+
+static __device__ float block_min(float v, float* sm) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nw = blockDim.x >> 5;
+  for (int off = 16; off > 0; off >>= 1) v = fminf(v, __shfl_down_sync(0xffffffffu, v, off));
+  if (lane == 0) sm[warp] = v;
+  __syncthreads();
+  if (warp == 0) {
+    v = lane < nw ? sm[lane] : INFINITY;
+    for (int off = 16; off > 0; off >>= 1) v = fminf(v, __shfl_down_sync(0xffffffffu, v, off));
+    if (lane == 0) sm[0] = v;
+  }
+  __syncthreads();
+  v = sm[0];
+  __syncthreads();
+  return v;
+}
+
+
+// Exclusive prefix sum over the block (thread order); all threads get their prefix.
+static __device__ int block_excl_scan(int v, int* sw) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nw = blockDim.x >> 5;
+  int x = v;
+  for (int off = 1; off < 32; off <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, off);
+    if (lane >= off) x += y;
+  }
+  if (lane == 31) sw[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int w = lane < nw ? sw[lane] : 0;
+    for (int off = 1; off < 32; off <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, w, off);
+      if (lane >= off) w += y;
+    }
+    sw[lane] = w;
+  }
+  __syncthreads();
+  const int prefix = warp > 0 ? sw[warp - 1] : 0;
+  return prefix + x - v;
+}
+
 }  // namespace ss

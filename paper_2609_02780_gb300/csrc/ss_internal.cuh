@@ -97,6 +97,21 @@ struct Prob {
   int32_t* frames;
   int32_t* counts;             // n_pool, n_sel, n_exp, n_frames
   uint32_t* status;
+  // general path (one list per layer, or centroids of compressed windows as candidates):
+  // every candidate is scored into a dense row per list
+  int n_cand;                  // candidates per list
+  int n_raw_tok;               // of which raw history tokens (the rest are centroids)
+  int n_c, wu, wcap;           // centroids per window, units per window, window capacity
+  const __nv_bfloat16* cent;   // [P*Hkv][wcap*n_c][d]
+  const int32_t* mcnt;         // [P*Hkv][wcap][n_c][wu]
+  const int32_t* msize;        // [P*Hkv][wcap][n_c]
+  const int32_t* win_slot;     // [ucap / wu] window of each window slot or -1
+  const int32_t* win_u0;       // [wcap] first unit of each window
+  int32_t* raw_units;          // [ucap] history units not covered by a window, ascending
+  int32_t* raw_rank;           // [ucap] position of a unit in raw_units, or -1
+  float2* head_ml;             // [P*Hq] (M, L) of each head's softmax (one list per layer)
+  float* aval;                 // [P][cand_cap] head-averaged weight of every token
+  int32_t* aid;                // [P][cand_cap]
   // launch mapping of the score kernel
   int cta_begin;               // first score CTA of this problem
   int chunks;                  // score CTAs per slab (they share the slab's units)
@@ -111,6 +126,7 @@ struct Batch {
   int n_prev;
   int q_agg;
   int head_agg;
+  int use_clusters;
   int score_ctas;              // total CTAs of the score kernel
 };
 static_assert(sizeof(Batch) <= 32000, "kernel parameter block too large");
@@ -189,6 +205,10 @@ cudaError_t launch_prep(const Batch& B, cudaStream_t s);
 int sample_units(int k, int tokens_per_unit, int hist_units);
 cudaError_t launch_score(const Batch& B, cudaStream_t s);
 cudaError_t launch_select(const Batch& B, int max_lists, cudaStream_t s);
+cudaError_t launch_select_general(const Batch& B, int max_lists, cudaStream_t s);
+cudaError_t launch_general_score(const Batch& B, int max_cand, int max_slabs,
+                                 int max_score_lists, cudaStream_t s);
+cudaError_t launch_mass_general(const Batch& B, int max_hist_units, cudaStream_t s);
 cudaError_t launch_mass(const Batch& B, int max_hist_units, cudaStream_t s);
 
 cudaError_t launch_pool(const Batch& B, int max_hist_units, cudaStream_t s);

@@ -10,6 +10,7 @@
 // No floating-point atomics: every float reduction has a fixed order, so results are
 // bit-identical from run to run.
 #include "ss_internal.cuh"
+#include "ss_device.cuh"
 
 namespace ss {
 
@@ -113,56 +114,6 @@ __device__ __forceinline__ int next_pow2(int x) {
   return p;
 }
 
-// Block reduction of (max, sum 2^(s - max)) pairs in a fixed order; result to all.
-__device__ void block_ml(float& m, float& l, float* sm, float* sl) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int nw = blockDim.x >> 5;
-  for (int off = 16; off > 0; off >>= 1) {
-    const float mo = __shfl_down_sync(0xffffffffu, m, off);
-    const float lo = __shfl_down_sync(0xffffffffu, l, off);
-    ml_combine(m, l, mo, lo);
-  }
-  if (lane == 0) {
-    sm[warp] = m;
-    sl[warp] = l;
-  }
-  __syncthreads();
-  if (warp == 0) {
-    m = lane < nw ? sm[lane] : -INFINITY;
-    l = lane < nw ? sl[lane] : 0.f;
-    for (int off = 16; off > 0; off >>= 1) {
-      const float mo = __shfl_down_sync(0xffffffffu, m, off);
-      const float lo = __shfl_down_sync(0xffffffffu, l, off);
-      ml_combine(m, l, mo, lo);
-    }
-    if (lane == 0) {
-      sm[0] = m;
-      sl[0] = l;
-    }
-  }
-  __syncthreads();
-  m = sm[0];
-  l = sl[0];
-  __syncthreads();
-}
-
-__device__ float block_min(float v, float* sm) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int nw = blockDim.x >> 5;
-  for (int off = 16; off > 0; off >>= 1) v = fminf(v, __shfl_down_sync(0xffffffffu, v, off));
-  if (lane == 0) sm[warp] = v;
-  __syncthreads();
-  if (warp == 0) {
-    v = lane < nw ? sm[lane] : INFINITY;
-    for (int off = 16; off > 0; off >>= 1) v = fminf(v, __shfl_down_sync(0xffffffffu, v, off));
-    if (lane == 0) sm[0] = v;
-  }
-  __syncthreads();
-  v = sm[0];
-  __syncthreads();
-  return v;
-}
-
 // ---------------------------------------------------------------------------
 // Exact top-k of one list (Eq. 11). The candidate array holds every token whose score
 // reached a lower bound `lo` of the list's k-th best score. A 2048-bin histogram of
@@ -171,7 +122,11 @@ __device__ float block_min(float v, float* sm) {
 // If they do not fit (massive ties), an 8-pass radix select on the 64-bit keys over
 // the candidate array finds the n-th key exactly.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ Batch B) {
+// kGeneral: the general path (one list per layer, or centroid candidates). Its lists
+// hold every candidate (a dense row), its softmax statistics come from that row, and
+// with one list per layer the row holds the head-averaged weights themselves.
+template <bool kGeneral>
+__global__ void __launch_bounds__(kSelThreads) k_select_t(const __grid_constant__ Batch B) {
   extern __shared__ unsigned long long skeys[];
   __shared__ int s_hist[kFineBins];
   __shared__ float s_m[32], s_l[32];
@@ -183,44 +138,68 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
   const int pi = blockIdx.y;
   if (pi >= B.n) return;
   const Prob& P = B.p[pi];
-  const int n_lists = P.P * P.Hq;
+  const bool mean = kGeneral && B.head_agg == 1;  // one list per layer
+  const int n_lists = mean ? P.P : P.P * P.Hq;
   const int L = blockIdx.x;
   if (L >= n_lists) return;
   const int tid = threadIdx.x, lane = tid & 31;
   const int k = B.k;
 
-  // softmax statistics from the per-unit pairs in a fixed order (thread t takes units
-  // t, t + 1024, ...; then a fixed tree), whichever warps scored the units
   float M = -INFINITY, Ls = 0.f;
-  {
+  if constexpr (!kGeneral) {
+    // softmax statistics from the per-unit pairs in a fixed order (thread t takes units
+    // t, t + 1024, ...; then a fixed tree), whichever warps scored the units
     const float2* us = P.ustats + (int64_t)L * P.ucap;
     for (int u = tid; u < P.Uh; u += blockDim.x) {
       const float2 v = us[u];
       ml_combine(M, Ls, v.x, v.y);
     }
     block_ml(M, Ls, s_m, s_l);
+    if (tid == 0) P.list_ml[L] = make_float2(M, Ls);
   }
-  if (tid == 0) P.list_ml[L] = make_float2(M, Ls);
 
   int32_t* tok_out = P.topk_tok + (int64_t)L * k;
   float* w_out = P.topk_w + (int64_t)L * k;
-  const int64_t n_tok = (int64_t)P.Uh * P.Tu;
+  const int64_t n_tok = kGeneral ? (int64_t)P.n_cand : (int64_t)P.Uh * P.Tu;
   int n = (int)min((int64_t)k, n_tok);
   if (n == 0) {
+    if (kGeneral && tid == 0) P.list_ml[L] = make_float2(-INFINITY, 0.f);
     for (int r = tid; r < k; r += blockDim.x) {
       tok_out[r] = -1;
       w_out[r] = 0.f;
     }
     return;
   }
-  const int cnt = P.cand_cnt[L];
-  const float* cs = P.cand_s + (int64_t)L * P.cand_cap;
-  const int32_t* ci = P.cand_id + (int64_t)L * P.cand_cap;
-  float lo = ordered_to_float(P.gthr[L]);
+  const int cnt = kGeneral ? P.n_cand : P.cand_cnt[L];
+  const float* cs = (mean ? P.aval : P.cand_s) + (int64_t)L * P.cand_cap;
+  const int32_t* ci = (mean ? P.aid : P.cand_id) + (int64_t)L * P.cand_cap;
+  float lo = -INFINITY;
+  if constexpr (kGeneral) {
+    // statistics of the dense row in a fixed order: (max, sum 2^(s - max)) of the
+    // scores, or (max, sum) of the head-averaged weights
+    float m = -INFINITY, l = 0.f;
+    if (mean) {
+      for (int x = tid; x < cnt; x += blockDim.x) {
+        const float v = cs[x];
+        m = fmaxf(m, v);
+        l += v;
+      }
+      l = block_sum(l, s_l);
+      m = -block_min(-m, s_m);
+    } else {
+      for (int x = tid; x < cnt; x += blockDim.x) ml_combine(m, l, cs[x], 1.f);
+      block_ml(m, l, s_m, s_l);
+    }
+    M = m;
+    Ls = l;
+    if (tid == 0) P.list_ml[L] = make_float2(M, Ls);
+  } else {
+    lo = ordered_to_float(P.gthr[L]);
+  }
   // A tighter bound from the list's completed ladder of appended-score counts: if the
   // levels >= i hold n tokens, the n-th best score is at least level i's lower edge
   // (one level of margin for the rounding of the level computation).
-  if (tid < 32) {
+  if (!kGeneral && tid < 32) {
     constexpr int per = kLadderLevels / 32;
     const int* lad = P.ladder + (int64_t)L * kLadderLevels;
     int cntl[per];
@@ -252,9 +231,11 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
       }
     }
   }
-  __syncthreads();
-  lo = fmaxf(lo, s_m[0]);
-  __syncthreads();
+  if constexpr (!kGeneral) {
+    __syncthreads();
+    lo = fmaxf(lo, s_m[0]);
+    __syncthreads();
+  }
   if (lo == -INFINITY) {
     // no bound: start from the smallest real candidate (unused reserved slots hold
     // -inf and are never candidates)
@@ -420,9 +401,21 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
       const float s = ordered_to_float((uint32_t)(key >> 32));
       const int32_t id = (int32_t)(~(uint32_t)key);
       tok_out[r] = id;
-      w_out[r] = fast_exp2(s - M) * inv_l;
+      w_out[r] = mean ? s : fast_exp2(s - M) * inv_l;
       // one vote for the token's unit (integer atomics: exact)
-      if (id >= 0 && id / P.Tu < P.Uh) atomicAdd(&P.votes[id / P.Tu], 1);
+      if (id >= 0 && (uint32_t)id < kCentroidIdBase) {
+        if (id / P.Tu < P.Uh) atomicAdd(&P.votes[id / P.Tu], 1);
+      } else if (kGeneral && id >= 0) {
+        // a centroid: one vote per member token, to the member's unit
+        const int e = id - (int)kCentroidIdBase, w = e / P.n_c, c = e - w * P.n_c;
+        const int slab = (L / P.Hq) * P.Hkv + (L % P.Hq) / P.G;
+        const int32_t* mc = P.mcnt + (((int64_t)slab * P.wcap + w) * P.n_c + c) * P.wu;
+        const int u0 = P.win_u0[w];
+        for (int x = 0; x < P.wu; ++x) {
+          const int m = mc[x];
+          if (m && u0 + x < P.Uh) atomicAdd(&P.votes[u0 + x], m);
+        }
+      }
     } else {
       tok_out[r] = -1;
       w_out[r] = 0.f;
@@ -433,9 +426,18 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
 
 cudaError_t launch_select(const Batch& B, int max_lists, cudaStream_t s) {
   const int smem = kSelCap * (int)sizeof(unsigned long long);
-  cudaError_t e = cudaFuncSetAttribute(k_select, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaError_t e = cudaFuncSetAttribute(k_select_t<false>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  return launch_pdl(k_select, dim3(max_lists, B.n), dim3(kSelThreads), (size_t)smem, s, B);
+  return launch_pdl(k_select_t<false>, dim3(max_lists, B.n), dim3(kSelThreads), (size_t)smem, s, B);
+}
+
+cudaError_t launch_select_general(const Batch& B, int max_lists, cudaStream_t s) {
+  const int smem = kSelCap * (int)sizeof(unsigned long long);
+  cudaError_t e = cudaFuncSetAttribute(k_select_t<true>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  return launch_pdl(k_select_t<true>, dim3(max_lists, B.n), dim3(kSelThreads), (size_t)smem, s, B);
 }
 
 // ---------------------------------------------------------------------------
@@ -484,29 +486,6 @@ cudaError_t launch_mass(const Batch& B, int max_hist_units, cudaStream_t s) {
 // Vote-ranked pool: all history units sorted in shared memory by
 // (votes desc, mass desc, id asc); the first pool_n are the pool.
 // ---------------------------------------------------------------------------
-__device__ int block_excl_scan(int v, int* sw) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int nw = blockDim.x >> 5;
-  int x = v;
-  for (int off = 1; off < 32; off <<= 1) {
-    const int y = __shfl_up_sync(0xffffffffu, x, off);
-    if (lane >= off) x += y;
-  }
-  if (lane == 31) sw[warp] = x;
-  __syncthreads();
-  if (warp == 0) {
-    int w = lane < nw ? sw[lane] : 0;
-    for (int off = 1; off < 32; off <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, w, off);
-      if (lane >= off) w += y;
-    }
-    sw[lane] = w;
-  }
-  __syncthreads();
-  const int prefix = warp > 0 ? sw[warp - 1] : 0;
-  return prefix + x - v;
-}
-
 __device__ __forceinline__ bool unit_before(unsigned long long ka, int ia,
                                             unsigned long long kb, int ib) {
   return ka > kb || (ka == kb && ia < ib);

@@ -32,26 +32,37 @@ LOG2E = 1.0 / math.log(2.0)
 
 
 def check_topk(s: np.ndarray, tok: np.ndarray, w_gpu: np.ndarray, w_ref: np.ndarray,
-               k: int, lists=None) -> dict:
-    """s, w_ref: oracle scores / weights [lists][n_tok]; tok, w_gpu: GPU [lists][k]."""
+               k: int, lists=None, ids: np.ndarray | None = None, rel_tol: float = 0.0) -> dict:
+    """s, w_ref: oracle scores / weights [lists][n_cand]; tok, w_gpu: GPU [lists][k].
+
+    ids: the candidate id of each oracle column (default: the column index, i.e. token
+    ids). rel_tol > 0 ranks by values whose rounding is relative (head-averaged
+    weights): the band is then rel_tol * theta instead of TOL_SCORE."""
     n_tok = s.shape[1]
     n = min(k, n_tok)
     lists = range(s.shape[0]) if lists is None else lists
+    pos_of = None if ids is None else {int(v): j for j, v in enumerate(ids)}
     ambiguous = 0
     for li in lists:
         row_tok = tok[li]
         assert (row_tok[n:] == -1).all(), f"list {li}: entries past n must be -1"
-        got = row_tok[:n].astype(np.int64)
-        assert (got >= 0).all() and (got < n_tok).all(), f"list {li}: token id out of range"
+        if pos_of is None:
+            got = row_tok[:n].astype(np.int64)
+            assert (got >= 0).all() and (got < n_tok).all(), f"list {li}: token id out of range"
+        else:
+            assert all(int(v) in pos_of for v in row_tok[:n]), f"list {li}: unknown candidate id"
+            got = np.array([pos_of[int(v)] for v in row_tok[:n]], dtype=np.int64)
         assert len(set(got.tolist())) == n, f"list {li}: duplicate tokens"
         srow = s[li]
         theta = np.partition(srow, n_tok - n)[n_tok - n]
-        must = np.nonzero(srow > theta + TOL_SCORE)[0]
+        tol = rel_tol * abs(theta) if rel_tol > 0 else TOL_SCORE
+        must = np.nonzero(srow > theta + tol)[0]
         assert np.isin(must, got).all(), f"list {li}: missed a token above the band"
-        assert (srow[got] >= theta - TOL_SCORE).all(), f"list {li}: token below the band"
+        assert (srow[got] >= theta - tol).all(), f"list {li}: token below the band"
         # GPU order is (score desc, id asc) up to the score tolerance
         sg = srow[got]
-        assert (np.diff(sg) <= TOL_SCORE).all(), f"list {li}: order disagrees with scores"
+        otol = rel_tol * np.abs(sg[1:]) if rel_tol > 0 else TOL_SCORE
+        assert (np.diff(sg) <= otol).all(), f"list {li}: order disagrees with scores"
         wg = w_gpu[li, :n].astype(np.float64)
         assert np.abs(wg - w_ref[li, got]).max() <= TOL_W, f"list {li}: weight off"
         ref_set = set(np.lexsort((np.arange(n_tok), -srow))[:n].tolist())
@@ -73,12 +84,15 @@ def check_stats(s: np.ndarray, list_stats: np.ndarray, lists=None) -> None:
 
 
 def check_chain(gpu: dict, desc: np.ndarray, n_hist_units: int, tokens_per_unit: int,
-                budget: int, pool_mult: int, n_prev: int, frames_per_unit: int) -> dict:
+                budget: int, pool_mult: int, n_prev: int, frames_per_unit: int,
+                votes: np.ndarray | None = None) -> dict:
     """Votes, pool, max-min and expansion recomputed by the oracle from the GPU's own
-    upstream outputs."""
+    upstream outputs (votes: the oracle's votes from the GPU's lists, when they are not
+    plain token votes)."""
     tok = gpu["topk_tok"]
-    votes = R.unit_votes(tok[tok >= 0].reshape(1, -1) if (tok < 0).any() else tok,
-                         n_hist_units, tokens_per_unit)
+    if votes is None:
+        votes = R.unit_votes(tok[tok >= 0].reshape(1, -1) if (tok < 0).any() else tok,
+                             n_hist_units, tokens_per_unit)
     assert np.array_equal(votes, gpu["votes"]), "votes differ"
     pool = R.vote_pool(gpu["votes"], gpu["mass"].astype(np.float64), pool_mult * budget)
     assert np.array_equal(pool, gpu["pool"]), "pool differs"

@@ -1,0 +1,167 @@
+"""Parity of the general retrieval path (through the C ABI) with the CPU oracle:
+one list per layer (head-averaged weights) and retrieval over compressed windows."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import kmeans as KM
+from oracle import retrieval as R
+from tests import parity as PY
+
+pytestmark = pytest.mark.gpu
+
+# Head-averaged weights carry the relative rounding of the per-head weights they
+# average: |dw / w| <= |ds| (natural-log units) + fp32 rounding, with |ds| <= TOL_SCORE.
+REL_ALPHA = 1e-3
+
+
+def _ss():
+    import paper_2609_02780_gb300 as ss
+    return ss
+
+
+def _bits(t: torch.Tensor) -> np.ndarray:
+    return t.detach().contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
+
+
+def _keys_q(seed, P, Hq, Hkv, F, Tf, R_rows=4, scene=0):
+    g = torch.Generator().manual_seed(seed)
+    keys = torch.randn(P, Hkv, F * Tf, 128, generator=g)
+    if scene:
+        means = 0.7 * torch.randn(P, Hkv, F // scene + 1, 1, 128, generator=g)
+        keys += means.repeat_interleave(scene * Tf, 2)[:, :, :F * Tf, 0]
+    q = torch.randn(P, R_rows, Hq, 128, generator=g)
+    return keys.to(torch.bfloat16), q.to(torch.bfloat16)
+
+
+def _mean_case(keys, q, *, Tf, fpu, k, budget, n_recent, q_agg=0):
+    ss = _ss()
+    P, Hkv, N, _ = keys.shape
+    Hq = q.shape[2]
+    F = N // Tf
+    idx = ss.Index(P, Hq, Hkv, Tf, F, frames_per_unit=fpu, device="cuda")
+    idx.append(keys.cuda())
+    res = idx.retrieve(q.cuda(), k=k, budget=budget, n_recent=n_recent, q_agg=q_agg,
+                       head_agg=ss.H_MEAN)
+    res.check()
+    Tu, U = Tf * fpu, F // fpu
+    Uh = max(0, U - n_recent)
+    gpu = PY.gpu_outputs(res, Uh)
+    kb, qb = _bits(keys), _bits(q)
+    desc = R.descriptors(kb, U, Tu)
+    ref = R.retrieve(kb, qb, n_units=U, tokens_per_unit=Tu, k=k, budget=budget,
+                     frames_per_unit=fpu, n_recent=n_recent, q_agg=q_agg,
+                     head_agg=R.H_MEAN, desc=desc)
+    assert gpu["topk_tok"].shape[0] == P
+    info = PY.check_topk(ref["alpha"], gpu["topk_tok"], gpu["topk_w"], ref["alpha"], k,
+                         rel_tol=REL_ALPHA)
+    # list statistics of a layer list: (max alpha, sum alpha = 1)
+    st = gpu["list_stats"]
+    assert np.allclose(st[:, 0], ref["alpha"].max(1), rtol=REL_ALPHA)
+    assert np.allclose(st[:, 1], 1.0, atol=1e-4)
+    assert np.allclose(gpu["mass"], ref["mass"], rtol=1e-3, atol=1e-7)
+    info.update(PY.check_chain(gpu, desc, Uh, Tu, budget, 4, 1, fpu))
+    assert gpu["votes"].sum() == P * min(k, Uh * Tu)
+    if info["ambiguous_lists"] == 0 and info["close_maxmin_steps"] == 0:
+        assert gpu["sel"].tolist() == ref["sel"].tolist()
+        assert gpu["frames"].tolist() == ref["frames"].tolist()
+    return gpu, ref, info
+
+
+def test_head_averaged_lists_paper_configuration():
+    # Table 4's setting: 2-frame units, k = 64 per layer, pool 32, K = 8, 6 recent units
+    from paper_2609_02780_gb300 import synth
+    w = synth.PRESETS["paper_qwen"]
+    data = synth.make_workload(w, device="cpu")
+    _mean_case(data["keys"], data["q"], Tf=w.tokens_per_frame, fpu=w.frames_per_unit,
+               k=w.k, budget=w.budget, n_recent=w.n_recent)
+
+
+def test_head_averaged_lists_ragged_and_mean_logit_rows():
+    keys, q = _keys_q(31, P=2, Hq=8, Hkv=2, F=70, Tf=23, R_rows=5)
+    _mean_case(keys, q, Tf=23, fpu=1, k=200, budget=5, n_recent=3, q_agg=1)
+
+
+def test_head_averaged_lists_more_tokens_than_the_sort_buffer():
+    # 40,000 candidates per list: the top-k goes through the histogram fallback
+    keys, q = _keys_q(32, P=1, Hq=4, Hkv=1, F=200, Tf=200, R_rows=2)
+    _mean_case(keys, q, Tf=200, fpu=1, k=300, budget=6, n_recent=0)
+
+
+def _cluster_case(keys, q, *, Tf, fpu, WF, n_c, comp_frames, k, budget, n_recent,
+                  iters=3):
+    ss = _ss()
+    P, Hkv, N, _ = keys.shape
+    Hq = q.shape[2]
+    F = N // Tf
+    idx = ss.Index(P, Hq, Hkv, Tf, F, frames_per_unit=fpu, device="cuda")
+    idx.append(keys.cuda())
+    idx.compress(WF, n_centroids=n_c, iters=iters, first_frame=0, n_frames=comp_frames)
+    res = idx.retrieve(q.cuda(), k=k, budget=budget, n_recent=n_recent, use_clusters=1)
+    res.check()
+    cl = idx.clusters()
+    Tu, U = Tf * fpu, F // fpu
+    Uh = max(0, U - n_recent)
+    gpu = PY.gpu_outputs(res, Uh)
+    kb, qb = _bits(keys), _bits(q)
+    desc = R.descriptors(kb, U, Tu)
+    n_w = comp_frames // WF
+    cbits = _bits(cl["centroids"])                           # the GPU's own clusters
+    A = cl["assignment"].cpu().numpy()[:, :, :n_w * WF * Tf].reshape(P, Hkv, n_w, WF * Tf)
+    comp = {"centroid_bits": cbits, "assign": A.astype(np.int64), "first_frame": 0,
+            "window_frames": WF}
+    ref = KM.retrieve_compressed(kb, qb, comp, n_units=U, tokens_per_unit=Tu,
+                                 frames_per_unit=fpu, tokens_per_frame=Tf, k=k,
+                                 budget=budget, n_recent=n_recent, desc=desc)
+    info = PY.check_topk(ref["s"], gpu["topk_tok"], gpu["topk_w"], ref["w"], k,
+                         ids=ref["ids"])
+    PY.check_stats(ref["s"], gpu["list_stats"])
+    assert np.allclose(gpu["mass"], ref["mass"], rtol=1e-3, atol=1e-7)
+    votes = KM.compressed_votes(gpu["topk_tok"], A, n_q_heads=Hq, n_kv_heads=Hkv,
+                                n_centroids=n_c, first_frame=0, window_frames=WF,
+                                tokens_per_frame=Tf, tokens_per_unit=Tu, n_hist_units=Uh)
+    info.update(PY.check_chain(gpu, desc, Uh, Tu, budget, 4, 1, fpu, votes=votes))
+    # a selected centroid votes once per member token
+    sizes = cl["member_sizes"].cpu().numpy()
+    expect = 0
+    for li in range(P * Hq):
+        i, g = li // Hq, (li % Hq) // (Hq // Hkv)
+        for v in gpu["topk_tok"][li]:
+            if v >= KM.CID_BASE:
+                w, c = divmod(int(v) - KM.CID_BASE, n_c)
+                expect += int(sizes[i, g, w, c])
+            elif v >= 0:
+                expect += 1
+    assert gpu["votes"].sum() <= expect          # members past the history do not vote
+    if info["ambiguous_lists"] == 0 and info["close_maxmin_steps"] == 0:
+        assert gpu["sel"].tolist() == ref["sel"].tolist()
+        assert gpu["frames"].tolist() == ref["frames"].tolist()
+    return gpu, ref, info
+
+
+def test_compressed_windows_and_raw_tail():
+    # 12 of 20 windows compressed; the raw tail and the recent units stay tokens
+    keys, q = _keys_q(33, P=2, Hq=8, Hkv=2, F=80, Tf=30, scene=8)
+    gpu, ref, _ = _cluster_case(keys, q, Tf=30, fpu=1, WF=4, n_c=16, comp_frames=48,
+                                k=120, budget=6, n_recent=5)
+    assert (gpu["topk_tok"] >= KM.CID_BASE).any() and (
+        (gpu["topk_tok"] >= 0) & (gpu["topk_tok"] < KM.CID_BASE)).any()
+
+
+def test_all_history_compressed_two_frame_units_window_past_history():
+    # every window compressed; with 3 recent units the last window straddles the history
+    keys, q = _keys_q(34, P=1, Hq=4, Hkv=1, F=48, Tf=20, scene=6)
+    _cluster_case(keys, q, Tf=20, fpu=2, WF=4, n_c=10, comp_frames=48, k=40, budget=4,
+                  n_recent=3)
+
+
+def test_general_path_errors():
+    ss = _ss()
+    keys, q = _keys_q(35, P=1, Hq=4, Hkv=1, F=8, Tf=10)
+    idx = ss.Index(1, 4, 1, 10, 8, device="cuda")
+    idx.append(keys.cuda())
+    with pytest.raises(ss.ShallowStreamError, match="STATE"):
+        idx.retrieve(q.cuda(), k=5, budget=2, use_clusters=1)
+    idx.compress(4, n_centroids=8, iters=2)
+    with pytest.raises(ss.ShallowStreamError, match="UNSUPPORTED"):
+        idx.retrieve(q.cuda(), k=5, budget=2, use_clusters=1, head_agg=ss.H_MEAN)
