@@ -187,26 +187,40 @@ def retrieve_compressed(key_bits: np.ndarray, q_bits: np.ndarray, comp: dict, *,
     tok = ids[pos]
     tw = np.take_along_axis(w_all, pos, axis=1)
 
-    def member_units(i, g, w, c):
-        return _member_units(A, i, g, w, c, f0, WF, tokens_per_frame, tokens_per_unit)
-
     votes = compressed_votes(tok, A, n_q_heads=Hq, n_kv_heads=Hkv, n_centroids=n_c,
                              first_frame=f0, window_frames=WF,
                              tokens_per_frame=tokens_per_frame,
                              tokens_per_unit=tokens_per_unit, n_hist_units=U_h)
     # mass: raw weights to their unit, centroid weights by member share
+    # (per window and key head: share[c][x] = members of c in the window's unit x / |c|,
+    # so a list's centroid weights spread over units as w_c @ share)
     mass = np.zeros(U_h, dtype=np.float64)
     n_raw = len(raw_tok)
+    raw_unit = raw_tok // tokens_per_unit
+    Wt = WF * tokens_per_frame
+    shares: dict[tuple[int, int, int], tuple[int, np.ndarray]] = {}
+
+    def share_of(i, g, w):
+        if (i, g, w) not in shares:
+            t0 = (f0 + w * WF) * tokens_per_frame
+            u = (t0 + np.arange(Wt)) // tokens_per_unit
+            u_first = int(u[0])
+            cnt = np.zeros((n_c, int(u[-1]) - u_first + 1), dtype=np.float64)
+            np.add.at(cnt, (A[i, g, w].astype(np.int64), u - u_first), 1.0)
+            size = cnt.sum(axis=1, keepdims=True)
+            shares[(i, g, w)] = (u_first, np.divide(cnt, size, out=np.zeros_like(cnt),
+                                                    where=size > 0))
+        return shares[(i, g, w)]
+
     for li in range(n_lists):
         i, g = li // Hq, (li % Hq) // G
-        for j in range(n_raw):
-            mass[raw_tok[j] // tokens_per_unit] += w_all[li, j]
-        for j in range(n_raw, len(ids)):
-            w, c = divmod(int(ids[j]) - CID_BASE, n_c)
-            mu = member_units(i, g, w, c)
-            for u in mu:
-                if u < U_h:
-                    mass[u] += w_all[li, j] / len(mu)
+        np.add.at(mass, raw_unit, w_all[li, :n_raw])
+        for k_w, w in enumerate(live_w):
+            u_first, sh = share_of(i, g, w)
+            cols = slice(n_raw + k_w * n_c, n_raw + (k_w + 1) * n_c)
+            add = w_all[li, cols] @ sh
+            hi = min(U_h, u_first + sh.shape[1])
+            mass[u_first:hi] += add[:hi - u_first]
     pool = vote_pool(votes, mass, pool_mult * budget)
     sel = maxmin_select(pool, desc, budget)
     exp = expand_units(sel, n_prev)

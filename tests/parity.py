@@ -65,7 +65,10 @@ def check_topk(s: np.ndarray, tok: np.ndarray, w_gpu: np.ndarray, w_ref: np.ndar
         assert (np.diff(sg) <= otol).all(), f"list {li}: order disagrees with scores"
         wg = w_gpu[li, :n].astype(np.float64)
         assert np.abs(wg - w_ref[li, got]).max() <= TOL_W, f"list {li}: weight off"
-        ref_set = set(np.lexsort((np.arange(n_tok), -srow))[:n].tolist())
+        top = np.nonzero(srow >= theta)[0]            # the n best, ties at theta to low ids
+        if len(top) > n:
+            top = top[np.lexsort((top, -srow[top]))[:n]]
+        ref_set = set(top.tolist())
         if ref_set != set(got.tolist()):
             ambiguous += 1
     return {"ambiguous_lists": ambiguous}
