@@ -1,0 +1,211 @@
+"""Parity at the full sizes of the benchmark workloads, through the calls bench.py times.
+
+The oracle scores every (layer, query head) list in fp64, one (layer, key head) slab at
+a time, so every list is checked: the top-k band, the softmax statistics and weights,
+the attention mass of every history unit, and, chained from the GPU's own lists,
+votes and mass, the votes (exact), pool, max-min and expansion.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import kmeans as KM
+from oracle import retrieval as R
+from tests import parity as PY
+
+pytestmark = pytest.mark.gpu
+
+
+def _ss():
+    import paper_2609_02780_gb300 as ss
+    return ss
+
+
+def _preset(name):
+    from paper_2609_02780_gb300 import synth
+    return synth, synth.PRESETS[name]
+
+
+def _params(w, **over):
+    ss = _ss()
+    kw = dict(k=w.k, budget=w.budget, pool_mult=w.pool_mult, n_prev=w.n_prev,
+              n_recent=w.n_recent, q_agg=w.q_agg, head_agg=w.head_agg)
+    kw.update(over)
+    return ss.RetrieveParams(**kw)
+
+
+def _index(w, keys):
+    ss = _ss()
+    idx = ss.Index(w.n_layers, w.n_q_heads, w.n_kv_heads, w.tokens_per_frame, w.n_frames,
+                   frames_per_unit=w.frames_per_unit, device=keys.device)
+    idx.append(keys)
+    return idx
+
+
+def _retrieve(idx, q, p):
+    """One retrieval the way bench.py times it: preallocated result and workspace."""
+    ss = _ss()
+    res = ss.Result(idx, p)
+    ws = torch.empty(idx.workspace_bytes(q.shape[1], p), dtype=torch.uint8, device=q.device)
+    idx.retrieve(q, k=p.k, budget=p.budget, pool_mult=p.pool_mult, n_prev=p.n_prev,
+                 n_recent=p.n_recent, q_agg=p.q_agg, head_agg=p.head_agg,
+                 use_clusters=p.use_clusters, out=res, workspace=ws)
+    res.check()
+    return res
+
+
+def _check_problem(kb, qb, gpu, w):
+    """Every list of one problem against the oracle; returns (ambiguous lists, chain)."""
+    P, Hkv = kb.shape[0], kb.shape[1]
+    Hq = qb.shape[2]
+    G = Hq // Hkv
+    Tu = w.tokens_per_frame * w.frames_per_unit
+    U = w.n_frames // w.frames_per_unit
+    Uh = U - w.n_recent
+    n_tok = Uh * Tu
+    qe = R.query_effective(qb, w.q_agg)
+    mass = np.zeros(Uh)
+    amb = 0
+    for i in range(P):
+        for g in range(Hkv):
+            s = R.scores(qe, kb, n_tok, lists=[(i, g * G + h) for h in range(G)])
+            for h in range(G):
+                L = i * Hq + g * G + h
+                wrow = R.softmax(s[h:h + 1])
+                mass += R.unit_mass(wrow, Uh, Tu)
+                info = PY.check_topk(s[h:h + 1], gpu["topk_tok"][L:L + 1],
+                                     gpu["topk_w"][L:L + 1], wrow, w.k)
+                amb += info["ambiguous_lists"]
+                PY.check_stats(s[h:h + 1], gpu["list_stats"][L:L + 1])
+            del s
+    assert np.allclose(gpu["mass"], mass, rtol=1e-4, atol=1e-7)
+    assert gpu["votes"].sum() == P * Hq * min(w.k, n_tok)
+    desc = R.descriptors(kb, U, Tu)
+    chain = PY.check_chain(gpu, desc, Uh, Tu, w.budget, w.pool_mult, w.n_prev,
+                           w.frames_per_unit)
+    return amb, chain
+
+
+def _run_single(name):
+    synth, w = _preset(name)
+    data = synth.make_workload(w, device=torch.device("cuda"))
+    idx = _index(w, data["keys"])
+    res = _retrieve(idx, data["q"], _params(w))
+    Uh = w.n_frames // w.frames_per_unit - w.n_recent
+    gpu = PY.gpu_outputs(res, Uh)
+    kb, qb = synth.bf16_bits(data["keys"]), synth.bf16_bits(data["q"])
+    del data, idx
+    torch.cuda.empty_cache()
+    amb, chain = _check_problem(kb, qb, gpu, w)
+    # the planted frames carry the question's direction: most of them are selected
+    return gpu, amb, chain
+
+
+def test_one_hour_index_every_list():
+    gpu, amb, chain = _run_single("hour1")
+    assert amb <= 4 and chain["close_maxmin_steps"] <= 2
+
+
+def test_three_hour_index_every_list():
+    gpu, amb, chain = _run_single("hour3")
+    assert amb <= 8
+
+
+def test_sixteen_streams_batched():
+    ss = _ss()
+    synth, w = _preset("batched16")
+    idxs, qs, kbs = [], [], []
+    for st in range(w.n_streams):
+        data = synth.make_workload(w, device=torch.device("cuda"), stream=st)
+        idxs.append(_index(w, data["keys"]))
+        qs.append(data["q"])
+        if st in (0, 7, 15):
+            kbs.append((st, synth.bf16_bits(data["keys"]), synth.bf16_bits(data["q"])))
+        del data
+    p = _params(w)
+    ws = torch.empty(ss.workspace_bytes(idxs, [q.shape[1] for q in qs], p),
+                     dtype=torch.uint8, device="cuda")
+    outs = ss.retrieve_batched(idxs, qs, p, workspace=ws)
+    Uh = w.n_frames // w.frames_per_unit - w.n_recent
+    Tu = w.tokens_per_frame * w.frames_per_unit
+    gpus = [PY.gpu_outputs(o, Uh) for o in outs]
+    for o in outs:
+        o.check()
+    # every stream: exact chained votes and the vote total, mass summing to the lists
+    for gpu in gpus:
+        tok = gpu["topk_tok"]
+        assert np.array_equal(R.unit_votes(tok, Uh, Tu), gpu["votes"])
+        assert gpu["votes"].sum() == w.n_layers * w.n_q_heads * w.k
+        assert abs(gpu["mass"].sum() - w.n_layers * w.n_q_heads) <= 1e-3 * w.n_layers * w.n_q_heads
+    del idxs, outs, ws
+    torch.cuda.empty_cache()
+    for st, kb, qb in kbs:
+        amb, _ = _check_problem(kb, qb, gpus[st], w)
+        assert amb <= 4
+
+
+def test_one_hour_index_compressed():
+    """The 1-hour index compressed in 20-frame windows to 64 centroids (5 rounds), then
+    retrieval over centroids with k = 512."""
+    synth, w = _preset("hour1_kmeans")
+    data = synth.make_workload(w, device=torch.device("cuda"))
+    WF, n_c, T = w.window_frames, w.n_centroids, w.kmeans_iters
+    Wt = WF * w.tokens_per_frame
+    kb, qb = synth.bf16_bits(data["keys"]), synth.bf16_bits(data["q"])
+    # Lloyd rounds of a few (window, slab) pairs, chained round by round
+    sample = [(0, 0, 0), (1, 2, 97), (3, 3, 179)]            # (layer, key head, window)
+    rounds = []
+    for t in range(1, T + 1):
+        idx = _index(w, data["keys"])
+        idx.compress(WF, n_centroids=n_c, iters=t)
+        cl = idx.clusters()
+        rounds.append({(i, g, wi): (cl["assignment"][i, g, wi * Wt:(wi + 1) * Wt].cpu().numpy(),
+                                    synth.bf16_bits(cl["centroids"][i, g, wi]))
+                       for i, g, wi in sample})
+        if t < T:
+            del idx, cl
+            torch.cuda.empty_cache()
+    for key in sample:
+        i, g, wi = key
+        X = R.bf16_to_f64(kb[i, g, wi * Wt:(wi + 1) * Wt])
+        C = X[:n_c].copy()
+        for t in range(T):
+            a, cbits = rounds[t][key]
+            a = a.astype(np.int64)
+            D = ((X[:, None, :] - C[None]) ** 2).sum(-1)
+            tol = 1e-4 * ((X * X).sum(1) + (C * C).sum(1).max())
+            assert (D[np.arange(len(X)), a] <= D.min(1) + tol).all()
+            C = C.copy()
+            for c in range(n_c):
+                if (a == c).any():
+                    C[c] = X[a == c].mean(0)
+            assert np.all(np.abs(R.bf16_to_f64(cbits) - C) <= 2.0 ** -8 * np.abs(C) + 1e-6)
+    # retrieval over the compressed index (the last index: 5 rounds)
+    p = _params(w, use_clusters=1)
+    res = _retrieve(idx, data["q"], p)
+    Uh = w.n_frames // w.frames_per_unit - w.n_recent
+    Tu = w.tokens_per_frame * w.frames_per_unit
+    gpu = PY.gpu_outputs(res, Uh)
+    n_w = w.n_frames // WF
+    A = cl["assignment"].cpu().numpy()[:, :, :n_w * Wt].reshape(w.n_layers, w.n_kv_heads, n_w, Wt)
+    comp = {"centroid_bits": synth.bf16_bits(cl["centroids"]), "assign": A.astype(np.int64),
+            "first_frame": 0, "window_frames": WF}
+    del data, idx, cl
+    torch.cuda.empty_cache()
+    desc = R.descriptors(kb, w.n_frames // w.frames_per_unit, Tu)
+    ref = KM.retrieve_compressed(kb, qb, comp, n_units=w.n_frames // w.frames_per_unit,
+                                 tokens_per_unit=Tu, frames_per_unit=w.frames_per_unit,
+                                 tokens_per_frame=w.tokens_per_frame, k=w.k,
+                                 budget=w.budget, n_recent=w.n_recent, q_agg=w.q_agg,
+                                 desc=desc)
+    info = PY.check_topk(ref["s"], gpu["topk_tok"], gpu["topk_w"], ref["w"], w.k,
+                         ids=ref["ids"])
+    PY.check_stats(ref["s"], gpu["list_stats"])
+    assert np.allclose(gpu["mass"], ref["mass"], rtol=1e-3, atol=1e-7)
+    votes = KM.compressed_votes(gpu["topk_tok"], A, n_q_heads=w.n_q_heads,
+                                n_kv_heads=w.n_kv_heads, n_centroids=n_c, first_frame=0,
+                                window_frames=WF, tokens_per_frame=w.tokens_per_frame,
+                                tokens_per_unit=Tu, n_hist_units=Uh)
+    PY.check_chain(gpu, desc, Uh, Tu, w.budget, w.pool_mult, w.n_prev, w.frames_per_unit,
+                   votes=votes)
+    assert info["ambiguous_lists"] <= 4
