@@ -207,6 +207,29 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+# DRAM bytes of one k_score launch on the full 1-hour workload, from the 1-pass ncu
+# capture summarised in profiles/k_score_dram_traffic.md; valid only for the kernel
+# sources it was taken on (their sha256 below), reported as null otherwise.
+TRAFFIC_RECORD = {"workload": "hour1", "sources_sha256": None, "dram_bytes": None}
+SCORE_SOURCES = ("ss_score.cu", "ss_internal.cuh", "ss_device.cuh")
+
+
+def score_sources_sha256() -> str:
+    import hashlib
+    h = hashlib.sha256()
+    for f in SCORE_SOURCES:
+        with open(os.path.join(ROOT, "paper_2609_02780_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def recorded_traffic(w) -> float | None:
+    r = TRAFFIC_RECORD
+    if r["dram_bytes"] is None or w.name != r["workload"] or w.window_frames:
+        return None
+    return float(r["dram_bytes"]) if score_sources_sha256() == r["sources_sha256"] else None
+
+
 def run_ours(args):
     import numpy as np
     import torch
@@ -219,24 +242,41 @@ def run_ours(args):
     if args.frames:
         w = w.replace(n_frames=args.frames,
                       n_planted=max(1, w.n_planted * args.frames // w.n_frames))
-    data = synth.make_workload(w, device=dev, stream=rank)
-    idx = ss.Index(w.n_layers, w.n_q_heads, w.n_kv_heads, w.tokens_per_frame, w.n_frames,
-                   frames_per_unit=w.frames_per_unit, device=dev)
-    idx.append(data["keys"])
-    q = data["q"]
-    keys_cpu = None
-    if rank == 0 and not args.no_cpu_baseline:
-        frames = min(args.cpu_frames, w.n_frames)
-        keys_cpu = data["keys"][:, :, : frames * w.tokens_per_frame].cpu()
-    q_cpu = q.cpu()
-    del data
+    n_streams = w.n_streams
+    clusters = w.window_frames > 0
+    idxs, qs = [], []
+    keys_cpu = q_cpu = None
+    compress_ms = None
+    for st in range(n_streams):
+        data = synth.make_workload(w, device=dev, stream=rank * n_streams + st)
+        idx = ss.Index(w.n_layers, w.n_q_heads, w.n_kv_heads, w.tokens_per_frame, w.n_frames,
+                       frames_per_unit=w.frames_per_unit, device=dev)
+        idx.append(data["keys"])
+        if clusters:
+            c0 = torch.cuda.Event(enable_timing=True)
+            c1 = torch.cuda.Event(enable_timing=True)
+            c0.record()
+            idx.compress(w.window_frames, n_centroids=w.n_centroids, iters=w.kmeans_iters)
+            c1.record()
+            torch.cuda.synchronize(dev)
+            compress_ms = c0.elapsed_time(c1)
+        if st == 0:
+            if rank == 0 and not args.no_cpu_baseline:
+                frames = min(args.cpu_frames, w.n_frames)
+                keys_cpu = data["keys"][:, :, : frames * w.tokens_per_frame].cpu()
+            q_cpu = data["q"].cpu()
+        idxs.append(idx)
+        qs.append(data["q"])
+        del data
     torch.cuda.synchronize(dev)
     torch.cuda.empty_cache()
 
     p = ss.RetrieveParams(k=w.k, budget=w.budget, pool_mult=w.pool_mult, n_prev=w.n_prev,
-                          n_recent=w.n_recent, q_agg=w.q_agg, head_agg=w.head_agg)
-    res = ss.Result(idx, p)
-    ws = torch.empty(idx.workspace_bytes(q.shape[1], p), dtype=torch.uint8, device=dev)
+                          n_recent=w.n_recent, q_agg=w.q_agg, head_agg=w.head_agg,
+                          use_clusters=int(clusters))
+    outs = [ss.Result(ix, p) for ix in idxs]
+    ws = torch.empty(ss.workspace_bytes(idxs, [q.shape[1] for q in qs], p),
+                     dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
     k_begin = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     k_end = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
@@ -247,13 +287,12 @@ def run_ours(args):
 
     def step(i=None):
         tr = (k_begin[i], k_end[i]) if i is not None else None
-        idx.retrieve(q, k=p.k, budget=p.budget, pool_mult=p.pool_mult, n_prev=p.n_prev,
-                     n_recent=p.n_recent, q_agg=p.q_agg, head_agg=p.head_agg, out=res,
-                     workspace=ws, trace=tr)
+        ss.retrieve_batched(idxs, qs, p, outs=outs, workspace=ws, trace=tr)
 
     for _ in range(max(3, args.warmup)):
         step()
-    res.check()
+    for o in outs:
+        o.check()
     clocks = ClockSampler(local)
     barrier(world)
     torch.cuda.synchronize(dev)
@@ -269,17 +308,19 @@ def run_ours(args):
     torch.cuda.synchronize(dev)
     barrier(world)
     clk = clocks.stop()
-    res.check()
+    for o in outs:
+        o.check()
     total_ms = t_all0.elapsed_time(t_all1)
     total_ms = max_over_ranks(total_ms, world)
     step_ms = sorted(s_begin[i].elapsed_time(s_end[i]) for i in range(args.steps))
     k1_ms = [k_begin[i].elapsed_time(k_end[i]) for i in range(args.steps)]
-    keys = w.keys_per_query
+    keys = w.keys_per_query * n_streams
     value = keys * args.steps * world / (total_ms / 1e3)
 
     # end to end through the public API: host question in, host selection out
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and n_streams == 1:
+        idx = idxs[0]
         q_pin = q_cpu.pin_memory()
         for _ in range(3):
             idx.retrieve_host(q_pin, p, workspace=ws)
@@ -301,34 +342,54 @@ def run_ours(args):
         return
     peak, peak_kind = measured_peak_gbs()
     k1_avg_s = statistics.mean(k1_ms) / 1e3
-    alg_bytes = keys * 256
+    if clusters:
+        # the scoring stage reads the centroids of every window of every slab
+        n_cand = w.n_slabs * (w.n_frames // w.window_frames) * w.n_centroids * n_streams
+        alg_bytes = n_cand * 256
+        kernel = "k_dense"
+        launches = 9   # k_sample, k_cluster_map, k_dense, k_select, k_centroid_weight,
+        #                k_mass, k_pool, k_gram, k_maxmin
+    else:
+        alg_bytes = keys * 256
+        kernel = "k_score"
+        launches = 7   # k_sample, k_score, k_select, k_mass, k_pool, k_gram, k_maxmin
     achieved = alg_bytes / k1_avg_s / 1e9
-    traffic = None
+    traffic = recorded_traffic(w) if not args.frames and n_streams == 1 else None
     cpu = None
     if keys_cpu is not None:
         cpu = cpu_baseline(w, keys_cpu, q_cpu, keys_cpu.shape[2] // w.tokens_per_frame)
+    desc = (f"{w.name}: {w.n_layers} layers x {w.n_kv_heads} kv heads x "
+            f"{w.n_frames} frames x {w.tokens_per_frame} tokens, Hq {w.n_q_heads}, "
+            f"R {w.n_rows}, k {w.k}, budget {w.budget}, pool {w.pool_mult * w.budget}")
+    if n_streams > 1:
+        desc += f", {n_streams} streams per GPU in one batched call"
+    if clusters:
+        desc += (f", windows of {w.window_frames} frames compressed to {w.n_centroids} "
+                 f"centroids ({w.kmeans_iters} Lloyd rounds), retrieval over centroids")
+    config = {"workload": desc, "keys_per_step": keys, "index_bytes": w.key_bytes * n_streams,
+              "l2": f"inputs larger than L2 ({w.key_bytes * n_streams / 1e9:.2f} GB index vs "
+                    f"129 MB L2), no flush",
+              "parallelism": f"replicas x{world} (independent streams per GPU)"}
+    if clusters:
+        config["compress_ms"] = compress_ms
+        config["candidates_per_step"] = n_cand
+        config["l2"] = (f"{alg_bytes / 1e6:.1f} MB of centroids per step: below L2, so the "
+                        f"timed steps read them from L2 (no flush)")
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": max(3, args.warmup),
         "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": f"{w.name}: {w.n_layers} layers x {w.n_kv_heads} kv heads x "
-                               f"{w.n_frames} frames x {w.tokens_per_frame} tokens, "
-                               f"Hq {w.n_q_heads}, R {w.n_rows}, k {w.k}, budget {w.budget}, "
-                               f"pool {w.pool_mult * w.budget}",
-                   "keys_per_step": keys, "index_bytes": w.key_bytes,
-                   "l2": f"inputs larger than L2 ({w.key_bytes / 1e9:.2f} GB index vs "
-                         f"129 MB L2), no flush",
-                   "parallelism": f"replicas x{world} (one independent stream per GPU)"},
+        "config": config,
         "latency_ms": {"p50": statistics.median(step_ms),
                        "p90": step_ms[min(len(step_ms) - 1, int(0.9 * len(step_ms)))],
                        "score_kernel_avg": statistics.mean(k1_ms)},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
-                     "kernel": "k_score", "peak_kind": peak_kind,
+                     "kernel": kernel, "peak_kind": peak_kind,
                      "algorithmic_bytes_per_launch": alg_bytes},
         "clocks": clk,
-        "gpu_launches": 8 * args.steps,
+        "gpu_launches": launches * args.steps,
         "e2e": e2e,
         "cpu_baseline": cpu,
     }

@@ -98,7 +98,7 @@ int64_t cand_cap_of(const ss_index* ix) {
 // Workspace regions of one problem (offsets from the problem's base).
 struct Layout {
   size_t qeff, cand_s, cand_id, cand_cnt, gthr, ladder, samp_max, ustats, next_unit, gram;
-  size_t raw_units, raw_rank, head_ml, aval, aid;  // general path only
+  size_t raw_units, raw_rank, cw, head_ml, aval, aid;  // general path only
   size_t topk_tok, topk_w, list_ml, votes, mass, pool, sel, exp_units, frames, counts,
       status, qstage;
   size_t total;
@@ -142,6 +142,7 @@ Layout layout_of(const ss_index* ix, int R, const ss_retrieve_params* p) {
   if (p->use_clusters) {
     l.raw_units = take(ix->ucap * 4);
     l.raw_rank = take(ix->ucap * 4);
+    l.cw = take((size_t)c.n_layers * c.n_kv_heads * ix->wcap * ix->n_centroids * 4);
   }
   if (p->head_agg == SS_H_MEAN) {
     l.head_ml = take(score_lists * 8);
@@ -221,7 +222,7 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
   B.use_clusters = p->use_clusters;
   const bool general = p->head_agg == SS_H_MEAN || p->use_clusters;
   int max_lists = 0, max_uh = 0, max_pool = 0, n_slabs_total = 0;
-  int max_cand = 0, max_slabs = 0, max_score_lists = 0;
+  int max_cand = 0, max_slabs = 0, max_score_lists = 0, max_cent = 0;
   char* base = static_cast<char*>(ws);
   for (int j = 0; j < n; ++j) {
     const ss_index* x = ix[j];
@@ -292,6 +293,7 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
         P.win_u0 = x->win_u0;
         P.raw_units = reinterpret_cast<int32_t*>(base + l.raw_units);
         P.raw_rank = reinterpret_cast<int32_t*>(base + l.raw_rank);
+        P.cw = reinterpret_cast<float*>(base + l.cw);
       }
       P.n_raw_tok = (int)((P.Uh - covered) * P.Tu);
       P.n_cand = (int)(P.n_raw_tok + n_live * P.n_c);
@@ -301,6 +303,7 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
         P.aid = reinterpret_cast<int32_t*>(base + l.aid);
       }
       max_cand = max(max_cand, P.n_cand);
+      max_cent = max(max_cent, P.n_cand - P.n_raw_tok);
       max_slabs = max(max_slabs, P.P * P.Hkv);
       max_score_lists = max(max_score_lists, P.P * P.Hq);
     }
@@ -334,7 +337,7 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
   if (tr && tr->score_end) SS_CUDA(cudaEventRecord((cudaEvent_t)tr->score_end, st));
   if (general) {
     SS_CUDA(launch_select_general(B, max_lists, st));
-    SS_CUDA(launch_mass_general(B, max_uh, st));
+    SS_CUDA(launch_mass_general(B, max_cent, max_slabs, max_uh, st));
   } else {
     SS_CUDA(launch_select(B, max_lists, st));
     SS_CUDA(launch_mass(B, max_uh, st));

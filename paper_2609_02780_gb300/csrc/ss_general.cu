@@ -15,6 +15,7 @@
 //   k_dense        scores every candidate of every list into a dense row (tensor cores)
 //   k_head_stats   per-head softmax statistics (one list per layer only)
 //   k_alpha        head-averaged weights of every token (one list per layer only)
+//   k_centroid_weight  each centroid's weight summed over its slab's lists
 //   k_mass_general attention mass of every history unit from the dense rows
 // The top-k of a dense row is k_select's general variant (ss_select.cu).
 #include "ss_internal.cuh"
@@ -175,33 +176,58 @@ __global__ void __launch_bounds__(256) k_alpha(const __grid_constant__ Batch B) 
 }
 
 // ---------------------------------------------------------------------------
+// Weight of every centroid summed over the G lists of its slab (heads in order):
+// cw[slab][e] = sum_h 2^(s_{list0 + h, e} - M) / L.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_centroid_weight(const __grid_constant__ Batch B) {
+  pdl_wait();
+  pdl_release();
+  const int pi = blockIdx.z;
+  if (pi >= B.n) return;
+  const Prob& P = B.p[pi];
+  const int slab = blockIdx.y;
+  if (slab >= P.P * P.Hkv) return;
+  const int e = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= P.n_cand - P.n_raw_tok) return;
+  const int i = slab / P.Hkv, gk = slab - i * P.Hkv;
+  const int list0 = i * P.Hq + gk * P.G;
+  float a = 0.f;
+  for (int h = 0; h < P.G; ++h) {
+    const float2 ml = P.list_ml[list0 + h];
+    a += fast_exp2(P.cand_s[(int64_t)(list0 + h) * P.cand_cap + P.n_raw_tok + e] - ml.x) *
+         (1.0f / ml.y);
+  }
+  P.cw[(int64_t)slab * P.wcap * P.n_c + e] = a;
+}
+
+// ---------------------------------------------------------------------------
 // Attention mass of every history unit: the sum over lists of the normalised weights of
 // the unit's tokens; a compressed unit gets, from each centroid of its window, the
-// centroid's weight times (members in the unit) / (members). One warp per unit; the
-// lanes take the (list, token or centroid) terms in a fixed order, then a fixed tree.
+// centroid's weight times (members in the unit) / (members). One block per unit; the
+// threads take the (list, token) or (slab, centroid) terms in a fixed order, then a
+// fixed tree.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) k_mass_general(const __grid_constant__ Batch B) {
+  __shared__ float sm[32];
   pdl_wait();
   pdl_release();
   const int pi = blockIdx.y;
   if (pi >= B.n) return;
   const Prob& P = B.p[pi];
-  const int lane = threadIdx.x & 31;
-  const int u = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int u = blockIdx.x;
   if (u >= P.Uh) return;
-  const int Tu = P.Tu;
+  const int Tu = P.Tu, tid = threadIdx.x;
   float acc = 0.f;
   if (B.head_agg == 1) {
-    for (int t = lane; t < P.P * Tu; t += 32) {
+    for (int t = tid; t < P.P * Tu; t += blockDim.x) {
       const int i = t / Tu, r = t - i * Tu;
       acc += P.aval[(int64_t)i * P.cand_cap + (int64_t)u * Tu + r];
     }
   } else {
-    const int n_lists = P.P * P.Hq;
     const int rr = B.use_clusters ? P.raw_rank[u] : u;
     if (rr >= 0) {
       const int64_t j0 = (int64_t)rr * Tu;
-      for (int t = lane; t < n_lists * Tu; t += 32) {
+      for (int t = tid; t < P.P * P.Hq * Tu; t += blockDim.x) {
         const int L = t / Tu, r = t - L * Tu;
         const float2 ml = P.list_ml[L];
         acc += fast_exp2(P.cand_s[(int64_t)L * P.cand_cap + j0 + r] - ml.x) * (1.0f / ml.y);
@@ -210,23 +236,16 @@ __global__ void __launch_bounds__(256) k_mass_general(const __grid_constant__ Ba
       const int w = P.win_slot[u / P.wu];
       const int x = u - P.win_u0[w];
       const int n_c = P.n_c;
-      const int64_t base = (int64_t)P.n_raw_tok + (int64_t)w * n_c;
-      for (int t = lane; t < n_lists * n_c; t += 32) {
-        const int L = t / n_c, c = t - L * n_c;
-        const int slab = (L / P.Hq) * P.Hkv + (L % P.Hq) / P.G;
+      for (int t = tid; t < P.P * P.Hkv * n_c; t += blockDim.x) {
+        const int slab = t / n_c, c = t - slab * n_c;
         const int64_t wc = ((int64_t)slab * P.wcap + w) * n_c + c;
         const int m = P.mcnt[wc * P.wu + x];
-        if (m) {
-          const float2 ml = P.list_ml[L];
-          const float wgt = fast_exp2(P.cand_s[(int64_t)L * P.cand_cap + base + c] - ml.x) *
-                            (1.0f / ml.y);
-          acc += wgt * (float)m / (float)P.msize[wc];
-        }
+        if (m) acc += P.cw[wc] * (float)m / (float)P.msize[wc];
       }
     }
   }
-  for (int off = 16; off > 0; off >>= 1) acc += __shfl_down_sync(0xffffffffu, acc, off);
-  if (lane == 0) P.mass[u] = acc;
+  acc = block_sum(acc, sm);
+  if (tid == 0) P.mass[u] = acc;
 }
 
 cudaError_t launch_general_score(const Batch& B, int max_cand, int max_slabs,
@@ -251,9 +270,15 @@ cudaError_t launch_general_score(const Batch& B, int max_cand, int max_slabs,
   return cudaSuccess;
 }
 
-cudaError_t launch_mass_general(const Batch& B, int max_hist_units, cudaStream_t s) {
+cudaError_t launch_mass_general(const Batch& B, int max_cent, int max_slabs,
+                                int max_hist_units, cudaStream_t s) {
+  if (B.use_clusters && max_cent > 0) {
+    const cudaError_t e = launch_pdl(k_centroid_weight, dim3((max_cent + 255) / 256, max_slabs, B.n),
+                                     dim3(256), 0, s, B);
+    if (e != cudaSuccess) return e;
+  }
   if (max_hist_units <= 0) return cudaSuccess;
-  return launch_pdl(k_mass_general, dim3((max_hist_units + 7) / 8, B.n), dim3(256), 0, s, B);
+  return launch_pdl(k_mass_general, dim3(max_hist_units, B.n), dim3(256), 0, s, B);
 }
 
 }  // namespace ss

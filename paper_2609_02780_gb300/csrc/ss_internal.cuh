@@ -109,6 +109,8 @@ struct Prob {
   const int32_t* win_u0;       // [wcap] first unit of each window
   int32_t* raw_units;          // [ucap] history units not covered by a window, ascending
   int32_t* raw_rank;           // [ucap] position of a unit in raw_units, or -1
+  float* cw;                   // [P*Hkv][wcap*n_c] summed weight of each centroid over
+                               // the G lists of its slab
   float2* head_ml;             // [P*Hq] (M, L) of each head's softmax (one list per layer)
   float* aval;                 // [P][cand_cap] head-averaged weight of every token
   int32_t* aid;                // [P][cand_cap]
@@ -208,7 +210,8 @@ cudaError_t launch_select(const Batch& B, int max_lists, cudaStream_t s);
 cudaError_t launch_select_general(const Batch& B, int max_lists, cudaStream_t s);
 cudaError_t launch_general_score(const Batch& B, int max_cand, int max_slabs,
                                  int max_score_lists, cudaStream_t s);
-cudaError_t launch_mass_general(const Batch& B, int max_hist_units, cudaStream_t s);
+cudaError_t launch_mass_general(const Batch& B, int max_cent, int max_slabs,
+                                int max_hist_units, cudaStream_t s);
 cudaError_t launch_mass(const Batch& B, int max_hist_units, cudaStream_t s);
 
 cudaError_t launch_pool(const Batch& B, int max_hist_units, cudaStream_t s);

@@ -246,10 +246,12 @@ __global__ void __launch_bounds__(kSelThreads) k_select_t(const __grid_constant_
     }
     lo = block_min(mn, s_m);
   }
+  // A dense row of more than 2048 candidates goes straight to the histogram below.
+  const bool dense = kGeneral && cnt > 2 * kSelThreads;
   // collect the candidates at or above the bound (warp-aggregated slot counter)
   if (tid == 0) s_n = 0;
   __syncthreads();
-  {
+  if (!dense) {
     // each thread scans 4 consecutive slots per step (one 16-byte load; the list's slots
     // start 256-byte aligned), with the next step's load issued before this one's work
     const float4* cs4 = reinterpret_cast<const float4*>(cs);
@@ -278,7 +280,7 @@ __global__ void __launch_bounds__(kSelThreads) k_select_t(const __grid_constant_
     }
   }
   __syncthreads();
-  int ns = s_n;
+  int ns = dense ? kSelCap + 1 : s_n;
   if (ns > kSelCap) {
     // Too many: a 2048-bin histogram of the candidates over [lo, max] locates the bin
     // of the n-th best; keep the candidates from that bin up.
