@@ -84,6 +84,13 @@ def max_over_ranks(x: float, world: int) -> float:
     return float(t.item())
 
 
+def whole_job_rate(units_per_step_per_rank: int, steps: int, world: int,
+                   max_ms_over_ranks: float) -> float:
+    """Units per second of the whole job: every rank processes its own units (weak
+    scaling), timed by the slowest rank."""
+    return units_per_step_per_rank * steps * world / (max_ms_over_ranks / 1e3)
+
+
 class ClockSampler:
     """nvidia-smi clock / throttle samples while the timed region runs."""
 
@@ -315,7 +322,7 @@ def run_ours(args):
     step_ms = sorted(s_begin[i].elapsed_time(s_end[i]) for i in range(args.steps))
     k1_ms = [k_begin[i].elapsed_time(k_end[i]) for i in range(args.steps)]
     keys = w.keys_per_query * n_streams
-    value = keys * args.steps * world / (total_ms / 1e3)
+    value = whole_job_rate(keys, args.steps, world, total_ms)
 
     # end to end through the public API: host question in, host selection out
     e2e = None
