@@ -306,8 +306,9 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
   const int local = b - P.cta_begin;
   const int n_slabs = P.P * P.Hkv;
   if (P.chunks <= 0) return;
-  const int slab = local / P.chunks;
-  if (slab >= n_slabs) return;
+  // consecutive CTAs go to different slabs, so each slab's CTAs spread over the SMs
+  if (local >= n_slabs * P.chunks) return;
+  const int slab = local % n_slabs;
 
   const int i = slab / P.Hkv, kvh = slab - i * P.Hkv;
   const int G = P.G;
