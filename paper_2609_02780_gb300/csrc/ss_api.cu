@@ -325,6 +325,7 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
     cta += P.P * P.Hkv * P.chunks;
   }
   B.score_ctas = cta;
+  B.score_spread = cta <= score_slots(ix[0]->sm_count) ? 1 : 0;
 
   SS_CUDA(cudaSetDevice(dev));
   SS_CUDA(launch_prep(B, st));
@@ -336,10 +337,10 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
   }
   if (tr && tr->score_end) SS_CUDA(cudaEventRecord((cudaEvent_t)tr->score_end, st));
   if (general) {
-    SS_CUDA(launch_select_general(B, max_lists, st));
+    SS_CUDA(launch_select_general(B, max_lists, ix[0]->sm_count, st));
     SS_CUDA(launch_mass_general(B, max_cent, max_slabs, max_uh, st));
   } else {
-    SS_CUDA(launch_select(B, max_lists, st));
+    SS_CUDA(launch_select(B, max_lists, ix[0]->sm_count, st));
     SS_CUDA(launch_mass(B, max_uh, st));
   }
   SS_CUDA(launch_pool(B, max_uh, st));

@@ -130,6 +130,7 @@ struct Batch {
   int head_agg;
   int use_clusters;
   int score_ctas;              // total CTAs of the score kernel
+  int score_spread;            // 1: one wave; slab = CTA index mod slabs
 };
 static_assert(sizeof(Batch) <= 32000, "kernel parameter block too large");
 
@@ -206,8 +207,8 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
 cudaError_t launch_prep(const Batch& B, cudaStream_t s);
 int sample_units(int k, int tokens_per_unit, int hist_units);
 cudaError_t launch_score(const Batch& B, cudaStream_t s);
-cudaError_t launch_select(const Batch& B, int max_lists, cudaStream_t s);
-cudaError_t launch_select_general(const Batch& B, int max_lists, cudaStream_t s);
+cudaError_t launch_select(const Batch& B, int max_lists, int sm_count, cudaStream_t s);
+cudaError_t launch_select_general(const Batch& B, int max_lists, int sm_count, cudaStream_t s);
 cudaError_t launch_general_score(const Batch& B, int max_cand, int max_slabs,
                                  int max_score_lists, cudaStream_t s);
 cudaError_t launch_mass_general(const Batch& B, int max_cent, int max_slabs,
@@ -229,4 +230,5 @@ cudaError_t launch_descriptors(const __nv_bfloat16* keys, int64_t ncap, int P, i
                                int Tu, int64_t u_begin, int64_t u_end, float* desc,
                                cudaStream_t s);
 int score_chunks_per_slab(int n_slabs_total, int hist_units, int sm_count);
+int score_slots(int sm_count);
 }  // namespace ss

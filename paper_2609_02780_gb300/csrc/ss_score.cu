@@ -306,9 +306,10 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
   const int local = b - P.cta_begin;
   const int n_slabs = P.P * P.Hkv;
   if (P.chunks <= 0) return;
-  // consecutive CTAs go to different slabs, so each slab's CTAs spread over the SMs
+  // In a one-wave grid consecutive CTAs go to different slabs, so each slab's CTAs
+  // spread over the SMs; a grid of several waves keeps a slab's CTAs together.
   if (local >= n_slabs * P.chunks) return;
-  const int slab = local % n_slabs;
+  const int slab = B.score_spread ? local % n_slabs : local / P.chunks;
 
   const int i = slab / P.Hkv, kvh = slab - i * P.Hkv;
   const int G = P.G;
@@ -587,6 +588,8 @@ int score_chunks_per_slab(int n_slabs_total, int hist_units, int sm_count) {
   }
   return best_c;
 }
+
+int score_slots(int sm_count) { return sm_count * kScoreCtasPerSm; }
 
 cudaError_t launch_score(const Batch& B, cudaStream_t s) {
   if (B.score_ctas <= 0) return cudaSuccess;

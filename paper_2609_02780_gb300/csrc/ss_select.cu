@@ -14,9 +14,11 @@
 
 namespace ss {
 
-constexpr int kSelThreads = 1024;
+// k_select runs 1024 threads per list with room for 16384 survivors, or, when the lists
+// outnumber the SMs, 512 threads with room for 8192 so that two lists share an SM.
 constexpr int kMassUnits = 32;     // history units per mass block
-constexpr int kSelCap = 16384;   // survivors sorted in shared memory
+template <int kThreads>
+constexpr int sel_cap() { return kThreads >= 1024 ? 16384 : 8192; }  // survivors in smem
 constexpr int kFineBins = 2048;  // second-level score histogram of k_select
 
 __device__ __forceinline__ unsigned long long cand_key(float s, int32_t id) {
@@ -108,6 +110,75 @@ __device__ void bitonic_desc_hybrid(unsigned long long* a, int n2) {
   __syncthreads();
 }
 
+// Descending sort of keys[0, ns) by bucketing on the score (the upper 32 bits of a key):
+// 2048 buckets over [lo, hi] (every key's score lies there), a counting scatter in
+// bucket order, then an insertion sort inside each bucket. Needs ns <= kSelCap / 2
+// (the upper half of `keys` holds the input copy) and buckets of at most kBucketMax
+// keys; returns false, with keys untouched, when a bucket is larger (then the caller
+// sorts another way). All threads of the block call it.
+constexpr int kBucketMax = 32;
+
+template <int kThreads>
+__device__ bool bucket_sort_desc(unsigned long long* keys, int ns, float lo, float hi,
+                                 int* hist, int* cursor, int* sflag) {
+  const int tid = threadIdx.x;
+  const uint32_t klo = float_to_ordered(lo), khi = float_to_ordered(hi);
+  const uint64_t span = (uint64_t)(khi - klo) + 1u;
+  auto bucket = [&](unsigned long long key) -> int {
+    const uint32_t ok = (uint32_t)(key >> 32);
+    const uint64_t d = ok > klo ? (uint64_t)(ok - klo) : 0u;
+    const int b = (int)((d * kFineBins) / span);
+    return kFineBins - 1 - min(b, kFineBins - 1);  // best scores first
+  };
+  for (int b = tid; b < kFineBins; b += blockDim.x) hist[b] = 0;
+  if (tid == 0) *sflag = 0;
+  __syncthreads();
+  for (int i = tid; i < ns; i += blockDim.x) atomicAdd(&hist[bucket(keys[i])], 1);
+  __syncthreads();
+  // exclusive scan of the bucket counts (each thread owns consecutive buckets)
+  constexpr int kPerT = kFineBins / kThreads;
+  int c[kPerT], tot = 0;
+#pragma unroll
+  for (int q = 0; q < kPerT; ++q) {
+    c[q] = hist[kPerT * tid + q];
+    tot += c[q];
+    if (c[q] > kBucketMax) *sflag = 1;
+  }
+  __shared__ int sw[32];
+  int run = block_excl_scan(tot, sw);
+  const bool big = *sflag != 0;
+  __syncthreads();
+  if (big) return false;
+#pragma unroll
+  for (int q = 0; q < kPerT; ++q) {
+    hist[kPerT * tid + q] = run;
+    cursor[kPerT * tid + q] = run;
+    run += c[q];
+  }
+  unsigned long long* in = keys + sel_cap<kThreads>() / 2;
+  for (int i = tid; i < ns; i += blockDim.x) in[i] = keys[i];
+  __syncthreads();
+  for (int i = tid; i < ns; i += blockDim.x) {
+    const unsigned long long key = in[i];
+    keys[atomicAdd(&cursor[bucket(key)], 1)] = key;
+  }
+  __syncthreads();
+  for (int b = tid; b < kFineBins; b += blockDim.x) {
+    const int b0 = hist[b], b1 = cursor[b];  // after the scatter: the bucket's end
+    for (int i = b0 + 1; i < b1; ++i) {
+      const unsigned long long x = keys[i];
+      int j = i - 1;
+      while (j >= b0 && keys[j] < x) {
+        keys[j + 1] = keys[j];
+        --j;
+      }
+      keys[j + 1] = x;
+    }
+  }
+  __syncthreads();
+  return true;
+}
+
 __device__ __forceinline__ int next_pow2(int x) {
   int p = 1;
   while (p < x) p <<= 1;
@@ -125,10 +196,13 @@ __device__ __forceinline__ int next_pow2(int x) {
 // kGeneral: the general path (one list per layer, or centroid candidates). Its lists
 // hold every candidate (a dense row), its softmax statistics come from that row, and
 // with one list per layer the row holds the head-averaged weights themselves.
-template <bool kGeneral>
-__global__ void __launch_bounds__(kSelThreads) k_select_t(const __grid_constant__ Batch B) {
+template <bool kGeneral, int kThreads>
+__global__ void __launch_bounds__(kThreads) k_select_t(const __grid_constant__ Batch B) {
+  constexpr int kSelCap = sel_cap<kThreads>();
   extern __shared__ unsigned long long skeys[];
   __shared__ int s_hist[kFineBins];
+  __shared__ int s_cursor[kFineBins];
+  __shared__ int s_flag;
   __shared__ float s_m[32], s_l[32];
   __shared__ int s_n, s_bstar, s_rem;
   __shared__ unsigned long long s_prefix;
@@ -247,34 +321,54 @@ __global__ void __launch_bounds__(kSelThreads) k_select_t(const __grid_constant_
     lo = block_min(mn, s_m);
   }
   // A dense row of more than 2048 candidates goes straight to the histogram below.
-  const bool dense = kGeneral && cnt > 2 * kSelThreads;
+  const bool dense = kGeneral && cnt > 2 * kThreads;
   // collect the candidates at or above the bound (warp-aggregated slot counter)
   if (tid == 0) s_n = 0;
   __syncthreads();
   if (!dense) {
-    // each thread scans 4 consecutive slots per step (one 16-byte load; the list's slots
-    // start 256-byte aligned), with the next step's load issued before this one's work
+    // each thread loads 4 x 4 consecutive slots per round (16-byte loads; the list's slots
+    // start 256-byte aligned); a warp claims the round's output slots with one atomic
+    constexpr int kU = 4096 / kThreads;
     const float4* cs4 = reinterpret_cast<const float4*>(cs);
     const int n4 = (cnt + 3) >> 2;
-    const int step = blockDim.x;
-    float4 nxt = tid < n4 ? cs4[tid] : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
-    for (int b0 = 0; b0 < n4; b0 += step) {
-      const int x4 = b0 + tid;
-      const float4 cur = nxt;
-      const int y4 = x4 + step;
-      nxt = y4 < n4 ? cs4[y4] : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
-      const float v[4] = {cur.x, cur.y, cur.z, cur.w};
+    const float4 ninf = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+    for (int b0 = 0; b0 < n4; b0 += kU * (int)blockDim.x) {
+      float4 v4[kU];
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int x = 4 * x4 + e;
-        const bool keep = x < cnt && v[e] >= lo;
-        const unsigned m = __ballot_sync(0xffffffffu, keep);
-        int base = 0;
-        if (lane == 0 && m) base = atomicAdd(&s_n, __popc(m));
-        base = __shfl_sync(0xffffffffu, base, 0);
-        if (keep) {
-          const int pos = base + __popc(m & ((1u << lane) - 1u));
+      for (int u = 0; u < kU; ++u) {
+        const int x4 = b0 + u * blockDim.x + tid;
+        v4[u] = x4 < n4 ? cs4[x4] : ninf;
+      }
+      float v[4 * kU];
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        v[4 * u] = v4[u].x;
+        v[4 * u + 1] = v4[u].y;
+        v[4 * u + 2] = v4[u].z;
+        v[4 * u + 3] = v4[u].w;
+      }
+      unsigned kb = 0u;
+#pragma unroll
+      for (int e = 0; e < 4 * kU; ++e) {
+        const int x = 4 * (b0 + (e >> 2) * blockDim.x + tid) + (e & 3);
+        if (x < cnt && v[e] >= lo) kb |= 1u << e;
+      }
+      const int c = __popc(kb);
+      int incl = c;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off) incl += y;
+      }
+      int base = 0;
+      if (lane == 31 && incl) base = atomicAdd(&s_n, incl);
+      int pos = __shfl_sync(0xffffffffu, base, 31) + incl - c;
+#pragma unroll
+      for (int e = 0; e < 4 * kU; ++e) {
+        if ((kb >> e) & 1u) {
+          const int x = 4 * (b0 + (e >> 2) * blockDim.x + tid) + (e & 3);
           if (pos < kSelCap) skeys[pos] = cand_key(v[e], ci[x]);
+          ++pos;
         }
       }
     }
@@ -388,13 +482,18 @@ __global__ void __launch_bounds__(kSelThreads) k_select_t(const __grid_constant_
     if (tid == 0) atomicOr(P.status, kStatusInternal);
     n = ns;
   }
-  const int n2 = max(64, next_pow2(max(ns, 1)));
-  for (int x = ns + tid; x < n2; x += blockDim.x) skeys[x] = 0ull;
-  __syncthreads();
-  if (n2 <= 2 * kSelThreads) {
-    bitonic_desc_hybrid(skeys, n2);
-  } else {
-    bitonic_desc(skeys, n2);
+  const bool bucketed =
+      ns > 64 && ns <= kSelCap / 2 &&
+      bucket_sort_desc<kThreads>(skeys, ns, lo, M, s_hist, s_cursor, &s_flag);
+  if (!bucketed) {
+    const int n2 = max(64, next_pow2(max(ns, 1)));
+    for (int x = ns + tid; x < n2; x += blockDim.x) skeys[x] = 0ull;
+    __syncthreads();
+    if (n2 <= 2 * kThreads) {
+      bitonic_desc_hybrid(skeys, n2);
+    } else {
+      bitonic_desc(skeys, n2);
+    }
   }
   const float inv_l = 1.0f / Ls;
   for (int r = tid; r < k; r += blockDim.x) {
@@ -426,20 +525,24 @@ __global__ void __launch_bounds__(kSelThreads) k_select_t(const __grid_constant_
   (void)lane;
 }
 
-cudaError_t launch_select(const Batch& B, int max_lists, cudaStream_t s) {
-  const int smem = kSelCap * (int)sizeof(unsigned long long);
-  cudaError_t e = cudaFuncSetAttribute(k_select_t<false>,
+template <bool kGeneral, int kThreads>
+cudaError_t launch_select_t(const Batch& B, int max_lists, cudaStream_t s) {
+  const int smem = sel_cap<kThreads>() * (int)sizeof(unsigned long long);
+  cudaError_t e = cudaFuncSetAttribute(k_select_t<kGeneral, kThreads>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  return launch_pdl(k_select_t<false>, dim3(max_lists, B.n), dim3(kSelThreads), (size_t)smem, s, B);
+  return launch_pdl(k_select_t<kGeneral, kThreads>, dim3(max_lists, B.n), dim3(kThreads),
+                    (size_t)smem, s, B);
 }
 
-cudaError_t launch_select_general(const Batch& B, int max_lists, cudaStream_t s) {
-  const int smem = kSelCap * (int)sizeof(unsigned long long);
-  cudaError_t e = cudaFuncSetAttribute(k_select_t<true>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  if (e != cudaSuccess) return e;
-  return launch_pdl(k_select_t<true>, dim3(max_lists, B.n), dim3(kSelThreads), (size_t)smem, s, B);
+cudaError_t launch_select(const Batch& B, int max_lists, int sm_count, cudaStream_t s) {
+  if ((int64_t)max_lists * B.n <= sm_count) return launch_select_t<false, 1024>(B, max_lists, s);
+  return launch_select_t<false, 512>(B, max_lists, s);
+}
+
+cudaError_t launch_select_general(const Batch& B, int max_lists, int sm_count, cudaStream_t s) {
+  if ((int64_t)max_lists * B.n <= sm_count) return launch_select_t<true, 1024>(B, max_lists, s);
+  return launch_select_t<true, 512>(B, max_lists, s);
 }
 
 // ---------------------------------------------------------------------------
