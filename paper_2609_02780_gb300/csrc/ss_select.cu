@@ -767,14 +767,30 @@ __global__ void __launch_bounds__(256) k_gram(const __grid_constant__ Batch B) {
   if (a < pn && b < pn && a <= b) P.gram[tri_off(a, pn) + (b - a)] = acc;
 }
 
-// Greedy max-min (DivTopK) by one warp over the packed Gram triangle (in shared memory
-// when it fits), then the expansion (Nbr of Eq. 12) by the whole block. Lane l owns
-// the pool ranks l, l + 32, ...; kPer = ranks per lane.
-constexpr int kMaxMinSmemPool = 320;   // packed triangle of 320 ranks = 201 KB
+// Greedy max-min (DivTopK) by one warp over the packed Gram triangle, then the
+// expansion (Nbr of Eq. 12) by the whole block. Lane l owns the pool ranks l, l + 32,
+// ...; kPer = ranks per lane. The triangle sits in shared memory as fp32 up to 320
+// ranks (201 KB), as 24-bit fixed point (2^-22 steps, far below the fp32 Gram's own
+// rounding at the distances compared) up to 384 ranks (222 KB), else in global memory.
+constexpr int kMaxMinSmemPool = 320;
+constexpr int kMaxMinFixedPool = 384;
 constexpr int kMaxMinThreads = kMaxHistUnits / 32;  // one bitmap word per thread
 
-template <int kPer>
-__device__ void greedy_maxmin(const Prob& P, const float* pk, const int* pool, int* sel,
+struct TriF32 {  // fp32 triangle (shared or global memory)
+  const float* p;
+  __device__ __forceinline__ float operator()(int i) const { return p[i]; }
+};
+struct TriFix24 {  // 24-bit fixed point split into 16 high and 8 low bits
+  const uint16_t* hi;
+  const uint8_t* lo;
+  __device__ __forceinline__ float operator()(int i) const {
+    const int x = ((int)(((uint32_t)hi[i] << 16) | ((uint32_t)lo[i] << 8))) >> 8;
+    return (float)x * (1.0f / 4194304.0f);
+  }
+};
+
+template <int kPer, class Tri>
+__device__ void greedy_maxmin(const Prob& P, const Tri pk, const int* pool, int* sel,
                               int pn, int ns) {
   const int lane = threadIdx.x & 31;
   float mind[kPer];
@@ -783,7 +799,7 @@ __device__ void greedy_maxmin(const Prob& P, const float* pk, const int* pool, i
   for (int q = 0; q < kPer; ++q) {
     const int c = lane + 32 * q;
     toff[q] = tri_off(c, pn);
-    mind[q] = c < pn ? 1.0f - pk[c] : -INFINITY;  // row 0 of the triangle is G[0][*]
+    mind[q] = c < pn ? 1.0f - pk(c) : -INFINITY;  // row 0 of the triangle is G[0][*]
   }
   uint32_t taken = lane == 0 ? 1u : 0u;  // bit q: rank lane + 32 q is picked
   if (lane == 0) sel[0] = pool[0];
@@ -829,7 +845,7 @@ __device__ void greedy_maxmin(const Prob& P, const float* pk, const int* pool, i
     for (int q = 0; q < kPer; ++q) {
       const int c = lane + 32 * q;
       if (c < pn) {
-        const float g = c >= best ? pk[rowoff + c] : pk[toff[q] + best - c];
+        const float g = pk(c >= best ? rowoff + c : toff[q] + best - c);
         mind[q] = fminf(mind[q], 1.0f - g);
       }
     }
@@ -847,11 +863,22 @@ __global__ void __launch_bounds__(kMaxMinThreads) k_maxmin(const __grid_constant
   const int pn = P.pool_n, ns = P.n_sel;
   const int tid = threadIdx.x, warp = tid >> 5;
   const bool in_smem = pn <= kMaxMinSmemPool;
+  const bool fixed24 = !in_smem && pn <= kMaxMinFixedPool;
+  const int total = tri_off(pn, pn);
+  uint16_t* fhi = reinterpret_cast<uint16_t*>(pks4);
+  uint8_t* flo = reinterpret_cast<uint8_t*>(fhi + total);
   for (int x = tid; x < pn; x += blockDim.x) spool[x] = P.pool[x];
   if (in_smem) {
-    const int total4 = (tri_off(pn, pn) + 3) / 4;
+    const int total4 = (total + 3) / 4;
     const float4* g4 = reinterpret_cast<const float4*>(P.gram);
     for (int x = tid; x < total4; x += blockDim.x) pks4[x] = g4[x];
+  } else if (fixed24) {
+    for (int x = tid; x < total; x += blockDim.x) {
+      const float g = fminf(fmaxf(P.gram[x], -1.99f), 1.99f);
+      const int v = __float2int_rn(g * 4194304.0f);
+      fhi[x] = (uint16_t)((uint32_t)v >> 8);
+      flo[x] = (uint8_t)((uint32_t)v & 0xffu);
+    }
   }
   __syncthreads();
   // One warp does the rest: warps parked at a barrier would slow its serial greedy.
@@ -862,15 +889,18 @@ __global__ void __launch_bounds__(kMaxMinThreads) k_maxmin(const __grid_constant
     // to the compiler, so the greedy's reads are plain shared-memory loads when staged
     const int per = (pn + 31) / 32;
     if (in_smem) {
-      const float* sk = reinterpret_cast<const float*>(pks4);
+      const TriF32 sk{reinterpret_cast<const float*>(pks4)};
       if (per <= 1) greedy_maxmin<1>(P, sk, spool, ssel, pn, ns);
       else if (per <= 2) greedy_maxmin<2>(P, sk, spool, ssel, pn, ns);
       else if (per <= 4) greedy_maxmin<4>(P, sk, spool, ssel, pn, ns);
       else if (per <= 8) greedy_maxmin<8>(P, sk, spool, ssel, pn, ns);
       else greedy_maxmin<16>(P, sk, spool, ssel, pn, ns);   // pool <= 320 here
+    } else if (fixed24) {
+      greedy_maxmin<12>(P, TriFix24{fhi, flo}, spool, ssel, pn, ns);   // 320 < pool <= 384
     } else {
-      if (per <= 16) greedy_maxmin<16>(P, P.gram, spool, ssel, pn, ns);
-      else greedy_maxmin<32>(P, P.gram, spool, ssel, pn, ns);
+      const TriF32 gk{P.gram};
+      if (per <= 16) greedy_maxmin<16>(P, gk, spool, ssel, pn, ns);
+      else greedy_maxmin<32>(P, gk, spool, ssel, pn, ns);
     }
   }
   __syncwarp();
@@ -929,8 +959,9 @@ cudaError_t launch_maxmin(const Batch& B, int max_pool, cudaStream_t s) {
     e = launch_pdl(k_gram, grid, dim3(kGramTile * kGramTile), (size_t)smem, s, B);
     if (e != cudaSuccess) return e;
   }
-  const int pk_n = max_pool <= kMaxMinSmemPool ? max_pool * (max_pool + 1) / 2 : 0;
-  const int smem = ((max(pk_n, 1) + 3) / 4) * (int)sizeof(float4);
+  const int tri = max_pool * (max_pool + 1) / 2;
+  const int bytes = max_pool <= kMaxMinSmemPool ? tri * 4 : max_pool <= kMaxMinFixedPool ? tri * 3 : 4;
+  const int smem = ((bytes + 15) / 16) * (int)sizeof(float4);
   cudaError_t e = cudaFuncSetAttribute(k_maxmin, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   return launch_pdl(k_maxmin, dim3(B.n), dim3(kMaxMinThreads), (size_t)smem, s, B);

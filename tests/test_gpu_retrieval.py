@@ -203,3 +203,11 @@ def test_invalid_arguments_fail_before_launch():
         idx.retrieve(q, k=5, budget=0)
     with pytest.raises(ss.ShallowStreamError, match="UNSUPPORTED"):
         ss.Index(1, 4, 2, 8, 10, head_dim=64, device="cuda")
+
+
+def test_maxmin_pool_sizes_across_the_gram_storage_forms():
+    # the Gram triangle of the pool is held in fp32 (pool <= 320), 24-bit fixed point
+    # (320 < pool <= 384) or global memory (larger); each must give a valid greedy
+    keys, q = gaussian_case(12, P=1, Hq=4, Hkv=1, F=420, Tf=8, R_rows=2)
+    for budget in (80, 96, 105):              # pools 320, 384, 420
+        run_case(keys, q, tokens_per_frame=8, k=64, budget=budget, check_e2e=False)
