@@ -118,8 +118,10 @@ Layout layout_of(const ss_index* ix, int R, const ss_retrieve_params* p) {
   const int64_t pc = pool_cap_of(ix, p);
   const int64_t nexp = (int64_t)p->budget_units * (1 + p->n_prev);
   l.qeff = take(score_lists * kHeadDim * 2);
-  l.cand_s = take(score_lists * cand_cap_of(ix) * 4);
-  l.cand_id = take(score_lists * cand_cap_of(ix) * 4);
+  // candidate (score, id) pairs of the default path; the general path's dense score
+  // and id rows are the two halves of the same region
+  l.cand_s = take(score_lists * cand_cap_of(ix) * 8);
+  l.cand_id = l.cand_s + score_lists * cand_cap_of(ix) * 4;
   l.cand_cnt = take(score_lists * 4);
   l.gthr = take(score_lists * 4);
   l.ladder = take(score_lists * kLadderLevels * 4);
@@ -244,6 +246,7 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
     P.q = static_cast<const __nv_bfloat16*>(q[j]);
     P.R = R[j];
     P.qeff = reinterpret_cast<__nv_bfloat16*>(base + l.qeff);
+    P.cand_pair = reinterpret_cast<float2*>(base + l.cand_s);
     P.cand_s = reinterpret_cast<float*>(base + l.cand_s);
     P.cand_id = reinterpret_cast<int32_t*>(base + l.cand_id);
     P.cand_cap = cand_cap_of(x);

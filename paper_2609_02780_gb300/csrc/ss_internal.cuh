@@ -74,8 +74,10 @@ struct Prob {
   int R;
   // workspace
   __nv_bfloat16* qeff;         // [P][Hq][d]
-  float* cand_s;               // [n_score_lists][cand_cap]
-  int32_t* cand_id;
+  float2* cand_pair;           // [n_score_lists][cand_cap] (score, id bits): the score
+                               // kernel's appended candidates
+  float* cand_s;               // [n_score_lists][cand_cap] dense rows (general path),
+  int32_t* cand_id;            // over the same memory as cand_pair
   int64_t cand_cap;
   int32_t* cand_cnt;           // [n_score_lists]
   uint32_t* gthr;              // [n_score_lists] ordered-float threshold

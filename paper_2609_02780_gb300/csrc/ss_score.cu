@@ -397,26 +397,22 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
     auto slot1 = [&](int r) { return cbase1 + (r < rl1 ? rp1 + r : nb1 + (r - rl1)); };
     if (p00) {
       const int64_t pos = slot0(__popc(b00 & lt_mask));
-      P.cand_s[pos] = s00;
-      P.cand_id[pos] = tok0;
+      P.cand_pair[pos] = make_float2(s00, __int_as_float(tok0));
       ladder_add(S, c0, s00, an0);
     }
     if (p10) {
       const int64_t pos = slot0(__popc(b00) + __popc(b10 & lt_mask));
-      P.cand_s[pos] = s10;
-      P.cand_id[pos] = tok1;
+      P.cand_pair[pos] = make_float2(s10, __int_as_float(tok1));
       ladder_add(S, c0, s10, an0);
     }
     if (p01) {
       const int64_t pos = slot1(__popc(b01 & lt_mask));
-      P.cand_s[pos] = s01;
-      P.cand_id[pos] = tok0;
+      P.cand_pair[pos] = make_float2(s01, __int_as_float(tok0));
       ladder_add(S, c1, s01, an1);
     }
     if (p11) {
       const int64_t pos = slot1(__popc(b01) + __popc(b11 & lt_mask));
-      P.cand_s[pos] = s11;
-      P.cand_id[pos] = tok1;
+      P.cand_pair[pos] = make_float2(s11, __int_as_float(tok1));
       ladder_add(S, c1, s11, an1);
     }
     if (need0) {
@@ -549,8 +545,8 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
     }
   }
   // unused reserved slots are marked empty (score -inf)
-  for (int x = g; x < rl0; x += 8) P.cand_s[cbase0 + rp0 + x] = -INFINITY;
-  for (int x = g; x < rl1; x += 8) P.cand_s[cbase1 + rp1 + x] = -INFINITY;
+  for (int x = g; x < rl0; x += 8) P.cand_pair[cbase0 + rp0 + x].x = -INFINITY;
+  for (int x = g; x < rl1; x += 8) P.cand_pair[cbase1 + rp1 + x].x = -INFINITY;
   if (aborted) {
     // report, then let the copies already in flight land before the CTA exits
     if (lane == 0) atomicOr(P.status, kStatusTimeout);

@@ -245,8 +245,19 @@ __global__ void __launch_bounds__(kThreads) k_select_t(const __grid_constant__ B
     return;
   }
   const int cnt = kGeneral ? P.n_cand : P.cand_cnt[L];
+  // candidates: (score, id) pairs appended by the score kernel, or the general path's
+  // dense rows of values and ids
   const float* cs = (mean ? P.aval : P.cand_s) + (int64_t)L * P.cand_cap;
   const int32_t* ci = (mean ? P.aid : P.cand_id) + (int64_t)L * P.cand_cap;
+  const float2* cp = P.cand_pair + (int64_t)L * P.cand_cap;
+  auto sc_at = [&](int x) -> float {
+    if constexpr (kGeneral) return cs[x];
+    else return cp[x].x;
+  };
+  auto id_at = [&](int x) -> int32_t {
+    if constexpr (kGeneral) return ci[x];
+    else return __float_as_int(cp[x].y);
+  };
   float lo = -INFINITY;
   if constexpr (kGeneral) {
     // statistics of the dense row in a fixed order: (max, sum 2^(s - max)) of the
@@ -315,7 +326,7 @@ __global__ void __launch_bounds__(kThreads) k_select_t(const __grid_constant__ B
     // -inf and are never candidates)
     float mn = INFINITY;
     for (int x = tid; x < cnt; x += blockDim.x) {
-      const float s = cs[x];
+      const float s = sc_at(x);
       if (s > -INFINITY) mn = fminf(mn, s);
     }
     lo = block_min(mn, s_m);
@@ -325,7 +336,48 @@ __global__ void __launch_bounds__(kThreads) k_select_t(const __grid_constant__ B
   // collect the candidates at or above the bound (warp-aggregated slot counter)
   if (tid == 0) s_n = 0;
   __syncthreads();
-  if (!dense) {
+  if constexpr (!kGeneral) {
+    // each thread loads 4 x 2 consecutive (score, id) slots per round (16-byte loads; the
+    // list's slots start 256-byte aligned); a warp claims its output slots with one atomic
+    constexpr int kU = 4096 / kThreads;
+    const float4* cp4 = reinterpret_cast<const float4*>(cp);
+    const int n2p = (cnt + 1) >> 1;
+    const float4 ninf = make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
+    for (int b0 = 0; b0 < n2p; b0 += kU * (int)blockDim.x) {
+      float4 v4[kU];
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const int x2 = b0 + u * blockDim.x + tid;
+        v4[u] = x2 < n2p ? cp4[x2] : ninf;
+      }
+      unsigned kb = 0u;
+#pragma unroll
+      for (int e = 0; e < 2 * kU; ++e) {
+        const int x = 2 * (b0 + (e >> 1) * blockDim.x + tid) + (e & 1);
+        const float v = (e & 1) ? v4[e >> 1].z : v4[e >> 1].x;
+        if (x < cnt && v >= lo) kb |= 1u << e;
+      }
+      const int c = __popc(kb);
+      int incl = c;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off) incl += y;
+      }
+      int base = 0;
+      if (lane == 31 && incl) base = atomicAdd(&s_n, incl);
+      int pos = __shfl_sync(0xffffffffu, base, 31) + incl - c;
+#pragma unroll
+      for (int e = 0; e < 2 * kU; ++e) {
+        if ((kb >> e) & 1u) {
+          const float v = (e & 1) ? v4[e >> 1].z : v4[e >> 1].x;
+          const float idf = (e & 1) ? v4[e >> 1].w : v4[e >> 1].y;
+          if (pos < kSelCap) skeys[pos] = cand_key(v, __float_as_int(idf));
+          ++pos;
+        }
+      }
+    }
+  } else if (!dense) {
     // each thread loads 4 x 4 consecutive slots per round (16-byte loads; the list's slots
     // start 256-byte aligned); a warp claims the round's output slots with one atomic
     constexpr int kU = 4096 / kThreads;
@@ -387,7 +439,7 @@ __global__ void __launch_bounds__(kThreads) k_select_t(const __grid_constant__ B
     for (int x = tid; x < kFineBins; x += blockDim.x) s_hist[x] = 0;
     __syncthreads();
     for (int x = tid; x < cnt; x += blockDim.x) {
-      const float s = cs[x];
+      const float s = sc_at(x);
       if (s >= lo) atomicAdd(&s_hist[fbin(s)], 1);
     }
     __syncthreads();
@@ -422,10 +474,10 @@ __global__ void __launch_bounds__(kThreads) k_select_t(const __grid_constant__ B
     if (bstar < 0 && tid == 0) atomicOr(P.status, kStatusInternal);
     const int bmin = max(bstar, 0);
     for (int x = tid; x < cnt; x += blockDim.x) {
-      const float s = cs[x];
+      const float s = sc_at(x);
       if (s >= lo && fbin(s) >= bmin) {
         const int pos = atomicAdd(&s_n, 1);
-        if (pos < kSelCap) skeys[pos] = cand_key(s, ci[x]);
+        if (pos < kSelCap) skeys[pos] = cand_key(s, id_at(x));
       }
     }
     __syncthreads();
@@ -444,9 +496,9 @@ __global__ void __launch_bounds__(kThreads) k_select_t(const __grid_constant__ B
       const unsigned long long prefix = s_prefix;
       const unsigned long long hmask = (shift == 56) ? 0ull : (~0ull << (shift + 8));
       for (int x = tid; x < cnt; x += blockDim.x) {
-        const float s = cs[x];
+        const float s = sc_at(x);
         if (s < lo) continue;
-        const unsigned long long key = cand_key(s, ci[x]);
+        const unsigned long long key = cand_key(s, id_at(x));
         if ((key & hmask) != (prefix & hmask)) continue;
         atomicAdd(&s_hist[(key >> shift) & 255u], 1);
       }
@@ -466,9 +518,9 @@ __global__ void __launch_bounds__(kThreads) k_select_t(const __grid_constant__ B
     if (tid == 0) s_n = 0;
     __syncthreads();
     for (int x = tid; x < cnt; x += blockDim.x) {
-      const float s = cs[x];
+      const float s = sc_at(x);
       if (s < lo) continue;
-      const unsigned long long key = cand_key(s, ci[x]);
+      const unsigned long long key = cand_key(s, id_at(x));
       if (key >= kth) {
         const int pos = atomicAdd(&s_n, 1);
         if (pos < kSelCap) skeys[pos] = key;
