@@ -197,7 +197,7 @@ __device__ __forceinline__ int next_pow2(int x) {
 // hold every candidate (a dense row), its softmax statistics come from that row, and
 // with one list per layer the row holds the head-averaged weights themselves.
 template <bool kGeneral, int kThreads>
-__global__ void __launch_bounds__(kThreads) k_select_t(const __grid_constant__ Batch B) {
+__global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __grid_constant__ Batch B) {
   constexpr int kSelCap = sel_cap<kThreads>();
   extern __shared__ unsigned long long skeys[];
   __shared__ int s_hist[kFineBins];
@@ -339,7 +339,7 @@ __global__ void __launch_bounds__(kThreads) k_select_t(const __grid_constant__ B
   if constexpr (!kGeneral) {
     // each thread loads 4 x 2 consecutive (score, id) slots per round (16-byte loads; the
     // list's slots start 256-byte aligned); a warp claims its output slots with one atomic
-    constexpr int kU = 4096 / kThreads;
+    constexpr int kU = 4;
     const float4* cp4 = reinterpret_cast<const float4*>(cp);
     const int n2p = (cnt + 1) >> 1;
     const float4 ninf = make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
@@ -380,7 +380,7 @@ __global__ void __launch_bounds__(kThreads) k_select_t(const __grid_constant__ B
   } else if (!dense) {
     // each thread loads 4 x 4 consecutive slots per round (16-byte loads; the list's slots
     // start 256-byte aligned); a warp claims the round's output slots with one atomic
-    constexpr int kU = 4096 / kThreads;
+    constexpr int kU = 4;
     const float4* cs4 = reinterpret_cast<const float4*>(cs);
     const int n4 = (cnt + 3) >> 2;
     const float4 ninf = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
@@ -583,6 +583,10 @@ cudaError_t launch_select_t(const Batch& B, int max_lists, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(k_select_t<kGeneral, kThreads>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
+  // all of the SM's unified memory as shared memory, so that two 512-thread lists fit
+  e = cudaFuncSetAttribute(k_select_t<kGeneral, kThreads>,
+                           cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+  if (e != cudaSuccess) return e;
   return launch_pdl(k_select_t<kGeneral, kThreads>, dim3(max_lists, B.n), dim3(kThreads),
                     (size_t)smem, s, B);
 }
@@ -668,9 +672,18 @@ __global__ void __launch_bounds__(1024) k_pool(const __grid_constant__ Batch B) 
   for (int x = tid; x < kVoteBins; x += blockDim.x) vh[x] = 0;
   if (tid == 0) s_c = 0;
   __syncthreads();
-  for (int u0 = 0; u0 < Uh; u0 += blockDim.x) {
-    const int u = u0 + tid;
-    const int b = u < Uh ? min(P.votes[u], kVoteBins - 1) : -1;
+  // every thread's units' votes are loaded at once and kept for step (2)
+  constexpr int kUnitsPerThread = kMaxHistUnits / 1024;
+  int vt[kUnitsPerThread];
+#pragma unroll
+  for (int q = 0; q < kUnitsPerThread; ++q) {
+    const int u = q * 1024 + tid;
+    vt[q] = u < Uh ? P.votes[u] : -1;
+  }
+#pragma unroll
+  for (int q = 0; q < kUnitsPerThread; ++q) {
+    if (q * 1024 >= Uh) break;
+    const int b = vt[q] >= 0 ? min(vt[q], kVoteBins - 1) : -1;
     const unsigned same = __match_any_sync(0xffffffffu, b);   // most units share a few levels
     if (b >= 0 && (__ffs(same) - 1) == (tid & 31)) atomicAdd(&vh[b], __popc(same));
   }
@@ -694,11 +707,13 @@ __global__ void __launch_bounds__(1024) k_pool(const __grid_constant__ Batch B) 
   // (2) the units at or above level V, ranked by (votes desc, mass desc, id asc)
   unsigned long long* ck = reinterpret_cast<unsigned long long*>(smem_raw);
   int* ci = reinterpret_cast<int*>(ck + kRankMax);
-  for (int u = tid; u < Uh; u += blockDim.x) {
-    if (min(P.votes[u], kVoteBins - 1) >= V) {
+#pragma unroll
+  for (int q = 0; q < kUnitsPerThread; ++q) {
+    const int u = q * 1024 + tid;
+    if (u < Uh && min(vt[q], kVoteBins - 1) >= V) {
       const int pos = atomicAdd(&s_c, 1);
       if (pos < kRankMax) {
-        ck[pos] = ((unsigned long long)(uint32_t)P.votes[u] << 32) | __float_as_uint(P.mass[u]);
+        ck[pos] = ((unsigned long long)(uint32_t)vt[q] << 32) | __float_as_uint(P.mass[u]);
         ci[pos] = u;
       }
     }
@@ -800,16 +815,31 @@ __global__ void __launch_bounds__(256) k_gram(const __grid_constant__ Batch B) {
   }
   __syncthreads();
   const int d4 = dim / 4;
-  for (int x = threadIdx.x; x < kGramTile * d4; x += blockDim.x) {
-    const int r = x / d4, e = 4 * (x - r * d4);
-    const float4 va = ua[r] >= 0 ? *reinterpret_cast<const float4*>(P.desc + (int64_t)ua[r] * dim + e)
-                                 : make_float4(0.f, 0.f, 0.f, 0.f);
-    const float4 vb = ub[r] >= 0 ? *reinterpret_cast<const float4*>(P.desc + (int64_t)ub[r] * dim + e)
-                                 : make_float4(0.f, 0.f, 0.f, 0.f);
-    float* pa = A + r * ld + e;
-    float* pb = Bm + r * ld + e;
-    pa[0] = va.x; pa[1] = va.y; pa[2] = va.z; pa[3] = va.w;
-    pb[0] = vb.x; pb[1] = vb.y; pb[2] = vb.z; pb[3] = vb.w;
+  // the rows' float4s, 4 + 4 per thread in flight before any is stored
+  constexpr int kB = 4;
+  for (int x0 = 0; x0 < kGramTile * d4; x0 += kB * blockDim.x) {
+    float4 va[kB], vb[kB];
+#pragma unroll
+    for (int q = 0; q < kB; ++q) {
+      const int x = x0 + q * blockDim.x + threadIdx.x;
+      const int r = x / d4, e = 4 * (x - r * d4);
+      const bool in = x < kGramTile * d4;
+      va[q] = in && ua[r] >= 0 ? *reinterpret_cast<const float4*>(P.desc + (int64_t)ua[r] * dim + e)
+                               : make_float4(0.f, 0.f, 0.f, 0.f);
+      vb[q] = in && ub[r] >= 0 ? *reinterpret_cast<const float4*>(P.desc + (int64_t)ub[r] * dim + e)
+                               : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int q = 0; q < kB; ++q) {
+      const int x = x0 + q * blockDim.x + threadIdx.x;
+      if (x < kGramTile * d4) {
+        const int r = x / d4, e = 4 * (x - r * d4);
+        float* pa = A + r * ld + e;
+        float* pb = Bm + r * ld + e;
+        pa[0] = va[q].x; pa[1] = va[q].y; pa[2] = va[q].z; pa[3] = va[q].w;
+        pb[0] = vb[q].x; pb[1] = vb[q].y; pb[2] = vb[q].z; pb[3] = vb[q].w;
+      }
+    }
   }
   __syncthreads();
   const int r = threadIdx.x / kGramTile, c = threadIdx.x % kGramTile;
