@@ -3,6 +3,8 @@
 Named to be collected last, so that it runs both after the rest of the GPU suite and,
 when selected alone, with the library's per-device set-up done by its own first call.
 """
+import gc
+
 import pytest
 import torch
 
@@ -53,12 +55,25 @@ def test_static_scratch_matches_workspace_entry_point_twice_in_a_row():
         refs.append(r)
     outs = [ss.Result(idx, p) for _ in range(3)]
     torch.cuda.synchronize()
-    before = (torch.cuda.memory_allocated(dev), torch.cuda.memory_reserved(dev))
-    # two calls in a row on the same question, then a call on another question
-    for out, j in zip(outs, (0, 0, 1)):
-        idx.retrieve_static(qs[j], p, out)
-    torch.cuda.synchronize()
-    assert (torch.cuda.memory_allocated(dev), torch.cuda.memory_reserved(dev)) == before
+
+    def allocations():
+        # cumulative count of device allocations made through torch (the binding's
+        # allocator too), and the memory torch holds: frees of earlier tests' tensors
+        # lower neither
+        st = torch.cuda.memory_stats(dev)
+        return st["allocation.all.allocated"], torch.cuda.memory_reserved(dev)
+
+    gc.collect()
+    gc.disable()
+    try:
+        before = allocations()
+        # two calls in a row on the same question, then a call on another question
+        for out, j in zip(outs, (0, 0, 1)):
+            idx.retrieve_static(qs[j], p, out)
+        torch.cuda.synchronize()
+        assert allocations() == before
+    finally:
+        gc.enable()
     for out, j in zip(outs, (0, 0, 1)):
         out.check()
         _same(out, refs[j], uh)
