@@ -218,7 +218,9 @@ def run_reference(args):
 # DRAM bytes of one k_score launch on the full 1-hour workload, from the 1-pass ncu
 # capture summarised in profiles/k_score_dram_traffic.md; valid only for the kernel
 # sources it was taken on (their sha256 below), reported as null otherwise.
-TRAFFIC_RECORD = {"workload": "hour1", "sources_sha256": None, "dram_bytes": None}
+TRAFFIC_RECORD = {"workload": "hour1",
+                  "sources_sha256": "deeb9d4c243fc9b5ba71e0da9c6d7ec1fd28368f191c341843c29aa7c7e38244",
+                  "dram_bytes": 2895287040 + 40795648}  # read + write
 SCORE_SOURCES = ("ss_score.cu", "ss_internal.cuh", "ss_device.cuh")
 
 
