@@ -104,7 +104,19 @@ __global__ void __launch_bounds__(256) k_sample(const __grid_constant__ Batch B)
     __syncthreads();
     const uint4* src = reinterpret_cast<const uint4*>(sk + (int64_t)rb * kHeadDim);
     uint4* dst = reinterpret_cast<uint4*>(kt);
-    for (int x = tid; x < nr * (kHeadDim / 8); x += blockDim.x) dst[x] = src[x];
+    // the pass's rows as 16-byte vectors, all of a thread's loads in flight at once
+    constexpr int kPerThread = kSampleRows * (kHeadDim / 8) / 256;
+    uint4 vbuf[kPerThread];
+#pragma unroll
+    for (int q = 0; q < kPerThread; ++q) {
+      const int x = q * 256 + tid;
+      if (x < nr * (kHeadDim / 8)) vbuf[q] = src[x];
+    }
+#pragma unroll
+    for (int q = 0; q < kPerThread; ++q) {
+      const int x = q * 256 + tid;
+      if (x < nr * (kHeadDim / 8)) dst[x] = vbuf[q];
+    }
     __syncthreads();
     // warp w scores rows [16 w, 16 w + 16) of this pass
     const int tr = kTileRows * warp;

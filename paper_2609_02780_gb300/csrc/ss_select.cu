@@ -258,23 +258,44 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
     if constexpr (kGeneral) return ci[x];
     else return __float_as_int(cp[x].y);
   };
+  // Visits every candidate x < cnt with its value: thread t takes x = t, t + T, ... in
+  // increasing order, loading four values before using them (loads in flight).
+  auto each = [&](auto&& f) {
+    for (int x0 = tid; x0 < cnt; x0 += 4 * (int)blockDim.x) {
+      float v[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int x = x0 + e * blockDim.x;
+        v[e] = x < cnt ? sc_at(x) : 0.f;
+      }
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int x = x0 + e * blockDim.x;
+        if (x < cnt) f(x, v[e]);
+      }
+    }
+  };
   float lo = -INFINITY;
   if constexpr (kGeneral) {
     // statistics of the dense row in a fixed order: (max, sum 2^(s - max)) of the
-    // scores, or (max, sum) of the head-averaged weights
-    float m = -INFINITY, l = 0.f;
+    // scores, or (max, sum) of the head-averaged weights; and its minimum (the bound)
+    float m = -INFINITY, l = 0.f, mn = INFINITY;
     if (mean) {
-      for (int x = tid; x < cnt; x += blockDim.x) {
-        const float v = cs[x];
+      each([&](int, float v) {
         m = fmaxf(m, v);
         l += v;
-      }
+        mn = fminf(mn, v);
+      });
       l = block_sum(l, s_l);
       m = -block_min(-m, s_m);
     } else {
-      for (int x = tid; x < cnt; x += blockDim.x) ml_combine(m, l, cs[x], 1.f);
+      each([&](int, float v) {
+        ml_combine(m, l, v, 1.f);
+        mn = fminf(mn, v);
+      });
       block_ml(m, l, s_m, s_l);
     }
+    lo = block_min(mn, s_m);
     M = m;
     Ls = l;
     if (tid == 0) P.list_ml[L] = make_float2(M, Ls);
@@ -325,10 +346,9 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
     // no bound: start from the smallest real candidate (unused reserved slots hold
     // -inf and are never candidates)
     float mn = INFINITY;
-    for (int x = tid; x < cnt; x += blockDim.x) {
-      const float s = sc_at(x);
+    each([&](int, float s) {
       if (s > -INFINITY) mn = fminf(mn, s);
-    }
+    });
     lo = block_min(mn, s_m);
   }
   // A dense row of more than 2048 candidates goes straight to the histogram below.
@@ -438,10 +458,9 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
     };
     for (int x = tid; x < kFineBins; x += blockDim.x) s_hist[x] = 0;
     __syncthreads();
-    for (int x = tid; x < cnt; x += blockDim.x) {
-      const float s = sc_at(x);
+    each([&](int, float s) {
       if (s >= lo) atomicAdd(&s_hist[fbin(s)], 1);
-    }
+    });
     __syncthreads();
     if (tid < 32) {
       constexpr int per = kFineBins / 32;  // lane 0 holds the top bins
@@ -473,13 +492,12 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
     const int bstar = s_bstar;
     if (bstar < 0 && tid == 0) atomicOr(P.status, kStatusInternal);
     const int bmin = max(bstar, 0);
-    for (int x = tid; x < cnt; x += blockDim.x) {
-      const float s = sc_at(x);
+    each([&](int x, float s) {
       if (s >= lo && fbin(s) >= bmin) {
         const int pos = atomicAdd(&s_n, 1);
         if (pos < kSelCap) skeys[pos] = cand_key(s, id_at(x));
       }
-    }
+    });
     __syncthreads();
     ns = s_n;
   }
@@ -721,13 +739,29 @@ __global__ void __launch_bounds__(1024) k_pool(const __grid_constant__ Batch B) 
   __syncthreads();
   const int C = s_c;
   if (C <= kRankMax) {
-    if (tid < C) {
-      const unsigned long long mk = ck[tid];
-      const int mi = ci[tid];
-      int rank = 0;
-      for (int o = 0; o < C; ++o) rank += unit_before(ck[o], ci[o], mk, mi) ? 1 : 0;
-      if (rank < pn) P.pool[rank] = mi;
+    // rank = the number of candidates ordered before; the block's threads split the
+    // comparisons: thread t counts for candidate t % C over part t / C of the others
+    int* rk = reinterpret_cast<int*>(ci + kRankMax);
+    for (int x = tid; x < C; x += blockDim.x) rk[x] = 0;
+    __syncthreads();
+    const int parts = max(1, (int)blockDim.x / max(C, 1));
+    const int i = tid % max(C, 1), part = tid / max(C, 1);
+    if (C > 0 && part < parts) {
+      const unsigned long long mk = ck[i];
+      const int mi = ci[i];
+      const int o0 = (int)(((int64_t)C * part) / parts), o1 = (int)(((int64_t)C * (part + 1)) / parts);
+      int r[4] = {0, 0, 0, 0};  // independent partial counts keep the loads in flight
+      int o = o0;
+      for (; o + 4 <= o1; o += 4) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) r[e] += unit_before(ck[o + e], ci[o + e], mk, mi) ? 1 : 0;
+      }
+      for (; o < o1; ++o) r[0] += unit_before(ck[o], ci[o], mk, mi) ? 1 : 0;
+      atomicAdd(&rk[i], r[0] + r[1] + r[2] + r[3]);
     }
+    __syncthreads();
+    for (int x = tid; x < C; x += blockDim.x)
+      if (rk[x] < pn) P.pool[rk[x]] = ci[x];
     return;
   }
   // (3) too many ties at level V: sort every history unit
@@ -770,7 +804,8 @@ __global__ void __launch_bounds__(1024) k_pool(const __grid_constant__ Batch B) 
 cudaError_t launch_pool(const Batch& B, int max_hist_units, cudaStream_t s) {
   int n2 = 1;
   while (n2 < max_hist_units) n2 <<= 1;
-  const int smem = max(n2, kRankMax) * (int)(sizeof(unsigned long long) + sizeof(int));
+  const int smem = max(n2, kRankMax) * (int)(sizeof(unsigned long long) + sizeof(int)) +
+                   kRankMax * (int)sizeof(int);
   cudaError_t e = cudaFuncSetAttribute(k_pool, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   return launch_pdl(k_pool, dim3(B.n), dim3(1024), (size_t)smem, s, B);
@@ -843,8 +878,12 @@ __global__ void __launch_bounds__(256) k_gram(const __grid_constant__ Batch B) {
   }
   __syncthreads();
   const int r = threadIdx.x / kGramTile, c = threadIdx.x % kGramTile;
-  float acc = 0.f;
-  for (int d = 0; d < dim; ++d) acc = fmaf(A[r * ld + d], Bm[c * ld + d], acc);
+  float a4[4] = {0.f, 0.f, 0.f, 0.f};  // four independent FMA chains (dim % 4 == 0)
+  for (int d = 0; d < dim; d += 4) {
+#pragma unroll
+    for (int e = 0; e < 4; ++e) a4[e] = fmaf(A[r * ld + d + e], Bm[c * ld + d + e], a4[e]);
+  }
+  const float acc = (a4[0] + a4[1]) + (a4[2] + a4[3]);
   const int a = ta * kGramTile + r, b = tb * kGramTile + c;
   if (a < pn && b < pn && a <= b) P.gram[tri_off(a, pn) + (b - a)] = acc;
 }
