@@ -165,3 +165,31 @@ def test_general_path_errors():
     idx.compress(4, n_centroids=8, iters=2)
     with pytest.raises(ss.ShallowStreamError, match="UNSUPPORTED"):
         idx.retrieve(q.cuda(), k=5, budget=2, use_clusters=1, head_agg=ss.H_MEAN)
+
+
+def test_general_path_batched_equals_single():
+    # one launch per stage over problems of different lengths and compression states
+    ss = _ss()
+    for mode in ("mean", "clusters"):
+        idxs, qs = [], []
+        for j, F in enumerate((40, 64, 24)):
+            keys, q = _keys_q(40 + j, P=2, Hq=8, Hkv=2, F=F, Tf=20, scene=4)
+            ix = ss.Index(2, 8, 2, 20, F, device="cuda")
+            ix.append(keys.cuda())
+            if mode == "clusters":
+                ix.compress(4, n_centroids=8, iters=2, first_frame=0, n_frames=(F // 2) // 4 * 4)
+            idxs.append(ix)
+            qs.append(q.cuda())
+        p = ss.RetrieveParams(k=30, budget=4, n_recent=1,
+                              head_agg=ss.H_MEAN if mode == "mean" else ss.H_PER_QHEAD,
+                              use_clusters=1 if mode == "clusters" else 0)
+        batched = ss.retrieve_batched(idxs, qs, p)
+        for ix, q, rb in zip(idxs, qs, batched):
+            rs = ix.retrieve(q, k=p.k, budget=p.budget, n_recent=p.n_recent,
+                             head_agg=p.head_agg, use_clusters=p.use_clusters)
+            uh = ix.n_units - p.n_recent
+            for name in ("topk_tok", "topk_w", "list_stats", "counts"):
+                assert torch.equal(getattr(rb, name), getattr(rs, name)), (mode, name)
+            assert torch.equal(rb.unit_votes[:uh], rs.unit_votes[:uh]), mode
+            assert torch.equal(rb.unit_mass[:uh], rs.unit_mass[:uh]), mode
+            assert rb.host() == rs.host(), mode
