@@ -202,7 +202,8 @@ cudaError_t launch_prep(const Batch& B, cudaStream_t s) {
 // Each unit's softmax statistics (max, sum 2^(s - max)) are written per list; the
 // list totals are combined later in unit order, whichever warp scored a unit.
 // ---------------------------------------------------------------------------
-constexpr int kUnitQueue = 8;  // > units a warp's issue cursor can run ahead
+constexpr int kUnitQueue = 8;
+constexpr int kStagePairs = 16;  // staged candidates per (warp, list) before a write-out  // > units a warp's issue cursor can run ahead
 
 struct ScoreShared {
   int lad[kMaxGroup][kLadderLevels];  // this CTA's appended-score counts not yet merged
@@ -211,6 +212,8 @@ struct ScoreShared {
   int all_done;
   unsigned long long bar[kScoreWarps][kScoreStages];  // one mbarrier per warp stage
   int uq[kScoreWarps][kUnitQueue];      // per warp: units taken, in order
+  // per warp and list: appended (score, id) pairs waiting to be written out together
+  float2 stage[kScoreWarps][kMaxGroup][kStagePairs];
 };
 
 // One column (query head) of a tile: online (max, sum 2^(s - max)) over valid rows.
@@ -388,6 +391,40 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
 
   // Appends the scores of keys tok0 (row g) and tok0 + 8 (row g + 8) that reach the
   // current thresholds, and counts them in the CTA's ladder.
+  // Staged pairs of this lane group's two lists (counts identical in its 8 lanes).
+  int sc0 = 0, sc1 = 0;
+  // Writes the staged pairs of every lane group to their lists' reserved slots (8 lanes
+  // store 64 contiguous bytes at a time), reserving a new slot block when one runs out.
+  // The whole warp calls it.
+  auto flush = [&]() {
+    __syncwarp();
+    const bool need0 = sc0 > rl0, need1 = sc1 > rl1;
+    int nb0 = 0, nb1 = 0;
+    if (g == 0 && need0) nb0 = atomicAdd(P.cand_cnt + L0, kReserve);
+    if (g == 0 && need1) nb1 = atomicAdd(P.cand_cnt + L1, kReserve);
+    nb0 = __shfl_sync(0xffffffffu, nb0, t4);
+    nb1 = __shfl_sync(0xffffffffu, nb1, t4);
+    for (int r = g; r < sc0; r += 8)
+      P.cand_pair[cbase0 + (r < rl0 ? rp0 + r : nb0 + (r - rl0))] = S.stage[warp][c0][r];
+    for (int r = g; r < sc1; r += 8)
+      P.cand_pair[cbase1 + (r < rl1 ? rp1 + r : nb1 + (r - rl1))] = S.stage[warp][c1][r];
+    if (need0) {
+      rp0 = nb0 + (sc0 - rl0);
+      rl0 = kReserve - (sc0 - rl0);
+    } else {
+      rp0 += sc0;
+      rl0 -= sc0;
+    }
+    if (need1) {
+      rp1 = nb1 + (sc1 - rl1);
+      rl1 = kReserve - (sc1 - rl1);
+    } else {
+      rp1 += sc1;
+      rl1 -= sc1;
+    }
+    sc0 = sc1 = 0;
+    __syncwarp();
+  };
   auto append = [&](float s00, float s01, float s10, float s11, int tok0, bool v0, bool v1,
                     float thr0, float thr1) {
     const bool p00 = hv0 && v0 && s00 >= thr0, p10 = hv0 && v1 && s10 >= thr0;
@@ -398,49 +435,27 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
     const unsigned b01 = __ballot_sync(0xffffffffu, p01) & gmask;
     const unsigned b11 = __ballot_sync(0xffffffffu, p11) & gmask;
     const int n0 = __popc(b00) + __popc(b10), n1 = __popc(b01) + __popc(b11);
-    // slots: continue the reserved block, reserve a new one when it runs out
-    const bool need0 = n0 > rl0, need1 = n1 > rl1;
-    int nb0 = 0, nb1 = 0;
-    if (g == 0 && need0) nb0 = atomicAdd(P.cand_cnt + L0, kReserve);
-    if (g == 0 && need1) nb1 = atomicAdd(P.cand_cnt + L1, kReserve);
-    nb0 = __shfl_sync(0xffffffffu, nb0, t4);
-    nb1 = __shfl_sync(0xffffffffu, nb1, t4);
-    auto slot0 = [&](int r) { return cbase0 + (r < rl0 ? rp0 + r : nb0 + (r - rl0)); };
-    auto slot1 = [&](int r) { return cbase1 + (r < rl1 ? rp1 + r : nb1 + (r - rl1)); };
+    if (__any_sync(0xffffffffu, sc0 + n0 > kStagePairs || sc1 + n1 > kStagePairs)) flush();
     if (p00) {
-      const int64_t pos = slot0(__popc(b00 & lt_mask));
-      P.cand_pair[pos] = make_float2(s00, __int_as_float(tok0));
+      S.stage[warp][c0][sc0 + __popc(b00 & lt_mask)] = make_float2(s00, __int_as_float(tok0));
       ladder_add(S, c0, s00, an0);
     }
     if (p10) {
-      const int64_t pos = slot0(__popc(b00) + __popc(b10 & lt_mask));
-      P.cand_pair[pos] = make_float2(s10, __int_as_float(tok1));
+      S.stage[warp][c0][sc0 + __popc(b00) + __popc(b10 & lt_mask)] =
+          make_float2(s10, __int_as_float(tok1));
       ladder_add(S, c0, s10, an0);
     }
     if (p01) {
-      const int64_t pos = slot1(__popc(b01 & lt_mask));
-      P.cand_pair[pos] = make_float2(s01, __int_as_float(tok0));
+      S.stage[warp][c1][sc1 + __popc(b01 & lt_mask)] = make_float2(s01, __int_as_float(tok0));
       ladder_add(S, c1, s01, an1);
     }
     if (p11) {
-      const int64_t pos = slot1(__popc(b01) + __popc(b11 & lt_mask));
-      P.cand_pair[pos] = make_float2(s11, __int_as_float(tok1));
+      S.stage[warp][c1][sc1 + __popc(b01) + __popc(b11 & lt_mask)] =
+          make_float2(s11, __int_as_float(tok1));
       ladder_add(S, c1, s11, an1);
     }
-    if (need0) {
-      rp0 = nb0 + (n0 - rl0);
-      rl0 = kReserve - (n0 - rl0);
-    } else {
-      rp0 += n0;
-      rl0 -= n0;
-    }
-    if (need1) {
-      rp1 = nb1 + (n1 - rl1);
-      rl1 = kReserve - (n1 - rl1);
-    } else {
-      rp1 += n1;
-      rl1 -= n1;
-    }
+    sc0 += n0;
+    sc1 += n1;
   };
 
   // Lane 0 starts the bulk copy of tile t (unit uu, tile jj of the unit) into its
@@ -556,6 +571,7 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
       }
     }
   }
+  flush();
   // unused reserved slots are marked empty (score -inf)
   for (int x = g; x < rl0; x += 8) P.cand_pair[cbase0 + rp0 + x].x = -INFINITY;
   for (int x = g; x < rl1; x += 8) P.cand_pair[cbase1 + rp1 + x].x = -INFINITY;
