@@ -219,8 +219,8 @@ def run_reference(args):
 # capture summarised in profiles/k_score_dram_traffic.md; valid only for the kernel
 # sources it was taken on (their sha256 below), reported as null otherwise.
 TRAFFIC_RECORD = {"workload": "hour1",
-                  "sources_sha256": "deeb9d4c243fc9b5ba71e0da9c6d7ec1fd28368f191c341843c29aa7c7e38244",
-                  "dram_bytes": 2895287040 + 40795648}  # read + write
+                  "sources_sha256": "ea4b862881ead41678505adfd48da72db6f93ed1947de6956b929c715284732a",
+                  "dram_bytes": 2893158144 + 29731328}  # read + write
 SCORE_SOURCES = ("ss_score.cu", "ss_internal.cuh", "ss_device.cuh")
 
 
