@@ -391,13 +391,15 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
 
   // Appends the scores of keys tok0 (row g) and tok0 + 8 (row g + 8) that reach the
   // current thresholds, and counts them in the CTA's ladder.
-  // Staged pairs of this lane group's two lists (counts identical in its 8 lanes).
-  int sc0 = 0, sc1 = 0;
+  // Staged pairs of this lane group's two lists (counts identical in its 8 lanes),
+  // packed as sc0 | sc1 << 8.
+  int scp = 0;
   // Writes the staged pairs of every lane group to their lists' reserved slots (8 lanes
   // store 64 contiguous bytes at a time), reserving a new slot block when one runs out.
   // The whole warp calls it.
   auto flush = [&]() {
     __syncwarp();
+    const int sc0 = scp & 0xff, sc1 = scp >> 8;
     const bool need0 = sc0 > rl0, need1 = sc1 > rl1;
     int nb0 = 0, nb1 = 0;
     if (g == 0 && need0) nb0 = atomicAdd(P.cand_cnt + L0, kReserve);
@@ -422,7 +424,7 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
       rp1 += sc1;
       rl1 -= sc1;
     }
-    sc0 = sc1 = 0;
+    scp = 0;
     __syncwarp();
   };
   auto append = [&](float s00, float s01, float s10, float s11, int tok0, bool v0, bool v1,
@@ -435,7 +437,9 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
     const unsigned b01 = __ballot_sync(0xffffffffu, p01) & gmask;
     const unsigned b11 = __ballot_sync(0xffffffffu, p11) & gmask;
     const int n0 = __popc(b00) + __popc(b10), n1 = __popc(b01) + __popc(b11);
-    if (__any_sync(0xffffffffu, sc0 + n0 > kStagePairs || sc1 + n1 > kStagePairs)) flush();
+    if (__any_sync(0xffffffffu, (scp & 0xff) + n0 > kStagePairs || (scp >> 8) + n1 > kStagePairs))
+      flush();
+    const int sc0 = scp & 0xff, sc1 = scp >> 8;
     if (p00) {
       S.stage[warp][c0][sc0 + __popc(b00 & lt_mask)] = make_float2(s00, __int_as_float(tok0));
       ladder_add(S, c0, s00, an0);
@@ -454,8 +458,7 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
           make_float2(s11, __int_as_float(tok1));
       ladder_add(S, c1, s11, an1);
     }
-    sc0 += n0;
-    sc1 += n1;
+    scp += n0 + (n1 << 8);
   };
 
   // Lane 0 starts the bulk copy of tile t (unit uu, tile jj of the unit) into its
