@@ -239,22 +239,38 @@ __device__ __forceinline__ void ladder_add(ScoreShared& S, int c, float s, float
 // derives from those the lower bound thr of each list's k-th best score: if the
 // levels >= i hold at least k appended tokens (of any CTA), the k-th best score is at
 // least level i's lower edge. One level of margin covers the rounding of the level
-// computation.
-__device__ void threshold_warp(ScoreShared& S, const Prob& P, int list0, int k) {
-  constexpr int per = kLadderLevels / 32;  // levels per lane; lane 0 holds the top ones
+// computation. Lane l handles the levels 255 - (32 q + l), q = 0..7, so that a warp's
+// accesses to one block of 32 levels are consecutive words (no shared-memory bank
+// conflicts, one 128-byte global transaction).
+__device__ __noinline__ void threshold_warp(ScoreShared& S, const Prob& P, int list0, int k) {
+  constexpr int per = kLadderLevels / 32;  // blocks of 32 levels; block 0 the top ones
   const int lane = threadIdx.x & 31;
   const int G = P.G;
   volatile int* vdone = &S.all_done;
   volatile float* vthr = S.thr;
+  auto level = [&](int q) { return kLadderLevels - 1 - (32 * q + lane); };
   for (int iter = 0; iter < (1 << 21); ++iter) {
     const int done = *vdone;
-    for (int c = 0; c < G; ++c) {
-      int* gl = P.ladder + (int64_t)(list0 + c) * kLadderLevels;
+    // the bounds other CTAs published (lane c holds list c's), in flight while merging
+    const float pub = lane < G ? ordered_to_float(*(volatile uint32_t*)(P.gthr + list0 + lane))
+                               : -INFINITY;
+    // merge this CTA's new counts into the global ladder, 2 lists at a time: all the
+    // exchanges first, then the additions (no atomic result is waited for)
 #pragma unroll
-      for (int q = 0; q < per; ++q) {
-        const int lv = kLadderLevels - 1 - (per * lane + q);
-        const int dv = atomicExch(&S.lad[c][lv], 0);
-        if (dv) atomicAdd(gl + lv, dv);
+    for (int c0 = 0; c0 < kMaxGroup; c0 += 2) {
+      int dv[2][per];
+#pragma unroll
+      for (int cc = 0; cc < 2; ++cc) {
+#pragma unroll
+        for (int q = 0; q < per; ++q)
+          dv[cc][q] = c0 + cc < G ? atomicExch(&S.lad[c0 + cc][level(q)], 0) : 0;
+      }
+#pragma unroll
+      for (int cc = 0; cc < 2; ++cc) {
+        int* gl = P.ladder + (int64_t)(list0 + c0 + cc) * kLadderLevels;
+#pragma unroll
+        for (int q = 0; q < per; ++q)
+          if (dv[cc][q]) atomicAdd(gl + level(q), dv[cc][q]);
       }
     }
     // the global counts of 4 lists per round trip
@@ -267,42 +283,42 @@ __device__ void threshold_warp(ScoreShared& S, const Prob& P, int list0, int k) 
         const int c = c0 + cc;
         const volatile int* gl = P.ladder + (int64_t)(list0 + (c < G ? c : 0)) * kLadderLevels;
 #pragma unroll
-        for (int q = 0; q < per; ++q)
-          cnt[cc][q] = c < G ? gl[kLadderLevels - 1 - (per * lane + q)] : 0;
+        for (int q = 0; q < per; ++q) cnt[cc][q] = c < G ? gl[level(q)] : 0;
       }
 #pragma unroll
       for (int cc = 0; cc < 4; ++cc) {
         const int c = c0 + cc;
         if (c >= G) break;
-        int sum = 0;
+        // the first block of 32 levels where the count from the top reaches k, then the
+        // first level inside it
+        int above = 0, qf = -1;
 #pragma unroll
-        for (int q = 0; q < per; ++q) sum += cnt[cc][q];
-        int cum = sum;
-#pragma unroll
-        for (int off = 1; off < 32; off <<= 1) {
-          const int y = __shfl_up_sync(0xffffffffu, cum, off);
-          if (lane >= off) cum += y;
+        for (int q = 0; q < per; ++q) {
+          const int tq = __reduce_add_sync(0xffffffffu, (unsigned)cnt[cc][q]);
+          if (qf < 0 && above + tq >= k) qf = q;
+          if (qf < 0) above += tq;
         }
-        const unsigned hit = __ballot_sync(0xffffffffu, cum >= k);
-        if (hit) {
-          const int f = __ffs(hit) - 1;
-          if (lane == f) {
-            int run = cum - sum, qf = per - 1;
+        float t = -INFINITY;
+        if (qf >= 0) {
+          int mine = 0;
 #pragma unroll
-            for (int q = 0; q < per; ++q) {
-              run += cnt[cc][q];
-              if (run >= k && qf == per - 1 && q < per - 1) qf = q;
-            }
-            const int lv = kLadderLevels - 1 - (per * lane + qf);
-            float t = S.anchor[c] + (float)(lv - kLadderZero - 1) / kLadderPerUnit;
-            const uint32_t old = atomicMax(P.gthr + list0 + c, float_to_ordered(t));
-            t = fmaxf(t, ordered_to_float(old));
-            if (t > vthr[c]) vthr[c] = t;
+          for (int q = 0; q < per; ++q)
+            if (q == qf) mine = cnt[cc][q];
+          int cum = mine;
+#pragma unroll
+          for (int off = 1; off < 32; off <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, cum, off);
+            if (lane >= off) cum += y;
           }
-        } else if (lane == 0) {
-          const float t = ordered_to_float(*(volatile uint32_t*)(P.gthr + list0 + c));
-          if (t > vthr[c]) vthr[c] = t;
+          const unsigned hit = __ballot_sync(0xffffffffu, above + cum >= k);
+          const int f = __ffs(hit) - 1;
+          const int lv = kLadderLevels - 1 - (32 * qf + f);
+          t = S.anchor[c] + (float)(lv - kLadderZero - 1) / kLadderPerUnit;
+          if (lane == 0) atomicMax(P.gthr + list0 + c, float_to_ordered(t));  // not waited for
         }
+        const float other = __shfl_sync(0xffffffffu, pub, c);
+        t = fmaxf(t, other);
+        if (lane == 0 && t > vthr[c]) vthr[c] = t;
       }
     }
     __syncwarp();
