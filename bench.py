@@ -219,8 +219,8 @@ def run_reference(args):
 # capture summarised in profiles/k_score_dram_traffic.md; valid only for the kernel
 # sources it was taken on (their sha256 below), reported as null otherwise.
 TRAFFIC_RECORD = {"workload": "hour1",
-                  "sources_sha256": "ea4b862881ead41678505adfd48da72db6f93ed1947de6956b929c715284732a",
-                  "dram_bytes": 2893158144 + 29731328}  # read + write
+                  "sources_sha256": "35317f499ce0eb6a4afcefec55c6d33c25041cda68ff03619a611536d2715fa5",
+                  "dram_bytes": 2893401344 + 30992640}  # read + write
 SCORE_SOURCES = ("ss_score.cu", "ss_internal.cuh", "ss_device.cuh")
 
 
