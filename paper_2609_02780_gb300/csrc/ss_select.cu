@@ -824,6 +824,47 @@ constexpr int kGramTile = 16;
 
 __device__ __forceinline__ int tri_off(int a, int pn) { return a * pn - (a * (a - 1)) / 2; }
 
+// Storage of the triangle (total = pn (pn + 1) / 2 entries) in the workspace: fp32 up to
+// kMaxMinSmemPool ranks (staged whole into shared memory by k_maxmin), 24-bit fixed
+// point up to kMaxMinFixedPool ranks (also staged: the 16 high bits of every entry from
+// the region's start, the 8 low bits from the next 16-byte boundary; 2^-22 steps, far
+// below the fp32 Gram's own rounding at the distances compared), fp32 read from global
+// memory beyond.
+constexpr int kMaxMinSmemPool = 320;
+constexpr int kMaxMinFixedPool = 384;
+__host__ __device__ __forceinline__ int round16(int bytes) { return (bytes + 15) & ~15; }
+__host__ __device__ __forceinline__ int tri_entries(int pn) { return pn * (pn + 1) / 2; }
+__host__ __device__ __forceinline__ bool gram_fixed24(int pn) {
+  return pn > kMaxMinSmemPool && pn <= kMaxMinFixedPool;
+}
+// bytes of the triangle that k_maxmin copies into shared memory
+__host__ __device__ __forceinline__ int gram_stage_bytes(int pn) {
+  if (pn <= kMaxMinSmemPool) return round16(4 * tri_entries(pn));
+  if (pn <= kMaxMinFixedPool) return round16(2 * tri_entries(pn)) + round16(tri_entries(pn));
+  return 0;
+}
+// pool ranks per lane of the greedy (its instantiation) for a pool of pn ranks
+__host__ __device__ __forceinline__ int maxmin_per(int pn) {
+  const int need = (pn + 31) / 32;
+  if (pn <= kMaxMinSmemPool) return need <= 1 ? 1 : need <= 2 ? 2 : need <= 4 ? 4 : need <= 8 ? 8 : 16;
+  if (pn <= kMaxMinFixedPool) return 12;
+  return need <= 16 ? 16 : 32;
+}
+// Entries of the triangle's storage that the greedy reads: the row of rank b is read at
+// tri_off(b) - b + c for every lane rank c >= b, so the ranks past the pool (c up to
+// 32 maxmin_per - 1) reach past the triangle's end (values never used).
+__host__ __device__ __forceinline__ int maxmin_reach(int pn) {
+  return tri_entries(pn) - pn + 32 * maxmin_per(pn);
+}
+// shared-memory bytes k_maxmin needs for a pool of pn ranks: the staged triangle and
+// the reads past it (fixed point: the high parts' reads past end inside the low part)
+__host__ __device__ __forceinline__ int gram_smem_bytes(int pn) {
+  const int t = tri_entries(pn), r = maxmin_reach(pn);
+  if (pn <= kMaxMinSmemPool) return round16(4 * (r > t ? r : t));
+  if (pn <= kMaxMinFixedPool) return round16(2 * t) + round16(r > t ? r : t);
+  return 0;
+}
+
 __global__ void __launch_bounds__(256) k_gram(const __grid_constant__ Batch B) {
   extern __shared__ float gsm[];
   pdl_wait();
@@ -885,16 +926,23 @@ __global__ void __launch_bounds__(256) k_gram(const __grid_constant__ Batch B) {
   }
   const float acc = (a4[0] + a4[1]) + (a4[2] + a4[3]);
   const int a = ta * kGramTile + r, b = tb * kGramTile + c;
-  if (a < pn && b < pn && a <= b) P.gram[tri_off(a, pn) + (b - a)] = acc;
+  if (a < pn && b < pn && a <= b) {
+    const int x = tri_off(a, pn) + (b - a);
+    if (gram_fixed24(pn)) {
+      uint8_t* g8 = reinterpret_cast<uint8_t*>(P.gram);
+      const int v = __float2int_rn(fminf(fmaxf(acc, -1.99f), 1.99f) * 4194304.0f);
+      reinterpret_cast<uint16_t*>(g8)[x] = (uint16_t)((uint32_t)v >> 8);
+      g8[round16(2 * tri_entries(pn)) + x] = (uint8_t)((uint32_t)v & 0xffu);
+    } else {
+      P.gram[x] = acc;
+    }
+  }
 }
 
 // Greedy max-min (DivTopK) by one warp over the packed Gram triangle, then the
-// expansion (Nbr of Eq. 12) by the whole block. Lane l owns the pool ranks l, l + 32,
-// ...; kPer = ranks per lane. The triangle sits in shared memory as fp32 up to 320
-// ranks (201 KB), as 24-bit fixed point (2^-22 steps, far below the fp32 Gram's own
-// rounding at the distances compared) up to 384 ranks (222 KB), else in global memory.
-constexpr int kMaxMinSmemPool = 320;
-constexpr int kMaxMinFixedPool = 384;
+// expansion (Nbr of Eq. 12). Lane l owns the pool ranks l, l + 32, ...; kPer = ranks
+// per lane. The triangle sits in shared memory as fp32 up to 320 ranks (201 KB), as
+// 24-bit fixed point up to 384 ranks (222 KB), else in global memory.
 constexpr int kMaxMinThreads = kMaxHistUnits / 32;  // one bitmap word per thread
 
 struct TriF32 {  // fp32 triangle (shared or global memory)
@@ -911,8 +959,7 @@ struct TriFix24 {  // 24-bit fixed point split into 16 high and 8 low bits
 };
 
 template <int kPer, class Tri>
-__device__ void greedy_maxmin(const Prob& P, const Tri pk, const int* pool, int* sel,
-                              int pn, int ns) {
+__device__ void greedy_maxmin(const Prob& P, const Tri pk, int* sel, int pn, int ns) {
   const int lane = threadIdx.x & 31;
   float mind[kPer];
   int toff[kPer];  // start of candidate c's row in the packed triangle
@@ -923,7 +970,7 @@ __device__ void greedy_maxmin(const Prob& P, const Tri pk, const int* pool, int*
     mind[q] = c < pn ? 1.0f - pk(c) : -INFINITY;  // row 0 of the triangle is G[0][*]
   }
   uint32_t taken = lane == 0 ? 1u : 0u;  // bit q: rank lane + 32 q is picked
-  if (lane == 0) sel[0] = pool[0];
+  if (lane == 0) sel[0] = 0;
   for (int step = 1; step < ns; ++step) {
     // best distance over the unpicked ranks, then the smallest rank holding it; distances
     // are >= 0 (or NaN, which ranks last), so their bit patterns order as unsigned ints
@@ -958,18 +1005,20 @@ __device__ void greedy_maxmin(const Prob& P, const Tri pk, const int* pool, int*
       return;
     }
     if ((best & 31) == lane) taken |= 1u << (best >> 5);
-    if (lane == 0) sel[step] = pool[best];
+    if (lane == 0) sel[step] = best;  // a pool rank; mapped to its unit afterwards
     // row best of the triangle: ranks >= best are contiguous, ranks < best sit in
     // column best of their own rows
+    // all loads of the row are issued before any is used; ranks past the pool read
+    // past the triangle (storage sized by maxmin_reach), their distance stays -inf
     const int rowoff = tri_off(best, pn) - best;
+    float g[kPer];
 #pragma unroll
     for (int q = 0; q < kPer; ++q) {
       const int c = lane + 32 * q;
-      if (c < pn) {
-        const float g = pk(c >= best ? rowoff + c : toff[q] + best - c);
-        mind[q] = fminf(mind[q], 1.0f - g);
-      }
+      g[q] = pk(c >= best ? rowoff + c : toff[q] + best - c);
     }
+#pragma unroll
+    for (int q = 0; q < kPer; ++q) mind[q] = fminf(mind[q], 1.0f - g[q]);
   }
 }
 
@@ -978,60 +1027,76 @@ __global__ void __launch_bounds__(kMaxMinThreads) k_maxmin(const __grid_constant
   __shared__ uint32_t bits[kMaxHistUnits / 32];
   __shared__ int spool[kMaxPool];
   __shared__ int ssel[kMaxPool];
+  __shared__ __align__(8) uint64_t tri_bar;
   pdl_wait();
   pdl_release();
   const Prob& P = B.p[blockIdx.x];
   const int pn = P.pool_n, ns = P.n_sel;
   const int tid = threadIdx.x, warp = tid >> 5;
   const bool in_smem = pn <= kMaxMinSmemPool;
-  const bool fixed24 = !in_smem && pn <= kMaxMinFixedPool;
-  const int total = tri_off(pn, pn);
-  uint16_t* fhi = reinterpret_cast<uint16_t*>(pks4);
-  uint8_t* flo = reinterpret_cast<uint8_t*>(fhi + total);
-  for (int x = tid; x < pn; x += blockDim.x) spool[x] = P.pool[x];
-  if (in_smem) {
-    const int total4 = (total + 3) / 4;
-    const float4* g4 = reinterpret_cast<const float4*>(P.gram);
-    for (int x = tid; x < total4; x += blockDim.x) pks4[x] = g4[x];
-  } else if (fixed24) {
-    for (int x = tid; x < total; x += blockDim.x) {
-      const float g = fminf(fmaxf(P.gram[x], -1.99f), 1.99f);
-      const int v = __float2int_rn(g * 4194304.0f);
-      fhi[x] = (uint16_t)((uint32_t)v >> 8);
-      flo[x] = (uint8_t)((uint32_t)v & 0xffu);
+  const bool fixed24 = gram_fixed24(pn);
+  const int hi_bytes = round16(2 * tri_entries(pn));
+  const uint16_t* fhi = reinterpret_cast<const uint16_t*>(pks4);
+  const uint8_t* flo = reinterpret_cast<const uint8_t*>(pks4) + hi_bytes;
+  // one thread stages the triangle with bulk copies (both parts of the fixed-point form
+  // lie at 16-byte boundaries; the rounded-up tails stay inside the workspace region)
+  const bool staged = ns > 0 && (in_smem || fixed24);
+  const uint32_t bar = smem_u32(&tri_bar);
+  if (staged && tid == 0) {
+    mbar_init(bar, 1u);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    const uint8_t* g8 = reinterpret_cast<const uint8_t*>(P.gram);
+    mbar_expect_tx(bar, (uint32_t)gram_stage_bytes(pn));
+    if (in_smem) {
+      bulk_load(smem_u32(pks4), g8, (uint32_t)round16(4 * tri_entries(pn)), bar);
+    } else {
+      bulk_load(smem_u32(pks4), g8, (uint32_t)hi_bytes, bar);
+      bulk_load(smem_u32(flo), g8 + hi_bytes, (uint32_t)round16(tri_entries(pn)), bar);
     }
   }
+  for (int x = tid; x < pn; x += blockDim.x) spool[x] = P.pool[x];
+  const int Uh = P.Uh;
+  const int nwords = (Uh + 31) >> 5;
+  for (int x = tid; x < nwords; x += blockDim.x) bits[x] = 0u;
   __syncthreads();
   // One warp does the rest: warps parked at a barrier would slow its serial greedy.
   if (warp != 0) return;
   const int lane = tid;
+  if (staged && !mbar_wait_bounded(bar, 0u)) {
+    // report, then let the copies in flight land before the CTA exits
+    if (lane == 0) atomicOr(P.status, kStatusTimeout);
+    mbar_wait_bounded(bar, 0u);
+    return;
+  }
   if (ns > 0) {
     // separate call sites keep the triangle's address space (shared or global) known
     // to the compiler, so the greedy's reads are plain shared-memory loads when staged
-    const int per = (pn + 31) / 32;
+    const int per = maxmin_per(pn);
     if (in_smem) {
       const TriF32 sk{reinterpret_cast<const float*>(pks4)};
-      if (per <= 1) greedy_maxmin<1>(P, sk, spool, ssel, pn, ns);
-      else if (per <= 2) greedy_maxmin<2>(P, sk, spool, ssel, pn, ns);
-      else if (per <= 4) greedy_maxmin<4>(P, sk, spool, ssel, pn, ns);
-      else if (per <= 8) greedy_maxmin<8>(P, sk, spool, ssel, pn, ns);
-      else greedy_maxmin<16>(P, sk, spool, ssel, pn, ns);   // pool <= 320 here
+      if (per <= 1) greedy_maxmin<1>(P, sk, ssel, pn, ns);
+      else if (per <= 2) greedy_maxmin<2>(P, sk, ssel, pn, ns);
+      else if (per <= 4) greedy_maxmin<4>(P, sk, ssel, pn, ns);
+      else if (per <= 8) greedy_maxmin<8>(P, sk, ssel, pn, ns);
+      else greedy_maxmin<16>(P, sk, ssel, pn, ns);   // pool <= 320 here
     } else if (fixed24) {
-      greedy_maxmin<12>(P, TriFix24{fhi, flo}, spool, ssel, pn, ns);   // 320 < pool <= 384
+      greedy_maxmin<12>(P, TriFix24{fhi, flo}, ssel, pn, ns);   // 320 < pool <= 384
     } else {
       const TriF32 gk{P.gram};
-      if (per <= 16) greedy_maxmin<16>(P, gk, spool, ssel, pn, ns);
-      else greedy_maxmin<32>(P, gk, spool, ssel, pn, ns);
+      if (per <= 16) greedy_maxmin<16>(P, gk, ssel, pn, ns);
+      else greedy_maxmin<32>(P, gk, ssel, pn, ns);
     }
   }
   __syncwarp();
-  for (int r = lane; r < ns; r += 32) P.sel[r] = ssel[r];
+  for (int r = lane; r < ns; r += 32) {
+    const int rk = ssel[r];  // left unset past a failed step (status already raised)
+    const int u = rk >= 0 && rk < pn ? spool[rk] : -1;
+    ssel[r] = u;
+    P.sel[r] = u;
+  }
+  __syncwarp();
 
   // expansion: each pick and its n_prev predecessors, deduplicated, ascending
-  const int Uh = P.Uh;
-  const int nwords = (Uh + 31) >> 5;
-  for (int x = lane; x < nwords; x += 32) bits[x] = 0u;
-  __syncwarp();
   for (int r = lane; r < ns; r += 32) {
     const int u = ssel[r];
     for (int j = 0; j <= B.n_prev; ++j) {
@@ -1080,9 +1145,10 @@ cudaError_t launch_maxmin(const Batch& B, int max_pool, cudaStream_t s) {
     e = launch_pdl(k_gram, grid, dim3(kGramTile * kGramTile), (size_t)smem, s, B);
     if (e != cudaSuccess) return e;
   }
-  const int tri = max_pool * (max_pool + 1) / 2;
-  const int bytes = max_pool <= kMaxMinSmemPool ? tri * 4 : max_pool <= kMaxMinFixedPool ? tri * 3 : 4;
-  const int smem = ((bytes + 15) / 16) * (int)sizeof(float4);
+  // the largest staged triangle of any problem of the batch (the two forms' sizes are
+  // not monotonic across the switch to fixed point)
+  int smem = 16;
+  for (int j = 0; j < B.n; ++j) smem = max(smem, gram_smem_bytes(B.p[j].pool_n));
   cudaError_t e = cudaFuncSetAttribute(k_maxmin, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   return launch_pdl(k_maxmin, dim3(B.n), dim3(kMaxMinThreads), (size_t)smem, s, B);
