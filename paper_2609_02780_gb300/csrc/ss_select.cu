@@ -206,6 +206,7 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
   __shared__ float s_m[32], s_l[32];
   __shared__ int s_n, s_bstar, s_rem;
   __shared__ unsigned long long s_prefix;
+  __shared__ float s_lb;
 
   pdl_wait();
   pdl_release();
@@ -220,22 +221,71 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
   const int k = B.k;
 
   float M = -INFINITY, Ls = 0.f;
+  const int64_t n_tok = kGeneral ? (int64_t)P.n_cand : (int64_t)P.Uh * P.Tu;
+  int n = (int)min((int64_t)k, n_tok);
+  float lo = -INFINITY;
   if constexpr (!kGeneral) {
-    // softmax statistics from the per-unit pairs in a fixed order (thread t takes units
-    // t, t + 1024, ...; then a fixed tree), whichever warps scored the units
-    const float2* us = P.ustats + (int64_t)L * P.ucap;
-    for (int u = tid; u < P.Uh; u += blockDim.x) {
-      const float2 v = us[u];
-      ml_combine(M, Ls, v.x, v.y);
+    const uint32_t gthr = P.gthr[L];  // the bound the score kernel published
+    // Warp 0 first derives a tighter bound from the list's completed ladder of
+    // appended-score counts (its loads overlap the other warps' statistics loads): if
+    // the levels >= i hold n tokens, the n-th best score is at least level i's lower
+    // edge (one level of margin for the rounding of the level computation).
+    if (tid < 32) {
+      constexpr int per = kLadderLevels / 32;
+      const int* lad = P.ladder + (int64_t)L * kLadderLevels;
+      const float anchor = list_anchor(P, L);
+      int cntl[per];
+      int sum = 0;
+#pragma unroll
+      for (int q = 0; q < per; ++q) {
+        cntl[q] = lad[kLadderLevels - 1 - (per * lane + q)];
+        sum += cntl[q];
+      }
+      int cum = sum;
+      for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, cum, off);
+        if (lane >= off) cum += y;
+      }
+      const unsigned hit = __ballot_sync(0xffffffffu, cum >= n);
+      if (hit == 0u) {
+        if (lane == 0) s_lb = -INFINITY;
+      } else {
+        const int f = __ffs(hit) - 1;
+        if (lane == f) {
+          int run = cum - sum, qf = per - 1;
+#pragma unroll
+          for (int q = 0; q < per; ++q) {
+            run += cntl[q];
+            if (run >= n && qf == per - 1 && q < per - 1) qf = q;
+          }
+          const int lv = kLadderLevels - 1 - (per * lane + qf);
+          s_lb = anchor + (float)(lv - kLadderZero - 1) / kLadderPerUnit;
+        }
+      }
     }
-    block_ml(M, Ls, s_m, s_l);
+    // softmax statistics from the per-unit pairs in a fixed order (thread t takes units
+    // t, t + 1024, ...; then a fixed tree), whichever warps scored the units; four
+    // loads in flight per thread
+    const float2* us = P.ustats + (int64_t)L * P.ucap;
+    const int Uh = P.Uh;
+    for (int u0 = tid; u0 < Uh; u0 += 4 * (int)blockDim.x) {
+      float2 v[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int u = u0 + e * blockDim.x;
+        v[e] = u < Uh ? us[u] : make_float2(0.f, 0.f);
+      }
+#pragma unroll
+      for (int e = 0; e < 4; ++e)
+        if (u0 + e * (int)blockDim.x < Uh) ml_combine(M, Ls, v[e].x, v[e].y);
+    }
+    block_ml(M, Ls, s_m, s_l);  // its barriers also publish s_lb
     if (tid == 0) P.list_ml[L] = make_float2(M, Ls);
+    lo = fmaxf(ordered_to_float(gthr), s_lb);
   }
 
   int32_t* tok_out = P.topk_tok + (int64_t)L * k;
   float* w_out = P.topk_w + (int64_t)L * k;
-  const int64_t n_tok = kGeneral ? (int64_t)P.n_cand : (int64_t)P.Uh * P.Tu;
-  int n = (int)min((int64_t)k, n_tok);
   if (n == 0) {
     if (kGeneral && tid == 0) P.list_ml[L] = make_float2(-INFINITY, 0.f);
     for (int r = tid; r < k; r += blockDim.x) {
@@ -275,7 +325,6 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
       }
     }
   };
-  float lo = -INFINITY;
   if constexpr (kGeneral) {
     // statistics of the dense row in a fixed order: (max, sum 2^(s - max)) of the
     // scores, or (max, sum) of the head-averaged weights; and its minimum (the bound)
@@ -299,48 +348,6 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
     M = m;
     Ls = l;
     if (tid == 0) P.list_ml[L] = make_float2(M, Ls);
-  } else {
-    lo = ordered_to_float(P.gthr[L]);
-  }
-  // A tighter bound from the list's completed ladder of appended-score counts: if the
-  // levels >= i hold n tokens, the n-th best score is at least level i's lower edge
-  // (one level of margin for the rounding of the level computation).
-  if (!kGeneral && tid < 32) {
-    constexpr int per = kLadderLevels / 32;
-    const int* lad = P.ladder + (int64_t)L * kLadderLevels;
-    int cntl[per];
-    int sum = 0;
-#pragma unroll
-    for (int q = 0; q < per; ++q) {
-      cntl[q] = lad[kLadderLevels - 1 - (per * lane + q)];
-      sum += cntl[q];
-    }
-    int cum = sum;
-    for (int off = 1; off < 32; off <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, cum, off);
-      if (lane >= off) cum += y;
-    }
-    const unsigned hit = __ballot_sync(0xffffffffu, cum >= n);
-    if (lane == 0) s_m[0] = -INFINITY;
-    __syncwarp();
-    if (hit) {
-      const int f = __ffs(hit) - 1;
-      if (lane == f) {
-        int run = cum - sum, qf = per - 1;
-#pragma unroll
-        for (int q = 0; q < per; ++q) {
-          run += cntl[q];
-          if (run >= n && qf == per - 1 && q < per - 1) qf = q;
-        }
-        const int lv = kLadderLevels - 1 - (per * lane + qf);
-        s_m[0] = list_anchor(P, L) + (float)(lv - kLadderZero - 1) / kLadderPerUnit;
-      }
-    }
-  }
-  if constexpr (!kGeneral) {
-    __syncthreads();
-    lo = fmaxf(lo, s_m[0]);
-    __syncthreads();
   }
   if (lo == -INFINITY) {
     // no bound: start from the smallest real candidate (unused reserved slots hold
@@ -1028,6 +1035,10 @@ __global__ void __launch_bounds__(kMaxMinThreads) k_maxmin(const __grid_constant
   __shared__ int spool[kMaxPool];
   __shared__ int ssel[kMaxPool];
   __shared__ __align__(8) uint64_t tri_bar;
+  // the expansion's arguments, copied from the parameter block by another warp while
+  // warp 0 runs the greedy (its constant-cache misses stay off the serial path)
+  __shared__ int* xa_ptr[4];  // sel, exp_units, frames, counts
+  __shared__ int xa_int[2];   // frames per unit, n_prev
   pdl_wait();
   pdl_release();
   const Prob& P = B.p[blockIdx.x];
@@ -1058,6 +1069,14 @@ __global__ void __launch_bounds__(kMaxMinThreads) k_maxmin(const __grid_constant
   const int Uh = P.Uh;
   const int nwords = (Uh + 31) >> 5;
   for (int x = tid; x < nwords; x += blockDim.x) bits[x] = 0u;
+  if (tid == 32) {
+    xa_ptr[0] = P.sel;
+    xa_ptr[1] = P.exp_units;
+    xa_ptr[2] = P.frames;
+    xa_ptr[3] = P.counts;
+    xa_int[0] = P.fpu;
+    xa_int[1] = B.n_prev;
+  }
   __syncthreads();
   // One warp does the rest: warps parked at a barrier would slow its serial greedy.
   if (warp != 0) return;
@@ -1088,18 +1107,17 @@ __global__ void __launch_bounds__(kMaxMinThreads) k_maxmin(const __grid_constant
     }
   }
   __syncwarp();
+  int* const sel_out = xa_ptr[0];
+  int* const exp_out = xa_ptr[1];
+  int* const frames_out = xa_ptr[2];
+  const int fpu = xa_int[0], n_prev = xa_int[1];
+  // the picks' units, then the expansion: each pick and its n_prev predecessors,
+  // deduplicated, ascending
   for (int r = lane; r < ns; r += 32) {
     const int rk = ssel[r];  // left unset past a failed step (status already raised)
     const int u = rk >= 0 && rk < pn ? spool[rk] : -1;
-    ssel[r] = u;
-    P.sel[r] = u;
-  }
-  __syncwarp();
-
-  // expansion: each pick and its n_prev predecessors, deduplicated, ascending
-  for (int r = lane; r < ns; r += 32) {
-    const int u = ssel[r];
-    for (int j = 0; j <= B.n_prev; ++j) {
+    sel_out[r] = u;
+    for (int j = 0; j <= n_prev; ++j) {
       const int v = u - j;
       if (v >= 0 && v < Uh) atomicOr(&bits[v >> 5], 1u << (v & 31));
     }
@@ -1107,29 +1125,30 @@ __global__ void __launch_bounds__(kMaxMinThreads) k_maxmin(const __grid_constant
   __syncwarp();
   // lane l compacts the words [l * wpl, (l + 1) * wpl) in order
   const int wpl = (nwords + 31) / 32;
+  const int x0 = min(nwords, lane * wpl), x1 = min(nwords, x0 + wpl);
   int c = 0;
-  for (int x = lane * wpl; x < min(nwords, (lane + 1) * wpl); ++x) c += __popc(bits[x]);
+  for (int x = x0; x < x1; ++x) c += __popc(bits[x]);
   int incl = c;
   for (int off = 1; off < 32; off <<= 1) {
     const int y = __shfl_up_sync(0xffffffffu, incl, off);
     if (lane >= off) incl += y;
   }
   int q = incl - c;
-  for (int x = lane * wpl; x < min(nwords, (lane + 1) * wpl); ++x) {
+  for (int x = x0; x < x1; ++x) {
     uint32_t rest = bits[x];
     while (rest) {
-      const int bpos = __ffs(rest) - 1;
+      const int u = x * 32 + __ffs(rest) - 1;
       rest &= rest - 1u;
-      const int u = x * 32 + bpos;
-      P.exp_units[q] = u;
-      for (int f = 0; f < P.fpu; ++f) P.frames[q * P.fpu + f] = u * P.fpu + f;
+      exp_out[q] = u;
+      for (int f = 0; f < fpu; ++f) frames_out[q * fpu + f] = u * fpu + f;
       ++q;
     }
   }
   if (lane == 31) {
-    P.counts[1] = ns;
-    P.counts[2] = incl;
-    P.counts[3] = incl * P.fpu;
+    int* const counts = xa_ptr[3];
+    counts[1] = ns;
+    counts[2] = incl;
+    counts[3] = incl * fpu;
   }
 }
 
