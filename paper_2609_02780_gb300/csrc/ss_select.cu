@@ -112,10 +112,10 @@ __device__ void bitonic_desc_hybrid(unsigned long long* a, int n2) {
 
 // Descending sort of keys[0, ns) by bucketing on the score (the upper 32 bits of a key):
 // 2048 buckets over [lo, hi] (every key's score lies there), a counting scatter in
-// bucket order, then an insertion sort inside each bucket. Needs ns <= kSelCap / 2
-// (the upper half of `keys` holds the input copy) and buckets of at most kBucketMax
-// keys; returns false, with keys untouched, when a bucket is larger (then the caller
-// sorts another way). All threads of the block call it.
+// bucket order into the upper half of `keys`, then every key placed by its rank inside
+// its bucket. Needs ns <= kSelCap / 2 and buckets of at most kBucketMax keys; returns
+// false, with keys untouched, when a bucket is larger (then the caller sorts another
+// way). All threads of the block call it.
 constexpr int kBucketMax = 32;
 
 template <int kThreads>
@@ -123,11 +123,13 @@ __device__ bool bucket_sort_desc(unsigned long long* keys, int ns, float lo, flo
                                  int* hist, int* cursor, int* sflag) {
   const int tid = threadIdx.x;
   const uint32_t klo = float_to_ordered(lo), khi = float_to_ordered(hi);
-  const uint64_t span = (uint64_t)(khi - klo) + 1u;
+  // buckets linear in the ordered score bits, in fp32 (rounding keeps the map
+  // monotonic, which is all the order needs)
+  const float scale = (float)kFineBins / ((float)(khi - klo) + 1.0f);
   auto bucket = [&](unsigned long long key) -> int {
     const uint32_t ok = (uint32_t)(key >> 32);
-    const uint64_t d = ok > klo ? (uint64_t)(ok - klo) : 0u;
-    const int b = (int)((d * kFineBins) / span);
+    const uint32_t d = ok > klo ? ok - klo : 0u;
+    const int b = (int)((float)d * scale);
     return kFineBins - 1 - min(b, kFineBins - 1);  // best scores first
   };
   for (int b = tid; b < kFineBins; b += blockDim.x) hist[b] = 0;
@@ -155,25 +157,26 @@ __device__ bool bucket_sort_desc(unsigned long long* keys, int ns, float lo, flo
     cursor[kPerT * tid + q] = run;
     run += c[q];
   }
-  unsigned long long* in = keys + sel_cap<kThreads>() / 2;
-  for (int i = tid; i < ns; i += blockDim.x) in[i] = keys[i];
-  __syncthreads();
+  __syncthreads();  // every bucket's start is set before any thread scatters
+  // scatter into the upper half (ns <= half the capacity), bucket by bucket
+  unsigned long long* tmp = keys + sel_cap<kThreads>() / 2;
   for (int i = tid; i < ns; i += blockDim.x) {
-    const unsigned long long key = in[i];
-    keys[atomicAdd(&cursor[bucket(key)], 1)] = key;
+    const unsigned long long key = keys[i];
+    tmp[atomicAdd(&cursor[bucket(key)], 1)] = key;
   }
   __syncthreads();
-  for (int b = tid; b < kFineBins; b += blockDim.x) {
+  // every key's place inside its bucket: the bucket's keys above it (equal keys by
+  // position), at most kBucketMax comparisons per key
+  for (int i = tid; i < ns; i += blockDim.x) {
+    const unsigned long long key = tmp[i];
+    const int b = bucket(key);
     const int b0 = hist[b], b1 = cursor[b];  // after the scatter: the bucket's end
-    for (int i = b0 + 1; i < b1; ++i) {
-      const unsigned long long x = keys[i];
-      int j = i - 1;
-      while (j >= b0 && keys[j] < x) {
-        keys[j + 1] = keys[j];
-        --j;
-      }
-      keys[j + 1] = x;
+    int r = 0;
+    for (int j = b0; j < b1; ++j) {
+      const unsigned long long y = tmp[j];
+      r += (y > key || (y == key && j < i)) ? 1 : 0;
     }
+    keys[b0 + r] = key;
   }
   __syncthreads();
   return true;
