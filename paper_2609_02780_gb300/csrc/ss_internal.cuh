@@ -24,12 +24,14 @@ constexpr uint32_t kCentroidIdBase = 0x40000000u;
 constexpr int kMaxCentroids = 128;     // per window (k-means compression)
 constexpr int kMaxWindowTokens = 65536;
 
-// Score-kernel geometry: kScoreWarps compute warps + 1 threshold warp per CTA.
+// Score-kernel geometry: kScoreWarps compute warps + 2 threshold warps per CTA (each
+// threshold warp serves half of the group's lists).
 #ifndef SS_SCORE_WARPS
 #define SS_SCORE_WARPS 8
 #endif
 constexpr int kScoreWarps = SS_SCORE_WARPS;
-constexpr int kScoreThreads = (kScoreWarps + 1) * 32;
+constexpr int kThresholdWarps = 2;
+constexpr int kScoreThreads = (kScoreWarps + kThresholdWarps) * 32;
 #ifndef SS_SCORE_CTAS_PER_SM
 #define SS_SCORE_CTAS_PER_SM 2
 #endif

@@ -178,7 +178,7 @@ cudaError_t launch_prep(const Batch& B, cudaStream_t s) {
 // Scoring kernel.
 //
 // Grid: P.chunks CTAs per (problem, slab = (layer i, key head g)), one wave.
-// Block: kScoreWarps compute warps + 1 threshold warp.
+// Block: kScoreWarps compute warps + 2 threshold warps.
 //
 // All compute warps of a slab's CTAs take history units from the slab's shared unit
 // counter, so SMs that run faster score more units, and walk each unit in tiles of 16
@@ -194,7 +194,7 @@ cudaError_t launch_prep(const Batch& B, cudaStream_t s) {
 // Candidate filter: a token is appended to its list when s >= thr[h], where thr[h] is
 // always a lower bound of the list's k-th best score, so every top-k token is
 // appended. Every appended score also counts in the CTA's ladder for its list (256
-// levels 1/16 apart in log2 units, anchored at the list's best sampled unit); the
+// levels 1/16 apart in log2 units, anchored at the list's best sampled unit); a
 // threshold warp merges the CTA's counts into the list's global ladder and scans it
 // from the top: the level where the count first reaches k bounds the k-th best score
 // from below, because at least k appended tokens (of any CTA) score that much. The
@@ -235,6 +235,8 @@ __device__ __forceinline__ void ladder_add(ScoreShared& S, int c, float s, float
   if (lv >= 0) atomicAdd(&S.lad[c][min(lv, kLadderLevels - 1)], 1);
 }
 
+constexpr int kThrLists = kMaxGroup / kThresholdWarps;  // lists per threshold warp
+
 // The threshold warp merges this CTA's ladder counts into the lists' global counts and
 // derives from those the lower bound thr of each list's k-th best score: if the
 // levels >= i hold at least k appended tokens (of any CTA), the k-th best score is at
@@ -242,84 +244,72 @@ __device__ __forceinline__ void ladder_add(ScoreShared& S, int c, float s, float
 // computation. Lane l handles the levels 255 - (32 q + l), q = 0..7, so that a warp's
 // accesses to one block of 32 levels are consecutive words (no shared-memory bank
 // conflicts, one 128-byte global transaction).
-__device__ __noinline__ void threshold_warp(ScoreShared& S, const Prob& P, int list0, int k) {
+__device__ __noinline__ void threshold_warp(ScoreShared& S, const Prob& P, int list0, int k,
+                                           int c0) {
   constexpr int per = kLadderLevels / 32;  // blocks of 32 levels; block 0 the top ones
   const int lane = threadIdx.x & 31;
   const int G = P.G;
+  if (c0 >= G) return;  // no list of this warp's half
   volatile int* vdone = &S.all_done;
   volatile float* vthr = S.thr;
   auto level = [&](int q) { return kLadderLevels - 1 - (32 * q + lane); };
   for (int iter = 0; iter < (1 << 21); ++iter) {
     const int done = *vdone;
-    // the bounds other CTAs published (lane c holds list c's), in flight while merging
+    // the bounds other CTAs published (lane c holds list c's)
     const float pub = lane < G ? ordered_to_float(*(volatile uint32_t*)(P.gthr + list0 + lane))
                                : -INFINITY;
-    // merge this CTA's new counts into the global ladder, 2 lists at a time: all the
-    // exchanges first, then the additions (no atomic result is waited for)
+    // the global counts of this warp's lists, all in flight at once (one round trip per
+    // pass); they predate this pass's merge, whose counts are added to them here
+    int cnt[kThrLists][per];
 #pragma unroll
-    for (int c0 = 0; c0 < kMaxGroup; c0 += 2) {
-      int dv[2][per];
+    for (int j = 0; j < kThrLists; ++j) {
+      const int c = c0 + j;
+      const volatile int* gl = P.ladder + (int64_t)(list0 + (c < G ? c : 0)) * kLadderLevels;
 #pragma unroll
-      for (int cc = 0; cc < 2; ++cc) {
-#pragma unroll
-        for (int q = 0; q < per; ++q)
-          dv[cc][q] = c0 + cc < G ? atomicExch(&S.lad[c0 + cc][level(q)], 0) : 0;
-      }
-#pragma unroll
-      for (int cc = 0; cc < 2; ++cc) {
-        int* gl = P.ladder + (int64_t)(list0 + c0 + cc) * kLadderLevels;
-#pragma unroll
-        for (int q = 0; q < per; ++q)
-          if (dv[cc][q]) atomicAdd(gl + level(q), dv[cc][q]);
-      }
+      for (int q = 0; q < per; ++q) cnt[j][q] = c < G ? gl[level(q)] : 0;
     }
-    // the global counts of 4 lists per round trip
 #pragma unroll
-    for (int c0 = 0; c0 < kMaxGroup; c0 += 4) {
-      if (c0 >= G) break;
-      int cnt[4][per];
+    for (int j = 0; j < kThrLists; ++j) {
+      const int c = c0 + j;
+      if (c >= G) break;
+      // merge this CTA's new counts of list c into the global ladder (not waited for)
+      int* gl = P.ladder + (int64_t)(list0 + c) * kLadderLevels;
 #pragma unroll
-      for (int cc = 0; cc < 4; ++cc) {
-        const int c = c0 + cc;
-        const volatile int* gl = P.ladder + (int64_t)(list0 + (c < G ? c : 0)) * kLadderLevels;
-#pragma unroll
-        for (int q = 0; q < per; ++q) cnt[cc][q] = c < G ? gl[level(q)] : 0;
+      for (int q = 0; q < per; ++q) {
+        const int dv = atomicExch(&S.lad[c][level(q)], 0);
+        if (dv) atomicAdd(gl + level(q), dv);
+        cnt[j][q] += dv;
       }
+      // the first block of 32 levels where the count from the top reaches k, then the
+      // first level inside it
+      int above = 0, qf = -1;
 #pragma unroll
-      for (int cc = 0; cc < 4; ++cc) {
-        const int c = c0 + cc;
-        if (c >= G) break;
-        // the first block of 32 levels where the count from the top reaches k, then the
-        // first level inside it
-        int above = 0, qf = -1;
-#pragma unroll
-        for (int q = 0; q < per; ++q) {
-          const int tq = __reduce_add_sync(0xffffffffu, (unsigned)cnt[cc][q]);
-          if (qf < 0 && above + tq >= k) qf = q;
-          if (qf < 0) above += tq;
-        }
-        float t = -INFINITY;
-        if (qf >= 0) {
-          int mine = 0;
-#pragma unroll
-          for (int q = 0; q < per; ++q)
-            if (q == qf) mine = cnt[cc][q];
-          int cum = mine;
-#pragma unroll
-          for (int off = 1; off < 32; off <<= 1) {
-            const int y = __shfl_up_sync(0xffffffffu, cum, off);
-            if (lane >= off) cum += y;
-          }
-          const unsigned hit = __ballot_sync(0xffffffffu, above + cum >= k);
-          const int f = __ffs(hit) - 1;
-          const int lv = kLadderLevels - 1 - (32 * qf + f);
-          t = S.anchor[c] + (float)(lv - kLadderZero - 1) / kLadderPerUnit;
-          if (lane == 0) atomicMax(P.gthr + list0 + c, float_to_ordered(t));  // not waited for
-        }
-        const float other = __shfl_sync(0xffffffffu, pub, c);
-        t = fmaxf(t, other);
-        if (lane == 0 && t > vthr[c]) vthr[c] = t;
+      for (int q = 0; q < per; ++q) {
+        const int tq = __reduce_add_sync(0xffffffffu, (unsigned)cnt[j][q]);
+        if (qf < 0 && above + tq >= k) qf = q;
+        if (qf < 0) above += tq;
       }
+      float t = -INFINITY;
+      if (qf >= 0) {
+        int mine = 0;
+#pragma unroll
+        for (int q = 0; q < per; ++q)
+          if (q == qf) mine = cnt[j][q];
+        int cum = mine;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+          const int y = __shfl_up_sync(0xffffffffu, cum, off);
+          if (lane >= off) cum += y;
+        }
+        const unsigned hit = __ballot_sync(0xffffffffu, above + cum >= k);
+        const int f = __ffs(hit) - 1;
+        const int lv = kLadderLevels - 1 - (32 * qf + f);
+        t = S.anchor[c] + (float)(lv - kLadderZero - 1) / kLadderPerUnit;
+        if (lane == 0) atomicMax(P.gthr + list0 + c, float_to_ordered(t));  // not waited for
+      }
+      const float other = __shfl_sync(0xffffffffu, pub, c);
+      t = fmaxf(t, other);
+      if (lane == 0 && t > vthr[c]) vthr[c] = t;
     }
     __syncwarp();
     if (done >= kScoreWarps) break;
@@ -362,8 +352,8 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int k = B.k;
-  if (warp == kScoreWarps) {
-    threshold_warp(S, P, list0, k);
+  if (warp >= kScoreWarps) {
+    threshold_warp(S, P, list0, k, (warp - kScoreWarps) * kThrLists);
     return;
   }
 
