@@ -38,8 +38,8 @@ __global__ void __launch_bounds__(256) k_sample(const __grid_constant__ Batch B)
   __shared__ __align__(16) __nv_bfloat16 qsb[kMaxGroup][kHeadDim];
   __shared__ float wmax[8][kMaxGroup];
   __shared__ __align__(16) unsigned char kt[kSampleRows * kHeadDim * 2];
-  pdl_wait();     // keys, queries and the previous call's use of the workspace
-  pdl_release();
+  // Before the wait for the previous kernel: only reads of the inputs (query rows and
+  // the first pass of the sampled unit's keys), which no kernel of the chain writes.
   const int pi = blockIdx.y;
   if (pi >= B.n) return;
   const Prob& P = B.p[pi];
@@ -50,6 +50,21 @@ __global__ void __launch_bounds__(256) k_sample(const __grid_constant__ Batch B)
   const int list0 = i * P.Hq + gk * G;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t row_stride = (int64_t)P.Hq * kHeadDim;
+  const bool sampling = z < P.n_sample;
+  const int64_t u = sampling ? ((int64_t)z * P.Uh) / P.n_sample : 0;
+  const __nv_bfloat16* sk = P.keys + ((int64_t)slab * P.ncap + u * P.Tu) * kHeadDim;
+  // a pass's rows as 16-byte vectors, all of a thread's loads in flight at once
+  constexpr int kPerThread = kSampleRows * (kHeadDim / 8) / 256;
+  uint4 vbuf[kPerThread];
+  auto load_pass = [&](int rb, int nr) {
+    const uint4* src = reinterpret_cast<const uint4*>(sk + (int64_t)rb * kHeadDim);
+#pragma unroll
+    for (int q = 0; q < kPerThread; ++q) {
+      const int x = q * 256 + tid;
+      if (x < nr * (kHeadDim / 8)) vbuf[q] = src[x];
+    }
+  };
+  if (sampling) load_pass(0, min(kSampleRows, P.Tu));
   for (int x = tid; x < kMaxGroup * kHeadDim; x += blockDim.x) {
     const int hh = x / kHeadDim, d = x - hh * kHeadDim;
     __nv_bfloat16 qe = __float2bfloat16_rn(0.f);
@@ -64,26 +79,27 @@ __global__ void __launch_bounds__(256) k_sample(const __grid_constant__ Batch B)
         v = __fdiv_rn(acc, (float)P.R);
       }
       qe = __float2bfloat16_rn(v);
-      if (z == 0) P.qeff[(int64_t)(list0 + hh) * kHeadDim + d] = qe;
     }
     qsb[hh][d] = qe;
   }
+  pdl_wait();     // the previous call's use of the workspace
+  pdl_release();
   if (z == 0) {
+    for (int x = tid; x < G * kHeadDim; x += blockDim.x)  // each thread's own qsb entries
+      P.qeff[(int64_t)list0 * kHeadDim + x] = qsb[x / kHeadDim][x % kHeadDim];
     if (tid < G) {
       P.cand_cnt[list0 + tid] = 0;
       P.gthr[list0 + tid] = float_to_ordered(-INFINITY);
     }
     for (int x = tid; x < G * kLadderLevels; x += blockDim.x)
       P.ladder[(int64_t)list0 * kLadderLevels + x] = 0;
-    if (tid == 0) P.next_unit[slab] = 0;
-    for (int u = slab * blockDim.x + tid; u < P.ucap; u += n_slabs * blockDim.x) P.votes[u] = 0;
+    if (tid == 0) P.next_unit[slab] = P.chunks * kScoreWarps;  // past the fixed first units
+    for (int v = slab * blockDim.x + tid; v < P.ucap; v += n_slabs * blockDim.x) P.votes[v] = 0;
     if (slab == 0 && tid < 4) P.counts[tid] = 0;
     if (slab == 0 && tid == 0) *P.status = 0u;
   }
   __syncthreads();
-  if (z >= P.n_sample) return;
-  const int64_t u = ((int64_t)z * P.Uh) / P.n_sample;
-  const __nv_bfloat16* sk = P.keys + ((int64_t)slab * P.ncap + u * P.Tu) * kHeadDim;
+  if (!sampling) return;
   // query fragments, permuted like the key fragments (as in the scoring kernel)
   const int g = lane >> 2, t4 = lane & 3;
   uint32_t qf[8][2];
@@ -102,16 +118,8 @@ __global__ void __launch_bounds__(256) k_sample(const __grid_constant__ Batch B)
   for (int rb = 0; rb < P.Tu; rb += kSampleRows) {
     const int nr = min(kSampleRows, P.Tu - rb);
     __syncthreads();
-    const uint4* src = reinterpret_cast<const uint4*>(sk + (int64_t)rb * kHeadDim);
     uint4* dst = reinterpret_cast<uint4*>(kt);
-    // the pass's rows as 16-byte vectors, all of a thread's loads in flight at once
-    constexpr int kPerThread = kSampleRows * (kHeadDim / 8) / 256;
-    uint4 vbuf[kPerThread];
-#pragma unroll
-    for (int q = 0; q < kPerThread; ++q) {
-      const int x = q * 256 + tid;
-      if (x < nr * (kHeadDim / 8)) vbuf[q] = src[x];
-    }
+    if (rb > 0) load_pass(rb, nr);  // the first pass was loaded before the wait
 #pragma unroll
     for (int q = 0; q < kPerThread; ++q) {
       const int x = q * 256 + tid;
@@ -335,22 +343,61 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
   const int i = slab / P.Hkv, kvh = slab - i * P.Hkv;
   const int G = P.G;
   const int list0 = i * P.Hq + kvh * G;
-  pdl_wait();     // q_eff, anchors and resets of the prep kernel
-  pdl_release();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int x = threadIdx.x; x < kMaxGroup * kLadderLevels; x += blockDim.x)
     (&S.lad[0][0])[x] = 0;
-  if (threadIdx.x < kMaxGroup) {
-    // a CTA that starts late begins with the bound published by the earlier ones
-    S.thr[threadIdx.x] = threadIdx.x < G ? ordered_to_float(P.gthr[list0 + threadIdx.x]) : -INFINITY;
-    S.anchor[threadIdx.x] = threadIdx.x < G ? list_anchor(P, list0 + threadIdx.x) : 0.f;
-  }
   if (threadIdx.x == 0) S.all_done = 0;
   if (threadIdx.x < kScoreWarps * kScoreStages)
     mbar_init(smem_u32(&S.bar[0][0] + threadIdx.x), 1u);
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   __syncthreads();
 
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int Tu = P.Tu;
+  const int tpu = (Tu + kTileRows - 1) / kTileRows;
+  const int Uh = P.Uh;
+  const __nv_bfloat16* slab_keys = P.keys + (int64_t)slab * P.ncap * kHeadDim;
+  unsigned char* my_tiles = tiles + (size_t)(warp < kScoreWarps ? warp : 0) * kScoreStages * kTileBytes;
+  const uint32_t my_tiles_s = smem_u32(my_tiles);
+  const uint32_t my_bars = smem_u32(&S.bar[warp < kScoreWarps ? warp : 0][0]);
+  // Lane 0 starts the bulk copy of tile t (unit uu, tile jj of the unit) into its
+  // stage once the warp's reads of that stage are ordered before the async write.
+  auto issue = [&](int t, int uu, int jj) {
+    if (uu >= Uh) return;
+    const int r0 = kTileRows * jj;
+    const int nrows = min(kTileRows, Tu - r0);
+    const int st = t % kScoreStages;
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      const uint32_t bar = my_bars + 8u * st;
+      const uint32_t bytes = (uint32_t)nrows * kHeadDim * 2u;
+      mbar_expect_tx(bar, bytes);
+      bulk_load(my_tiles_s + (uint32_t)st * kTileBytes,
+                slab_keys + ((int64_t)uu * Tu + r0) * kHeadDim, bytes, bar);
+    }
+  };
+  // Each compute warp's first unit is fixed (a slab's CTAs take units idx * kScoreWarps
+  // + warp; the slab's counter, reset by the prep kernel, hands out the rest), so its
+  // first tiles are requested before the wait for the prep kernel: they read only the
+  // keys, which no kernel of the chain writes.
+  int iu = Uh;
+  int n_pre = 0;
+  if (warp < kScoreWarps) {
+    const int idx = B.score_spread ? local / n_slabs : local - slab * P.chunks;
+    const int first = idx * kScoreWarps + warp;
+    iu = first < Uh ? first : Uh;
+    n_pre = min(kScoreStages, tpu);
+    for (int t = 0; t < n_pre; ++t) issue(t, iu, t);
+  }
+  pdl_wait();     // q_eff, anchors and resets of the prep kernel
+  pdl_release();
+  if (threadIdx.x < kMaxGroup) {
+    // a CTA that starts late begins with the bound published by the earlier ones
+    S.thr[threadIdx.x] = threadIdx.x < G ? ordered_to_float(P.gthr[list0 + threadIdx.x]) : -INFINITY;
+    S.anchor[threadIdx.x] = threadIdx.x < G ? list_anchor(P, list0 + threadIdx.x) : 0.f;
+  }
+  __syncthreads();
+
   const int k = B.k;
   if (warp >= kScoreWarps) {
     threshold_warp(S, P, list0, k, (warp - kScoreWarps) * kThrLists);
@@ -378,16 +425,9 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
   const int c0 = 2 * t4, c1 = 2 * t4 + 1;
   const bool hv0 = c0 < G, hv1 = c1 < G;
   const int L0 = list0 + c0, L1 = list0 + c1;
-  const int Tu = P.Tu;
-  const int tpu = (Tu + kTileRows - 1) / kTileRows;
-  const int Uh = P.Uh;
   int* next_unit = P.next_unit + slab;
-  const __nv_bfloat16* slab_keys = P.keys + (int64_t)slab * P.ncap * kHeadDim;
   const int64_t cbase0 = (int64_t)(hv0 ? L0 : list0) * P.cand_cap;
   const int64_t cbase1 = (int64_t)(hv1 ? L1 : list0) * P.cand_cap;
-  unsigned char* my_tiles = tiles + (size_t)warp * kScoreStages * kTileBytes;
-  const uint32_t my_tiles_s = smem_u32(my_tiles);
-  const uint32_t my_bars = smem_u32(&S.bar[warp][0]);
   const volatile float* vthr = S.thr;
   const unsigned gmask = 0x11111111u << t4;
   const unsigned lt_mask = (1u << lane) - 1u;
@@ -467,28 +507,10 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
     scp += n0 + (n1 << 8);
   };
 
-  // Lane 0 starts the bulk copy of tile t (unit uu, tile jj of the unit) into its
-  // stage once the warp's reads of that stage are ordered before the async write.
-  auto issue = [&](int t, int uu, int jj) {
-    if (uu >= Uh) return;
-    const int r0 = kTileRows * jj;
-    const int nrows = min(kTileRows, Tu - r0);
-    const int st = t % kScoreStages;
-    fence_proxy_async_smem();
-    __syncwarp();
-    if (lane == 0) {
-      const uint32_t bar = my_bars + 8u * st;
-      const uint32_t bytes = (uint32_t)nrows * kHeadDim * 2u;
-      mbar_expect_tx(bar, bytes);
-      bulk_load(my_tiles_s + (uint32_t)st * kTileBytes,
-                slab_keys + ((int64_t)uu * Tu + r0) * kHeadDim, bytes, bar);
-    }
-  };
-
-  // Units come from the slab's shared counter: every warp of the slab's CTAs takes the
-  // next unit when it needs one, so faster SMs score more units. Lane 0 takes its next
-  // unit one unit ahead (the atomic's latency hides behind a unit of work); the units a
-  // warp takes are queued in shared memory for its consume cursor.
+  // After the first, units come from the slab's shared counter: every warp of the
+  // slab's CTAs takes the next unit when it needs one, so faster SMs score more units.
+  // Lane 0 takes its next unit one unit ahead (the atomic's latency hides behind a unit
+  // of work); the units a warp takes are queued in shared memory for its consume cursor.
   int* uq = S.uq[warp];
   int pre = lane == 0 ? atomicAdd(next_unit, 1) : 0;
   auto take = [&]() {
@@ -496,7 +518,7 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
     if (lane == 0) pre = u < Uh ? atomicAdd(next_unit, 1) : Uh;
     return min(u, Uh);
   };
-  int iu = take(), ij = 0, nq = 0;     // issue position, units queued
+  int ij = 0, nq = 0;                  // issue position (unit iu, tile ij), units queued
   if (lane == 0) uq[0] = iu;
   nq = 1;
   __syncwarp();
@@ -511,7 +533,7 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
     }
   };
   for (int t = 0; t < kScoreStages; ++t) {
-    issue(t, iu, ij);
+    if (t >= n_pre) issue(t, iu, ij);  // the first n_pre went out before the wait
     advance_issue();
   }
 
