@@ -687,7 +687,7 @@ __global__ void __launch_bounds__(1024) k_pool(const __grid_constant__ Batch B) 
   extern __shared__ unsigned char smem_raw[];
   __shared__ int vh[kVoteBins];
   __shared__ int sw[32];
-  __shared__ int s_v, s_c;
+  __shared__ int s_v, s_c, s_vmax;
   pdl_wait();
   pdl_release();
   const Prob& P = B.p[blockIdx.x];
@@ -698,7 +698,10 @@ __global__ void __launch_bounds__(1024) k_pool(const __grid_constant__ Batch B) 
   // (1) histogram of votes (clipped): the pool's smallest vote level V is the highest
   //     level whose units and all better ones number at least pool_n
   for (int x = tid; x < kVoteBins; x += blockDim.x) vh[x] = 0;
-  if (tid == 0) s_c = 0;
+  if (tid == 0) {
+    s_c = 0;
+    s_vmax = 0;
+  }
   __syncthreads();
   // every thread's units' votes are loaded at once and kept for step (2)
   constexpr int kUnitsPerThread = kMaxHistUnits / 1024;
@@ -743,6 +746,7 @@ __global__ void __launch_bounds__(1024) k_pool(const __grid_constant__ Batch B) 
       if (pos < kRankMax) {
         ck[pos] = ((unsigned long long)(uint32_t)vt[q] << 32) | __float_as_uint(P.mass[u]);
         ci[pos] = u;
+        atomicMax(&s_vmax, vt[q]);
       }
     }
   }
@@ -750,9 +754,21 @@ __global__ void __launch_bounds__(1024) k_pool(const __grid_constant__ Batch B) 
   const int C = s_c;
   if (C <= kRankMax) {
     // rank = the number of candidates ordered before; the block's threads split the
-    // comparisons: thread t counts for candidate t % C over part t / C of the others
+    // comparisons: thread t counts for candidate t % C over part t / C of the others.
+    // When the votes fit 19 bits one 64-bit key orders a candidate exactly: votes, the
+    // mass's bits (31: masses are sums of non-negative weights, so the sign bit is clear
+    // and the bits order as the values) and 16383 - id (14 bits: ids < kMaxHistUnits),
+    // so a comparison is one 64-bit compare.
+    static_assert(kMaxHistUnits <= (1 << 14), "unit ids must fit 14 bits");
+    const bool packed = s_vmax < (1 << 19);
     int* rk = reinterpret_cast<int*>(ci + kRankMax);
-    for (int x = tid; x < C; x += blockDim.x) rk[x] = 0;
+    for (int x = tid; x < C; x += blockDim.x) {
+      rk[x] = 0;
+      if (packed) {
+        const unsigned long long v = ck[x] >> 32, mb = (uint32_t)ck[x] & 0x7fffffffu;
+        ck[x] = (v << 45) | (mb << 14) | (unsigned long long)(16383 - ci[x]);
+      }
+    }
     __syncthreads();
     const int parts = max(1, (int)blockDim.x / max(C, 1));
     const int i = tid % max(C, 1), part = tid / max(C, 1);
@@ -762,11 +778,19 @@ __global__ void __launch_bounds__(1024) k_pool(const __grid_constant__ Batch B) 
       const int o0 = (int)(((int64_t)C * part) / parts), o1 = (int)(((int64_t)C * (part + 1)) / parts);
       int r[4] = {0, 0, 0, 0};  // independent partial counts keep the loads in flight
       int o = o0;
-      for (; o + 4 <= o1; o += 4) {
+      if (packed) {
+        for (; o + 4 <= o1; o += 4) {
 #pragma unroll
-        for (int e = 0; e < 4; ++e) r[e] += unit_before(ck[o + e], ci[o + e], mk, mi) ? 1 : 0;
+          for (int e = 0; e < 4; ++e) r[e] += ck[o + e] > mk ? 1 : 0;
+        }
+        for (; o < o1; ++o) r[0] += ck[o] > mk ? 1 : 0;
+      } else {
+        for (; o + 4 <= o1; o += 4) {
+#pragma unroll
+          for (int e = 0; e < 4; ++e) r[e] += unit_before(ck[o + e], ci[o + e], mk, mi) ? 1 : 0;
+        }
+        for (; o < o1; ++o) r[0] += unit_before(ck[o], ci[o], mk, mi) ? 1 : 0;
       }
-      for (; o < o1; ++o) r[0] += unit_before(ck[o], ci[o], mk, mi) ? 1 : 0;
       atomicAdd(&rk[i], r[0] + r[1] + r[2] + r[3]);
     }
     __syncthreads();
