@@ -914,7 +914,7 @@ __global__ void __launch_bounds__(256) k_gram(const __grid_constant__ Batch B) {
   }
   if (ta >= T) return;
   const int tb = ta + rem;
-  const int ld = dim + 1;
+  const int ld = dim + 4;  // rows 16-byte aligned; float4 reads of 8 rows hit distinct banks
   float* A = gsm;
   float* Bm = gsm + kGramTile * ld;
   __shared__ int ua[kGramTile], ub[kGramTile];
@@ -925,8 +925,8 @@ __global__ void __launch_bounds__(256) k_gram(const __grid_constant__ Batch B) {
   }
   __syncthreads();
   const int d4 = dim / 4;
-  // the rows' float4s, 4 + 4 per thread in flight before any is stored
-  constexpr int kB = 4;
+  // the rows' float4s, 8 + 8 per thread in flight before any is stored
+  constexpr int kB = 8;
   for (int x0 = 0; x0 < kGramTile * d4; x0 += kB * blockDim.x) {
     float4 va[kB], vb[kB];
 #pragma unroll
@@ -944,19 +944,25 @@ __global__ void __launch_bounds__(256) k_gram(const __grid_constant__ Batch B) {
       const int x = x0 + q * blockDim.x + threadIdx.x;
       if (x < kGramTile * d4) {
         const int r = x / d4, e = 4 * (x - r * d4);
-        float* pa = A + r * ld + e;
-        float* pb = Bm + r * ld + e;
-        pa[0] = va[q].x; pa[1] = va[q].y; pa[2] = va[q].z; pa[3] = va[q].w;
-        pb[0] = vb[q].x; pb[1] = vb[q].y; pb[2] = vb[q].z; pb[3] = vb[q].w;
+        *reinterpret_cast<float4*>(A + r * ld + e) = va[q];
+        *reinterpret_cast<float4*>(Bm + r * ld + e) = vb[q];
       }
     }
   }
   __syncthreads();
   const int r = threadIdx.x / kGramTile, c = threadIdx.x % kGramTile;
-  float a4[4] = {0.f, 0.f, 0.f, 0.f};  // four independent FMA chains (dim % 4 == 0)
-  for (int d = 0; d < dim; d += 4) {
-#pragma unroll
-    for (int e = 0; e < 4; ++e) a4[e] = fmaf(A[r * ld + d + e], Bm[c * ld + d + e], a4[e]);
+  // four independent FMA chains (chain e takes the dimensions = e mod 4), fed by float4
+  // reads (dim % 4 == 0)
+  float a4[4] = {0.f, 0.f, 0.f, 0.f};
+  const float4* A4 = reinterpret_cast<const float4*>(A + r * ld);
+  const float4* B4 = reinterpret_cast<const float4*>(Bm + c * ld);
+#pragma unroll 4
+  for (int d4 = 0; d4 < dim / 4; ++d4) {
+    const float4 x = A4[d4], y = B4[d4];
+    a4[0] = fmaf(x.x, y.x, a4[0]);
+    a4[1] = fmaf(x.y, y.y, a4[1]);
+    a4[2] = fmaf(x.z, y.z, a4[2]);
+    a4[3] = fmaf(x.w, y.w, a4[3]);
   }
   const float acc = (a4[0] + a4[1]) + (a4[2] + a4[3]);
   const int a = ta * kGramTile + r, b = tb * kGramTile + c;
@@ -1184,7 +1190,7 @@ cudaError_t launch_maxmin(const Batch& B, int max_pool, cudaStream_t s) {
   for (int j = 0; j < B.n; ++j) max_dim = max(max_dim, B.p[j].Hkv * kHeadDim);
   if (max_pool > 0) {
     const int T = (max_pool + kGramTile - 1) / kGramTile;
-    const int smem = 2 * kGramTile * (max_dim + 1) * (int)sizeof(float);
+    const int smem = 2 * kGramTile * (max_dim + 4) * (int)sizeof(float);
     cudaError_t e = cudaFuncSetAttribute(k_gram, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     dim3 grid(T * (T + 1) / 2, B.n);
