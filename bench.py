@@ -219,8 +219,8 @@ def run_reference(args):
 # capture summarised in profiles/k_score_dram_traffic.md; valid only for the kernel
 # sources it was taken on (their sha256 below), reported as null otherwise.
 TRAFFIC_RECORD = {"workload": "hour1",
-                  "sources_sha256": "35317f499ce0eb6a4afcefec55c6d33c25041cda68ff03619a611536d2715fa5",
-                  "dram_bytes": 2893401344 + 30992640}  # read + write
+                  "sources_sha256": "ef162c2d43d35d7063f4b7fac93ada9a0d71705e7ca959ea4c1861203a5782b7",
+                  "dram_bytes": 2893943296 + 26276864}  # read + write
 SCORE_SOURCES = ("ss_score.cu", "ss_internal.cuh", "ss_device.cuh")
 
 
