@@ -53,18 +53,22 @@ __global__ void __launch_bounds__(256) k_sample(const __grid_constant__ Batch B)
   const bool sampling = z < P.n_sample;
   const int64_t u = sampling ? ((int64_t)z * P.Uh) / P.n_sample : 0;
   const __nv_bfloat16* sk = P.keys + ((int64_t)slab * P.ncap + u * P.Tu) * kHeadDim;
-  // a pass's rows as 16-byte vectors, all of a thread's loads in flight at once
+  // a pass's rows as 16-byte vectors, all of a thread's loads in flight at once; the
+  // first two passes are loaded before the wait
   constexpr int kPerThread = kSampleRows * (kHeadDim / 8) / 256;
-  uint4 vbuf[kPerThread];
-  auto load_pass = [&](int rb, int nr) {
+  uint4 vbuf[kPerThread], vbuf2[kPerThread];
+  auto load_pass = [&](uint4 (&vb)[kPerThread], int rb, int nr) {
     const uint4* src = reinterpret_cast<const uint4*>(sk + (int64_t)rb * kHeadDim);
 #pragma unroll
     for (int q = 0; q < kPerThread; ++q) {
       const int x = q * 256 + tid;
-      if (x < nr * (kHeadDim / 8)) vbuf[q] = src[x];
+      if (x < nr * (kHeadDim / 8)) vb[q] = src[x];
     }
   };
-  if (sampling) load_pass(0, min(kSampleRows, P.Tu));
+  if (sampling) {
+    load_pass(vbuf, 0, min(kSampleRows, P.Tu));
+    if (P.Tu > kSampleRows) load_pass(vbuf2, kSampleRows, min(kSampleRows, P.Tu - kSampleRows));
+  }
   for (int x = tid; x < kMaxGroup * kHeadDim; x += blockDim.x) {
     const int hh = x / kHeadDim, d = x - hh * kHeadDim;
     __nv_bfloat16 qe = __float2bfloat16_rn(0.f);
@@ -119,7 +123,12 @@ __global__ void __launch_bounds__(256) k_sample(const __grid_constant__ Batch B)
     const int nr = min(kSampleRows, P.Tu - rb);
     __syncthreads();
     uint4* dst = reinterpret_cast<uint4*>(kt);
-    if (rb > 0) load_pass(rb, nr);  // the first pass was loaded before the wait
+    if (rb == kSampleRows) {
+#pragma unroll
+      for (int q = 0; q < kPerThread; ++q) vbuf[q] = vbuf2[q];
+    } else if (rb > kSampleRows) {
+      load_pass(vbuf, rb, nr);  // the first two passes were loaded before the wait
+    }
 #pragma unroll
     for (int q = 0; q < kPerThread; ++q) {
       const int x = q * 256 + tid;

@@ -637,8 +637,6 @@ cudaError_t launch_select_general(const Batch& B, int max_lists, int sm_count, c
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(1024) k_mass(const __grid_constant__ Batch B) {
   __shared__ float part[32][33];
-  pdl_wait();
-  pdl_release();
   const int pi = blockIdx.y;
   if (pi >= B.n) return;
   const Prob& P = B.p[pi];
@@ -646,10 +644,31 @@ __global__ void __launch_bounds__(1024) k_mass(const __grid_constant__ Batch B) 
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   if ((int)blockIdx.x * kMassUnits >= P.Uh) return;
   const int u = blockIdx.x * kMassUnits + lane;
+  // The per-unit pairs of the warp's first lists are loaded before the wait for the
+  // select kernel: they come from the score kernel, which completed before the select
+  // kernel started (only the lists' totals come from the select kernel).
+  constexpr int kPre = 4;
+  float2 st0[kPre];
+#pragma unroll
+  for (int i = 0; i < kPre; ++i) {
+    const int L = warp + 32 * i;
+    st0[i] = u < P.Uh && L < n_lists ? P.ustats[(int64_t)L * P.ucap + u]
+                                     : make_float2(-INFINITY, 0.f);
+  }
+  pdl_wait();
+  pdl_release();
   float acc = 0.f;
   if (u < P.Uh) {
+#pragma unroll
+    for (int i = 0; i < kPre; ++i) {
+      const int L = warp + 32 * i;
+      if (L < n_lists) {
+        const float2 m = P.list_ml[L];
+        if (st0[i].x != -INFINITY) acc += st0[i].y * fast_exp2(st0[i].x - m.x) / m.y;
+      }
+    }
 #pragma unroll 4
-    for (int L = warp; L < n_lists; L += 32) {
+    for (int L = warp + 32 * kPre; L < n_lists; L += 32) {
       const float2 st = P.ustats[(int64_t)L * P.ucap + u];
       const float2 m = P.list_ml[L];
       if (st.x != -INFINITY) acc += st.y * fast_exp2(st.x - m.x) / m.y;
