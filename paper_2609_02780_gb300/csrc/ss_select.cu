@@ -707,21 +707,21 @@ __global__ void __launch_bounds__(1024) k_pool(const __grid_constant__ Batch B) 
   __shared__ int vh[kVoteBins];
   __shared__ int sw[32];
   __shared__ int s_v, s_c, s_vmax;
-  pdl_wait();
-  pdl_release();
-  const Prob& P = B.p[blockIdx.x];
-  const int Uh = P.Uh, pn = P.pool_n;
   const int tid = threadIdx.x;
-  if (tid == 0) P.counts[0] = pn;
-  if (pn == 0) return;
-  // (1) histogram of votes (clipped): the pool's smallest vote level V is the highest
-  //     level whose units and all better ones number at least pool_n
+  // shared-memory set-up before the wait for the previous kernel
   for (int x = tid; x < kVoteBins; x += blockDim.x) vh[x] = 0;
   if (tid == 0) {
     s_c = 0;
     s_vmax = 0;
   }
-  __syncthreads();
+  pdl_wait();
+  pdl_release();
+  const Prob& P = B.p[blockIdx.x];
+  const int Uh = P.Uh, pn = P.pool_n;
+  if (tid == 0) P.counts[0] = pn;
+  if (pn == 0) return;
+  // (1) histogram of votes (clipped): the pool's smallest vote level V is the highest
+  //     level whose units and all better ones number at least pool_n
   // every thread's units' votes are loaded at once and kept for step (2)
   constexpr int kUnitsPerThread = kMaxHistUnits / 1024;
   int vt[kUnitsPerThread];
@@ -730,6 +730,7 @@ __global__ void __launch_bounds__(1024) k_pool(const __grid_constant__ Batch B) 
     const int u = q * 1024 + tid;
     vt[q] = u < Uh ? P.votes[u] : -1;
   }
+  __syncthreads();  // the zeroed bins
 #pragma unroll
   for (int q = 0; q < kUnitsPerThread; ++q) {
     if (q * 1024 >= Uh) break;
@@ -1091,11 +1092,23 @@ __global__ void __launch_bounds__(kMaxMinThreads) k_maxmin(const __grid_constant
   // warp 0 runs the greedy (its constant-cache misses stay off the serial path)
   __shared__ int* xa_ptr[4];  // sel, exp_units, frames, counts
   __shared__ int xa_int[2];   // frames per unit, n_prev
-  pdl_wait();
-  pdl_release();
   const Prob& P = B.p[blockIdx.x];
   const int pn = P.pool_n, ns = P.n_sel;
   const int tid = threadIdx.x, warp = tid >> 5;
+  // Before the wait for the Gram kernel: the pool (written by the pool kernel, which
+  // completed before the Gram kernel started) and the shared-memory set-up.
+  for (int x = tid; x < pn; x += blockDim.x) spool[x] = P.pool[x];
+  const int Uh = P.Uh;
+  const int nwords = (Uh + 31) >> 5;
+  for (int x = tid; x < nwords; x += blockDim.x) bits[x] = 0u;
+  if (tid == 32) {
+    xa_ptr[0] = P.sel;
+    xa_ptr[1] = P.exp_units;
+    xa_ptr[2] = P.frames;
+    xa_ptr[3] = P.counts;
+    xa_int[0] = P.fpu;
+    xa_int[1] = B.n_prev;
+  }
   const bool in_smem = pn <= kMaxMinSmemPool;
   const bool fixed24 = gram_fixed24(pn);
   const int hi_bytes = round16(2 * tri_entries(pn));
@@ -1108,6 +1121,10 @@ __global__ void __launch_bounds__(kMaxMinThreads) k_maxmin(const __grid_constant
   if (staged && tid == 0) {
     mbar_init(bar, 1u);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  pdl_wait();
+  pdl_release();
+  if (staged && tid == 0) {
     const uint8_t* g8 = reinterpret_cast<const uint8_t*>(P.gram);
     mbar_expect_tx(bar, (uint32_t)gram_stage_bytes(pn));
     if (in_smem) {
@@ -1116,18 +1133,6 @@ __global__ void __launch_bounds__(kMaxMinThreads) k_maxmin(const __grid_constant
       bulk_load(smem_u32(pks4), g8, (uint32_t)hi_bytes, bar);
       bulk_load(smem_u32(flo), g8 + hi_bytes, (uint32_t)round16(tri_entries(pn)), bar);
     }
-  }
-  for (int x = tid; x < pn; x += blockDim.x) spool[x] = P.pool[x];
-  const int Uh = P.Uh;
-  const int nwords = (Uh + 31) >> 5;
-  for (int x = tid; x < nwords; x += blockDim.x) bits[x] = 0u;
-  if (tid == 32) {
-    xa_ptr[0] = P.sel;
-    xa_ptr[1] = P.exp_units;
-    xa_ptr[2] = P.frames;
-    xa_ptr[3] = P.counts;
-    xa_int[0] = P.fpu;
-    xa_int[1] = B.n_prev;
   }
   __syncthreads();
   // One warp does the rest: warps parked at a barrier would slow its serial greedy.
