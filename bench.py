@@ -219,8 +219,8 @@ def run_reference(args):
 # capture summarised in profiles/k_score_dram_traffic.md; valid only for the kernel
 # sources it was taken on (their sha256 below), reported as null otherwise.
 TRAFFIC_RECORD = {"workload": "hour1",
-                  "sources_sha256": "ef162c2d43d35d7063f4b7fac93ada9a0d71705e7ca959ea4c1861203a5782b7",
-                  "dram_bytes": 2893943296 + 26276864}  # read + write
+                  "sources_sha256": "4f87011495fa30cedafb92d0876e2f247fac32d565206cf5e68006e21dde28c2",
+                  "dram_bytes": 2893074176 + 25865472}  # read + write
 SCORE_SOURCES = ("ss_score.cu", "ss_internal.cuh", "ss_device.cuh")
 
 

@@ -37,7 +37,7 @@ constexpr int kScoreThreads = (kScoreWarps + kThresholdWarps) * 32;
 #endif
 constexpr int kScoreCtasPerSm = SS_SCORE_CTAS_PER_SM;
 #ifndef SS_SCORE_STAGES
-#define SS_SCORE_STAGES 3
+#define SS_SCORE_STAGES 2
 #endif
 constexpr int kScoreStages = SS_SCORE_STAGES;  // bulk-copy stages per compute warp
 constexpr int kTileRows = 16;                  // key rows per stage (one MMA tile)
