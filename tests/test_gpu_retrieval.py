@@ -211,3 +211,12 @@ def test_maxmin_pool_sizes_across_the_gram_storage_forms():
     keys, q = gaussian_case(12, P=1, Hq=4, Hkv=1, F=420, Tf=8, R_rows=2)
     for budget in (80, 96, 105):              # pools 320, 384, 420
         run_case(keys, q, tokens_per_frame=8, k=64, budget=budget, check_e2e=False)
+
+
+def test_maxmin_pool_sizes_that_leave_lanes_past_the_pool():
+    # pools that are not a multiple of the greedy's ranks per warp: the lanes' ranks past
+    # the pool read past the end of the triangle (fp32 in shared memory: 36 and 260,
+    # fixed point: 324, global memory: 516) and must not change the selection
+    keys, q = gaussian_case(13, P=1, Hq=4, Hkv=1, F=600, Tf=8, R_rows=2)
+    for budget in (9, 65, 81, 129):           # pools 36, 260, 324, 516
+        run_case(keys, q, tokens_per_frame=8, k=64, budget=budget, check_e2e=False)
