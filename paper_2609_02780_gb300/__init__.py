@@ -311,10 +311,18 @@ class Index:
         nbytes = self.workspace_bytes(R, p)
         ws = workspace if workspace is not None else self._workspace(nbytes)
         nexp = p.budget * (1 + p.n_prev)
-        sel = torch.empty(p.budget, dtype=torch.int32).pin_memory()
-        exp = torch.empty(nexp, dtype=torch.int32).pin_memory()
-        frames = torch.empty(nexp * self.frames_per_unit, dtype=torch.int32).pin_memory()
-        counts = torch.empty(4, dtype=torch.int32).pin_memory()
+        # pinned result buffers, kept per shape (the call copies them out before returning)
+        key = (p.budget, nexp)
+        bufs = self._host_bufs.get(key) if hasattr(self, "_host_bufs") else None
+        if bufs is None:
+            bufs = (torch.empty(p.budget, dtype=torch.int32).pin_memory(),
+                    torch.empty(nexp, dtype=torch.int32).pin_memory(),
+                    torch.empty(nexp * self.frames_per_unit, dtype=torch.int32).pin_memory(),
+                    torch.empty(4, dtype=torch.int32).pin_memory())
+            if not hasattr(self, "_host_bufs"):
+                self._host_bufs = {}
+            self._host_bufs[key] = bufs
+        sel, exp, frames, counts = bufs
         hr = _abi.HostResult(sel.data_ptr(), exp.data_ptr(), frames.data_ptr(),
                              counts.data_ptr())
         with torch.cuda.device(self.device):

@@ -630,7 +630,21 @@ SS_EXPORT ss_status ss_retrieve_host(ss_index* ix, const void* q_host, int32_t R
   SS_CUDA(cudaMemcpyAsync(out->exp_units, r.exp_units, nexp * 4, cudaMemcpyDeviceToHost, st));
   SS_CUDA(cudaMemcpyAsync(out->frames, r.frames, nexp * c.frames_per_unit * 4, cudaMemcpyDeviceToHost, st));
   SS_CUDA(cudaMemcpyAsync(out->counts, r.counts, 16, cudaMemcpyDeviceToHost, st));
-  return ss_status_sync(r.status, stream);
+  // the status word comes back with the outputs (one synchronisation per call)
+  struct PinnedWord {
+    uint32_t* p = nullptr;
+    ~PinnedWord() {
+      if (p) cudaFreeHost(p);
+    }
+  };
+  static thread_local PinnedWord hstat;
+  if (!hstat.p) SS_CUDA(cudaMallocHost(reinterpret_cast<void**>(&hstat.p), sizeof(uint32_t)));
+  SS_CUDA(cudaMemcpyAsync(hstat.p, r.status, sizeof(uint32_t), cudaMemcpyDeviceToHost, st));
+  SS_CUDA(cudaStreamSynchronize(st));
+  const uint32_t v = *hstat.p;
+  if (v & kStatusTimeout) return fail(SS_ERR_TIMEOUT, "a bounded device-side wait gave up");
+  if (v & kStatusInternal) return fail(SS_ERR_INTERNAL, "a device-side consistency check failed");
+  return SS_OK;
 }
 
 // ---------------------------------------------------------------------------

@@ -10,6 +10,8 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 
+#include <map>
+#include <mutex>
 #include <utility>
 
 namespace ss {
@@ -207,6 +209,27 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+// Raises a kernel's dynamic shared-memory limit (and sets its carveout, when asked) on
+// the current device, once per larger size: the attributes persist in the context, so a
+// call that needs no more than an earlier one costs a map lookup instead of driver calls.
+inline cudaError_t ensure_smem(const void* kernel, int bytes, int carveout = -1) {
+  static std::mutex mu;
+  static std::map<std::pair<const void*, int>, int> done;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = done.find({kernel, dev});
+  if (it != done.end() && it->second >= bytes) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e != cudaSuccess) return e;
+  if (carveout >= 0) {
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, carveout);
+    if (e != cudaSuccess) return e;
+  }
+  done[{kernel, dev}] = bytes;
+  return cudaSuccess;
 }
 cudaError_t launch_prep(const Batch& B, cudaStream_t s);
 int sample_units(int k, int tokens_per_unit, int hist_units);

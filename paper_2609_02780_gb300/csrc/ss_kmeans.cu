@@ -262,7 +262,7 @@ cudaError_t launch_kmeans(const __nv_bfloat16* keys, int64_t ncap, int n_slabs,
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const size_t smem = kmeans_smem_bytes(n_c, J.Wt);
-  e = cudaFuncSetAttribute(k_kmeans, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  e = ensure_smem((const void*)k_kmeans, (int)smem);
   if (e != cudaSuccess) return e;
   k_kmeans<<<dim3(n_new, n_slabs), kKmThreads, smem, s>>>(J);
   return cudaGetLastError();

@@ -658,7 +658,7 @@ int score_slots(int sm_count) { return sm_count * kScoreCtasPerSm; }
 cudaError_t launch_score(const Batch& B, cudaStream_t s) {
   if (B.score_ctas <= 0) return cudaSuccess;
   const int smem = kScoreWarps * kScoreStages * kTileBytes;
-  cudaError_t e = cudaFuncSetAttribute(k_score, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaError_t e = ensure_smem((const void*)k_score, smem);
   if (e != cudaSuccess) return e;
   return launch_pdl(k_score, dim3(B.score_ctas), dim3(kScoreThreads), (size_t)smem, s, B);
 }

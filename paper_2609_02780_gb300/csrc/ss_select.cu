@@ -608,12 +608,8 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
 template <bool kGeneral, int kThreads>
 cudaError_t launch_select_t(const Batch& B, int max_lists, cudaStream_t s) {
   const int smem = sel_cap<kThreads>() * (int)sizeof(unsigned long long);
-  cudaError_t e = cudaFuncSetAttribute(k_select_t<kGeneral, kThreads>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  if (e != cudaSuccess) return e;
   // all of the SM's unified memory as shared memory, so that two 512-thread lists fit
-  e = cudaFuncSetAttribute(k_select_t<kGeneral, kThreads>,
-                           cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+  cudaError_t e = ensure_smem((const void*)k_select_t<kGeneral, kThreads>, smem, 100);
   if (e != cudaSuccess) return e;
   return launch_pdl(k_select_t<kGeneral, kThreads>, dim3(max_lists, B.n), dim3(kThreads),
                     (size_t)smem, s, B);
@@ -860,7 +856,7 @@ cudaError_t launch_pool(const Batch& B, int max_hist_units, cudaStream_t s) {
   while (n2 < max_hist_units) n2 <<= 1;
   const int smem = max(n2, kRankMax) * (int)(sizeof(unsigned long long) + sizeof(int)) +
                    kRankMax * (int)sizeof(int);
-  cudaError_t e = cudaFuncSetAttribute(k_pool, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaError_t e = ensure_smem((const void*)k_pool, smem);
   if (e != cudaSuccess) return e;
   return launch_pdl(k_pool, dim3(B.n), dim3(1024), (size_t)smem, s, B);
 }
@@ -1215,7 +1211,7 @@ cudaError_t launch_maxmin(const Batch& B, int max_pool, cudaStream_t s) {
   if (max_pool > 0) {
     const int T = (max_pool + kGramTile - 1) / kGramTile;
     const int smem = 2 * kGramTile * (max_dim + 4) * (int)sizeof(float);
-    cudaError_t e = cudaFuncSetAttribute(k_gram, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaError_t e = ensure_smem((const void*)k_gram, smem);
     if (e != cudaSuccess) return e;
     dim3 grid(T * (T + 1) / 2, B.n);
     e = launch_pdl(k_gram, grid, dim3(kGramTile * kGramTile), (size_t)smem, s, B);
@@ -1225,7 +1221,7 @@ cudaError_t launch_maxmin(const Batch& B, int max_pool, cudaStream_t s) {
   // not monotonic across the switch to fixed point)
   int smem = 16;
   for (int j = 0; j < B.n; ++j) smem = max(smem, gram_smem_bytes(B.p[j].pool_n));
-  cudaError_t e = cudaFuncSetAttribute(k_maxmin, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaError_t e = ensure_smem((const void*)k_maxmin, smem);
   if (e != cudaSuccess) return e;
   return launch_pdl(k_maxmin, dim3(B.n), dim3(kMaxMinThreads), (size_t)smem, s, B);
 }
