@@ -240,6 +240,15 @@ def recorded_traffic(w) -> float | None:
     return float(r["dram_bytes"]) if score_sources_sha256() == r["sources_sha256"] else None
 
 
+def host_copy_bytes(budget: int, nexp: int, frames_per_unit: int) -> int:
+    """Bytes of the one device-to-host copy of ss_retrieve_host: the selection, expansion,
+    frames, counts and status regions of the workspace, each starting at a 256-byte
+    boundary, up to the end of the status word."""
+    def a256(n):
+        return (n + 255) // 256 * 256
+    return a256(4 * budget) + a256(4 * nexp) + a256(4 * nexp * frames_per_unit) + 256 + 4
+
+
 def run_ours(args):
     import numpy as np
     import torch
@@ -350,7 +359,7 @@ def run_ours(args):
         nexp = p.budget * (1 + p.n_prev)
         e2e = {"value": keys * args.steps * world / dt, "unit": UNIT,
                "h2d_bytes_per_step": int(q_pin.numel() * 2),
-               "d2h_bytes_per_step": int(4 * (p.budget + nexp + nexp * w.frames_per_unit + 4 + 1)),
+               "d2h_bytes_per_step": host_copy_bytes(p.budget, nexp, w.frames_per_unit),
                "ms_per_step": dt / args.steps * 1e3}
 
     if rank != 0:

@@ -146,7 +146,7 @@ typedef struct {
   uint32_t* status;          /* [1] device status word, 0 = ok (required) */
 } ss_result;
 
-/* Host-side outputs of ss_retrieve_host (plain host arrays, pinned for speed). */
+/* Host-side outputs of ss_retrieve_host (plain host arrays, pinned or not). */
 typedef struct {
   int32_t* sel_units;        /* [K] */
   int32_t* exp_units;        /* [K * (1 + n_prev)] */
@@ -262,10 +262,12 @@ ss_status ss_retrieve_batched(ss_index* const* indexes, const void* const* q,
                               void* workspace, size_t workspace_bytes, void* stream,
                               const ss_trace* trace);
 
-/* ss_retrieve from host memory: copies `q_host` (bf16 [P][R][Hq][d]) to the device,
- * retrieves with every result array in the workspace, copies the selection back into
- * `out` and synchronizes `stream`. Returns the device status as well (TIMEOUT or
- * INTERNAL). Errors as ss_retrieve. */
+/* ss_retrieve from host memory: copies `q_host` (bf16 [P][R][Hq][d]; pinned memory
+ * makes the copy asynchronous) to the device, retrieves with every result array in the
+ * workspace, brings the selection back with one copy into pinned memory that the
+ * library keeps per host thread (allocated on the thread's first call, at least the
+ * largest selection seen), unpacks it into `out` and synchronizes `stream`. Returns the
+ * device status as well (TIMEOUT or INTERNAL). Errors as ss_retrieve. */
 ss_status ss_retrieve_host(ss_index* index, const void* q_host, int32_t n_rows,
                            const ss_retrieve_params* params, const ss_host_result* out,
                            void* workspace, size_t workspace_bytes, void* stream);

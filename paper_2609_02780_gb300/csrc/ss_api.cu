@@ -626,24 +626,35 @@ SS_EXPORT ss_status ss_retrieve_host(ss_index* ix, const void* q_host, int32_t R
   if (s != SS_OK) return s;
   const size_t nsel = (size_t)p->budget_units;
   const size_t nexp = nsel * (1 + p->n_prev);
-  SS_CUDA(cudaMemcpyAsync(out->sel_units, r.sel_units, nsel * 4, cudaMemcpyDeviceToHost, st));
-  SS_CUDA(cudaMemcpyAsync(out->exp_units, r.exp_units, nexp * 4, cudaMemcpyDeviceToHost, st));
-  SS_CUDA(cudaMemcpyAsync(out->frames, r.frames, nexp * c.frames_per_unit * 4, cudaMemcpyDeviceToHost, st));
-  SS_CUDA(cudaMemcpyAsync(out->counts, r.counts, 16, cudaMemcpyDeviceToHost, st));
-  // the status word comes back with the outputs (one synchronisation per call)
-  struct PinnedWord {
-    uint32_t* p = nullptr;
-    ~PinnedWord() {
+  // The selection, expansion, frames, counts and status words are consecutive regions of
+  // the workspace: one copy brings them back (into pinned memory kept per host thread),
+  // then they are unpacked into the caller's buffers.
+  struct PinnedStage {
+    char* p = nullptr;
+    size_t bytes = 0;
+    ~PinnedStage() {
       if (p) cudaFreeHost(p);
     }
   };
-  static thread_local PinnedWord hstat;
-  if (!hstat.p) SS_CUDA(cudaMallocHost(reinterpret_cast<void**>(&hstat.p), sizeof(uint32_t)));
-  SS_CUDA(cudaMemcpyAsync(hstat.p, r.status, sizeof(uint32_t), cudaMemcpyDeviceToHost, st));
+  static thread_local PinnedStage stage;
+  const size_t span = l.status + sizeof(uint32_t) - l.sel;
+  if (stage.bytes < span) {
+    if (stage.p) cudaFreeHost(stage.p);
+    stage.p = nullptr;
+    stage.bytes = 0;
+    SS_CUDA(cudaMallocHost(reinterpret_cast<void**>(&stage.p), span));
+    stage.bytes = span;
+  }
+  SS_CUDA(cudaMemcpyAsync(stage.p, base + l.sel, span, cudaMemcpyDeviceToHost, st));
   SS_CUDA(cudaStreamSynchronize(st));
-  const uint32_t v = *hstat.p;
+  uint32_t v = 0;
+  std::memcpy(&v, stage.p + (l.status - l.sel), sizeof(v));
   if (v & kStatusTimeout) return fail(SS_ERR_TIMEOUT, "a bounded device-side wait gave up");
   if (v & kStatusInternal) return fail(SS_ERR_INTERNAL, "a device-side consistency check failed");
+  std::memcpy(out->sel_units, stage.p, nsel * 4);
+  std::memcpy(out->exp_units, stage.p + (l.exp_units - l.sel), nexp * 4);
+  std::memcpy(out->frames, stage.p + (l.frames - l.sel), nexp * c.frames_per_unit * 4);
+  std::memcpy(out->counts, stage.p + (l.counts - l.sel), 16);
   return SS_OK;
 }
 
