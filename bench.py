@@ -358,7 +358,9 @@ def run_ours(args):
         dt = max_over_ranks(time.perf_counter() - t0, world)
         nexp = p.budget * (1 + p.n_prev)
         e2e = {"value": keys * args.steps * world / dt, "unit": UNIT,
-               "h2d_bytes_per_step": int(q_pin.numel() * 2),
+               # the host call copies only the rows the path reads (the last one of each
+               # layer under the default LAST reading, every row otherwise)
+               "h2d_bytes_per_step": int(q_pin.numel() * 2 // (q_pin.shape[1] if p.q_agg == 0 else 1)),
                "d2h_bytes_per_step": host_copy_bytes(p.budget, nexp, w.frames_per_unit),
                "ms_per_step": dt / args.steps * 1e3}
 

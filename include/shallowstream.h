@@ -263,7 +263,8 @@ ss_status ss_retrieve_batched(ss_index* const* indexes, const void* const* q,
                               const ss_trace* trace);
 
 /* ss_retrieve from host memory: copies `q_host` (bf16 [P][R][Hq][d]; pinned memory
- * makes the copy asynchronous) to the device, retrieves with every result array in the
+ * makes the copy asynchronous; with SS_Q_LAST only each layer's last row, the only one
+ * read, is copied) to the device, retrieves with every result array in the
  * workspace, brings the selection back with one copy into pinned memory that the
  * library keeps per host thread (allocated on the thread's first call, at least the
  * largest selection seen), unpacks it into `out` and synchronizes `stream`. Returns the

@@ -615,7 +615,16 @@ SS_EXPORT ss_status ss_retrieve_host(ss_index* ix, const void* q_host, int32_t R
   char* base = static_cast<char*>(ws);
   const size_t qbytes = (size_t)c.n_layers * R * c.n_q_heads * kHeadDim * 2;
   SS_CUDA(cudaSetDevice(ix->device));
-  SS_CUDA(cudaMemcpyAsync(base + l.qstage, q_host, qbytes, cudaMemcpyHostToDevice, st));
+  if (p->q_agg == SS_Q_LAST) {
+    // only each layer's last question row is read: one strided copy of those rows
+    const size_t row = (size_t)c.n_q_heads * kHeadDim * 2;
+    SS_CUDA(cudaMemcpy2DAsync(base + l.qstage + (size_t)(R - 1) * row, (size_t)R * row,
+                              static_cast<const char*>(q_host) + (size_t)(R - 1) * row,
+                              (size_t)R * row, row, (size_t)c.n_layers,
+                              cudaMemcpyHostToDevice, st));
+  } else {
+    SS_CUDA(cudaMemcpyAsync(base + l.qstage, q_host, qbytes, cudaMemcpyHostToDevice, st));
+  }
   ss_result r{};
   r.sel_units = reinterpret_cast<int32_t*>(base + l.sel);
   r.exp_units = reinterpret_cast<int32_t*>(base + l.exp_units);
