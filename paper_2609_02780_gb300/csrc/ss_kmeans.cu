@@ -112,15 +112,22 @@ __global__ void __launch_bounds__(kKmThreads) k_kmeans(const KmJob J) {
   const int ngrp = n_c8 / 8;
   for (int it = 0; it < J.iters; ++it) {
     // ---- assign: nearest centroid of every key (tensor cores) ----
-    for (int tile = warp; tile < ntile; tile += kKmWarps) {
-      const int r0 = tile * 16 + g, r1 = r0 + 8;
-      uint4 ra[4], rb[4];
-      const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+    // a warp walks its tiles with the next tile's key fragments already in flight
+    const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+    auto load_tile = [&](int tile, uint4 (&fa)[4], uint4 (&fb)[4]) {
+      const int q0 = tile * 16 + g, q1 = q0 + 8;
 #pragma unroll
       for (int v = 0; v < 4; ++v) {
-        ra[v] = r0 < Wt ? ld_stream(X + (int64_t)r0 * kHeadDim + 8 * (4 * v + t4)) : z;
-        rb[v] = r1 < Wt ? ld_stream(X + (int64_t)r1 * kHeadDim + 8 * (4 * v + t4)) : z;
+        fa[v] = tile < ntile && q0 < Wt ? ld_stream(X + (int64_t)q0 * kHeadDim + 8 * (4 * v + t4)) : z;
+        fb[v] = tile < ntile && q1 < Wt ? ld_stream(X + (int64_t)q1 * kHeadDim + 8 * (4 * v + t4)) : z;
       }
+    };
+    uint4 ra[4], rb[4];
+    load_tile(warp, ra, rb);
+    for (int tile = warp; tile < ntile; tile += kKmWarps) {
+      const int r0 = tile * 16 + g, r1 = r0 + 8;
+      uint4 na[4], nb[4];
+      load_tile(tile + kKmWarps, na, nb);
       float bd0 = INFINITY, bd1 = INFINITY;
       int bc0 = 0, bc1 = 0;
       for (int grp = 0; grp < ngrp; ++grp) {
@@ -159,17 +166,42 @@ __global__ void __launch_bounds__(kKmThreads) k_kmeans(const KmJob J) {
         if (r0 < Wt) a[r0] = (uint8_t)bc0;
         if (r1 < Wt) a[r1] = (uint8_t)bc1;
       }
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        ra[v] = na[v];
+        rb[v] = nb[v];
+      }
     }
     __syncthreads();
     // ---- update: fp32 sums in token order; warp w owns centroids w, w + 8, ... ----
     for (int x = tid; x < n_c8 * kHeadDim; x += blockDim.x) S[x] = 0.f;
     for (int c = tid; c < n_c8; c += blockDim.x) cnt[c] = 0;
     __syncthreads();
+    // the chunks pass through shared memory in token order; each thread's share of the
+    // next chunk is loaded into registers while the current one is summed
+    constexpr int kPer = kKmChunk * 16 / kKmThreads;
+    uint4 nxt[kPer];
+    auto load_chunk = [&](int q0) {
+      const int nr = min(kKmChunk, Wt - q0);
+#pragma unroll
+      for (int e = 0; e < kPer; ++e) {
+        const int x = e * kKmThreads + tid;
+        if (q0 < Wt && x < nr * 16) nxt[e] = ld_stream(X + (int64_t)q0 * kHeadDim + 8 * x);
+      }
+    };
+    auto store_chunk = [&](int q0) {
+      const int nr = min(kKmChunk, Wt - q0);
+#pragma unroll
+      for (int e = 0; e < kPer; ++e) {
+        const int x = e * kKmThreads + tid;
+        if (q0 < Wt && x < nr * 16) reinterpret_cast<uint4*>(chunk)[x] = nxt[e];
+      }
+    };
+    load_chunk(0);
+    store_chunk(0);
     for (int p0 = 0; p0 < Wt; p0 += kKmChunk) {
       const int nrow = min(kKmChunk, Wt - p0);
-      for (int x = tid; x < nrow * 16; x += blockDim.x)
-        reinterpret_cast<uint4*>(chunk)[x] =
-            ld_stream(X + (int64_t)p0 * kHeadDim + 8 * x);
+      load_chunk(p0 + kKmChunk);
       __syncthreads();
       for (int c = warp; c < n_c; c += kKmWarps) {
         float4 acc = *reinterpret_cast<const float4*>(S + c * kHeadDim + 4 * lane);
@@ -192,6 +224,7 @@ __global__ void __launch_bounds__(kKmThreads) k_kmeans(const KmJob J) {
         if (lane == 0) cnt[c] += n;
       }
       __syncthreads();
+      store_chunk(p0 + kKmChunk);
     }
     for (int x = tid; x < n_c * kHeadDim; x += blockDim.x) {
       const int c = x >> 7;
