@@ -219,8 +219,8 @@ def run_reference(args):
 # capture summarised in profiles/k_score_dram_traffic.md; valid only for the kernel
 # sources it was taken on (their sha256 below), reported as null otherwise.
 TRAFFIC_RECORD = {"workload": "hour1",
-                  "sources_sha256": "a1000e207f05c2908f5272c23fce106b66d70fcd2f7bb87b5b316065bf9a6186",
-                  "dram_bytes": 2892953600 + 25359872}  # read + write
+                  "sources_sha256": "ccd64b2df9c8db37f476b6b0aecc761ffbb0d7b2f306cd603548475c94679c10",
+                  "dram_bytes": 2892998144 + 25918208}  # read + write
 SCORE_SOURCES = ("ss_score.cu", "ss_internal.cuh", "ss_device.cuh")
 
 

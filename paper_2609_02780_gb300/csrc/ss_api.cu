@@ -98,7 +98,7 @@ int64_t cand_cap_of(const ss_index* ix) {
 // Workspace regions of one problem (offsets from the problem's base).
 struct Layout {
   size_t qeff, cand_s, cand_id, cand_cnt, gthr, ladder, samp_max, ustats, next_unit, gram;
-  size_t raw_units, raw_rank, cw, head_ml, aval, aid;  // general path only
+  size_t raw_units, raw_rank, cw, csel, head_ml, aval, aid;  // general path only
   size_t topk_tok, topk_w, list_ml, votes, mass, pool, sel, exp_units, frames, counts,
       status, qstage;
   size_t total;
@@ -145,6 +145,7 @@ Layout layout_of(const ss_index* ix, int R, const ss_retrieve_params* p) {
     l.raw_units = take(ix->ucap * 4);
     l.raw_rank = take(ix->ucap * 4);
     l.cw = take((size_t)c.n_layers * c.n_kv_heads * ix->wcap * ix->n_centroids * 4);
+    l.csel = take((size_t)c.n_layers * c.n_kv_heads * ix->wcap * ix->n_centroids * 4);
   }
   if (p->head_agg == SS_H_MEAN) {
     l.head_ml = take(score_lists * 8);
@@ -297,6 +298,7 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
         P.raw_units = reinterpret_cast<int32_t*>(base + l.raw_units);
         P.raw_rank = reinterpret_cast<int32_t*>(base + l.raw_rank);
         P.cw = reinterpret_cast<float*>(base + l.cw);
+        P.csel = reinterpret_cast<int32_t*>(base + l.csel);
       }
       P.n_raw_tok = (int)((P.Uh - covered) * P.Tu);
       P.n_cand = (int)(P.n_raw_tok + n_live * P.n_c);

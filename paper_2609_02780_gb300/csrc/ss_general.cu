@@ -84,6 +84,12 @@ __global__ void __launch_bounds__(kDenseWarps * 32) k_dense(const __grid_constan
   if (slab >= P.P * P.Hkv) return;
   const bool clusters = B.use_clusters != 0;
   const bool mean = B.head_agg == 1;
+  if (clusters) {
+    // this call's per-centroid selection counts start at zero (the select kernel adds)
+    const int per_slab = P.wcap * P.n_c;
+    for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < per_slab; e += gridDim.x * blockDim.x)
+      P.csel[(int64_t)slab * per_slab + e] = 0;
+  }
   const int i = slab / P.Hkv, gk = slab - i * P.Hkv, G = P.G;
   const int list0 = i * P.Hq + gk * G;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -233,15 +239,31 @@ __global__ void __launch_bounds__(256) k_mass_general(const __grid_constant__ Ba
         acc += fast_exp2(P.cand_s[(int64_t)L * P.cand_cap + j0 + r] - ml.x) * (1.0f / ml.y);
       }
     } else {
+      // a compressed unit: its mass and its votes, both from the window's centroids (a
+      // centroid's weight shared by member count; one vote per member token for every
+      // list that selected the centroid)
       const int w = P.win_slot[u / P.wu];
       const int x = u - P.win_u0[w];
       const int n_c = P.n_c;
+      int vs = 0;
       for (int t = tid; t < P.P * P.Hkv * n_c; t += blockDim.x) {
         const int slab = t / n_c, c = t - slab * n_c;
         const int64_t wc = ((int64_t)slab * P.wcap + w) * n_c + c;
         const int m = P.mcnt[wc * P.wu + x];
-        if (m) acc += P.cw[wc] * (float)m / (float)P.msize[wc];
+        if (m) {
+          acc += P.cw[wc] * (float)m / (float)P.msize[wc];
+          vs += P.csel[wc] * m;
+        }
       }
+      // integer block sum (exact in any order)
+      __shared__ int svs;
+      if (tid == 0) svs = 0;
+      __syncthreads();
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) vs += __shfl_down_sync(0xffffffffu, vs, off);
+      if ((tid & 31) == 0 && vs) atomicAdd(&svs, vs);
+      __syncthreads();
+      if (tid == 0) P.votes[u] = svs;
     }
   }
   acc = block_sum(acc, sm);

@@ -117,6 +117,8 @@ struct Prob {
   int32_t* raw_rank;           // [ucap] position of a unit in raw_units, or -1
   float* cw;                   // [P*Hkv][wcap*n_c] summed weight of each centroid over
                                // the G lists of its slab
+  int32_t* csel;               // [P*Hkv][wcap*n_c] lists of its slab that selected each
+                               // centroid
   float2* head_ml;             // [P*Hq] (M, L) of each head's softmax (one list per layer)
   float* aval;                 // [P][cand_cap] head-averaged weight of every token
   int32_t* aid;                // [P][cand_cap]

@@ -587,15 +587,11 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
       if (id >= 0 && (uint32_t)id < kCentroidIdBase) {
         if (id / P.Tu < P.Uh) atomicAdd(&P.votes[id / P.Tu], 1);
       } else if (kGeneral && id >= 0) {
-        // a centroid: one vote per member token, to the member's unit
+        // a centroid: its slab's count of lists that selected it (each selection is one
+        // vote per member token, cast per unit by the mass kernel)
         const int e = id - (int)kCentroidIdBase, w = e / P.n_c, c = e - w * P.n_c;
         const int slab = (L / P.Hq) * P.Hkv + (L % P.Hq) / P.G;
-        const int32_t* mc = P.mcnt + (((int64_t)slab * P.wcap + w) * P.n_c + c) * P.wu;
-        const int u0 = P.win_u0[w];
-        for (int x = 0; x < P.wu; ++x) {
-          const int m = mc[x];
-          if (m && u0 + x < P.Uh) atomicAdd(&P.votes[u0 + x], m);
-        }
+        atomicAdd(P.csel + ((int64_t)slab * P.wcap + w) * P.n_c + c, 1);
       }
     } else {
       tok_out[r] = -1;
