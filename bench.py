@@ -219,8 +219,8 @@ def run_reference(args):
 # capture summarised in profiles/k_score_dram_traffic.md; valid only for the kernel
 # sources it was taken on (their sha256 below), reported as null otherwise.
 TRAFFIC_RECORD = {"workload": "hour1",
-                  "sources_sha256": "ccd64b2df9c8db37f476b6b0aecc761ffbb0d7b2f306cd603548475c94679c10",
-                  "dram_bytes": 2892998144 + 25918208}  # read + write
+                  "sources_sha256": "eeb1a0dd68295312e854fb9683aaabfdd1343078e307fc056375dee7bd6c4abf",
+                  "dram_bytes": 2891569152 + 23497984}  # read + write
 SCORE_SOURCES = ("ss_score.cu", "ss_internal.cuh", "ss_device.cuh")
 
 

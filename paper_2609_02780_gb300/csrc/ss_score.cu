@@ -219,8 +219,10 @@ cudaError_t launch_prep(const Batch& B, cudaStream_t s) {
 // Each unit's softmax statistics (max, sum 2^(s - max)) are written per list; the
 // list totals are combined later in unit order, whichever warp scored a unit.
 // ---------------------------------------------------------------------------
-constexpr int kUnitQueue = 8;
-constexpr int kStagePairs = 16;  // staged candidates per (warp, list) before a write-out  // > units a warp's issue cursor can run ahead
+constexpr int kUnitQueue = 8;    // > units a warp's issue cursor can run ahead
+constexpr int kStagePairs = 64;  // staged candidates per (warp, list) before a write-out
+static_assert(kStagePairs <= kReserve, "a write-out overflows into one new slot block");
+static_assert(kStagePairs < 256, "staged counts are packed in 8 bits");
 
 struct ScoreShared {
   int lad[kMaxGroup][kLadderLevels];  // this CTA's appended-score counts not yet merged
