@@ -93,11 +93,14 @@ def whole_job_rate(units_per_step_per_rank: int, steps: int, world: int,
 
 
 class ClockSampler:
-    """nvidia-smi clock / throttle samples while the timed region runs."""
+    """nvidia-smi clock / throttle samples around the timed region. The sampler starts
+    before the warm-up (so that nvidia-smi's start-up is not inside the region) and keeps
+    the samples stamped within one sampling period of the region."""
 
-    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    QUERY = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    PERIOD_S = 0.1
 
     def __init__(self, gpu_index: int):
         self.gpu = gpu_index
@@ -108,7 +111,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
-                 "--format=csv,noheader,nounits", "-lms", "100"],
+                 "--format=csv,noheader,nounits", "-lms", str(int(self.PERIOD_S * 1000))],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.thread = threading.Thread(target=self._read, daemon=True)
             self.thread.start()
@@ -119,7 +122,32 @@ class ClockSampler:
         for line in self.proc.stdout:
             self.lines.append(line.strip())
 
-    def stop(self) -> dict:
+    @staticmethod
+    def parse(lines: list[str], t0: float | None = None, t1: float | None = None,
+              pad: float = 0.1) -> dict:
+        """Median SM clock, max clock and active throttle reasons of the samples stamped
+        in [t0 - pad, t1 + pad] (host epoch seconds), or of all samples if none is."""
+        import datetime
+        rows = []
+        for ln in lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 10:
+                continue
+            try:
+                ts = datetime.datetime.strptime(f[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+                rows.append((ts, float(f[2]), float(f[3]), f[6:10]))
+            except ValueError:
+                continue
+        inside = [r for r in rows if t0 is None or t0 - pad <= r[0] <= t1 + pad]
+        use = inside or rows
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = {nm for r in use for nm, v in zip(names, r[3]) if v.lower() == "active"}
+        return {"sm_mhz": statistics.median(r[1] for r in use) if use else None,
+                "sm_max_mhz": max(r[2] for r in use) if use else None,
+                "reasons": sorted(reasons), "samples": len(use),
+                "window": "timed region" if inside else "whole run"}
+
+    def stop(self, t0: float | None = None, t1: float | None = None) -> dict:
         if self.proc is None:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
         self.proc.terminate()
@@ -127,23 +155,7 @@ class ClockSampler:
             self.proc.wait(timeout=5)
         except subprocess.TimeoutExpired:
             self.proc.kill()
-        sm, mx, reasons = [], [], set()
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for ln in self.lines:
-            f = [x.strip() for x in ln.split(",")]
-            if len(f) < 9:
-                continue
-            try:
-                sm.append(float(f[1]))
-                mx.append(float(f[2]))
-            except ValueError:
-                continue
-            for nm, v in zip(names, f[5:9]):
-                if v.lower() == "active":
-                    reasons.add(nm)
-        return {"sm_mhz": statistics.median(sm) if sm else None,
-                "sm_max_mhz": max(mx) if mx else None,
-                "reasons": sorted(reasons), "samples": len(sm)}
+        return self.parse(self.lines, t0, t1, self.PERIOD_S)
 
 
 def measured_peak_gbs() -> tuple[float, str]:
@@ -312,14 +324,15 @@ def run_ours(args):
     def step(tr=None):
         ss.retrieve_batched(idxs, qs, p, outs=outs, workspace=ws, trace=tr)
 
+    clocks = ClockSampler(local)
+    clocks.start()
     for _ in range(max(3, args.warmup)):
         step()
     for o in outs:
         o.check()
-    clocks = ClockSampler(local)
     barrier(world)
     torch.cuda.synchronize(dev)
-    clocks.start()
+    wall0 = time.time()
     t_all0 = torch.cuda.Event(enable_timing=True)
     t_all1 = torch.cuda.Event(enable_timing=True)
     t_all0.record(stream)
@@ -328,13 +341,14 @@ def run_ours(args):
         step((k_begin[j], k_end[j]) if i % TRACE_EVERY == 0 else None)
     t_all1.record(stream)
     torch.cuda.synchronize(dev)
+    wall1 = time.time()
     barrier(world)
     for i in range(n_lat):
         s_begin[i].record(stream)
         step()
         s_end[i].record(stream)
     torch.cuda.synchronize(dev)
-    clk = clocks.stop()
+    clk = clocks.stop(wall0, wall1)
     for o in outs:
         o.check()
     total_ms = t_all0.elapsed_time(t_all1)

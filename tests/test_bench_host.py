@@ -1,0 +1,42 @@
+"""Host-side pieces of bench.py that need no GPU: the clock record of the timed region
+and the byte count of the host call's device-to-host copy."""
+import datetime
+import os
+import sys
+import time
+
+sys.path.insert(0, os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
+
+
+def _line(t, sm, reasons):
+    ts = datetime.datetime.fromtimestamp(t).strftime("%Y/%m/%d %H:%M:%S.%f")[:-3]
+    flags = ", ".join("Active" if r else "Not Active" for r in reasons)
+    return f"{ts}, 0, {sm}, 2070, 1000.0, 0x0, {flags}"
+
+
+def test_clock_samples_are_those_of_the_timed_region():
+    import bench
+    t = time.time()
+    lines = [_line(t - 2.0, 1000, (1, 0, 0, 0)),   # warm-up, throttled: not in the region
+             _line(t, 2070, (0, 0, 0, 1)),
+             _line(t + 0.05, 2050, (0, 0, 0, 0)),
+             _line(t + 2.0, 900, (0, 1, 0, 0))]    # after the region
+    c = bench.ClockSampler.parse(lines, t - 0.01, t + 0.06, pad=0.1)
+    assert c["samples"] == 2 and c["window"] == "timed region"
+    assert c["sm_mhz"] == 2060.0 and c["sm_max_mhz"] == 2070.0
+    assert c["reasons"] == ["sw_power_cap"]
+
+
+def test_clock_record_falls_back_to_the_whole_run():
+    import bench
+    t = time.time()
+    lines = [_line(t - 2.0, 1800, (0, 0, 0, 0)), "garbage", _line(t + 2.0, 2070, (0, 0, 0, 0))]
+    c = bench.ClockSampler.parse(lines, t, t + 0.01, pad=0.1)
+    assert c["samples"] == 2 and c["window"] == "whole run" and c["sm_mhz"] == 1935.0
+
+
+def test_host_copy_bytes_follow_the_workspace_alignment():
+    import bench
+    # hour1: K = 64, n_prev = 1, one frame per unit
+    assert bench.host_copy_bytes(64, 128, 1) == 256 + 512 + 512 + 256 + 4
+    assert bench.host_copy_bytes(1, 2, 2) == 256 + 256 + 256 + 256 + 4
