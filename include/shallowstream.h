@@ -281,7 +281,9 @@ ss_status ss_retrieve_host(ss_index* index, const void* q_host, int32_t n_rows,
  * implicit device synchronisation. The workspace is a fixed 64 MiB array in the
  * library's device memory (one per device, reserved when the library's device code is
  * loaded). The first call on each device looks up that array's address with the
- * device current (one-time set-up); make that first call before any stream capture.
+ * device current (one-time set-up, repeated only if the device's context is destroyed
+ * and made again, as cudaDeviceReset does); make that first call before any stream
+ * capture.
  * Nothing in the scratch has to start at zero: the first kernel of every call resets
  * the counters that later kernels accumulate into. Every call on a device uses the same
  * scratch, so calls that overlap (other streams or host threads on that device, before
@@ -293,6 +295,16 @@ ss_status ss_retrieve_host(ss_index* index, const void* q_host, int32_t n_rows,
 ss_status ss_retrieve_static(ss_index* index, const void* q, int32_t n_rows,
                              const ss_retrieve_params* params, const ss_result* result,
                              void* stream);
+
+/* Sets how long the key-scoring kernel's waits for its key copies may take before
+ * they give up: `polls` polls of the copy's barrier (each wait also gives up after about
+ * one second), or -1 for the default (2^26 polls). A wait that gives up records
+ * SS_ERR_TIMEOUT in the retrieval's status word, lets its copies in flight land and
+ * ends its warp; the retrieval's later kernels then skip their work and leave the
+ * counts at 0. 0 makes every such wait give up at once, which makes the failure path
+ * testable without a fault. Process-wide; takes effect for retrievals issued after the
+ * call. Errors: INVALID_ARG (polls < -1 or >= 2^32). */
+ss_status ss_set_wait_limit(int64_t polls);
 
 /* Synchronizes `stream` and returns the status recorded in the device word `status`
  * by earlier retrievals on it (SS_OK, SS_ERR_TIMEOUT or SS_ERR_INTERNAL). */

@@ -15,10 +15,13 @@ scored by Eq. 13) is the closest text; the token-level k-means reading is:
       update  c = mean of its members; a centroid with no members keeps its value.
     Members are the last round's assignment; the stored centroid is the last
     round's mean rounded to bf16.
+  * Windows start on multiples of W frames but need not be adjacent: compressions
+    made one after another can leave raw frames before, between and after them.
   * Retrieval candidates of a list: the centroids of every compressed window whose
     first unit is in the history, and the raw tokens of the history units that no
     compressed window covers. Softmax over all of them; top-k by (score desc, id
-    asc) with centroid (w, c) given id CID_BASE + w * n_c + c, after all token ids.
+    asc) with centroid (w, c) given id CID_BASE + w * n_c + c, after all token ids
+    (w counts windows in the order they were compressed).
   * A selected centroid gives one vote to each member token's unit (history units
     only); its weight is apportioned to units by member share |members in u| /
     |members|. Empty centroids stay candidates but vote for nothing.
@@ -87,24 +90,40 @@ def compress(key_bits: np.ndarray, *, tokens_per_frame: int, first_frame: int,
                 C[i, g, w], A[i, g, w] = lloyd(X, n_centroids, iters)
     bits = f32_to_bf16_rne(C.astype(np.float32))
     return {"centroids": C, "centroid_bits": bits, "assign": A,
-            "first_frame": first_frame, "window_frames": window_frames}
+            "first_frame": first_frame, "window_frames": window_frames,
+            "window_first_frames": [first_frame + w * window_frames for w in range(n_w)]}
 
 
-def _member_units(A, i, g, w, c, f0, WF, tokens_per_frame, tokens_per_unit):
-    """Units of the member tokens of centroid c of window w at (layer i, key head g)."""
+def window_first_frames(comp: dict, n_windows: int) -> list[int]:
+    """First frame of every window: comp["window_first_frames"] when given (windows of
+    several compressions), else adjacent windows from comp["first_frame"]."""
+    if "window_first_frames" in comp:
+        f = [int(x) for x in comp["window_first_frames"]]
+        if len(f) != n_windows:
+            raise ValueError("one first frame per window is needed")
+        return f
+    return [int(comp["first_frame"]) + w * int(comp["window_frames"]) for w in range(n_windows)]
+
+
+def _member_units(A, i, g, w, c, win_f0, tokens_per_frame, tokens_per_unit):
+    """Units of the member tokens of centroid c of window w (first frame win_f0[w]) at
+    (layer i, key head g)."""
     m = np.nonzero(A[i, g, w] == c)[0]
-    t = (f0 + w * WF) * tokens_per_frame + m
+    t = win_f0[w] * tokens_per_frame + m
     return t // tokens_per_unit
 
 
 def compressed_votes(tok: np.ndarray, A: np.ndarray, *, n_q_heads: int, n_kv_heads: int,
-                     n_centroids: int, first_frame: int, window_frames: int,
-                     tokens_per_frame: int, tokens_per_unit: int,
-                     n_hist_units: int) -> np.ndarray:
+                     n_centroids: int, window_frames: int, tokens_per_frame: int,
+                     tokens_per_unit: int, n_hist_units: int, first_frame: int = 0,
+                     window_first: list[int] | None = None) -> np.ndarray:
     """Unit votes of per-(layer, query head) lists that mix token ids and centroid ids:
     a token votes for its unit, a centroid once for the unit of each member token
-    (history units only). A: assignments [P][Hkv][n_w][W * T_f]."""
+    (history units only). A: assignments [P][Hkv][n_w][W * T_f]; window_first: the
+    first frame of every window (default: adjacent windows from first_frame)."""
     G = n_q_heads // n_kv_heads
+    if window_first is None:
+        window_first = [first_frame + w * window_frames for w in range(A.shape[2])]
     votes = np.zeros(n_hist_units, dtype=np.int64)
     for li in range(tok.shape[0]):
         i, g = li // n_q_heads, (li % n_q_heads) // G
@@ -116,8 +135,8 @@ def compressed_votes(tok: np.ndarray, A: np.ndarray, *, n_q_heads: int, n_kv_hea
                 votes[cand // tokens_per_unit] += 1
                 continue
             w, c = divmod(cand - CID_BASE, n_centroids)
-            for u in _member_units(A, i, g, w, c, first_frame, window_frames,
-                                   tokens_per_frame, tokens_per_unit):
+            for u in _member_units(A, i, g, w, c, window_first, tokens_per_frame,
+                                   tokens_per_unit):
                 if u < n_hist_units:
                     votes[u] += 1
     return votes
@@ -146,14 +165,14 @@ def retrieve_compressed(key_bits: np.ndarray, q_bits: np.ndarray, comp: dict, *,
     A = comp["assign"] if assignment is None else assignment
     n_w, n_c = cb.shape[2], cb.shape[3]
     WF = comp["window_frames"]
-    f0 = comp["first_frame"]
+    win_f0 = window_first_frames(comp, n_w)
     U_h = history_units(n_units, n_recent)
     if desc is None:
         desc = descriptors(key_bits, n_units, tokens_per_unit)
     qe = query_effective(q_bits, q_agg)
 
     # windows as unit ranges; which are candidates; which units stay detailed
-    win_u0 = [(f0 + w * WF) // frames_per_unit for w in range(n_w)]
+    win_u0 = [f // frames_per_unit for f in win_f0]
     win_nu = WF // frames_per_unit
     covered = np.zeros(max(n_units, 1), dtype=bool)
     for u0 in win_u0:
@@ -188,7 +207,7 @@ def retrieve_compressed(key_bits: np.ndarray, q_bits: np.ndarray, comp: dict, *,
     tw = np.take_along_axis(w_all, pos, axis=1)
 
     votes = compressed_votes(tok, A, n_q_heads=Hq, n_kv_heads=Hkv, n_centroids=n_c,
-                             first_frame=f0, window_frames=WF,
+                             window_frames=WF, window_first=win_f0,
                              tokens_per_frame=tokens_per_frame,
                              tokens_per_unit=tokens_per_unit, n_hist_units=U_h)
     # mass: raw weights to their unit, centroid weights by member share
@@ -202,7 +221,7 @@ def retrieve_compressed(key_bits: np.ndarray, q_bits: np.ndarray, comp: dict, *,
 
     def share_of(i, g, w):
         if (i, g, w) not in shares:
-            t0 = (f0 + w * WF) * tokens_per_frame
+            t0 = win_f0[w] * tokens_per_frame
             u = (t0 + np.arange(Wt)) // tokens_per_unit
             u_first = int(u[0])
             cnt = np.zeros((n_c, int(u[-1]) - u_first + 1), dtype=np.float64)

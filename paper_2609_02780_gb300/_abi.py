@@ -87,6 +87,7 @@ SIGNATURES = {
                                       C.POINTER(RetrieveParams), C.POINTER(Result),
                                       C.c_void_p]),
     "ss_status_sync": (c_status, [C.c_void_p, C.c_void_p]),
+    "ss_set_wait_limit": (c_status, [C.c_int64]),
 }
 
 _LIB = None

@@ -1,10 +1,13 @@
 // C ABI of the library (include/shallowstream.h): argument validation, device memory
 // of the index, workspace layout and the launch sequence of one retrieval.
+#include <atomic>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
 #include <mutex>
 #include <vector>
+
+#include <cuda.h>
 
 #include "shallowstream.h"
 #include "ss_internal.cuh"
@@ -42,6 +45,9 @@ struct ss_index {
 namespace {
 
 thread_local char g_err[512] = "";
+
+// Polls after which the score kernel's waits for its key copies give up (process-wide).
+std::atomic<uint32_t> g_wait_polls{kDefaultWaitPolls};
 
 ss_status fail(ss_status s, const char* fmt, ...) {
   va_list ap;
@@ -223,6 +229,7 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
   B.q_agg = p->q_agg;
   B.head_agg = p->head_agg;
   B.use_clusters = p->use_clusters;
+  B.wait_polls = g_wait_polls.load(std::memory_order_relaxed);
   const bool general = p->head_agg == SS_H_MEAN || p->use_clusters;
   int max_lists = 0, max_uh = 0, max_pool = 0, n_slabs_total = 0;
   int max_cand = 0, max_slabs = 0, max_score_lists = 0, max_cent = 0;
@@ -372,7 +379,14 @@ SS_EXPORT const char* ss_status_string(ss_status s) {
 
 SS_EXPORT const char* ss_last_error(void) { return g_err; }
 
-SS_EXPORT const char* ss_version(void) { return "shallowstream-gb300 0.1 (sm_103a)"; }
+SS_EXPORT const char* ss_version(void) { return "shallowstream-gb300 0.2 (sm_103a)"; }
+
+SS_EXPORT ss_status ss_set_wait_limit(int64_t polls) {
+  if (polls < -1 || polls > (int64_t)UINT32_MAX)
+    return fail(SS_ERR_INVALID_ARG, "polls must be -1 (default) or in [0, 2^32)");
+  g_wait_polls.store(polls < 0 ? kDefaultWaitPolls : (uint32_t)polls, std::memory_order_relaxed);
+  return SS_OK;
+}
 
 SS_EXPORT ss_status ss_index_create(const ss_index_config* cfg, const ss_allocator* alloc,
                                     void* stream, ss_index** out) {
@@ -687,20 +701,47 @@ __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
 
 std::mutex g_static_mu;
 void* g_static_ptr[kMaxStaticDevices] = {};
+void* g_static_ctx[kMaxStaticDevices] = {};   // the context each address belongs to
 
-// The scratch's device address on `dev` (which must be current); looked up once per
-// device, on that device's first call.
+// The current CUDA context (driver cuCtxGetCurrent, found through the runtime so that
+// the library needs no link to the driver library).
+ss_status current_context(void** ctx) {
+  using Fn = CUresult (*)(CUcontext*);
+  static Fn fn = nullptr;
+  if (!fn) {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    const cudaError_t e = cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 12000,
+                                                           cudaEnableDefault, &q);
+    if (e != cudaSuccess || !f || q != cudaDriverEntryPointSuccess)
+      return fail(SS_ERR_CUDA, "cuCtxGetCurrent is not available");
+    fn = reinterpret_cast<Fn>(f);
+  }
+  CUcontext c = nullptr;
+  if (fn(&c) != CUDA_SUCCESS || !c) return fail(SS_ERR_CUDA, "no current CUDA context");
+  *ctx = c;
+  return SS_OK;
+}
+
+// The scratch's device address on `dev` (which must be current). It is looked up on the
+// first call in each CUDA context of the device: once per device, unless the device's
+// context is destroyed and made again (cudaDeviceReset), which loads the library's
+// device code again at another address.
 ss_status static_scratch(int dev, void** out) {
   if (dev < 0 || dev >= kMaxStaticDevices)
     return fail(SS_ERR_UNSUPPORTED, "device %d: static scratch supports devices [0, %d)", dev,
                 kMaxStaticDevices);
   std::lock_guard<std::mutex> lock(g_static_mu);
-  if (!g_static_ptr[dev]) {
+  void* ctx = nullptr;
+  ss_status s = current_context(&ctx);
+  if (s != SS_OK) return s;
+  if (!g_static_ptr[dev] || g_static_ctx[dev] != ctx) {
     void* p = nullptr;
     const cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch);
     if (e != cudaSuccess)
       return fail(SS_ERR_CUDA, "cudaGetSymbolAddress(static scratch): %s", cudaGetErrorString(e));
     g_static_ptr[dev] = p;
+    g_static_ctx[dev] = ctx;
   }
   *out = g_static_ptr[dev];
   return SS_OK;

@@ -65,15 +65,21 @@ __device__ __forceinline__ uint64_t global_ns() {
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
   return t;
 }
-// Bounded wait for a stage's bulk copy: gives up after ~1 s (or 2^26 polls).
-static __device__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity) {
+// Bounded wait for a phase of an mbarrier: gives up after `polls` polls or ~1 s,
+// whichever comes first (0 polls: gives up at once, without looking).
+static __device__ bool mbar_wait_limit(uint32_t bar, uint32_t parity, uint32_t polls) {
+  if (polls == 0u) return false;
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_ns();
-  for (uint32_t i = 1; i < (1u << 26); ++i) {
+  for (uint32_t i = 1; i < polls; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((i & 1023u) == 0u && global_ns() - t0 > 1000000000ull) break;
   }
   return false;
+}
+// The default limit: 2^26 polls or ~1 s.
+static __device__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity) {
+  return mbar_wait_limit(bar, parity, kDefaultWaitPolls);
 }
 
 // ---- fixed-order block reductions (deterministic) ----

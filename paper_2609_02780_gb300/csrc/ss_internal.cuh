@@ -59,6 +59,8 @@ constexpr int kMaxChunksPerSlab = 128;
 // Device status word bits (ss_result::status).
 constexpr uint32_t kStatusInternal = 1u;
 constexpr uint32_t kStatusTimeout = 2u;
+// Polls after which a bounded wait gives up (it also gives up after ~1 s).
+constexpr uint32_t kDefaultWaitPolls = 1u << 26;
 
 // log2(e) / sqrt(128): scores are kept in the log2 domain, s2 = (q.k) * kScoreScale,
 // so softmax weights are 2^(s2 - M) / L.
@@ -139,6 +141,7 @@ struct Batch {
   int use_clusters;
   int score_ctas;              // total CTAs of the score kernel
   int score_spread;            // 1: one wave; slab = CTA index mod slabs
+  uint32_t wait_polls;         // limit of the score kernel's waits for its key copies
 };
 static_assert(sizeof(Batch) <= 32000, "kernel parameter block too large");
 
@@ -184,6 +187,13 @@ __device__ __forceinline__ float list_anchor(const Prob& P, int L) {
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_release() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// True when an earlier kernel of this retrieval gave up a bounded wait: the later
+// kernels then skip their work (the caller reads SS_ERR_TIMEOUT from the status word).
+// Read after pdl_wait(): no kernel that runs at the same time writes the word.
+__device__ __forceinline__ bool retrieval_timed_out(const Prob& P) {
+  return (*(volatile const uint32_t*)P.status & kStatusTimeout) != 0u;
 }
 
 __device__ __forceinline__ int problem_of_block(const Batch& B, int b) {

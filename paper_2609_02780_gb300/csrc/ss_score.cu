@@ -553,7 +553,8 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
   bool aborted = false;
   for (; cu < Uh; ++t) {
     const int st = t % kScoreStages;
-    const bool ok = mbar_wait_bounded(my_bars + 8u * st, (uint32_t)((t / kScoreStages) & 1));
+    const bool ok = mbar_wait_limit(my_bars + 8u * st, (uint32_t)((t / kScoreStages) & 1),
+                                    B.wait_polls);
     if (!__all_sync(0xffffffffu, ok)) {
       aborted = true;
       break;
@@ -618,7 +619,8 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
   for (int x = g; x < rl0; x += 8) P.cand_pair[cbase0 + rp0 + x].x = -INFINITY;
   for (int x = g; x < rl1; x += 8) P.cand_pair[cbase1 + rp1 + x].x = -INFINITY;
   if (aborted) {
-    // report, then let the copies already in flight land before the CTA exits
+    // report, then let the copies already in flight land before the CTA exits (with the
+    // default limit: the copies were issued and complete)
     if (lane == 0) atomicOr(P.status, kStatusTimeout);
     // stages of tiles t .. t + kScoreStages - 1 that were issued (units < Uh)
     int ru = cu, rj = cj, rq = qh;

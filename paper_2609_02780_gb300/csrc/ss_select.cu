@@ -216,6 +216,7 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
   const int pi = blockIdx.y;
   if (pi >= B.n) return;
   const Prob& P = B.p[pi];
+  if (retrieval_timed_out(P)) return;
   const bool mean = kGeneral && B.head_agg == 1;  // one list per layer
   const int n_lists = mean ? P.P : P.P * P.Hq;
   const int L = blockIdx.x;
@@ -649,6 +650,7 @@ __global__ void __launch_bounds__(1024) k_mass(const __grid_constant__ Batch B) 
   }
   pdl_wait();
   pdl_release();
+  if (retrieval_timed_out(P)) return;
   float acc = 0.f;
   if (u < P.Uh) {
 #pragma unroll
@@ -709,6 +711,7 @@ __global__ void __launch_bounds__(1024) k_pool(const __grid_constant__ Batch B) 
   pdl_wait();
   pdl_release();
   const Prob& P = B.p[blockIdx.x];
+  if (retrieval_timed_out(P)) return;   // counts stay 0 (reset by the prep kernel)
   const int Uh = P.Uh, pn = P.pool_n;
   if (tid == 0) P.counts[0] = pn;
   if (pn == 0) return;
@@ -916,6 +919,7 @@ __global__ void __launch_bounds__(256) k_gram(const __grid_constant__ Batch B) {
   pdl_wait();
   pdl_release();
   const Prob& P = B.p[blockIdx.y];
+  if (retrieval_timed_out(P)) return;
   const int pn = P.pool_n;
   const int dim = P.Hkv * kHeadDim;
   const int T = (pn + kGramTile - 1) / kGramTile;
@@ -1116,6 +1120,7 @@ __global__ void __launch_bounds__(kMaxMinThreads) k_maxmin(const __grid_constant
   }
   pdl_wait();
   pdl_release();
+  if (retrieval_timed_out(P)) return;   // no copy was issued
   if (staged && tid == 0) {
     const uint8_t* g8 = reinterpret_cast<const uint8_t*>(P.gram);
     mbar_expect_tx(bar, (uint32_t)gram_stage_bytes(pn));

@@ -66,6 +66,7 @@ def _check_problem(kb, qb, gpu, w):
     qe = R.query_effective(qb, w.q_agg)
     mass = np.zeros(Uh)
     amb = 0
+    tok_ref = np.empty((P * Hq, min(w.k, n_tok)), dtype=np.int64)   # the oracle's own lists
     for i in range(P):
         for g in range(Hkv):
             s = R.scores(qe, kb, n_tok, lists=[(i, g * G + h) for h in range(G)])
@@ -77,12 +78,18 @@ def _check_problem(kb, qb, gpu, w):
                                      gpu["topk_w"][L:L + 1], wrow, w.k)
                 amb += info["ambiguous_lists"]
                 PY.check_stats(s[h:h + 1], gpu["list_stats"][L:L + 1])
+                tok_ref[L] = R.topk_rows(s[h:h + 1], w.k)[0]
             del s
-    assert np.allclose(gpu["mass"], mass, rtol=1e-4, atol=1e-7)
+    assert np.allclose(gpu["mass"], mass, rtol=PY.TOL_MASS, atol=1e-7)
     assert gpu["votes"].sum() == P * Hq * min(w.k, n_tok)
     desc = R.descriptors(kb, U, Tu)
     chain = PY.check_chain(gpu, desc, Uh, Tu, w.budget, w.pool_mult, w.n_prev,
                            w.frames_per_unit)
+    ref = R.select_from_lists(tok_ref, mass, desc, Uh, Tu, w.budget, w.pool_mult, w.n_prev,
+                              w.frames_per_unit)
+    chain["e2e"] = PY.check_end_to_end(gpu, ref, amb, desc, w.budget, w.pool_mult)
+    print(f"{w.name}: ambiguous lists {amb}, close max-min steps (GPU chain) "
+          f"{chain['close_maxmin_steps']}, {chain['e2e']}")
     return amb, chain
 
 
@@ -186,10 +193,8 @@ def test_one_hour_index_compressed():
     Uh = w.n_frames // w.frames_per_unit - w.n_recent
     Tu = w.tokens_per_frame * w.frames_per_unit
     gpu = PY.gpu_outputs(res, Uh)
-    n_w = w.n_frames // WF
-    A = cl["assignment"].cpu().numpy()[:, :, :n_w * Wt].reshape(w.n_layers, w.n_kv_heads, n_w, Wt)
-    comp = {"centroid_bits": synth.bf16_bits(cl["centroids"]), "assign": A.astype(np.int64),
-            "first_frame": 0, "window_frames": WF}
+    comp = PY.gpu_comp(cl, w.tokens_per_frame, w.frames_per_unit)
+    assert comp["window_first_frames"] == list(range(0, w.n_frames, WF))
     del data, idx, cl
     torch.cuda.empty_cache()
     desc = R.descriptors(kb, w.n_frames // w.frames_per_unit, Tu)
@@ -202,10 +207,16 @@ def test_one_hour_index_compressed():
                          ids=ref["ids"])
     PY.check_stats(ref["s"], gpu["list_stats"])
     assert np.allclose(gpu["mass"], ref["mass"], rtol=1e-3, atol=1e-7)
-    votes = KM.compressed_votes(gpu["topk_tok"], A, n_q_heads=w.n_q_heads,
-                                n_kv_heads=w.n_kv_heads, n_centroids=n_c, first_frame=0,
-                                window_frames=WF, tokens_per_frame=w.tokens_per_frame,
+    votes = KM.compressed_votes(gpu["topk_tok"], comp["assign"], n_q_heads=w.n_q_heads,
+                                n_kv_heads=w.n_kv_heads, n_centroids=n_c,
+                                window_frames=WF, window_first=comp["window_first_frames"],
+                                tokens_per_frame=w.tokens_per_frame,
                                 tokens_per_unit=Tu, n_hist_units=Uh)
-    PY.check_chain(gpu, desc, Uh, Tu, w.budget, w.pool_mult, w.n_prev, w.frames_per_unit,
-                   votes=votes)
+    chain = PY.check_chain(gpu, desc, Uh, Tu, w.budget, w.pool_mult, w.n_prev,
+                           w.frames_per_unit, votes=votes)
+    # end to end: the oracle's own lists, votes, mass, pool, selection and frames
+    e2e = PY.check_end_to_end(gpu, ref, info["ambiguous_lists"], desc, w.budget,
+                              w.pool_mult, rel_mass=1e-3)
+    print(f"hour1_kmeans: ambiguous lists {info['ambiguous_lists']}, close max-min steps "
+          f"{chain['close_maxmin_steps']}, {e2e}")
     assert info["ambiguous_lists"] <= 4

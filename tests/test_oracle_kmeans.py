@@ -1,6 +1,11 @@
 """Pins of the k-means compression oracle (oracle/kmeans.py): a library k-means on
-separated data, the identity special case, Lloyd invariants, and the reduction of
-retrieval over one-token clusters to plain token retrieval."""
+separated data, the identity special case, Lloyd invariants, the reduction of
+retrieval over one-token clusters to plain token retrieval, and a hand-worked
+retrieval over windows that start after frame 0, leave a raw gap and hold a recent
+unit (tests/golden/compressed_example.*)."""
+import json
+import os
+
 import numpy as np
 import pytest
 import torch
@@ -110,3 +115,92 @@ def test_compressed_vote_total_is_member_count():
     # candidates: 4 raw units (0, 1, 8, 9) of 8 tokens and 2 windows of 5 centroids
     assert len(out["ids"]) == 4 * 8 + 2 * 5
     assert np.allclose(out["mass"].sum(), P * Hq, atol=1e-12)   # no empty centroid here
+
+
+# ---------------------------------------------------------------- hand-worked example
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "compressed_example.json")
+
+
+def _golden():
+    with open(GOLDEN) as f:
+        g = json.load(f)
+    keys = to_bf16_bits(np.array(g["keys"], np.float32))[None, None]        # [1][1][16][4]
+    q = to_bf16_bits(np.array(g["q_last_row"], np.float32))[None, None]     # [1][1][2][4]
+    cb = to_bf16_bits(np.array(g["centroids"], np.float32))[None, None]     # [1][1][2][2][4]
+    A = np.array(g["assignment"], np.int64)[None, None]                      # [1][1][2][4]
+    comp = {"centroid_bits": cb, "assign": A, "window_frames": g["window_frames"],
+            "window_first_frames": g["window_first_frames"]}
+    sh = g["shape"]
+    kw = dict(n_units=sh["n_units"], tokens_per_unit=sh["tokens_per_frame"] * sh["frames_per_unit"],
+              frames_per_unit=sh["frames_per_unit"], tokens_per_frame=sh["tokens_per_frame"],
+              k=g["k"], pool_mult=2, n_prev=1, n_recent=sh["n_recent"])
+    return g, keys, q, comp, kw
+
+
+def test_hand_example_compressed_retrieval():
+    g, keys, q, comp, kw = _golden()
+    tol = g["tolerance"]
+    out = KM.retrieve_compressed(keys, q, comp, budget=2, **kw)
+    assert out["ids"].tolist() == g["candidate_ids"]
+    assert np.allclose(out["s"], g["scores"], atol=0, rtol=0)
+    assert out["topk_tok"].tolist() == g["topk_tok"]
+    assert np.allclose(out["topk_w"], g["topk_w"], atol=tol)
+    assert out["votes"].tolist() == g["votes"]
+    assert np.allclose(out["mass"], g["mass"], atol=tol)
+    assert abs(out["mass"].sum() - g["mass_total"]) <= tol
+    assert np.allclose(R.descriptors(keys, 8, 2), g["descriptors"], atol=tol)
+    for key in ("pool", "sel", "expanded", "frames"):
+        assert out[key].tolist() == g["budget2"][key], key
+    out3 = KM.retrieve_compressed(keys, q, comp, budget=3, **kw)
+    for key in ("pool", "sel", "expanded", "frames"):
+        assert out3[key].tolist() == g["budget3"][key], key
+
+
+def test_hand_example_compressed_votes_direct():
+    g, keys, q, comp, kw = _golden()
+    tok = np.array(g["topk_tok"], np.int64)
+    v = KM.compressed_votes(tok, comp["assign"], n_q_heads=2, n_kv_heads=1, n_centroids=2,
+                            window_frames=2, window_first=g["window_first_frames"],
+                            tokens_per_frame=2, tokens_per_unit=2, n_hist_units=7)
+    assert v.tolist() == g["votes"]
+    # the same windows placed adjacent from frame 0 put A0's votes on units 0 and 1
+    v0 = KM.compressed_votes(tok, comp["assign"], n_q_heads=2, n_kv_heads=1,
+                             n_centroids=2, window_frames=2, first_frame=0,
+                             tokens_per_frame=2, tokens_per_unit=2, n_hist_units=7)
+    assert v0.tolist() != g["votes"]
+
+
+def test_hand_example_catches_planted_mistakes(monkeypatch):
+    """Plausible mistakes in the compressed path, planted in the oracle (CPU only), each
+    fail the hand-worked values."""
+    g, keys, q, comp, kw = _golden()
+
+    def fails(**over) -> bool:
+        out = KM.retrieve_compressed(keys, q, comp, budget=2, **kw)
+        return (out["votes"].tolist() != g["votes"]
+                or not np.allclose(out["mass"], g["mass"], atol=g["tolerance"]))
+
+    assert not fails()
+    # (a) the window's first frame dropped from the member-token positions
+    orig = KM._member_units
+    monkeypatch.setattr(KM, "_member_units",
+                        lambda A, i, gg, w, c, f0, tpf, tpu: orig(A, i, gg, w, c, [0] * len(f0), tpf, tpu))
+    assert fails()
+    monkeypatch.setattr(KM, "_member_units", orig)
+    # (b) windows taken as adjacent from the first one (the raw gap ignored)
+    comp_adj = dict(comp)
+    comp_adj["window_first_frames"] = [2, 4]
+    out = KM.retrieve_compressed(keys, q, comp_adj, budget=2, **kw)
+    assert out["votes"].tolist() != g["votes"]
+    # (c) a centroid's weight spread evenly over its window's units, not by member count
+    A_even = comp["assign"].copy()
+    A_even[0, 0, 0] = [0, 1, 0, 1]            # A0 then has one member in each unit
+    comp_even = dict(comp, assign=A_even)
+    out = KM.retrieve_compressed(keys, q, comp_even, budget=2, **kw)
+    assert not np.allclose(out["mass"], g["mass"], atol=g["tolerance"])
+    # (d) members in the recent unit counted as votes
+    tok = np.array(g["topk_tok"], np.int64)
+    v8 = KM.compressed_votes(tok, comp["assign"], n_q_heads=2, n_kv_heads=1, n_centroids=2,
+                             window_frames=2, window_first=g["window_first_frames"],
+                             tokens_per_frame=2, tokens_per_unit=2, n_hist_units=8)
+    assert v8[:7].tolist() == g["votes"] and v8[7] == 2
