@@ -208,14 +208,18 @@ ss_status ss_index_get_view(const ss_index* index, ss_index_view* view);
  * (bf16, nearest-even) and memberships. Distances are compared as ||c||^2 - 2 x . c in
  * fp32 (x . c on the tensor cores with c split into two bf16 parts), so a key whose two
  * nearest centroids are within that rounding of each other may take either; the sums
- * of the update run in token order (results repeat bit for bit). The first call fixes
+ * of the update run in a fixed order (results repeat bit for bit). The first call fixes
  * window_frames and
  * n_centroids (later calls must match, with windows after those already compressed)
  * and allocates the cluster arrays from the index's allocator.
+ * With n_centroids <= 64 and windows of <= 16384 tokens the rounds run on the tcgen05
+ * tensor cores (one read of the window's keys per round; member sums accumulated by the
+ * tensor cores in a fixed order), otherwise on mma.sync tensor cores. A device-side wait
+ * of the compression that gives up (SS_ERR_TIMEOUT) is reported in the status word of
+ * every later retrieval on the index.
  * Errors: INVALID_ARG (misaligned ranges, frames not yet appended, overlap with a
  * compressed window), UNSUPPORTED (n_centroids > 128 or > window tokens, windows of more
- * than 65536 tokens), ALLOC,
- * CUDA. */
+ * than 65536 tokens), ALLOC (nothing is kept; the call can be repeated), CUDA. */
 ss_status ss_index_compress(ss_index* index, const ss_compress_params* params,
                             void* stream);
 

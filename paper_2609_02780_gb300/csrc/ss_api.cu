@@ -40,6 +40,7 @@ struct ss_index {
   int32_t* win_slot;    // [ucap / units per window]: window of each window slot, or -1
   int32_t* mcnt;        // [P*Hkv][wcap][nc][units per window] members per (centroid, unit)
   int32_t* msize;       // [P*Hkv][wcap][nc] members per centroid
+  uint32_t* kstatus;    // device word: a compression's wait gave up (kStatusTimeout)
 };
 
 namespace {
@@ -251,6 +252,7 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
     P.U = (int)x->n_units;
     P.Uh = (int)hist_units_of(x, p);
     P.ucap = (int)x->ucap;
+    P.index_status = x->kstatus;
     P.q = static_cast<const __nv_bfloat16*>(q[j]);
     P.R = R[j];
     P.qeff = reinterpret_cast<__nv_bfloat16*>(base + l.qeff);
@@ -448,6 +450,7 @@ SS_EXPORT ss_status ss_index_destroy(ss_index* ix) {
   dev_free(ix, ix->win_slot);
   dev_free(ix, ix->mcnt);
   dev_free(ix, ix->msize);
+  dev_free(ix, ix->kstatus);
   delete ix;
   return SS_OK;
 }
@@ -543,19 +546,24 @@ SS_EXPORT ss_status ss_index_compress(ss_index* ix, const ss_compress_params* cp
     ix->msize = static_cast<int32_t*>(dev_alloc(ix, sb, st));
     ix->win_u0 = static_cast<int32_t*>(dev_alloc(ix, (size_t)wcap * 4, st));
     ix->win_slot = static_cast<int32_t*>(dev_alloc(ix, (size_t)n_slots * 4, st));
-    if (!ix->cent || !ix->assign || !ix->mcnt || !ix->msize || !ix->win_u0 || !ix->win_slot) {
+    ix->kstatus = static_cast<uint32_t*>(dev_alloc(ix, 256, st));
+    if (!ix->cent || !ix->assign || !ix->mcnt || !ix->msize || !ix->win_u0 || !ix->win_slot ||
+        !ix->kstatus) {
       dev_free(ix, ix->cent);
       dev_free(ix, ix->assign);
       dev_free(ix, ix->mcnt);
       dev_free(ix, ix->msize);
       dev_free(ix, ix->win_u0);
       dev_free(ix, ix->win_slot);
+      dev_free(ix, ix->kstatus);
       ix->cent = nullptr;
       ix->assign = nullptr;
       ix->mcnt = ix->msize = ix->win_u0 = ix->win_slot = nullptr;
+      ix->kstatus = nullptr;
       return fail(SS_ERR_ALLOC, "device allocation of the cluster arrays failed");
     }
     SS_CUDA(cudaMemsetAsync(ix->win_slot, 0xff, (size_t)n_slots * 4, st));
+    SS_CUDA(cudaMemsetAsync(ix->kstatus, 0, 4, st));
     ix->wcap = (int32_t)wcap;
     ix->win_frames = q.window_frames;
     ix->n_centroids = q.n_centroids;
@@ -564,7 +572,7 @@ SS_EXPORT ss_status ss_index_compress(ss_index* ix, const ss_compress_params* cp
   SS_CUDA(launch_kmeans(ix->keys, ix->ncap, n_slabs, ix->cent, ix->assign, ix->mcnt, ix->msize,
                         ix->win_u0, ix->win_slot, ix->wcap, ix->n_windows, n_new, q.first_frame,
                         q.window_frames, c.tokens_per_frame, c.frames_per_unit, q.n_centroids,
-                        q.iters, st));
+                        q.iters, ix->kstatus, st));
   for (int j = 0; j < n_new; ++j)
     ix->win_first_frame.push_back(q.first_frame + (int64_t)j * q.window_frames);
   ix->n_windows += n_new;

@@ -115,6 +115,7 @@ struct Prob {
   const int32_t* msize;        // [P*Hkv][wcap][n_c]
   const int32_t* win_slot;     // [ucap / wu] window of each window slot or -1
   const int32_t* win_u0;       // [wcap] first unit of each window
+  const uint32_t* index_status;  // device word of the index's compressions, or NULL
   int32_t* raw_units;          // [ucap] history units not covered by a window, ascending
   int32_t* raw_rank;           // [ucap] position of a unit in raw_units, or -1
   float* cw;                   // [P*Hkv][wcap*n_c] summed weight of each centroid over
@@ -264,7 +265,8 @@ cudaError_t launch_kmeans(const __nv_bfloat16* keys, int64_t ncap, int n_slabs,
                           __nv_bfloat16* cent, uint8_t* assign, int32_t* mcnt, int32_t* msize,
                           int32_t* win_u0, int32_t* win_slot, int wcap, int w_begin, int n_new,
                           int64_t first_frame, int window_frames, int tokens_per_frame,
-                          int frames_per_unit, int n_c, int iters, cudaStream_t s);
+                          int frames_per_unit, int n_c, int iters, uint32_t* status,
+                          cudaStream_t s);
 cudaError_t launch_descriptors(const __nv_bfloat16* keys, int64_t ncap, int P, int Hkv,
                                int Tu, int64_t u_begin, int64_t u_end, float* desc,
                                cudaStream_t s);

@@ -11,8 +11,12 @@
 //     update  c = mean of the keys assigned to c; a centroid with no keys keeps its value
 // and the index stores the last update's centroids (bf16, nearest-even), the last
 // assignment, and per (centroid, unit of the window) member counts for retrieval.
+//
+// Two kernels: k_kmeans_tc (tcgen05 MMAs, TMA-staged keys, one key read per round) for
+// n_c <= 64 and windows of <= 16384 tokens, and k_kmeans (mma.sync) for the rest.
 #include "ss_internal.cuh"
 #include "ss_device.cuh"
+#include "ss_tc.cuh"
 
 namespace ss {
 
@@ -251,6 +255,440 @@ __global__ void __launch_bounds__(kKmThreads) k_kmeans(const KmJob J) {
   for (int c = tid; c < n_c; c += blockDim.x) ms[c] = cnt[c];
 }
 
+// ---------------------------------------------------------------------------
+// Lloyd rounds on the 5th-generation tensor cores (n_c <= 64, windows of <= 16384
+// tokens). One CTA per (window, slab); every round streams the window's keys once, in
+// tiles of 128 tokens, through a ring of shared-memory stages filled by tiled TMA
+// copies (128-byte swizzle; a 4-D tensor map [slab][window][token][dim] whose token
+// extent is the window, so a ragged last tile reads zeros). Per tile:
+//   MMA1  D1[token][c]      = x . c_hi,  D1[token][n16 + c] = x . c_lo
+//         (M = 128 tokens, N = 2 n16, K = 128 dims; c_hi = bf16(c), c_lo = bf16(c - c_hi),
+//         so x . c carries ~16 significant bits of c; fp32 accumulation in TMEM)
+//   assign a(x) = argmin_c ||c||^2 - 2 (x . c_hi + x . c_lo), lowest id on ties; the
+//         epilogue writes the one-hot row of a(x) (bf16 1.0) into shared memory
+//   MMA2  D2[dim][c] += sum_x x[dim] * onehot[x][c]
+//         (M = 128 dims, N = 64, K = 128 tokens: the key tile read MN-major, the same
+//         bytes as MMA1's K-major operand, so each key is loaded once per round)
+// At the end of a round the member sums D2 and the counts give the new centroids
+// (c = sum / count; an empty centroid keeps its value), from which the epilogue builds
+// the next round's split operands. Every sum has a fixed order (the tensor core's
+// accumulation order over the window's tiles), so results repeat bit for bit.
+//
+// Warp roles: warp 0 issues the TMA copies, warp 1 allocates tensor memory and issues
+// the MMAs (one thread), warps 2-5 are the epilogue (thread e owns TMEM lane e: token e
+// of a tile for MMA1, dim e for MMA2). All waits are bounded; a wait that gives up
+// raises a shared abort flag that ends every role's loop, then the copies and MMAs in
+// flight are drained and the tensor memory is freed.
+// ---------------------------------------------------------------------------
+constexpr int kTcStages = 4;
+constexpr int kTcTile = 128;                            // tokens per tile
+constexpr int kTcStageBytes = kTcTile * kHeadDim * 2;   // 32 KB
+constexpr int kTcEpiWarps = 8;                          // two per TMEM lane quarter
+constexpr int kTcEpiThreads = kTcEpiWarps * 32;
+constexpr int kTcThreads = 64 + kTcEpiThreads;          // + TMA warp + MMA warp
+constexpr int kTcMaxCentroids = 64;
+constexpr int kTcMaxWindowTokens = 16384;
+constexpr int kTcD1Bufs = 3;
+// tensor memory: D1 in three buffers of 128 columns, D2 (64 columns), the fp32
+// centroids (lane = dim, column = centroid; 64 columns)
+constexpr uint32_t kTcTmemCols = 512;
+constexpr uint32_t kTcD2Col = 384;
+constexpr uint32_t kTcCfCol = 448;
+
+struct TcJob {
+  __nv_bfloat16* cent;        // [n_slabs][wcap * n_c][d]
+  uint8_t* assign;            // [n_slabs][ncap]
+  int32_t* mcnt;              // [n_slabs][wcap][n_c][wu]
+  int32_t* msize;             // [n_slabs][wcap][n_c]
+  const __nv_bfloat16* keys;  // [n_slabs][ncap][d] (initial centroids)
+  int64_t ncap;
+  int64_t tok_first;
+  int Wt, Tu, wu, w_begin, wcap, n_c, n16, iters;
+  uint32_t* status;           // device word: kStatusTimeout on a wait that gave up
+};
+
+struct TcBars {
+  unsigned long long full[kTcStages], empty[kTcStages];
+  unsigned long long d1_full[kTcD1Bufs], epi_done[kTcD1Bufs], mma2_done[2];
+  unsigned long long d2_full, b1_ready, final_mma;
+  uint32_t taddr;
+  int abort;
+  int cnt[kTcMaxCentroids];
+  float cn2[kTcMaxCentroids];
+  float xbest[2][2][kTcTile];  // [tile parity][centroid half][row]: nearest distance
+  int xbc[2][2][kTcTile];      // and its centroid
+};
+
+// ring, B1 operand (128 rows x 256 B), one-hot rows (2 x 128 x 128 B, which also hold
+// the fp32 centroids [64][128] at the end of a round), assignment bytes
+size_t kmeans_tc_smem_bytes(int Wt) {
+  return 1024 + (size_t)kTcStages * kTcStageBytes + 128 * 256 + 2 * kTcTile * 128 +
+         (size_t)((Wt + 15) & ~15);
+}
+
+bool kmeans_tc_supported(int n_c, int Wt) {
+  return n_c <= kTcMaxCentroids && Wt <= kTcMaxWindowTokens && Wt >= 1;
+}
+
+// Bounded wait that also gives up when another role raised the abort flag; a wait that
+// runs out raises it.
+__device__ __forceinline__ bool tc_wait(uint32_t bar, uint32_t parity, volatile int* abort) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (uint32_t i = 1; i < kDefaultWaitPolls; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 255u) == 0u) {
+      if (*abort) return false;
+      if (global_ns() - t0 > 1000000000ull) break;
+    }
+  }
+  *abort = 1;
+  return false;
+}
+
+// Writes centroid c's split operand rows (c_hi in row c, c_lo in row n16 + c) at dim e of
+// the 128-byte swizzled K-major tile B1 (two halves of 64 dims, each N1 rows x 128 B).
+__device__ __forceinline__ void tc_put_split(unsigned char* B1, int N1, int row, int e, float x) {
+  const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+  const __nv_bfloat16 lo = __float2bfloat16_rn(x - __bfloat162float(hi));
+  const int half = e >> 6, b = (e & 63) * 2;
+  const int r2 = row + (N1 >> 1);
+  unsigned char* h0 = B1 + half * (N1 * 128);
+  *reinterpret_cast<__nv_bfloat16*>(h0 + row * 128 + ((((b >> 4) ^ (row & 7))) << 4) + (b & 15)) = hi;
+  *reinterpret_cast<__nv_bfloat16*>(h0 + r2 * 128 + ((((b >> 4) ^ (r2 & 7))) << 4) + (b & 15)) = lo;
+}
+
+__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+
+// New round operands from the fp32 centroids cf[0..31] = centroids 32 h .. 32 h + 31 at
+// this thread's dim er: the centroids to tensor memory, the split rows of B1 and, through
+// the staging rows Ct (fp32 [64][128]), ||c||^2 of every centroid (thread i < n16 sums
+// centroid i over the dims starting at its own index: a fixed order, no bank conflicts).
+__device__ __forceinline__ void tc_round_operands(const float* cf, int h, int er, int ei, int n_c,
+                                                  int n16, unsigned char* B1, float* Ct,
+                                                  float* cn2, uint32_t cf_taddr, bool build_b1) {
+  float w[32];
+#pragma unroll
+  for (int c = 0; c < 32; ++c) w[c] = cf[c];
+  tmem_st32(cf_taddr + 32 * h, w);
+#pragma unroll
+  for (int c = 0; c < 32; ++c)
+    if (32 * h + c < n16) Ct[(32 * h + c) * kHeadDim + er] = cf[c];
+  if (build_b1)
+#pragma unroll
+    for (int c = 0; c < 32; ++c)
+      if (32 * h + c < n16) tc_put_split(B1, 2 * n16, 32 * h + c, er, cf[c]);
+  epi_bar();
+  if (ei < n16) {
+    float s2 = INFINITY;   // padding centroids are never nearest
+    if (ei < n_c) {
+      s2 = 0.f;
+      const float* row = Ct + ei * kHeadDim;
+      for (int t = 0; t < kHeadDim; ++t) {
+        const float x = row[(ei + t) & (kHeadDim - 1)];
+        s2 = fmaf(x, x, s2);
+      }
+    }
+    cn2[ei] = s2;
+  }
+}
+
+__global__ void __launch_bounds__(kTcThreads, 1)
+    k_kmeans_tc(const __grid_constant__ CUtensorMap kmap, const TcJob J) {
+  extern __shared__ unsigned char sm_raw[];
+  __shared__ TcBars S;
+  unsigned char* sm = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  unsigned char* ring = sm;
+  unsigned char* B1 = ring + kTcStages * kTcStageBytes;
+  unsigned char* onehot = B1 + 128 * 256;
+  float* Ct = reinterpret_cast<float*>(onehot);   // staging rows at the end of a round
+  uint8_t* a_s = onehot + 2 * kTcTile * 128;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int wl = blockIdx.x, slab = blockIdx.y;
+  const int n_c = J.n_c, n16 = J.n16, N1 = 2 * n16, Wt = J.Wt;
+  const int ntile = (Wt + kTcTile - 1) / kTcTile;
+  const int J_tiles = J.iters * ntile;
+  volatile int* abort = &S.abort;
+
+  if (tid == 0) {
+    for (int s = 0; s < kTcStages; ++s) {
+      mbar_init(smem_u32(&S.full[s]), 1);
+      mbar_init(smem_u32(&S.empty[s]), 1);
+    }
+    for (int b = 0; b < kTcD1Bufs; ++b) {
+      mbar_init(smem_u32(&S.d1_full[b]), 1);
+      mbar_init(smem_u32(&S.epi_done[b]), kTcEpiThreads);
+    }
+    for (int b = 0; b < 2; ++b) mbar_init(smem_u32(&S.mma2_done[b]), 1);
+    mbar_init(smem_u32(&S.d2_full), 1);
+    mbar_init(smem_u32(&S.b1_ready), 1);
+    mbar_init(smem_u32(&S.final_mma), 1);
+    S.abort = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (tid < kTcMaxCentroids) S.cnt[tid] = 0;
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&S.taddr), kTcTmemCols);
+    tmem_relinquish();
+  }
+  if (warp == 0 && lane == 0) tma_prefetch_map(&kmap);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tbase = S.taddr;
+
+  if (warp == 0) {
+    // ---- TMA producer ----
+    if (lane == 0) {
+      int issued_last[kTcStages];
+      for (int s = 0; s < kTcStages; ++s) issued_last[s] = -1;
+      for (int j = 0; j < J_tiles && !*abort; ++j) {
+        const int st = j % kTcStages;
+        if (j >= kTcStages && !tc_wait(smem_u32(&S.empty[st]), ((j / kTcStages) - 1) & 1, abort))
+          break;
+        const uint32_t bar = smem_u32(&S.full[st]);
+        const uint32_t dst = smem_u32(ring + st * kTcStageBytes);
+        const int y = (j % ntile) * kTcTile;
+        mbar_expect_tx(bar, kTcStageBytes);
+        tma_load_4d(dst, &kmap, bar, 0, y, wl, slab);
+        tma_load_4d(dst + kTcStageBytes / 2, &kmap, bar, 64, y, wl, slab);
+        issued_last[st] = j;
+      }
+      // let every issued copy land before the CTA can exit
+      for (int s = 0; s < kTcStages; ++s)
+        if (issued_last[s] >= 0)
+          mbar_wait_bounded(smem_u32(&S.full[s]), (issued_last[s] / kTcStages) & 1);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ---- MMA issuer: issues MMA1 of a tile as soon as its keys, a free D1 buffer and
+    // (at a round's first tile) the round's operands are ready, and MMA2 of the oldest
+    // tile whose one-hot rows are written, whichever comes first ----
+    if (lane == 0) {
+      const uint32_t id1 = idesc_bf16_f32(128, N1, false, false);
+      const uint32_t id2 = idesc_bf16_f32(128, 64, true, true);
+      const uint32_t b1s = smem_u32(B1);
+      int n1 = 0, n2 = 0;                       // next tile for MMA1, for MMA2
+      uint64_t t_idle = 0;
+      uint32_t idle = 0;
+      while (n2 < J_tiles) {
+        bool did = false;
+        if (n1 < J_tiles && n1 - n2 < kTcD1Bufs) {
+          const int tile = n1 % ntile, st = n1 % kTcStages, buf = n1 % kTcD1Bufs;
+          bool ready = tile != 0 || (n2 == n1 && mbar_try_wait(smem_u32(&S.b1_ready), (n1 / ntile) & 1));
+          ready = ready && mbar_try_wait(smem_u32(&S.full[st]), (n1 / kTcStages) & 1);
+          if (ready) {
+            tc_fence_after();
+            const uint32_t as = smem_u32(ring + st * kTcStageBytes);
+            const uint32_t d1 = tbase + (uint32_t)buf * 128u;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              const uint32_t ka = (k >> 2) * (kTcStageBytes / 2) + (k & 3) * 32;
+              const uint32_t kb = (k >> 2) * (N1 * 128) + (k & 3) * 32;
+              umma_bf16(d1, sdesc_sw128(as + ka, 16, 1024), sdesc_sw128(b1s + kb, 16, 1024), id1,
+                        k > 0 ? 1u : 0u);
+            }
+            umma_commit(smem_u32(&S.d1_full[buf]));
+            ++n1;
+            did = true;
+          }
+        }
+        if (n2 < n1 && mbar_try_wait(smem_u32(&S.epi_done[n2 % kTcD1Bufs]), (n2 / kTcD1Bufs) & 1)) {
+          tc_fence_after();
+          const uint32_t xs = smem_u32(ring + (n2 % kTcStages) * kTcStageBytes);
+          const uint32_t os = smem_u32(onehot + (n2 & 1) * (kTcTile * 128));
+          const bool first = (n2 % ntile) == 0;
+#pragma unroll
+          for (int k = 0; k < 8; ++k)
+            umma_bf16(tbase + kTcD2Col, sdesc_sw128(xs + k * 2048, kTcStageBytes / 2, 1024),
+                      sdesc_sw128(os + k * 2048, kTcStageBytes / 2, 1024), id2,
+                      (first && k == 0) ? 0u : 1u);
+          umma_commit(smem_u32(&S.mma2_done[n2 & 1]));
+          umma_commit(smem_u32(&S.empty[n2 % kTcStages]));
+          if ((n2 % ntile) == ntile - 1) umma_commit(smem_u32(&S.d2_full));
+          ++n2;
+          did = true;
+        }
+        if (did) {
+          idle = 0;
+        } else if ((++idle & 255u) == 0u) {
+          // bounded: give up after ~1 s without progress, or when another role did
+          const uint64_t now = global_ns();
+          if (idle == 256u) t_idle = now;
+          if (*abort || now - t_idle > 1000000000ull || idle >= kDefaultWaitPolls) {
+            *abort = 1;
+            break;
+          }
+        }
+      }
+      // every MMA issued has completed before the tensor memory is freed
+      umma_commit(smem_u32(&S.final_mma));
+      mbar_wait_bounded(smem_u32(&S.final_mma), 0);
+    }
+    __syncwarp();
+  } else {
+    // ---- epilogue: warps 2-9. Thread (h, er): TMEM lane er (token er of a tile for
+    // MMA1, dim er for MMA2) and centroids 32 h .. 32 h + 31 ----
+    // Every epilogue thread runs the same sequence of named barriers whatever happens
+    // (a wait that gives up clears `ok` and the work is skipped, never the barriers).
+    const int q = warp & 3;                      // the lane quarter this warp may access
+    const int h = (warp - 2) >> 2;               // centroid half
+    const int er = q * 32 + lane;
+    const int ei = h * 128 + er;                 // 0 .. 255
+    const uint32_t lane_addr = tbase + ((uint32_t)(q * 32) << 16);
+    const __nv_bfloat16* X0 =
+        J.keys + ((int64_t)slab * J.ncap + J.tok_first + (int64_t)wl * Wt) * kHeadDim;
+    const int c_lo = 32 * h;                     // this thread's first centroid
+    const int n_mine = max(0, min(32, n16 - c_lo));
+    bool ok = true;
+    {
+      // C0 = the window's first n_c keys; the round-0 operands
+      float cf[32];
+#pragma unroll
+      for (int c = 0; c < 32; ++c)
+        cf[c] = c_lo + c < n_c ? __bfloat162float(X0[(int64_t)(c_lo + c) * kHeadDim + er]) : 0.f;
+      tc_round_operands(cf, h, er, ei, n_c, n16, B1, Ct, S.cn2, lane_addr + kTcCfCol, true);
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    epi_bar();
+    if (ei == 0) mbar_arrive(smem_u32(&S.b1_ready));
+
+    for (int j = 0; j < J_tiles; ++j) {
+      const int tile = j % ntile, round = j / ntile, buf = j % kTcD1Bufs, x = j & 1;
+      ok = ok && tc_wait(smem_u32(&S.d1_full[buf]), (j / kTcD1Bufs) & 1, abort);
+      tc_fence_after();
+      // nearest of this half's centroids to token tile * 128 + er
+      float best = INFINITY;
+      int bc = c_lo;
+      if (ok && n_mine > 0) {
+        const uint32_t d1 = lane_addr + (uint32_t)buf * 128u;
+        if (n_mine == 32) {
+          float hi[32], lo[32];
+          tmem_ld32(d1 + c_lo, hi);
+          tmem_ld32(d1 + n16 + c_lo, lo);
+#pragma unroll
+          for (int c = 0; c < 32; ++c) {
+            const float dist = fmaf(-2.f, hi[c] + lo[c], S.cn2[c_lo + c]);
+            if (dist < best) {
+              best = dist;
+              bc = c_lo + c;
+            }
+          }
+        } else {
+          for (int c0 = 0; c0 < n_mine; c0 += 16) {
+            float hi[16], lo[16];
+            tmem_ld16(d1 + c_lo + c0, hi);
+            tmem_ld16(d1 + n16 + c_lo + c0, lo);
+#pragma unroll
+            for (int t = 0; t < 16; ++t) {
+              const float dist = fmaf(-2.f, hi[t] + lo[t], S.cn2[c_lo + c0 + t]);
+              if (dist < best) {
+                best = dist;
+                bc = c_lo + c0 + t;
+              }
+            }
+          }
+        }
+      }
+      // both halves' candidates (double-buffered by tile parity): the nearest, the lower
+      // half on a tie (lower ids), is the row's centroid in both halves
+      S.xbest[x][h][er] = best;
+      S.xbc[x][h][er] = bc;
+      epi_bar();
+      {
+        const float b0 = S.xbest[x][0][er], b1 = S.xbest[x][1][er];
+        bc = b1 < b0 ? S.xbc[x][1][er] : S.xbc[x][0][er];
+      }
+      const int tok = tile * kTcTile + er;
+      const bool valid = tok < Wt;
+      ok = ok && (j < 2 || tc_wait(smem_u32(&S.mma2_done[x]), ((j >> 1) - 1) & 1, abort));
+      if (ok) {
+        // half h writes chunks 4 h .. 4 h + 3 of the row's one-hot (8 centroids each)
+        unsigned char* row = onehot + x * (kTcTile * 128) + er * 128;
+#pragma unroll
+        for (int qq = 0; qq < 4; ++qq) {
+          const int qc = 4 * h + qq;
+          uint4 v = make_uint4(0u, 0u, 0u, 0u);
+          if (valid && (bc >> 3) == qc) {
+            const uint32_t one = 0x3F80u << (16 * (bc & 1));   // bf16 1.0
+            const int w = (bc & 7) >> 1;
+            if (w == 0) v.x = one;
+            else if (w == 1) v.y = one;
+            else if (w == 2) v.z = one;
+            else v.w = one;
+          }
+          *reinterpret_cast<uint4*>(row + ((qc ^ (er & 7)) << 4)) = v;
+        }
+        if (h == 0 && valid) {
+          a_s[tok] = (uint8_t)bc;
+          atomicAdd(&S.cnt[bc], 1);
+        }
+      }
+      fence_proxy_async_smem();
+      tc_fence_before();
+      mbar_arrive(smem_u32(&S.epi_done[buf]));
+
+      if (tile == ntile - 1) {
+        // ---- end of a round: new centroids from the member sums ----
+        // (every MMA of the round has completed once d2_full does, so the one-hot rows
+        // are free to stage the fp32 centroids)
+        epi_bar();                                            // every count is in
+        ok = ok && tc_wait(smem_u32(&S.d2_full), round & 1, abort);
+        tc_fence_after();
+        float cf[32];
+#pragma unroll
+        for (int c = 0; c < 32; ++c) cf[c] = 0.f;
+        if (ok) {
+          float sum[32];
+          tmem_ld32(lane_addr + kTcD2Col + c_lo, sum);
+          tmem_ld32(lane_addr + kTcCfCol + c_lo, cf);
+#pragma unroll
+          for (int c = 0; c < 32; ++c) {
+            const int n = c_lo + c < n_c ? S.cnt[c_lo + c] : 0;
+            if (n > 0) cf[c] = sum[c] / (float)n;
+          }
+        }
+        const bool more = round + 1 < J.iters;
+        tc_round_operands(cf, h, er, ei, n_c, n16, B1, Ct, S.cn2, lane_addr + kTcCfCol,
+                          ok && more);
+        if (more) {
+          if (ei < kTcMaxCentroids) S.cnt[ei] = 0;
+          fence_proxy_async_smem();
+          tc_fence_before();
+          epi_bar();
+          if (ei == 0 && ok) mbar_arrive(smem_u32(&S.b1_ready));
+        } else if (!*abort) {
+          // ---- outputs: centroids (bf16), assignment, member counts ----
+          __nv_bfloat16* co = J.cent + ((int64_t)slab * J.wcap * n_c +
+                                        (int64_t)(J.w_begin + wl) * n_c) * kHeadDim;
+#pragma unroll
+          for (int c = 0; c < 32; ++c)
+            if (c_lo + c < n_c) co[(int64_t)(c_lo + c) * kHeadDim + er] = __float2bfloat16_rn(cf[c]);
+          const int64_t tok0 = J.tok_first + (int64_t)wl * Wt;
+          uint8_t* ao = J.assign + (int64_t)slab * J.ncap + tok0;
+          int32_t* mc = J.mcnt + ((int64_t)slab * J.wcap + J.w_begin + wl) * n_c * J.wu;
+          for (int p = ei; p < Wt; p += kTcEpiThreads) {
+            const int c = a_s[p];
+            ao[p] = (uint8_t)c;
+            atomicAdd(mc + c * J.wu + p / J.Tu, 1);
+          }
+          int32_t* ms = J.msize + ((int64_t)slab * J.wcap + J.w_begin + wl) * n_c;
+          if (ei < n_c) ms[ei] = S.cnt[ei];
+        }
+      }
+    }
+    epi_bar();
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (tid == 0 && *abort) atomicOr(J.status, kStatusTimeout);
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tbase, kTcTmemCols);
+}
+
 // Window metadata: first unit of each new window and the window of each window slot
 // (slot = first unit / units per window; windows start on window boundaries).
 __global__ void k_window_meta(int32_t* win_u0, int32_t* win_slot, int w_begin, int n_new,
@@ -266,7 +704,8 @@ cudaError_t launch_kmeans(const __nv_bfloat16* keys, int64_t ncap, int n_slabs,
                           __nv_bfloat16* cent, uint8_t* assign, int32_t* mcnt, int32_t* msize,
                           int32_t* win_u0, int32_t* win_slot, int wcap, int w_begin, int n_new,
                           int64_t first_frame, int window_frames, int tokens_per_frame,
-                          int frames_per_unit, int n_c, int iters, cudaStream_t s) {
+                          int frames_per_unit, int n_c, int iters, uint32_t* status,
+                          cudaStream_t s) {
   if (n_new <= 0) return cudaSuccess;
   const int wu = window_frames / frames_per_unit;
   const int Tu = tokens_per_frame * frames_per_unit;
@@ -294,6 +733,39 @@ cudaError_t launch_kmeans(const __nv_bfloat16* keys, int64_t ncap, int n_slabs,
                                                      first_frame / frames_per_unit, wu);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  if (kmeans_tc_supported(n_c, J.Wt)) {
+    // keys of this call's windows as [slab][window][token][dim]: the token extent is the
+    // window, so a tile past the window's end reads zeros
+    const uint64_t dims[4] = {(uint64_t)kHeadDim, (uint64_t)J.Wt, (uint64_t)n_new, (uint64_t)n_slabs};
+    const uint64_t strides[3] = {(uint64_t)kHeadDim * 2, (uint64_t)J.Wt * kHeadDim * 2,
+                                 (uint64_t)ncap * kHeadDim * 2};
+    const uint32_t box[4] = {64, kTcTile, 1, 1};
+    CUtensorMap map;
+    e = encode_bf16_map(&map, keys + J.tok_first * kHeadDim, 4, dims, strides, box);
+    if (e != cudaSuccess) return e;
+    TcJob T;
+    T.cent = cent;
+    T.assign = assign;
+    T.mcnt = mcnt;
+    T.msize = msize;
+    T.keys = keys;
+    T.ncap = ncap;
+    T.tok_first = J.tok_first;
+    T.Wt = J.Wt;
+    T.Tu = Tu;
+    T.wu = wu;
+    T.w_begin = w_begin;
+    T.wcap = wcap;
+    T.n_c = n_c;
+    T.n16 = (n_c + 15) & ~15;
+    T.iters = iters;
+    T.status = status;
+    const size_t smem = kmeans_tc_smem_bytes(J.Wt);
+    e = ensure_smem((const void*)k_kmeans_tc, (int)smem);
+    if (e != cudaSuccess) return e;
+    k_kmeans_tc<<<dim3(n_new, n_slabs), kTcThreads, smem, s>>>(map, T);
+    return cudaGetLastError();
+  }
   const size_t smem = kmeans_smem_bytes(n_c, J.Wt);
   e = ensure_smem((const void*)k_kmeans, (int)smem);
   if (e != cudaSuccess) return e;

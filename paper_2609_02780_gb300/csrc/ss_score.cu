@@ -100,7 +100,8 @@ __global__ void __launch_bounds__(256) k_sample(const __grid_constant__ Batch B)
     if (tid == 0) P.next_unit[slab] = P.chunks * kScoreWarps;  // past the fixed first units
     for (int v = slab * blockDim.x + tid; v < P.ucap; v += n_slabs * blockDim.x) P.votes[v] = 0;
     if (slab == 0 && tid < 4) P.counts[tid] = 0;
-    if (slab == 0 && tid == 0) *P.status = 0u;
+    // a compression whose wait gave up is reported by every later retrieval
+    if (slab == 0 && tid == 0) *P.status = P.index_status ? (*P.index_status & kStatusTimeout) : 0u;
   }
   __syncthreads();
   if (!sampling) return;

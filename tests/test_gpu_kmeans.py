@@ -7,11 +7,14 @@ stored centroids after round t against the fp64 means of its own round-t assignm
 A run with `iters = t` is the first t rounds of a longer run (the kernel is
 deterministic), so one index per t gives every round.
 
-Distance tolerance: the kernel compares ||c||^2 - 2 x . c in fp32, with x . c on the
-tensor cores from c split into two bf16 parts (|c - c_hi - c_lo| <= 2^-18 |c| per
-element) and 256 products accumulated in fp32 (<= 256 * 2^-23 relative), and ||c||^2
-as a 128-term fp32 sum. Each distance is then off by at most about
-3e-5 * (||x||^2 + ||c||^2); a difference of two by twice that. TOL_REL = 1e-4 covers it.
+Distance tolerance: both kernels (tcgen05 for n_c <= 64, mma.sync above) compare
+||c||^2 - 2 x . c in fp32, with x . c on the tensor cores from c split into two bf16
+parts (|c - c_hi - c_lo| <= 2^-18 |c| per element) and 256 products accumulated in fp32
+(<= 256 * 2^-23 relative), and ||c||^2 as a 128-term fp32 sum. Each distance is then
+off by at most about 3e-5 * (||x||^2 + ||c||^2); a difference of two by twice that.
+TOL_REL = 1e-4 covers it. The member sums behind each mean are fp32 sums of exact
+bf16 keys (tensor-core accumulation on the tcgen05 path), far inside the half-ulp bound
+the stored bf16 centroids are checked with.
 """
 import numpy as np
 import pytest
@@ -174,3 +177,24 @@ def test_oracle_compress_agrees_on_a_clear_case():
     cg = _bits(r["centroids"][0, 0, 0]).astype(np.int64)
     cr = ref["centroid_bits"][0, 0, 0].astype(np.int64)
     assert np.abs(cg - cr).max() <= 1          # bf16 of an fp32 vs an fp64 mean
+
+
+def test_more_than_64_centroids_take_the_mma_sync_kernel():
+    # n_c = 96 is past the tcgen05 kernel's limit: the other kernel, same contract
+    g = torch.Generator().manual_seed(26)
+    keys = (torch.randn(1, 2, 12 * 50, 128, generator=g) +
+            0.5 * torch.randn(1, 2, 12, 1, 128, generator=g).repeat_interleave(50, 2)
+            .reshape(1, 2, 600, 128)).to(torch.bfloat16)
+    _, amb = _chained(keys, Tf=50, WF=4, n_c=96, T=3)     # 3 windows of 200 keys
+    assert amb < 0.05
+
+
+def test_window_of_one_partial_tile_and_many_full_tiles():
+    # 100-token windows (one ragged 128-token tile) and 1,300-token windows (10 full
+    # tiles and a ragged one), 40 centroids (padded to 48 operand rows)
+    g = torch.Generator().manual_seed(27)
+    keys = torch.randn(1, 1, 26 * 100, 128, generator=g).to(torch.bfloat16)
+    _, amb = _chained(keys, Tf=100, WF=1, n_c=40, T=3)
+    assert amb < 0.05
+    _, amb = _chained(keys, Tf=100, WF=13, n_c=40, T=3)
+    assert amb < 0.05
