@@ -315,12 +315,12 @@ struct TcBars {
   int abort;
   int cnt[kTcMaxCentroids];
   float cn2[kTcMaxCentroids];
-  float xbest[2][2][kTcTile];  // [tile parity][centroid half][row]: nearest distance
-  int xbc[2][2][kTcTile];      // and its centroid
+  float part[4][kTcMaxCentroids];  // ||c||^2 partial sums of each lane quarter
+  float xbest[2][2][kTcTile];      // [tile parity][centroid half][row]: nearest distance
+  int xbc[2][2][kTcTile];          // and its centroid
 };
 
-// ring, B1 operand (128 rows x 256 B), one-hot rows (2 x 128 x 128 B, which also hold
-// the fp32 centroids [64][128] at the end of a round), assignment bytes
+// ring, B1 operand (128 rows x 256 B), one-hot rows (2 x 128 x 128 B), assignment bytes
 size_t kmeans_tc_smem_bytes(int Wt) {
   return 1024 + (size_t)kTcStages * kTcStageBytes + 128 * 256 + 2 * kTcTile * 128 +
          (size_t)((Wt + 15) & ~15);
@@ -358,39 +358,50 @@ __device__ __forceinline__ void tc_put_split(unsigned char* B1, int N1, int row,
   *reinterpret_cast<__nv_bfloat16*>(h0 + r2 * 128 + ((((b >> 4) ^ (r2 & 7))) << 4) + (b & 15)) = lo;
 }
 
+// Byte offset of centroid c in row r of a one-hot tile (MN-major, 128-byte swizzle).
+__device__ __forceinline__ int onehot_off(int r, int c) {
+  return r * 128 + ((((c >> 3) ^ (r & 7))) << 4) + (c & 7) * 2;
+}
+
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+// The two warps of one TMEM lane quarter (barriers 2-5).
+__device__ __forceinline__ void pair_bar(int q) {
+  asm volatile("bar.sync %0, 64;" ::"r"(2 + q) : "memory");
+}
 
 // New round operands from the fp32 centroids cf[0..31] = centroids 32 h .. 32 h + 31 at
-// this thread's dim er: the centroids to tensor memory, the split rows of B1 and, through
-// the staging rows Ct (fp32 [64][128]), ||c||^2 of every centroid (thread i < n16 sums
-// centroid i over the dims starting at its own index: a fixed order, no bank conflicts).
-__device__ __forceinline__ void tc_round_operands(const float* cf, int h, int er, int ei, int n_c,
-                                                  int n16, unsigned char* B1, float* Ct,
-                                                  float* cn2, uint32_t cf_taddr, bool build_b1) {
+// this thread's dim er: the centroids to tensor memory, the split rows of B1 and
+// ||c||^2 of every centroid (squares summed over each warp's 32 dims by a shuffle tree,
+// then over the four lane quarters in order: a fixed order). On return this thread holds
+// the squared norms of its own 32 centroids in cn2r.
+__device__ __forceinline__ void tc_round_operands(const float* cf, int h, int q, int lane, int er,
+                                                  int ei, int n_c, int n16, unsigned char* B1,
+                                                  TcBars& S, uint32_t cf_taddr, bool build_b1,
+                                                  float (&cn2r)[32]) {
   float w[32];
 #pragma unroll
   for (int c = 0; c < 32; ++c) w[c] = cf[c];
   tmem_st32(cf_taddr + 32 * h, w);
-#pragma unroll
-  for (int c = 0; c < 32; ++c)
-    if (32 * h + c < n16) Ct[(32 * h + c) * kHeadDim + er] = cf[c];
   if (build_b1)
 #pragma unroll
     for (int c = 0; c < 32; ++c)
       if (32 * h + c < n16) tc_put_split(B1, 2 * n16, 32 * h + c, er, cf[c]);
+#pragma unroll
+  for (int c = 0; c < 32; ++c) {
+    float v = cf[c] * cf[c];
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+    if (lane == 0) S.part[q][32 * h + c] = v;
+  }
   epi_bar();
   if (ei < n16) {
     float s2 = INFINITY;   // padding centroids are never nearest
-    if (ei < n_c) {
-      s2 = 0.f;
-      const float* row = Ct + ei * kHeadDim;
-      for (int t = 0; t < kHeadDim; ++t) {
-        const float x = row[(ei + t) & (kHeadDim - 1)];
-        s2 = fmaf(x, x, s2);
-      }
-    }
-    cn2[ei] = s2;
+    if (ei < n_c) s2 = ((S.part[0][ei] + S.part[1][ei]) + S.part[2][ei]) + S.part[3][ei];
+    S.cn2[ei] = s2;
   }
+  epi_bar();
+#pragma unroll
+  for (int c = 0; c < 32; ++c) cn2r[c] = 32 * h + c < n16 ? S.cn2[32 * h + c] : INFINITY;
 }
 
 __global__ void __launch_bounds__(kTcThreads, 1)
@@ -402,7 +413,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   unsigned char* ring = sm;
   unsigned char* B1 = ring + kTcStages * kTcStageBytes;
   unsigned char* onehot = B1 + 128 * 256;
-  float* Ct = reinterpret_cast<float*>(onehot);   // staging rows at the end of a round
   uint8_t* a_s = onehot + 2 * kTcTile * 128;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -429,6 +439,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (tid < kTcMaxCentroids) S.cnt[tid] = 0;
+  // the one-hot tiles start at zero; afterwards only the single 1.0 of a row changes
+  for (int x = tid; x < 2 * kTcTile * 128 / 16; x += kTcThreads)
+    reinterpret_cast<uint4*>(onehot)[x] = make_uint4(0u, 0u, 0u, 0u);
   if (warp == 1) {
     tmem_alloc(smem_u32(&S.taddr), kTcTmemCols);
     tmem_relinquish();
@@ -542,6 +555,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         J.keys + ((int64_t)slab * J.ncap + J.tok_first + (int64_t)wl * Wt) * kHeadDim;
     const int c_lo = 32 * h;                     // this thread's first centroid
     const int n_mine = max(0, min(32, n16 - c_lo));
+    float cn2r[32];                              // ||c||^2 of this thread's centroids
+    int prev[2] = {-1, -1};                      // the 1.0 each one-hot tile holds in row er
     bool ok = true;
     {
       // C0 = the window's first n_c keys; the round-0 operands
@@ -549,7 +564,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 #pragma unroll
       for (int c = 0; c < 32; ++c)
         cf[c] = c_lo + c < n_c ? __bfloat162float(X0[(int64_t)(c_lo + c) * kHeadDim + er]) : 0.f;
-      tc_round_operands(cf, h, er, ei, n_c, n16, B1, Ct, S.cn2, lane_addr + kTcCfCol, true);
+      tc_round_operands(cf, h, q, lane, er, ei, n_c, n16, B1, S, lane_addr + kTcCfCol, true, cn2r);
     }
     fence_proxy_async_smem();
     tc_fence_before();
@@ -571,70 +586,61 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           tmem_ld32(d1 + n16 + c_lo, lo);
 #pragma unroll
           for (int c = 0; c < 32; ++c) {
-            const float dist = fmaf(-2.f, hi[c] + lo[c], S.cn2[c_lo + c]);
+            const float dist = fmaf(-2.f, hi[c] + lo[c], cn2r[c]);
             if (dist < best) {
               best = dist;
               bc = c_lo + c;
             }
           }
         } else {
-          for (int c0 = 0; c0 < n_mine; c0 += 16) {
-            float hi[16], lo[16];
-            tmem_ld16(d1 + c_lo + c0, hi);
-            tmem_ld16(d1 + n16 + c_lo + c0, lo);
 #pragma unroll
-            for (int t = 0; t < 16; ++t) {
-              const float dist = fmaf(-2.f, hi[t] + lo[t], S.cn2[c_lo + c0 + t]);
-              if (dist < best) {
-                best = dist;
-                bc = c_lo + c0 + t;
+          for (int c0 = 0; c0 < 32; c0 += 16) {
+            if (c0 < n_mine) {
+              float hi[16], lo[16];
+              tmem_ld16(d1 + c_lo + c0, hi);
+              tmem_ld16(d1 + n16 + c_lo + c0, lo);
+#pragma unroll
+              for (int t = 0; t < 16; ++t) {
+                const float dist = fmaf(-2.f, hi[t] + lo[t], cn2r[c0 + t]);
+                if (dist < best) {
+                  best = dist;
+                  bc = c_lo + c0 + t;
+                }
               }
             }
           }
         }
       }
-      // both halves' candidates (double-buffered by tile parity): the nearest, the lower
-      // half on a tie (lower ids), is the row's centroid in both halves
-      S.xbest[x][h][er] = best;
-      S.xbc[x][h][er] = bc;
-      epi_bar();
-      {
-        const float b0 = S.xbest[x][0][er], b1 = S.xbest[x][1][er];
-        bc = b1 < b0 ? S.xbc[x][1][er] : S.xbc[x][0][er];
+      // the two halves' candidates (double-buffered by tile parity): the nearest, the
+      // lower half on a tie (lower ids), is the row's centroid
+      if (h == 1) {
+        S.xbest[x][1][er] = best;
+        S.xbc[x][1][er] = bc;
       }
+      pair_bar(q);
       const int tok = tile * kTcTile + er;
       const bool valid = tok < Wt;
-      ok = ok && (j < 2 || tc_wait(smem_u32(&S.mma2_done[x]), ((j >> 1) - 1) & 1, abort));
-      if (ok) {
-        // half h writes chunks 4 h .. 4 h + 3 of the row's one-hot (8 centroids each)
-        unsigned char* row = onehot + x * (kTcTile * 128) + er * 128;
-#pragma unroll
-        for (int qq = 0; qq < 4; ++qq) {
-          const int qc = 4 * h + qq;
-          uint4 v = make_uint4(0u, 0u, 0u, 0u);
-          if (valid && (bc >> 3) == qc) {
-            const uint32_t one = 0x3F80u << (16 * (bc & 1));   // bf16 1.0
-            const int w = (bc & 7) >> 1;
-            if (w == 0) v.x = one;
-            else if (w == 1) v.y = one;
-            else if (w == 2) v.z = one;
-            else v.w = one;
+      if (h == 0) {
+        if (S.xbest[x][1][er] < best) bc = S.xbc[x][1][er];
+        ok = ok && (j < 2 || tc_wait(smem_u32(&S.mma2_done[x]), ((j >> 1) - 1) & 1, abort));
+        if (ok) {
+          // one 2-byte store clears the row's previous 1.0 in this tile, one sets the new
+          unsigned char* t1 = onehot + x * (kTcTile * 128);
+          if (prev[x] >= 0) *reinterpret_cast<uint16_t*>(t1 + onehot_off(er, prev[x])) = 0;
+          prev[x] = valid ? bc : -1;
+          if (valid) {
+            *reinterpret_cast<uint16_t*>(t1 + onehot_off(er, bc)) = 0x3F80;   // bf16 1.0
+            a_s[tok] = (uint8_t)bc;
+            atomicAdd(&S.cnt[bc], 1);
           }
-          *reinterpret_cast<uint4*>(row + ((qc ^ (er & 7)) << 4)) = v;
         }
-        if (h == 0 && valid) {
-          a_s[tok] = (uint8_t)bc;
-          atomicAdd(&S.cnt[bc], 1);
-        }
+        fence_proxy_async_smem();
       }
-      fence_proxy_async_smem();
       tc_fence_before();
       mbar_arrive(smem_u32(&S.epi_done[buf]));
 
       if (tile == ntile - 1) {
         // ---- end of a round: new centroids from the member sums ----
-        // (every MMA of the round has completed once d2_full does, so the one-hot rows
-        // are free to stage the fp32 centroids)
         epi_bar();                                            // every count is in
         ok = ok && tc_wait(smem_u32(&S.d2_full), round & 1, abort);
         tc_fence_after();
@@ -652,8 +658,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           }
         }
         const bool more = round + 1 < J.iters;
-        tc_round_operands(cf, h, er, ei, n_c, n16, B1, Ct, S.cn2, lane_addr + kTcCfCol,
-                          ok && more);
+        tc_round_operands(cf, h, q, lane, er, ei, n_c, n16, B1, S, lane_addr + kTcCfCol,
+                          ok && more, cn2r);
         if (more) {
           if (ei < kTcMaxCentroids) S.cnt[ei] = 0;
           fence_proxy_async_smem();
