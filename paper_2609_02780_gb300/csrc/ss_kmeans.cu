@@ -490,8 +490,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         bool did = false;
         if (n1 < J_tiles && n1 - n2 < kTcD1Bufs) {
           const int tile = n1 % ntile, st = n1 % kTcStages, buf = n1 % kTcD1Bufs;
-          bool ready = tile != 0 || (n2 == n1 && mbar_try_wait(smem_u32(&S.b1_ready), (n1 / ntile) & 1));
-          ready = ready && mbar_try_wait(smem_u32(&S.full[st]), (n1 / kTcStages) & 1);
+          // (non-blocking tests: a suspended try_wait here would hold back the other queue)
+          bool ready = tile != 0 || (n2 == n1 && mbar_test_wait(smem_u32(&S.b1_ready), (n1 / ntile) & 1));
+          ready = ready && mbar_test_wait(smem_u32(&S.full[st]), (n1 / kTcStages) & 1);
           if (ready) {
             tc_fence_after();
             const uint32_t as = smem_u32(ring + st * kTcStageBytes);
@@ -508,7 +509,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             did = true;
           }
         }
-        if (n2 < n1 && mbar_try_wait(smem_u32(&S.epi_done[n2 % kTcD1Bufs]), (n2 / kTcD1Bufs) & 1)) {
+        if (n2 < n1 && mbar_test_wait(smem_u32(&S.epi_done[n2 % kTcD1Bufs]), (n2 / kTcD1Bufs) & 1)) {
           tc_fence_after();
           const uint32_t xs = smem_u32(ring + (n2 % kTcStages) * kTcStageBytes);
           const uint32_t os = smem_u32(onehot + (n2 & 1) * (kTcTile * 128));
@@ -526,7 +527,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
         if (did) {
           idle = 0;
-        } else if ((++idle & 255u) == 0u) {
+        } else if (__nanosleep(32), (++idle & 255u) == 0u) {
+          // (the short sleep keeps this polling loop from taking the issue slots of the
+          // epilogue warps that share its scheduler)
           // bounded: give up after ~1 s without progress, or when another role did
           const uint64_t now = global_ns();
           if (idle == 256u) t_idle = now;
@@ -582,8 +585,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const uint32_t d1 = lane_addr + (uint32_t)buf * 128u;
         if (n_mine == 32) {
           float hi[32], lo[32];
-          tmem_ld32(d1 + c_lo, hi);
-          tmem_ld32(d1 + n16 + c_lo, lo);
+          tmem_ld32x2(d1 + c_lo, d1 + n16 + c_lo, hi, lo);
 #pragma unroll
           for (int c = 0; c < 32; ++c) {
             const float dist = fmaf(-2.f, hi[c] + lo[c], cn2r[c]);
@@ -649,12 +651,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         for (int c = 0; c < 32; ++c) cf[c] = 0.f;
         if (ok) {
           float sum[32];
-          tmem_ld32(lane_addr + kTcD2Col + c_lo, sum);
-          tmem_ld32(lane_addr + kTcCfCol + c_lo, cf);
+          tmem_ld32x2(lane_addr + kTcD2Col + c_lo, lane_addr + kTcCfCol + c_lo, sum, cf);
+          // mean = sum * (1 / n): the reciprocal rounded once, then one rounded product
 #pragma unroll
           for (int c = 0; c < 32; ++c) {
             const int n = c_lo + c < n_c ? S.cnt[c_lo + c] : 0;
-            if (n > 0) cf[c] = sum[c] / (float)n;
+            if (n > 0) cf[c] = __fmul_rn(sum[c], __frcp_rn((float)n));
           }
         }
         const bool more = round + 1 < J.iters;
@@ -666,23 +668,39 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           tc_fence_before();
           epi_bar();
           if (ei == 0 && ok) mbar_arrive(smem_u32(&S.b1_ready));
-        } else if (!*abort) {
+        } else {
+          // (the barriers below run whatever `write` says: abort may be raised between the
+          // threads' reads of it)
+          const bool write = !*abort;
           // ---- outputs: centroids (bf16), assignment, member counts ----
           __nv_bfloat16* co = J.cent + ((int64_t)slab * J.wcap * n_c +
                                         (int64_t)(J.w_begin + wl) * n_c) * kHeadDim;
 #pragma unroll
           for (int c = 0; c < 32; ++c)
-            if (c_lo + c < n_c) co[(int64_t)(c_lo + c) * kHeadDim + er] = __float2bfloat16_rn(cf[c]);
+            if (write && c_lo + c < n_c)
+              co[(int64_t)(c_lo + c) * kHeadDim + er] = __float2bfloat16_rn(cf[c]);
+          // member counts per (centroid, unit of the window) tallied in shared memory (the
+          // one-hot tiles' space: every MMA has completed), then written out
           const int64_t tok0 = J.tok_first + (int64_t)wl * Wt;
           uint8_t* ao = J.assign + (int64_t)slab * J.ncap + tok0;
           int32_t* mc = J.mcnt + ((int64_t)slab * J.wcap + J.w_begin + wl) * n_c * J.wu;
-          for (int p = ei; p < Wt; p += kTcEpiThreads) {
+          int* tally = reinterpret_cast<int*>(onehot);
+          const int n_tally = n_c * J.wu;
+          const bool in_smem = n_tally <= 2 * kTcTile * 128 / 4;
+          if (write && in_smem)
+            for (int x = ei; x < n_tally; x += kTcEpiThreads) tally[x] = 0;
+          epi_bar();
+          for (int p = ei; write && p < Wt; p += kTcEpiThreads) {
             const int c = a_s[p];
             ao[p] = (uint8_t)c;
-            atomicAdd(mc + c * J.wu + p / J.Tu, 1);
+            if (in_smem) atomicAdd(&tally[c * J.wu + p / J.Tu], 1);
+            else atomicAdd(mc + c * J.wu + p / J.Tu, 1);
           }
+          epi_bar();
+          if (write && in_smem)
+            for (int x = ei; x < n_tally; x += kTcEpiThreads) mc[x] = tally[x];
           int32_t* ms = J.msize + ((int64_t)slab * J.wcap + J.w_begin + wl) * n_c;
-          if (ei < n_c) ms[ei] = S.cnt[ei];
+          if (write && ei < n_c) ms[ei] = S.cnt[ei];
         }
       }
     }

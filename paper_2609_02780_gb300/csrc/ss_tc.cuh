@@ -95,6 +95,29 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
 #pragma unroll
   for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
 }
+// 2 x 32 columns at two column offsets, one wait.
+__device__ __forceinline__ void tmem_ld32x2(uint32_t a0, uint32_t a1, float (&v0)[32],
+                                            float (&v1)[32]) {
+  uint32_t r[64];
+#define SS_R8(b) "=r"(r[b]), "=r"(r[b + 1]), "=r"(r[b + 2]), "=r"(r[b + 3]), "=r"(r[b + 4]), \
+                 "=r"(r[b + 5]), "=r"(r[b + 6]), "=r"(r[b + 7])
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%64];\n"
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,"
+      "%43,%44,%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63},"
+      " [%65];\n"
+      "tcgen05.wait::ld.sync.aligned;\n"
+      : SS_R8(0), SS_R8(8), SS_R8(16), SS_R8(24), SS_R8(32), SS_R8(40), SS_R8(48), SS_R8(56)
+      : "r"(a0), "r"(a1)
+      : "memory");
+#undef SS_R8
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    v0[j] = __uint_as_float(r[j]);
+    v1[j] = __uint_as_float(r[32 + j]);
+  }
+}
 // 16 columns.
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
   uint32_t r[16];
