@@ -154,6 +154,47 @@ typedef struct {
   int32_t* counts;           /* [4] as in ss_result */
 } ss_host_result;
 
+/* Device outputs of one shard of a retrieval over an index split by token range (see
+ * ss_retrieve_shard). n_lists = P * Hq; Uh = the shard's history units. */
+typedef struct {
+  int32_t* topk_tok;         /* [n_lists][k] the shard's top-k tokens per list, stream token
+                                ids (shard unit u is stream unit unit_begin + u), sorted by
+                                (score desc, id asc); -1 past the shard's tokens */
+  float* topk_s;             /* [n_lists][k] their log2-scaled scores s * log2(e);
+                                -infinity past the shard's tokens */
+  float* list_stats;         /* [n_lists][2] (M, L) over the shard's history tokens, as in
+                                ss_result */
+  float* unit_stats;         /* [n_lists][Uh][2] (m, l) over each history unit's tokens:
+                                m = max s * log2(e), l = sum 2^(s * log2(e) - m) */
+  uint32_t* status;          /* [1] device status word (required) */
+} ss_shard_result;
+
+/* One shard's payload as the merge reads it (host arrays). */
+typedef struct {
+  int64_t unit_begin;        /* stream unit of the shard's first history unit */
+  int32_t n_units;           /* the shard's history units */
+  const int32_t* topk_tok;   /* [n_lists][k] as ss_shard_result */
+  const float* topk_s;       /* [n_lists][k] */
+  const float* list_stats;   /* [n_lists][2] */
+  const float* unit_stats;   /* [n_lists][n_units][2] */
+  const float* desc;         /* [n_units][desc_dim] the units' descriptors (Eq. 3) */
+} ss_shard;
+
+/* Host outputs of ss_merge_shards; sizes as ss_result's with U = the stream's history
+ * units (the shards' n_units summed). All required. */
+typedef struct {
+  int32_t* topk_tok;         /* [n_lists][k] */
+  float* topk_w;             /* [n_lists][k] */
+  float* list_stats;         /* [n_lists][2] */
+  int32_t* unit_votes;       /* [U] */
+  float* unit_mass;          /* [U] */
+  int32_t* pool;             /* [min(pool_mult * K, U)] */
+  int32_t* sel_units;        /* [K] */
+  int32_t* exp_units;        /* [K * (1 + n_prev)] */
+  int32_t* frames;           /* [K * (1 + n_prev) * frames_per_unit] */
+  int32_t* counts;           /* [4] n_pool, n_sel, n_exp, n_frames */
+} ss_merge_result;
+
 /* Optional instrumentation: cudaEvent_t handles recorded on the call's stream
  * immediately before and after the key-scoring kernel. NULL members are skipped. */
 typedef struct {
@@ -309,6 +350,38 @@ ss_status ss_retrieve_static(ss_index* index, const void* q, int32_t n_rows,
  * testable without a fault. Process-wide; takes effect for retrievals issued after the
  * call. Errors: INVALID_ARG (polls < -1 or >= 2^32). */
 ss_status ss_set_wait_limit(int64_t polls);
+
+/* One shard of a retrieval over a stream whose history is split by unit range across
+ * GPUs, each GPU holding the keys of its range in its own index (appended in order; its
+ * unit 0 is stream unit unit_begin). The shard scores its own history keys exactly as
+ * ss_retrieve does (Sec. 4.2) and stops after each list's top-k (Eq. 11), writing to
+ * `out` its top-k tokens with their scores, its list statistics and its per-(list, unit)
+ * statistics; with those, ss_merge_shards finishes the retrieval on one host. A token of
+ * a list's global top-k is always in the top-k of its shard, and a list's (M, L) and a
+ * unit's attention mass combine exactly from the shards' statistics, so the merged
+ * result is the unsharded one (up to floating-point rounding). The shard's n_recent_units
+ * counts its own latest units (0 except on the shard that holds the stream's latest
+ * units). Only per-query-head lists over tokens (head_agg SS_H_PER_QHEAD, use_clusters 0)
+ * are supported. `workspace` as ss_retrieve's (same size). Errors as ss_retrieve, plus
+ * UNSUPPORTED for other list kinds. */
+ss_status ss_retrieve_shard(ss_index* index, const void* q, int32_t n_rows,
+                            const ss_retrieve_params* params, int64_t unit_begin,
+                            const ss_shard_result* out, void* workspace,
+                            size_t workspace_bytes, void* stream);
+
+/* Merges the payloads of n_shards shards (host arrays, shards in stream order, their
+ * history unit ranges tiling [0, U)) into the retrieval of the whole stream, on the host:
+ * per list the first k of the shards' candidates by (score desc, id asc) and their
+ * weights under the list's combined softmax statistics (M, L), the unit votes, the units'
+ * attention mass (each unit's per-list statistics under the list's combined (M, L)), the
+ * vote-ranked pool, max-min diversity over the descriptors and the expansion, with the
+ * same rules as ss_retrieve (Sec. 4.2, Eq. 11-12). The merge's arithmetic is fp64.
+ * Errors: INVALID_ARG (NULL, shards not tiling the history in order, a token outside its
+ * shard), UNSUPPORTED (head_agg or use_clusters set). Runs on the calling thread; needs
+ * no GPU. */
+ss_status ss_merge_shards(const ss_shard* shards, int32_t n_shards, int32_t n_lists,
+                          int32_t tokens_per_unit, int32_t frames_per_unit, int32_t desc_dim,
+                          const ss_retrieve_params* params, const ss_merge_result* out);
 
 /* Synchronizes `stream` and returns the status recorded in the device word `status`
  * by earlier retrievals on it (SS_OK, SS_ERR_TIMEOUT or SS_ERR_INTERNAL). */

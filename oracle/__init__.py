@@ -12,5 +12,8 @@ Plain, slow, fp64 numpy written from the paper's definitions:
   kmeans.py     token-level k-means compression of 20-frame windows and retrieval
                 over the centroids with member expansion (the cluster-compressed
                 index variant; closest paper text Sec. 4.1 Eq. 5-7 and Eq. 13)
+  shard.py      one shard's share of a retrieval over an index split by token range
+                (its top-k candidates with scores, softmax statistics per list and
+                per unit, descriptors)
 """
-from . import retrieval, kmeans  # noqa: F401
+from . import retrieval, kmeans, shard  # noqa: F401

@@ -302,6 +302,35 @@ class Index:
         out._keep = (q,)
         return out
 
+    def retrieve_shard(self, q: torch.Tensor, p: RetrieveParams, unit_begin: int,
+                       workspace: torch.Tensor | None = None) -> dict:
+        """This index as one shard (stream units from unit_begin) of a retrieval split by
+        token range: ss_retrieve_shard. Returns device tensors: topk_tok (stream ids),
+        topk_s, list_stats, unit_stats, status; the descriptors are descriptors()."""
+        if q.dtype != torch.bfloat16 or q.dim() != 4 or not q.is_contiguous() or q.device != self.device:
+            raise ValueError("q must be contiguous bf16 [P][R][Hq][128] on the index's device")
+        n_lists = self.n_layers * self.n_q_heads
+        uh = max(0, self.n_units - p.n_recent)
+        dev = self.device
+        out = {"topk_tok": torch.empty(n_lists, p.k, dtype=torch.int32, device=dev),
+               "topk_s": torch.empty(n_lists, p.k, dtype=torch.float32, device=dev),
+               "list_stats": torch.empty(n_lists, 2, dtype=torch.float32, device=dev),
+               "unit_stats": torch.empty(n_lists, max(uh, 1), 2, dtype=torch.float32, device=dev),
+               "status": torch.zeros(1, dtype=torch.int32, device=dev)}
+        nbytes = self.workspace_bytes(q.shape[1], p)
+        ws = workspace if workspace is not None else self._workspace(nbytes)
+        sr = _abi.ShardResult(*[out[k].data_ptr() for k in ("topk_tok", "topk_s", "list_stats",
+                                                             "unit_stats", "status")])
+        with torch.cuda.device(dev):
+            _check(_lib().ss_retrieve_shard(self.handle, C.c_void_p(q.data_ptr()), q.shape[1],
+                                            C.byref(p.to_c()), int(unit_begin), C.byref(sr),
+                                            C.c_void_p(ws.data_ptr()), ws.numel(),
+                                            C.c_void_p(_stream_ptr(dev))))
+        out["unit_stats"] = out["unit_stats"][:, :uh]
+        out["unit_begin"], out["n_units"] = int(unit_begin), uh
+        out["_keep"] = (q, ws)
+        return out
+
     def retrieve_host(self, q_host: torch.Tensor, p: RetrieveParams,
                       workspace: torch.Tensor | None = None) -> dict:
         """ss_retrieve_host: q in (pinned) host memory, selection copied back to host."""
@@ -381,3 +410,45 @@ def retrieve_batched(indexes: list[Index], qs: list[torch.Tensor], p: RetrievePa
     for o in outs:
         o._keep = (workspace, qs)
     return outs
+
+
+def merge_shards(shards: list[dict], n_lists: int, tokens_per_unit: int, p: RetrieveParams,
+                 frames_per_unit: int = 1) -> dict:
+    """ss_merge_shards on the host: the shards' payloads (numpy arrays or CPU tensors with
+    keys unit_begin, n_units, topk_tok int32 [n_lists][k], topk_s fp32 [n_lists][k],
+    list_stats fp32 [n_lists][2], unit_stats fp32 [n_lists][n_units][2], desc fp32
+    [n_units][D]), in stream order. Returns numpy arrays of the merged retrieval."""
+    import numpy as np
+
+    def arr(x, dt):
+        if isinstance(x, torch.Tensor):
+            x = x.detach().cpu().numpy()
+        return np.ascontiguousarray(x, dtype=dt)
+
+    keep = []
+    cs = (_abi.Shard * len(shards))()
+    D = None
+    for j, sh in enumerate(shards):
+        a = [arr(sh["topk_tok"], np.int32), arr(sh["topk_s"], np.float32),
+             arr(sh["list_stats"], np.float32), arr(sh["unit_stats"], np.float32),
+             arr(sh["desc"], np.float32)]
+        keep.append(a)
+        D = a[4].shape[1] if a[4].ndim == 2 and a[4].shape[0] else (D or 1)
+        cs[j] = _abi.Shard(int(sh["unit_begin"]), int(sh["n_units"]),
+                           *[x.ctypes.data for x in a])
+    U = sum(int(sh["n_units"]) for sh in shards)
+    nexp = p.budget * (1 + p.n_prev)
+    out = {"topk_tok": np.empty((n_lists, p.k), np.int32), "topk_w": np.empty((n_lists, p.k), np.float32),
+           "list_stats": np.empty((n_lists, 2), np.float32), "votes": np.empty(U, np.int32),
+           "mass": np.empty(U, np.float32), "pool": np.empty(max(1, min(p.pool_mult * p.budget, U)), np.int32),
+           "sel": np.empty(p.budget, np.int32), "expanded": np.empty(nexp, np.int32),
+           "frames": np.empty(nexp * frames_per_unit, np.int32), "counts": np.zeros(4, np.int32)}
+    mr = _abi.MergeResult(*[out[k].ctypes.data for k in ("topk_tok", "topk_w", "list_stats",
+                                                         "votes", "mass", "pool", "sel",
+                                                         "expanded", "frames", "counts")])
+    _check(_lib().ss_merge_shards(cs, len(shards), n_lists, tokens_per_unit, frames_per_unit,
+                                  int(D or 1), C.byref(p.to_c()), C.byref(mr)))
+    c = out["counts"]
+    out["pool"], out["sel"] = out["pool"][:c[0]], out["sel"][:c[1]]
+    out["expanded"], out["frames"] = out["expanded"][:c[2]], out["frames"][:c[3]]
+    return out

@@ -55,6 +55,24 @@ class HostResult(C.Structure):
                 ("counts", C.c_void_p)]
 
 
+class ShardResult(C.Structure):
+    _fields_ = [("topk_tok", C.c_void_p), ("topk_s", C.c_void_p), ("list_stats", C.c_void_p),
+                ("unit_stats", C.c_void_p), ("status", C.c_void_p)]
+
+
+class Shard(C.Structure):
+    _fields_ = [("unit_begin", C.c_int64), ("n_units", C.c_int32), ("topk_tok", C.c_void_p),
+                ("topk_s", C.c_void_p), ("list_stats", C.c_void_p),
+                ("unit_stats", C.c_void_p), ("desc", C.c_void_p)]
+
+
+class MergeResult(C.Structure):
+    _fields_ = [("topk_tok", C.c_void_p), ("topk_w", C.c_void_p), ("list_stats", C.c_void_p),
+                ("unit_votes", C.c_void_p), ("unit_mass", C.c_void_p), ("pool", C.c_void_p),
+                ("sel_units", C.c_void_p), ("exp_units", C.c_void_p), ("frames", C.c_void_p),
+                ("counts", C.c_void_p)]
+
+
 class Trace(C.Structure):
     _fields_ = [("score_begin", C.c_void_p), ("score_end", C.c_void_p)]
 
@@ -88,6 +106,13 @@ SIGNATURES = {
                                       C.c_void_p]),
     "ss_status_sync": (c_status, [C.c_void_p, C.c_void_p]),
     "ss_set_wait_limit": (c_status, [C.c_int64]),
+    "ss_retrieve_shard": (c_status, [C.c_void_p, C.c_void_p, C.c_int32,
+                                     C.POINTER(RetrieveParams), C.c_int64,
+                                     C.POINTER(ShardResult), C.c_void_p, C.c_size_t,
+                                     C.c_void_p]),
+    "ss_merge_shards": (c_status, [C.POINTER(Shard), C.c_int32, C.c_int32, C.c_int32,
+                                   C.c_int32, C.c_int32, C.POINTER(RetrieveParams),
+                                   C.POINTER(MergeResult)]),
 }
 
 _LIB = None

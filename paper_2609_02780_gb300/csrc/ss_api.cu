@@ -44,8 +44,18 @@ struct ss_index {
 };
 
 namespace {
-
 thread_local char g_err[512] = "";
+}  // namespace
+
+ss_status ss::fail_status(ss_status s, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return s;
+}
+
+namespace {
 
 // Polls after which the score kernel's waits for its key copies give up (process-wide).
 std::atomic<uint32_t> g_wait_polls{kDefaultWaitPolls};
@@ -194,9 +204,18 @@ T* pick(T* user, char* base, size_t off) {
   return user ? user : reinterpret_cast<T*>(base + off);
 }
 
+// A shard of a retrieval split by token range: the select kernel also writes the lists'
+// scores, and the retrieval ends with the export of the shard's payload.
+struct ShardOut {
+  int64_t tok_offset;
+  float* topk_s;
+  float2* unit_stats;
+};
+
 ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t* R, int n,
                         const ss_retrieve_params* p, const ss_result* res, void* ws,
-                        size_t ws_bytes, cudaStream_t st, const ss_trace* tr) {
+                        size_t ws_bytes, cudaStream_t st, const ss_trace* tr,
+                        const ShardOut* shard = nullptr) {
   if (n < 1 || n > kMaxProbs) return fail(SS_ERR_INVALID_ARG, "n must be in [1, %d]", kMaxProbs);
   if (!ix || !q || !R || !res) return fail(SS_ERR_INVALID_ARG, "NULL argument");
   ss_status s = check_params(p);
@@ -270,6 +289,7 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
     const ss_result& r = res[j];
     P.topk_tok = pick(r.topk_tok, base, l.topk_tok);
     P.topk_w = pick(r.topk_w, base, l.topk_w);
+    P.topk_s = shard ? shard->topk_s : nullptr;
     P.list_ml = pick(reinterpret_cast<float2*>(r.list_stats), base, l.list_ml);
     P.votes = pick(r.unit_votes, base, l.votes);
     P.mass = pick(r.unit_mass, base, l.mass);
@@ -355,6 +375,10 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
     SS_CUDA(launch_mass_general(B, max_cent, max_slabs, max_uh, st));
   } else {
     SS_CUDA(launch_select(B, max_lists, ix[0]->sm_count, st));
+    if (shard) {
+      SS_CUDA(launch_shard_export(B, shard->tok_offset, shard->unit_stats, st));
+      return SS_OK;
+    }
     SS_CUDA(launch_mass(B, max_uh, st));
   }
   SS_CUDA(launch_pool(B, max_uh, st));
@@ -610,6 +634,41 @@ SS_EXPORT ss_status ss_retrieve_batched(ss_index* const* ix, const void* const* 
                                         void* ws, size_t ws_bytes, void* stream,
                                         const ss_trace* tr) {
   return retrieve_impl(ix, q, R, n, p, res, ws, ws_bytes, static_cast<cudaStream_t>(stream), tr);
+}
+
+SS_EXPORT ss_status ss_retrieve_shard(ss_index* ix, const void* q, int32_t R,
+                                      const ss_retrieve_params* p, int64_t unit_begin,
+                                      const ss_shard_result* out, void* ws, size_t ws_bytes,
+                                      void* stream) {
+  if (!ix || !out) return fail(SS_ERR_INVALID_ARG, "NULL argument");
+  ss_status s = check_params(p);
+  if (s != SS_OK) return s;
+  if (p->head_agg != SS_H_PER_QHEAD || p->use_clusters)
+    return fail(SS_ERR_UNSUPPORTED, "sharded retrieval needs per-query-head lists over tokens");
+  if (unit_begin < 0) return fail(SS_ERR_INVALID_ARG, "unit_begin must be >= 0");
+  if (!out->topk_tok || !out->topk_s || !out->list_stats || !out->unit_stats || !out->status)
+    return fail(SS_ERR_INVALID_ARG, "every shard output array is required");
+  const int64_t Tu = (int64_t)ix->cfg.tokens_per_frame * ix->cfg.frames_per_unit;
+  if ((unit_begin + ix->ucap) * Tu > (int64_t)0x3fffffff)
+    return fail(SS_ERR_UNSUPPORTED, "stream token ids past 2^30");
+  // the per-list outputs go straight to the caller's arrays; the rest of ss_result is
+  // the workspace's
+  ss_result r{};
+  r.topk_tok = out->topk_tok;
+  r.list_stats = out->list_stats;
+  r.status = out->status;
+  const Layout l = layout_of(ix, R < 1 ? 1 : R, p);
+  if (!ws || ws_bytes < l.total) return fail(SS_ERR_INVALID_ARG, "workspace too small");
+  char* base = static_cast<char*>(ws);
+  r.sel_units = reinterpret_cast<int32_t*>(base + l.sel);
+  r.exp_units = reinterpret_cast<int32_t*>(base + l.exp_units);
+  r.frames = reinterpret_cast<int32_t*>(base + l.frames);
+  r.counts = reinterpret_cast<int32_t*>(base + l.counts);
+  ShardOut so{unit_begin * Tu, out->topk_s, reinterpret_cast<float2*>(out->unit_stats)};
+  ss_index* const arr[1] = {ix};
+  const void* const qa[1] = {q};
+  return retrieve_impl(arr, qa, &R, 1, p, &r, ws, ws_bytes, static_cast<cudaStream_t>(stream),
+                       nullptr, &so);
 }
 
 SS_EXPORT ss_status ss_status_sync(const uint32_t* status, void* stream) {

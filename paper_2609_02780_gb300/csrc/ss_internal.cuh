@@ -14,7 +14,13 @@
 #include <mutex>
 #include <utility>
 
+#include "shallowstream.h"
+
 namespace ss {
+
+// Records a printf-style message as the calling thread's last error (ss_last_error) and
+// returns `s`.
+ss_status fail_status(ss_status s, const char* fmt, ...);
 
 constexpr int kHeadDim = 128;          // d (only 128 is supported)
 constexpr int kMaxProbs = 32;          // problems per batched launch
@@ -96,6 +102,7 @@ struct Prob {
   // outputs
   int32_t* topk_tok;           // [n_lists][k]
   float* topk_w;
+  float* topk_s;               // [n_lists][k] log2-scaled scores of the list, or NULL
   float2* list_ml;             // [n_lists] (M, L)
   int32_t* votes;              // [ucap]
   float* mass;                 // [ucap]
@@ -256,6 +263,8 @@ cudaError_t launch_mass_general(const Batch& B, int max_cent, int max_slabs,
 cudaError_t launch_mass(const Batch& B, int max_hist_units, cudaStream_t s);
 
 cudaError_t launch_pool(const Batch& B, int max_hist_units, cudaStream_t s);
+cudaError_t launch_shard_export(const Batch& B, int64_t tok_offset, float2* unit_stats,
+                                cudaStream_t s);
 cudaError_t launch_maxmin(const Batch& B, int max_pool, cudaStream_t s);
 cudaError_t launch_append(__nv_bfloat16* keys, int64_t ncap, int64_t tok0,
                           const __nv_bfloat16* src, int64_t src_stride_tokens,

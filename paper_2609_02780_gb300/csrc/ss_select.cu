@@ -290,11 +290,13 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
 
   int32_t* tok_out = P.topk_tok + (int64_t)L * k;
   float* w_out = P.topk_w + (int64_t)L * k;
+  float* s_out = P.topk_s ? P.topk_s + (int64_t)L * k : nullptr;
   if (n == 0) {
     if (kGeneral && tid == 0) P.list_ml[L] = make_float2(-INFINITY, 0.f);
     for (int r = tid; r < k; r += blockDim.x) {
       tok_out[r] = -1;
       w_out[r] = 0.f;
+      if (s_out) s_out[r] = -INFINITY;
     }
     return;
   }
@@ -584,6 +586,7 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
       const int32_t id = (int32_t)(~(uint32_t)key);
       tok_out[r] = id;
       w_out[r] = mean ? s : fast_exp2(s - M) * inv_l;
+      if (s_out) s_out[r] = s;
       // one vote for the token's unit (integer atomics: exact)
       if (id >= 0 && (uint32_t)id < kCentroidIdBase) {
         if (id / P.Tu < P.Uh) atomicAdd(&P.votes[id / P.Tu], 1);
@@ -597,6 +600,7 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
     } else {
       tok_out[r] = -1;
       w_out[r] = 0.f;
+      if (s_out) s_out[r] = -INFINITY;
     }
   }
   (void)lane;
