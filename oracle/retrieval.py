@@ -12,7 +12,9 @@ design notes):
   * query representation: the last question row ("final prompt token", Sec. 4.2 and
     Table 4) by default; optionally the row mean, whose logit is the mean logit.
     The row mean is formed in fp32 in row order and rounded to bf16 (nearest-even),
-    a defined step that both sides take.
+    a defined step that both sides take. Third option: every question row attends on
+    its own and a list's weight of a token is the mean over the rows of the rows'
+    softmax weights (row_softmax_mean); the list ranks tokens by that mean weight.
   * scale 1/sqrt(d) on post-RoPE q and k; softmax over the candidate history tokens.
   * per-query-head lists (P * Hq lists of k tokens) by default; "average over heads"
     (Eq. 11 as printed) as the mean of the per-head softmax weights, P lists.
@@ -29,7 +31,7 @@ from __future__ import annotations
 
 import numpy as np
 
-Q_LAST, Q_MEAN_LOGIT = 0, 1
+Q_LAST, Q_MEAN_LOGIT, Q_MEAN_SOFTMAX = 0, 1, 2
 H_PER_QHEAD, H_MEAN = 0, 1
 
 
@@ -113,6 +115,20 @@ def scores(q_eff: np.ndarray, key_bits: np.ndarray, n_hist_tokens: int,
             cache[(i, g)] = bf16_to_f64(key_bits[i, g, :n_hist_tokens])
         out[li] = cache[(i, g)] @ q_eff[i, h] / np.sqrt(d)
     return out
+
+
+def row_softmax_mean(q_bits: np.ndarray, key_bits: np.ndarray, n_hist_tokens: int) -> np.ndarray:
+    """alpha[list][p] = (1/R) sum_r softmax_p(q_r . k_p / sqrt(d)) per (layer, query head)
+    list: the mean over the question rows of each row's attention weights (Sec. 4.2's
+    scored Q-K attention, taken for every question row instead of the last one).
+    q_bits: bf16 bits [P][R][Hq][d]."""
+    q_bits = np.asarray(q_bits, dtype=np.uint16)
+    R = q_bits.shape[1]
+    acc = None
+    for r in range(R):
+        w = softmax(scores(bf16_to_f64(q_bits[:, r]), key_bits, n_hist_tokens))
+        acc = w if acc is None else acc + w
+    return acc / R
 
 
 def softmax(s: np.ndarray) -> np.ndarray:
@@ -281,6 +297,23 @@ def retrieve(key_bits: np.ndarray, q_bits: np.ndarray, *, n_units: int,
     n_tok = U_h * tokens_per_unit
     if desc is None:
         desc = descriptors(key_bits, n_units, tokens_per_unit)
+    if q_agg == Q_MEAN_SOFTMAX:
+        if head_agg != H_PER_QHEAD:
+            raise ValueError("the mean of the rows' softmaxes is defined for per-query-head lists")
+        out = {"n_hist_units": U_h}
+        if U_h == 0:
+            empty = np.zeros(0, dtype=np.int64)
+            out.update(topk_tok=np.zeros((P * Hq, 0), np.int64), topk_w=np.zeros((0, 0)),
+                       votes=empty, mass=np.zeros(0), pool=empty, sel=empty, expanded=empty,
+                       frames=empty)
+            return out
+        alpha = row_softmax_mean(q_bits, key_bits, n_tok)          # [P*Hq][n_tok]
+        tok = topk_rows(alpha, k)
+        out.update(alpha=alpha, topk_tok=tok, topk_w=np.take_along_axis(alpha, tok, axis=1))
+        out.update(select_from_lists(tok, unit_mass(alpha, U_h, tokens_per_unit), desc, U_h,
+                                     tokens_per_unit, budget, pool_mult, n_prev,
+                                     frames_per_unit))
+        return out
     qe = query_effective(q_bits, q_agg)
     out = {"q_eff": qe, "n_hist_units": U_h}
     if U_h == 0:

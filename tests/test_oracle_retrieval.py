@@ -324,3 +324,45 @@ def test_planted_units_are_found():
     # one (the planted units share a descriptor direction, so max-min spreads out)
     assert set(out["pool"][:3].tolist()) == set(planted)
     assert out["sel"][0] == out["pool"][0]
+
+
+# ---------------------------------------------------------------- mean of the rows' softmaxes
+def test_hand_example_mean_of_row_softmaxes(hand):
+    g, keys, q_bits = hand
+    tol = g["tolerance"]
+    ex = g["mean_softmax"]
+    out = R.retrieve(keys, q_bits, n_units=4, tokens_per_unit=2, k=g["k"], budget=2,
+                     pool_mult=2, n_prev=1, q_agg=R.Q_MEAN_SOFTMAX)
+    assert np.allclose(out["alpha"], ex["alpha"], atol=tol)
+    assert out["topk_tok"].tolist() == ex["topk_tok"]
+    assert out["votes"].tolist() == ex["votes"]
+    assert np.allclose(out["mass"], ex["mass"], atol=tol)
+    assert out["pool"].tolist() == ex["pool_mult2_budget2"]
+
+
+def test_mean_of_row_softmaxes_against_library_softmax():
+    sp = pytest.importorskip("scipy.special")
+    rng = np.random.default_rng(11)
+    P, R_, Hq, Hkv, N = 2, 3, 4, 2, 40
+    keys = to_bf16_bits(rng.standard_normal((P, Hkv, N, 128)).astype(np.float32))
+    q = to_bf16_bits(rng.standard_normal((P, R_, Hq, 128)).astype(np.float32))
+    alpha = R.row_softmax_mean(q, keys, N)
+    K = torch.tensor(R.bf16_to_f64(keys))
+    Q = torch.tensor(R.bf16_to_f64(q))
+    for i in range(P):
+        for h in range(Hq):
+            s = (Q[i, :, h] @ K[i, h // 2].T / math.sqrt(128)).numpy()   # [R][N]
+            ref = sp.softmax(s, axis=1).mean(axis=0)
+            assert np.allclose(alpha[i * Hq + h], ref, rtol=1e-12, atol=0)
+    assert np.allclose(alpha.sum(1), 1.0, atol=1e-12)
+
+
+def test_mean_of_row_softmaxes_with_one_row_is_the_last_row_softmax():
+    rng = np.random.default_rng(12)
+    keys = to_bf16_bits(rng.standard_normal((1, 1, 30, 128)).astype(np.float32))
+    q = to_bf16_bits(rng.standard_normal((1, 1, 2, 128)).astype(np.float32))
+    a = R.retrieve(keys, q, n_units=5, tokens_per_unit=6, k=7, budget=2, q_agg=R.Q_MEAN_SOFTMAX)
+    b = R.retrieve(keys, q, n_units=5, tokens_per_unit=6, k=7, budget=2, q_agg=R.Q_LAST)
+    assert np.allclose(a["alpha"], b["w"], rtol=1e-14)
+    for key in ("topk_tok", "votes", "pool", "sel", "frames"):
+        assert np.array_equal(a[key], b[key]), key
