@@ -106,7 +106,16 @@ typedef struct {
   int64_t n_frames;          /* multiple of window_frames */
 } ss_compress_params;
 
-typedef enum { SS_Q_LAST = 0, SS_Q_MEAN_LOGIT = 1 } ss_q_agg;
+/* Which question rows attend (Sec. 4.2 uses the final prompt token):
+ *   SS_Q_LAST         the last row;
+ *   SS_Q_MEAN_LOGIT   the rows' mean (fp32 sum in row order / R, rounded to bf16): its
+ *                     logit is the rows' mean logit;
+ *   SS_Q_MEAN_SOFTMAX every row attends on its own; a list's weight of a token is the
+ *                     mean over the rows of the rows' softmax weights, and the list ranks
+ *                     tokens by it (two passes over the keys: each row's softmax
+ *                     statistics, then the weights; per-query-head lists over tokens only,
+ *                     R <= 64 and (Hq / Hkv) * (R rounded up to 16) <= 512). */
+typedef enum { SS_Q_LAST = 0, SS_Q_MEAN_LOGIT = 1, SS_Q_MEAN_SOFTMAX = 2 } ss_q_agg;
 typedef enum { SS_H_PER_QHEAD = 0, SS_H_MEAN = 1 } ss_head_agg;
 
 /* Evidence-selection parameters (Sec. 4.2; Table 4 gives k = 64, pool 32 = 4 x 8,
@@ -130,10 +139,12 @@ typedef struct {
                                 token id p, or 0x40000000 + window * n_c + centroid for a
                                 centroid; -1 past the number of candidates */
   float* topk_w;             /* [n_lists][k] normalised attention weight of each entry
-                                (SS_H_MEAN: the head-averaged weight alpha) */
+                                (SS_H_MEAN: the head-averaged weight alpha;
+                                SS_Q_MEAN_SOFTMAX: the row-averaged weight) */
   float* list_stats;         /* [n_lists][2] softmax stats (M, L): M = max over candidates
                                 of the log2-scaled score s * log2(e), L = sum 2^(s' - M)
-                                (SS_H_MEAN: M = max alpha, L = sum alpha = 1) */
+                                (SS_H_MEAN, SS_Q_MEAN_SOFTMAX: M = max weight,
+                                L = sum of the weights = 1) */
   int32_t* unit_votes;       /* [U_cap] votes of each history unit */
   float* unit_mass;          /* [U_cap] attention mass of each history unit */
   int32_t* pool;             /* [pool_mult * K] vote-ranked pool, best first */
@@ -283,7 +294,9 @@ ss_status ss_retrieve_workspace_size(const ss_index* const* indexes, int32_t n,
  * 1 - cosine, from its nearest pick; ties to the better pool rank) picks min(K, pool)
  * units; each pick and its n_prev predecessors, deduplicated and ascending, form
  * exp_units and frames (Eq. 12). With SS_H_MEAN the lists are per layer, ranked by the
- * mean over query heads of the per-head weights. With use_clusters, compressed
+ * mean over query heads of the per-head weights. With SS_Q_MEAN_SOFTMAX every question
+ * row attends on its own and a list ranks tokens by the mean of the rows' weights. With
+ * use_clusters, compressed
  * windows contribute their centroids as candidates instead of their tokens (only with
  * SS_H_PER_QHEAD); a selected centroid votes once per member token and its weight is
  * shared among member units by member count. These two modes keep every candidate's

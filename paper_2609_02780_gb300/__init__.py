@@ -21,7 +21,7 @@ import torch
 
 from . import _abi
 
-Q_LAST, Q_MEAN_LOGIT = 0, 1
+Q_LAST, Q_MEAN_LOGIT, Q_MEAN_SOFTMAX = 0, 1, 2
 H_PER_QHEAD, H_MEAN = 0, 1
 CENTROID_ID_BASE = 0x40000000
 STATUS_NAMES = ("OK", "INVALID_ARG", "UNSUPPORTED", "CAPACITY", "STATE", "ALLOC", "CUDA",

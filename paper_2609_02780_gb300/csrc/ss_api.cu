@@ -112,10 +112,18 @@ int64_t cand_cap_of(const ss_index* ix) {
   return (c + 63) & ~(int64_t)63;  // keeps every list's slots 256-byte aligned
 }
 
+// CTAs per slab of the row-averaged passes, at most (the workspace is sized for it).
+int rm_max_chunks(const ss_index* ix) {
+  const int n_slabs = ix->cfg.n_layers * ix->cfg.n_kv_heads;
+  const int64_t hist_tok = ix->ucap * ix->cfg.tokens_per_frame * ix->cfg.frames_per_unit;
+  return rowmean_chunks(n_slabs, (int)(hist_tok > 0x3fffffff ? 0x3fffffff : hist_tok),
+                        ix->sm_count);
+}
+
 // Workspace regions of one problem (offsets from the problem's base).
 struct Layout {
   size_t qeff, cand_s, cand_id, cand_cnt, gthr, ladder, samp_max, ustats, next_unit, gram;
-  size_t raw_units, raw_rank, cw, csel, head_ml, aval, aid;  // general path only
+  size_t raw_units, raw_rank, cw, csel, head_ml, aval, rm;  // general path only
   size_t topk_tok, topk_w, list_ml, votes, mass, pool, sel, exp_units, frames, counts,
       status, qstage;
   size_t total;
@@ -167,8 +175,10 @@ Layout layout_of(const ss_index* ix, int R, const ss_retrieve_params* p) {
   if (p->head_agg == SS_H_MEAN) {
     l.head_ml = take(score_lists * 8);
     l.aval = take((size_t)c.n_layers * cand_cap_of(ix) * 4);
-    l.aid = take((size_t)c.n_layers * cand_cap_of(ix) * 4);
   }
+  if (p->q_agg == SS_Q_MEAN_SOFTMAX)
+    l.rm = take(rowmean_workspace_bytes(c.n_layers * c.n_kv_heads, R,
+                                        c.n_q_heads / c.n_kv_heads, rm_max_chunks(ix)));
   l.total = align256(cur);
   return l;
 }
@@ -183,8 +193,10 @@ ss_status check_params(const ss_retrieve_params* p) {
     return fail(SS_ERR_UNSUPPORTED, "pool_mult * budget_units > %d is not supported", kMaxPool);
   if (p->n_prev < 0) return fail(SS_ERR_INVALID_ARG, "n_prev must be >= 0");
   if (p->n_recent_units < 0) return fail(SS_ERR_INVALID_ARG, "n_recent_units must be >= 0");
-  if (p->q_agg != SS_Q_LAST && p->q_agg != SS_Q_MEAN_LOGIT)
+  if (p->q_agg != SS_Q_LAST && p->q_agg != SS_Q_MEAN_LOGIT && p->q_agg != SS_Q_MEAN_SOFTMAX)
     return fail(SS_ERR_INVALID_ARG, "unknown q_agg %d", p->q_agg);
+  if (p->q_agg == SS_Q_MEAN_SOFTMAX && (p->head_agg != SS_H_PER_QHEAD || p->use_clusters))
+    return fail(SS_ERR_UNSUPPORTED, "q_agg SS_Q_MEAN_SOFTMAX needs per-query-head lists over tokens");
   if (p->head_agg != SS_H_PER_QHEAD && p->head_agg != SS_H_MEAN)
     return fail(SS_ERR_INVALID_ARG, "unknown head_agg %d", p->head_agg);
   if (p->use_clusters != 0 && p->use_clusters != 1)
@@ -233,6 +245,11 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
       return fail(SS_ERR_UNSUPPORTED, "more than %d history units", kMaxHistUnits);
     if (p->use_clusters && ix[j]->n_windows == 0)
       return fail(SS_ERR_STATE, "index %d has no compressed windows", j);
+    if (p->q_agg == SS_Q_MEAN_SOFTMAX &&
+        !rowmean_supported(R[j], ix[j]->cfg.n_q_heads / ix[j]->cfg.n_kv_heads))
+      return fail(SS_ERR_UNSUPPORTED,
+                  "q_agg SS_Q_MEAN_SOFTMAX supports up to 64 rows and (heads per key head) x "
+                  "(rows rounded up to 16) <= 512");
     const ss_result& r = res[j];
     if (!r.sel_units || !r.exp_units || !r.frames || !r.counts || !r.status)
       return fail(SS_ERR_INVALID_ARG, "result %d: sel_units, exp_units, frames, counts and status are required", j);
@@ -250,7 +267,8 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
   B.head_agg = p->head_agg;
   B.use_clusters = p->use_clusters;
   B.wait_polls = g_wait_polls.load(std::memory_order_relaxed);
-  const bool general = p->head_agg == SS_H_MEAN || p->use_clusters;
+  const bool general = p->head_agg == SS_H_MEAN || p->use_clusters ||
+                       p->q_agg == SS_Q_MEAN_SOFTMAX;
   int max_lists = 0, max_uh = 0, max_pool = 0, n_slabs_total = 0;
   int max_cand = 0, max_slabs = 0, max_score_lists = 0, max_cent = 0;
   char* base = static_cast<char*>(ws);
@@ -334,7 +352,10 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
       if (p->head_agg == SS_H_MEAN) {
         P.head_ml = reinterpret_cast<float2*>(base + l.head_ml);
         P.aval = reinterpret_cast<float*>(base + l.aval);
-        P.aid = reinterpret_cast<int32_t*>(base + l.aid);
+      }
+      if (p->q_agg == SS_Q_MEAN_SOFTMAX) {
+        P.rm_scratch = reinterpret_cast<float2*>(base + l.rm);
+        P.rm_chunks = rowmean_chunks(P.P * P.Hkv, P.Uh * P.Tu, x->sm_count);
       }
       max_cand = max(max_cand, P.n_cand);
       max_cent = max(max_cent, P.n_cand - P.n_raw_tok);
@@ -364,7 +385,10 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
   SS_CUDA(cudaSetDevice(dev));
   SS_CUDA(launch_prep(B, st));
   if (tr && tr->score_begin) SS_CUDA(cudaEventRecord((cudaEvent_t)tr->score_begin, st));
-  if (general) {
+  if (p->q_agg == SS_Q_MEAN_SOFTMAX) {
+    for (int j = 0; j < n; ++j)
+      SS_CUDA(launch_rowmean(B, j, B.p[j].rm_scratch, B.p[j].rm_chunks, st));
+  } else if (general) {
     SS_CUDA(launch_general_score(B, max_cand, max_slabs, max_score_lists, st));
   } else {
     SS_CUDA(launch_score(B, st));

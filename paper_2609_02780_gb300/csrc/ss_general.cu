@@ -177,8 +177,7 @@ __global__ void __launch_bounds__(256) k_alpha(const __grid_constant__ Batch B) 
     const float2 ml = P.head_ml[L];
     a += fast_exp2(P.cand_s[(int64_t)L * P.cand_cap + j] - ml.x) * (1.0f / ml.y);
   }
-  P.aval[(int64_t)i * P.cand_cap + j] = a / (float)P.Hq;
-  P.aid[(int64_t)i * P.cand_cap + j] = j;
+  P.aval[(int64_t)i * P.cand_cap + j] = a / (float)P.Hq;   // (its id is its position j)
 }
 
 // ---------------------------------------------------------------------------
@@ -228,6 +227,12 @@ __global__ void __launch_bounds__(256) k_mass_general(const __grid_constant__ Ba
     for (int t = tid; t < P.P * Tu; t += blockDim.x) {
       const int i = t / Tu, r = t - i * Tu;
       acc += P.aval[(int64_t)i * P.cand_cap + (int64_t)u * Tu + r];
+    }
+  } else if (B.q_agg == 2) {
+    // per-query-head lists of row-averaged weights: the rows hold the weights
+    for (int t = tid; t < P.P * P.Hq * Tu; t += blockDim.x) {
+      const int L = t / Tu, r = t - L * Tu;
+      acc += P.cand_s[(int64_t)L * P.cand_cap + (int64_t)u * Tu + r];
     }
   } else {
     const int rr = B.use_clusters ? P.raw_rank[u] : u;

@@ -130,8 +130,9 @@ struct Prob {
   int32_t* csel;               // [P*Hkv][wcap*n_c] lists of its slab that selected each
                                // centroid
   float2* head_ml;             // [P*Hq] (M, L) of each head's softmax (one list per layer)
+  float2* rm_scratch;          // row-averaged lists: per-row softmax statistics
+  int rm_chunks;               // CTAs per slab of the row-averaged passes
   float* aval;                 // [P][cand_cap] head-averaged weight of every token
-  int32_t* aid;                // [P][cand_cap]
   // launch mapping of the score kernel
   int cta_begin;               // first score CTA of this problem
   int chunks;                  // score CTAs per slab (they share the slab's units)
@@ -144,7 +145,7 @@ struct Batch {
   int n;
   int k;
   int n_prev;
-  int q_agg;
+  int q_agg;                   // 0 last row, 1 row mean, 2 mean of the rows' softmaxes
   int head_agg;
   int use_clusters;
   int score_ctas;              // total CTAs of the score kernel
@@ -263,6 +264,10 @@ cudaError_t launch_mass_general(const Batch& B, int max_cent, int max_slabs,
 cudaError_t launch_mass(const Batch& B, int max_hist_units, cudaStream_t s);
 
 cudaError_t launch_pool(const Batch& B, int max_hist_units, cudaStream_t s);
+bool rowmean_supported(int R, int G);
+size_t rowmean_workspace_bytes(int n_slabs, int R, int G, int max_chunks);
+int rowmean_chunks(int n_slabs, int hist_tokens, int sm_count);
+cudaError_t launch_rowmean(const Batch& B, int pi, float2* scratch, int chunks, cudaStream_t s);
 cudaError_t launch_shard_export(const Batch& B, int64_t tok_offset, float2* unit_stats,
                                 cudaStream_t s);
 cudaError_t launch_maxmin(const Batch& B, int max_pool, cudaStream_t s);

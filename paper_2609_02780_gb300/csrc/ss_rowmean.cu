@@ -1,0 +1,456 @@
+// Lists ranked by the mean over the question rows of the rows' softmax weights.
+//
+// Sec. 4.2 scores the candidates against the final prompt token. With every question row
+// attending on its own, token p's weight in list (layer i, query head h) is
+//   alpha(p) = (1/R) sum_r 2^(s_r(p) - M_r) / L_r,   s_r(p) = q_r . k_p * log2(e) / sqrt(d),
+// where (M_r, L_r) are row r's softmax statistics over the history tokens. Every row's
+// statistics must be known before any alpha, so the keys are read twice:
+//   pass 1  k_rm_stats: S^T = Q . K^T on the tcgen05 tensor cores, the question rows of a
+//           key head's G query heads on the TMEM lanes (M = 128 rows per MMA, N = 128
+//           tokens, K = 128 dims), each epilogue thread keeping its row's online
+//           (max, sum) over the tokens; partial statistics per CTA, combined in a fixed
+//           order by k_rm_combine;
+//   pass 2  k_rm_alpha: S = K . Q^T, the tokens on the TMEM lanes (M = 128 tokens,
+//           N = the G * R rows), each epilogue thread summing its token's weights over a
+//           head's rows; alpha goes to the list's dense row, ranked by the general top-k
+//           (ids = positions) and summed per unit by the general mass kernel.
+// Keys reach shared memory through tiled TMA copies (128-byte swizzle), the question
+// rows once per CTA. The rows of head h occupy positions h * Rp .. h * Rp + R - 1
+// (Rp = R rounded up to 16; the padding rows are zero and ignored).
+#include "ss_internal.cuh"
+#include "ss_device.cuh"
+#include "ss_tc.cuh"
+
+namespace ss {
+
+constexpr int kRmTile = 128;                           // tokens per tile
+constexpr int kRmStageBytes = kRmTile * kHeadDim * 2;  // 32 KB
+
+struct RmJob {
+  int prob;            // problem index in the batch
+  int Rp;              // rows per head, padded to 16
+  int GRp;             // G * Rp
+  int chunks;          // CTAs per slab
+  int nbuf;            // TMEM accumulator buffers
+  int stages;          // key stages
+  float2* part;        // [slabs][GRp][chunks] partial (m, l) of pass 1
+  float2* stat;        // [slabs][GRp] (M, 1 / L) of every row
+};
+
+__device__ __forceinline__ void rm_bar(int nthreads) {
+  asm volatile("bar.sync 1, %0;" ::"r"(nthreads) : "memory");
+}
+
+// Copies the question rows of slab (i, g) into a 128-byte swizzled K-major operand:
+// row rho = h * Rp + r (h < G, r < R) from q[i][r][g * G + h][:], zero elsewhere, in
+// blocks of `rows_per_block` rows (each block: two halves of rows_per_block x 128 B).
+__device__ void rm_load_q(const Prob& P, int slab, int Rp, int n_rows, int rows_per_block,
+                          unsigned char* dst, int t0, int nt) {
+  const int i = slab / P.Hkv, g = slab - i * P.Hkv;
+  const int64_t row_stride = (int64_t)P.Hq * kHeadDim;
+  for (int e = t0; e < n_rows * 16; e += nt) {
+    const int rho = e >> 4, c = e & 15;
+    const int h = rho / Rp, r = rho - h * Rp;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (h < P.G && r < P.R)
+      v = *reinterpret_cast<const uint4*>(P.q + (int64_t)i * P.R * row_stride +
+                                          (int64_t)r * row_stride +
+                                          (int64_t)(g * P.G + h) * kHeadDim + 8 * c);
+    const int b = rho / rows_per_block, n = rho - b * rows_per_block;
+    unsigned char* blk = dst + (size_t)b * rows_per_block * 256;
+    *reinterpret_cast<uint4*>(blk + (c >> 3) * (rows_per_block * 128) + n * 128 +
+                              ((((c & 7) ^ (n & 7))) << 4)) = v;
+  }
+}
+
+// Bounded wait that gives up when another role raised the abort flag.
+__device__ __forceinline__ bool rm_wait(uint32_t bar, uint32_t parity, volatile int* abort) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (uint32_t i = 1; i < kDefaultWaitPolls; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 255u) == 0u) {
+      if (*abort) return false;
+      if (global_ns() - t0 > 1000000000ull) break;
+    }
+  }
+  *abort = 1;
+  return false;
+}
+
+struct RmBars {
+  unsigned long long full[4], empty[4], d_full[2], epi_done[2], q_ready, final_mma;
+  uint32_t taddr;
+  int abort;
+};
+
+// Producer / MMA / drain shared by both passes. The MMA thread calls `mma(j, stage, buf)`
+// for each tile j once its keys and a free accumulator buffer are there.
+template <typename MmaFn>
+__device__ void rm_pipeline(const CUtensorMap* kmap, RmBars& S, unsigned char* ring, int stages,
+                            int nbuf, int n_epi, int n_tiles, int64_t row0, MmaFn&& mma) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  volatile int* abort = &S.abort;
+  if (warp == 0 && lane == 0) {
+    int issued_last[4] = {-1, -1, -1, -1};
+    for (int j = 0; j < n_tiles && !*abort; ++j) {
+      const int st = j % stages;
+      if (j >= stages && !rm_wait(smem_u32(&S.empty[st]), ((j / stages) - 1) & 1, abort)) break;
+      const uint32_t bar = smem_u32(&S.full[st]);
+      const uint32_t dst = smem_u32(ring + st * kRmStageBytes);
+      const int y = (int)(row0 + (int64_t)j * kRmTile);
+      mbar_expect_tx(bar, kRmStageBytes);
+      tma_load_2d(dst, kmap, bar, 0, y);
+      tma_load_2d(dst + kRmStageBytes / 2, kmap, bar, 64, y);
+      issued_last[st] = j;
+    }
+    for (int s = 0; s < stages; ++s)
+      if (issued_last[s] >= 0) mbar_wait_bounded(smem_u32(&S.full[s]), (issued_last[s] / stages) & 1);
+  } else if (warp == 1 && lane == 0) {
+    if (rm_wait(smem_u32(&S.q_ready), 0, abort)) {
+      for (int j = 0; j < n_tiles; ++j) {
+        const int st = j % stages, buf = j % nbuf;
+        if (j >= nbuf && !rm_wait(smem_u32(&S.epi_done[buf]), ((j / nbuf) - 1) & 1, abort)) break;
+        if (!rm_wait(smem_u32(&S.full[st]), (j / stages) & 1, abort)) break;
+        tc_fence_after();
+        mma(j, smem_u32(ring + st * kRmStageBytes), buf);
+        umma_commit(smem_u32(&S.d_full[buf]));
+        umma_commit(smem_u32(&S.empty[st]));
+      }
+    }
+    umma_commit(smem_u32(&S.final_mma));
+    mbar_wait_bounded(smem_u32(&S.final_mma), 0);
+  }
+  (void)n_epi;
+}
+
+__device__ __forceinline__ void rm_init(RmBars& S, int stages, int nbuf, int n_epi, uint32_t cols) {
+  const int warp = threadIdx.x >> 5;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < stages; ++s) {
+      mbar_init(smem_u32(&S.full[s]), 1);
+      mbar_init(smem_u32(&S.empty[s]), 1);
+    }
+    for (int b = 0; b < nbuf; ++b) {
+      mbar_init(smem_u32(&S.d_full[b]), 1);
+      mbar_init(smem_u32(&S.epi_done[b]), n_epi);
+    }
+    mbar_init(smem_u32(&S.q_ready), 1);
+    mbar_init(smem_u32(&S.final_mma), 1);
+    S.abort = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&S.taddr), cols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+}
+
+// The tiles [t0, t1) of history tokens of chunk `c` of a slab.
+__device__ __forceinline__ void rm_chunk(const Prob& P, int chunks, int c, int& t0, int& t1) {
+  const int n_tok = P.Uh * P.Tu;
+  const int T = (n_tok + kRmTile - 1) / kRmTile;
+  t0 = (int)((int64_t)T * c / chunks);
+  t1 = (int)((int64_t)T * (c + 1) / chunks);
+}
+
+// ---------------------------------------------------------------------------
+// Pass 1: per-row (max, sum) of the log2-scaled scores over the chunk's tokens.
+// Warps: 0 TMA, 1 MMA (+ TMEM), then 4 per 128-row block (NMB blocks).
+// ---------------------------------------------------------------------------
+template <int NMB>
+__global__ void __launch_bounds__(64 + 128 * NMB, 1)
+    k_rm_stats(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ Batch B,
+               const RmJob J) {
+  extern __shared__ unsigned char sm_raw[];
+  __shared__ RmBars S;
+  unsigned char* sm = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  unsigned char* qs = sm;                                // NMB x 32 KB
+  unsigned char* ring = qs + NMB * 32768;
+  constexpr int n_epi = 128 * NMB;
+  const int nbuf = J.nbuf, stages = J.stages;
+  const uint32_t cols = nbuf * NMB * 128 <= 256 ? 256u : 512u;
+  rm_init(S, stages, nbuf, n_epi, cols);
+  const uint32_t tbase = S.taddr;
+  const Prob& P = B.p[J.prob];
+  const int slab = blockIdx.y, chunk = blockIdx.x;
+  int t0, t1;
+  rm_chunk(P, J.chunks, chunk, t0, t1);
+  const int n_tiles = t1 - t0;
+  const int n_tok = P.Uh * P.Tu;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  volatile int* abort = &S.abort;
+  if (warp < 2) {
+    rm_pipeline(&kmap, S, ring, stages, nbuf, n_epi, n_tiles,
+                (int64_t)slab * P.ncap + (int64_t)t0 * kRmTile,
+                [&](int j, uint32_t ks, int buf) {
+                  const uint32_t id = idesc_bf16_f32(128, 128, false, false);
+#pragma unroll
+                  for (int b = 0; b < NMB; ++b) {
+                    const uint32_t d = tbase + (uint32_t)(buf * NMB + b) * 128u;
+                    const uint32_t as = smem_u32(qs + b * 32768);
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) {
+                      const uint32_t ko = (k >> 2) * 16384 + (k & 3) * 32;
+                      umma_bf16(d, sdesc_sw128(as + ko, 16, 1024), sdesc_sw128(ks + ko, 16, 1024),
+                                id, k > 0 ? 1u : 0u);
+                    }
+                  }
+                  (void)j;
+                });
+  } else {
+    pdl_release();
+    const int e = threadIdx.x - 64;
+    const int b = e >> 7, q = warp & 3;
+    const int rho = b * 128 + q * 32 + lane;            // this thread's row
+    // the slab's question rows (written before the wait: inputs only)
+    rm_load_q(P, slab, J.Rp, NMB * 128, 128, qs, e, n_epi);
+    fence_proxy_async_smem();
+    rm_bar(n_epi);
+    if (e == 0) mbar_arrive(smem_u32(&S.q_ready));
+    const uint32_t lane_addr = tbase + ((uint32_t)(q * 32) << 16);
+    float m = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int j = 0; j < n_tiles; ++j) {
+      const int buf = j % nbuf;
+      ok = ok && rm_wait(smem_u32(&S.d_full[buf]), (j / nbuf) & 1, abort);
+      tc_fence_after();
+      if (ok) {
+        const uint32_t d = lane_addr + (uint32_t)(buf * NMB + b) * 128u;
+        const int nv = min(kRmTile, n_tok - (t0 + j) * kRmTile);   // valid tokens
+        // the tile's 128 token columns in two halves of 64 (online update per half)
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+          float v0[32], v1[32];
+          tmem_ld32x2(d + 64 * hh, d + 64 * hh + 32, v0, v1);
+          float mt = -INFINITY;
+#pragma unroll
+          for (int c = 0; c < 32; ++c) {
+            if (64 * hh + c < nv) mt = fmaxf(mt, v0[c] * kScoreScale);
+            if (64 * hh + 32 + c < nv) mt = fmaxf(mt, v1[c] * kScoreScale);
+          }
+          if (mt > m) {
+            l = (m == -INFINITY) ? 0.f : l * fast_exp2(m - mt);
+            m = mt;
+          }
+          float acc = 0.f;
+#pragma unroll
+          for (int c = 0; c < 32; ++c) {
+            if (64 * hh + c < nv) acc += fast_exp2(fmaf(v0[c], kScoreScale, -m));
+            if (64 * hh + 32 + c < nv) acc += fast_exp2(fmaf(v1[c], kScoreScale, -m));
+          }
+          l += acc;
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(smem_u32(&S.epi_done[buf]));
+    }
+    const int h = rho / J.Rp, r = rho - h * J.Rp;
+    pdl_wait();   // the previous kernel of the call (its resets) has completed
+    if (ok && !*abort && h < P.G && r < P.R)
+      J.part[((int64_t)slab * J.GRp + rho) * J.chunks + chunk] = make_float2(m, l);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (threadIdx.x == 0) pdl_wait();
+  if (threadIdx.x == 0 && S.abort) atomicOr(P.status, kStatusTimeout);
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tbase, cols);
+}
+
+// (M, 1 / L) of every row from the chunks' partials, in chunk order.
+__global__ void __launch_bounds__(256) k_rm_combine(const __grid_constant__ Batch B, const RmJob J) {
+  pdl_wait();
+  pdl_release();
+  const Prob& P = B.p[J.prob];
+  const int x = blockIdx.x * blockDim.x + threadIdx.x;
+  const int n_slabs = P.P * P.Hkv;
+  if (x >= n_slabs * J.GRp) return;
+  const int rho = x % J.GRp;
+  const int h = rho / J.Rp, r = rho - h * J.Rp;
+  if (h >= P.G || r >= P.R) return;
+  float m = -INFINITY, l = 0.f;
+  for (int c = 0; c < J.chunks; ++c) {
+    const float2 v = J.part[(int64_t)x * J.chunks + c];
+    if (v.y > 0.f) ml_combine(m, l, v.x, v.y);
+  }
+  J.stat[x] = make_float2(m, l > 0.f ? 1.0f / l : 0.f);
+}
+
+// ---------------------------------------------------------------------------
+// Pass 2: alpha of every history token of the chunk for the slab's G lists.
+// Warps: 0 TMA, 1 MMA (+ TMEM), 2-9 epilogue (two groups of four, heads split).
+// ---------------------------------------------------------------------------
+constexpr int kRmEpi2 = 256;
+
+__global__ void __launch_bounds__(64 + kRmEpi2, 1)
+    k_rm_alpha(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ Batch B,
+               const RmJob J) {
+  extern __shared__ unsigned char sm_raw[];
+  __shared__ RmBars S;
+  __shared__ float2 st[512];
+  unsigned char* sm = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  const int GRp = J.GRp;
+  // question rows as the B operand: one tile of GRp rows, or two of NE rows each
+  const int two = GRp > 256;
+  const int NE = two ? ((GRp / 2 + 15) & ~15) : GRp;
+  unsigned char* qs = sm;
+  const int q_bytes = (two ? 2 : 1) * NE * 256;
+  unsigned char* ring = qs + ((q_bytes + 1023) & ~1023);
+  const int nbuf = J.nbuf, stages = J.stages;
+  const uint32_t cols = nbuf * (two ? 2 * NE : NE) <= 256 ? 256u : 512u;
+  rm_init(S, stages, nbuf, kRmEpi2, cols);
+  const uint32_t tbase = S.taddr;
+  const Prob& P = B.p[J.prob];
+  const int slab = blockIdx.y, chunk = blockIdx.x;
+  int t0, t1;
+  rm_chunk(P, J.chunks, chunk, t0, t1);
+  const int n_tiles = t1 - t0;
+  const int n_tok = P.Uh * P.Tu;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t buf_cols = two ? 2 * NE : NE;
+  volatile int* abort = &S.abort;
+  if (warp < 2) {
+    rm_pipeline(&kmap, S, ring, stages, nbuf, kRmEpi2, n_tiles,
+                (int64_t)slab * P.ncap + (int64_t)t0 * kRmTile,
+                [&](int j, uint32_t ks, int buf) {
+                  const uint32_t id = idesc_bf16_f32(128, NE, false, false);
+                  for (int t = 0; t < 1 + two; ++t) {
+                    const uint32_t d = tbase + (uint32_t)buf * buf_cols + (uint32_t)(t * NE);
+                    const uint32_t bs = smem_u32(qs + t * NE * 256);
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) {
+                      const uint32_t ka = (k >> 2) * 16384 + (k & 3) * 32;
+                      const uint32_t kb = (k >> 2) * (NE * 128) + (k & 3) * 32;
+                      umma_bf16(d, sdesc_sw128(ks + ka, 16, 1024), sdesc_sw128(bs + kb, 16, 1024),
+                                id, k > 0 ? 1u : 0u);
+                    }
+                  }
+                  (void)j;
+                });
+  } else {
+    const int e = threadIdx.x - 64;
+    const int grp = e >> 7, q = warp & 3;
+    const int tl = q * 32 + lane;                        // token lane
+    rm_load_q(P, slab, J.Rp, (two ? 2 : 1) * NE, NE, qs, e, kRmEpi2);
+    fence_proxy_async_smem();
+    rm_bar(kRmEpi2);
+    if (e == 0) mbar_arrive(smem_u32(&S.q_ready));
+    pdl_wait();                                          // the rows' statistics (pass 1)
+    for (int x = e; x < GRp; x += kRmEpi2)
+      st[x] = J.stat[(int64_t)slab * GRp + x];
+    rm_bar(kRmEpi2);
+    pdl_release();
+    const int G = P.G, Rp = J.Rp;
+    const int hh = (G + 1) / 2;                          // heads of group 0
+    const int h_begin = grp ? hh : 0, h_end = grp ? G : hh;
+    const int i = slab / P.Hkv, g = slab - i * P.Hkv;
+    const float invR = 1.0f / (float)P.R;
+    const uint32_t lane_addr = tbase + ((uint32_t)(q * 32) << 16);
+    bool ok = true;
+    for (int j = 0; j < n_tiles; ++j) {
+      const int buf = j % nbuf;
+      ok = ok && rm_wait(smem_u32(&S.d_full[buf]), (j / nbuf) & 1, abort);
+      tc_fence_after();
+      const int tok = (t0 + j) * kRmTile + tl;
+      if (ok) {
+        for (int h = h_begin; h < h_end; ++h) {
+          float a = 0.f;
+          for (int r0 = 0; r0 < Rp; r0 += 16) {
+            float v[16];
+            tmem_ld16(lane_addr + (uint32_t)buf * buf_cols + (uint32_t)(h * Rp + r0), v);
+#pragma unroll
+            for (int t = 0; t < 16; ++t) {
+              if (r0 + t < P.R) {
+                const float2 s2 = st[h * Rp + r0 + t];
+                a = fmaf(fast_exp2(fmaf(v[t], kScoreScale, -s2.x)), s2.y, a);
+              }
+            }
+          }
+          if (tok < n_tok)
+            P.cand_s[(int64_t)(i * P.Hq + g * G + h) * P.cand_cap + tok] = a * invR;
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(smem_u32(&S.epi_done[buf]));
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (threadIdx.x == 0) pdl_wait();
+  if (threadIdx.x == 0 && S.abort) atomicOr(P.status, kStatusTimeout);
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tbase, cols);
+}
+
+// Host: both passes for problem `pi` of the batch (its own key tensor map).
+bool rowmean_supported(int R, int G) {
+  const int Rp = (R + 15) & ~15;
+  return R >= 1 && Rp <= 64 && G * Rp <= 512;
+}
+
+size_t rowmean_workspace_bytes(int n_slabs, int R, int G, int max_chunks) {
+  const int GRp = G * ((R + 15) & ~15);
+  return (size_t)n_slabs * GRp * (max_chunks + 1) * sizeof(float2);
+}
+
+int rowmean_chunks(int n_slabs, int hist_tokens, int sm_count) {
+  const int T = (hist_tokens + kRmTile - 1) / kRmTile;
+  int c = (sm_count + n_slabs - 1) / n_slabs;
+  c = c < 1 ? 1 : c;
+  return T < c ? (T < 1 ? 1 : T) : c;
+}
+
+cudaError_t launch_rowmean(const Batch& B, int pi, float2* scratch, int chunks, cudaStream_t s) {
+  const Prob& P = B.p[pi];
+  const int n_slabs = P.P * P.Hkv;
+  const int Rp = (P.R + 15) & ~15, GRp = P.G * Rp;
+  if (P.Uh <= 0) return cudaSuccess;
+  RmJob J;
+  J.prob = pi;
+  J.Rp = Rp;
+  J.GRp = GRp;
+  J.chunks = chunks;
+  J.part = scratch;
+  J.stat = scratch + (size_t)n_slabs * GRp * chunks;
+  // keys of every slab: rows [slab * ncap + token], 128 dims
+  const uint64_t dims[2] = {(uint64_t)kHeadDim, (uint64_t)n_slabs * (uint64_t)P.ncap};
+  const uint64_t strides[1] = {(uint64_t)kHeadDim * 2};
+  const uint32_t box[2] = {64, kRmTile};
+  CUtensorMap map;
+  cudaError_t e = encode_bf16_map(&map, P.keys, 2, dims, strides, box);
+  if (e != cudaSuccess) return e;
+  const int nmb = (GRp + 127) / 128;
+  {
+    J.nbuf = nmb <= 2 ? 2 : 1;
+    J.stages = nmb <= 2 ? 4 : 2;
+    const size_t smem = 1024 + (size_t)nmb * 32768 + (size_t)J.stages * kRmStageBytes;
+    auto kern = nmb == 1 ? k_rm_stats<1> : nmb == 2 ? k_rm_stats<2> : nmb == 3 ? k_rm_stats<3>
+                                                                              : k_rm_stats<4>;
+    e = ensure_smem((const void*)kern, (int)smem);
+    if (e != cudaSuccess) return e;
+    e = launch_pdl(kern, dim3(chunks, n_slabs), dim3(64 + 128 * nmb), smem, s, map, B, J);
+    if (e != cudaSuccess) return e;
+  }
+  e = launch_pdl(k_rm_combine, dim3((n_slabs * GRp + 255) / 256), dim3(256), 0, s, B, J);
+  if (e != cudaSuccess) return e;
+  {
+    const bool two = GRp > 256;
+    const int NE = two ? ((GRp / 2 + 15) & ~15) : GRp;
+    const int qb = ((two ? 2 : 1) * NE * 256 + 1023) & ~1023;
+    J.nbuf = (two ? 2 * NE : NE) <= 256 ? 2 : 1;
+    J.stages = qb <= 64 * 1024 ? 4 : 3;
+    const size_t smem = 1024 + (size_t)qb + (size_t)J.stages * kRmStageBytes;
+    e = ensure_smem((const void*)k_rm_alpha, (int)smem);
+    if (e != cudaSuccess) return e;
+    e = launch_pdl(k_rm_alpha, dim3(chunks, n_slabs), dim3(64 + kRmEpi2), smem, s, map, B, J);
+  }
+  return e;
+}
+
+}  // namespace ss

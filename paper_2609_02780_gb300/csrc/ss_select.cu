@@ -217,8 +217,10 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
   if (pi >= B.n) return;
   const Prob& P = B.p[pi];
   if (retrieval_timed_out(P)) return;
-  const bool mean = kGeneral && B.head_agg == 1;  // one list per layer
-  const int n_lists = mean ? P.P : P.P * P.Hq;
+  // rows of weights rather than scores: one list per layer (head-averaged weights) or
+  // per-query-head lists of row-averaged weights; their candidate ids are the positions
+  const bool mean = kGeneral && (B.head_agg == 1 || B.q_agg == 2);
+  const int n_lists = (kGeneral && B.head_agg == 1) ? P.P : P.P * P.Hq;
   const int L = blockIdx.x;
   if (L >= n_lists) return;
   const int tid = threadIdx.x, lane = tid & 31;
@@ -303,15 +305,15 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
   const int cnt = kGeneral ? P.n_cand : P.cand_cnt[L];
   // candidates: (score, id) pairs appended by the score kernel, or the general path's
   // dense rows of values and ids
-  const float* cs = (mean ? P.aval : P.cand_s) + (int64_t)L * P.cand_cap;
-  const int32_t* ci = (mean ? P.aid : P.cand_id) + (int64_t)L * P.cand_cap;
+  const float* cs = (B.head_agg == 1 ? P.aval : P.cand_s) + (int64_t)L * P.cand_cap;
+  const int32_t* ci = P.cand_id + (int64_t)L * P.cand_cap;
   const float2* cp = P.cand_pair + (int64_t)L * P.cand_cap;
   auto sc_at = [&](int x) -> float {
     if constexpr (kGeneral) return cs[x];
     else return cp[x].x;
   };
   auto id_at = [&](int x) -> int32_t {
-    if constexpr (kGeneral) return ci[x];
+    if constexpr (kGeneral) return mean ? (int32_t)x : ci[x];
     else return __float_as_int(cp[x].y);
   };
   // Visits every candidate x < cnt with its value: thread t takes x = t, t + T, ... in
@@ -452,7 +454,7 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
       for (int e = 0; e < 4 * kU; ++e) {
         if ((kb >> e) & 1u) {
           const int x = 4 * (b0 + (e >> 2) * blockDim.x + tid) + (e & 3);
-          if (pos < kSelCap) skeys[pos] = cand_key(v[e], ci[x]);
+          if (pos < kSelCap) skeys[pos] = cand_key(v[e], id_at(x));
           ++pos;
         }
       }
