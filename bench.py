@@ -451,6 +451,12 @@ def run_ours(args):
         kernel = "k_dense"
         launches = 9   # k_sample, k_cluster_map, k_dense, k_select, k_centroid_weight,
         #                k_mass, k_pool, k_gram, k_maxmin
+    elif w.q_agg == 2:
+        # every question row attends: two passes over the keys (statistics, weights)
+        alg_bytes = 2 * keys * 256
+        kernel = "k_rm_stats + k_rm_combine + k_rm_alpha"
+        launches = 9   # k_sample, the three passes, k_select, k_mass_general, k_pool,
+        #                k_gram, k_maxmin
     else:
         alg_bytes = keys * 256
         kernel = "k_score"

@@ -444,7 +444,7 @@ cudaError_t launch_rowmean(const Batch& B, int pi, float2* scratch, int chunks, 
     const int NE = two ? ((GRp / 2 + 15) & ~15) : GRp;
     const int qb = ((two ? 2 : 1) * NE * 256 + 1023) & ~1023;
     J.nbuf = (two ? 2 * NE : NE) <= 256 ? 2 : 1;
-    J.stages = qb <= 64 * 1024 ? 4 : 3;
+    J.stages = qb <= 64 * 1024 ? 4 : qb <= 115 * 1024 ? 3 : 2;
     const size_t smem = 1024 + (size_t)qb + (size_t)J.stages * kRmStageBytes;
     e = ensure_smem((const void*)k_rm_alpha, (int)smem);
     if (e != cudaSuccess) return e;

@@ -101,6 +101,11 @@ PRESETS = {
     "batched16": Workload("batched16", n_layers=4, n_frames=1800, tokens_per_frame=196,
                           n_rows=32, k=1024, budget=48, n_planted=16,
                           keys="drift_outlier", seed=0, n_streams=16),
+    # the 1-hour stream with lists ranked by the mean of all 32 question rows' softmax
+    # weights (every row attends on its own)
+    "hour1_msm": Workload("hour1_msm", n_layers=4, n_frames=3600, tokens_per_frame=196,
+                          n_rows=32, k=1024, budget=64, n_planted=16,
+                          keys="drift_outlier", seed=0, q_agg=2),
     # Table 4 evidence-selection settings (Qwen3-VL column: 2-frame units, P = 5,
     # 64 candidates per layer averaged over heads, pool 32, K = 8, 6 recent units).
     "paper_qwen": Workload("paper_qwen", n_layers=5, n_frames=256, tokens_per_frame=64,
