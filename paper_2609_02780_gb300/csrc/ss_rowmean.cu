@@ -227,23 +227,39 @@ __global__ void __launch_bounds__(64 + 128 * NMB, 1)
         for (int hh = 0; hh < 2; ++hh) {
           float v0[32], v1[32];
           tmem_ld32x2(d + 64 * hh, d + 64 * hh + 32, v0, v1);
+          // (a full tile needs no per-column test; the max is taken on the raw dot
+          // products and scaled once)
           float mt = -INFINITY;
+          if (nv == kRmTile) {
 #pragma unroll
-          for (int c = 0; c < 32; ++c) {
-            if (64 * hh + c < nv) mt = fmaxf(mt, v0[c] * kScoreScale);
-            if (64 * hh + 32 + c < nv) mt = fmaxf(mt, v1[c] * kScoreScale);
+            for (int c = 0; c < 32; ++c) mt = fmaxf(mt, fmaxf(v0[c], v1[c]));
+          } else {
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+              if (64 * hh + c < nv) mt = fmaxf(mt, v0[c]);
+              if (64 * hh + 32 + c < nv) mt = fmaxf(mt, v1[c]);
+            }
           }
+          mt *= kScoreScale;
           if (mt > m) {
             l = (m == -INFINITY) ? 0.f : l * fast_exp2(m - mt);
             m = mt;
           }
-          float acc = 0.f;
+          float acc0 = 0.f, acc1 = 0.f;
+          if (nv == kRmTile) {
 #pragma unroll
-          for (int c = 0; c < 32; ++c) {
-            if (64 * hh + c < nv) acc += fast_exp2(fmaf(v0[c], kScoreScale, -m));
-            if (64 * hh + 32 + c < nv) acc += fast_exp2(fmaf(v1[c], kScoreScale, -m));
+            for (int c = 0; c < 32; ++c) {
+              acc0 += fast_exp2(fmaf(v0[c], kScoreScale, -m));
+              acc1 += fast_exp2(fmaf(v1[c], kScoreScale, -m));
+            }
+          } else {
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+              if (64 * hh + c < nv) acc0 += fast_exp2(fmaf(v0[c], kScoreScale, -m));
+              if (64 * hh + 32 + c < nv) acc1 += fast_exp2(fmaf(v1[c], kScoreScale, -m));
+            }
           }
-          l += acc;
+          l += acc0 + acc1;
         }
       }
       tc_fence_before();
@@ -262,7 +278,8 @@ __global__ void __launch_bounds__(64 + 128 * NMB, 1)
   if (warp == 1) tmem_dealloc(tbase, cols);
 }
 
-// (M, 1 / L) of every row from the chunks' partials, in chunk order.
+// The exponent offset M + log2(L) (and 1 / L) of every row from the chunks' partials,
+// combined in chunk order.
 __global__ void __launch_bounds__(256) k_rm_combine(const __grid_constant__ Batch B, const RmJob J) {
   pdl_wait();
   pdl_release();
@@ -278,7 +295,8 @@ __global__ void __launch_bounds__(256) k_rm_combine(const __grid_constant__ Batc
     const float2 v = J.part[(int64_t)x * J.chunks + c];
     if (v.y > 0.f) ml_combine(m, l, v.x, v.y);
   }
-  J.stat[x] = make_float2(m, l > 0.f ? 1.0f / l : 0.f);
+  // 2^(s - M) / L = 2^(s - (M + log2 L)): the weight needs one exponent offset per row
+  J.stat[x] = make_float2(l > 0.f ? m + __log2f(l) : INFINITY, l > 0.f ? 1.0f / l : 0.f);
 }
 
 // ---------------------------------------------------------------------------
@@ -292,7 +310,7 @@ __global__ void __launch_bounds__(64 + kRmEpi2, 1)
                const RmJob J) {
   extern __shared__ unsigned char sm_raw[];
   __shared__ RmBars S;
-  __shared__ float2 st[512];
+  __shared__ __align__(16) float st[512];   // exponent offset of every row
   unsigned char* sm = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const int GRp = J.GRp;
@@ -342,8 +360,11 @@ __global__ void __launch_bounds__(64 + kRmEpi2, 1)
     rm_bar(kRmEpi2);
     if (e == 0) mbar_arrive(smem_u32(&S.q_ready));
     pdl_wait();                                          // the rows' statistics (pass 1)
-    for (int x = e; x < GRp; x += kRmEpi2)
-      st[x] = J.stat[(int64_t)slab * GRp + x];
+    for (int x = e; x < GRp; x += kRmEpi2) {
+      const int hr = x / J.Rp, rr = x - hr * J.Rp;
+      // rows past R get an offset that makes their terms 0
+      st[x] = (hr < P.G && rr < P.R) ? J.stat[(int64_t)slab * GRp + x].x : INFINITY;
+    }
     rm_bar(kRmEpi2);
     pdl_release();
     const int G = P.G, Rp = J.Rp;
@@ -360,20 +381,40 @@ __global__ void __launch_bounds__(64 + kRmEpi2, 1)
       const int tok = (t0 + j) * kRmTile + tl;
       if (ok) {
         for (int h = h_begin; h < h_end; ++h) {
-          float a = 0.f;
-          for (int r0 = 0; r0 < Rp; r0 += 16) {
-            float v[16];
-            tmem_ld16(lane_addr + (uint32_t)buf * buf_cols + (uint32_t)(h * Rp + r0), v);
+          const uint32_t col = lane_addr + (uint32_t)buf * buf_cols + (uint32_t)(h * Rp);
+          const float* sh = st + h * Rp;
+          float a = 0.f, a2 = 0.f;
+          // a head's rows in one load and one wait where they fit 32 or 64 columns; the
+          // offsets four at a time (padding rows add 2^-inf = 0)
+          auto add = [&](const float (&v)[32], int r0) {
 #pragma unroll
-            for (int t = 0; t < 16; ++t) {
-              if (r0 + t < P.R) {
-                const float2 s2 = st[h * Rp + r0 + t];
-                a = fmaf(fast_exp2(fmaf(v[t], kScoreScale, -s2.x)), s2.y, a);
-              }
+            for (int t = 0; t < 32; t += 4) {
+              const float4 o = *reinterpret_cast<const float4*>(sh + r0 + t);
+              a += fast_exp2(fmaf(v[t], kScoreScale, -o.x));
+              a2 += fast_exp2(fmaf(v[t + 1], kScoreScale, -o.y));
+              a += fast_exp2(fmaf(v[t + 2], kScoreScale, -o.z));
+              a2 += fast_exp2(fmaf(v[t + 3], kScoreScale, -o.w));
+            }
+          };
+          if (Rp == 32) {
+            float v[32];
+            tmem_ld32(col, v);
+            add(v, 0);
+          } else if (Rp == 64) {
+            float v0[32], v1[32];
+            tmem_ld32x2(col, col + 32, v0, v1);
+            add(v0, 0);
+            add(v1, 32);
+          } else {
+            for (int r0 = 0; r0 < Rp; r0 += 16) {
+              float v[16];
+              tmem_ld16(col + (uint32_t)r0, v);
+#pragma unroll
+              for (int t = 0; t < 16; ++t) a += fast_exp2(fmaf(v[t], kScoreScale, -sh[r0 + t]));
             }
           }
           if (tok < n_tok)
-            P.cand_s[(int64_t)(i * P.Hq + g * G + h) * P.cand_cap + tok] = a * invR;
+            P.cand_s[(int64_t)(i * P.Hq + g * G + h) * P.cand_cap + tok] = (a + a2) * invR;
         }
       }
       tc_fence_before();
@@ -399,9 +440,10 @@ size_t rowmean_workspace_bytes(int n_slabs, int R, int G, int max_chunks) {
   return (size_t)n_slabs * GRp * (max_chunks + 1) * sizeof(float2);
 }
 
+// CTAs per slab: as many as fit in one wave (one CTA per SM), at least one.
 int rowmean_chunks(int n_slabs, int hist_tokens, int sm_count) {
   const int T = (hist_tokens + kRmTile - 1) / kRmTile;
-  int c = (sm_count + n_slabs - 1) / n_slabs;
+  int c = sm_count / n_slabs;
   c = c < 1 ? 1 : c;
   return T < c ? (T < 1 ? 1 : T) : c;
 }
