@@ -49,6 +49,9 @@ def parse():
                     help="frames of the stream one reference-arm step scores")
     ap.add_argument("--frames", type=int, default=0,
                     help="truncate the stream to this many frames (small profiling case)")
+    ap.add_argument("--sweep", action="store_true",
+                    help="query latency versus history length (64 frames to 3 h), with and "
+                         "without window compression; one JSON line per length")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args()
@@ -512,8 +515,69 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+SWEEP_FRAMES = (64, 128, 256, 512, 1024, 1800, 3600, 7200, 10800)
+
+
+def run_sweep(args):
+    """Query-time latency of one retrieval versus the length of the retained history (the
+    1-hour stream's shape at 1 fps: 64 frames to 3 hours), without compression (every key
+    scored) and with the history's 20-frame windows compressed to 64 centroids except the
+    latest 60 frames (LC-on: centroids and the recent raw tail scored). Device time of
+    the retrieval with CUDA events, p50 of the timed steps."""
+    import torch
+    import paper_2609_02780_gb300 as ss
+    from paper_2609_02780_gb300 import synth
+    dev = torch.device("cuda", 0)
+    base = synth.PRESETS["hour1"]
+    steps = max(10, args.steps)
+
+    def p50(fn):
+        for _ in range(3):
+            fn()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(steps)]
+        for a, b in ev:
+            a.record()
+            fn()
+            b.record()
+        torch.cuda.synchronize(dev)
+        return statistics.median(a.elapsed_time(b) for a, b in ev)
+
+    for frames in SWEEP_FRAMES:
+        w = base.replace(n_frames=frames, n_planted=max(1, min(16, frames // 64)))
+        data = synth.make_workload(w, device=dev)
+        idx = ss.Index(w.n_layers, w.n_q_heads, w.n_kv_heads, w.tokens_per_frame, frames,
+                       device=dev)
+        idx.append(data["keys"])
+        p = ss.RetrieveParams(k=w.k, budget=w.budget)
+        res = ss.Result(idx, p)
+        ws = torch.empty(idx.workspace_bytes(w.n_rows, p), dtype=torch.uint8, device=dev)
+        q = data["q"]
+        off = p50(lambda: idx.retrieve(q, k=p.k, budget=p.budget, out=res, workspace=ws))
+        on = None
+        n_comp = (max(0, frames - 60) // 20) * 20
+        if n_comp:
+            idx.compress(20, n_centroids=64, iters=5, first_frame=0, n_frames=n_comp)
+            pc = ss.RetrieveParams(k=512, budget=w.budget, use_clusters=1)
+            rc = ss.Result(idx, pc)
+            wc = torch.empty(idx.workspace_bytes(w.n_rows, pc), dtype=torch.uint8, device=dev)
+            on = p50(lambda: idx.retrieve(q, k=pc.k, budget=pc.budget, use_clusters=1, out=rc,
+                                          workspace=wc))
+        keys = w.keys_per_query
+        print(json.dumps({"sweep": "query latency vs history", "frames": frames,
+                          "hours": round(frames / 3600, 3), "keys": keys,
+                          "index_bytes": w.key_bytes, "lc_off_ms": off,
+                          "lc_off_keys_per_s": keys / (off / 1e3),
+                          "lc_on_ms": on, "lc_on_compressed_frames": n_comp}), flush=True)
+        del idx, data, res, ws
+        torch.cuda.empty_cache()
+
+
 def main():
     args = parse()
+    if args.sweep:
+        run_sweep(args)
+        return
     if args.impl == "reference":
         run_reference(args)
     else:
