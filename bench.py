@@ -311,12 +311,10 @@ def time_compress(ss, w, keys, dev, reps: int = 3) -> tuple[float, list[float]]:
 
 
 def host_copy_bytes(budget: int, nexp: int, frames_per_unit: int) -> int:
-    """Bytes of the one device-to-host copy of ss_retrieve_host: the selection, expansion,
-    frames, counts and status regions of the workspace, each starting at a 256-byte
-    boundary, up to the end of the status word."""
-    def a256(n):
-        return (n + 255) // 256 * 256
-    return a256(4 * budget) + a256(4 * nexp) + a256(4 * nexp * frames_per_unit) + 256 + 4
+    """Bytes that ss_retrieve_host's kernels write into page-locked host memory per call,
+    at most: the selection (K ids), the expansion and its frames (at most K (1 + n_prev)
+    units, times frames per unit), the four counts and the status word."""
+    return 4 * budget + 4 * nexp + 4 * nexp * frames_per_unit + 16 + 4
 
 
 def run_ours(args):
@@ -434,8 +432,8 @@ def run_ours(args):
         assert got["frames"] == call.frames(), "host entry point results differ"
         nexp = p.budget * (1 + p.n_prev)
         e2e = {"value": keys * args.steps * world / dt, "unit": UNIT,
-               # the host call copies only the rows the path reads (the last one of each
-               # layer under the default LAST reading, every row otherwise)
+               # the kernels read only the rows the path needs from the page-locked
+               # question (the last one of each layer under the default LAST reading)
                "h2d_bytes_per_step": int(q_pin.numel() * 2 // (q_pin.shape[1] if p.q_agg == 0 else 1)),
                "d2h_bytes_per_step": host_copy_bytes(p.budget, nexp, w.frames_per_unit),
                "ms_per_step": dt / args.steps * 1e3}

@@ -320,13 +320,15 @@ ss_status ss_retrieve_batched(ss_index* const* indexes, const void* const* q,
                               void* workspace, size_t workspace_bytes, void* stream,
                               const ss_trace* trace);
 
-/* ss_retrieve from host memory: copies `q_host` (bf16 [P][R][Hq][d]; pinned memory
- * makes the copy asynchronous; with SS_Q_LAST only each layer's last row, the only one
- * read, is copied) to the device, retrieves with every result array in the
- * workspace, brings the selection back with one copy into pinned memory that the
- * library keeps per host thread (allocated on the thread's first call, at least the
- * largest selection seen), unpacks it into `out` and synchronizes `stream`. Returns the
- * device status as well (TIMEOUT or INTERNAL). Errors as ss_retrieve. */
+/* ss_retrieve from host memory. `q_host` (bf16 [P][R][Hq][d]) in page-locked memory is
+ * read by the kernels in place through the device's mapping of it (on GB300 over
+ * NVLink-C2C; only the rows the query reading needs are read); pageable rows are first
+ * copied into the workspace (under SS_Q_LAST only each layer's last row). The
+ * selection, expansion, frames and counts are written by the kernels directly into
+ * page-locked host memory that the library keeps per host thread (allocated with
+ * cudaHostAlloc on the thread's first call, grown to the largest selection seen),
+ * then unpacked into `out` once `stream` is synchronized. Returns the device status
+ * as well (TIMEOUT or INTERNAL). Errors as ss_retrieve. */
 ss_status ss_retrieve_host(ss_index* index, const void* q_host, int32_t n_rows,
                            const ss_retrieve_params* params, const ss_host_result* out,
                            void* workspace, size_t workspace_bytes, void* stream);

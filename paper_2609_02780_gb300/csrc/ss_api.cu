@@ -227,7 +227,7 @@ struct ShardOut {
 ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t* R, int n,
                         const ss_retrieve_params* p, const ss_result* res, void* ws,
                         size_t ws_bytes, cudaStream_t st, const ss_trace* tr,
-                        const ShardOut* shard = nullptr) {
+                        const ShardOut* shard = nullptr, uint32_t* host_status = nullptr) {
   if (n < 1 || n > kMaxProbs) return fail(SS_ERR_INVALID_ARG, "n must be in [1, %d]", kMaxProbs);
   if (!ix || !q || !R || !res) return fail(SS_ERR_INVALID_ARG, "NULL argument");
   ss_status s = check_params(p);
@@ -317,6 +317,7 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
     P.frames = r.frames;
     P.counts = r.counts;
     P.status = r.status;
+    P.host_status = host_status;
     const int64_t pc = (int64_t)p->pool_mult * p->budget_units;
     P.pool_n = (int)(pc < P.Uh ? pc : P.Uh);
     P.n_sample = sample_units(p->k, P.Tu, P.Uh);
@@ -722,55 +723,77 @@ SS_EXPORT ss_status ss_retrieve_host(ss_index* ix, const void* q_host, int32_t R
   char* base = static_cast<char*>(ws);
   const size_t qbytes = (size_t)c.n_layers * R * c.n_q_heads * kHeadDim * 2;
   SS_CUDA(cudaSetDevice(ix->device));
-  if (p->q_agg == SS_Q_LAST) {
-    // only each layer's last question row is read: one strided copy of those rows
-    const size_t row = (size_t)c.n_q_heads * kHeadDim * 2;
-    SS_CUDA(cudaMemcpy2DAsync(base + l.qstage + (size_t)(R - 1) * row, (size_t)R * row,
-                              static_cast<const char*>(q_host) + (size_t)(R - 1) * row,
-                              (size_t)R * row, row, (size_t)c.n_layers,
-                              cudaMemcpyHostToDevice, st));
-  } else {
-    SS_CUDA(cudaMemcpyAsync(base + l.qstage, q_host, qbytes, cudaMemcpyHostToDevice, st));
+  // Question rows in page-locked host memory are read by the kernels in place (the device
+  // maps them; on GB300 through NVLink-C2C); pageable rows are copied into the workspace.
+  const void* q_dev = nullptr;
+  {
+    cudaPointerAttributes a{};
+    if (cudaPointerGetAttributes(&a, q_host) == cudaSuccess && a.type == cudaMemoryTypeHost &&
+        a.devicePointer)
+      q_dev = a.devicePointer;
+    cudaGetLastError();
   }
-  ss_result r{};
-  r.sel_units = reinterpret_cast<int32_t*>(base + l.sel);
-  r.exp_units = reinterpret_cast<int32_t*>(base + l.exp_units);
-  r.frames = reinterpret_cast<int32_t*>(base + l.frames);
-  r.counts = reinterpret_cast<int32_t*>(base + l.counts);
-  r.status = reinterpret_cast<uint32_t*>(base + l.status);
-  s = ss_retrieve(ix, base + l.qstage, R, p, &r, ws, ws_bytes, stream, nullptr);
-  if (s != SS_OK) return s;
+  if (!q_dev) {
+    if (p->q_agg == SS_Q_LAST) {
+      // only each layer's last question row is read: one strided copy of those rows
+      const size_t row = (size_t)c.n_q_heads * kHeadDim * 2;
+      SS_CUDA(cudaMemcpy2DAsync(base + l.qstage + (size_t)(R - 1) * row, (size_t)R * row,
+                                static_cast<const char*>(q_host) + (size_t)(R - 1) * row,
+                                (size_t)R * row, row, (size_t)c.n_layers,
+                                cudaMemcpyHostToDevice, st));
+    } else {
+      SS_CUDA(cudaMemcpyAsync(base + l.qstage, q_host, qbytes, cudaMemcpyHostToDevice, st));
+    }
+    q_dev = base + l.qstage;
+  }
+  // The selection, expansion, frames, counts and status copy are written by the kernels
+  // straight into page-locked host memory that the library keeps per host thread
+  // (allocated on the thread's first call, grown to the largest selection seen).
   const size_t nsel = (size_t)p->budget_units;
   const size_t nexp = nsel * (1 + p->n_prev);
-  // The selection, expansion, frames, counts and status words are consecutive regions of
-  // the workspace: one copy brings them back (into pinned memory kept per host thread),
-  // then they are unpacked into the caller's buffers.
+  const size_t nfr = nexp * c.frames_per_unit;
+  const size_t o_exp = align256(nsel * 4), o_fr = o_exp + align256(nexp * 4),
+               o_cnt = o_fr + align256(nfr * 4), o_st = o_cnt + 256, span = o_st + 256;
   struct PinnedStage {
     char* p = nullptr;
+    char* d = nullptr;
     size_t bytes = 0;
     ~PinnedStage() {
       if (p) cudaFreeHost(p);
     }
   };
   static thread_local PinnedStage stage;
-  const size_t span = l.status + sizeof(uint32_t) - l.sel;
   if (stage.bytes < span) {
     if (stage.p) cudaFreeHost(stage.p);
-    stage.p = nullptr;
+    stage.p = stage.d = nullptr;
     stage.bytes = 0;
-    SS_CUDA(cudaMallocHost(reinterpret_cast<void**>(&stage.p), span));
+    SS_CUDA(cudaHostAlloc(reinterpret_cast<void**>(&stage.p), span, cudaHostAllocMapped));
+    SS_CUDA(cudaHostGetDevicePointer(reinterpret_cast<void**>(&stage.d), stage.p, 0));
     stage.bytes = span;
   }
-  SS_CUDA(cudaMemcpyAsync(stage.p, base + l.sel, span, cudaMemcpyDeviceToHost, st));
+  ss_result r{};
+  r.sel_units = reinterpret_cast<int32_t*>(stage.d);
+  r.exp_units = reinterpret_cast<int32_t*>(stage.d + o_exp);
+  r.frames = reinterpret_cast<int32_t*>(stage.d + o_fr);
+  r.counts = reinterpret_cast<int32_t*>(stage.d + o_cnt);
+  r.status = reinterpret_cast<uint32_t*>(base + l.status);   // device-side atomics stay in HBM
+  uint32_t* host_status = reinterpret_cast<uint32_t*>(stage.d + o_st);
+  *reinterpret_cast<volatile uint32_t*>(stage.p + o_st) = 0xffffffffu;  // set by the last kernel
+  {
+    ss_index* const arr[1] = {ix};
+    const void* const qa[1] = {q_dev};
+    s = retrieve_impl(arr, qa, &R, 1, p, &r, ws, ws_bytes, st, nullptr, nullptr, host_status);
+  }
+  if (s != SS_OK) return s;
   SS_CUDA(cudaStreamSynchronize(st));
-  uint32_t v = 0;
-  std::memcpy(&v, stage.p + (l.status - l.sel), sizeof(v));
+  const uint32_t v = *reinterpret_cast<volatile uint32_t*>(stage.p + o_st);
+  if (v == 0xffffffffu) return fail(SS_ERR_INTERNAL, "the retrieval did not report its status");
   if (v & kStatusTimeout) return fail(SS_ERR_TIMEOUT, "a bounded device-side wait gave up");
   if (v & kStatusInternal) return fail(SS_ERR_INTERNAL, "a device-side consistency check failed");
   std::memcpy(out->sel_units, stage.p, nsel * 4);
-  std::memcpy(out->exp_units, stage.p + (l.exp_units - l.sel), nexp * 4);
-  std::memcpy(out->frames, stage.p + (l.frames - l.sel), nexp * c.frames_per_unit * 4);
-  std::memcpy(out->counts, stage.p + (l.counts - l.sel), 16);
+  std::memcpy(out->exp_units, stage.p + o_exp, nexp * 4);
+  std::memcpy(out->frames, stage.p + o_fr, nfr * 4);
+  std::memcpy(out->counts, stage.p + o_cnt, 16);
   return SS_OK;
 }
 

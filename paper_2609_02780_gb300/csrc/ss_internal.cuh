@@ -112,6 +112,7 @@ struct Prob {
   int32_t* frames;
   int32_t* counts;             // n_pool, n_sel, n_exp, n_frames
   uint32_t* status;
+  uint32_t* host_status;       // copy of the final status word in mapped host memory, or NULL
   // general path (one list per layer, or centroids of compressed windows as candidates):
   // every candidate is scored into a dense row per list
   int n_cand;                  // candidates per list

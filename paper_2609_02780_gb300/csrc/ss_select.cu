@@ -1126,7 +1126,14 @@ __global__ void __launch_bounds__(kMaxMinThreads) k_maxmin(const __grid_constant
   }
   pdl_wait();
   pdl_release();
-  if (retrieval_timed_out(P)) return;   // no copy was issued
+  // the last kernel of a retrieval: it also copies the status word for a host caller
+  auto publish_status = [&]() {
+    if (P.host_status) *(volatile uint32_t*)P.host_status = *(volatile const uint32_t*)P.status;
+  };
+  if (retrieval_timed_out(P)) {   // no copy was issued
+    if (tid == 0) publish_status();
+    return;
+  }
   if (staged && tid == 0) {
     const uint8_t* g8 = reinterpret_cast<const uint8_t*>(P.gram);
     mbar_expect_tx(bar, (uint32_t)gram_stage_bytes(pn));
@@ -1143,7 +1150,11 @@ __global__ void __launch_bounds__(kMaxMinThreads) k_maxmin(const __grid_constant
   const int lane = tid;
   if (staged && !mbar_wait_bounded(bar, 0u)) {
     // report, then let the copies in flight land before the CTA exits
-    if (lane == 0) atomicOr(P.status, kStatusTimeout);
+    if (lane == 0) {
+      atomicOr(P.status, kStatusTimeout);
+      __threadfence();
+      publish_status();
+    }
     mbar_wait_bounded(bar, 0u);
     return;
   }
@@ -1209,6 +1220,11 @@ __global__ void __launch_bounds__(kMaxMinThreads) k_maxmin(const __grid_constant
     counts[1] = ns;
     counts[2] = incl;
     counts[3] = incl * fpu;
+  }
+  __syncwarp();
+  if (lane == 0) {
+    __threadfence();
+    publish_status();
   }
 }
 

@@ -1,5 +1,5 @@
 """Host-side pieces of bench.py that need no GPU: the clock record of the timed region
-and the byte count of the host call's device-to-host copy."""
+and the byte count of what the host call's kernels write into host memory."""
 import datetime
 import os
 import sys
@@ -35,8 +35,8 @@ def test_clock_record_falls_back_to_the_whole_run():
     assert c["samples"] == 2 and c["window"] == "whole run" and c["sm_mhz"] == 1935.0
 
 
-def test_host_copy_bytes_follow_the_workspace_alignment():
+def test_host_copy_bytes_count_what_the_kernels_write_to_host_memory():
     import bench
-    # hour1: K = 64, n_prev = 1, one frame per unit
-    assert bench.host_copy_bytes(64, 128, 1) == 256 + 512 + 512 + 256 + 4
-    assert bench.host_copy_bytes(1, 2, 2) == 256 + 256 + 256 + 256 + 4
+    # hour1: K = 64, n_prev = 1, one frame per unit: ids, expansion, frames, counts, status
+    assert bench.host_copy_bytes(64, 128, 1) == 256 + 512 + 512 + 16 + 4
+    assert bench.host_copy_bytes(1, 2, 2) == 4 + 8 + 16 + 16 + 4

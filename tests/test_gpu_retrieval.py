@@ -191,13 +191,17 @@ def test_host_entry_point_matches_device_path():
     # repeated calls with other questions (the host call copies only the rows it reads
     # under LAST, every row under MEAN_LOGIT) agree with the device path each time
     _, q2 = gaussian_case(12, P=2, Hq=8, Hkv=2, F=64, Tf=32)
-    for q_agg in (0, 1):
+    # page-locked rows are read by the kernels in place, pageable rows are copied first;
+    # both agree with the device path, under every row reading
+    for q_agg in (0, 1, 2):
         pq = ss.RetrieveParams(k=70, budget=6, q_agg=q_agg)
-        for qq in (q2, q, q2):
+        for qq in (q2, q.pin_memory(), q2.pin_memory(), q):
             host = idx.retrieve_host(qq, pq)
             dev = idx.retrieve(qq.cuda(), k=70, budget=6, q_agg=q_agg).host()
             assert host["sel"] == dev["sel"] and host["frames"] == dev["frames"]
             assert host["expanded"] == dev["expanded"]
+            assert host["counts"][1:] == [len(dev["sel"]), len(dev["expanded"]),
+                                          len(dev["frames"])]
 
 
 def test_invalid_arguments_fail_before_launch():
