@@ -15,5 +15,8 @@ Plain, slow, fp64 numpy written from the paper's definitions:
   shard.py      one shard's share of a retrieval over an index split by token range
                 (its top-k candidates with scores, softmax statistics per list and
                 per unit, descriptors)
+  unit_clusters.py  the paper's long-history compression (Sec. 4.1, Eq. 5-7: units
+                leaving the detailed window clustered online, representative keys as
+                running averages) and the cluster evidence of Eq. 13
 """
-from . import retrieval, kmeans, shard  # noqa: F401
+from . import retrieval, kmeans, shard, unit_clusters  # noqa: F401
