@@ -94,6 +94,14 @@ typedef struct {
   const int32_t* member_counts; /* device int32 [P][Hkv][W_cap][n_centroids][window units]:
                                    members of each centroid in each unit of its window */
   const int32_t* member_sizes;  /* device int32 [P][Hkv][W_cap][n_centroids] */
+  /* long-history compression (ss_index_cluster_units) */
+  int64_t n_clustered_units;    /* units [0, n) have left the detailed window */
+  int32_t cluster_capacity;     /* 0 until the first clustering */
+  const int32_t* unit_cluster;  /* device int32 [U_cap]: cluster of a clustered unit, -1 */
+  const int32_t* cluster_count; /* device int32 [1]: clusters so far */
+  const float* cluster_centroids; /* device fp32 [capacity][Hkv * d] (unit norm) */
+  const int32_t* cluster_sizes; /* device int32 [capacity] members */
+  const float* cluster_keys;    /* device fp32 [capacity][P][Hkv][T_u][d] representative keys */
 } ss_index_view;
 
 /* k-means compression of the frames [first_frame, first_frame + n_frames) in
@@ -274,6 +282,42 @@ ss_status ss_index_get_view(const ss_index* index, ss_index_view* view);
  * than 65536 tokens), ALLOC (nothing is kept; the call can be repeated), CUDA. */
 ss_status ss_index_compress(ss_index* index, const ss_compress_params* params,
                             void* stream);
+
+/* The paper's long-history compression (Sec. 4.1, Eq. 6-7): the next n_units oldest
+ * detailed units leave the detailed window, in order. A leaving unit t joins the latest
+ * cluster C_j when its descriptor k_t (Eq. 3) satisfies k_t . c_j >= tau, and then
+ * c_j <- Norm((n_j c_j + k_t) / (n_j + 1)); otherwise it starts the next cluster with
+ * c = k_t (the first unit to leave starts cluster 0). Each cluster keeps representative
+ * keys, the running average (n K + K_t) / (n + 1) of its members' keys at every (layer,
+ * key head, token slot of a unit, dim), in fp32. Retrieval then scores only the detailed
+ * units (the clustered ones get no votes and no mass; a selected unit's predecessor is
+ * added only if it is detailed), and ss_select_clusters gives the cluster evidence.
+ * Decisions use fp32 dot products reduced in a fixed order, so repeated calls give the
+ * same clusters. The first call fixes max_clusters (1..16384, at most the unit capacity)
+ * and allocates fp32 [max_clusters][P][Hkv][T_u][d] for the representatives. More
+ * clusters than that raise SS_ERR_INTERNAL in the status of later retrievals.
+ * Errors: INVALID_ARG (n_units beyond the complete detailed units, NaN tau, another
+ * max_clusters), STATE (the index has k-means windows), ALLOC, CUDA. */
+ss_status ss_index_cluster_units(ss_index* index, int64_t n_units, float tau,
+                                 int32_t max_clusters, void* stream);
+
+/* Eq. 5 as a budget on the detailed units' keys: *n_units = how many of the oldest
+ * detailed units must leave the detailed window so that the detailed keys fit
+ * budget_bytes, never taking units from the latest near_term_units (the near-term and
+ * recent context). Host-only. */
+ss_status ss_index_units_over_budget(const ss_index* index, int64_t budget_bytes,
+                                     int64_t near_term_units, int64_t* n_units);
+
+/* The cluster evidence of a question (Sec. 4.2, Eq. 13): every cluster's centroid scored
+ * against the query state of the last shallow layer, score_j = (1/Hq) sum_h
+ * q_h . c_j[h / G] / sqrt(d), with q_h the last question row (SS_Q_LAST) or the rows'
+ * mean rounded to bf16 (the other readings), and c_j[g] the 128 entries of key head g;
+ * then the first min(k_l, clusters) clusters by (score desc, id asc). Device outputs:
+ * ids [k_l] (-1 past the count), scores [k_l], count [1]. Errors: INVALID_ARG, STATE (no
+ * clusters), UNSUPPORTED (k_l outside [1, 1024]), CUDA. */
+ss_status ss_select_clusters(ss_index* index, const void* q, int32_t n_rows, int32_t q_agg,
+                             int32_t k_l, int32_t* ids, float* scores, int32_t* count,
+                             void* stream);
 
 /* Bytes of device workspace that ss_retrieve_batched needs for these indexes, row
  * counts and parameters (ss_retrieve: n = 1). Depends on the indexes' capacities, not

@@ -233,6 +233,53 @@ class Index:
                 "window_first_unit": wf[:nw], "window_frames": v.window_frames,
                 "n_centroids": nc}
 
+    def cluster_units(self, n_units: int, tau: float, max_clusters: int) -> None:
+        """ss_index_cluster_units: the next n_units oldest detailed units leave the detailed
+        window and join clusters (Sec. 4.1, Eq. 6-7)."""
+        with torch.cuda.device(self.device):
+            _check(_lib().ss_index_cluster_units(self.handle, int(n_units), float(tau),
+                                                 int(max_clusters),
+                                                 C.c_void_p(_stream_ptr(self.device))))
+
+    def units_over_budget(self, budget_bytes: int, near_term_units: int) -> int:
+        """ss_index_units_over_budget (Eq. 5): detailed units that must leave."""
+        n = C.c_int64()
+        _check(_lib().ss_index_units_over_budget(self.handle, int(budget_bytes),
+                                                 int(near_term_units), C.byref(n)))
+        return n.value
+
+    def unit_clusters(self) -> dict:
+        """Views of the long-history compression's device arrays: unit_cluster [n_clustered],
+        centroids [C][Hkv * 128], sizes [C], keys fp32 [C][P][Hkv][T_u][128]."""
+        v = self.view()
+        if v.cluster_capacity == 0:
+            raise ValueError("the index has no unit clusters")
+        cap = v.cluster_capacity
+        tu = self.tokens_per_frame * self.frames_per_unit
+        cnt = self._block_view(v.cluster_count, torch.int32, (1,))
+        n_c = int(cnt.item())
+        uc = self._block_view(v.unit_cluster, torch.int32, (self.unit_capacity,))
+        cen = self._block_view(v.cluster_centroids, torch.float32, (cap, self.n_kv_heads * 128))
+        sz = self._block_view(v.cluster_sizes, torch.int32, (cap,))
+        ck = self._block_view(v.cluster_keys, torch.float32,
+                              (cap, self.n_layers, self.n_kv_heads, tu, 128))
+        return {"n_clustered_units": v.n_clustered_units, "unit_cluster": uc[:v.n_clustered_units],
+                "centroids": cen[:n_c], "sizes": sz[:n_c], "keys": ck[:n_c]}
+
+    def select_clusters(self, q: torch.Tensor, k_l: int, q_agg: int = Q_LAST) -> dict:
+        """ss_select_clusters (Eq. 13): the top k_l clusters for question rows q."""
+        if q.dtype != torch.bfloat16 or q.dim() != 4 or not q.is_contiguous() or q.device != self.device:
+            raise ValueError("q must be contiguous bf16 [P][R][Hq][128] on the index's device")
+        ids = torch.empty(k_l, dtype=torch.int32, device=self.device)
+        sc = torch.empty(k_l, dtype=torch.float32, device=self.device)
+        cnt = torch.empty(1, dtype=torch.int32, device=self.device)
+        with torch.cuda.device(self.device):
+            _check(_lib().ss_select_clusters(self.handle, C.c_void_p(q.data_ptr()), q.shape[1],
+                                             int(q_agg), int(k_l), C.c_void_p(ids.data_ptr()),
+                                             C.c_void_p(sc.data_ptr()), C.c_void_p(cnt.data_ptr()),
+                                             C.c_void_p(_stream_ptr(self.device))))
+        return {"ids": ids, "scores": sc, "count": cnt, "_keep": q}
+
     def append(self, keys: torch.Tensor, n_frames: int | None = None) -> None:
         """Appends frames of shallow keys bf16 [P][Hkv][S][128] (the first
         n_frames * T_f tokens of each slab; S may exceed that)."""

@@ -29,7 +29,10 @@ class IndexView(C.Structure):
                 ("window_frames", C.c_int32), ("n_centroids", C.c_int32),
                 ("centroids", C.c_void_p), ("assignment", C.c_void_p),
                 ("window_first_unit", C.c_void_p), ("member_counts", C.c_void_p),
-                ("member_sizes", C.c_void_p)]
+                ("member_sizes", C.c_void_p), ("n_clustered_units", C.c_int64),
+                ("cluster_capacity", C.c_int32), ("unit_cluster", C.c_void_p),
+                ("cluster_count", C.c_void_p), ("cluster_centroids", C.c_void_p),
+                ("cluster_sizes", C.c_void_p), ("cluster_keys", C.c_void_p)]
 
 
 class CompressParams(C.Structure):
@@ -110,6 +113,12 @@ SIGNATURES = {
                                      C.POINTER(RetrieveParams), C.c_int64,
                                      C.POINTER(ShardResult), C.c_void_p, C.c_size_t,
                                      C.c_void_p]),
+    "ss_index_cluster_units": (c_status, [C.c_void_p, C.c_int64, C.c_float, C.c_int32,
+                                          C.c_void_p]),
+    "ss_index_units_over_budget": (c_status, [C.c_void_p, C.c_int64, C.c_int64,
+                                              C.POINTER(C.c_int64)]),
+    "ss_select_clusters": (c_status, [C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_int32,
+                                      C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
     "ss_merge_shards": (c_status, [C.POINTER(Shard), C.c_int32, C.c_int32, C.c_int32,
                                    C.c_int32, C.c_int32, C.POINTER(RetrieveParams),
                                    C.POINTER(MergeResult)]),

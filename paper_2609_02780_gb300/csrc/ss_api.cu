@@ -41,6 +41,17 @@ struct ss_index {
   int32_t* mcnt;        // [P*Hkv][wcap][nc][units per window] members per (centroid, unit)
   int32_t* msize;       // [P*Hkv][wcap][nc] members per centroid
   uint32_t* kstatus;    // device word: a compression's wait gave up (kStatusTimeout)
+  // long-history compression (clusters of units that left the detailed window)
+  int64_t n_clustered;  // clustered units: the prefix [0, n_clustered)
+  int32_t uc_cap;       // cluster capacity (0 until the first clustering)
+  int32_t* unit_cluster;
+  float* cdesc;
+  int32_t* ccount;
+  float* creps;
+  int32_t* cfirst;
+  int32_t* cprev;
+  int32_t* uc_count;    // device: [0] clusters, [1] first cluster the last call touched
+  float* uc_work;
 };
 
 namespace {
@@ -206,8 +217,10 @@ ss_status check_params(const ss_retrieve_params* p) {
   return SS_OK;
 }
 
+// History units scored by a retrieval: the detailed units after the clustered prefix,
+// minus the recent ones (Eq. 4).
 int64_t hist_units_of(const ss_index* ix, const ss_retrieve_params* p) {
-  const int64_t u = ix->n_units - p->n_recent_units;
+  const int64_t u = ix->n_units - ix->n_clustered - p->n_recent_units;
   return u > 0 ? u : 0;
 }
 
@@ -245,6 +258,8 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
       return fail(SS_ERR_UNSUPPORTED, "more than %d history units", kMaxHistUnits);
     if (p->use_clusters && ix[j]->n_windows == 0)
       return fail(SS_ERR_STATE, "index %d has no compressed windows", j);
+    if (shard && ix[j]->n_clustered > 0)
+      return fail(SS_ERR_UNSUPPORTED, "a shard with clustered units");
     if (p->q_agg == SS_Q_MEAN_SOFTMAX &&
         !rowmean_supported(R[j], ix[j]->cfg.n_q_heads / ix[j]->cfg.n_kv_heads))
       return fail(SS_ERR_UNSUPPORTED,
@@ -277,8 +292,13 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
     const ss_index_config& c = x->cfg;
     const Layout l = layout_of(x, R[j], p);
     Prob& P = B.p[j];
-    P.keys = x->keys;
-    P.desc = x->desc;
+    // with clustered units the kernels see the index from its first detailed unit on;
+    // k_uc_shift moves the outputs back to stream numbering
+    const int64_t uoff = x->n_clustered;
+    const int64_t tu = (int64_t)c.tokens_per_frame * c.frames_per_unit;
+    P.unit_offset = (int)uoff;
+    P.keys = x->keys + uoff * tu * kHeadDim;
+    P.desc = x->desc + uoff * c.n_kv_heads * kHeadDim;
     P.ncap = x->ncap;
     P.P = c.n_layers;
     P.Hq = c.n_q_heads;
@@ -286,9 +306,9 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
     P.G = c.n_q_heads / c.n_kv_heads;
     P.fpu = c.frames_per_unit;
     P.Tu = c.tokens_per_frame * c.frames_per_unit;
-    P.U = (int)x->n_units;
+    P.U = (int)(x->n_units - uoff);
     P.Uh = (int)hist_units_of(x, p);
-    P.ucap = (int)x->ucap;
+    P.ucap = (int)(x->ucap - uoff);
     P.index_status = x->kstatus;
     P.q = static_cast<const __nv_bfloat16*>(q[j]);
     P.R = R[j];
@@ -309,8 +329,10 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
     P.topk_w = pick(r.topk_w, base, l.topk_w);
     P.topk_s = shard ? shard->topk_s : nullptr;
     P.list_ml = pick(reinterpret_cast<float2*>(r.list_stats), base, l.list_ml);
-    P.votes = pick(r.unit_votes, base, l.votes);
-    P.mass = pick(r.unit_mass, base, l.mass);
+    P.votes_base = pick(r.unit_votes, base, l.votes);
+    P.mass_base = pick(r.unit_mass, base, l.mass);
+    P.votes = P.votes_base + uoff;
+    P.mass = P.mass_base + uoff;
     P.pool = pick(r.pool, base, l.pool);
     P.sel = r.sel_units;
     P.exp_units = r.exp_units;
@@ -408,6 +430,9 @@ ss_status retrieve_impl(ss_index* const* ix, const void* const* q, const int32_t
   }
   SS_CUDA(launch_pool(B, max_uh, st));
   SS_CUDA(launch_maxmin(B, max_pool, st));
+  bool shifted = false;
+  for (int j = 0; j < n; ++j) shifted = shifted || B.p[j].unit_offset > 0;
+  if (shifted) SS_CUDA(launch_uc_shift(B, st));
   return SS_OK;
 }
 
@@ -500,6 +525,14 @@ SS_EXPORT ss_status ss_index_destroy(ss_index* ix) {
   dev_free(ix, ix->mcnt);
   dev_free(ix, ix->msize);
   dev_free(ix, ix->kstatus);
+  dev_free(ix, ix->unit_cluster);
+  dev_free(ix, ix->cdesc);
+  dev_free(ix, ix->ccount);
+  dev_free(ix, ix->creps);
+  dev_free(ix, ix->cfirst);
+  dev_free(ix, ix->cprev);
+  dev_free(ix, ix->uc_count);
+  dev_free(ix, ix->uc_work);
   delete ix;
   return SS_OK;
 }
@@ -547,6 +580,13 @@ SS_EXPORT ss_status ss_index_get_view(const ss_index* ix, ss_index_view* v) {
   v->window_first_unit = ix->win_u0;
   v->member_counts = ix->mcnt;
   v->member_sizes = ix->msize;
+  v->n_clustered_units = ix->n_clustered;
+  v->cluster_capacity = ix->uc_cap;
+  v->unit_cluster = ix->unit_cluster;
+  v->cluster_count = ix->uc_count;
+  v->cluster_centroids = ix->cdesc;
+  v->cluster_sizes = ix->ccount;
+  v->cluster_keys = ix->creps;
   return SS_OK;
 }
 
@@ -577,6 +617,8 @@ SS_EXPORT ss_status ss_index_compress(ss_index* ix, const ss_compress_params* cp
     if (q.first_frame < end)
       return fail(SS_ERR_INVALID_ARG, "frames before %lld are already compressed", (long long)end);
   }
+  if (ix->n_clustered > 0)
+    return fail(SS_ERR_STATE, "the index already clusters units (ss_index_cluster_units)");
   if (q.n_frames == 0) return SS_OK;
   const cudaStream_t st = static_cast<cudaStream_t>(stream);
   SS_CUDA(cudaSetDevice(ix->device));
@@ -625,6 +667,125 @@ SS_EXPORT ss_status ss_index_compress(ss_index* ix, const ss_compress_params* cp
   for (int j = 0; j < n_new; ++j)
     ix->win_first_frame.push_back(q.first_frame + (int64_t)j * q.window_frames);
   ix->n_windows += n_new;
+  return SS_OK;
+}
+
+SS_EXPORT ss_status ss_index_cluster_units(ss_index* ix, int64_t n_units, float tau,
+                                           int32_t max_clusters, void* stream) {
+  if (!ix) return fail(SS_ERR_INVALID_ARG, "index is NULL");
+  if (n_units < 0) return fail(SS_ERR_INVALID_ARG, "n_units must be >= 0");
+  if (tau != tau) return fail(SS_ERR_INVALID_ARG, "tau is NaN");
+  if (ix->n_windows > 0)
+    return fail(SS_ERR_STATE, "the index already has k-means windows (ss_index_compress)");
+  if (ix->n_clustered + n_units > ix->n_units)
+    return fail(SS_ERR_INVALID_ARG, "only %lld detailed units are complete",
+                (long long)(ix->n_units - ix->n_clustered));
+  const ss_index_config& c = ix->cfg;
+  const int D = c.n_kv_heads * kHeadDim;
+  if (ix->uc_cap == 0) {
+    if (max_clusters < 1 || max_clusters > ix->ucap || max_clusters > 16384)
+      return fail(SS_ERR_INVALID_ARG, "max_clusters must be in [1, min(unit capacity, 16384)]");
+  } else if (max_clusters != ix->uc_cap) {
+    return fail(SS_ERR_INVALID_ARG, "max_clusters differs from the first clustering call");
+  }
+  if (n_units == 0) return SS_OK;
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  SS_CUDA(cudaSetDevice(ix->device));
+  const int n_slabs = c.n_layers * c.n_kv_heads;
+  const int64_t Tu = (int64_t)c.tokens_per_frame * c.frames_per_unit;
+  if (ix->uc_cap == 0) {
+    const int64_t cap = max_clusters;
+    ix->unit_cluster = static_cast<int32_t*>(dev_alloc(ix, (size_t)ix->ucap * 4, st));
+    ix->cdesc = static_cast<float*>(dev_alloc(ix, (size_t)cap * D * 4, st));
+    ix->ccount = static_cast<int32_t*>(dev_alloc(ix, (size_t)cap * 4, st));
+    ix->creps = static_cast<float*>(dev_alloc(ix, (size_t)cap * n_slabs * Tu * kHeadDim * 4, st));
+    ix->cfirst = static_cast<int32_t*>(dev_alloc(ix, (size_t)cap * 4, st));
+    ix->cprev = static_cast<int32_t*>(dev_alloc(ix, (size_t)cap * 4, st));
+    ix->uc_count = static_cast<int32_t*>(dev_alloc(ix, 256, st));
+    ix->uc_work = static_cast<float*>(dev_alloc(ix, (size_t)cap * 4, st));
+    if (!ix->kstatus) ix->kstatus = static_cast<uint32_t*>(dev_alloc(ix, 256, st));
+    if (!ix->unit_cluster || !ix->cdesc || !ix->ccount || !ix->creps || !ix->cfirst ||
+        !ix->cprev || !ix->uc_count || !ix->uc_work || !ix->kstatus) {
+      void** arrs[] = {(void**)&ix->unit_cluster, (void**)&ix->cdesc, (void**)&ix->ccount,
+                       (void**)&ix->creps, (void**)&ix->cfirst, (void**)&ix->cprev,
+                       (void**)&ix->uc_count, (void**)&ix->uc_work};
+      for (void** a : arrs) {
+        dev_free(ix, *a);
+        *a = nullptr;
+      }
+      return fail(SS_ERR_ALLOC, "device allocation of the cluster arrays failed");
+    }
+    SS_CUDA(cudaMemsetAsync(ix->unit_cluster, 0xff, (size_t)ix->ucap * 4, st));
+    SS_CUDA(cudaMemsetAsync(ix->uc_count, 0, 256, st));
+    SS_CUDA(cudaMemsetAsync(ix->kstatus, 0, 4, st));
+    ix->uc_cap = max_clusters;
+  }
+  UcJob J;
+  J.desc = ix->desc;
+  J.keys = ix->keys;
+  J.ncap = ix->ncap;
+  J.n_slabs = n_slabs;
+  J.Tu = (int)Tu;
+  J.D = D;
+  J.u0 = (int)ix->n_clustered;
+  J.n = (int)n_units;
+  J.tau = tau;
+  J.cap = ix->uc_cap;
+  J.n_clusters = ix->uc_count;
+  J.cdesc = ix->cdesc;
+  J.ccount = ix->ccount;
+  J.creps = ix->creps;
+  J.unit_cluster = ix->unit_cluster;
+  J.cfirst = ix->cfirst;
+  J.cprev = ix->cprev;
+  J.first_touched = ix->uc_count + 1;
+  J.status = ix->kstatus;
+  SS_CUDA(launch_uc_cluster(J, st));
+  ix->n_clustered += n_units;
+  return SS_OK;
+}
+
+SS_EXPORT ss_status ss_index_units_over_budget(const ss_index* ix, int64_t budget_bytes,
+                                               int64_t near_term_units, int64_t* n_units) {
+  if (!ix || !n_units) return fail(SS_ERR_INVALID_ARG, "NULL argument");
+  if (budget_bytes < 0 || near_term_units < 0)
+    return fail(SS_ERR_INVALID_ARG, "budget_bytes and near_term_units must be >= 0");
+  const ss_index_config& c = ix->cfg;
+  const int64_t unit_bytes = (int64_t)c.n_layers * c.n_kv_heads * c.tokens_per_frame *
+                             c.frames_per_unit * kHeadDim * 2;
+  const int64_t detailed = ix->n_units - ix->n_clustered;
+  int64_t keep = budget_bytes / unit_bytes;
+  if (keep < near_term_units) keep = near_term_units;
+  *n_units = detailed > keep ? detailed - keep : 0;
+  return SS_OK;
+}
+
+SS_EXPORT ss_status ss_select_clusters(ss_index* ix, const void* q, int32_t R, int32_t q_agg,
+                                       int32_t k_l, int32_t* ids, float* scores,
+                                       int32_t* count, void* stream) {
+  if (!ix || !q || !ids || !scores || !count) return fail(SS_ERR_INVALID_ARG, "NULL argument");
+  if (R < 1) return fail(SS_ERR_INVALID_ARG, "n_rows must be >= 1");
+  if (q_agg != SS_Q_LAST && q_agg != SS_Q_MEAN_LOGIT && q_agg != SS_Q_MEAN_SOFTMAX)
+    return fail(SS_ERR_INVALID_ARG, "unknown q_agg %d", q_agg);
+  if (k_l < 1 || k_l > 1024) return fail(SS_ERR_UNSUPPORTED, "k_l must be in [1, 1024]");
+  if (ix->uc_cap == 0) return fail(SS_ERR_STATE, "the index has no unit clusters");
+  const ss_index_config& c = ix->cfg;
+  UcSel S;
+  S.q = static_cast<const __nv_bfloat16*>(q);
+  S.P = c.n_layers;
+  S.R = R;
+  S.Hq = c.n_q_heads;
+  S.Hkv = c.n_kv_heads;
+  S.q_agg = q_agg;
+  S.k_l = k_l;
+  S.cdesc = ix->cdesc;
+  S.n_clusters = ix->uc_count;
+  S.work = ix->uc_work;
+  S.ids = ids;
+  S.scores = scores;
+  S.count = count;
+  SS_CUDA(cudaSetDevice(ix->device));
+  SS_CUDA(launch_uc_select(S, ix->uc_cap, static_cast<cudaStream_t>(stream)));
   return SS_OK;
 }
 

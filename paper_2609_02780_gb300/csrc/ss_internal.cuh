@@ -134,6 +134,10 @@ struct Prob {
   float2* rm_scratch;          // row-averaged lists: per-row softmax statistics
   int rm_chunks;               // CTAs per slab of the row-averaged passes
   float* aval;                 // [P][cand_cap] head-averaged weight of every token
+  // an index with clustered units: the view above starts at its first detailed unit
+  int unit_offset;             // clustered units before it (0: none)
+  int32_t* votes_base;         // the caller's votes / mass arrays in stream numbering
+  float* mass_base;
   // launch mapping of the score kernel
   int cta_begin;               // first score CTA of this problem
   int chunks;                  // score CTAs per slab (they share the slab's units)
@@ -154,6 +158,38 @@ struct Batch {
   uint32_t wait_polls;         // limit of the score kernel's waits for its key copies
 };
 static_assert(sizeof(Batch) <= 32000, "kernel parameter block too large");
+
+// Online clustering of units leaving the detailed window (one call).
+struct UcJob {
+  const float* desc;           // [ucap][D]
+  const __nv_bfloat16* keys;   // [n_slabs][ncap][d]
+  int64_t ncap;
+  int n_slabs, Tu, D;
+  int u0, n;                   // the units leaving, in order
+  float tau;
+  int cap;                     // cluster capacity
+  int32_t* n_clusters;         // device count
+  float* cdesc;                // [cap][D] centroids
+  int32_t* ccount;             // [cap] members
+  float* creps;                // [cap][n_slabs][Tu][d] representative keys
+  int32_t* unit_cluster;       // [ucap]
+  int32_t* cfirst;             // [cap] first member unit in the current call
+  int32_t* cprev;              // [cap] members before the current call
+  int32_t* first_touched;      // device: the first cluster the call touched
+  uint32_t* status;            // device status word of the index
+};
+
+// Cluster evidence of a question (Eq. 13).
+struct UcSel {
+  const __nv_bfloat16* q;      // [P][R][Hq][d]
+  int P, R, Hq, Hkv, q_agg, k_l;
+  const float* cdesc;
+  const int32_t* n_clusters;
+  float* work;                 // [cap] scores
+  int32_t* ids;                // [k_l]
+  float* scores;               // [k_l]
+  int32_t* count;              // [1]
+};
 
 // ---------------------------------------------------------------------------
 // Device helpers
@@ -269,6 +305,9 @@ bool rowmean_supported(int R, int G);
 size_t rowmean_workspace_bytes(int n_slabs, int R, int G, int max_chunks);
 int rowmean_chunks(int n_slabs, int hist_tokens, int sm_count);
 cudaError_t launch_rowmean(const Batch& B, int pi, float2* scratch, int chunks, cudaStream_t s);
+cudaError_t launch_uc_shift(const Batch& B, cudaStream_t s);
+cudaError_t launch_uc_cluster(const UcJob& J, cudaStream_t s);
+cudaError_t launch_uc_select(const UcSel& S, int cap, cudaStream_t s);
 cudaError_t launch_shard_export(const Batch& B, int64_t tok_offset, float2* unit_stats,
                                 cudaStream_t s);
 cudaError_t launch_maxmin(const Batch& B, int max_pool, cudaStream_t s);
