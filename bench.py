@@ -561,13 +561,38 @@ def run_sweep(args):
             wc = torch.empty(idx.workspace_bytes(w.n_rows, pc), dtype=torch.uint8, device=dev)
             on = p50(lambda: idx.retrieve(q, k=pc.k, budget=pc.budget, use_clusters=1, out=rc,
                                           workspace=wc))
+        # LC-on with the paper's compression: units older than the latest 60 leave the
+        # detailed window into online clusters (tau 0.9); a question is answered by token
+        # voting over the detailed units plus the top-8 clusters (Eq. 13)
+        del idx, res, ws
+        torch.cuda.empty_cache()
+        on_units = None
+        if frames > 60:
+            ix2 = ss.Index(w.n_layers, w.n_q_heads, w.n_kv_heads, w.tokens_per_frame, frames,
+                           device=dev)
+            ix2.append(data["keys"])
+            n_leave = ix2.units_over_budget(0, 60)
+            ix2.cluster_units(n_leave, 0.9, max_clusters=min(frames, 16384))
+            r2 = ss.Result(ix2, p)
+            w2 = torch.empty(ix2.workspace_bytes(w.n_rows, p), dtype=torch.uint8, device=dev)
+
+            def both():
+                ix2.retrieve(q, k=p.k, budget=p.budget, out=r2, workspace=w2)
+                ix2.select_clusters(q, k_l=8)
+            on_units = p50(both)
+            n_clusters = int(ix2.unit_clusters()["sizes"].numel())
+            del ix2, r2, w2
+            torch.cuda.empty_cache()
         keys = w.keys_per_query
         print(json.dumps({"sweep": "query latency vs history", "frames": frames,
                           "hours": round(frames / 3600, 3), "keys": keys,
                           "index_bytes": w.key_bytes, "lc_off_ms": off,
                           "lc_off_keys_per_s": keys / (off / 1e3),
-                          "lc_on_ms": on, "lc_on_compressed_frames": n_comp}), flush=True)
-        del idx, data, res, ws
+                          "lc_on_ms": on, "lc_on_compressed_frames": n_comp,
+                          "lc_units_ms": on_units,
+                          "lc_units_clusters": n_clusters if on_units is not None else None}),
+              flush=True)
+        del data
         torch.cuda.empty_cache()
 
 
