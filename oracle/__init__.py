@@ -18,5 +18,8 @@ Plain, slow, fp64 numpy written from the paper's definitions:
   unit_clusters.py  the paper's long-history compression (Sec. 4.1, Eq. 5-7: units
                 leaving the detailed window clustered online, representative keys as
                 running averages) and the cluster evidence of Eq. 13
+  forward.py    the question's forward pass through the shallow layers (Eq. 10):
+                synthetic pre-norm GQA decoder layers whose attention reads the stored
+                keys and values, yielding the query states the retrieval scores
 """
-from . import retrieval, kmeans, shard, unit_clusters  # noqa: F401
+from . import retrieval, kmeans, shard, unit_clusters, forward  # noqa: F401
