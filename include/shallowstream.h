@@ -102,6 +102,9 @@ typedef struct {
   const float* cluster_centroids; /* device fp32 [capacity][Hkv * d] (unit norm) */
   const int32_t* cluster_sizes; /* device int32 [capacity] members */
   const float* cluster_keys;    /* device fp32 [capacity][P][Hkv][T_u][d] representative keys */
+  /* stored values (ss_index_append_values), read by the question's forward only */
+  const void* values;           /* device bf16 [P][Hkv][N_cap][d] or NULL */
+  int64_t n_value_frames;       /* frames whose values are stored */
 } ss_index_view;
 
 /* k-means compression of the frames [first_frame, first_frame + n_frames) in
@@ -214,6 +217,26 @@ typedef struct {
   int32_t* counts;           /* [4] n_pool, n_sel, n_exp, n_frames */
 } ss_merge_result;
 
+/* The question's forward through the shallow layers (ss_question_forward). */
+typedef struct {
+  int32_t intermediate;      /* I, the MLP width: a positive multiple of 128 */
+  float rms_eps;             /* RMSNorm epsilon, > 0 */
+  float rope_theta;          /* RoPE base theta, > 1 */
+  int64_t pos0;              /* position of question row 0; < 0: the stored token count
+                                (the question follows the retained history) */
+} ss_forward_params;
+
+/* One shallow layer's weights: device bf16, row-major, 16-byte aligned. D = Hq * d. */
+typedef struct {
+  const void* ln1;           /* [D] RMSNorm weight before attention */
+  const void* wqkv;          /* [(Hq + 2 Hkv) d][D]: q rows (head-major), k rows, v rows */
+  const void* bqkv;          /* [(Hq + 2 Hkv) d] projection bias, or NULL for none */
+  const void* wo;            /* [D][Hq d] output projection */
+  const void* ln2;           /* [D] RMSNorm weight before the MLP */
+  const void* wgu;           /* [2 I][D]: gate rows, then up rows */
+  const void* wd;            /* [D][I] down projection */
+} ss_layer_weights;
+
 /* Optional instrumentation: cudaEvent_t handles recorded on the call's stream
  * immediately before and after the key-scoring kernel. NULL members are skipped. */
 typedef struct {
@@ -258,6 +281,45 @@ ss_status ss_index_append(ss_index* index, const void* keys, int32_t n_frames,
 
 /* Fills *view with the index's current state. Device arrays are owned by the index. */
 ss_status ss_index_get_view(const ss_index* index, ss_index_view* view);
+
+/* Stores the values that the shallow layers produced for the next n_frames frames
+ * whose keys are already stored (the layer-i KV cache C^i_T of Eq. 10 holds keys and
+ * values; only the question's forward reads the values). `values` is device bf16
+ * [P][Hkv][slab_stride_tokens][d], the key layout of ss_index_append (stride 0 =
+ * n_frames * T_f). The first call allocates [P][Hkv][N_cap][d] from the index's
+ * allocator. Errors: INVALID_ARG, STATE (values past the stored keys), ALLOC, CUDA. */
+ss_status ss_index_append_values(ss_index* index, const void* values, int32_t n_frames,
+                                 int64_t slab_stride_tokens, void* stream);
+
+/* Bytes of device workspace ss_question_forward needs for this index, row count and
+ * parameters (depends on the stored token count through the attention's chunking: take
+ * it again after appends). Errors as ss_question_forward's argument checks. */
+ss_status ss_forward_workspace_size(const ss_index* index, int32_t n_rows,
+                                    const ss_forward_params* params, size_t* bytes);
+
+/* The question's forward through the shallow layers (Sec. 4.2, Eq. 10): the question's
+ * R embedded rows `h_in` (device bf16 [R][D], D = Hq * d) pass through layers [0, P),
+ * each a pre-norm GQA decoder layer with the caller's weights `layers` [P]:
+ *   x = bf16(RMSNorm(H) * ln1);  [q; k; v] = x Wqkv^T + bqkv
+ *   q, k = bf16(RoPE(q, k)) at positions pos0 + r (rotate-half pairs (j, j + d/2),
+ *          angle pos * theta^(-2j/d), computed in fp64), v = bf16(v)
+ *   o = softmax(q k^T / sqrt(d)) v over the layer's stored tokens (their keys and values
+ *       as stored) and the question's rows 0..r, query head h reading key head h / G
+ *   H += bf16(o) Wo^T;  x2 = bf16(RMSNorm(H) * ln2);  H += bf16(silu(x2 Wg^T) * (x2 Wu^T)) Wd^T
+ * Outputs: q_out (device bf16 [P][R][Hq][d]) = each layer's post-RoPE query rows Q^i,
+ * the retrieval's input layout (ss_retrieve's q); h_out (device fp32 [R][D], or NULL) =
+ * the hidden states after layer P - 1. H is carried in fp32; products run on the tensor
+ * cores in bf16 with fp32 accumulation; attention weights are rounded to bf16 for the
+ * tensor cores and normalised by the sum of the rounded weights. `status` (device word,
+ * or NULL for one in the workspace) records SS_ERR_TIMEOUT as in ss_status_sync.
+ * Needs R <= 64, (Hq / Hkv) * (R rounded up to 16) <= 256, values stored for every
+ * stored frame, and an index without compressed windows or clusters.
+ * Errors: INVALID_ARG (NULL, misaligned, bad parameters), UNSUPPORTED, STATE (values
+ * missing, compressed index), CAPACITY (workspace too small), CUDA. */
+ss_status ss_question_forward(ss_index* index, const ss_layer_weights* layers,
+                              const ss_forward_params* params, const void* h_in,
+                              int32_t n_rows, void* q_out, float* h_out, uint32_t* status,
+                              void* workspace, size_t workspace_bytes, void* stream);
 
 /* k-means compression of already appended frames (the cluster-compressed variant;
  * closest paper text Sec. 4.1 Eq. 5-7). For every window of `window_frames` frames in

@@ -80,34 +80,43 @@ def silu(x: np.ndarray) -> np.ndarray:
 
 
 def attention(q: np.ndarray, hist_k: np.ndarray, hist_v: np.ndarray,
-              own_k: np.ndarray, own_v: np.ndarray) -> np.ndarray:
+              own_k: np.ndarray, own_v: np.ndarray, spread: bool = False):
     """q [R][Hq][d]; hist_k, hist_v [Hkv][N][d] (the layer's stored tokens); own_k, own_v
     [R][Hkv][d] (the question's rows). Row r of head h attends to the N stored tokens of
-    key head h // G and to the question's rows 0..r. Returns o [R][Hq][d] (fp64)."""
+    key head h // G and to the question's rows 0..r. Returns o [R][Hq][d] (fp64); with
+    spread=True also sum_j p_j |v_j - o| per element (how far a change of the weights by a
+    relative e can move o: at most e times this)."""
     R, Hq, d = q.shape
     Hkv = hist_k.shape[0]
     G = Hq // Hkv
     out = np.zeros((R, Hq, d), dtype=np.float64)
+    spr = np.zeros((R, Hq, d), dtype=np.float64) if spread else None
     scale = 1.0 / np.sqrt(d)
+    causal = np.tril(np.ones((R, R), dtype=bool))                           # row r sees 0..r
     for h in range(Hq):
         g = h // G
-        for r in range(R):
-            keys = np.concatenate([hist_k[g], own_k[:r + 1, g]], axis=0)     # [N + r + 1][d]
-            vals = np.concatenate([hist_v[g], own_v[:r + 1, g]], axis=0)
-            s = keys @ q[r, h] * scale
-            p = np.exp(s - s.max())
-            p /= p.sum()
-            out[r, h] = p @ vals
-    return out
+        keys = np.concatenate([hist_k[g], own_k[:, g]], axis=0)              # [N + R][d]
+        vals = np.concatenate([hist_v[g], own_v[:, g]], axis=0)
+        s = q[:, h] @ keys.T * scale                                         # [R][N + R]
+        s[:, hist_k.shape[1]:][~causal] = -np.inf
+        p = np.exp(s - s.max(axis=1, keepdims=True))
+        p /= p.sum(axis=1, keepdims=True)
+        out[:, h] = p @ vals
+        if spread:
+            for r in range(R):
+                spr[r, h] = p[r] @ np.abs(vals - out[r, h][None, :])
+    return (out, spr) if spread else out
 
 
 def layer(h: np.ndarray, w: dict, hist_k_bits: np.ndarray, hist_v_bits: np.ndarray,
-          *, n_q_heads: int, n_kv_heads: int, pos0: int, eps: float, theta: float) -> dict:
+          *, n_q_heads: int, n_kv_heads: int, pos0: int, eps: float, theta: float,
+          with_spread: bool = False) -> dict:
     """One shallow layer F^i (Eq. 10). h [R][D] (fp64 hidden states). w: bf16 bit arrays
     ln1 [D], wqkv [(Hq + 2 Hkv) d][D], bqkv [(Hq + 2 Hkv) d] or None, wo [D][Hq d],
     ln2 [D], wgu [2 I][D] (gate rows, then up rows), wd [D][I]. hist_k_bits,
     hist_v_bits: the layer's stored keys and values, bf16 bits [Hkv][N][d].
-    Returns {"h": H^{i+1} fp64, "q_bits": Q^i bf16 bits [R][Hq][d], "k", "v", "o", "a"}."""
+    Returns {"h": H^{i+1} fp64, "q_bits": Q^i bf16 bits [R][Hq][d], and the intermediate
+    values (q, k, v, o, a and their values before rounding)}."""
     h = np.asarray(h, dtype=np.float64)
     R, D = h.shape
     Hq, Hkv = n_q_heads, n_kv_heads
@@ -121,11 +130,14 @@ def layer(h: np.ndarray, w: dict, hist_k_bits: np.ndarray, hist_v_bits: np.ndarr
     yq = y[:, :Hq * d].reshape(R, Hq, d)
     yk = y[:, Hq * d:(Hq + Hkv) * d].reshape(R, Hkv, d)
     yv = y[:, (Hq + Hkv) * d:].reshape(R, Hkv, d)
-    q = bf16_round(rope(yq, pos, theta))
+    q_pre = rope(yq, pos, theta)
+    q = bf16_round(q_pre)
     k = bf16_round(rope(yk, pos, theta))
     v = bf16_round(yv)
-    o = attention(q, bf16_to_f64(hist_k_bits), bf16_to_f64(hist_v_bits), k, v)
-    o = bf16_round(o.reshape(R, Hq * d))
+    att = attention(q, bf16_to_f64(hist_k_bits), bf16_to_f64(hist_v_bits), k, v,
+                    spread=with_spread)
+    o_pre, o_spread = att if with_spread else (att, None)
+    o = bf16_round(o_pre.reshape(R, Hq * d))
     h1 = h + o @ f("wo").T
     x2 = bf16_round(rms_norm(h1, f("ln2"), eps))
     wgu = f("wgu")
@@ -135,7 +147,9 @@ def layer(h: np.ndarray, w: dict, hist_k_bits: np.ndarray, hist_v_bits: np.ndarr
     a = bf16_round(silu(g) * u)
     h2 = h1 + a @ f("wd").T
     return {"h": h2, "h_mid": h1, "q_bits": f32_to_bf16_rne(q.astype(np.float32)),
-            "q": q, "k": k, "v": v, "o": o, "x": x, "x2": x2, "a": a}
+            "q": q, "q_pre": q_pre, "k": k, "v": v, "o": o, "o_pre": o_pre.reshape(R, Hq * d),
+            "o_spread": None if o_spread is None else o_spread.reshape(R, Hq * d),
+            "x": x, "x2": x2, "a": a, "a_pre": silu(g) * u}
 
 
 def forward(h_in_bits: np.ndarray, layers: list, key_bits: np.ndarray, value_bits: np.ndarray,

@@ -121,6 +121,19 @@ class Result:
         return self.host()["frames"]
 
 
+@dataclass
+class ForwardParams:
+    """ss_forward_params: MLP width, RMSNorm epsilon, RoPE base, position of row 0
+    (< 0: the stored token count)."""
+    intermediate: int
+    rms_eps: float = 1e-6
+    rope_theta: float = 1e6
+    pos0: int = -1
+
+    def abi(self) -> _abi.ForwardParams:
+        return _abi.ForwardParams(self.intermediate, self.rms_eps, self.rope_theta, self.pos0)
+
+
 class Index:
     """A shallow key index (Eq. 2) of one video stream, resident on one GPU."""
 
@@ -299,6 +312,95 @@ class Index:
                                           int(n_frames), int(S),
                                           C.c_void_p(_stream_ptr(self.device))))
         self._last_src = keys  # keep the source alive until the stream passes the copy
+
+    def append_values(self, values: torch.Tensor, n_frames: int | None = None) -> None:
+        """Stores the values bf16 [P][Hkv][S][128] of the next frames whose keys are
+        stored (ss_index_append_values; the question's forward reads them)."""
+        if values.dtype != torch.bfloat16 or values.dim() != 4 or values.device != self.device:
+            raise ValueError("values must be bf16 [P][Hkv][S][128] on the index's device")
+        if (values.stride(3) != 1 or values.stride(2) != 128 or
+                values.stride(0) != values.shape[1] * values.stride(1)):
+            raise ValueError("values must be row-major per slab")
+        S = values.stride(1) // 128
+        if n_frames is None:
+            if values.shape[2] % self.tokens_per_frame:
+                raise ValueError("token count is not a whole number of frames")
+            n_frames = values.shape[2] // self.tokens_per_frame
+        with torch.cuda.device(self.device):
+            _check(_lib().ss_index_append_values(self.handle, C.c_void_p(values.data_ptr()),
+                                                 int(n_frames), int(S),
+                                                 C.c_void_p(_stream_ptr(self.device))))
+        self._last_vsrc = values
+
+    def values(self) -> torch.Tensor:
+        """Device bf16 [P][Hkv][capacity][128] value slabs, a view."""
+        v = self.view()
+        if not v.values:
+            raise ValueError("the index stores no values")
+        return self._block_view(v.values, torch.bfloat16,
+                                (self.n_layers, self.n_kv_heads, v.token_capacity, 128))
+
+    def forward_workspace_bytes(self, n_rows: int, params: "ForwardParams") -> int:
+        n = C.c_size_t()
+        fp = params.abi()
+        _check(_lib().ss_forward_workspace_size(self.handle, int(n_rows), C.byref(fp),
+                                                C.byref(n)))
+        return n.value
+
+    def forward(self, layers: list[dict], h_in: torch.Tensor, params: "ForwardParams", *,
+                q_out: torch.Tensor | None = None, h_out: torch.Tensor | None = None,
+                status: torch.Tensor | None = None,
+                workspace: torch.Tensor | None = None) -> tuple[torch.Tensor, torch.Tensor]:
+        """ss_question_forward (Sec. 4.2, Eq. 10): the question's rows h_in bf16 [R][D]
+        through the P shallow layers (weights: one dict per layer of bf16 device tensors
+        ln1, wqkv, bqkv (or None), wo, ln2, wgu, wd). Returns (q bf16 [P][R][Hq][128], the
+        retrieval's input, and H fp32 [R][D]). Asynchronous on the current stream."""
+        if len(layers) != self.n_layers:
+            raise ValueError("one weight dict per shallow layer")
+        D = self.n_q_heads * 128
+        if (h_in.dtype != torch.bfloat16 or h_in.dim() != 2 or h_in.shape[1] != D or
+                not h_in.is_contiguous() or h_in.device != self.device):
+            raise ValueError("h_in must be contiguous bf16 [R][Hq * 128] on the index's device")
+        R = h_in.shape[0]
+        if q_out is None:
+            q_out = torch.empty(self.n_layers, R, self.n_q_heads, 128, dtype=torch.bfloat16,
+                                device=self.device)
+        if h_out is None:
+            h_out = torch.empty(R, D, dtype=torch.float32, device=self.device)
+        W = (_abi.LayerWeights * self.n_layers)()
+        keep = []
+        for i, w in enumerate(layers):
+            ptrs = []
+            for name in ("ln1", "wqkv", "bqkv", "wo", "ln2", "wgu", "wd"):
+                t = w.get(name)
+                if t is None:
+                    if name != "bqkv":
+                        raise ValueError(f"layer {i}: {name} missing")
+                    ptrs.append(None)
+                    continue
+                if (t.dtype != torch.bfloat16 or not t.is_contiguous() or t.device != self.device):
+                    raise ValueError(f"layer {i}: {name} must be contiguous bf16 on the device")
+                keep.append(t)
+                ptrs.append(t.data_ptr())
+            W[i] = _abi.LayerWeights(*ptrs)
+        nbytes = self.forward_workspace_bytes(R, params)
+        ws = workspace if workspace is not None else self._fw_workspace(nbytes)
+        fp = params.abi()
+        with torch.cuda.device(self.device):
+            _check(_lib().ss_question_forward(
+                self.handle, W, C.byref(fp), C.c_void_p(h_in.data_ptr()), R,
+                C.c_void_p(q_out.data_ptr()), C.c_void_p(h_out.data_ptr()),
+                C.c_void_p(status.data_ptr() if status is not None else None),
+                C.c_void_p(ws.data_ptr()), ws.numel(), C.c_void_p(_stream_ptr(self.device))))
+        self._fw_keep = keep
+        return q_out, h_out
+
+    def _fw_workspace(self, nbytes: int) -> torch.Tensor:
+        ws = getattr(self, "_fws", None)
+        if ws is None or ws.numel() < nbytes:
+            ws = torch.empty(nbytes, dtype=torch.uint8, device=self.device)
+            self._fws = ws
+        return ws
 
     def compress(self, window_frames: int, n_centroids: int = 64, iters: int = 5,
                  first_frame: int = 0, n_frames: int | None = None) -> None:

@@ -32,7 +32,8 @@ class IndexView(C.Structure):
                 ("member_sizes", C.c_void_p), ("n_clustered_units", C.c_int64),
                 ("cluster_capacity", C.c_int32), ("unit_cluster", C.c_void_p),
                 ("cluster_count", C.c_void_p), ("cluster_centroids", C.c_void_p),
-                ("cluster_sizes", C.c_void_p), ("cluster_keys", C.c_void_p)]
+                ("cluster_sizes", C.c_void_p), ("cluster_keys", C.c_void_p),
+                ("values", C.c_void_p), ("n_value_frames", C.c_int64)]
 
 
 class CompressParams(C.Structure):
@@ -74,6 +75,16 @@ class MergeResult(C.Structure):
                 ("unit_votes", C.c_void_p), ("unit_mass", C.c_void_p), ("pool", C.c_void_p),
                 ("sel_units", C.c_void_p), ("exp_units", C.c_void_p), ("frames", C.c_void_p),
                 ("counts", C.c_void_p)]
+
+
+class ForwardParams(C.Structure):
+    _fields_ = [("intermediate", C.c_int32), ("rms_eps", C.c_float), ("rope_theta", C.c_float),
+                ("pos0", C.c_int64)]
+
+
+class LayerWeights(C.Structure):
+    _fields_ = [("ln1", C.c_void_p), ("wqkv", C.c_void_p), ("bqkv", C.c_void_p),
+                ("wo", C.c_void_p), ("ln2", C.c_void_p), ("wgu", C.c_void_p), ("wd", C.c_void_p)]
 
 
 class Trace(C.Structure):
@@ -119,6 +130,14 @@ SIGNATURES = {
                                               C.POINTER(C.c_int64)]),
     "ss_select_clusters": (c_status, [C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_int32,
                                       C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
+    "ss_index_append_values": (c_status, [C.c_void_p, C.c_void_p, C.c_int32, C.c_int64,
+                                          C.c_void_p]),
+    "ss_forward_workspace_size": (c_status, [C.c_void_p, C.c_int32, C.POINTER(ForwardParams),
+                                             C.POINTER(C.c_size_t)]),
+    "ss_question_forward": (c_status, [C.c_void_p, C.POINTER(LayerWeights),
+                                       C.POINTER(ForwardParams), C.c_void_p, C.c_int32,
+                                       C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                                       C.c_size_t, C.c_void_p]),
     "ss_merge_shards": (c_status, [C.POINTER(Shard), C.c_int32, C.c_int32, C.c_int32,
                                    C.c_int32, C.c_int32, C.POINTER(RetrieveParams),
                                    C.POINTER(MergeResult)]),

@@ -52,6 +52,9 @@ struct ss_index {
   int32_t* cprev;
   int32_t* uc_count;    // device: [0] clusters, [1] first cluster the last call touched
   float* uc_work;
+  // stored values (the question's forward attends over keys and values)
+  __nv_bfloat16* vals;  // [P*Hkv][ncap][d], allocated by the first value append
+  int64_t n_vframes;    // frames whose values are stored
 };
 
 namespace {
@@ -533,6 +536,7 @@ SS_EXPORT ss_status ss_index_destroy(ss_index* ix) {
   dev_free(ix, ix->cprev);
   dev_free(ix, ix->uc_count);
   dev_free(ix, ix->uc_work);
+  dev_free(ix, ix->vals);
   delete ix;
   return SS_OK;
 }
@@ -587,6 +591,125 @@ SS_EXPORT ss_status ss_index_get_view(const ss_index* ix, ss_index_view* v) {
   v->cluster_centroids = ix->cdesc;
   v->cluster_sizes = ix->ccount;
   v->cluster_keys = ix->creps;
+  v->values = ix->vals;
+  v->n_value_frames = ix->n_vframes;
+  return SS_OK;
+}
+
+SS_EXPORT ss_status ss_index_append_values(ss_index* ix, const void* values, int32_t n_frames,
+                                           int64_t stride, void* stream) {
+  if (!ix) return fail(SS_ERR_INVALID_ARG, "index is NULL");
+  if (n_frames < 0) return fail(SS_ERR_INVALID_ARG, "n_frames must be >= 0");
+  if (n_frames == 0) return SS_OK;
+  if (!values) return fail(SS_ERR_INVALID_ARG, "values is NULL");
+  if ((uintptr_t)values & 15u) return fail(SS_ERR_INVALID_ARG, "values must be 16-byte aligned");
+  const ss_index_config& c = ix->cfg;
+  const int64_t n_tok = (int64_t)n_frames * c.tokens_per_frame;
+  if (stride == 0) stride = n_tok;
+  if (stride < n_tok) return fail(SS_ERR_INVALID_ARG, "slab_stride_tokens < n_frames * tokens_per_frame");
+  if (ix->n_vframes + n_frames > ix->n_frames)
+    return fail(SS_ERR_STATE, "values of %d frames would pass the %lld frames whose keys are stored",
+                n_frames, (long long)ix->n_frames);
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  SS_CUDA(cudaSetDevice(ix->device));
+  if (!ix->vals) {
+    const size_t vb = (size_t)c.n_layers * c.n_kv_heads * ix->ncap * kHeadDim * 2;
+    ix->vals = static_cast<__nv_bfloat16*>(dev_alloc(ix, vb, st));
+    if (!ix->vals || ((uintptr_t)ix->vals & 15u)) {
+      dev_free(ix, ix->vals);
+      ix->vals = nullptr;
+      return fail(SS_ERR_ALLOC, "device allocation of %zu bytes for the values failed", vb);
+    }
+  }
+  SS_CUDA(launch_append(ix->vals, ix->ncap, ix->n_vframes * c.tokens_per_frame,
+                        static_cast<const __nv_bfloat16*>(values), stride,
+                        c.n_layers * c.n_kv_heads, n_tok, st));
+  ix->n_vframes += n_frames;
+  return SS_OK;
+}
+
+namespace {
+ss_status forward_shape(const ss_index* ix, int32_t R, const ss_forward_params* fp, FwShape* F) {
+  if (!ix || !fp) return fail(SS_ERR_INVALID_ARG, "NULL argument");
+  const ss_index_config& c = ix->cfg;
+  if (R < 1) return fail(SS_ERR_INVALID_ARG, "n_rows must be >= 1");
+  if (!forward_supported(R, c.n_q_heads, c.n_kv_heads))
+    return fail(SS_ERR_UNSUPPORTED,
+                "the forward needs R <= 64 and (Hq / Hkv) * (R rounded up to 16) <= 256");
+  if (fp->intermediate < 128 || fp->intermediate % 128)
+    return fail(SS_ERR_INVALID_ARG, "intermediate must be a positive multiple of 128");
+  if (!(fp->rms_eps > 0.f) || !(fp->rope_theta > 1.f))
+    return fail(SS_ERR_INVALID_ARG, "rms_eps must be > 0 and rope_theta > 1");
+  if ((int64_t)c.n_q_heads * kHeadDim > 16384)
+    return fail(SS_ERR_UNSUPPORTED, "hidden size above 16384");
+  F->P = c.n_layers;
+  F->Hq = c.n_q_heads;
+  F->Hkv = c.n_kv_heads;
+  F->R = R;
+  F->I = fp->intermediate;
+  F->ncap = ix->ncap;
+  F->n_tok = (int)(ix->n_frames * c.tokens_per_frame);
+  F->sm_count = ix->sm_count;
+  F->eps = fp->rms_eps;
+  F->theta = (double)fp->rope_theta;
+  F->pos0 = fp->pos0 < 0 ? (int64_t)F->n_tok : fp->pos0;
+  F->keys = ix->keys;
+  F->values = ix->vals;
+  return SS_OK;
+}
+}  // namespace
+
+SS_EXPORT ss_status ss_forward_workspace_size(const ss_index* ix, int32_t n_rows,
+                                              const ss_forward_params* fp, size_t* bytes) {
+  if (!bytes) return fail(SS_ERR_INVALID_ARG, "bytes is NULL");
+  FwShape F{};
+  const ss_status s = forward_shape(ix, n_rows, fp, &F);
+  if (s != SS_OK) return s;
+  *bytes = forward_workspace_bytes(F);
+  return SS_OK;
+}
+
+SS_EXPORT ss_status ss_question_forward(ss_index* ix, const ss_layer_weights* layers,
+                                        const ss_forward_params* fp, const void* h_in,
+                                        int32_t n_rows, void* q_out, float* h_out,
+                                        uint32_t* status, void* workspace,
+                                        size_t workspace_bytes, void* stream) {
+  FwShape F{};
+  ss_status s = forward_shape(ix, n_rows, fp, &F);
+  if (s != SS_OK) return s;
+  if (!layers || !h_in || !q_out || !workspace)
+    return fail(SS_ERR_INVALID_ARG, "NULL argument");
+  if (ix->n_clustered > 0 || ix->n_windows > 0)
+    return fail(SS_ERR_UNSUPPORTED, "the forward reads an uncompressed index only");
+  if (ix->n_vframes != ix->n_frames)
+    return fail(SS_ERR_STATE, "values are stored for %lld of %lld frames",
+                (long long)ix->n_vframes, (long long)ix->n_frames);
+  if (F.n_tok > 0 && !ix->vals) return fail(SS_ERR_STATE, "the index stores no values");
+  const size_t need = forward_workspace_bytes(F);
+  if (workspace_bytes < need)
+    return fail(SS_ERR_CAPACITY, "workspace of %zu bytes < %zu needed", workspace_bytes, need);
+  auto al16 = [](const void* p) { return ((uintptr_t)p & 15u) == 0u; };
+  if (((uintptr_t)workspace & 255u) || !al16(h_in) || !al16(q_out) || (h_out && !al16(h_out)) ||
+      (status && ((uintptr_t)status & 3u)))
+    return fail(SS_ERR_INVALID_ARG, "workspace must be 256-byte aligned, h_in, q_out and h_out 16-byte aligned");
+  std::vector<FwLayerW> W(F.P);
+  for (int i = 0; i < F.P; ++i) {
+    const ss_layer_weights& w = layers[i];
+    if (!w.ln1 || !w.wqkv || !w.wo || !w.ln2 || !w.wgu || !w.wd)
+      return fail(SS_ERR_INVALID_ARG, "layer %d: a weight pointer is NULL (only bqkv may be)", i);
+    for (const void* p : {w.ln1, w.wqkv, w.bqkv, w.wo, w.ln2, w.wgu, w.wd})
+      if (p && !al16(p)) return fail(SS_ERR_INVALID_ARG, "layer %d: weights must be 16-byte aligned", i);
+    W[i] = FwLayerW{w.ln1, w.wqkv, w.bqkv, w.wo, w.ln2, w.wgu, w.wd};
+  }
+  FwArgs A;
+  A.layers = W.data();
+  A.h_in = h_in;
+  A.q_out = q_out;
+  A.h_out = h_out;
+  A.status = status;
+  A.workspace = workspace;
+  SS_CUDA(cudaSetDevice(ix->device));
+  SS_CUDA(launch_forward(F, A, static_cast<cudaStream_t>(stream)));
   return SS_OK;
 }
 

@@ -1,0 +1,855 @@
+// The question's forward through the shallow layers (Sec. 4.2, Eq. 10).
+//
+// Eq. 10 appends the question to the retained shallow history and runs it through layers
+// [0, P); layer i's attention reads the layer's stored keys and values, and the layer
+// yields the question's query states Q^i, which the retrieval scores (Eq. 11). The
+// backbone is synthetic: pre-norm GQA decoder layers (RMSNorm, q/k/v projections with
+// bias, rotate-half RoPE, attention, output projection, SwiGLU MLP, residual adds).
+// Rounding points: the operands of every matrix product and the outputs q, k, v are
+// bf16 (nearest-even); the hidden states H stay fp32.
+//
+// Kernels per layer (R question rows, Rp = R rounded up to 16):
+//   k_fw_norm     H (+)= the split-K partial sums of the previous product (fixed order),
+//                 then X = bf16(RMSNorm(H) * w)
+//   k_fw_gemm     partial[split] = X W^T on the tcgen05 tensor cores: 128 output features
+//                 of W on the TMEM lanes (A operand), the Rp rows as N, K split over CTAs;
+//                 W and X tiles by TMA (128-byte swizzle) through a ring of stages
+//   k_fw_qkv      q, k, v from the partials (+ bias), RoPE on q and k with exact (fp64)
+//                 angles; q goes to the caller's Q^i
+//   k_fw_attn     the question rows of one key head against a chunk of the layer's
+//                 stored tokens: S = Q K^T (rows on the TMEM lanes), P = 2^(s - m) in bf16,
+//                 O += P V on the tensor cores, with the running max raised lazily (only
+//                 when a tile's max exceeds it by 8, scaling O and l then); per chunk the
+//                 unnormalised (m, l, O)
+//   k_fw_attn_out the chunks and the question's own rows (causal) merged per (row, head)
+//                 in a fixed order, o = bf16(O / L)
+//   k_fw_swiglu   a = bf16(silu(g) * u) from the gate and up partials
+#include "ss_internal.cuh"
+#include "ss_device.cuh"
+#include "ss_tc.cuh"
+
+#include <algorithm>
+
+namespace ss {
+
+// Bounded wait that gives up when another role of the CTA raised the abort flag; a wait
+// that runs out raises it.
+__device__ __forceinline__ bool fw_wait(uint32_t bar, uint32_t parity, volatile int* abort) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (uint32_t i = 1; i < kDefaultWaitPolls; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 255u) == 0u) {
+      if (*abort) return false;
+      if (global_ns() - t0 > 1000000000ull) break;
+    }
+  }
+  *abort = 1;
+  return false;
+}
+
+__device__ __forceinline__ void fw_bar(int id, int nthreads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+// ===========================================================================
+// Skinny GEMM: part[split][r][n] = sum over the split's K range of X[r][k] W[n][k].
+// ===========================================================================
+constexpr int kGmThreads = 192;           // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
+constexpr int kGmMaxStages = 8;
+constexpr int kGmABytes = 128 * 128;      // 128 rows of W x 64 bf16
+
+struct GemmJob {
+  float* part;       // [splits][Rp][n_out]
+  int n_out;
+  int R, Rp;
+  int kblocks;       // K / 64
+  int splits;
+  int stages;
+  uint32_t* status;
+};
+
+struct GmBars {
+  unsigned long long full[kGmMaxStages], empty[kGmMaxStages], d_full;
+  uint32_t taddr;
+  int abort;
+};
+
+__global__ void __launch_bounds__(kGmThreads, 1)
+    k_fw_gemm(const __grid_constant__ CUtensorMap wmap, const __grid_constant__ CUtensorMap xmap,
+              const GemmJob J) {
+  extern __shared__ unsigned char sm_raw[];
+  __shared__ GmBars S;
+  unsigned char* sm = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  const int stages = J.stages;
+  const int b_bytes = J.Rp * 128;
+  const int stage_bytes = kGmABytes + b_bytes;   // a multiple of 1024 (Rp % 16 == 0)
+  const int m0 = blockIdx.x * 128, split = blockIdx.y;
+  const int kb0 = (int)((int64_t)J.kblocks * split / J.splits);
+  const int kb1 = (int)((int64_t)J.kblocks * (split + 1) / J.splits);
+  const int n = kb1 - kb0;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  volatile int* abort = &S.abort;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < stages; ++s) {
+      mbar_init(smem_u32(&S.full[s]), 1);
+      mbar_init(smem_u32(&S.empty[s]), 1);
+    }
+    mbar_init(smem_u32(&S.d_full), 1);
+    S.abort = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&S.taddr), 64);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tbase = S.taddr;
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_map(&wmap);
+    tma_prefetch_map(&xmap);
+    int issued_last[kGmMaxStages];
+    for (int s = 0; s < kGmMaxStages; ++s) issued_last[s] = -1;
+    for (int j = 0; j < n && !*abort; ++j) {
+      const int st = j % stages;
+      if (j >= stages && !fw_wait(smem_u32(&S.empty[st]), ((j / stages) - 1) & 1, abort)) break;
+      const uint32_t bar = smem_u32(&S.full[st]);
+      const uint32_t dst = smem_u32(sm + st * stage_bytes);
+      mbar_expect_tx(bar, (uint32_t)stage_bytes);
+      tma_load_2d(dst, &wmap, bar, (kb0 + j) * 64, m0);
+      tma_load_2d(dst + kGmABytes, &xmap, bar, (kb0 + j) * 64, 0);
+      issued_last[st] = j;
+    }
+    // the copies in flight land before the CTA ends
+    for (int s = 0; s < stages; ++s)
+      if (issued_last[s] >= 0) mbar_wait_bounded(smem_u32(&S.full[s]), (issued_last[s] / stages) & 1);
+  } else if (warp == 1 && lane == 0) {
+    const uint32_t id = idesc_bf16_f32(128, J.Rp, false, false);
+    for (int j = 0; j < n; ++j) {
+      const int st = j % stages;
+      if (!fw_wait(smem_u32(&S.full[st]), (j / stages) & 1, abort)) break;
+      tc_fence_after();
+      const uint32_t a = smem_u32(sm + st * stage_bytes);
+      const uint32_t b = a + kGmABytes;
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+        umma_bf16(tbase, sdesc_sw128(a + k * 32, 16, 1024), sdesc_sw128(b + k * 32, 16, 1024), id,
+                  (j > 0 || k > 0) ? 1u : 0u);
+      umma_commit(smem_u32(&S.empty[st]));
+    }
+    umma_commit(smem_u32(&S.d_full));
+    mbar_wait_bounded(smem_u32(&S.d_full), 0);
+  } else if (warp >= 2) {
+    const int qd = warp & 3;                       // TMEM lane quarter of this warp
+    const int f = m0 + qd * 32 + lane;             // this thread's output feature
+    bool ok = fw_wait(smem_u32(&S.d_full), 0, abort) && n > 0;
+    ok = __all_sync(0xffffffffu, ok) && !*abort;
+    tc_fence_after();
+    if (ok) {
+      const uint32_t la = tbase + ((uint32_t)(qd * 32) << 16);
+      float* out = J.part + (int64_t)split * J.Rp * J.n_out + f;
+      for (int c0 = 0; c0 < J.Rp; c0 += 16) {
+        float v[16];
+        tmem_ld16(la + (uint32_t)c0, v);
+#pragma unroll
+        for (int c = 0; c < 16; ++c)
+          if (c0 + c < J.R) out[(int64_t)(c0 + c) * J.n_out] = v[c];
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (threadIdx.x == 0 && S.abort) atomicOr(J.status, kStatusTimeout);
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tbase, 64);
+}
+
+// ===========================================================================
+// Element-wise steps
+// ===========================================================================
+struct NormJob {
+  float* H;                    // [R][D]
+  const __nv_bfloat16* h_in;   // [R][D] or NULL: H = h_in instead of H += partials
+  const float* part;           // [splits][Rp][D] or NULL
+  int splits;
+  const __nv_bfloat16* w;      // [D] or NULL: no normalisation
+  __nv_bfloat16* X;            // [Rp][D] (rows >= R zero)
+  int D, R, Rp;
+  float eps;
+};
+
+// One CTA per row of Rp: the residual add in split order, then RMSNorm with the sum of
+// squares reduced in a fixed order.
+__global__ void __launch_bounds__(256) k_fw_norm(const NormJob J) {
+  __shared__ float red[8];
+  const int r = blockIdx.x, t = threadIdx.x;
+  const int D = J.D;
+  if (r >= J.R) {
+    if (J.w)
+      for (int x = t; x < D; x += 256) J.X[(int64_t)r * D + x] = __float2bfloat16_rn(0.f);
+    return;
+  }
+  float ss = 0.f;
+  for (int x = t; x < D; x += 256) {
+    float h = J.h_in ? __bfloat162float(J.h_in[(int64_t)r * D + x]) : J.H[(int64_t)r * D + x];
+    if (J.part)
+      for (int s = 0; s < J.splits; ++s) h += J.part[((int64_t)s * J.Rp + r) * D + x];
+    J.H[(int64_t)r * D + x] = h;
+    ss = fmaf(h, h, ss);
+  }
+  if (!J.w) return;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  if ((t & 31) == 0) red[t >> 5] = ss;
+  __syncthreads();
+  float tot = 0.f;
+#pragma unroll
+  for (int w = 0; w < 8; ++w) tot += red[w];
+  const float inv = 1.0f / sqrtf(tot / (float)D + J.eps);
+  for (int x = t; x < D; x += 256)
+    J.X[(int64_t)r * D + x] =
+        __float2bfloat16_rn(J.H[(int64_t)r * D + x] * inv * __bfloat162float(J.w[x]));
+}
+
+struct QkvJob {
+  const float* part;           // [splits][Rp][(Hq + 2 Hkv) d]
+  int splits, Rp, R;
+  const __nv_bfloat16* bias;   // [(Hq + 2 Hkv) d] or NULL
+  int Hq, Hkv;
+  int64_t pos0;
+  double theta;
+  __nv_bfloat16* q;            // [R][Hq][d] (the caller's Q^i)
+  __nv_bfloat16* k;            // [R][Hkv][d]
+  __nv_bfloat16* v;            // [R][Hkv][d]
+};
+
+// Grid (R, Hq + 2 Hkv); thread j < 64 owns the pair (j, j + 64) of one head.
+__global__ void __launch_bounds__(64) k_fw_qkv(const QkvJob J) {
+  const int r = blockIdx.x, t = blockIdx.y, j = threadIdx.x;
+  const int n_out = (J.Hq + 2 * J.Hkv) * kHeadDim;
+  const int f0 = t * kHeadDim + j, f1 = f0 + 64;
+  float y0 = 0.f, y1 = 0.f;
+  for (int s = 0; s < J.splits; ++s) {
+    const float* p = J.part + ((int64_t)s * J.Rp + r) * n_out;
+    y0 += p[f0];
+    y1 += p[f1];
+  }
+  if (J.bias) {
+    y0 += __bfloat162float(J.bias[f0]);
+    y1 += __bfloat162float(J.bias[f1]);
+  }
+  __nv_bfloat16* dst;
+  if (t < J.Hq + J.Hkv) {
+    // angle = pos * theta^(-2j/d) in fp64 (exact enough at any stream position)
+    const double inv = pow(J.theta, -2.0 * (double)j / (double)kHeadDim);
+    const double ang = (double)(J.pos0 + r) * inv;
+    double sd, cd;
+    sincos(ang, &sd, &cd);
+    const float c = (float)cd, sn = (float)sd;
+    const float a = fmaf(y0, c, -y1 * sn);
+    const float b = fmaf(y1, c, y0 * sn);
+    y0 = a;
+    y1 = b;
+    dst = t < J.Hq ? J.q + ((int64_t)r * J.Hq + t) * kHeadDim
+                   : J.k + ((int64_t)r * J.Hkv + (t - J.Hq)) * kHeadDim;
+  } else {
+    dst = J.v + ((int64_t)r * J.Hkv + (t - J.Hq - J.Hkv)) * kHeadDim;
+  }
+  dst[j] = __float2bfloat16_rn(y0);
+  dst[j + 64] = __float2bfloat16_rn(y1);
+}
+
+struct SwigluJob {
+  const float* part;           // [splits][Rp][2 I]
+  int splits, Rp, R, I;
+  __nv_bfloat16* A;            // [Rp][I]
+};
+
+__global__ void __launch_bounds__(256) k_fw_swiglu(const SwigluJob J) {
+  const int64_t x = (int64_t)blockIdx.x * 256 + threadIdx.x;
+  if (x >= (int64_t)J.Rp * J.I) return;
+  const int r = (int)(x / J.I), f = (int)(x - (int64_t)r * J.I);
+  float a = 0.f;
+  if (r < J.R) {
+    float g = 0.f, u = 0.f;
+    for (int s = 0; s < J.splits; ++s) {
+      const float* p = J.part + ((int64_t)s * J.Rp + r) * (2 * J.I);
+      g += p[f];
+      u += p[J.I + f];
+    }
+    a = g / (1.0f + expf(-g)) * u;
+  }
+  J.A[x] = __float2bfloat16_rn(a);
+}
+
+// ===========================================================================
+// Attention of the question rows over the layer's stored tokens
+// ===========================================================================
+constexpr int kAtThreads = 192;            // warp 0 TMA, warp 1 MMA, warps 2-5 rows
+constexpr int kAtTile = 128;               // tokens per tile
+constexpr int kAtTileBytes = kAtTile * kHeadDim * 2;   // 32 KB
+constexpr float kAtLazy = 8.0f;            // raise the running max only past this margin
+
+struct AttnJob {
+  int layer;
+  int Hq, Hkv, G, R, Rp, GRp, halves;
+  int n_tok;                       // stored tokens of every slab
+  int chunks;
+  const __nv_bfloat16* q;          // [R][Hq][d] this layer's question rows
+  float* opart;                    // [Hkv][chunks][halves * 128][d] unnormalised O
+  float2* mlpart;                  // [Hkv][chunks][halves * 128] (m, l)
+  uint32_t* status;
+};
+
+struct AtBars {
+  unsigned long long kfull[2], kempty[2], vfull[2], vempty[2], sfull[2], sempty[2];
+  unsigned long long pfull, pvdone, q_ready, final_mma;
+  uint32_t taddr;
+  int abort;
+};
+
+// grid (chunks, halves, Hkv). Rows rho = h * Rp + r (h < G) of key head g; this CTA
+// takes rho in [128 * half, 128 * half + 128).
+__global__ void __launch_bounds__(kAtThreads, 1)
+    k_fw_attn(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
+              const AttnJob J) {
+  extern __shared__ unsigned char sm_raw[];
+  __shared__ AtBars S;
+  unsigned char* sm = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  unsigned char* qs = sm;                    // A operand of S = Q K^T: 128 rows x 128 dims
+  unsigned char* ps = qs + kAtTileBytes;     // A operand of O += P V: 128 rows x 128 tokens
+  unsigned char* kr = ps + kAtTileBytes;     // 2 key stages
+  unsigned char* vr = kr + 2 * kAtTileBytes; // 2 value stages
+  const int chunk = blockIdx.x, half = blockIdx.y, g = blockIdx.z;
+  const int T = (J.n_tok + kAtTile - 1) / kAtTile;
+  const int t0 = (int)((int64_t)T * chunk / J.chunks);
+  const int t1 = (int)((int64_t)T * (chunk + 1) / J.chunks);
+  const int n = t1 - t0;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  volatile int* abort = &S.abort;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(smem_u32(&S.kfull[s]), 1);
+      mbar_init(smem_u32(&S.kempty[s]), 1);
+      mbar_init(smem_u32(&S.vfull[s]), 1);
+      mbar_init(smem_u32(&S.vempty[s]), 1);
+      mbar_init(smem_u32(&S.sfull[s]), 1);
+      mbar_init(smem_u32(&S.sempty[s]), 128);
+    }
+    mbar_init(smem_u32(&S.pfull), 128);
+    mbar_init(smem_u32(&S.pvdone), 1);
+    mbar_init(smem_u32(&S.q_ready), 1);
+    mbar_init(smem_u32(&S.final_mma), 1);
+    S.abort = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&S.taddr), 512);   // S in columns 0-255 (two buffers), O at 256
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tbase = S.taddr;
+  // tensor maps [P][Hkv][n_tok][d]: a tile past the stored tokens reads zeros
+  const int y0 = t0 * kAtTile;
+  if (warp == 0 && lane == 0) {
+    // ---- TMA producer: K(j) and V(j) into their rings ----
+    int klast[2] = {-1, -1}, vlast[2] = {-1, -1};
+    for (int j = 0; j < n && !*abort; ++j) {
+      const int st = j & 1;
+      const int y = y0 + j * kAtTile;
+      if (j >= 2 && !fw_wait(smem_u32(&S.kempty[st]), ((j >> 1) - 1) & 1, abort)) break;
+      uint32_t bar = smem_u32(&S.kfull[st]);
+      uint32_t dst = smem_u32(kr + st * kAtTileBytes);
+      mbar_expect_tx(bar, kAtTileBytes);
+      tma_load_4d(dst, &kmap, bar, 0, y, g, J.layer);
+      tma_load_4d(dst + kAtTileBytes / 2, &kmap, bar, 64, y, g, J.layer);
+      klast[st] = j;
+      if (j >= 2 && !fw_wait(smem_u32(&S.vempty[st]), ((j >> 1) - 1) & 1, abort)) break;
+      bar = smem_u32(&S.vfull[st]);
+      dst = smem_u32(vr + st * kAtTileBytes);
+      mbar_expect_tx(bar, kAtTileBytes);
+      tma_load_4d(dst, &vmap, bar, 0, y, g, J.layer);
+      tma_load_4d(dst + kAtTileBytes / 2, &vmap, bar, 64, y, g, J.layer);
+      vlast[st] = j;
+    }
+    for (int s = 0; s < 2; ++s) {
+      if (klast[s] >= 0) mbar_wait_bounded(smem_u32(&S.kfull[s]), (klast[s] >> 1) & 1);
+      if (vlast[s] >= 0) mbar_wait_bounded(smem_u32(&S.vfull[s]), (vlast[s] >> 1) & 1);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ---- MMA issuer: S(j) = Q K(j)^T, then O += P(j - 1) V(j - 1) ----
+    const uint32_t id1 = idesc_bf16_f32(128, 128, false, false);
+    const uint32_t id2 = idesc_bf16_f32(128, 128, false, true);
+    const uint32_t qa = smem_u32(qs), pa = smem_u32(ps);
+    if (fw_wait(smem_u32(&S.q_ready), 0, abort)) {
+      for (int j = 0; j <= n; ++j) {
+        if (j < n) {
+          const int st = j & 1;
+          if (!fw_wait(smem_u32(&S.kfull[st]), (j >> 1) & 1, abort)) break;
+          if (j >= 2 && !fw_wait(smem_u32(&S.sempty[st]), ((j >> 1) - 1) & 1, abort)) break;
+          tc_fence_after();
+          const uint32_t ka = smem_u32(kr + st * kAtTileBytes);
+          const uint32_t d = tbase + (uint32_t)st * 128u;
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const uint32_t ko = (k >> 2) * 16384 + (k & 3) * 32;
+            umma_bf16(d, sdesc_sw128(qa + ko, 16, 1024), sdesc_sw128(ka + ko, 16, 1024), id1,
+                      k > 0 ? 1u : 0u);
+          }
+          umma_commit(smem_u32(&S.sfull[st]));
+          umma_commit(smem_u32(&S.kempty[st]));
+        }
+        if (j >= 1) {
+          const int jp = j - 1, st = jp & 1;
+          if (!fw_wait(smem_u32(&S.pfull), jp & 1, abort)) break;
+          if (!fw_wait(smem_u32(&S.vfull[st]), (jp >> 1) & 1, abort)) break;
+          tc_fence_after();
+          const uint32_t va = smem_u32(vr + st * kAtTileBytes);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            // P: K-major, tokens in two 64-token halves; V: N = dims MN-major (two 64-dim
+            // blocks 16 KB apart), 16 tokens = 2048 bytes per K step
+            const uint32_t pk = (k >> 2) * 16384 + (k & 3) * 32;
+            umma_bf16(tbase + 256u, sdesc_sw128(pa + pk, 16, 1024),
+                      sdesc_sw128(va + k * 2048, 16384, 1024), id2, (jp > 0 || k > 0) ? 1u : 0u);
+          }
+          umma_commit(smem_u32(&S.vempty[st]));
+          umma_commit(smem_u32(&S.pvdone));
+        }
+      }
+    }
+    umma_commit(smem_u32(&S.final_mma));
+    mbar_wait_bounded(smem_u32(&S.final_mma), 0);
+  } else if (warp >= 2) {
+    // ---- rows: one per thread (TMEM lane) ----
+    const int e = threadIdx.x - 64;
+    const int qd = warp & 3;
+    const int rl = qd * 32 + lane;                 // row within the CTA's 128
+    const int rho = half * 128 + rl;
+    const int hl = rho / J.Rp, r = rho - hl * J.Rp;
+    const bool valid = hl < J.G && r < J.R;
+    // question rows -> 128-byte swizzled K-major tile (two halves of 64 dims)
+    for (int x = e; x < 128 * 16; x += 128) {
+      const int row = x >> 4, c = x & 15;
+      const int rr = half * 128 + row;
+      const int h2 = rr / J.Rp, r2 = rr - h2 * J.Rp;
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      if (h2 < J.G && r2 < J.R)
+        v = *reinterpret_cast<const uint4*>(J.q + ((int64_t)r2 * J.Hq + g * J.G + h2) * kHeadDim +
+                                            8 * c);
+      *reinterpret_cast<uint4*>(qs + (c >> 3) * 16384 + row * 128 + (((c & 7) ^ (row & 7)) << 4)) = v;
+    }
+    fence_proxy_async_smem();
+    fw_bar(1, 128);
+    if (e == 0) mbar_arrive(smem_u32(&S.q_ready));
+    const uint32_t la = tbase + ((uint32_t)(qd * 32) << 16);
+    unsigned char* prow = ps + rl * 128;
+    float m = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int j = 0; j < n; ++j) {
+      const int st = j & 1;
+      ok = ok && fw_wait(smem_u32(&S.sfull[st]), (j >> 1) & 1, abort);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) break;
+      tc_fence_after();
+      float s[128];
+      tmem_ld32x4(la + st * 128u, la + st * 128u + 32u, la + st * 128u + 64u, la + st * 128u + 96u,
+                  s);
+      tc_fence_before();
+      mbar_arrive(smem_u32(&S.sempty[st]));
+      const int nv = min(kAtTile, J.n_tok - (t0 + j) * kAtTile);   // valid tokens
+      float mt = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < 128; ++c) mt = fmaxf(mt, c < nv ? s[c] : -INFINITY);
+      mt *= kScoreScale;
+      const bool raise = mt > m + kAtLazy;
+      const float m_new = raise ? mt : m;
+      // P = 2^(s - m_new) in bf16; l sums the rounded values the MMA uses
+      uint32_t pk[64];
+      float lt = 0.f;
+#pragma unroll
+      for (int c = 0; c < 64; ++c) {
+        const float p0 = 2 * c < nv ? fast_exp2(fmaf(s[2 * c], kScoreScale, -m_new)) : 0.f;
+        const float p1 = 2 * c + 1 < nv ? fast_exp2(fmaf(s[2 * c + 1], kScoreScale, -m_new)) : 0.f;
+        const __nv_bfloat162 b2 = __floats2bfloat162_rn(p0, p1);
+        lt += __low2float(b2) + __high2float(b2);
+        pk[c] = *reinterpret_cast<const uint32_t*>(&b2);
+      }
+      // O and the P buffer are free once the previous tile's O += P V has completed
+      if (j >= 1) {
+        ok = fw_wait(smem_u32(&S.pvdone), (j - 1) & 1, abort);
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok) break;
+        tc_fence_after();
+        const float fac = raise ? fast_exp2(m - m_new) : 1.0f;
+        if (__any_sync(0xffffffffu, raise)) {
+#pragma unroll 1
+          for (int c0 = 0; c0 < 128; c0 += 32) {
+            float o[32];
+            tmem_ld32(la + 256u + (uint32_t)c0, o);
+#pragma unroll
+            for (int c = 0; c < 32; ++c) o[c] *= fac;
+            tmem_st32(la + 256u + (uint32_t)c0, o);
+          }
+        }
+        l *= fac;
+      }
+      m = m_new;
+      l += lt;
+      // the P row: tokens 0-63 in half 0, 64-127 in half 1; 16-byte chunks swizzled
+#pragma unroll
+      for (int c = 0; c < 16; ++c) {
+        const uint4 w = make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+        *reinterpret_cast<uint4*>(prow + (c >> 3) * 16384 + (((c & 7) ^ (rl & 7)) << 4)) = w;
+      }
+      fence_proxy_async_smem();
+      tc_fence_before();
+      mbar_arrive(smem_u32(&S.pfull));
+    }
+    if (ok && n > 0) {
+      ok = fw_wait(smem_u32(&S.pvdone), (n - 1) & 1, abort);
+      ok = __all_sync(0xffffffffu, ok);
+    }
+    tc_fence_after();
+    const int64_t prow_out = ((int64_t)g * J.chunks + chunk) * (J.halves * 128) + rho;
+    if (ok && !*abort) {
+      for (int c0 = 0; c0 < 128; c0 += 32) {
+        float o[32];
+        tmem_ld32(la + 256u + (uint32_t)c0, o);
+        if (valid && n > 0) {
+          float4* dst = reinterpret_cast<float4*>(J.opart + prow_out * kHeadDim + c0);
+#pragma unroll
+          for (int c = 0; c < 8; ++c) dst[c] = make_float4(o[4 * c], o[4 * c + 1], o[4 * c + 2], o[4 * c + 3]);
+        }
+      }
+      if (valid) J.mlpart[prow_out] = n > 0 ? make_float2(m, l) : make_float2(-INFINITY, 0.f);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (threadIdx.x == 0 && S.abort) atomicOr(J.status, kStatusTimeout);
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tbase, 512);
+}
+
+struct AttnOutJob {
+  int Hq, Hkv, G, R, Rp, halves, chunks;
+  const __nv_bfloat16* q;          // [R][Hq][d]
+  const __nv_bfloat16* k;          // [R][Hkv][d] the question's own keys
+  const __nv_bfloat16* v;          // [R][Hkv][d]
+  const float* opart;
+  const float2* mlpart;
+  __nv_bfloat16* o;                // [Rp][Hq d] (rows >= R zero)
+  const uint32_t* status;
+};
+
+// One warp per (row of Rp, head): the chunks in chunk order, then the question's own
+// rows 0..r; lane owns dims 4 lane .. 4 lane + 3.
+__global__ void __launch_bounds__(256) k_fw_attn_out(const AttnOutJob J) {
+  const int wid = (blockIdx.x * 256 + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (wid >= J.Rp * J.Hq) return;
+  const int r = wid / J.Hq, h = wid - r * J.Hq;
+  __nv_bfloat16* dst = J.o + (int64_t)r * J.Hq * kHeadDim + h * kHeadDim + 4 * lane;
+  if (r >= J.R || (*(volatile const uint32_t*)J.status & kStatusTimeout)) {
+    const __nv_bfloat162 z = __floats2bfloat162_rn(0.f, 0.f);
+    reinterpret_cast<__nv_bfloat162*>(dst)[0] = z;
+    reinterpret_cast<__nv_bfloat162*>(dst)[1] = z;
+    return;
+  }
+  const int g = h / J.G, hl = h - g * J.G;
+  const int rho = hl * J.Rp + r;
+  const int rows = J.halves * 128;
+  float M = -INFINITY;
+  for (int c = 0; c < J.chunks; ++c) {
+    const float2 ml = J.mlpart[((int64_t)g * J.chunks + c) * rows + rho];
+    if (ml.y > 0.f) M = fmaxf(M, ml.x);
+  }
+  // own rows: s_j = q_r . k_j in the log2 domain (dot products reduced in a fixed order)
+  const uint2 qv = *reinterpret_cast<const uint2*>(J.q + ((int64_t)r * J.Hq + h) * kHeadDim + 4 * lane);
+  const float q0 = __uint_as_float(qv.x << 16), q1 = __uint_as_float(qv.x & 0xffff0000u);
+  const float q2 = __uint_as_float(qv.y << 16), q3 = __uint_as_float(qv.y & 0xffff0000u);
+  float own[64];
+  for (int jr = 0; jr <= r; ++jr) {
+    const uint2 kv = *reinterpret_cast<const uint2*>(J.k + ((int64_t)jr * J.Hkv + g) * kHeadDim + 4 * lane);
+    float d = q0 * __uint_as_float(kv.x << 16);
+    d = fmaf(q1, __uint_as_float(kv.x & 0xffff0000u), d);
+    d = fmaf(q2, __uint_as_float(kv.y << 16), d);
+    d = fmaf(q3, __uint_as_float(kv.y & 0xffff0000u), d);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) d += __shfl_xor_sync(0xffffffffu, d, o);
+    own[jr] = d * kScoreScale;
+    M = fmaxf(M, own[jr]);
+  }
+  float L = 0.f;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int c = 0; c < J.chunks; ++c) {
+    const int64_t pr = ((int64_t)g * J.chunks + c) * rows + rho;
+    const float2 ml = J.mlpart[pr];
+    if (!(ml.y > 0.f)) continue;
+    const float w = fast_exp2(ml.x - M);
+    L = fmaf(ml.y, w, L);
+    const float4 ov = reinterpret_cast<const float4*>(J.opart + pr * kHeadDim)[lane];
+    acc.x = fmaf(ov.x, w, acc.x);
+    acc.y = fmaf(ov.y, w, acc.y);
+    acc.z = fmaf(ov.z, w, acc.z);
+    acc.w = fmaf(ov.w, w, acc.w);
+  }
+  for (int jr = 0; jr <= r; ++jr) {
+    const float w = fast_exp2(own[jr] - M);
+    L += w;
+    const uint2 vv = *reinterpret_cast<const uint2*>(J.v + ((int64_t)jr * J.Hkv + g) * kHeadDim + 4 * lane);
+    acc.x = fmaf(__uint_as_float(vv.x << 16), w, acc.x);
+    acc.y = fmaf(__uint_as_float(vv.x & 0xffff0000u), w, acc.y);
+    acc.z = fmaf(__uint_as_float(vv.y << 16), w, acc.z);
+    acc.w = fmaf(__uint_as_float(vv.y & 0xffff0000u), w, acc.w);
+  }
+  const float inv = 1.0f / L;
+  reinterpret_cast<__nv_bfloat162*>(dst)[0] = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
+  reinterpret_cast<__nv_bfloat162*>(dst)[1] = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
+}
+
+// ===========================================================================
+// Host: one forward
+// ===========================================================================
+namespace {
+
+int gemm_stages(int Rp) {
+  const int stage = kGmABytes + Rp * 128;
+  int s = (110 * 1024) / stage;              // two CTAs per SM
+  return s < 2 ? 2 : (s > kGmMaxStages ? kGmMaxStages : s);
+}
+
+int gemm_splits(int n_out, int kblocks, int sm_count) {
+  const int tiles = n_out / 128;
+  int s = (2 * sm_count + tiles / 2) / tiles;
+  if (s < 1) s = 1;
+  if (s > kblocks) s = kblocks;
+  if (s > 16) s = 16;
+  return s;
+}
+
+struct Seg {
+  size_t off = 0;
+  template <typename T>
+  size_t take(size_t count) {
+    const size_t o = off;
+    off = (off + count * sizeof(T) + 255) & ~(size_t)255;
+    return o;
+  }
+};
+
+struct FwLayout {
+  size_t H, X, A, part, k, v, opart, ml, status, total;
+  int Rp, halves, chunks, sp_qkv, sp_o, sp_gu, sp_d;
+};
+
+FwLayout fw_layout(const FwShape& F) {
+  FwLayout L{};
+  const int D = F.Hq * kHeadDim;
+  L.Rp = (F.R + 15) & ~15;
+  const int G = F.Hq / F.Hkv;
+  L.halves = (G * L.Rp + 127) / 128;
+  const int T = (F.n_tok + kAtTile - 1) / kAtTile;
+  int c = F.sm_count / (L.halves * F.Hkv);
+  c = c < 1 ? 1 : c;
+  L.chunks = T < 1 ? 1 : (T < c ? T : c);
+  const int nqkv = (F.Hq + 2 * F.Hkv) * kHeadDim;
+  L.sp_qkv = gemm_splits(nqkv, D / 64, F.sm_count);
+  L.sp_o = gemm_splits(D, D / 64, F.sm_count);
+  L.sp_gu = gemm_splits(2 * F.I, D / 64, F.sm_count);
+  L.sp_d = gemm_splits(D, F.I / 64, F.sm_count);
+  size_t part = (size_t)L.sp_qkv * nqkv;
+  part = std::max(part, (size_t)L.sp_o * D);
+  part = std::max(part, (size_t)L.sp_gu * 2 * F.I);
+  part = std::max(part, (size_t)L.sp_d * D);
+  Seg s;
+  L.H = s.take<float>((size_t)F.R * D);
+  L.X = s.take<__nv_bfloat16>((size_t)L.Rp * D);
+  L.A = s.take<__nv_bfloat16>((size_t)L.Rp * F.I);
+  L.part = s.take<float>(part * L.Rp);
+  L.k = s.take<__nv_bfloat16>((size_t)F.R * F.Hkv * kHeadDim);
+  L.v = s.take<__nv_bfloat16>((size_t)F.R * F.Hkv * kHeadDim);
+  L.opart = s.take<float>((size_t)F.Hkv * L.chunks * L.halves * 128 * kHeadDim);
+  L.ml = s.take<float2>((size_t)F.Hkv * L.chunks * L.halves * 128);
+  L.status = s.take<uint32_t>(1);
+  L.total = s.off;
+  return L;
+}
+
+cudaError_t gemm(const void* W, int n_out, int K, const __nv_bfloat16* X, int R, int Rp,
+                 int splits, float* part, uint32_t* status, cudaStream_t st) {
+  CUtensorMap wm, xm;
+  const uint64_t wd[2] = {(uint64_t)K, (uint64_t)n_out}, ws[1] = {(uint64_t)K * 2};
+  const uint32_t wb[2] = {64, 128};
+  cudaError_t e = encode_bf16_map(&wm, W, 2, wd, ws, wb);
+  if (e != cudaSuccess) return e;
+  const uint64_t xd[2] = {(uint64_t)K, (uint64_t)Rp}, xs[1] = {(uint64_t)K * 2};
+  const uint32_t xb[2] = {64, (uint32_t)Rp};
+  e = encode_bf16_map(&xm, X, 2, xd, xs, xb);
+  if (e != cudaSuccess) return e;
+  GemmJob J;
+  J.part = part;
+  J.n_out = n_out;
+  J.R = R;
+  J.Rp = Rp;
+  J.kblocks = K / 64;
+  J.splits = splits;
+  J.stages = gemm_stages(Rp);
+  J.status = status;
+  const int smem = J.stages * (kGmABytes + Rp * 128) + 1024;
+  e = ensure_smem((const void*)k_fw_gemm, smem);
+  if (e != cudaSuccess) return e;
+  k_fw_gemm<<<dim3(n_out / 128, splits), kGmThreads, smem, st>>>(wm, xm, J);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool forward_supported(int R, int Hq, int Hkv) {
+  const int Rp = (R + 15) & ~15;
+  return R >= 1 && R <= 64 && (Hq / Hkv) * Rp <= 256;
+}
+
+size_t forward_workspace_bytes(const FwShape& F) { return fw_layout(F).total; }
+
+cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
+  const FwLayout L = fw_layout(F);
+  unsigned char* ws = static_cast<unsigned char*>(A.workspace);
+  float* H = reinterpret_cast<float*>(ws + L.H);
+  __nv_bfloat16* X = reinterpret_cast<__nv_bfloat16*>(ws + L.X);
+  __nv_bfloat16* Ab = reinterpret_cast<__nv_bfloat16*>(ws + L.A);
+  float* part = reinterpret_cast<float*>(ws + L.part);
+  __nv_bfloat16* kown = reinterpret_cast<__nv_bfloat16*>(ws + L.k);
+  __nv_bfloat16* vown = reinterpret_cast<__nv_bfloat16*>(ws + L.v);
+  float* opart = reinterpret_cast<float*>(ws + L.opart);
+  float2* ml = reinterpret_cast<float2*>(ws + L.ml);
+  uint32_t* status = A.status ? A.status : reinterpret_cast<uint32_t*>(ws + L.status);
+  const int D = F.Hq * kHeadDim, G = F.Hq / F.Hkv;
+  const int nqkv = (F.Hq + 2 * F.Hkv) * kHeadDim;
+  cudaError_t e = cudaMemsetAsync(status, 0, sizeof(uint32_t), st);
+  if (e != cudaSuccess) return e;
+  // stored keys and values of every layer as [P][Hkv][n_tok][d] (the stored tokens of a
+  // slab only, so the last tile's rows past them read zeros), tiles of 128 tokens
+  CUtensorMap km, vm;
+  const uint64_t dims[4] = {(uint64_t)kHeadDim, (uint64_t)F.n_tok, (uint64_t)F.Hkv, (uint64_t)F.P};
+  const uint64_t strides[3] = {(uint64_t)kHeadDim * 2, (uint64_t)F.ncap * kHeadDim * 2,
+                               (uint64_t)F.Hkv * F.ncap * kHeadDim * 2};
+  const uint32_t box[4] = {64, (uint32_t)kAtTile, 1, 1};
+  if (F.n_tok > 0) {
+    e = encode_bf16_map(&km, F.keys, 4, dims, strides, box);
+    if (e != cudaSuccess) return e;
+    e = encode_bf16_map(&vm, F.values, 4, dims, strides, box);
+    if (e != cudaSuccess) return e;
+    e = ensure_smem((const void*)k_fw_attn, 6 * kAtTileBytes + 1024);
+    if (e != cudaSuccess) return e;
+  }
+  NormJob nj{};
+  nj.H = H;
+  nj.D = D;
+  nj.R = F.R;
+  nj.Rp = L.Rp;
+  nj.eps = F.eps;
+  for (int i = 0; i < F.P; ++i) {
+    const FwLayerW& W = A.layers[i];
+    __nv_bfloat16* q = static_cast<__nv_bfloat16*>(A.q_out) + (int64_t)i * F.R * F.Hq * kHeadDim;
+    // X = bf16(RMSNorm(H) * ln1); layer 0 starts from the question's rows, later layers
+    // add the previous layer's down-projection partials first
+    nj.h_in = i == 0 ? static_cast<const __nv_bfloat16*>(A.h_in) : nullptr;
+    nj.part = i == 0 ? nullptr : part;
+    nj.splits = L.sp_d;
+    nj.w = static_cast<const __nv_bfloat16*>(W.ln1);
+    nj.X = X;
+    k_fw_norm<<<L.Rp, 256, 0, st>>>(nj);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = gemm(W.wqkv, nqkv, D, X, F.R, L.Rp, L.sp_qkv, part, status, st)) != cudaSuccess) return e;
+    QkvJob qj;
+    qj.part = part;
+    qj.splits = L.sp_qkv;
+    qj.Rp = L.Rp;
+    qj.R = F.R;
+    qj.bias = static_cast<const __nv_bfloat16*>(W.bqkv);
+    qj.Hq = F.Hq;
+    qj.Hkv = F.Hkv;
+    qj.pos0 = F.pos0;
+    qj.theta = F.theta;
+    qj.q = q;
+    qj.k = kown;
+    qj.v = vown;
+    k_fw_qkv<<<dim3(F.R, F.Hq + 2 * F.Hkv), 64, 0, st>>>(qj);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if (F.n_tok > 0) {
+      AttnJob aj;
+      aj.layer = i;
+      aj.Hq = F.Hq;
+      aj.Hkv = F.Hkv;
+      aj.G = G;
+      aj.R = F.R;
+      aj.Rp = L.Rp;
+      aj.GRp = G * L.Rp;
+      aj.halves = L.halves;
+      aj.n_tok = F.n_tok;
+      aj.chunks = L.chunks;
+      aj.q = q;
+      aj.opart = opart;
+      aj.mlpart = ml;
+      aj.status = status;
+      k_fw_attn<<<dim3(L.chunks, L.halves, F.Hkv), kAtThreads, 6 * kAtTileBytes + 1024, st>>>(km, vm, aj);
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    AttnOutJob oj;
+    oj.Hq = F.Hq;
+    oj.Hkv = F.Hkv;
+    oj.G = G;
+    oj.R = F.R;
+    oj.Rp = L.Rp;
+    oj.halves = L.halves;
+    oj.chunks = F.n_tok > 0 ? L.chunks : 0;
+    oj.q = q;
+    oj.k = kown;
+    oj.v = vown;
+    oj.opart = opart;
+    oj.mlpart = ml;
+    oj.o = X;
+    oj.status = status;
+    const int warps = L.Rp * F.Hq;
+    k_fw_attn_out<<<(warps * 32 + 255) / 256, 256, 0, st>>>(oj);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = gemm(W.wo, D, D, X, F.R, L.Rp, L.sp_o, part, status, st)) != cudaSuccess) return e;
+    // H += o Wo^T; X = bf16(RMSNorm(H) * ln2)
+    nj.h_in = nullptr;
+    nj.part = part;
+    nj.splits = L.sp_o;
+    nj.w = static_cast<const __nv_bfloat16*>(W.ln2);
+    k_fw_norm<<<L.Rp, 256, 0, st>>>(nj);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = gemm(W.wgu, 2 * F.I, D, X, F.R, L.Rp, L.sp_gu, part, status, st)) != cudaSuccess) return e;
+    SwigluJob sj;
+    sj.part = part;
+    sj.splits = L.sp_gu;
+    sj.Rp = L.Rp;
+    sj.R = F.R;
+    sj.I = F.I;
+    sj.A = Ab;
+    k_fw_swiglu<<<(int)(((int64_t)L.Rp * F.I + 255) / 256), 256, 0, st>>>(sj);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = gemm(W.wd, D, F.I, Ab, F.R, L.Rp, L.sp_d, part, status, st)) != cudaSuccess) return e;
+  }
+  // H += the last down projection
+  nj.h_in = nullptr;
+  nj.part = part;
+  nj.splits = L.sp_d;
+  nj.w = nullptr;
+  k_fw_norm<<<L.Rp, 256, 0, st>>>(nj);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if (A.h_out)
+    return cudaMemcpyAsync(A.h_out, H, (size_t)F.R * D * sizeof(float), cudaMemcpyDeviceToDevice, st);
+  return cudaSuccess;
+}
+
+}  // namespace ss

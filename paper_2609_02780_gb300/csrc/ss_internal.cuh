@@ -326,4 +326,31 @@ cudaError_t launch_descriptors(const __nv_bfloat16* keys, int64_t ncap, int P, i
                                cudaStream_t s);
 int score_chunks_per_slab(int n_slabs_total, int hist_units, int sm_count);
 int score_slots(int sm_count);
+
+// The question's forward through the shallow layers (ss_forward.cu).
+struct FwShape {
+  int P, Hq, Hkv, R, I;
+  int64_t ncap;                 // tokens per slab of the index's arrays
+  int n_tok;                    // stored tokens per slab
+  int sm_count;
+  float eps;
+  double theta;
+  int64_t pos0;
+  const void* keys;             // bf16 [P][Hkv][ncap][d]
+  const void* values;           // bf16 [P][Hkv][ncap][d]
+};
+struct FwLayerW {
+  const void *ln1, *wqkv, *bqkv, *wo, *ln2, *wgu, *wd;
+};
+struct FwArgs {
+  const FwLayerW* layers;       // [P]
+  const void* h_in;             // bf16 [R][D]
+  void* q_out;                  // bf16 [P][R][Hq][d]
+  float* h_out;                 // fp32 [R][D] or NULL
+  uint32_t* status;             // device word or NULL (then in the workspace)
+  void* workspace;
+};
+bool forward_supported(int R, int Hq, int Hkv);
+size_t forward_workspace_bytes(const FwShape& F);
+cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st);
 }  // namespace ss

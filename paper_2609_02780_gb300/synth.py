@@ -12,7 +12,9 @@ consume its bytes.
 
 Layouts (all contiguous, bf16):
   keys    [P][Hkv][F * T_f][d]   token id p = frame * T_f + slot
+  values  [P][Hkv][F * T_f][d]   (the question's forward only)
   queries [P][R][Hq][d]
+  question rows [R][Hq d] and decoder-layer weights (the question's forward only)
 """
 from __future__ import annotations
 
@@ -106,6 +108,12 @@ PRESETS = {
     "hour1_msm": Workload("hour1_msm", n_layers=4, n_frames=3600, tokens_per_frame=196,
                           n_rows=32, k=1024, budget=64, n_planted=16,
                           keys="drift_outlier", seed=0, q_agg=2),
+    # the 1-hour stream with the question's forward through the shallow layers (Eq. 10):
+    # synthetic decoder layers of hidden size 28 * 128 and MLP width 18944 produce the
+    # query rows the retrieval scores
+    "hour1_fwd": Workload("hour1_fwd", n_layers=4, n_frames=3600, tokens_per_frame=196,
+                          n_rows=32, k=1024, budget=64, n_planted=16,
+                          keys="drift_outlier", seed=0, extra={"intermediate": 18944}),
     # Table 4 evidence-selection settings (Qwen3-VL column: 2-frame units, P = 5,
     # 64 candidates per layer averaged over heads, pool 32, K = 8, 6 recent units).
     "paper_qwen": Workload("paper_qwen", n_layers=5, n_frames=256, tokens_per_frame=64,
@@ -208,6 +216,56 @@ def make_keys(w: Workload, q: torch.Tensor, device="cpu",
                 z[f * Tf:(f + 1) * Tf] += shift[i, j]
             out[i, j] = z.to(torch.bfloat16)
     return out
+
+
+def make_values(w: Workload, device="cpu", seed: int | None = None) -> torch.Tensor:
+    """Shallow values, bf16 [P][Hkv][F*T_f][d] ~ N(0, 1), drawn per layer, per kv head."""
+    s = w.seed if seed is None else seed
+    g = _gen(2_000_003 + s, device)
+    P, Hkv, N, d = w.n_layers, w.n_kv_heads, w.n_frames * w.tokens_per_frame, w.head_dim
+    out = torch.empty(P, Hkv, N, d, dtype=torch.bfloat16, device=device)
+    for i in range(P):
+        for j in range(Hkv):
+            out[i, j] = torch.randn(N, d, generator=g, device=device).to(torch.bfloat16)
+    return out
+
+
+def make_forward_weights(w: Workload, intermediate: int, device="cpu", seed: int | None = None,
+                         bias: bool = True) -> list[dict]:
+    """Synthetic weights of the P shallow decoder layers (one dict per layer, bf16):
+    RMSNorm weights 1 + N(0, 0.1^2); projections N(0, 1 / fan_in); q/k/v bias N(0, 0.1^2).
+    Layouts as ss_layer_weights: wqkv [(Hq + 2 Hkv) d][D], wo [D][Hq d], wgu [2 I][D]
+    (gate rows, then up rows), wd [D][I]."""
+    s = w.seed if seed is None else seed
+    g = _gen(3_000_017 + s, device)
+    D = w.n_q_heads * w.head_dim
+    nqkv = (w.n_q_heads + 2 * w.n_kv_heads) * w.head_dim
+    I = intermediate
+
+    def rnd(*shape, std=1.0, mean=0.0):
+        x = torch.randn(*shape, generator=g, device=device) * std + mean
+        return x.to(torch.bfloat16).contiguous()
+
+    layers = []
+    for _ in range(w.n_layers):
+        layers.append({
+            "ln1": rnd(D, std=0.1, mean=1.0),
+            "wqkv": rnd(nqkv, D, std=D ** -0.5),
+            "bqkv": rnd(nqkv, std=0.1) if bias else None,
+            "wo": rnd(D, D, std=D ** -0.5),
+            "ln2": rnd(D, std=0.1, mean=1.0),
+            "wgu": rnd(2 * I, D, std=D ** -0.5),
+            "wd": rnd(D, I, std=I ** -0.5),
+        })
+    return layers
+
+
+def make_question_rows(w: Workload, device="cpu", seed: int | None = None) -> torch.Tensor:
+    """The question's embedded rows entering the first shallow layer, bf16 [R][Hq d] ~ N(0, 1)."""
+    s = w.seed if seed is None else seed
+    g = _gen(4_000_037 + s, device)
+    D = w.n_q_heads * w.head_dim
+    return torch.randn(w.n_rows, D, generator=g, device=device).to(torch.bfloat16)
 
 
 def make_workload(w: Workload, device="cpu", stream: int = 0) -> dict:

@@ -233,7 +233,7 @@ def test_planted_mistakes_fail_the_library_comparison(monkeypatch):
                            theta=1e4)
             assert np.abs(bad["q"] - lib["q"].numpy()).max() > 1e-3
 
-    def shifted_attention(q, hist_k, hist_v, own_k, own_v):
+    def shifted_attention(q, hist_k, hist_v, own_k, own_v, spread=False):
         # rows r >= 1 see one own row too few (a causal mask off by one)
         R_, Hq_, d_ = q.shape
         G_ = Hq_ // hist_k.shape[0]
