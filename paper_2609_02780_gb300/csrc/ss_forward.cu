@@ -177,41 +177,96 @@ struct NormJob {
   int splits;
   const __nv_bfloat16* w;      // [D] or NULL: no normalisation
   __nv_bfloat16* X;            // [Rp][D] (rows >= R zero)
-  int D, R, Rp;
+  float* ssq;                  // [R][chunks] partial sums of squares
+  unsigned int* ticket;        // [R] arrival counters (never reset: taken modulo chunks)
+  int D, R, Rp, chunks;
   float eps;
 };
 
-// One CTA per row of Rp: the residual add in split order, then RMSNorm with the sum of
-// squares reduced in a fixed order.
+constexpr int kNormCols = 512;   // columns per CTA (2 per thread)
+
+// Grid (chunks = D / 512, Rp). Each CTA adds the partial sums of its 512 columns of a row
+// in split order and writes H; with normalisation it also writes its sum of squares, and
+// the CTA that completes the row's count (an atomic ticket) sums the chunks' squares in
+// chunk order and writes X = bf16(H * rsqrt * w) for the whole row.
 __global__ void __launch_bounds__(256) k_fw_norm(const NormJob J) {
   __shared__ float red[8];
-  const int r = blockIdx.x, t = threadIdx.x;
+  __shared__ int s_last;
+  const int r = blockIdx.y, c0 = blockIdx.x * kNormCols, t = threadIdx.x;
   const int D = J.D;
+  const int x = c0 + 2 * t;                 // this thread's two columns (D is even)
+  const bool in = x < D;
   if (r >= J.R) {
-    if (J.w)
-      for (int x = t; x < D; x += 256) J.X[(int64_t)r * D + x] = __float2bfloat16_rn(0.f);
+    if (J.w && in)
+      reinterpret_cast<__nv_bfloat162*>(J.X + (int64_t)r * D)[x >> 1] = __floats2bfloat162_rn(0.f, 0.f);
     return;
   }
-  float ss = 0.f;
-  for (int x = t; x < D; x += 256) {
-    float h = J.h_in ? __bfloat162float(J.h_in[(int64_t)r * D + x]) : J.H[(int64_t)r * D + x];
-    if (J.part)
-      for (int s = 0; s < J.splits; ++s) h += J.part[((int64_t)s * J.Rp + r) * D + x];
-    J.H[(int64_t)r * D + x] = h;
-    ss = fmaf(h, h, ss);
+  float2 h = make_float2(0.f, 0.f);
+  if (in) {
+    if (J.h_in) {
+      const __nv_bfloat162 b = reinterpret_cast<const __nv_bfloat162*>(J.h_in + (int64_t)r * D)[x >> 1];
+      h = make_float2(__low2float(b), __high2float(b));
+    } else {
+      h = reinterpret_cast<const float2*>(J.H + (int64_t)r * D)[x >> 1];
+    }
+    if (J.part) {
+      int s = 0;
+      for (; s + 4 <= J.splits; s += 4) {
+        float2 v[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          v[u] = reinterpret_cast<const float2*>(J.part + ((int64_t)(s + u) * J.Rp + r) * D)[x >> 1];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          h.x += v[u].x;
+          h.y += v[u].y;
+        }
+      }
+      for (; s < J.splits; ++s) {
+        const float2 v = reinterpret_cast<const float2*>(J.part + ((int64_t)s * J.Rp + r) * D)[x >> 1];
+        h.x += v.x;
+        h.y += v.y;
+      }
+    }
+    reinterpret_cast<float2*>(J.H + (int64_t)r * D)[x >> 1] = h;
   }
   if (!J.w) return;
+  float ss = fmaf(h.y, h.y, h.x * h.x);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
   if ((t & 31) == 0) red[t >> 5] = ss;
   __syncthreads();
-  float tot = 0.f;
+  if (t == 0) {
+    float tot = 0.f;
 #pragma unroll
-  for (int w = 0; w < 8; ++w) tot += red[w];
+    for (int w = 0; w < 8; ++w) tot += red[w];
+    J.ssq[(int64_t)r * J.chunks + blockIdx.x] = tot;
+    __threadfence();
+    const unsigned int old = atomicAdd(J.ticket + r, 1u);
+    s_last = (old % (unsigned)J.chunks) == (unsigned)(J.chunks - 1);
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  float tot = 0.f;
+  for (int c = 0; c < J.chunks; ++c) tot += __ldcg(J.ssq + (int64_t)r * J.chunks + c);
   const float inv = 1.0f / sqrtf(tot / (float)D + J.eps);
-  for (int x = t; x < D; x += 256)
-    J.X[(int64_t)r * D + x] =
-        __float2bfloat16_rn(J.H[(int64_t)r * D + x] * inv * __bfloat162float(J.w[x]));
+  for (int y = 2 * t; y < D; y += 512) {
+    const float2 hv = __ldcg(reinterpret_cast<const float2*>(J.H + (int64_t)r * D + y));
+    const __nv_bfloat162 wv = reinterpret_cast<const __nv_bfloat162*>(J.w)[y >> 1];
+    reinterpret_cast<__nv_bfloat162*>(J.X + (int64_t)r * D)[y >> 1] =
+        __floats2bfloat162_rn(hv.x * inv * __low2float(wv), hv.y * inv * __high2float(wv));
+  }
+}
+
+// cos and sin of the RoPE angles pos * theta^(-2j/d) of every question row (computed in
+// fp64, stored as fp32): [R][64] pairs.
+__global__ void __launch_bounds__(64) k_fw_rope(float2* tab, int64_t pos0, double theta) {
+  const int r = blockIdx.x, j = threadIdx.x;
+  const double inv = pow(theta, -2.0 * (double)j / (double)kHeadDim);
+  double sd, cd;
+  sincos((double)(pos0 + r) * inv, &sd, &cd);
+  tab[r * 64 + j] = make_float2((float)cd, (float)sd);
 }
 
 struct QkvJob {
@@ -219,8 +274,7 @@ struct QkvJob {
   int splits, Rp, R;
   const __nv_bfloat16* bias;   // [(Hq + 2 Hkv) d] or NULL
   int Hq, Hkv;
-  int64_t pos0;
-  double theta;
+  const float2* rope;          // [R][64] (cos, sin)
   __nv_bfloat16* q;            // [R][Hq][d] (the caller's Q^i)
   __nv_bfloat16* k;            // [R][Hkv][d]
   __nv_bfloat16* v;            // [R][Hkv][d]
@@ -232,7 +286,22 @@ __global__ void __launch_bounds__(64) k_fw_qkv(const QkvJob J) {
   const int n_out = (J.Hq + 2 * J.Hkv) * kHeadDim;
   const int f0 = t * kHeadDim + j, f1 = f0 + 64;
   float y0 = 0.f, y1 = 0.f;
-  for (int s = 0; s < J.splits; ++s) {
+  int s = 0;
+  for (; s + 4 <= J.splits; s += 4) {
+    float a[4], b[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const float* p = J.part + ((int64_t)(s + u) * J.Rp + r) * n_out;
+      a[u] = p[f0];
+      b[u] = p[f1];
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      y0 += a[u];
+      y1 += b[u];
+    }
+  }
+  for (; s < J.splits; ++s) {
     const float* p = J.part + ((int64_t)s * J.Rp + r) * n_out;
     y0 += p[f0];
     y1 += p[f1];
@@ -243,14 +312,9 @@ __global__ void __launch_bounds__(64) k_fw_qkv(const QkvJob J) {
   }
   __nv_bfloat16* dst;
   if (t < J.Hq + J.Hkv) {
-    // angle = pos * theta^(-2j/d) in fp64 (exact enough at any stream position)
-    const double inv = pow(J.theta, -2.0 * (double)j / (double)kHeadDim);
-    const double ang = (double)(J.pos0 + r) * inv;
-    double sd, cd;
-    sincos(ang, &sd, &cd);
-    const float c = (float)cd, sn = (float)sd;
-    const float a = fmaf(y0, c, -y1 * sn);
-    const float b = fmaf(y1, c, y0 * sn);
+    const float2 cs = J.rope[r * 64 + j];
+    const float a = fmaf(y0, cs.x, -y1 * cs.y);
+    const float b = fmaf(y1, cs.x, y0 * cs.y);
     y0 = a;
     y1 = b;
     dst = t < J.Hq ? J.q + ((int64_t)r * J.Hq + t) * kHeadDim
@@ -288,10 +352,33 @@ __global__ void __launch_bounds__(256) k_fw_swiglu(const SwigluJob J) {
 // ===========================================================================
 // Attention of the question rows over the layer's stored tokens
 // ===========================================================================
-constexpr int kAtThreads = 192;            // warp 0 TMA, warp 1 MMA, warps 2-5 rows
+constexpr int kAtThreads = 320;            // warp 0 TMA, warp 1 MMA, warps 2-9 rows
+constexpr int kAtEpi = 256;                // two threads per row, 64 columns each
 constexpr int kAtTile = 128;               // tokens per tile
 constexpr int kAtTileBytes = kAtTile * kHeadDim * 2;   // 32 KB
+constexpr int kAtSmem = 7 * kAtTileBytes + 1024;       // Q, 2 P, 2 K, 2 V stages
 constexpr float kAtLazy = 8.0f;            // raise the running max only past this margin
+
+// Packed fp32 pairs (the .f32x2 arithmetic of sm_100 and later): one instruction for two
+// lanes of a row's scores.
+__device__ __forceinline__ unsigned long long f2pack(float a, float b) {
+  return (unsigned long long)__float_as_uint(a) | ((unsigned long long)__float_as_uint(b) << 32);
+}
+__device__ __forceinline__ float f2lo(unsigned long long v) { return __uint_as_float((uint32_t)v); }
+__device__ __forceinline__ float f2hi(unsigned long long v) {
+  return __uint_as_float((uint32_t)(v >> 32));
+}
+__device__ __forceinline__ unsigned long long ffma2(unsigned long long a, unsigned long long b,
+                                                    unsigned long long c) {
+  unsigned long long d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ unsigned long long fadd2(unsigned long long a, unsigned long long b) {
+  unsigned long long d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
 
 struct AttnJob {
   int layer;
@@ -306,13 +393,31 @@ struct AttnJob {
 
 struct AtBars {
   unsigned long long kfull[2], kempty[2], vfull[2], vempty[2], sfull[2], sempty[2];
-  unsigned long long pfull, pvdone, q_ready, final_mma;
+  unsigned long long pfull[2], pvdone[2], q_ready, final_mma;
   uint32_t taddr;
   int abort;
+  float xchg[2][128];             // per column half: a row's tile maximum, then its l
 };
 
+// Barrier of the two warps that share a TMEM lane quarter (ids 2-5, 64 threads); returns
+// the AND of `pred` over them, so both take the same branch after it.
+__device__ __forceinline__ bool pair_sync_and(int qd, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n"
+      " barrier.red.and.pred q, %2, 64, p;\n selp.u32 %0, 1, 0, q;\n}\n"
+      : "=r"(r)
+      : "r"((uint32_t)pred), "r"(2 + qd)
+      : "memory");
+  return r != 0;
+}
+
 // grid (chunks, halves, Hkv). Rows rho = h * Rp + r (h < G) of key head g; this CTA
-// takes rho in [128 * half, 128 * half + 128).
+// takes rho in [128 * half, 128 * half + 128). Pipeline per tile j of 128 tokens:
+//   TMA    K(j), V(j) into two-stage rings
+//   MMA    S(j) = Q K(j)^T into one of two TMEM buffers; O += P(j - 1) V(j - 1)
+//   rows   S(j) -> m, P(j) = bf16(2^(s - m)) into one of two shared-memory buffers
+// so the rows' exponentials of tile j overlap the tensor cores' P V of tile j - 1.
 __global__ void __launch_bounds__(kAtThreads, 1)
     k_fw_attn(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
               const AttnJob J) {
@@ -320,10 +425,10 @@ __global__ void __launch_bounds__(kAtThreads, 1)
   __shared__ AtBars S;
   unsigned char* sm = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  unsigned char* qs = sm;                    // A operand of S = Q K^T: 128 rows x 128 dims
-  unsigned char* ps = qs + kAtTileBytes;     // A operand of O += P V: 128 rows x 128 tokens
-  unsigned char* kr = ps + kAtTileBytes;     // 2 key stages
-  unsigned char* vr = kr + 2 * kAtTileBytes; // 2 value stages
+  unsigned char* qs = sm;                        // A operand of S = Q K^T: 128 rows x 128 dims
+  unsigned char* ps = qs + kAtTileBytes;         // 2 x A operand of O += P V: rows x tokens
+  unsigned char* kr = ps + 2 * kAtTileBytes;     // 2 key stages
+  unsigned char* vr = kr + 2 * kAtTileBytes;     // 2 value stages
   const int chunk = blockIdx.x, half = blockIdx.y, g = blockIdx.z;
   const int T = (J.n_tok + kAtTile - 1) / kAtTile;
   const int t0 = (int)((int64_t)T * chunk / J.chunks);
@@ -332,16 +437,16 @@ __global__ void __launch_bounds__(kAtThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   volatile int* abort = &S.abort;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < 2; ++s) {
-      mbar_init(smem_u32(&S.kfull[s]), 1);
-      mbar_init(smem_u32(&S.kempty[s]), 1);
-      mbar_init(smem_u32(&S.vfull[s]), 1);
-      mbar_init(smem_u32(&S.vempty[s]), 1);
-      mbar_init(smem_u32(&S.sfull[s]), 1);
-      mbar_init(smem_u32(&S.sempty[s]), 128);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(smem_u32(&S.kfull[b]), 1);
+      mbar_init(smem_u32(&S.kempty[b]), 1);
+      mbar_init(smem_u32(&S.vfull[b]), 1);
+      mbar_init(smem_u32(&S.vempty[b]), 1);
+      mbar_init(smem_u32(&S.sfull[b]), 1);
+      mbar_init(smem_u32(&S.sempty[b]), kAtEpi);
+      mbar_init(smem_u32(&S.pfull[b]), kAtEpi);
+      mbar_init(smem_u32(&S.pvdone[b]), 1);
     }
-    mbar_init(smem_u32(&S.pfull), 128);
-    mbar_init(smem_u32(&S.pvdone), 1);
     mbar_init(smem_u32(&S.q_ready), 1);
     mbar_init(smem_u32(&S.final_mma), 1);
     S.abort = 0;
@@ -359,6 +464,8 @@ __global__ void __launch_bounds__(kAtThreads, 1)
   const int y0 = t0 * kAtTile;
   if (warp == 0 && lane == 0) {
     // ---- TMA producer: K(j) and V(j) into their rings ----
+    tma_prefetch_map(&kmap);
+    tma_prefetch_map(&vmap);
     int klast[2] = {-1, -1}, vlast[2] = {-1, -1};
     for (int j = 0; j < n && !*abort; ++j) {
       const int st = j & 1;
@@ -378,15 +485,15 @@ __global__ void __launch_bounds__(kAtThreads, 1)
       tma_load_4d(dst + kAtTileBytes / 2, &vmap, bar, 64, y, g, J.layer);
       vlast[st] = j;
     }
-    for (int s = 0; s < 2; ++s) {
-      if (klast[s] >= 0) mbar_wait_bounded(smem_u32(&S.kfull[s]), (klast[s] >> 1) & 1);
-      if (vlast[s] >= 0) mbar_wait_bounded(smem_u32(&S.vfull[s]), (vlast[s] >> 1) & 1);
+    for (int b = 0; b < 2; ++b) {
+      if (klast[b] >= 0) mbar_wait_bounded(smem_u32(&S.kfull[b]), (klast[b] >> 1) & 1);
+      if (vlast[b] >= 0) mbar_wait_bounded(smem_u32(&S.vfull[b]), (vlast[b] >> 1) & 1);
     }
   } else if (warp == 1 && lane == 0) {
     // ---- MMA issuer: S(j) = Q K(j)^T, then O += P(j - 1) V(j - 1) ----
     const uint32_t id1 = idesc_bf16_f32(128, 128, false, false);
     const uint32_t id2 = idesc_bf16_f32(128, 128, false, true);
-    const uint32_t qa = smem_u32(qs), pa = smem_u32(ps);
+    const uint32_t qa = smem_u32(qs);
     if (fw_wait(smem_u32(&S.q_ready), 0, abort)) {
       for (int j = 0; j <= n; ++j) {
         if (j < n) {
@@ -407,10 +514,11 @@ __global__ void __launch_bounds__(kAtThreads, 1)
         }
         if (j >= 1) {
           const int jp = j - 1, st = jp & 1;
-          if (!fw_wait(smem_u32(&S.pfull), jp & 1, abort)) break;
+          if (!fw_wait(smem_u32(&S.pfull[st]), (jp >> 1) & 1, abort)) break;
           if (!fw_wait(smem_u32(&S.vfull[st]), (jp >> 1) & 1, abort)) break;
           tc_fence_after();
           const uint32_t va = smem_u32(vr + st * kAtTileBytes);
+          const uint32_t pa = smem_u32(ps + st * kAtTileBytes);
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
             // P: K-major, tokens in two 64-token halves; V: N = dims MN-major (two 64-dim
@@ -420,22 +528,23 @@ __global__ void __launch_bounds__(kAtThreads, 1)
                       sdesc_sw128(va + k * 2048, 16384, 1024), id2, (jp > 0 || k > 0) ? 1u : 0u);
           }
           umma_commit(smem_u32(&S.vempty[st]));
-          umma_commit(smem_u32(&S.pvdone));
+          umma_commit(smem_u32(&S.pvdone[st]));
         }
       }
     }
     umma_commit(smem_u32(&S.final_mma));
     mbar_wait_bounded(smem_u32(&S.final_mma), 0);
   } else if (warp >= 2) {
-    // ---- rows: one per thread (TMEM lane) ----
+    // ---- rows: two threads per row (TMEM lane), 64 columns each ----
     const int e = threadIdx.x - 64;
-    const int qd = warp & 3;
+    const int qd = warp & 3;                       // TMEM lane quarter
+    const int ch = (warp - 2) >> 2;                // column half: tokens / dims 64 ch .. + 63
     const int rl = qd * 32 + lane;                 // row within the CTA's 128
     const int rho = half * 128 + rl;
     const int hl = rho / J.Rp, r = rho - hl * J.Rp;
     const bool valid = hl < J.G && r < J.R;
     // question rows -> 128-byte swizzled K-major tile (two halves of 64 dims)
-    for (int x = e; x < 128 * 16; x += 128) {
+    for (int x = e; x < 128 * 16; x += kAtEpi) {
       const int row = x >> 4, c = x & 15;
       const int rr = half * 128 + row;
       const int h2 = rr / J.Rp, r2 = rr - h2 * J.Rp;
@@ -446,89 +555,122 @@ __global__ void __launch_bounds__(kAtThreads, 1)
       *reinterpret_cast<uint4*>(qs + (c >> 3) * 16384 + row * 128 + (((c & 7) ^ (row & 7)) << 4)) = v;
     }
     fence_proxy_async_smem();
-    fw_bar(1, 128);
+    fw_bar(1, kAtEpi);
     if (e == 0) mbar_arrive(smem_u32(&S.q_ready));
     const uint32_t la = tbase + ((uint32_t)(qd * 32) << 16);
-    unsigned char* prow = ps + rl * 128;
+    const uint32_t sc = (uint32_t)(64 * ch);       // this thread's columns within S and O
+    float* xm = S.xchg[ch];                        // the pair's exchange slots
+    float* xo = S.xchg[ch ^ 1];
     float m = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < n; ++j) {
       const int st = j & 1;
       ok = ok && fw_wait(smem_u32(&S.sfull[st]), (j >> 1) & 1, abort);
       ok = __all_sync(0xffffffffu, ok);
-      if (!ok) break;
-      tc_fence_after();
-      float s[128];
-      tmem_ld32x4(la + st * 128u, la + st * 128u + 32u, la + st * 128u + 64u, la + st * 128u + 96u,
-                  s);
-      tc_fence_before();
-      mbar_arrive(smem_u32(&S.sempty[st]));
-      const int nv = min(kAtTile, J.n_tok - (t0 + j) * kAtTile);   // valid tokens
+      float s[64];
+      if (ok) {
+        tc_fence_after();
+        tmem_ld32x2(la + st * 128u + sc, la + st * 128u + sc + 32u,
+                    *reinterpret_cast<float(*)[32]>(s), *reinterpret_cast<float(*)[32]>(s + 32));
+        tc_fence_before();
+        mbar_arrive(smem_u32(&S.sempty[st]));
+      }
+      const int nv = min(kAtTile, J.n_tok - (t0 + j) * kAtTile) - 64 * ch;   // valid columns
       float mt = -INFINITY;
+      if (ok) {
+        if (nv < 64) {
 #pragma unroll
-      for (int c = 0; c < 128; ++c) mt = fmaxf(mt, c < nv ? s[c] : -INFINITY);
-      mt *= kScoreScale;
+          for (int c = 0; c < 64; ++c)
+            if (c >= nv) s[c] = -INFINITY;
+        }
+        float a0 = s[0], a1 = s[1], a2 = s[2], a3 = s[3];
+#pragma unroll
+        for (int c = 4; c < 64; c += 4) {
+          a0 = fmaxf(a0, s[c]);
+          a1 = fmaxf(a1, s[c + 1]);
+          a2 = fmaxf(a2, s[c + 2]);
+          a3 = fmaxf(a3, s[c + 3]);
+        }
+        mt = fmaxf(fmaxf(a0, a1), fmaxf(a2, a3)) * kScoreScale;
+      }
+      // the pair agrees on the tile maximum and on going on (a barrier that also ANDs ok)
+      xm[rl] = mt;
+      ok = pair_sync_and(qd, ok);
+      if (!ok) break;
+      mt = fmaxf(mt, xo[rl]);
       const bool raise = mt > m + kAtLazy;
       const float m_new = raise ? mt : m;
-      // P = 2^(s - m_new) in bf16; l sums the rounded values the MMA uses
-      uint32_t pk[64];
-      float lt = 0.f;
+      // P = 2^(s - m_new) rounded to bf16 for the tensor cores; the scaling and l (the sum
+      // of the weights before rounding) on packed pairs
+      uint32_t pk[32];
+      const unsigned long long sc2 = f2pack(kScoreScale, kScoreScale);
+      const unsigned long long nm2 = f2pack(-m_new, -m_new);
+      unsigned long long acc0 = 0ull, acc1 = 0ull;
 #pragma unroll
-      for (int c = 0; c < 64; ++c) {
-        const float p0 = 2 * c < nv ? fast_exp2(fmaf(s[2 * c], kScoreScale, -m_new)) : 0.f;
-        const float p1 = 2 * c + 1 < nv ? fast_exp2(fmaf(s[2 * c + 1], kScoreScale, -m_new)) : 0.f;
+      for (int c = 0; c < 32; ++c) {
+        const unsigned long long x = ffma2(f2pack(s[2 * c], s[2 * c + 1]), sc2, nm2);
+        const float p0 = fast_exp2(f2lo(x)), p1 = fast_exp2(f2hi(x));
         const __nv_bfloat162 b2 = __floats2bfloat162_rn(p0, p1);
-        lt += __low2float(b2) + __high2float(b2);
         pk[c] = *reinterpret_cast<const uint32_t*>(&b2);
+        if (c & 1) acc1 = fadd2(acc1, f2pack(p0, p1));
+        else acc0 = fadd2(acc0, f2pack(p0, p1));
       }
-      // O and the P buffer are free once the previous tile's O += P V has completed
-      if (j >= 1) {
-        ok = fw_wait(smem_u32(&S.pvdone), (j - 1) & 1, abort);
-        ok = __all_sync(0xffffffffu, ok);
-        if (!ok) break;
+      const float lt0 = f2lo(acc0), lt1 = f2hi(acc0), lt2 = f2lo(acc1), lt3 = f2hi(acc1);
+      // the P buffer is free once O += P(j - 2) V(j - 2) has completed; a raised maximum
+      // rescales O (and l) once O += P(j - 1) V(j - 1) has completed
+      bool w_ok = true;
+      if (j >= 2) w_ok = fw_wait(smem_u32(&S.pvdone[st]), ((j - 2) >> 1) & 1, abort);
+      const bool any_raise = __any_sync(0xffffffffu, raise) && j >= 1;
+      if (any_raise) w_ok = w_ok && fw_wait(smem_u32(&S.pvdone[st ^ 1]), ((j - 1) >> 1) & 1, abort);
+      w_ok = __all_sync(0xffffffffu, w_ok);
+      ok = pair_sync_and(qd, w_ok);
+      if (!ok) break;
+      const float fac = raise ? fast_exp2(m - m_new) : 1.0f;
+      if (any_raise) {
         tc_fence_after();
-        const float fac = raise ? fast_exp2(m - m_new) : 1.0f;
-        if (__any_sync(0xffffffffu, raise)) {
 #pragma unroll 1
-          for (int c0 = 0; c0 < 128; c0 += 32) {
-            float o[32];
-            tmem_ld32(la + 256u + (uint32_t)c0, o);
+        for (int c0 = 0; c0 < 64; c0 += 32) {
+          float o[32];
+          tmem_ld32(la + 256u + sc + (uint32_t)c0, o);
 #pragma unroll
-            for (int c = 0; c < 32; ++c) o[c] *= fac;
-            tmem_st32(la + 256u + (uint32_t)c0, o);
-          }
+          for (int c = 0; c < 32; ++c) o[c] *= fac;
+          tmem_st32(la + 256u + sc + (uint32_t)c0, o);
         }
-        l *= fac;
       }
+      l = (j >= 1 ? l * fac : 0.f) + ((lt0 + lt1) + (lt2 + lt3));
       m = m_new;
-      l += lt;
-      // the P row: tokens 0-63 in half 0, 64-127 in half 1; 16-byte chunks swizzled
+      // this thread's 64 tokens of the P row: the half ch of the K-major operand
+      unsigned char* prow = ps + st * kAtTileBytes + ch * 16384 + rl * 128;
 #pragma unroll
-      for (int c = 0; c < 16; ++c) {
+      for (int c = 0; c < 8; ++c) {
         const uint4 w = make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
-        *reinterpret_cast<uint4*>(prow + (c >> 3) * 16384 + (((c & 7) ^ (rl & 7)) << 4)) = w;
+        *reinterpret_cast<uint4*>(prow + ((c ^ (rl & 7)) << 4)) = w;
       }
       fence_proxy_async_smem();
       tc_fence_before();
-      mbar_arrive(smem_u32(&S.pfull));
+      mbar_arrive(smem_u32(&S.pfull[st]));
     }
     if (ok && n > 0) {
-      ok = fw_wait(smem_u32(&S.pvdone), (n - 1) & 1, abort);
+      ok = fw_wait(smem_u32(&S.pvdone[(n - 1) & 1]), ((n - 1) >> 1) & 1, abort);
       ok = __all_sync(0xffffffffu, ok);
     }
+    // the row's l is the pair's sum
+    xm[rl] = l;
+    ok = pair_sync_and(qd, ok);
     tc_fence_after();
     const int64_t prow_out = ((int64_t)g * J.chunks + chunk) * (J.halves * 128) + rho;
     if (ok && !*abort) {
-      for (int c0 = 0; c0 < 128; c0 += 32) {
+      for (int c0 = 0; c0 < 64; c0 += 32) {
         float o[32];
-        tmem_ld32(la + 256u + (uint32_t)c0, o);
+        tmem_ld32(la + 256u + sc + (uint32_t)c0, o);
         if (valid && n > 0) {
-          float4* dst = reinterpret_cast<float4*>(J.opart + prow_out * kHeadDim + c0);
+          float4* dst = reinterpret_cast<float4*>(J.opart + prow_out * kHeadDim + sc + c0);
 #pragma unroll
           for (int c = 0; c < 8; ++c) dst[c] = make_float4(o[4 * c], o[4 * c + 1], o[4 * c + 2], o[4 * c + 3]);
         }
       }
-      if (valid) J.mlpart[prow_out] = n > 0 ? make_float2(m, l) : make_float2(-INFINITY, 0.f);
+      if (valid && ch == 0)
+        J.mlpart[prow_out] = n > 0 ? make_float2(m, l + xo[rl]) : make_float2(-INFINITY, 0.f);
     }
   }
   tc_fence_before();
@@ -549,8 +691,8 @@ struct AttnOutJob {
   const uint32_t* status;
 };
 
-// One warp per (row of Rp, head): the chunks in chunk order, then the question's own
-// rows 0..r; lane owns dims 4 lane .. 4 lane + 3.
+// One warp per (row of Rp, head): the chunks' (m, l, O) and the question's own rows
+// 0..r merged under their common maximum, in a fixed order; lane owns dims 4 lane .. +3.
 __global__ void __launch_bounds__(256) k_fw_attn_out(const AttnOutJob J) {
   const int wid = (blockIdx.x * 256 + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (wid >= J.Rp * J.Hq) return;
@@ -565,16 +707,12 @@ __global__ void __launch_bounds__(256) k_fw_attn_out(const AttnOutJob J) {
   const int g = h / J.G, hl = h - g * J.G;
   const int rho = hl * J.Rp + r;
   const int rows = J.halves * 128;
-  float M = -INFINITY;
-  for (int c = 0; c < J.chunks; ++c) {
-    const float2 ml = J.mlpart[((int64_t)g * J.chunks + c) * rows + rho];
-    if (ml.y > 0.f) M = fmaxf(M, ml.x);
-  }
-  // own rows: s_j = q_r . k_j in the log2 domain (dot products reduced in a fixed order)
+  // own rows' scores, lane jr < 32 (and jr + 32) holds row jr's (one dot per row, lanes
+  // summed in a fixed butterfly)
   const uint2 qv = *reinterpret_cast<const uint2*>(J.q + ((int64_t)r * J.Hq + h) * kHeadDim + 4 * lane);
   const float q0 = __uint_as_float(qv.x << 16), q1 = __uint_as_float(qv.x & 0xffff0000u);
   const float q2 = __uint_as_float(qv.y << 16), q3 = __uint_as_float(qv.y & 0xffff0000u);
-  float own[64];
+  float own0 = -INFINITY, own1 = -INFINITY;     // rows lane and lane + 32
   for (int jr = 0; jr <= r; ++jr) {
     const uint2 kv = *reinterpret_cast<const uint2*>(J.k + ((int64_t)jr * J.Hkv + g) * kHeadDim + 4 * lane);
     float d = q0 * __uint_as_float(kv.x << 16);
@@ -583,31 +721,63 @@ __global__ void __launch_bounds__(256) k_fw_attn_out(const AttnOutJob J) {
     d = fmaf(q3, __uint_as_float(kv.y & 0xffff0000u), d);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) d += __shfl_xor_sync(0xffffffffu, d, o);
-    own[jr] = d * kScoreScale;
-    M = fmaxf(M, own[jr]);
+    if (lane == (jr & 31)) {
+      if (jr < 32) own0 = d * kScoreScale;
+      else own1 = d * kScoreScale;
+    }
   }
+  // chunk statistics: lane c holds chunk c (and c + 32, ...)
+  float M = fmaxf(own0, own1);
+  for (int c = lane; c < J.chunks; c += 32) {
+    const float2 ml = J.mlpart[((int64_t)g * J.chunks + c) * rows + rho];
+    if (ml.y > 0.f) M = fmaxf(M, ml.x);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
   float L = 0.f;
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  for (int c = 0; c < J.chunks; ++c) {
+  int c = 0;
+  for (; c + 4 <= J.chunks; c += 4) {
+    float2 ml[4];
+    float4 ov[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int64_t pr = ((int64_t)g * J.chunks + c + u) * rows + rho;
+      ml[u] = J.mlpart[pr];
+      ov[u] = reinterpret_cast<const float4*>(J.opart + pr * kHeadDim)[lane];
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      if (!(ml[u].y > 0.f)) continue;
+      const float wgt = fast_exp2(ml[u].x - M);
+      L = fmaf(ml[u].y, wgt, L);
+      acc.x = fmaf(ov[u].x, wgt, acc.x);
+      acc.y = fmaf(ov[u].y, wgt, acc.y);
+      acc.z = fmaf(ov[u].z, wgt, acc.z);
+      acc.w = fmaf(ov[u].w, wgt, acc.w);
+    }
+  }
+  for (; c < J.chunks; ++c) {
     const int64_t pr = ((int64_t)g * J.chunks + c) * rows + rho;
     const float2 ml = J.mlpart[pr];
     if (!(ml.y > 0.f)) continue;
-    const float w = fast_exp2(ml.x - M);
-    L = fmaf(ml.y, w, L);
+    const float wgt = fast_exp2(ml.x - M);
     const float4 ov = reinterpret_cast<const float4*>(J.opart + pr * kHeadDim)[lane];
-    acc.x = fmaf(ov.x, w, acc.x);
-    acc.y = fmaf(ov.y, w, acc.y);
-    acc.z = fmaf(ov.z, w, acc.z);
-    acc.w = fmaf(ov.w, w, acc.w);
+    L = fmaf(ml.y, wgt, L);
+    acc.x = fmaf(ov.x, wgt, acc.x);
+    acc.y = fmaf(ov.y, wgt, acc.y);
+    acc.z = fmaf(ov.z, wgt, acc.z);
+    acc.w = fmaf(ov.w, wgt, acc.w);
   }
   for (int jr = 0; jr <= r; ++jr) {
-    const float w = fast_exp2(own[jr] - M);
-    L += w;
+    const float s = __shfl_sync(0xffffffffu, jr < 32 ? own0 : own1, jr & 31);
+    const float wgt = fast_exp2(s - M);
+    L += wgt;
     const uint2 vv = *reinterpret_cast<const uint2*>(J.v + ((int64_t)jr * J.Hkv + g) * kHeadDim + 4 * lane);
-    acc.x = fmaf(__uint_as_float(vv.x << 16), w, acc.x);
-    acc.y = fmaf(__uint_as_float(vv.x & 0xffff0000u), w, acc.y);
-    acc.z = fmaf(__uint_as_float(vv.y << 16), w, acc.z);
-    acc.w = fmaf(__uint_as_float(vv.y & 0xffff0000u), w, acc.w);
+    acc.x = fmaf(__uint_as_float(vv.x << 16), wgt, acc.x);
+    acc.y = fmaf(__uint_as_float(vv.x & 0xffff0000u), wgt, acc.y);
+    acc.z = fmaf(__uint_as_float(vv.y << 16), wgt, acc.z);
+    acc.w = fmaf(__uint_as_float(vv.y & 0xffff0000u), wgt, acc.w);
   }
   const float inv = 1.0f / L;
   reinterpret_cast<__nv_bfloat162*>(dst)[0] = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
@@ -645,8 +815,8 @@ struct Seg {
 };
 
 struct FwLayout {
-  size_t H, X, A, part, k, v, opart, ml, status, total;
-  int Rp, halves, chunks, sp_qkv, sp_o, sp_gu, sp_d;
+  size_t H, X, A, part, k, v, opart, ml, rope, ssq, ticket, total;
+  int Rp, halves, chunks, nchunks, sp_qkv, sp_o, sp_gu, sp_d;
 };
 
 FwLayout fw_layout(const FwShape& F) {
@@ -677,7 +847,10 @@ FwLayout fw_layout(const FwShape& F) {
   L.v = s.take<__nv_bfloat16>((size_t)F.R * F.Hkv * kHeadDim);
   L.opart = s.take<float>((size_t)F.Hkv * L.chunks * L.halves * 128 * kHeadDim);
   L.ml = s.take<float2>((size_t)F.Hkv * L.chunks * L.halves * 128);
-  L.status = s.take<uint32_t>(1);
+  L.rope = s.take<float2>((size_t)F.R * 64);
+  L.nchunks = (D + kNormCols - 1) / kNormCols;
+  L.ssq = s.take<float>((size_t)F.R * L.nchunks);
+  L.ticket = s.take<uint32_t>((size_t)F.R + 1);   // the row tickets, then the status word
   L.total = s.off;
   return L;
 }
@@ -729,11 +902,17 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
   __nv_bfloat16* vown = reinterpret_cast<__nv_bfloat16*>(ws + L.v);
   float* opart = reinterpret_cast<float*>(ws + L.opart);
   float2* ml = reinterpret_cast<float2*>(ws + L.ml);
-  uint32_t* status = A.status ? A.status : reinterpret_cast<uint32_t*>(ws + L.status);
+  float2* rope = reinterpret_cast<float2*>(ws + L.rope);
+  float* ssq = reinterpret_cast<float*>(ws + L.ssq);
+  unsigned int* ticket = reinterpret_cast<unsigned int*>(ws + L.ticket);
+  uint32_t* status = A.status ? A.status : reinterpret_cast<uint32_t*>(ticket + F.R);
   const int D = F.Hq * kHeadDim, G = F.Hq / F.Hkv;
   const int nqkv = (F.Hq + 2 * F.Hkv) * kHeadDim;
-  cudaError_t e = cudaMemsetAsync(status, 0, sizeof(uint32_t), st);
+  cudaError_t e = cudaMemsetAsync(ticket, 0, (size_t)(F.R + 1) * sizeof(uint32_t), st);
   if (e != cudaSuccess) return e;
+  if (A.status && (e = cudaMemsetAsync(status, 0, sizeof(uint32_t), st)) != cudaSuccess) return e;
+  k_fw_rope<<<F.R, 64, 0, st>>>(rope, F.pos0, F.theta);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
   // stored keys and values of every layer as [P][Hkv][n_tok][d] (the stored tokens of a
   // slab only, so the last tile's rows past them read zeros), tiles of 128 tokens
   CUtensorMap km, vm;
@@ -746,7 +925,7 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     e = encode_bf16_map(&vm, F.values, 4, dims, strides, box);
     if (e != cudaSuccess) return e;
-    e = ensure_smem((const void*)k_fw_attn, 6 * kAtTileBytes + 1024);
+    e = ensure_smem((const void*)k_fw_attn, kAtSmem);
     if (e != cudaSuccess) return e;
   }
   NormJob nj{};
@@ -755,6 +934,10 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
   nj.R = F.R;
   nj.Rp = L.Rp;
   nj.eps = F.eps;
+  nj.ssq = ssq;
+  nj.ticket = ticket;
+  nj.chunks = L.nchunks;
+  const dim3 ngrid(L.nchunks, L.Rp);
   for (int i = 0; i < F.P; ++i) {
     const FwLayerW& W = A.layers[i];
     __nv_bfloat16* q = static_cast<__nv_bfloat16*>(A.q_out) + (int64_t)i * F.R * F.Hq * kHeadDim;
@@ -765,7 +948,7 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
     nj.splits = L.sp_d;
     nj.w = static_cast<const __nv_bfloat16*>(W.ln1);
     nj.X = X;
-    k_fw_norm<<<L.Rp, 256, 0, st>>>(nj);
+    k_fw_norm<<<ngrid, 256, 0, st>>>(nj);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     if ((e = gemm(W.wqkv, nqkv, D, X, F.R, L.Rp, L.sp_qkv, part, status, st)) != cudaSuccess) return e;
     QkvJob qj;
@@ -776,8 +959,7 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
     qj.bias = static_cast<const __nv_bfloat16*>(W.bqkv);
     qj.Hq = F.Hq;
     qj.Hkv = F.Hkv;
-    qj.pos0 = F.pos0;
-    qj.theta = F.theta;
+    qj.rope = rope;
     qj.q = q;
     qj.k = kown;
     qj.v = vown;
@@ -799,7 +981,7 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
       aj.opart = opart;
       aj.mlpart = ml;
       aj.status = status;
-      k_fw_attn<<<dim3(L.chunks, L.halves, F.Hkv), kAtThreads, 6 * kAtTileBytes + 1024, st>>>(km, vm, aj);
+      k_fw_attn<<<dim3(L.chunks, L.halves, F.Hkv), kAtThreads, kAtSmem, st>>>(km, vm, aj);
       if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     AttnOutJob oj;
@@ -826,7 +1008,7 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
     nj.part = part;
     nj.splits = L.sp_o;
     nj.w = static_cast<const __nv_bfloat16*>(W.ln2);
-    k_fw_norm<<<L.Rp, 256, 0, st>>>(nj);
+    k_fw_norm<<<ngrid, 256, 0, st>>>(nj);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     if ((e = gemm(W.wgu, 2 * F.I, D, X, F.R, L.Rp, L.sp_gu, part, status, st)) != cudaSuccess) return e;
     SwigluJob sj;
@@ -845,7 +1027,7 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
   nj.part = part;
   nj.splits = L.sp_d;
   nj.w = nullptr;
-  k_fw_norm<<<L.Rp, 256, 0, st>>>(nj);
+  k_fw_norm<<<ngrid, 256, 0, st>>>(nj);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   if (A.h_out)
     return cudaMemcpyAsync(A.h_out, H, (size_t)F.R * D * sizeof(float), cudaMemcpyDeviceToDevice, st);

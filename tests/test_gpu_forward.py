@@ -11,11 +11,12 @@ sides still round differently (the oracle is fp64):
     accumulation over K = D terms errs by ~2^-24 sqrt(K) of that scale, 2^-18 leaves a
     margin, and eps stays a few percent of a bf16 step for q of order 1.
   * attention output o (Wo = identity and Wd = 0, so H_out - h_in = o exactly): the GPU
-    rounds the attention weights p to bf16 (relative error <= 2^-8) and normalises by their
-    rounded sum, which moves o by at most 2^-8 sum_j p_j |v_j - o| (the oracle's "spread");
-    a q or own k element at a rounding boundary moves a score by one bf16 step times a key
-    entry / sqrt(d) (< 2^-8 for these inputs), the same bound again; o is rounded to bf16
-    (half a step) on the GPU: |do| <= 2^-7 spread + step(o) / 2.
+    rounds the attention weights p to bf16 (relative error <= 2^-8) for the tensor cores
+    and normalises by the sum of the unrounded weights, which moves o by at most
+    2^-8 sum_j p_j |v_j| <= 2^-8 (spread + |o|), spread = sum_j p_j |v_j - o| (the
+    oracle's); a q or own k element at a rounding boundary moves a score by one bf16 step
+    times a key entry / sqrt(d) (< 2^-8 for these inputs), the same bound again; o is
+    rounded to bf16 (half a step) on the GPU: |do| <= 2^-7 (spread + |o|) + step(o) / 2.
   * MLP (Wo = 0, so H_mid = h_in and x2 = h_in / 2 exactly): H_out - h_in = a Wd^T with
     a = bf16(silu(g) u); an element of a whose oracle value lies within 1e-2 of a step of
     a rounding boundary may take the neighbouring value, so |dH_j| <= sum over those k of
@@ -176,7 +177,8 @@ def test_attention_and_q_of_one_layer(R, F, Tf):
                    theta=1e6, with_spread=True)
     n_q = _check_q(qb[0], ref["q_pre"], _q_scale(ref, _np_weights(layers)[0], w.n_q_heads))
     o_gpu = h - bf16_to_f64(hb)
-    tol = 2.0 ** -7 * ref["o_spread"] * 1.01 + 0.5 * _bf16_step(ref["o_pre"]) * 1.01 + 1e-7
+    tol = (2.0 ** -7 * (ref["o_spread"] + np.abs(ref["o_pre"])) * 1.01 +
+           0.5 * _bf16_step(ref["o_pre"]) * 1.01 + 1e-7)
     err = np.abs(o_gpu - ref["o_pre"])
     assert (err <= tol).all(), f"attention output off by {(err / tol).max():.2f} x its bound"
     print(f"q elements at a rounding boundary: {n_q}; o error / bound max {(err / tol).max():.3f}")
