@@ -107,15 +107,30 @@ __global__ void __launch_bounds__(kGmThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_release();
   const uint32_t tbase = S.taddr;
   if (warp == 0 && lane == 0) {
     tma_prefetch_map(&wmap);
     tma_prefetch_map(&xmap);
     int issued_last[kGmMaxStages];
     for (int s = 0; s < kGmMaxStages; ++s) issued_last[s] = -1;
-    for (int j = 0; j < n && !*abort; ++j) {
+    // the weights do not depend on the previous kernel: the first stages' weight tiles
+    // are requested before waiting for it, their rows of X after
+    const int pre = n < stages ? n : stages;
+    for (int j = 0; j < pre; ++j) {
+      const uint32_t bar = smem_u32(&S.full[j]);
+      mbar_expect_tx(bar, (uint32_t)stage_bytes);
+      tma_load_2d(smem_u32(sm + j * stage_bytes), &wmap, bar, (kb0 + j) * 64, m0);
+    }
+    pdl_wait();
+    for (int j = 0; j < pre; ++j) {
+      tma_load_2d(smem_u32(sm + j * stage_bytes) + kGmABytes, &xmap, smem_u32(&S.full[j]),
+                  (kb0 + j) * 64, 0);
+      issued_last[j] = j;
+    }
+    for (int j = pre; j < n && !*abort; ++j) {
       const int st = j % stages;
-      if (j >= stages && !fw_wait(smem_u32(&S.empty[st]), ((j / stages) - 1) & 1, abort)) break;
+      if (!fw_wait(smem_u32(&S.empty[st]), ((j / stages) - 1) & 1, abort)) break;
       const uint32_t bar = smem_u32(&S.full[st]);
       const uint32_t dst = smem_u32(sm + st * stage_bytes);
       mbar_expect_tx(bar, (uint32_t)stage_bytes);
@@ -192,6 +207,8 @@ constexpr int kNormCols = 512;   // columns per CTA (2 per thread)
 __global__ void __launch_bounds__(256) k_fw_norm(const NormJob J) {
   __shared__ float red[8];
   __shared__ int s_last;
+  pdl_wait();
+  pdl_release();
   const int r = blockIdx.y, c0 = blockIdx.x * kNormCols, t = threadIdx.x;
   const int D = J.D;
   const int x = c0 + 2 * t;                 // this thread's two columns (D is even)
@@ -263,6 +280,8 @@ __global__ void __launch_bounds__(256) k_fw_norm(const NormJob J) {
 // fp64, stored as fp32): [R][64] pairs.
 __global__ void __launch_bounds__(64) k_fw_rope(float2* tab, int64_t pos0, double theta) {
   const int r = blockIdx.x, j = threadIdx.x;
+  pdl_wait();     // (an earlier forward's kernels may still read the table)
+  pdl_release();
   const double inv = pow(theta, -2.0 * (double)j / (double)kHeadDim);
   double sd, cd;
   sincos((double)(pos0 + r) * inv, &sd, &cd);
@@ -283,6 +302,8 @@ struct QkvJob {
 // Grid (R, Hq + 2 Hkv); thread j < 64 owns the pair (j, j + 64) of one head.
 __global__ void __launch_bounds__(64) k_fw_qkv(const QkvJob J) {
   const int r = blockIdx.x, t = blockIdx.y, j = threadIdx.x;
+  pdl_wait();
+  pdl_release();
   const int n_out = (J.Hq + 2 * J.Hkv) * kHeadDim;
   const int f0 = t * kHeadDim + j, f1 = f0 + 64;
   float y0 = 0.f, y1 = 0.f;
@@ -334,6 +355,8 @@ struct SwigluJob {
 
 __global__ void __launch_bounds__(256) k_fw_swiglu(const SwigluJob J) {
   const int64_t x = (int64_t)blockIdx.x * 256 + threadIdx.x;
+  pdl_wait();
+  pdl_release();
   if (x >= (int64_t)J.Rp * J.I) return;
   const int r = (int)(x / J.I), f = (int)(x - (int64_t)r * J.I);
   float a = 0.f;
@@ -459,6 +482,7 @@ __global__ void __launch_bounds__(kAtThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_release();
   const uint32_t tbase = S.taddr;
   // tensor maps [P][Hkv][n_tok][d]: a tile past the stored tokens reads zeros
   const int y0 = t0 * kAtTile;
@@ -490,45 +514,69 @@ __global__ void __launch_bounds__(kAtThreads, 1)
       if (vlast[b] >= 0) mbar_wait_bounded(smem_u32(&S.vfull[b]), (vlast[b] >> 1) & 1);
     }
   } else if (warp == 1 && lane == 0) {
-    // ---- MMA issuer: S(j) = Q K(j)^T, then O += P(j - 1) V(j - 1) ----
+    // ---- MMA issuer, an event loop over two queues: S(j1) = Q K(j1)^T as soon as its
+    // keys are in and its TMEM buffer is read out, O += P(j2) V(j2) as soon as its weights
+    // are written (non-blocking tests, so neither queue holds back the other) ----
     const uint32_t id1 = idesc_bf16_f32(128, 128, false, false);
     const uint32_t id2 = idesc_bf16_f32(128, 128, false, true);
     const uint32_t qa = smem_u32(qs);
     if (fw_wait(smem_u32(&S.q_ready), 0, abort)) {
-      for (int j = 0; j <= n; ++j) {
-        if (j < n) {
-          const int st = j & 1;
-          if (!fw_wait(smem_u32(&S.kfull[st]), (j >> 1) & 1, abort)) break;
-          if (j >= 2 && !fw_wait(smem_u32(&S.sempty[st]), ((j >> 1) - 1) & 1, abort)) break;
-          tc_fence_after();
-          const uint32_t ka = smem_u32(kr + st * kAtTileBytes);
-          const uint32_t d = tbase + (uint32_t)st * 128u;
+      int j1 = 0, j2 = 0;
+      uint64_t t_idle = 0;
+      uint32_t idle = 0;
+      while (j2 < n) {
+        bool did = false;
+        if (j1 < n) {
+          const int st = j1 & 1;
+          bool ready = j1 < 2 || mbar_test_wait(smem_u32(&S.sempty[st]), ((j1 >> 1) - 1) & 1);
+          ready = ready && mbar_test_wait(smem_u32(&S.kfull[st]), (j1 >> 1) & 1);
+          if (ready) {
+            tc_fence_after();
+            const uint32_t ka = smem_u32(kr + st * kAtTileBytes);
+            const uint32_t d = tbase + (uint32_t)st * 128u;
 #pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            const uint32_t ko = (k >> 2) * 16384 + (k & 3) * 32;
-            umma_bf16(d, sdesc_sw128(qa + ko, 16, 1024), sdesc_sw128(ka + ko, 16, 1024), id1,
-                      k > 0 ? 1u : 0u);
+            for (int k = 0; k < 8; ++k) {
+              const uint32_t ko = (k >> 2) * 16384 + (k & 3) * 32;
+              umma_bf16(d, sdesc_sw128(qa + ko, 16, 1024), sdesc_sw128(ka + ko, 16, 1024), id1,
+                        k > 0 ? 1u : 0u);
+            }
+            umma_commit(smem_u32(&S.sfull[st]));
+            umma_commit(smem_u32(&S.kempty[st]));
+            ++j1;
+            did = true;
           }
-          umma_commit(smem_u32(&S.sfull[st]));
-          umma_commit(smem_u32(&S.kempty[st]));
         }
-        if (j >= 1) {
-          const int jp = j - 1, st = jp & 1;
-          if (!fw_wait(smem_u32(&S.pfull[st]), (jp >> 1) & 1, abort)) break;
-          if (!fw_wait(smem_u32(&S.vfull[st]), (jp >> 1) & 1, abort)) break;
-          tc_fence_after();
-          const uint32_t va = smem_u32(vr + st * kAtTileBytes);
-          const uint32_t pa = smem_u32(ps + st * kAtTileBytes);
+        if (j2 < j1) {
+          const int st = j2 & 1;
+          if (mbar_test_wait(smem_u32(&S.pfull[st]), (j2 >> 1) & 1) &&
+              mbar_test_wait(smem_u32(&S.vfull[st]), (j2 >> 1) & 1)) {
+            tc_fence_after();
+            const uint32_t va = smem_u32(vr + st * kAtTileBytes);
+            const uint32_t pa = smem_u32(ps + st * kAtTileBytes);
 #pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            // P: K-major, tokens in two 64-token halves; V: N = dims MN-major (two 64-dim
-            // blocks 16 KB apart), 16 tokens = 2048 bytes per K step
-            const uint32_t pk = (k >> 2) * 16384 + (k & 3) * 32;
-            umma_bf16(tbase + 256u, sdesc_sw128(pa + pk, 16, 1024),
-                      sdesc_sw128(va + k * 2048, 16384, 1024), id2, (jp > 0 || k > 0) ? 1u : 0u);
+            for (int k = 0; k < 8; ++k) {
+              // P: K-major, tokens in two 64-token halves; V: N = dims MN-major (two 64-dim
+              // blocks 16 KB apart), 16 tokens = 2048 bytes per K step
+              const uint32_t pk = (k >> 2) * 16384 + (k & 3) * 32;
+              umma_bf16(tbase + 256u, sdesc_sw128(pa + pk, 16, 1024),
+                        sdesc_sw128(va + k * 2048, 16384, 1024), id2, (j2 > 0 || k > 0) ? 1u : 0u);
+            }
+            umma_commit(smem_u32(&S.vempty[st]));
+            umma_commit(smem_u32(&S.pvdone[st]));
+            ++j2;
+            did = true;
           }
-          umma_commit(smem_u32(&S.vempty[st]));
-          umma_commit(smem_u32(&S.pvdone[st]));
+        }
+        if (did) {
+          idle = 0;
+        } else if (__nanosleep(32), (++idle & 255u) == 0u) {
+          // bounded: give up after ~1 s without progress, or when another role did
+          const uint64_t now = global_ns();
+          if (idle == 256u) t_idle = now;
+          if (*abort || now - t_idle > 1000000000ull || idle >= kDefaultWaitPolls) {
+            *abort = 1;
+            break;
+          }
         }
       }
     }
@@ -543,6 +591,8 @@ __global__ void __launch_bounds__(kAtThreads, 1)
     const int rho = half * 128 + rl;
     const int hl = rho / J.Rp, r = rho - hl * J.Rp;
     const bool valid = hl < J.G && r < J.R;
+    // (the keys and values stream in meanwhile: they do not depend on the previous kernel)
+    pdl_wait();
     // question rows -> 128-byte swizzled K-major tile (two halves of 64 dims)
     for (int x = e; x < 128 * 16; x += kAtEpi) {
       const int row = x >> 4, c = x & 15;
@@ -593,6 +643,11 @@ __global__ void __launch_bounds__(kAtThreads, 1)
         }
         mt = fmaxf(fmaxf(a0, a1), fmaxf(a2, a3)) * kScoreScale;
       }
+      // the P buffer is free once O += P(j - 2) V(j - 2) has completed
+      if (ok && j >= 2) {
+        ok = fw_wait(smem_u32(&S.pvdone[st]), ((j - 2) >> 1) & 1, abort);
+        ok = __all_sync(0xffffffffu, ok);
+      }
       // the pair agrees on the tile maximum and on going on (a barrier that also ANDs ok)
       xm[rl] = mt;
       ok = pair_sync_and(qd, ok);
@@ -616,15 +671,15 @@ __global__ void __launch_bounds__(kAtThreads, 1)
         else acc0 = fadd2(acc0, f2pack(p0, p1));
       }
       const float lt0 = f2lo(acc0), lt1 = f2hi(acc0), lt2 = f2lo(acc1), lt3 = f2hi(acc1);
-      // the P buffer is free once O += P(j - 2) V(j - 2) has completed; a raised maximum
-      // rescales O (and l) once O += P(j - 1) V(j - 1) has completed
-      bool w_ok = true;
-      if (j >= 2) w_ok = fw_wait(smem_u32(&S.pvdone[st]), ((j - 2) >> 1) & 1, abort);
+      // a raised maximum rescales O (and l) once O += P(j - 1) V(j - 1) has completed (the
+      // two warps of a pair hold the same rows, so both take this branch or neither)
       const bool any_raise = __any_sync(0xffffffffu, raise) && j >= 1;
-      if (any_raise) w_ok = w_ok && fw_wait(smem_u32(&S.pvdone[st ^ 1]), ((j - 1) >> 1) & 1, abort);
-      w_ok = __all_sync(0xffffffffu, w_ok);
-      ok = pair_sync_and(qd, w_ok);
-      if (!ok) break;
+      if (any_raise) {
+        bool w_ok = fw_wait(smem_u32(&S.pvdone[st ^ 1]), ((j - 1) >> 1) & 1, abort);
+        w_ok = __all_sync(0xffffffffu, w_ok);
+        ok = pair_sync_and(qd, w_ok);
+        if (!ok) break;
+      }
       const float fac = raise ? fast_exp2(m - m_new) : 1.0f;
       if (any_raise) {
         tc_fence_after();
@@ -695,6 +750,8 @@ struct AttnOutJob {
 // 0..r merged under their common maximum, in a fixed order; lane owns dims 4 lane .. +3.
 __global__ void __launch_bounds__(256) k_fw_attn_out(const AttnOutJob J) {
   const int wid = (blockIdx.x * 256 + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  pdl_wait();
+  pdl_release();
   if (wid >= J.Rp * J.Hq) return;
   const int r = wid / J.Hq, h = wid - r * J.Hq;
   __nv_bfloat16* dst = J.o + (int64_t)r * J.Hq * kHeadDim + h * kHeadDim + 4 * lane;
@@ -878,8 +935,7 @@ cudaError_t gemm(const void* W, int n_out, int K, const __nv_bfloat16* X, int R,
   const int smem = J.stages * (kGmABytes + Rp * 128) + 1024;
   e = ensure_smem((const void*)k_fw_gemm, smem);
   if (e != cudaSuccess) return e;
-  k_fw_gemm<<<dim3(n_out / 128, splits), kGmThreads, smem, st>>>(wm, xm, J);
-  return cudaGetLastError();
+  return launch_pdl(k_fw_gemm, dim3(n_out / 128, splits), dim3(kGmThreads), smem, st, wm, xm, J);
 }
 
 }  // namespace
@@ -911,8 +967,7 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
   cudaError_t e = cudaMemsetAsync(ticket, 0, (size_t)(F.R + 1) * sizeof(uint32_t), st);
   if (e != cudaSuccess) return e;
   if (A.status && (e = cudaMemsetAsync(status, 0, sizeof(uint32_t), st)) != cudaSuccess) return e;
-  k_fw_rope<<<F.R, 64, 0, st>>>(rope, F.pos0, F.theta);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if ((e = launch_pdl(k_fw_rope, dim3(F.R), dim3(64), 0, st, rope, F.pos0, F.theta)) != cudaSuccess) return e;
   // stored keys and values of every layer as [P][Hkv][n_tok][d] (the stored tokens of a
   // slab only, so the last tile's rows past them read zeros), tiles of 128 tokens
   CUtensorMap km, vm;
@@ -948,8 +1003,7 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
     nj.splits = L.sp_d;
     nj.w = static_cast<const __nv_bfloat16*>(W.ln1);
     nj.X = X;
-    k_fw_norm<<<ngrid, 256, 0, st>>>(nj);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = launch_pdl(k_fw_norm, ngrid, dim3(256), 0, st, nj)) != cudaSuccess) return e;
     if ((e = gemm(W.wqkv, nqkv, D, X, F.R, L.Rp, L.sp_qkv, part, status, st)) != cudaSuccess) return e;
     QkvJob qj;
     qj.part = part;
@@ -963,8 +1017,7 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
     qj.q = q;
     qj.k = kown;
     qj.v = vown;
-    k_fw_qkv<<<dim3(F.R, F.Hq + 2 * F.Hkv), 64, 0, st>>>(qj);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = launch_pdl(k_fw_qkv, dim3(F.R, F.Hq + 2 * F.Hkv), dim3(64), 0, st, qj)) != cudaSuccess) return e;
     if (F.n_tok > 0) {
       AttnJob aj;
       aj.layer = i;
@@ -981,8 +1034,9 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
       aj.opart = opart;
       aj.mlpart = ml;
       aj.status = status;
-      k_fw_attn<<<dim3(L.chunks, L.halves, F.Hkv), kAtThreads, kAtSmem, st>>>(km, vm, aj);
-      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+      if ((e = launch_pdl(k_fw_attn, dim3(L.chunks, L.halves, F.Hkv), dim3(kAtThreads), kAtSmem, st,
+                          km, vm, aj)) != cudaSuccess)
+        return e;
     }
     AttnOutJob oj;
     oj.Hq = F.Hq;
@@ -1000,16 +1054,15 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
     oj.o = X;
     oj.status = status;
     const int warps = L.Rp * F.Hq;
-    k_fw_attn_out<<<(warps * 32 + 255) / 256, 256, 0, st>>>(oj);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = launch_pdl(k_fw_attn_out, dim3((warps * 32 + 255) / 256), dim3(256), 0, st, oj)) != cudaSuccess)
+      return e;
     if ((e = gemm(W.wo, D, D, X, F.R, L.Rp, L.sp_o, part, status, st)) != cudaSuccess) return e;
     // H += o Wo^T; X = bf16(RMSNorm(H) * ln2)
     nj.h_in = nullptr;
     nj.part = part;
     nj.splits = L.sp_o;
     nj.w = static_cast<const __nv_bfloat16*>(W.ln2);
-    k_fw_norm<<<ngrid, 256, 0, st>>>(nj);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = launch_pdl(k_fw_norm, ngrid, dim3(256), 0, st, nj)) != cudaSuccess) return e;
     if ((e = gemm(W.wgu, 2 * F.I, D, X, F.R, L.Rp, L.sp_gu, part, status, st)) != cudaSuccess) return e;
     SwigluJob sj;
     sj.part = part;
@@ -1018,8 +1071,8 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
     sj.R = F.R;
     sj.I = F.I;
     sj.A = Ab;
-    k_fw_swiglu<<<(int)(((int64_t)L.Rp * F.I + 255) / 256), 256, 0, st>>>(sj);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = launch_pdl(k_fw_swiglu, dim3((unsigned)(((int64_t)L.Rp * F.I + 255) / 256)), dim3(256), 0, st, sj)) != cudaSuccess)
+      return e;
     if ((e = gemm(W.wd, D, F.I, Ab, F.R, L.Rp, L.sp_d, part, status, st)) != cudaSuccess) return e;
   }
   // H += the last down projection
@@ -1027,8 +1080,7 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
   nj.part = part;
   nj.splits = L.sp_d;
   nj.w = nullptr;
-  k_fw_norm<<<ngrid, 256, 0, st>>>(nj);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if ((e = launch_pdl(k_fw_norm, ngrid, dim3(256), 0, st, nj)) != cudaSuccess) return e;
   if (A.h_out)
     return cudaMemcpyAsync(A.h_out, H, (size_t)F.R * D * sizeof(float), cudaMemcpyDeviceToDevice, st);
   return cudaSuccess;
