@@ -331,6 +331,7 @@ def run_ours(args):
                       n_planted=max(1, w.n_planted * args.frames // w.n_frames))
     n_streams = w.n_streams
     clusters = w.window_frames > 0
+    fwd_I = int(w.extra.get("intermediate", 0))   # the question's forward (Eq. 10) too
     idxs, qs = [], []
     keys_cpu = q_cpu = None
     compress_ms = compress_all = None
@@ -339,11 +340,13 @@ def run_ours(args):
         idx = ss.Index(w.n_layers, w.n_q_heads, w.n_kv_heads, w.tokens_per_frame, w.n_frames,
                        frames_per_unit=w.frames_per_unit, device=dev)
         idx.append(data["keys"])
+        if fwd_I:
+            idx.append_values(synth.make_values(w, device=dev, seed=data["seed"]))
         if clusters:
             compress_ms, compress_all = time_compress(ss, w, data["keys"], dev)
             idx.compress(w.window_frames, n_centroids=w.n_centroids, iters=w.kmeans_iters)
         if st == 0:
-            if rank == 0 and not args.no_cpu_baseline:
+            if rank == 0 and not args.no_cpu_baseline and not fwd_I:
                 frames = min(args.cpu_frames, w.n_frames)
                 keys_cpu = data["keys"][:, :, : frames * w.tokens_per_frame].cpu()
             q_cpu = data["q"].cpu()
@@ -375,7 +378,30 @@ def run_ours(args):
     for ev in k_begin + k_end:
         ev.record(stream)  # create the events before handing them to the library
 
+    fw = None
+    if fwd_I:
+        # the question's forward through the shallow layers produces the query rows the
+        # retrieval scores (one stream per GPU)
+        fw_layers = synth.make_forward_weights(w, fwd_I, device=dev)
+        fw_h = synth.make_question_rows(w, device=dev)
+        fw_p = ss.ForwardParams(fwd_I)
+        fw_q = torch.empty_like(qs[0])
+        fw_hout = torch.empty(w.n_rows, w.n_q_heads * 128, dtype=torch.float32, device=dev)
+        fw_ws = torch.empty(idxs[0].forward_workspace_bytes(w.n_rows, fw_p), dtype=torch.uint8,
+                            device=dev)
+        fw_status = torch.zeros(1, dtype=torch.int32, device=dev)
+        fw_bytes = (sum(t.numel() * 2 for L in fw_layers for t in L.values() if t is not None) +
+                    2 * w.key_bytes)
+
+        def forward():
+            idxs[0].forward(fw_layers, fw_h, fw_p, q_out=fw_q, h_out=fw_hout, workspace=fw_ws,
+                            status=fw_status)
+        qs = [fw_q]
+        fw = {"bytes": fw_bytes, "ms": []}
+
     def step(tr=None):
+        if fw is not None:
+            forward()
         ss.retrieve_batched(idxs, qs, p, outs=outs, workspace=ws, trace=tr)
 
     clocks = ClockSampler(local)
@@ -403,6 +429,18 @@ def run_ours(args):
         s_end[i].record(stream)
     for j in range(n_traced, n_traced + n_kern):
         step((k_begin[j], k_end[j]))
+    if fw is not None:
+        # the forward alone, bracketed on each of n_kern calls
+        f_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                for _ in range(n_kern)]
+        for a, b in f_ev:
+            a.record(stream)
+            forward()
+            b.record(stream)
+        torch.cuda.synchronize(dev)
+        fw["ms"] = [a.elapsed_time(b) for a, b in f_ev]
+        if int(fw_status.item()) != 0:
+            raise RuntimeError(f"forward status {int(fw_status.item())}")
     torch.cuda.synchronize(dev)
     clk = clocks.stop(wall0, wall1)
     for o in outs:
@@ -417,7 +455,7 @@ def run_ours(args):
     # end to end through the C ABI's host entry point: the question's rows in pinned host
     # memory, the selection back in host memory, both copies inside the timed region
     e2e = None
-    if not args.no_e2e and n_streams == 1:
+    if not args.no_e2e and n_streams == 1 and fw is None:
         idx = idxs[0]
         q_pin = q_cpu.pin_memory()
         call = host_call(ss, idx, q_pin, p, ws, stream)
@@ -463,7 +501,15 @@ def run_ours(args):
         kernel = "k_score"
         launches = 7   # k_sample, k_score, k_select, k_mass, k_pool, k_gram, k_maxmin
     achieved = alg_bytes / k1_avg_s / 1e9
-    traffic = recorded_traffic(w) if not args.frames and n_streams == 1 else None
+    if fw is not None:
+        # the forward dominates the step: every layer's weights and stored keys and values
+        # read once per question
+        k1_avg_s = statistics.mean(fw["ms"]) / 1e3
+        alg_bytes = fw["bytes"]
+        kernel = "question forward (k_fw_norm, k_fw_gemm, k_fw_qkv, k_fw_attn, k_fw_attn_out, k_fw_swiglu)"
+        launches += 2 + 10 * w.n_layers   # RoPE table, final residual, 10 per layer
+        achieved = alg_bytes / k1_avg_s / 1e9
+    traffic = recorded_traffic(w) if not args.frames and n_streams == 1 and fw is None else None
     cpu = None
     if keys_cpu is not None:
         cpu = cpu_baseline(w, keys_cpu, q_cpu, keys_cpu.shape[2] // w.tokens_per_frame)
@@ -472,6 +518,10 @@ def run_ours(args):
             f"R {w.n_rows}, k {w.k}, budget {w.budget}, pool {w.pool_mult * w.budget}")
     if n_streams > 1:
         desc += f", {n_streams} streams per GPU in one batched call"
+    if fw is not None:
+        desc += (f", question forward through {w.n_layers} synthetic decoder layers (hidden "
+                 f"{w.n_q_heads * 128}, MLP {fwd_I}) attending to the stored keys and values, "
+                 f"then retrieval on its query rows")
     if clusters:
         desc += (f", windows of {w.window_frames} frames compressed to {w.n_centroids} "
                  f"centroids ({w.kmeans_iters} Lloyd rounds), retrieval over centroids")
@@ -479,6 +529,10 @@ def run_ours(args):
               "l2": f"inputs larger than L2 ({w.key_bytes * n_streams / 1e9:.2f} GB index vs "
                     f"129 MB L2), no flush",
               "parallelism": f"replicas x{world} (independent streams per GPU)"}
+    if fw is not None:
+        config["forward_ms"] = statistics.mean(fw["ms"])
+        config["forward_bytes"] = fw["bytes"]
+        config["index_bytes"] = 2 * w.key_bytes
     if clusters:
         config["compress_ms"] = compress_ms
         config["compress_ms_all"] = compress_all
