@@ -709,7 +709,11 @@ SS_EXPORT ss_status ss_question_forward(ss_index* ix, const ss_layer_weights* la
   A.status = status;
   A.workspace = workspace;
   SS_CUDA(cudaSetDevice(ix->device));
-  SS_CUDA(launch_forward(F, A, static_cast<cudaStream_t>(stream)));
+  const cudaError_t e = launch_forward(F, A, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) {
+    cudaGetLastError();   // a failed launch must not surface again in later calls
+    return fail(SS_ERR_CUDA, "question forward: %s", cudaGetErrorString(e));
+  }
   return SS_OK;
 }
 
