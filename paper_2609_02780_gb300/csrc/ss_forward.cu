@@ -27,6 +27,7 @@
 #include "ss_internal.cuh"
 #include "ss_device.cuh"
 #include "ss_tc.cuh"
+#include "ss_pack.cuh"
 
 #include <algorithm>
 
@@ -382,27 +383,6 @@ constexpr int kAtTileBytes = kAtTile * kHeadDim * 2;   // 32 KB
 constexpr int kAtSmem = 7 * kAtTileBytes + 1024;       // Q, 2 P, 2 K, 2 V stages
 constexpr float kAtLazy = 8.0f;            // raise the running max only past this margin
 
-// Packed fp32 pairs (the .f32x2 arithmetic of sm_100 and later): one instruction for two
-// lanes of a row's scores.
-__device__ __forceinline__ unsigned long long f2pack(float a, float b) {
-  return (unsigned long long)__float_as_uint(a) | ((unsigned long long)__float_as_uint(b) << 32);
-}
-__device__ __forceinline__ float f2lo(unsigned long long v) { return __uint_as_float((uint32_t)v); }
-__device__ __forceinline__ float f2hi(unsigned long long v) {
-  return __uint_as_float((uint32_t)(v >> 32));
-}
-__device__ __forceinline__ unsigned long long ffma2(unsigned long long a, unsigned long long b,
-                                                    unsigned long long c) {
-  unsigned long long d;
-  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
-  return d;
-}
-__device__ __forceinline__ unsigned long long fadd2(unsigned long long a, unsigned long long b) {
-  unsigned long long d;
-  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
-}
-
 struct AttnJob {
   int layer;
   int Hq, Hkv, G, R, Rp, GRp, halves;
@@ -633,15 +613,13 @@ __global__ void __launch_bounds__(kAtThreads, 1)
           for (int c = 0; c < 64; ++c)
             if (c >= nv) s[c] = -INFINITY;
         }
-        float a0 = s[0], a1 = s[1], a2 = s[2], a3 = s[3];
+        float a0 = -INFINITY, a1 = -INFINITY;
 #pragma unroll
-        for (int c = 4; c < 64; c += 4) {
-          a0 = fmaxf(a0, s[c]);
-          a1 = fmaxf(a1, s[c + 1]);
-          a2 = fmaxf(a2, s[c + 2]);
-          a3 = fmaxf(a3, s[c + 3]);
+        for (int c = 0; c < 64; c += 4) {
+          a0 = fmax3(a0, s[c], s[c + 1]);
+          a1 = fmax3(a1, s[c + 2], s[c + 3]);
         }
-        mt = fmaxf(fmaxf(a0, a1), fmaxf(a2, a3)) * kScoreScale;
+        mt = fmaxf(a0, a1) * kScoreScale;
       }
       // the P buffer is free once O += P(j - 2) V(j - 2) has completed
       if (ok && j >= 2) {

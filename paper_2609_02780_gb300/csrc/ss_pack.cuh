@@ -1,0 +1,37 @@
+// Packed arithmetic of sm_100 and later used by the exponential-heavy epilogues: fp32
+// pairs (.f32x2: one instruction for two lanes' values) and the three-operand max.
+#pragma once
+
+#include <stdint.h>
+
+namespace ss {
+
+// Packed fp32 pairs (the .f32x2 arithmetic of sm_100 and later): one instruction for two
+// lanes of a row's scores.
+__device__ __forceinline__ unsigned long long f2pack(float a, float b) {
+  return (unsigned long long)__float_as_uint(a) | ((unsigned long long)__float_as_uint(b) << 32);
+}
+__device__ __forceinline__ float f2lo(unsigned long long v) { return __uint_as_float((uint32_t)v); }
+__device__ __forceinline__ float f2hi(unsigned long long v) {
+  return __uint_as_float((uint32_t)(v >> 32));
+}
+__device__ __forceinline__ unsigned long long ffma2(unsigned long long a, unsigned long long b,
+                                                    unsigned long long c) {
+  unsigned long long d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ unsigned long long fadd2(unsigned long long a, unsigned long long b) {
+  unsigned long long d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
+// max(a, b, c) in one instruction (three-operand max of sm_100 and later).
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+}  // namespace ss

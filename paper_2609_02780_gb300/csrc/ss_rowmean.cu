@@ -20,6 +20,7 @@
 #include "ss_internal.cuh"
 #include "ss_device.cuh"
 #include "ss_tc.cuh"
+#include "ss_pack.cuh"
 
 namespace ss {
 
@@ -231,8 +232,13 @@ __global__ void __launch_bounds__(64 + 128 * NMB, 1)
           // products and scaled once)
           float mt = -INFINITY;
           if (nv == kRmTile) {
+            float a0 = -INFINITY, a1 = -INFINITY;
 #pragma unroll
-            for (int c = 0; c < 32; ++c) mt = fmaxf(mt, fmaxf(v0[c], v1[c]));
+            for (int c = 0; c < 32; c += 2) {
+              a0 = fmax3(a0, v0[c], v0[c + 1]);
+              a1 = fmax3(a1, v1[c], v1[c + 1]);
+            }
+            mt = fmaxf(a0, a1);
           } else {
 #pragma unroll
             for (int c = 0; c < 32; ++c) {
@@ -247,11 +253,19 @@ __global__ void __launch_bounds__(64 + 128 * NMB, 1)
           }
           float acc0 = 0.f, acc1 = 0.f;
           if (nv == kRmTile) {
+            // the scaling and the sums on packed pairs (columns c and 32 + c)
+            const unsigned long long sc2 = f2pack(kScoreScale, kScoreScale);
+            const unsigned long long nm2 = f2pack(-m, -m);
+            unsigned long long p0 = 0ull, p1 = 0ull;
 #pragma unroll
             for (int c = 0; c < 32; ++c) {
-              acc0 += fast_exp2(fmaf(v0[c], kScoreScale, -m));
-              acc1 += fast_exp2(fmaf(v1[c], kScoreScale, -m));
+              const unsigned long long x = ffma2(f2pack(v0[c], v1[c]), sc2, nm2);
+              const unsigned long long e = f2pack(fast_exp2(f2lo(x)), fast_exp2(f2hi(x)));
+              if (c & 1) p1 = fadd2(p1, e);
+              else p0 = fadd2(p0, e);
             }
+            acc0 = f2lo(p0) + f2lo(p1);
+            acc1 = f2hi(p0) + f2hi(p1);
           } else {
 #pragma unroll
             for (int c = 0; c < 32; ++c) {
@@ -363,7 +377,7 @@ __global__ void __launch_bounds__(64 + kRmEpi2, 1)
     for (int x = e; x < GRp; x += kRmEpi2) {
       const int hr = x / J.Rp, rr = x - hr * J.Rp;
       // rows past R get an offset that makes their terms 0
-      st[x] = (hr < P.G && rr < P.R) ? J.stat[(int64_t)slab * GRp + x].x : INFINITY;
+      st[x] = (hr < P.G && rr < P.R) ? -J.stat[(int64_t)slab * GRp + x].x : -INFINITY;
     }
     rm_bar(kRmEpi2);
     pdl_release();
@@ -386,15 +400,20 @@ __global__ void __launch_bounds__(64 + kRmEpi2, 1)
           float a = 0.f, a2 = 0.f;
           // a head's rows in one load and one wait where they fit 32 or 64 columns; the
           // offsets four at a time (padding rows add 2^-inf = 0)
+          // (the offsets are stored negated: s * scale - offset is one packed fma)
+          const unsigned long long sc2 = f2pack(kScoreScale, kScoreScale);
           auto add = [&](const float (&v)[32], int r0) {
+            unsigned long long p0 = 0ull, p1 = 0ull;
 #pragma unroll
             for (int t = 0; t < 32; t += 4) {
               const float4 o = *reinterpret_cast<const float4*>(sh + r0 + t);
-              a += fast_exp2(fmaf(v[t], kScoreScale, -o.x));
-              a2 += fast_exp2(fmaf(v[t + 1], kScoreScale, -o.y));
-              a += fast_exp2(fmaf(v[t + 2], kScoreScale, -o.z));
-              a2 += fast_exp2(fmaf(v[t + 3], kScoreScale, -o.w));
+              const unsigned long long x0 = ffma2(f2pack(v[t], v[t + 1]), sc2, f2pack(o.x, o.y));
+              const unsigned long long x1 = ffma2(f2pack(v[t + 2], v[t + 3]), sc2, f2pack(o.z, o.w));
+              p0 = fadd2(p0, f2pack(fast_exp2(f2lo(x0)), fast_exp2(f2hi(x0))));
+              p1 = fadd2(p1, f2pack(fast_exp2(f2lo(x1)), fast_exp2(f2hi(x1))));
             }
+            a += f2lo(p0) + f2lo(p1);
+            a2 += f2hi(p0) + f2hi(p1);
           };
           if (Rp == 32) {
             float v[32];
@@ -410,7 +429,7 @@ __global__ void __launch_bounds__(64 + kRmEpi2, 1)
               float v[16];
               tmem_ld16(col + (uint32_t)r0, v);
 #pragma unroll
-              for (int t = 0; t < 16; ++t) a += fast_exp2(fmaf(v[t], kScoreScale, -sh[r0 + t]));
+              for (int t = 0; t < 16; ++t) a += fast_exp2(fmaf(v[t], kScoreScale, sh[r0 + t]));
             }
           }
           if (tok < n_tok)
