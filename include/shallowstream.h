@@ -321,6 +321,23 @@ ss_status ss_question_forward(ss_index* index, const ss_layer_weights* layers,
                               int32_t n_rows, void* q_out, float* h_out, uint32_t* status,
                               void* workspace, size_t workspace_bytes, void* stream);
 
+/* The index's shape (as given to ss_index_create). Host-only. */
+ss_status ss_index_get_config(const ss_index* index, ss_index_config* config);
+
+/* Checkpoint of an index: writes its host metadata and every device array (keys, values,
+ * descriptors, compressed windows, unit clusters, at their full capacity) to the host file
+ * `path`, through a page-locked staging buffer on `stream` (the call returns when the file
+ * is written). The file is for this library version and a machine of the same byte order.
+ * Errors: INVALID_ARG (NULL, the file cannot be written), ALLOC, CUDA. */
+ss_status ss_index_save(const ss_index* index, const char* path, void* stream);
+
+/* Recreates an index from a file of ss_index_save on the current device, its device memory
+ * from `alloc` (NULL: cudaMalloc); the loaded index behaves as the saved one (appends,
+ * compression, retrieval continue from its state). Errors: INVALID_ARG (not such a file,
+ * truncated or inconsistent), ALLOC (nothing is kept), CUDA. */
+ss_status ss_index_load(const char* path, const ss_allocator* alloc, void* stream,
+                        ss_index** out);
+
 /* k-means compression of already appended frames (the cluster-compressed variant;
  * closest paper text Sec. 4.1 Eq. 5-7). For every window of `window_frames` frames in
  * [first_frame, first_frame + n_frames) and every (layer, key head): X = the window's

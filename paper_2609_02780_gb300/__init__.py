@@ -163,6 +163,39 @@ class Index:
                                        C.c_void_p(_stream_ptr(self.device)), C.byref(h)))
         self._h = h
 
+    @classmethod
+    def load(cls, path: str, device=None) -> "Index":
+        """ss_index_load: an index recreated from a checkpoint file of save()."""
+        lib = _lib()
+        self = cls.__new__(cls)
+        d = torch.device(device) if device is not None else torch.device("cuda")
+        self.device = d if d.index is not None else torch.device("cuda", torch.cuda.current_device())
+        self._blocks = {}
+        self._alloc_cb = _abi.ALLOC_FN(self._alloc)
+        self._free_cb = _abi.FREE_FN(self._free)
+        self._allocator = _abi.Allocator(self._alloc_cb, self._free_cb, None)
+        self._ws = None
+        self._host_calls = {}
+        self._h = None
+        h = C.c_void_p()
+        with torch.cuda.device(self.device):
+            _check(lib.ss_index_load(str(path).encode(), C.byref(self._allocator),
+                                     C.c_void_p(_stream_ptr(self.device)), C.byref(h)))
+        self._h = h
+        cfg = _abi.IndexConfig()
+        _check(lib.ss_index_get_config(h, C.byref(cfg)))
+        self.n_layers, self.n_q_heads, self.n_kv_heads = cfg.n_layers, cfg.n_q_heads, cfg.n_kv_heads
+        self.tokens_per_frame, self.frames_per_unit = cfg.tokens_per_frame, cfg.frames_per_unit
+        self.max_frames = cfg.max_frames
+        self.unit_capacity = cfg.max_frames // cfg.frames_per_unit
+        return self
+
+    def save(self, path: str) -> None:
+        """ss_index_save: writes a checkpoint of the index to `path` (synchronous)."""
+        with torch.cuda.device(self.device):
+            _check(_lib().ss_index_save(self.handle, str(path).encode(),
+                                        C.c_void_p(_stream_ptr(self.device))))
+
     # allocator callbacks: device memory comes from torch's caching allocator
     def _alloc(self, nbytes, stream, ctx):
         try:

@@ -130,6 +130,10 @@ SIGNATURES = {
                                               C.POINTER(C.c_int64)]),
     "ss_select_clusters": (c_status, [C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_int32,
                                       C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
+    "ss_index_get_config": (c_status, [C.c_void_p, C.POINTER(IndexConfig)]),
+    "ss_index_save": (c_status, [C.c_void_p, C.c_char_p, C.c_void_p]),
+    "ss_index_load": (c_status, [C.c_char_p, C.POINTER(Allocator), C.c_void_p,
+                                 C.POINTER(C.c_void_p)]),
     "ss_index_append_values": (c_status, [C.c_void_p, C.c_void_p, C.c_int32, C.c_int64,
                                           C.c_void_p]),
     "ss_forward_workspace_size": (c_status, [C.c_void_p, C.c_int32, C.POINTER(ForwardParams),

@@ -569,6 +569,209 @@ SS_EXPORT ss_status ss_index_append(ss_index* ix, const void* keys, int32_t n_fr
   return SS_OK;
 }
 
+SS_EXPORT ss_status ss_index_get_config(const ss_index* ix, ss_index_config* cfg) {
+  if (!ix || !cfg) return fail(SS_ERR_INVALID_ARG, "NULL argument");
+  *cfg = ix->cfg;
+  return SS_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Checkpoint: the index's host metadata and every device array, raw, at full capacity.
+// ---------------------------------------------------------------------------
+namespace {
+
+constexpr char kFileMagic[8] = {'S', 'S', 'I', 'D', 'X', 0, 0, 1};
+
+struct FileHeader {
+  ss_index_config cfg;
+  int64_t n_frames, n_units, n_vframes;
+  int32_t win_frames, n_centroids, n_windows, wcap;
+  int64_t n_clustered;
+  int32_t uc_cap, has_values;
+};
+
+// The device arrays of an index in file order, with their sizes (0 = not allocated).
+struct ArrayRef {
+  void** ptr;
+  size_t bytes;
+};
+
+std::vector<ArrayRef> index_arrays(ss_index* ix, bool values) {
+  const ss_index_config& c = ix->cfg;
+  const size_t n_slabs = (size_t)c.n_layers * c.n_kv_heads;
+  const size_t D = (size_t)c.n_kv_heads * kHeadDim;
+  const size_t Tu = (size_t)c.tokens_per_frame * c.frames_per_unit;
+  const size_t kb = n_slabs * ix->ncap * kHeadDim * 2;
+  std::vector<ArrayRef> a;
+  a.push_back({(void**)&ix->keys, kb});
+  a.push_back({(void**)&ix->desc, (size_t)ix->ucap * D * 4});
+  a.push_back({(void**)&ix->vals, values ? kb : 0});
+  const bool win = ix->win_frames > 0;
+  const size_t wcap = (size_t)ix->wcap, nc = (size_t)ix->n_centroids;
+  const size_t wu = win ? (size_t)(ix->win_frames / c.frames_per_unit) : 1;
+  const size_t n_slots = win ? ((size_t)ix->ucap + wu - 1) / wu : 0;
+  a.push_back({(void**)&ix->cent, win ? n_slabs * wcap * nc * kHeadDim * 2 : 0});
+  a.push_back({(void**)&ix->assign, win ? n_slabs * ix->ncap : 0});
+  a.push_back({(void**)&ix->win_u0, win ? wcap * 4 : 0});
+  a.push_back({(void**)&ix->win_slot, win ? n_slots * 4 : 0});
+  a.push_back({(void**)&ix->mcnt, win ? n_slabs * wcap * nc * wu * 4 : 0});
+  a.push_back({(void**)&ix->msize, win ? n_slabs * wcap * nc * 4 : 0});
+  const size_t cap = (size_t)ix->uc_cap;
+  const bool uc = cap > 0;
+  a.push_back({(void**)&ix->kstatus, (win || uc) ? (size_t)256 : (size_t)0});
+  a.push_back({(void**)&ix->unit_cluster, uc ? (size_t)ix->ucap * 4 : 0});
+  a.push_back({(void**)&ix->cdesc, uc ? cap * D * 4 : 0});
+  a.push_back({(void**)&ix->ccount, uc ? cap * 4 : 0});
+  a.push_back({(void**)&ix->creps, uc ? cap * n_slabs * Tu * kHeadDim * 4 : 0});
+  a.push_back({(void**)&ix->cfirst, uc ? cap * 4 : 0});
+  a.push_back({(void**)&ix->cprev, uc ? cap * 4 : 0});
+  a.push_back({(void**)&ix->uc_count, uc ? (size_t)256 : (size_t)0});
+  a.push_back({(void**)&ix->uc_work, uc ? cap * 4 : 0});
+  return a;
+}
+
+constexpr size_t kIoChunk = 64u << 20;   // host staging per copy
+
+}  // namespace
+
+SS_EXPORT ss_status ss_index_save(const ss_index* cix, const char* path, void* stream) {
+  if (!cix || !path) return fail(SS_ERR_INVALID_ARG, "NULL argument");
+  ss_index* ix = const_cast<ss_index*>(cix);
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  SS_CUDA(cudaSetDevice(ix->device));
+  FileHeader h{};
+  h.cfg = ix->cfg;
+  h.n_frames = ix->n_frames;
+  h.n_units = ix->n_units;
+  h.n_vframes = ix->n_vframes;
+  h.win_frames = ix->win_frames;
+  h.n_centroids = ix->n_centroids;
+  h.n_windows = ix->n_windows;
+  h.wcap = ix->wcap;
+  h.n_clustered = ix->n_clustered;
+  h.uc_cap = ix->uc_cap;
+  h.has_values = ix->vals != nullptr;
+  FILE* f = fopen(path, "wb");
+  if (!f) return fail(SS_ERR_INVALID_ARG, "cannot open %s for writing", path);
+  void* stage = nullptr;
+  if (cudaMallocHost(&stage, kIoChunk) != cudaSuccess) {
+    cudaGetLastError();
+    fclose(f);
+    return fail(SS_ERR_ALLOC, "page-locked staging buffer");
+  }
+  bool ok = fwrite(kFileMagic, 1, 8, f) == 8 && fwrite(&h, sizeof(h), 1, f) == 1;
+  for (int64_t fr : ix->win_first_frame) ok = ok && fwrite(&fr, 8, 1, f) == 1;
+  cudaError_t ce = cudaSuccess;
+  for (const ArrayRef& a : index_arrays(ix, ix->vals != nullptr)) {
+    const int64_t nb = (int64_t)a.bytes;
+    ok = ok && fwrite(&nb, 8, 1, f) == 1;
+    for (size_t off = 0; ok && ce == cudaSuccess && off < a.bytes; off += kIoChunk) {
+      const size_t n = a.bytes - off < kIoChunk ? a.bytes - off : kIoChunk;
+      ce = cudaMemcpyAsync(stage, static_cast<const char*>(*a.ptr) + off, n,
+                           cudaMemcpyDeviceToHost, st);
+      if (ce == cudaSuccess) ce = cudaStreamSynchronize(st);
+      ok = ok && ce == cudaSuccess && fwrite(stage, 1, n, f) == n;
+    }
+  }
+  cudaFreeHost(stage);
+  ok = (fclose(f) == 0) && ok;
+  if (ce != cudaSuccess) return fail(SS_ERR_CUDA, "device-to-host copy: %s", cudaGetErrorString(ce));
+  if (!ok) return fail(SS_ERR_INVALID_ARG, "write to %s failed", path);
+  return SS_OK;
+}
+
+SS_EXPORT ss_status ss_index_load(const char* path, const ss_allocator* alloc, void* stream,
+                                  ss_index** out) {
+  if (!path || !out) return fail(SS_ERR_INVALID_ARG, "NULL argument");
+  *out = nullptr;
+  FILE* f = fopen(path, "rb");
+  if (!f) return fail(SS_ERR_INVALID_ARG, "cannot open %s", path);
+  char magic[8];
+  FileHeader h{};
+  if (fread(magic, 1, 8, f) != 8 || memcmp(magic, kFileMagic, 8) != 0 ||
+      fread(&h, sizeof(h), 1, f) != 1) {
+    fclose(f);
+    return fail(SS_ERR_INVALID_ARG, "%s is not an index file of this version", path);
+  }
+  ss_index* ix = nullptr;
+  ss_status s = ss_index_create(&h.cfg, alloc, stream, &ix);
+  if (s != SS_OK) {
+    fclose(f);
+    return s;
+  }
+  const bool sane = h.n_frames >= 0 && h.n_frames <= h.cfg.max_frames && h.n_vframes >= 0 &&
+                    h.n_vframes <= h.n_frames && h.n_windows >= 0 && h.wcap >= 0 &&
+                    h.n_windows <= h.wcap && h.uc_cap >= 0 && h.n_clustered >= 0 &&
+                    h.n_centroids >= 0 && h.n_centroids <= kMaxCentroids &&
+                    h.win_frames >= 0 && h.n_units == h.n_frames / h.cfg.frames_per_unit &&
+                    (h.win_frames == 0 || h.win_frames % h.cfg.frames_per_unit == 0);
+  bool ok = sane;
+  for (int32_t w = 0; ok && w < h.n_windows; ++w) {
+    int64_t fr = 0;
+    ok = fread(&fr, 8, 1, f) == 1;
+    ix->win_first_frame.push_back(fr);
+  }
+  if (ok) {
+    ix->n_frames = h.n_frames;
+    ix->n_units = h.n_units;
+    ix->n_vframes = h.n_vframes;
+    ix->win_frames = h.win_frames;
+    ix->n_centroids = h.n_centroids;
+    ix->n_windows = h.n_windows;
+    ix->wcap = h.wcap;
+    ix->n_clustered = h.n_clustered;
+    ix->uc_cap = h.uc_cap;
+  }
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  void* stage = nullptr;
+  if (ok && cudaMallocHost(&stage, kIoChunk) != cudaSuccess) {
+    cudaGetLastError();
+    stage = nullptr;
+    ok = false;
+  }
+  cudaError_t ce = cudaSuccess;
+  bool alloc_failed = false;
+  if (ok) {
+    // the arrays the saved index had allocated are allocated here with the same sizes
+    // (the keys and descriptors come from ss_index_create)
+    if (h.win_frames == 0) ix->wcap = 0;
+    for (ArrayRef& a : index_arrays(ix, h.has_values != 0)) {
+      int64_t nb = -1;
+      if (!ok || fread(&nb, 8, 1, f) != 1 || nb != (int64_t)a.bytes) {
+        ok = false;
+        break;
+      }
+      if (a.bytes == 0) continue;
+      if (!*a.ptr) {
+        *a.ptr = dev_alloc(ix, a.bytes, st);
+        if (!*a.ptr) {
+          alloc_failed = true;
+          ok = false;
+          break;
+        }
+      }
+      for (size_t off = 0; ok && off < a.bytes; off += kIoChunk) {
+        const size_t n = a.bytes - off < kIoChunk ? a.bytes - off : kIoChunk;
+        ok = fread(stage, 1, n, f) == n;
+        if (ok) ce = cudaMemcpyAsync(static_cast<char*>(*a.ptr) + off, stage, n,
+                                     cudaMemcpyHostToDevice, st);
+        if (ok && ce == cudaSuccess) ce = cudaStreamSynchronize(st);
+        ok = ok && ce == cudaSuccess;
+      }
+    }
+  }
+  if (stage) cudaFreeHost(stage);
+  fclose(f);
+  if (!ok) {
+    ss_index_destroy(ix);
+    if (alloc_failed) return fail(SS_ERR_ALLOC, "device allocation while loading %s", path);
+    if (ce != cudaSuccess) return fail(SS_ERR_CUDA, "host-to-device copy: %s", cudaGetErrorString(ce));
+    return fail(SS_ERR_INVALID_ARG, "%s is truncated or inconsistent", path);
+  }
+  *out = ix;
+  return SS_OK;
+}
+
 SS_EXPORT ss_status ss_index_get_view(const ss_index* ix, ss_index_view* v) {
   if (!ix || !v) return fail(SS_ERR_INVALID_ARG, "NULL argument");
   v->n_frames = ix->n_frames;
