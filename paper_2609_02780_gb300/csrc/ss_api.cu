@@ -8,6 +8,7 @@
 #include <vector>
 
 #include <cuda.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include "shallowstream.h"
 #include "ss_internal.cuh"
@@ -59,6 +60,13 @@ struct ss_index {
 
 namespace {
 thread_local char g_err[512] = "";
+
+// A named NVTX range around a public call (visible to a profiler's timeline; near free when
+// no tool is attached).
+struct Range {
+  explicit Range(const char* name) { nvtxRangePushA(name); }
+  ~Range() { nvtxRangePop(); }
+};
 }  // namespace
 
 ss_status ss::fail_status(ss_status s, const char* fmt, ...) {
@@ -543,6 +551,7 @@ SS_EXPORT ss_status ss_index_destroy(ss_index* ix) {
 
 SS_EXPORT ss_status ss_index_append(ss_index* ix, const void* keys, int32_t n_frames,
                                     int64_t stride, void* stream) {
+  Range range_("ss_index_append");
   if (!ix) return fail(SS_ERR_INVALID_ARG, "index is NULL");
   if (n_frames < 0) return fail(SS_ERR_INVALID_ARG, "n_frames must be >= 0");
   if (n_frames == 0) return SS_OK;
@@ -635,6 +644,7 @@ constexpr size_t kIoChunk = 64u << 20;   // host staging per copy
 }  // namespace
 
 SS_EXPORT ss_status ss_index_save(const ss_index* cix, const char* path, void* stream) {
+  Range range_("ss_index_save");
   if (!cix || !path) return fail(SS_ERR_INVALID_ARG, "NULL argument");
   ss_index* ix = const_cast<ss_index*>(cix);
   const cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -682,6 +692,7 @@ SS_EXPORT ss_status ss_index_save(const ss_index* cix, const char* path, void* s
 
 SS_EXPORT ss_status ss_index_load(const char* path, const ss_allocator* alloc, void* stream,
                                   ss_index** out) {
+  Range range_("ss_index_load");
   if (!path || !out) return fail(SS_ERR_INVALID_ARG, "NULL argument");
   *out = nullptr;
   FILE* f = fopen(path, "rb");
@@ -801,6 +812,7 @@ SS_EXPORT ss_status ss_index_get_view(const ss_index* ix, ss_index_view* v) {
 
 SS_EXPORT ss_status ss_index_append_values(ss_index* ix, const void* values, int32_t n_frames,
                                            int64_t stride, void* stream) {
+  Range range_("ss_index_append_values");
   if (!ix) return fail(SS_ERR_INVALID_ARG, "index is NULL");
   if (n_frames < 0) return fail(SS_ERR_INVALID_ARG, "n_frames must be >= 0");
   if (n_frames == 0) return SS_OK;
@@ -877,6 +889,7 @@ SS_EXPORT ss_status ss_question_forward(ss_index* ix, const ss_layer_weights* la
                                         int32_t n_rows, void* q_out, float* h_out,
                                         uint32_t* status, void* workspace,
                                         size_t workspace_bytes, void* stream) {
+  Range range_("ss_question_forward");
   FwShape F{};
   ss_status s = forward_shape(ix, n_rows, fp, &F);
   if (s != SS_OK) return s;
@@ -921,6 +934,7 @@ SS_EXPORT ss_status ss_question_forward(ss_index* ix, const ss_layer_weights* la
 }
 
 SS_EXPORT ss_status ss_index_compress(ss_index* ix, const ss_compress_params* cp, void* stream) {
+  Range range_("ss_index_compress");
   if (!ix || !cp) return fail(SS_ERR_INVALID_ARG, "NULL argument");
   const ss_index_config& c = ix->cfg;
   const ss_compress_params& q = *cp;
@@ -1002,6 +1016,7 @@ SS_EXPORT ss_status ss_index_compress(ss_index* ix, const ss_compress_params* cp
 
 SS_EXPORT ss_status ss_index_cluster_units(ss_index* ix, int64_t n_units, float tau,
                                            int32_t max_clusters, void* stream) {
+  Range range_("ss_index_cluster_units");
   if (!ix) return fail(SS_ERR_INVALID_ARG, "index is NULL");
   if (n_units < 0) return fail(SS_ERR_INVALID_ARG, "n_units must be >= 0");
   if (tau != tau) return fail(SS_ERR_INVALID_ARG, "tau is NaN");
@@ -1093,6 +1108,7 @@ SS_EXPORT ss_status ss_index_units_over_budget(const ss_index* ix, int64_t budge
 SS_EXPORT ss_status ss_select_clusters(ss_index* ix, const void* q, int32_t R, int32_t q_agg,
                                        int32_t k_l, int32_t* ids, float* scores,
                                        int32_t* count, void* stream) {
+  Range range_("ss_select_clusters");
   if (!ix || !q || !ids || !scores || !count) return fail(SS_ERR_INVALID_ARG, "NULL argument");
   if (R < 1) return fail(SS_ERR_INVALID_ARG, "n_rows must be >= 1");
   if (q_agg != SS_Q_LAST && q_agg != SS_Q_MEAN_LOGIT && q_agg != SS_Q_MEAN_SOFTMAX)
@@ -1139,6 +1155,7 @@ SS_EXPORT ss_status ss_retrieve_workspace_size(const ss_index* const* ix, int32_
 SS_EXPORT ss_status ss_retrieve(ss_index* ix, const void* q, int32_t R,
                                 const ss_retrieve_params* p, const ss_result* res, void* ws,
                                 size_t ws_bytes, void* stream, const ss_trace* tr) {
+  Range range_("ss_retrieve");
   ss_index* const arr[1] = {ix};
   const void* const qa[1] = {q};
   return retrieve_impl(arr, qa, &R, 1, p, res, ws, ws_bytes, static_cast<cudaStream_t>(stream), tr);
@@ -1149,6 +1166,7 @@ SS_EXPORT ss_status ss_retrieve_batched(ss_index* const* ix, const void* const* 
                                         const ss_retrieve_params* p, const ss_result* res,
                                         void* ws, size_t ws_bytes, void* stream,
                                         const ss_trace* tr) {
+  Range range_("ss_retrieve_batched");
   return retrieve_impl(ix, q, R, n, p, res, ws, ws_bytes, static_cast<cudaStream_t>(stream), tr);
 }
 
@@ -1156,6 +1174,7 @@ SS_EXPORT ss_status ss_retrieve_shard(ss_index* ix, const void* q, int32_t R,
                                       const ss_retrieve_params* p, int64_t unit_begin,
                                       const ss_shard_result* out, void* ws, size_t ws_bytes,
                                       void* stream) {
+  Range range_("ss_retrieve_shard");
   if (!ix || !out) return fail(SS_ERR_INVALID_ARG, "NULL argument");
   ss_status s = check_params(p);
   if (s != SS_OK) return s;
@@ -1200,6 +1219,7 @@ SS_EXPORT ss_status ss_status_sync(const uint32_t* status, void* stream) {
 SS_EXPORT ss_status ss_retrieve_host(ss_index* ix, const void* q_host, int32_t R,
                                      const ss_retrieve_params* p, const ss_host_result* out,
                                      void* ws, size_t ws_bytes, void* stream) {
+  Range range_("ss_retrieve_host");
   if (!ix || !q_host || !out || !out->sel_units || !out->exp_units || !out->frames || !out->counts)
     return fail(SS_ERR_INVALID_ARG, "NULL argument");
   ss_status s = check_params(p);
@@ -1357,6 +1377,7 @@ ss_status static_scratch(int dev, void** out) {
 SS_EXPORT ss_status ss_retrieve_static(ss_index* ix, const void* q, int32_t R,
                                        const ss_retrieve_params* p, const ss_result* res,
                                        void* stream) {
+  Range range_("ss_retrieve_static");
   if (!ix || !q || !p || !res) return fail(SS_ERR_INVALID_ARG, "NULL argument");
   ss_status s = check_params(p);
   if (s != SS_OK) return s;
