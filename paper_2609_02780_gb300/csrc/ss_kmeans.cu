@@ -257,48 +257,53 @@ __global__ void __launch_bounds__(kKmThreads) k_kmeans(const KmJob J) {
 
 // ---------------------------------------------------------------------------
 // Lloyd rounds on the 5th-generation tensor cores (n_c <= 64, windows of <= 16384
-// tokens). One CTA per (window, slab); every round streams the window's keys once, in
-// tiles of 128 tokens, through a ring of shared-memory stages filled by tiled TMA
-// copies (128-byte swizzle; a 4-D tensor map [slab][window][token][dim] whose token
-// extent is the window, so a ragged last tile reads zeros). Per tile:
-//   MMA1  D1[token][c]      = x . c_hi,  D1[token][n16 + c] = x . c_lo
-//         (M = 128 tokens, N = 2 n16, K = 128 dims; c_hi = bf16(c), c_lo = bf16(c - c_hi),
+// tokens). One CTA per (window, slab), sized so that two CTAs share an SM: a CTA's rounds
+// are a chain of dependent steps per tile, and the second CTA's tiles fill its gaps.
+// Every round streams the window's keys once, in tiles of 128 tokens, through two
+// shared-memory stages filled by tiled TMA copies (128-byte swizzle; a 4-D tensor map
+// [slab][window][token][dim] whose token extent is the window, so a ragged last tile
+// reads zeros). Per tile:
+//   MMA1  D1[token][c] = x . c_hi + x . c_lo, the lo products accumulated onto the hi ones
+//         (M = 128 tokens, N = n16, K = 2 x 128 dims; c_hi = bf16(c), c_lo = bf16(c - c_hi),
 //         so x . c carries ~16 significant bits of c; fp32 accumulation in TMEM)
-//   assign a(x) = argmin_c ||c||^2 - 2 (x . c_hi + x . c_lo), lowest id on ties; the
-//         epilogue writes the one-hot row of a(x) (bf16 1.0) into shared memory
+//   assign a(x) = argmin_c ||c||^2 - 2 x . c, lowest id on ties; the epilogue writes the
+//         one-hot row of a(x) (bf16 1.0) into shared memory
 //   MMA2  D2[dim][c] += sum_x x[dim] * onehot[x][c]
 //         (M = 128 dims, N = 64, K = 128 tokens: the key tile read MN-major, the same
 //         bytes as MMA1's K-major operand, so each key is loaded once per round)
 // At the end of a round the member sums D2 and the counts give the new centroids
-// (c = sum / count; an empty centroid keeps its value), from which the epilogue builds
-// the next round's split operands. Every sum has a fixed order (the tensor core's
-// accumulation order over the window's tiles), so results repeat bit for bit.
+// (c = sum * (1 / count); an empty centroid keeps its value), from which the epilogue
+// builds the next round's split operands. Every sum has a fixed order (the tensor core's
+// accumulation order over the window's tiles), so results repeat bit for bit. The last
+// round's assignments and member counts per (centroid, unit) go straight to global memory.
 //
 // Warp roles: warp 0 issues the TMA copies, warp 1 allocates tensor memory and issues
 // the MMAs (one thread), warps 2-5 are the epilogue (thread e owns TMEM lane e: token e
-// of a tile for MMA1, dim e for MMA2). All waits are bounded; a wait that gives up
-// raises a shared abort flag that ends every role's loop, then the copies and MMAs in
-// flight are drained and the tensor memory is freed.
+// of a tile for MMA1, dim e for MMA2 and the update). All waits are bounded; a wait that
+// gives up raises a shared abort flag that ends every role's loop, then the copies and
+// MMAs in flight are drained and the tensor memory is freed. Every epilogue thread runs
+// the same sequence of named barriers whatever happens.
 // ---------------------------------------------------------------------------
-constexpr int kTcStages = 4;
+constexpr int kTcStages = 2;
 constexpr int kTcTile = 128;                            // tokens per tile
 constexpr int kTcStageBytes = kTcTile * kHeadDim * 2;   // 32 KB
-constexpr int kTcEpiWarps = 8;                          // two per TMEM lane quarter
-constexpr int kTcEpiThreads = kTcEpiWarps * 32;
+constexpr int kTcEpiThreads = 128;                      // one per TMEM lane
 constexpr int kTcThreads = 64 + kTcEpiThreads;          // + TMA warp + MMA warp
 constexpr int kTcMaxCentroids = 64;
 constexpr int kTcMaxWindowTokens = 16384;
-constexpr int kTcD1Bufs = 3;
-// tensor memory: D1 in three buffers of 128 columns, D2 (64 columns), the fp32
-// centroids (lane = dim, column = centroid; 64 columns)
-constexpr uint32_t kTcTmemCols = 512;
-constexpr uint32_t kTcD2Col = 384;
-constexpr uint32_t kTcCfCol = 448;
+constexpr int kTcD1Bufs = 2;
+constexpr int kTcB1Bytes = 128 * 256;                   // hi and lo rows, two 64-dim halves
+constexpr int kTcOneHotBytes = kTcTile * 128;           // 128 tokens x 64 centroids (bf16)
+// tensor memory (256 columns, half an SM's): D1 in two buffers at 0 and 64 (n16 columns
+// used), D2 at 128 (64 columns), the fp32 centroids at 192 (lane = dim, column = centroid)
+constexpr uint32_t kTcTmemCols = 256;
+constexpr uint32_t kTcD2Col = 128;
+constexpr uint32_t kTcCfCol = 192;
 
 struct TcJob {
   __nv_bfloat16* cent;        // [n_slabs][wcap * n_c][d]
   uint8_t* assign;            // [n_slabs][ncap]
-  int32_t* mcnt;              // [n_slabs][wcap][n_c][wu]
+  int32_t* mcnt;              // [n_slabs][wcap][n_c][wu] (zeroed by the launcher)
   int32_t* msize;             // [n_slabs][wcap][n_c]
   const __nv_bfloat16* keys;  // [n_slabs][ncap][d] (initial centroids)
   int64_t ncap;
@@ -307,23 +312,23 @@ struct TcJob {
   uint32_t* status;           // device word: kStatusTimeout on a wait that gave up
 };
 
+// Barriers and per-round tallies, at the end of the dynamic shared memory (the CTA has no
+// static shared memory, so the dynamic region starts on the 1024-byte boundary the
+// swizzled tiles need).
 struct TcBars {
   unsigned long long full[kTcStages], empty[kTcStages];
-  unsigned long long d1_full[kTcD1Bufs], epi_done[kTcD1Bufs], mma2_done[2];
+  unsigned long long d1_full[kTcD1Bufs], epi_done[kTcD1Bufs], mma2_done;
   unsigned long long d2_full, b1_ready, final_mma;
   uint32_t taddr;
   int abort;
   int cnt[kTcMaxCentroids];
   float cn2[kTcMaxCentroids];
-  float part[4][kTcMaxCentroids];  // ||c||^2 partial sums of each lane quarter
-  float xbest[2][2][kTcTile];      // [tile parity][centroid half][row]: nearest distance
-  int xbc[2][2][kTcTile];          // and its centroid
 };
 
-// ring, B1 operand (128 rows x 256 B), one-hot rows (2 x 128 x 128 B), assignment bytes
+// ring, B1 operand, one-hot rows, barriers
 size_t kmeans_tc_smem_bytes(int Wt) {
-  return 1024 + (size_t)kTcStages * kTcStageBytes + 128 * 256 + 2 * kTcTile * 128 +
-         (size_t)((Wt + 15) & ~15);
+  (void)Wt;
+  return (size_t)kTcStages * kTcStageBytes + kTcB1Bytes + kTcOneHotBytes + sizeof(TcBars);
 }
 
 bool kmeans_tc_supported(int n_c, int Wt) {
@@ -358,64 +363,56 @@ __device__ __forceinline__ void tc_put_split(unsigned char* B1, int N1, int row,
   *reinterpret_cast<__nv_bfloat16*>(h0 + r2 * 128 + ((((b >> 4) ^ (r2 & 7))) << 4) + (b & 15)) = lo;
 }
 
-// Byte offset of centroid c in row r of a one-hot tile (MN-major, 128-byte swizzle).
+// Byte offset of centroid c in row r of the one-hot tile (MN-major, 128-byte swizzle).
 __device__ __forceinline__ int onehot_off(int r, int c) {
   return r * 128 + ((((c >> 3) ^ (r & 7))) << 4) + (c & 7) * 2;
 }
 
-__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
-// The two warps of one TMEM lane quarter (barriers 2-5).
-__device__ __forceinline__ void pair_bar(int q) {
-  asm volatile("bar.sync %0, 64;" ::"r"(2 + q) : "memory");
-}
+__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
-// New round operands from the fp32 centroids cf[0..31] = centroids 32 h .. 32 h + 31 at
-// this thread's dim er: the centroids to tensor memory, the split rows of B1 and
-// ||c||^2 of every centroid (squares summed over each warp's 32 dims by a shuffle tree,
-// then over the four lane quarters in order: a fixed order). On return this thread holds
-// the squared norms of its own 32 centroids in cn2r.
-__device__ __forceinline__ void tc_round_operands(const float* cf, int h, int q, int lane, int er,
-                                                  int ei, int n_c, int n16, unsigned char* B1,
-                                                  TcBars& S, uint32_t cf_taddr, bool build_b1,
-                                                  float (&cn2r)[32]) {
-  float w[32];
-#pragma unroll
-  for (int c = 0; c < 32; ++c) w[c] = cf[c];
-  tmem_st32(cf_taddr + 32 * h, w);
-  if (build_b1)
+// One round's operands from 32 fp32 centroids cf[0..31] = centroids c0 .. c0 + 31 at this
+// thread's dim e: the centroids to tensor memory, their split rows of B1 (when `b1`), and
+// their squares summed over the warp's 32 dims by a shuffle tree into part[quarter][c].
+__device__ __forceinline__ void tc_put_centroids(const float (&cf)[32], int c0, int e, int q,
+                                                 int lane, int n16, unsigned char* B1,
+                                                 uint32_t cf_taddr, bool b1, float* part) {
+  tmem_st32(cf_taddr + (uint32_t)c0, cf);
+  if (b1)
 #pragma unroll
     for (int c = 0; c < 32; ++c)
-      if (32 * h + c < n16) tc_put_split(B1, 2 * n16, 32 * h + c, er, cf[c]);
+      if (c0 + c < n16) tc_put_split(B1, 2 * n16, c0 + c, e, cf[c]);
 #pragma unroll
   for (int c = 0; c < 32; ++c) {
     float v = cf[c] * cf[c];
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-    if (lane == 0) S.part[q][32 * h + c] = v;
+    if (lane == 0) part[q * kTcMaxCentroids + c0 + c] = v;
   }
-  epi_bar();
-  if (ei < n16) {
-    float s2 = INFINITY;   // padding centroids are never nearest
-    if (ei < n_c) s2 = ((S.part[0][ei] + S.part[1][ei]) + S.part[2][ei]) + S.part[3][ei];
-    S.cn2[ei] = s2;
-  }
-  epi_bar();
-#pragma unroll
-  for (int c = 0; c < 32; ++c) cn2r[c] = 32 * h + c < n16 ? S.cn2[32 * h + c] : INFINITY;
 }
 
-__global__ void __launch_bounds__(kTcThreads, 1)
+// ||c||^2 of every centroid from the four lane quarters' partial sums (in quarter order:
+// a fixed order); padding centroids get +inf, so they are never nearest.
+__device__ __forceinline__ void tc_norms(TcBars& S, const float* part, int e, int n_c, int n16) {
+  if (e < n16)
+    S.cn2[e] = e < n_c ? ((part[e] + part[kTcMaxCentroids + e]) + part[2 * kTcMaxCentroids + e]) +
+                             part[3 * kTcMaxCentroids + e]
+                       : INFINITY;
+}
+
+__global__ void __launch_bounds__(256, 2)
     k_kmeans_tc(const __grid_constant__ CUtensorMap kmap, const TcJob J) {
-  extern __shared__ unsigned char sm_raw[];
-  __shared__ TcBars S;
-  unsigned char* sm = reinterpret_cast<unsigned char*>(
-      (reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  extern __shared__ __align__(1024) unsigned char sm[];
   unsigned char* ring = sm;
   unsigned char* B1 = ring + kTcStages * kTcStageBytes;
-  unsigned char* onehot = B1 + 128 * 256;
-  uint8_t* a_s = onehot + 2 * kTcTile * 128;
+  unsigned char* onehot = B1 + kTcB1Bytes;
+  TcBars& S = *reinterpret_cast<TcBars*>(onehot + kTcOneHotBytes);
+  float* part = reinterpret_cast<float*>(onehot);    // the one-hot space between rounds
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if ((smem_u32(sm) & 1023u) != 0u) {                // the swizzled tiles need the boundary
+    if (tid == 0) atomicOr(J.status, kStatusInternal);
+    return;
+  }
   const int wl = blockIdx.x, slab = blockIdx.y;
   const int n_c = J.n_c, n16 = J.n16, N1 = 2 * n16, Wt = J.Wt;
   const int ntile = (Wt + kTcTile - 1) / kTcTile;
@@ -431,7 +428,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       mbar_init(smem_u32(&S.d1_full[b]), 1);
       mbar_init(smem_u32(&S.epi_done[b]), kTcEpiThreads);
     }
-    for (int b = 0; b < 2; ++b) mbar_init(smem_u32(&S.mma2_done[b]), 1);
+    mbar_init(smem_u32(&S.mma2_done), 1);
     mbar_init(smem_u32(&S.d2_full), 1);
     mbar_init(smem_u32(&S.b1_ready), 1);
     mbar_init(smem_u32(&S.final_mma), 1);
@@ -439,9 +436,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (tid < kTcMaxCentroids) S.cnt[tid] = 0;
-  // the one-hot tiles start at zero; afterwards only the single 1.0 of a row changes
-  for (int x = tid; x < 2 * kTcTile * 128 / 16; x += kTcThreads)
-    reinterpret_cast<uint4*>(onehot)[x] = make_uint4(0u, 0u, 0u, 0u);
   if (warp == 1) {
     tmem_alloc(smem_u32(&S.taddr), kTcTmemCols);
     tmem_relinquish();
@@ -476,13 +470,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
     __syncwarp();
   } else if (warp == 1) {
-    // ---- MMA issuer: issues MMA1 of a tile as soon as its keys, a free D1 buffer and
-    // (at a round's first tile) the round's operands are ready, and MMA2 of the oldest
-    // tile whose one-hot rows are written, whichever comes first ----
+    // ---- MMA issuer: MMA1 of a tile as soon as its keys, a free D1 buffer and (at a
+    // round's first tile) the round's operands are ready; MMA2 of the oldest tile whose
+    // one-hot rows are written ----
     if (lane == 0) {
-      const uint32_t id1 = idesc_bf16_f32(128, N1, false, false);
+      const uint32_t id1 = idesc_bf16_f32(128, n16, false, false);
       const uint32_t id2 = idesc_bf16_f32(128, 64, true, true);
       const uint32_t b1s = smem_u32(B1);
+      const uint32_t os = smem_u32(onehot);
       int n1 = 0, n2 = 0;                       // next tile for MMA1, for MMA2
       uint64_t t_idle = 0;
       uint32_t idle = 0;
@@ -496,11 +491,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           if (ready) {
             tc_fence_after();
             const uint32_t as = smem_u32(ring + st * kTcStageBytes);
-            const uint32_t d1 = tbase + (uint32_t)buf * 128u;
+            const uint32_t d1 = tbase + (uint32_t)buf * 64u;
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-              const uint32_t ka = (k >> 2) * (kTcStageBytes / 2) + (k & 3) * 32;
-              const uint32_t kb = (k >> 2) * (N1 * 128) + (k & 3) * 32;
+            for (int k = 0; k < 16; ++k) {
+              const int kk = k & 7;
+              const uint32_t ka = (kk >> 2) * (kTcStageBytes / 2) + (kk & 3) * 32;
+              const uint32_t kb = (kk >> 2) * (N1 * 128) + (kk & 3) * 32 + (k >> 3) * (n16 * 128);
               umma_bf16(d1, sdesc_sw128(as + ka, 16, 1024), sdesc_sw128(b1s + kb, 16, 1024), id1,
                         k > 0 ? 1u : 0u);
             }
@@ -512,14 +508,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         if (n2 < n1 && mbar_test_wait(smem_u32(&S.epi_done[n2 % kTcD1Bufs]), (n2 / kTcD1Bufs) & 1)) {
           tc_fence_after();
           const uint32_t xs = smem_u32(ring + (n2 % kTcStages) * kTcStageBytes);
-          const uint32_t os = smem_u32(onehot + (n2 & 1) * (kTcTile * 128));
           const bool first = (n2 % ntile) == 0;
 #pragma unroll
           for (int k = 0; k < 8; ++k)
             umma_bf16(tbase + kTcD2Col, sdesc_sw128(xs + k * 2048, kTcStageBytes / 2, 1024),
                       sdesc_sw128(os + k * 2048, kTcStageBytes / 2, 1024), id2,
                       (first && k == 0) ? 0u : 1u);
-          umma_commit(smem_u32(&S.mma2_done[n2 & 1]));
+          umma_commit(smem_u32(&S.mma2_done));
           umma_commit(smem_u32(&S.empty[n2 % kTcStages]));
           if ((n2 % ntile) == ntile - 1) umma_commit(smem_u32(&S.d2_full));
           ++n2;
@@ -528,8 +523,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         if (did) {
           idle = 0;
         } else if (__nanosleep(32), (++idle & 255u) == 0u) {
-          // (the short sleep keeps this polling loop from taking the issue slots of the
-          // epilogue warps that share its scheduler)
           // bounded: give up after ~1 s without progress, or when another role did
           const uint64_t now = global_ns();
           if (idle == 256u) t_idle = now;
@@ -545,99 +538,96 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
     __syncwarp();
   } else {
-    // ---- epilogue: warps 2-9. Thread (h, er): TMEM lane er (token er of a tile for
-    // MMA1, dim er for MMA2) and centroids 32 h .. 32 h + 31 ----
-    // Every epilogue thread runs the same sequence of named barriers whatever happens
-    // (a wait that gives up clears `ok` and the work is skipped, never the barriers).
+    // ---- epilogue: warps 2-5. Thread e: TMEM lane e (token e of a tile for MMA1, dim e
+    // for MMA2 and the update) ----
     const int q = warp & 3;                      // the lane quarter this warp may access
-    const int h = (warp - 2) >> 2;               // centroid half
-    const int er = q * 32 + lane;
-    const int ei = h * 128 + er;                 // 0 .. 255
+    const int e = q * 32 + lane;
     const uint32_t lane_addr = tbase + ((uint32_t)(q * 32) << 16);
     const __nv_bfloat16* X0 =
         J.keys + ((int64_t)slab * J.ncap + J.tok_first + (int64_t)wl * Wt) * kHeadDim;
-    const int c_lo = 32 * h;                     // this thread's first centroid
-    const int n_mine = max(0, min(32, n16 - c_lo));
-    float cn2r[32];                              // ||c||^2 of this thread's centroids
-    int prev[2] = {-1, -1};                      // the 1.0 each one-hot tile holds in row er
+    const int64_t tok0 = J.tok_first + (int64_t)wl * Wt;
+    uint8_t* ao = J.assign + (int64_t)slab * J.ncap + tok0;
+    int32_t* mc = J.mcnt + ((int64_t)slab * J.wcap + J.w_begin + wl) * n_c * J.wu;
+    int prev = -1;                               // the 1.0 the one-hot tile holds in row e
     bool ok = true;
     {
-      // C0 = the window's first n_c keys; the round-0 operands
-      float cf[32];
+      // C0 = the window's first n_c keys; the round-0 operands (the one-hot space holds
+      // the norms' partial sums first, then is cleared)
+#pragma unroll 1
+      for (int c0 = 0; c0 < 64; c0 += 32) {
+        float cf[32];
 #pragma unroll
-      for (int c = 0; c < 32; ++c)
-        cf[c] = c_lo + c < n_c ? __bfloat162float(X0[(int64_t)(c_lo + c) * kHeadDim + er]) : 0.f;
-      tc_round_operands(cf, h, q, lane, er, ei, n_c, n16, B1, S, lane_addr + kTcCfCol, true, cn2r);
+        for (int c = 0; c < 32; ++c)
+          cf[c] = c0 + c < n_c ? __bfloat162float(X0[(int64_t)(c0 + c) * kHeadDim + e]) : 0.f;
+        tc_put_centroids(cf, c0, e, q, lane, n16, B1, lane_addr + kTcCfCol, true, part);
+      }
+      epi_bar();
+      tc_norms(S, part, e, n_c, n16);
+      epi_bar();
+#pragma unroll
+      for (int x = 0; x < kTcOneHotBytes / 16 / kTcEpiThreads; ++x)
+        reinterpret_cast<uint4*>(onehot)[x * kTcEpiThreads + e] = make_uint4(0u, 0u, 0u, 0u);
     }
     fence_proxy_async_smem();
     tc_fence_before();
     epi_bar();
-    if (ei == 0) mbar_arrive(smem_u32(&S.b1_ready));
+    if (e == 0) mbar_arrive(smem_u32(&S.b1_ready));
 
     for (int j = 0; j < J_tiles; ++j) {
-      const int tile = j % ntile, round = j / ntile, buf = j % kTcD1Bufs, x = j & 1;
+      const int tile = j % ntile, round = j / ntile, buf = j % kTcD1Bufs;
+      const bool last = round + 1 == J.iters;
       ok = ok && tc_wait(smem_u32(&S.d1_full[buf]), (j / kTcD1Bufs) & 1, abort);
       tc_fence_after();
-      // nearest of this half's centroids to token tile * 128 + er
+      // nearest centroid of token tile * 128 + e (chunks of 32 columns)
       float best = INFINITY;
-      int bc = c_lo;
-      if (ok && n_mine > 0) {
-        const uint32_t d1 = lane_addr + (uint32_t)buf * 128u;
-        if (n_mine == 32) {
-          float hi[32], lo[32];
-          tmem_ld32x2(d1 + c_lo, d1 + n16 + c_lo, hi, lo);
+      int bc = 0;
+      if (ok) {
+        const uint32_t d1 = lane_addr + (uint32_t)buf * 64u;
+#pragma unroll 1
+        for (int c0 = 0; c0 < n16; c0 += 32) {
+          if (n16 - c0 >= 32) {
+            float xc[32];
+            tmem_ld32(d1 + (uint32_t)c0, xc);
 #pragma unroll
-          for (int c = 0; c < 32; ++c) {
-            const float dist = fmaf(-2.f, hi[c] + lo[c], cn2r[c]);
-            if (dist < best) {
-              best = dist;
-              bc = c_lo + c;
+            for (int c = 0; c < 32; ++c) {
+              const float dist = fmaf(-2.f, xc[c], S.cn2[c0 + c]);
+              if (dist < best) {
+                best = dist;
+                bc = c0 + c;
+              }
             }
-          }
-        } else {
+          } else {
+            float xc[16];
+            tmem_ld16(d1 + (uint32_t)c0, xc);
 #pragma unroll
-          for (int c0 = 0; c0 < 32; c0 += 16) {
-            if (c0 < n_mine) {
-              float hi[16], lo[16];
-              tmem_ld16(d1 + c_lo + c0, hi);
-              tmem_ld16(d1 + n16 + c_lo + c0, lo);
-#pragma unroll
-              for (int t = 0; t < 16; ++t) {
-                const float dist = fmaf(-2.f, hi[t] + lo[t], cn2r[c0 + t]);
-                if (dist < best) {
-                  best = dist;
-                  bc = c_lo + c0 + t;
-                }
+            for (int c = 0; c < 16; ++c) {
+              const float dist = fmaf(-2.f, xc[c], S.cn2[c0 + c]);
+              if (dist < best) {
+                best = dist;
+                bc = c0 + c;
               }
             }
           }
         }
       }
-      // the two halves' candidates (double-buffered by tile parity): the nearest, the
-      // lower half on a tie (lower ids), is the row's centroid
-      if (h == 1) {
-        S.xbest[x][1][er] = best;
-        S.xbc[x][1][er] = bc;
-      }
-      pair_bar(q);
-      const int tok = tile * kTcTile + er;
+      const int tok = tile * kTcTile + e;
       const bool valid = tok < Wt;
-      if (h == 0) {
-        if (S.xbest[x][1][er] < best) bc = S.xbc[x][1][er];
-        ok = ok && (j < 2 || tc_wait(smem_u32(&S.mma2_done[x]), ((j >> 1) - 1) & 1, abort));
-        if (ok) {
-          // one 2-byte store clears the row's previous 1.0 in this tile, one sets the new
-          unsigned char* t1 = onehot + x * (kTcTile * 128);
-          if (prev[x] >= 0) *reinterpret_cast<uint16_t*>(t1 + onehot_off(er, prev[x])) = 0;
-          prev[x] = valid ? bc : -1;
-          if (valid) {
-            *reinterpret_cast<uint16_t*>(t1 + onehot_off(er, bc)) = 0x3F80;   // bf16 1.0
-            a_s[tok] = (uint8_t)bc;
-            atomicAdd(&S.cnt[bc], 1);
+      // the one-hot tile is free once MMA2 of the previous tile has completed
+      ok = ok && (j == 0 || tc_wait(smem_u32(&S.mma2_done), (j - 1) & 1, abort));
+      if (ok) {
+        // one 2-byte store clears the row's previous 1.0, one sets the new
+        if (prev >= 0) *reinterpret_cast<uint16_t*>(onehot + onehot_off(e, prev)) = 0;
+        prev = valid ? bc : -1;
+        if (valid) {
+          *reinterpret_cast<uint16_t*>(onehot + onehot_off(e, bc)) = 0x3F80;   // bf16 1.0
+          atomicAdd(&S.cnt[bc], 1);
+          if (last) {
+            ao[tok] = (uint8_t)bc;
+            atomicAdd(mc + bc * J.wu + tok / J.Tu, 1);
           }
         }
-        fence_proxy_async_smem();
       }
+      fence_proxy_async_smem();
       tc_fence_before();
       mbar_arrive(smem_u32(&S.epi_done[buf]));
 
@@ -646,61 +636,52 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         epi_bar();                                            // every count is in
         ok = ok && tc_wait(smem_u32(&S.d2_full), round & 1, abort);
         tc_fence_after();
-        float cf[32];
+        // (every MMA of the round has completed: the one-hot space is free)
+        const bool write = !*abort;
+        __nv_bfloat16* co = J.cent + ((int64_t)slab * J.wcap * n_c +
+                                      (int64_t)(J.w_begin + wl) * n_c) * kHeadDim;
+#pragma unroll 1
+        for (int c0 = 0; c0 < 64; c0 += 32) {
+          float cf[32];
 #pragma unroll
-        for (int c = 0; c < 32; ++c) cf[c] = 0.f;
-        if (ok) {
-          float sum[32];
-          tmem_ld32x2(lane_addr + kTcD2Col + c_lo, lane_addr + kTcCfCol + c_lo, sum, cf);
-          // mean = sum * (1 / n): the reciprocal rounded once, then one rounded product
+          for (int c = 0; c < 32; ++c) cf[c] = 0.f;
+          if (ok) {
+            float sum[32];
+            tmem_ld32x2(lane_addr + kTcD2Col + (uint32_t)c0, lane_addr + kTcCfCol + (uint32_t)c0,
+                        sum, cf);
+            // mean = sum * (1 / n): the reciprocal rounded once, then one rounded product
 #pragma unroll
-          for (int c = 0; c < 32; ++c) {
-            const int n = c_lo + c < n_c ? S.cnt[c_lo + c] : 0;
-            if (n > 0) cf[c] = __fmul_rn(sum[c], __frcp_rn((float)n));
+            for (int c = 0; c < 32; ++c) {
+              const int n = c0 + c < n_c ? S.cnt[c0 + c] : 0;
+              if (n > 0) cf[c] = __fmul_rn(sum[c], __frcp_rn((float)n));
+            }
+          }
+          if (last) {
+#pragma unroll
+            for (int c = 0; c < 32; ++c)
+              if (write && c0 + c < n_c) co[(int64_t)(c0 + c) * kHeadDim + e] = __float2bfloat16_rn(cf[c]);
+          } else {
+            tc_put_centroids(cf, c0, e, q, lane, n16, B1, lane_addr + kTcCfCol, ok, part);
           }
         }
-        const bool more = round + 1 < J.iters;
-        tc_round_operands(cf, h, q, lane, er, ei, n_c, n16, B1, S, lane_addr + kTcCfCol,
-                          ok && more, cn2r);
-        if (more) {
-          if (ei < kTcMaxCentroids) S.cnt[ei] = 0;
+        if (!last) {
+          epi_bar();
+          tc_norms(S, part, e, n_c, n16);
+          if (e < kTcMaxCentroids) S.cnt[e] = 0;
+          epi_bar();
+          // the one-hot space back to zeros (the row's previous 1.0 is gone with it)
+#pragma unroll
+          for (int x = 0; x < kTcOneHotBytes / 16 / kTcEpiThreads; ++x)
+            reinterpret_cast<uint4*>(onehot)[x * kTcEpiThreads + e] = make_uint4(0u, 0u, 0u, 0u);
+          prev = -1;
           fence_proxy_async_smem();
           tc_fence_before();
           epi_bar();
-          if (ei == 0 && ok) mbar_arrive(smem_u32(&S.b1_ready));
+          if (e == 0 && ok) mbar_arrive(smem_u32(&S.b1_ready));
         } else {
-          // (the barriers below run whatever `write` says: abort may be raised between the
-          // threads' reads of it)
-          const bool write = !*abort;
-          // ---- outputs: centroids (bf16), assignment, member counts ----
-          __nv_bfloat16* co = J.cent + ((int64_t)slab * J.wcap * n_c +
-                                        (int64_t)(J.w_begin + wl) * n_c) * kHeadDim;
-#pragma unroll
-          for (int c = 0; c < 32; ++c)
-            if (write && c_lo + c < n_c)
-              co[(int64_t)(c_lo + c) * kHeadDim + er] = __float2bfloat16_rn(cf[c]);
-          // member counts per (centroid, unit of the window) tallied in shared memory (the
-          // one-hot tiles' space: every MMA has completed), then written out
-          const int64_t tok0 = J.tok_first + (int64_t)wl * Wt;
-          uint8_t* ao = J.assign + (int64_t)slab * J.ncap + tok0;
-          int32_t* mc = J.mcnt + ((int64_t)slab * J.wcap + J.w_begin + wl) * n_c * J.wu;
-          int* tally = reinterpret_cast<int*>(onehot);
-          const int n_tally = n_c * J.wu;
-          const bool in_smem = n_tally <= 2 * kTcTile * 128 / 4;
-          if (write && in_smem)
-            for (int x = ei; x < n_tally; x += kTcEpiThreads) tally[x] = 0;
           epi_bar();
-          for (int p = ei; write && p < Wt; p += kTcEpiThreads) {
-            const int c = a_s[p];
-            ao[p] = (uint8_t)c;
-            if (in_smem) atomicAdd(&tally[c * J.wu + p / J.Tu], 1);
-            else atomicAdd(mc + c * J.wu + p / J.Tu, 1);
-          }
-          epi_bar();
-          if (write && in_smem)
-            for (int x = ei; x < n_tally; x += kTcEpiThreads) mc[x] = tally[x];
           int32_t* ms = J.msize + ((int64_t)slab * J.wcap + J.w_begin + wl) * n_c;
-          if (write && ei < n_c) ms[ei] = S.cnt[ei];
+          if (write && e < n_c) ms[e] = S.cnt[e];
         }
       }
     }
