@@ -581,7 +581,28 @@ __global__ void __launch_bounds__(256, 2)
       // nearest centroid of token tile * 128 + e (chunks of 32 columns)
       float best = INFINITY;
       int bc = 0;
-      if (ok) {
+      if (ok && n16 == 64) {
+        // all 64 columns in one load and one wait
+        const uint32_t d1 = lane_addr + (uint32_t)buf * 64u;
+        float xa[32], xb[32];
+        tmem_ld32x2(d1, d1 + 32u, xa, xb);
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+          const float dist = fmaf(-2.f, xa[c], S.cn2[c]);
+          if (dist < best) {
+            best = dist;
+            bc = c;
+          }
+        }
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+          const float dist = fmaf(-2.f, xb[c], S.cn2[32 + c]);
+          if (dist < best) {
+            best = dist;
+            bc = 32 + c;
+          }
+        }
+      } else if (ok) {
         const uint32_t d1 = lane_addr + (uint32_t)buf * 64u;
 #pragma unroll 1
         for (int c0 = 0; c0 < n16; c0 += 32) {
