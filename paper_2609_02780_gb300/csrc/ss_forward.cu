@@ -376,11 +376,11 @@ __global__ void __launch_bounds__(256) k_fw_swiglu(const SwigluJob J) {
 // ===========================================================================
 // Attention of the question rows over the layer's stored tokens
 // ===========================================================================
-constexpr int kAtThreads = 320;            // warp 0 TMA, warp 1 MMA, warps 2-9 rows
-constexpr int kAtEpi = 256;                // two threads per row, 64 columns each
-constexpr int kAtTile = 128;               // tokens per tile
-constexpr int kAtTileBytes = kAtTile * kHeadDim * 2;   // 32 KB
-constexpr int kAtSmem = 7 * kAtTileBytes + 1024;       // Q, 2 P, 2 K, 2 V stages
+constexpr int kAtThreads = 192;            // warp 0 TMA, warp 1 MMA, warps 2-5 rows
+constexpr int kAtTile = 64;                // tokens per tile
+constexpr int kAtTileBytes = kAtTile * kHeadDim * 2;   // 16 KB of keys or values
+constexpr int kAtQBytes = 128 * kHeadDim * 2;          // 32 KB: 128 rows x 128 dims
+constexpr int kAtPBytes = 128 * kAtTile * 2;           // 16 KB: 128 rows x 64 tokens
 constexpr float kAtLazy = 8.0f;            // raise the running max only past this margin
 
 struct AttnJob {
@@ -394,50 +394,45 @@ struct AttnJob {
   uint32_t* status;
 };
 
+// Barriers, at the end of the dynamic shared memory (no static shared memory, so the
+// dynamic region starts on the 1024-byte boundary the swizzled tiles need).
 struct AtBars {
   unsigned long long kfull[2], kempty[2], vfull[2], vempty[2], sfull[2], sempty[2];
-  unsigned long long pfull[2], pvdone[2], q_ready, final_mma;
+  unsigned long long pfull, pvdone, q_ready, final_mma;
   uint32_t taddr;
   int abort;
-  float xchg[2][128];             // per column half: a row's tile maximum, then its l
 };
 
-// Barrier of the two warps that share a TMEM lane quarter (ids 2-5, 64 threads); returns
-// the AND of `pred` over them, so both take the same branch after it.
-__device__ __forceinline__ bool pair_sync_and(int qd, bool pred) {
-  uint32_t r;
-  asm volatile(
-      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n"
-      " barrier.red.and.pred q, %2, 64, p;\n selp.u32 %0, 1, 0, q;\n}\n"
-      : "=r"(r)
-      : "r"((uint32_t)pred), "r"(2 + qd)
-      : "memory");
-  return r != 0;
-}
+constexpr int kAtSmem = kAtQBytes + kAtPBytes + 4 * kAtTileBytes + (int)sizeof(AtBars);
 
-// grid (chunks, halves, Hkv). Rows rho = h * Rp + r (h < G) of key head g; this CTA
-// takes rho in [128 * half, 128 * half + 128). Pipeline per tile j of 128 tokens:
+// grid (chunks, halves, Hkv), two CTAs per SM (256 TMEM columns, ~113 KB of shared memory
+// each). Rows rho = h * Rp + r (h < G) of key head g; this CTA takes rho in
+// [128 * half, 128 * half + 128), one thread per row (TMEM lane). Per tile j of 64 tokens:
 //   TMA    K(j), V(j) into two-stage rings
-//   MMA    S(j) = Q K(j)^T into one of two TMEM buffers; O += P(j - 1) V(j - 1)
-//   rows   S(j) -> m, P(j) = bf16(2^(s - m)) into one of two shared-memory buffers
-// so the rows' exponentials of tile j overlap the tensor cores' P V of tile j - 1.
-__global__ void __launch_bounds__(kAtThreads, 1)
+//   MMA    S(j) = Q K(j)^T into one of two TMEM buffers (64 columns) as soon as K(j) is in
+//          and the buffer is read out; O += P(j) V(j) once P(j) is written (event loop)
+//   rows   S(j) -> m, P(j) = bf16(2^(s - m)) into shared memory, l; the running maximum
+//          raised only past 8 (log2), then O and l rescaled in TMEM
+// The second CTA on the SM fills the gaps of each CTA's chain of dependent steps.
+__global__ void __launch_bounds__(256, 2)
     k_fw_attn(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
               const AttnJob J) {
-  extern __shared__ unsigned char sm_raw[];
-  __shared__ AtBars S;
-  unsigned char* sm = reinterpret_cast<unsigned char*>(
-      (reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  extern __shared__ __align__(1024) unsigned char sm[];
   unsigned char* qs = sm;                        // A operand of S = Q K^T: 128 rows x 128 dims
-  unsigned char* ps = qs + kAtTileBytes;         // 2 x A operand of O += P V: rows x tokens
-  unsigned char* kr = ps + 2 * kAtTileBytes;     // 2 key stages
+  unsigned char* ps = qs + kAtQBytes;            // A operand of O += P V: 128 rows x 64 tokens
+  unsigned char* kr = ps + kAtPBytes;            // 2 key stages
   unsigned char* vr = kr + 2 * kAtTileBytes;     // 2 value stages
+  AtBars& S = *reinterpret_cast<AtBars*>(vr + 2 * kAtTileBytes);
   const int chunk = blockIdx.x, half = blockIdx.y, g = blockIdx.z;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if ((smem_u32(sm) & 1023u) != 0u) {             // the swizzled tiles need the boundary
+    if (threadIdx.x == 0) atomicOr(J.status, kStatusInternal);
+    return;
+  }
   const int T = (J.n_tok + kAtTile - 1) / kAtTile;
   const int t0 = (int)((int64_t)T * chunk / J.chunks);
   const int t1 = (int)((int64_t)T * (chunk + 1) / J.chunks);
   const int n = t1 - t0;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   volatile int* abort = &S.abort;
   if (threadIdx.x == 0) {
     for (int b = 0; b < 2; ++b) {
@@ -446,17 +441,17 @@ __global__ void __launch_bounds__(kAtThreads, 1)
       mbar_init(smem_u32(&S.vfull[b]), 1);
       mbar_init(smem_u32(&S.vempty[b]), 1);
       mbar_init(smem_u32(&S.sfull[b]), 1);
-      mbar_init(smem_u32(&S.sempty[b]), kAtEpi);
-      mbar_init(smem_u32(&S.pfull[b]), kAtEpi);
-      mbar_init(smem_u32(&S.pvdone[b]), 1);
+      mbar_init(smem_u32(&S.sempty[b]), 128);
     }
+    mbar_init(smem_u32(&S.pfull), 128);
+    mbar_init(smem_u32(&S.pvdone), 1);
     mbar_init(smem_u32(&S.q_ready), 1);
     mbar_init(smem_u32(&S.final_mma), 1);
     S.abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 1) {
-    tmem_alloc(smem_u32(&S.taddr), 512);   // S in columns 0-255 (two buffers), O at 256
+    tmem_alloc(smem_u32(&S.taddr), 256);   // S in columns 0-127 (two buffers), O at 128
     tmem_relinquish();
   }
   tc_fence_before();
@@ -497,9 +492,9 @@ __global__ void __launch_bounds__(kAtThreads, 1)
     // ---- MMA issuer, an event loop over two queues: S(j1) = Q K(j1)^T as soon as its
     // keys are in and its TMEM buffer is read out, O += P(j2) V(j2) as soon as its weights
     // are written (non-blocking tests, so neither queue holds back the other) ----
-    const uint32_t id1 = idesc_bf16_f32(128, 128, false, false);
+    const uint32_t id1 = idesc_bf16_f32(128, kAtTile, false, false);
     const uint32_t id2 = idesc_bf16_f32(128, 128, false, true);
-    const uint32_t qa = smem_u32(qs);
+    const uint32_t qa = smem_u32(qs), pa = smem_u32(ps);
     if (fw_wait(smem_u32(&S.q_ready), 0, abort)) {
       int j1 = 0, j2 = 0;
       uint64_t t_idle = 0;
@@ -513,11 +508,13 @@ __global__ void __launch_bounds__(kAtThreads, 1)
           if (ready) {
             tc_fence_after();
             const uint32_t ka = smem_u32(kr + st * kAtTileBytes);
-            const uint32_t d = tbase + (uint32_t)st * 128u;
+            const uint32_t d = tbase + (uint32_t)st * 64u;
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
-              const uint32_t ko = (k >> 2) * 16384 + (k & 3) * 32;
-              umma_bf16(d, sdesc_sw128(qa + ko, 16, 1024), sdesc_sw128(ka + ko, 16, 1024), id1,
+              // Q: two 64-dim halves 16 KB apart; K tile: two 64-dim halves 8 KB apart
+              const uint32_t qo = (k >> 2) * 16384 + (k & 3) * 32;
+              const uint32_t ko = (k >> 2) * (kAtTileBytes / 2) + (k & 3) * 32;
+              umma_bf16(d, sdesc_sw128(qa + qo, 16, 1024), sdesc_sw128(ka + ko, 16, 1024), id1,
                         k > 0 ? 1u : 0u);
             }
             umma_commit(smem_u32(&S.sfull[st]));
@@ -528,21 +525,20 @@ __global__ void __launch_bounds__(kAtThreads, 1)
         }
         if (j2 < j1) {
           const int st = j2 & 1;
-          if (mbar_test_wait(smem_u32(&S.pfull[st]), (j2 >> 1) & 1) &&
+          if (mbar_test_wait(smem_u32(&S.pfull), j2 & 1) &&
               mbar_test_wait(smem_u32(&S.vfull[st]), (j2 >> 1) & 1)) {
             tc_fence_after();
             const uint32_t va = smem_u32(vr + st * kAtTileBytes);
-            const uint32_t pa = smem_u32(ps + st * kAtTileBytes);
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-              // P: K-major, tokens in two 64-token halves; V: N = dims MN-major (two 64-dim
-              // blocks 16 KB apart), 16 tokens = 2048 bytes per K step
-              const uint32_t pk = (k >> 2) * 16384 + (k & 3) * 32;
-              umma_bf16(tbase + 256u, sdesc_sw128(pa + pk, 16, 1024),
-                        sdesc_sw128(va + k * 2048, 16384, 1024), id2, (j2 > 0 || k > 0) ? 1u : 0u);
+            for (int k = 0; k < 4; ++k) {
+              // P: K-major, 64 tokens in one 128-byte row; V: N = dims MN-major (two 64-dim
+              // blocks 8 KB apart), 16 tokens = 2048 bytes per K step
+              umma_bf16(tbase + 128u, sdesc_sw128(pa + k * 32, 16, 1024),
+                        sdesc_sw128(va + k * 2048, kAtTileBytes / 2, 1024), id2,
+                        (j2 > 0 || k > 0) ? 1u : 0u);
             }
             umma_commit(smem_u32(&S.vempty[st]));
-            umma_commit(smem_u32(&S.pvdone[st]));
+            umma_commit(smem_u32(&S.pvdone));
             ++j2;
             did = true;
           }
@@ -563,10 +559,9 @@ __global__ void __launch_bounds__(kAtThreads, 1)
     umma_commit(smem_u32(&S.final_mma));
     mbar_wait_bounded(smem_u32(&S.final_mma), 0);
   } else if (warp >= 2) {
-    // ---- rows: two threads per row (TMEM lane), 64 columns each ----
+    // ---- rows: one per thread (TMEM lane) ----
     const int e = threadIdx.x - 64;
-    const int qd = warp & 3;                       // TMEM lane quarter
-    const int ch = (warp - 2) >> 2;                // column half: tokens / dims 64 ch .. + 63
+    const int qd = warp & 3;
     const int rl = qd * 32 + lane;                 // row within the CTA's 128
     const int rho = half * 128 + rl;
     const int hl = rho / J.Rp, r = rho - hl * J.Rp;
@@ -574,7 +569,7 @@ __global__ void __launch_bounds__(kAtThreads, 1)
     // (the keys and values stream in meanwhile: they do not depend on the previous kernel)
     pdl_wait();
     // question rows -> 128-byte swizzled K-major tile (two halves of 64 dims)
-    for (int x = e; x < 128 * 16; x += kAtEpi) {
+    for (int x = e; x < 128 * 16; x += 128) {
       const int row = x >> 4, c = x & 15;
       const int rr = half * 128 + row;
       const int h2 = rr / J.Rp, r2 = rr - h2 * J.Rp;
@@ -585,58 +580,42 @@ __global__ void __launch_bounds__(kAtThreads, 1)
       *reinterpret_cast<uint4*>(qs + (c >> 3) * 16384 + row * 128 + (((c & 7) ^ (row & 7)) << 4)) = v;
     }
     fence_proxy_async_smem();
-    fw_bar(1, kAtEpi);
+    fw_bar(1, 128);
     if (e == 0) mbar_arrive(smem_u32(&S.q_ready));
     const uint32_t la = tbase + ((uint32_t)(qd * 32) << 16);
-    const uint32_t sc = (uint32_t)(64 * ch);       // this thread's columns within S and O
-    float* xm = S.xchg[ch];                        // the pair's exchange slots
-    float* xo = S.xchg[ch ^ 1];
+    unsigned char* prow = ps + rl * 128;
+    const unsigned long long sc2 = f2pack(kScoreScale, kScoreScale);
     float m = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < n; ++j) {
       const int st = j & 1;
       ok = ok && fw_wait(smem_u32(&S.sfull[st]), (j >> 1) & 1, abort);
       ok = __all_sync(0xffffffffu, ok);
-      float s[64];
-      if (ok) {
-        tc_fence_after();
-        tmem_ld32x2(la + st * 128u + sc, la + st * 128u + sc + 32u,
-                    *reinterpret_cast<float(*)[32]>(s), *reinterpret_cast<float(*)[32]>(s + 32));
-        tc_fence_before();
-        mbar_arrive(smem_u32(&S.sempty[st]));
-      }
-      const int nv = min(kAtTile, J.n_tok - (t0 + j) * kAtTile) - 64 * ch;   // valid columns
-      float mt = -INFINITY;
-      if (ok) {
-        if (nv < 64) {
-#pragma unroll
-          for (int c = 0; c < 64; ++c)
-            if (c >= nv) s[c] = -INFINITY;
-        }
-        float a0 = -INFINITY, a1 = -INFINITY;
-#pragma unroll
-        for (int c = 0; c < 64; c += 4) {
-          a0 = fmax3(a0, s[c], s[c + 1]);
-          a1 = fmax3(a1, s[c + 2], s[c + 3]);
-        }
-        mt = fmaxf(a0, a1) * kScoreScale;
-      }
-      // the P buffer is free once O += P(j - 2) V(j - 2) has completed
-      if (ok && j >= 2) {
-        ok = fw_wait(smem_u32(&S.pvdone[st]), ((j - 2) >> 1) & 1, abort);
-        ok = __all_sync(0xffffffffu, ok);
-      }
-      // the pair agrees on the tile maximum and on going on (a barrier that also ANDs ok)
-      xm[rl] = mt;
-      ok = pair_sync_and(qd, ok);
       if (!ok) break;
-      mt = fmaxf(mt, xo[rl]);
+      tc_fence_after();
+      float s[64];
+      tmem_ld32x2(la + st * 64u, la + st * 64u + 32u, *reinterpret_cast<float(*)[32]>(s),
+                  *reinterpret_cast<float(*)[32]>(s + 32));
+      tc_fence_before();
+      mbar_arrive(smem_u32(&S.sempty[st]));
+      const int nv = min(kAtTile, J.n_tok - (t0 + j) * kAtTile);   // valid tokens
+      if (nv < kAtTile) {
+#pragma unroll
+        for (int c = 0; c < kAtTile; ++c)
+          if (c >= nv) s[c] = -INFINITY;
+      }
+      float a0 = -INFINITY, a1 = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < kAtTile; c += 4) {
+        a0 = fmax3(a0, s[c], s[c + 1]);
+        a1 = fmax3(a1, s[c + 2], s[c + 3]);
+      }
+      const float mt = fmaxf(a0, a1) * kScoreScale;
       const bool raise = mt > m + kAtLazy;
       const float m_new = raise ? mt : m;
       // P = 2^(s - m_new) rounded to bf16 for the tensor cores; the scaling and l (the sum
       // of the weights before rounding) on packed pairs
       uint32_t pk[32];
-      const unsigned long long sc2 = f2pack(kScoreScale, kScoreScale);
       const unsigned long long nm2 = f2pack(-m_new, -m_new);
       unsigned long long acc0 = 0ull, acc1 = 0ull;
 #pragma unroll
@@ -648,32 +627,29 @@ __global__ void __launch_bounds__(kAtThreads, 1)
         if (c & 1) acc1 = fadd2(acc1, f2pack(p0, p1));
         else acc0 = fadd2(acc0, f2pack(p0, p1));
       }
-      const float lt0 = f2lo(acc0), lt1 = f2hi(acc0), lt2 = f2lo(acc1), lt3 = f2hi(acc1);
-      // a raised maximum rescales O (and l) once O += P(j - 1) V(j - 1) has completed (the
-      // two warps of a pair hold the same rows, so both take this branch or neither)
-      const bool any_raise = __any_sync(0xffffffffu, raise) && j >= 1;
-      if (any_raise) {
-        bool w_ok = fw_wait(smem_u32(&S.pvdone[st ^ 1]), ((j - 1) >> 1) & 1, abort);
-        w_ok = __all_sync(0xffffffffu, w_ok);
-        ok = pair_sync_and(qd, w_ok);
+      // the P buffer and O are free once O += P(j - 1) V(j - 1) has completed; a raised
+      // maximum then rescales O (and l)
+      if (j >= 1) {
+        ok = fw_wait(smem_u32(&S.pvdone), (j - 1) & 1, abort);
+        ok = __all_sync(0xffffffffu, ok);
         if (!ok) break;
-      }
-      const float fac = raise ? fast_exp2(m - m_new) : 1.0f;
-      if (any_raise) {
         tc_fence_after();
+        if (__any_sync(0xffffffffu, raise)) {
+          const float fac = raise ? fast_exp2(m - m_new) : 1.0f;
 #pragma unroll 1
-        for (int c0 = 0; c0 < 64; c0 += 32) {
-          float o[32];
-          tmem_ld32(la + 256u + sc + (uint32_t)c0, o);
+          for (int c0 = 0; c0 < 128; c0 += 32) {
+            float o[32];
+            tmem_ld32(la + 128u + (uint32_t)c0, o);
 #pragma unroll
-          for (int c = 0; c < 32; ++c) o[c] *= fac;
-          tmem_st32(la + 256u + sc + (uint32_t)c0, o);
+            for (int c = 0; c < 32; ++c) o[c] *= fac;
+            tmem_st32(la + 128u + (uint32_t)c0, o);
+          }
+          l *= fac;
         }
       }
-      l = (j >= 1 ? l * fac : 0.f) + ((lt0 + lt1) + (lt2 + lt3));
       m = m_new;
-      // this thread's 64 tokens of the P row: the half ch of the K-major operand
-      unsigned char* prow = ps + st * kAtTileBytes + ch * 16384 + rl * 128;
+      l += (f2lo(acc0) + f2hi(acc0)) + (f2lo(acc1) + f2hi(acc1));
+      // the P row: 64 tokens in 128 bytes, 16-byte chunks swizzled
 #pragma unroll
       for (int c = 0; c < 8; ++c) {
         const uint4 w = make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
@@ -681,36 +657,32 @@ __global__ void __launch_bounds__(kAtThreads, 1)
       }
       fence_proxy_async_smem();
       tc_fence_before();
-      mbar_arrive(smem_u32(&S.pfull[st]));
+      mbar_arrive(smem_u32(&S.pfull));
     }
     if (ok && n > 0) {
-      ok = fw_wait(smem_u32(&S.pvdone[(n - 1) & 1]), ((n - 1) >> 1) & 1, abort);
+      ok = fw_wait(smem_u32(&S.pvdone), (n - 1) & 1, abort);
       ok = __all_sync(0xffffffffu, ok);
     }
-    // the row's l is the pair's sum
-    xm[rl] = l;
-    ok = pair_sync_and(qd, ok);
     tc_fence_after();
     const int64_t prow_out = ((int64_t)g * J.chunks + chunk) * (J.halves * 128) + rho;
     if (ok && !*abort) {
-      for (int c0 = 0; c0 < 64; c0 += 32) {
+      for (int c0 = 0; c0 < 128; c0 += 32) {
         float o[32];
-        tmem_ld32(la + 256u + sc + (uint32_t)c0, o);
+        tmem_ld32(la + 128u + (uint32_t)c0, o);
         if (valid && n > 0) {
-          float4* dst = reinterpret_cast<float4*>(J.opart + prow_out * kHeadDim + sc + c0);
+          float4* dst = reinterpret_cast<float4*>(J.opart + prow_out * kHeadDim + c0);
 #pragma unroll
           for (int c = 0; c < 8; ++c) dst[c] = make_float4(o[4 * c], o[4 * c + 1], o[4 * c + 2], o[4 * c + 3]);
         }
       }
-      if (valid && ch == 0)
-        J.mlpart[prow_out] = n > 0 ? make_float2(m, l + xo[rl]) : make_float2(-INFINITY, 0.f);
+      if (valid) J.mlpart[prow_out] = n > 0 ? make_float2(m, l) : make_float2(-INFINITY, 0.f);
     }
   }
   tc_fence_before();
   __syncthreads();
   if (threadIdx.x == 0 && S.abort) atomicOr(J.status, kStatusTimeout);
   tc_fence_after();
-  if (warp == 1) tmem_dealloc(tbase, 512);
+  if (warp == 1) tmem_dealloc(tbase, 256);
 }
 
 struct AttnOutJob {
@@ -861,7 +833,7 @@ FwLayout fw_layout(const FwShape& F) {
   const int G = F.Hq / F.Hkv;
   L.halves = (G * L.Rp + 127) / 128;
   const int T = (F.n_tok + kAtTile - 1) / kAtTile;
-  int c = F.sm_count / (L.halves * F.Hkv);
+  int c = 2 * F.sm_count / (L.halves * F.Hkv);   // two attention CTAs per SM
   c = c < 1 ? 1 : c;
   L.chunks = T < 1 ? 1 : (T < c ? T : c);
   const int nqkv = (F.Hq + 2 * F.Hkv) * kHeadDim;
