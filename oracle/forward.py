@@ -80,12 +80,13 @@ def silu(x: np.ndarray) -> np.ndarray:
 
 
 def attention(q: np.ndarray, hist_k: np.ndarray, hist_v: np.ndarray,
-              own_k: np.ndarray, own_v: np.ndarray, spread: bool = False):
+              own_k: np.ndarray, own_v: np.ndarray, spread=False):
     """q [R][Hq][d]; hist_k, hist_v [Hkv][N][d] (the layer's stored tokens); own_k, own_v
     [R][Hkv][d] (the question's rows). Row r of head h attends to the N stored tokens of
     key head h // G and to the question's rows 0..r. Returns o [R][Hq][d] (fp64); with
     spread=True also sum_j p_j |v_j - o| per element (how far a change of the weights by a
-    relative e can move o: at most e times this)."""
+    relative e can move o: at most e times this); with spread="upper" the bound
+    sum_j p_j |v_j| + |o| of it instead (one product per head, for long histories)."""
     R, Hq, d = q.shape
     Hkv = hist_k.shape[0]
     G = Hq // Hkv
@@ -102,7 +103,9 @@ def attention(q: np.ndarray, hist_k: np.ndarray, hist_v: np.ndarray,
         p = np.exp(s - s.max(axis=1, keepdims=True))
         p /= p.sum(axis=1, keepdims=True)
         out[:, h] = p @ vals
-        if spread:
+        if spread == "upper":
+            spr[:, h] = p @ np.abs(vals) + np.abs(out[:, h])
+        elif spread:
             for r in range(R):
                 spr[r, h] = p[r] @ np.abs(vals - out[r, h][None, :])
     return (out, spr) if spread else out
@@ -110,7 +113,7 @@ def attention(q: np.ndarray, hist_k: np.ndarray, hist_v: np.ndarray,
 
 def layer(h: np.ndarray, w: dict, hist_k_bits: np.ndarray, hist_v_bits: np.ndarray,
           *, n_q_heads: int, n_kv_heads: int, pos0: int, eps: float, theta: float,
-          with_spread: bool = False) -> dict:
+          with_spread=False) -> dict:
     """One shallow layer F^i (Eq. 10). h [R][D] (fp64 hidden states). w: bf16 bit arrays
     ln1 [D], wqkv [(Hq + 2 Hkv) d][D], bqkv [(Hq + 2 Hkv) d] or None, wo [D][Hq d],
     ln2 [D], wgu [2 I][D] (gate rows, then up rows), wd [D][I]. hist_k_bits,

@@ -302,3 +302,38 @@ def test_forward_errors():
     small = torch.zeros(64, dtype=torch.uint8, device="cuda")
     with pytest.raises(ss.ShallowStreamError, match="CAPACITY"):
         idx.forward(layers, h_in.cuda(), params, workspace=small)
+
+
+def test_one_hour_layer_at_full_size():
+    """The bench's shapes: one layer of the 1-hour stream (705,600 stored tokens per key
+    head, G 7, R 32, MLP width 18944) in the launch configuration of the forward; q within
+    its band and the attention output of every row and head within the bound of the bf16
+    attention weights (with the per-row spread bounded by sum_j p_j |v_j| + |o|)."""
+    ss = _ss()
+    syn = _synth()
+    w = syn.PRESETS["hour1_fwd"]
+    dev = torch.device("cuda")
+    keys = syn.make_keys(w, syn.make_queries(w, device=dev), device=dev)[0:1].contiguous()
+    vals = syn.make_values(w, device=dev)[0:1].contiguous()
+    I = w.extra["intermediate"]
+    w1 = w.replace(n_layers=1)
+    layers = _unit_norm_weights(_attention_layers(syn.make_forward_weights(w1, I)))
+    h_in = _exact_norm_rows(w.n_rows, 28 * 128, seed=36)
+    idx = ss.Index(1, 28, 4, w.tokens_per_frame, w.n_frames, device=dev)
+    idx.append(keys)
+    idx.append_values(vals)
+    params = ss.ForwardParams(I, EXACT_EPS, 1e6)
+    qb, h = _run(idx, layers, h_in, params)
+    hb = to_bits(h_in)
+    N = w.n_frames * w.tokens_per_frame
+    npw = _np_weights(layers)[0]
+    ref = FW.layer(bf16_to_f64(hb), npw, to_bits(keys[0]), to_bits(vals[0]), n_q_heads=28,
+                   n_kv_heads=4, pos0=N, eps=EXACT_EPS, theta=1e6, with_spread="upper")
+    n_q = _check_q(qb[0], ref["q_pre"], _q_scale(ref, npw, 28))
+    o_gpu = h - bf16_to_f64(hb)
+    tol = (2.0 ** -7 * (ref["o_spread"] + np.abs(ref["o_pre"])) * 1.01 +
+           0.5 * _bf16_step(ref["o_pre"]) * 1.01 + 1e-7)
+    err = np.abs(o_gpu - ref["o_pre"])
+    assert (err <= tol).all(), f"attention output off by {(err / tol).max():.2f} x its bound"
+    print(f"full size: q elements at a rounding boundary {n_q}; o error / bound max "
+          f"{(err / tol).max():.3f}, median {np.median(err / tol):.4f}")

@@ -254,3 +254,15 @@ def test_planted_mistakes_fail_the_library_comparison(monkeypatch):
         bad = FW.layer(h, w, hk, hv, n_q_heads=Hq, n_kv_heads=Hkv, pos0=N, eps=1e-6,
                        theta=1e4)
         assert np.abs(bad["o"] - lib["o"].numpy()).max() > 1e-3
+
+
+def test_spread_upper_bound_holds():
+    rng = np.random.default_rng(8)
+    R, Hq, Hkv, d, N = 4, 4, 2, 8, 50
+    q = rng.standard_normal((R, Hq, d))
+    hk, hv = rng.standard_normal((Hkv, N, d)), rng.standard_normal((Hkv, N, d))
+    ok, ov = rng.standard_normal((R, Hkv, d)), rng.standard_normal((R, Hkv, d))
+    o1, exact = FW.attention(q, hk, hv, ok, ov, spread=True)
+    o2, upper = FW.attention(q, hk, hv, ok, ov, spread="upper")
+    np.testing.assert_array_equal(o1, o2)
+    assert (upper >= exact - 1e-12).all() and (exact > 0).all()
