@@ -160,19 +160,28 @@ __device__ __forceinline__ void rm_chunk(const Prob& P, int chunks, int c, int& 
 
 // ---------------------------------------------------------------------------
 // Pass 1: per-row (max, sum) of the log2-scaled scores over the chunk's tokens.
-// Warps: 0 TMA, 1 MMA (+ TMEM), then 4 per 128-row block (NMB blocks).
+// Warps: 0 TMA, 1 MMA (+ TMEM), then 4 per (128-row block, column part): NMB blocks,
+// each tile's 128 token columns split in CS parts, every part keeping its own (max, sum)
+// per row, combined in part order at the end.
 // ---------------------------------------------------------------------------
-template <int NMB>
-__global__ void __launch_bounds__(64 + 128 * NMB, 1)
+// Launch bound: the block's threads rounded up to whole groups of four warps (the unit
+// in which a block's registers are allocated).
+constexpr int rm_bound(int threads) { return (threads + 127) / 128 * 128; }
+
+template <int NMB, int CS>
+__global__ void __launch_bounds__(rm_bound(64 + 128 * NMB * CS), 1)
     k_rm_stats(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ Batch B,
                const RmJob J) {
   extern __shared__ unsigned char sm_raw[];
   __shared__ RmBars S;
+  __shared__ float2 part_s[(CS > 1 ? CS - 1 : 1) * NMB * 128];
   unsigned char* sm = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   unsigned char* qs = sm;                                // NMB x 32 KB
   unsigned char* ring = qs + NMB * 32768;
-  constexpr int n_epi = 128 * NMB;
+  constexpr int n_epi = 128 * NMB * CS;
+  constexpr int CW = kRmTile / CS;                       // columns of a part
+  constexpr int PW = CW >= 64 ? 64 : 32;                 // columns per TMEM load
   const int nbuf = J.nbuf, stages = J.stages;
   const uint32_t cols = nbuf * NMB * 128 <= 256 ? 256u : 512u;
   rm_init(S, stages, nbuf, n_epi, cols);
@@ -206,82 +215,104 @@ __global__ void __launch_bounds__(64 + 128 * NMB, 1)
   } else {
     pdl_release();
     const int e = threadIdx.x - 64;
-    const int b = e >> 7, q = warp & 3;
+    const int grp = e >> 7, b = grp % NMB, cp = grp / NMB, q = warp & 3;
     const int rho = b * 128 + q * 32 + lane;            // this thread's row
+    const int c0 = cp * CW;                             // its first token column
+    const int h = rho / J.Rp, r = rho - h * J.Rp;
+    const bool row_ok = h < P.G && r < P.R;
+    // a warp whose 32 rows are all padding only keeps the pipeline's count
+    const bool live = __any_sync(0xffffffffu, row_ok);
     // the slab's question rows (written before the wait: inputs only)
     rm_load_q(P, slab, J.Rp, NMB * 128, 128, qs, e, n_epi);
     fence_proxy_async_smem();
     rm_bar(n_epi);
     if (e == 0) mbar_arrive(smem_u32(&S.q_ready));
     const uint32_t lane_addr = tbase + ((uint32_t)(q * 32) << 16);
+    const unsigned long long sc2 = f2pack(kScoreScale, kScoreScale);
     float m = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < n_tiles; ++j) {
       const int buf = j % nbuf;
       ok = ok && rm_wait(smem_u32(&S.d_full[buf]), (j / nbuf) & 1, abort);
       tc_fence_after();
-      if (ok) {
-        const uint32_t d = lane_addr + (uint32_t)(buf * NMB + b) * 128u;
-        const int nv = min(kRmTile, n_tok - (t0 + j) * kRmTile);   // valid tokens
-        // the tile's 128 token columns in two halves of 64 (online update per half)
+      if (ok && live) {
+        const uint32_t d = lane_addr + (uint32_t)(buf * NMB + b) * 128u + (uint32_t)c0;
+        const int nv = min(kRmTile, n_tok - (t0 + j) * kRmTile) - c0;   // valid columns
+        // the part's columns PW at a time (online update per load); pairs (a[c], b[c])
+        // of the loaded columns go through the packed fp32x2 path
 #pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
+        for (int pc = 0; pc < CW; pc += PW) {
           float v0[32], v1[32];
-          tmem_ld32x2(d + 64 * hh, d + 64 * hh + 32, v0, v1);
-          // (a full tile needs no per-column test; the max is taken on the raw dot
-          // products and scaled once)
+          if constexpr (PW == 64) tmem_ld32x2(d + pc, d + pc + 32, v0, v1);
+          else tmem_ld32(d + pc, v0);
+          constexpr int NP = PW / 2;                    // packed pairs
+          auto A = [&](int c) -> float { return v0[c]; };
+          auto Bv = [&](int c) -> float {
+            if constexpr (PW == 64) return v1[c];
+            else return v0[16 + c];
+          };
           float mt = -INFINITY;
-          if (nv == kRmTile) {
+          if (nv >= pc + PW) {
+            // (a full load needs no per-column test; the max is taken on the raw dot
+            // products and scaled once)
             float a0 = -INFINITY, a1 = -INFINITY;
 #pragma unroll
-            for (int c = 0; c < 32; c += 2) {
-              a0 = fmax3(a0, v0[c], v0[c + 1]);
-              a1 = fmax3(a1, v1[c], v1[c + 1]);
+            for (int c = 0; c < NP; c += 2) {
+              a0 = fmax3(a0, A(c), A(c + 1));
+              a1 = fmax3(a1, Bv(c), Bv(c + 1));
             }
-            mt = fmaxf(a0, a1);
-          } else {
-#pragma unroll
-            for (int c = 0; c < 32; ++c) {
-              if (64 * hh + c < nv) mt = fmaxf(mt, v0[c]);
-              if (64 * hh + 32 + c < nv) mt = fmaxf(mt, v1[c]);
+            mt = fmaxf(a0, a1) * kScoreScale;
+            if (mt > m) {
+              l = (m == -INFINITY) ? 0.f : l * fast_exp2(m - mt);
+              m = mt;
             }
-          }
-          mt *= kScoreScale;
-          if (mt > m) {
-            l = (m == -INFINITY) ? 0.f : l * fast_exp2(m - mt);
-            m = mt;
-          }
-          float acc0 = 0.f, acc1 = 0.f;
-          if (nv == kRmTile) {
-            // the scaling and the sums on packed pairs (columns c and 32 + c)
-            const unsigned long long sc2 = f2pack(kScoreScale, kScoreScale);
             const unsigned long long nm2 = f2pack(-m, -m);
             unsigned long long p0 = 0ull, p1 = 0ull;
 #pragma unroll
-            for (int c = 0; c < 32; ++c) {
-              const unsigned long long x = ffma2(f2pack(v0[c], v1[c]), sc2, nm2);
-              const unsigned long long e = f2pack(fast_exp2(f2lo(x)), fast_exp2(f2hi(x)));
-              if (c & 1) p1 = fadd2(p1, e);
-              else p0 = fadd2(p0, e);
+            for (int c = 0; c < NP; ++c) {
+              const unsigned long long x = ffma2(f2pack(A(c), Bv(c)), sc2, nm2);
+              const unsigned long long ex = f2pack(fast_exp2(f2lo(x)), fast_exp2(f2hi(x)));
+              if (c & 1) p1 = fadd2(p1, ex);
+              else p0 = fadd2(p0, ex);
             }
-            acc0 = f2lo(p0) + f2lo(p1);
-            acc1 = f2hi(p0) + f2hi(p1);
-          } else {
+            l += (f2lo(p0) + f2lo(p1)) + (f2hi(p0) + f2hi(p1));
+          } else if (nv > pc) {
+            // the ragged last tile: column pc + c of A, pc + NP + c of Bv
 #pragma unroll
-            for (int c = 0; c < 32; ++c) {
-              if (64 * hh + c < nv) acc0 += fast_exp2(fmaf(v0[c], kScoreScale, -m));
-              if (64 * hh + 32 + c < nv) acc1 += fast_exp2(fmaf(v1[c], kScoreScale, -m));
+            for (int c = 0; c < NP; ++c) {
+              if (pc + c < nv) mt = fmaxf(mt, A(c));
+              if (pc + NP + c < nv) mt = fmaxf(mt, Bv(c));
             }
+            mt *= kScoreScale;
+            if (mt > m) {
+              l = (m == -INFINITY) ? 0.f : l * fast_exp2(m - mt);
+              m = mt;
+            }
+            float acc = 0.f;
+#pragma unroll
+            for (int c = 0; c < NP; ++c) {
+              if (pc + c < nv) acc += fast_exp2(fmaf(A(c), kScoreScale, -m));
+              if (pc + NP + c < nv) acc += fast_exp2(fmaf(Bv(c), kScoreScale, -m));
+            }
+            l += acc;
           }
-          l += acc0 + acc1;
         }
       }
       tc_fence_before();
       mbar_arrive(smem_u32(&S.epi_done[buf]));
     }
-    const int h = rho / J.Rp, r = rho - h * J.Rp;
+    // the column parts of a row, combined in part order
+    if constexpr (CS > 1) {
+      if (cp > 0) part_s[(cp - 1) * (NMB * 128) + rho] = make_float2(m, l);
+      rm_bar(n_epi);
+      if (cp == 0)
+        for (int c = 1; c < CS; ++c) {
+          const float2 v = part_s[(c - 1) * (NMB * 128) + rho];
+          if (v.y > 0.f) ml_combine(m, l, v.x, v.y);
+        }
+    }
     pdl_wait();   // the previous kernel of the call (its resets) has completed
-    if (ok && !*abort && h < P.G && r < P.R)
+    if (cp == 0 && ok && !*abort && row_ok)
       J.part[((int64_t)slab * J.GRp + rho) * J.chunks + chunk] = make_float2(m, l);
   }
   tc_fence_before();
@@ -315,11 +346,12 @@ __global__ void __launch_bounds__(256) k_rm_combine(const __grid_constant__ Batc
 
 // ---------------------------------------------------------------------------
 // Pass 2: alpha of every history token of the chunk for the slab's G lists.
-// Warps: 0 TMA, 1 MMA (+ TMEM), 2-9 epilogue (two groups of four, heads split).
+// Warps: 0 TMA, 1 MMA (+ TMEM), 2-17 epilogue (four groups of four, heads split).
 // ---------------------------------------------------------------------------
-constexpr int kRmEpi2 = 256;
+constexpr int kRmEpi2 = 512;
+constexpr int kRmGroups2 = kRmEpi2 / 128;
 
-__global__ void __launch_bounds__(64 + kRmEpi2, 1)
+__global__ void __launch_bounds__(rm_bound(64 + kRmEpi2), 1)
     k_rm_alpha(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ Batch B,
                const RmJob J) {
   extern __shared__ unsigned char sm_raw[];
@@ -382,8 +414,7 @@ __global__ void __launch_bounds__(64 + kRmEpi2, 1)
     rm_bar(kRmEpi2);
     pdl_release();
     const int G = P.G, Rp = J.Rp;
-    const int hh = (G + 1) / 2;                          // heads of group 0
-    const int h_begin = grp ? hh : 0, h_end = grp ? G : hh;
+    const int h_begin = G * grp / kRmGroups2, h_end = G * (grp + 1) / kRmGroups2;
     const int i = slab / P.Hkv, g = slab - i * P.Hkv;
     const float invR = 1.0f / (float)P.R;
     const uint32_t lane_addr = tbase + ((uint32_t)(q * 32) << 16);
@@ -491,11 +522,13 @@ cudaError_t launch_rowmean(const Batch& B, int pi, float2* scratch, int chunks, 
     J.nbuf = nmb <= 2 ? 2 : 1;
     J.stages = nmb <= 2 ? 4 : 2;
     const size_t smem = 1024 + (size_t)nmb * 32768 + (size_t)J.stages * kRmStageBytes;
-    auto kern = nmb == 1 ? k_rm_stats<1> : nmb == 2 ? k_rm_stats<2> : nmb == 3 ? k_rm_stats<3>
-                                                                              : k_rm_stats<4>;
+    // column parts: up to 16 epilogue warps per CTA
+    const int cs = nmb == 1 ? 4 : nmb == 2 ? 2 : 1;
+    auto kern = nmb == 1 ? k_rm_stats<1, 4> : nmb == 2 ? k_rm_stats<2, 2>
+              : nmb == 3 ? k_rm_stats<3, 1> : k_rm_stats<4, 1>;
     e = ensure_smem((const void*)kern, (int)smem);
     if (e != cudaSuccess) return e;
-    e = launch_pdl(kern, dim3(chunks, n_slabs), dim3(64 + 128 * nmb), smem, s, map, B, J);
+    e = launch_pdl(kern, dim3(chunks, n_slabs), dim3(64 + 128 * nmb * cs), smem, s, map, B, J);
     if (e != cudaSuccess) return e;
   }
   e = launch_pdl(k_rm_combine, dim3((n_slabs * GRp + 255) / 256), dim3(256), 0, s, B, J);

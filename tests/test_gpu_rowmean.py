@@ -74,6 +74,17 @@ def test_sixty_four_rows_two_operand_tiles():
     _case(62, P=1, Hq=14, Hkv=2, F=30, Tf=64, R_rows=64, k=100, budget=4)
 
 
+def test_forty_eight_rows_three_row_blocks():
+    # R = 48, G = 7: 336 rows, three row blocks in pass 1, two B tiles of 176 in pass 2
+    _case(65, P=1, Hq=14, Hkv=2, F=30, Tf=50, R_rows=48, k=80, budget=4)
+
+
+def test_twenty_rows_padding_inside_every_head():
+    # R = 20 (padded to 32): 12 padding rows inside each head's 32, two row blocks, the
+    # last warp of the second block padding only
+    _case(66, P=2, Hq=28, Hkv=4, F=24, Tf=61, R_rows=20, k=90, budget=4, n_recent=2)
+
+
 def test_group_of_eight_with_sixty_four_rows():
     # G = 8, R = 64: 512 rows, the largest supported
     _case(63, P=1, Hq=8, Hkv=1, F=24, Tf=50, R_rows=64, k=64, budget=3)
