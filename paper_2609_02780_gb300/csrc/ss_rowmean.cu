@@ -347,16 +347,30 @@ __global__ void __launch_bounds__(256) k_rm_combine(const __grid_constant__ Batc
 // ---------------------------------------------------------------------------
 // Pass 2: alpha of every history token of the chunk for the slab's G lists.
 // Warps: 0 TMA, 1 MMA (+ TMEM), 2-17 epilogue (four groups of four, heads split).
+// Each row's exponent offset enters the accumulator through one more MMA K step: A' (the
+// tokens, MN-major) is 1 in K columns 0-2, B' (the rows, MN-major) holds minus the row's
+// offset / scale split into three bf16 parts, so D = s - offset / scale and the epilogue
+// needs no per-row constants (no shared-memory loads next to the tensor cores' reads).
 // ---------------------------------------------------------------------------
 constexpr int kRmEpi2 = 512;
 constexpr int kRmGroups2 = kRmEpi2 / 128;
+constexpr int kRmXaBytes = 2 * 2048;                   // A': 2 blocks of 64 tokens x 16 K
+
+// Bytes of B' for one operand tile of `ne` rows: blocks of 64 rows x 16 K (2 KB each).
+__host__ __device__ constexpr int rm_xb_bytes(int ne) { return (ne + 63) / 64 * 2048; }
+
+// Element (k, n) of a 128-byte swizzled MN-major operand whose 64-element blocks are
+// 2048 bytes apart (16 K rows of 128 bytes each).
+__device__ __forceinline__ int rm_mn_offset(int k, int n) {
+  return (n >> 6) * 2048 + (k >> 3) * 1024 + (k & 7) * 128 + ((((n >> 3) & 7) ^ (k & 7)) << 4) +
+         (n & 7) * 2;
+}
 
 __global__ void __launch_bounds__(rm_bound(64 + kRmEpi2), 1)
     k_rm_alpha(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ Batch B,
                const RmJob J) {
   extern __shared__ unsigned char sm_raw[];
   __shared__ RmBars S;
-  __shared__ __align__(16) float st[512];   // exponent offset of every row
   unsigned char* sm = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const int GRp = J.GRp;
@@ -365,7 +379,10 @@ __global__ void __launch_bounds__(rm_bound(64 + kRmEpi2), 1)
   const int NE = two ? ((GRp / 2 + 15) & ~15) : GRp;
   unsigned char* qs = sm;
   const int q_bytes = (two ? 2 : 1) * NE * 256;
-  unsigned char* ring = qs + ((q_bytes + 1023) & ~1023);
+  unsigned char* xa = qs + ((q_bytes + 1023) & ~1023);   // A' (kRmXaBytes)
+  unsigned char* xb = xa + kRmXaBytes;                     // B' of each operand tile
+  const int xb_tile = rm_xb_bytes(NE);
+  unsigned char* ring = xb + (((two ? 2 : 1) * xb_tile + 1023) & ~1023);
   const int nbuf = J.nbuf, stages = J.stages;
   const uint32_t cols = nbuf * (two ? 2 * NE : NE) <= 256 ? 256u : 512u;
   rm_init(S, stages, nbuf, kRmEpi2, cols);
@@ -384,6 +401,7 @@ __global__ void __launch_bounds__(rm_bound(64 + kRmEpi2), 1)
                 (int64_t)slab * P.ncap + (int64_t)t0 * kRmTile,
                 [&](int j, uint32_t ks, int buf) {
                   const uint32_t id = idesc_bf16_f32(128, NE, false, false);
+                  const uint32_t idx = idesc_bf16_f32(128, NE, true, true);
                   for (int t = 0; t < 1 + two; ++t) {
                     const uint32_t d = tbase + (uint32_t)buf * buf_cols + (uint32_t)(t * NE);
                     const uint32_t bs = smem_u32(qs + t * NE * 256);
@@ -394,6 +412,9 @@ __global__ void __launch_bounds__(rm_bound(64 + kRmEpi2), 1)
                       umma_bf16(d, sdesc_sw128(ks + ka, 16, 1024), sdesc_sw128(bs + kb, 16, 1024),
                                 id, k > 0 ? 1u : 0u);
                     }
+                    // the offsets: D += A' B'^T
+                    umma_bf16(d, sdesc_sw128(smem_u32(xa), 2048, 1024),
+                              sdesc_sw128(smem_u32(xb + t * xb_tile), 2048, 1024), idx, 1u);
                   }
                   (void)j;
                 });
@@ -402,16 +423,38 @@ __global__ void __launch_bounds__(rm_bound(64 + kRmEpi2), 1)
     const int grp = e >> 7, q = warp & 3;
     const int tl = q * 32 + lane;                        // token lane
     rm_load_q(P, slab, J.Rp, (two ? 2 : 1) * NE, NE, qs, e, kRmEpi2);
+    // A': ones in K columns 0-2 for all 128 tokens, zeros elsewhere; B' zeroed
+    for (int x = e; x < 128 * 16; x += kRmEpi2) {
+      const int k = x >> 7, m = x & 127;
+      *reinterpret_cast<__nv_bfloat16*>(xa + rm_mn_offset(k, m)) =
+          __float2bfloat16_rn(k < 3 ? 1.f : 0.f);
+    }
+    for (int x = e; x < (two ? 2 : 1) * xb_tile / 16; x += kRmEpi2)
+      reinterpret_cast<uint4*>(xb)[x] = make_uint4(0u, 0u, 0u, 0u);
+    rm_bar(kRmEpi2);
+    pdl_wait();                                          // the rows' statistics (pass 1)
+    for (int x = e; x < (two ? 2 : 1) * NE; x += kRmEpi2) {
+      const int t = x / NE, n = x - t * NE;              // operand tile, its row
+      const int hr = x / J.Rp, rr = x - hr * J.Rp;
+      // offset / scale in three bf16 parts (24 significant bits); rows past R (or past
+      // the G heads) get one that takes their terms to 0
+      float v = 1e30f;
+      if (x < GRp && hr < P.G && rr < P.R) {
+        const float o = J.stat[(int64_t)slab * GRp + x].x;
+        if (o < INFINITY) v = o / kScoreScale;
+      }
+      const __nv_bfloat16 b1 = __float2bfloat16_rn(v);
+      const float r1 = v - __bfloat162float(b1);
+      const __nv_bfloat16 b2 = __float2bfloat16_rn(r1);
+      const __nv_bfloat16 b3 = __float2bfloat16_rn(r1 - __bfloat162float(b2));
+      unsigned char* tb = xb + t * xb_tile;
+      *reinterpret_cast<__nv_bfloat16*>(tb + rm_mn_offset(0, n)) = __hneg(b1);
+      *reinterpret_cast<__nv_bfloat16*>(tb + rm_mn_offset(1, n)) = __hneg(b2);
+      *reinterpret_cast<__nv_bfloat16*>(tb + rm_mn_offset(2, n)) = __hneg(b3);
+    }
     fence_proxy_async_smem();
     rm_bar(kRmEpi2);
     if (e == 0) mbar_arrive(smem_u32(&S.q_ready));
-    pdl_wait();                                          // the rows' statistics (pass 1)
-    for (int x = e; x < GRp; x += kRmEpi2) {
-      const int hr = x / J.Rp, rr = x - hr * J.Rp;
-      // rows past R get an offset that makes their terms 0
-      st[x] = (hr < P.G && rr < P.R) ? -J.stat[(int64_t)slab * GRp + x].x : -INFINITY;
-    }
-    rm_bar(kRmEpi2);
     pdl_release();
     const int G = P.G, Rp = J.Rp;
     const int h_begin = G * grp / kRmGroups2, h_end = G * (grp + 1) / kRmGroups2;
@@ -427,24 +470,22 @@ __global__ void __launch_bounds__(rm_bound(64 + kRmEpi2), 1)
       if (ok) {
         for (int h = h_begin; h < h_end; ++h) {
           const uint32_t col = lane_addr + (uint32_t)buf * buf_cols + (uint32_t)(h * Rp);
-          const float* sh = st + h * Rp;
           float a = 0.f, a2 = 0.f;
-          // a head's rows in one load and one wait where they fit 32 or 64 columns; the
-          // offsets four at a time (padding rows add 2^-inf = 0)
-          // (the offsets are stored negated: s * scale - offset is one packed fma)
+          // a head's rows in one load and one wait where they fit 32 or 64 columns (the
+          // accumulator already holds s - offset / scale: one packed multiply per pair)
           const unsigned long long sc2 = f2pack(kScoreScale, kScoreScale);
           auto add = [&](const float (&v)[32], int r0) {
             unsigned long long p0 = 0ull, p1 = 0ull;
 #pragma unroll
             for (int t = 0; t < 32; t += 4) {
-              const float4 o = *reinterpret_cast<const float4*>(sh + r0 + t);
-              const unsigned long long x0 = ffma2(f2pack(v[t], v[t + 1]), sc2, f2pack(o.x, o.y));
-              const unsigned long long x1 = ffma2(f2pack(v[t + 2], v[t + 3]), sc2, f2pack(o.z, o.w));
+              const unsigned long long x0 = fmul2(f2pack(v[t], v[t + 1]), sc2);
+              const unsigned long long x1 = fmul2(f2pack(v[t + 2], v[t + 3]), sc2);
               p0 = fadd2(p0, f2pack(fast_exp2(f2lo(x0)), fast_exp2(f2hi(x0))));
               p1 = fadd2(p1, f2pack(fast_exp2(f2lo(x1)), fast_exp2(f2hi(x1))));
             }
             a += f2lo(p0) + f2lo(p1);
             a2 += f2hi(p0) + f2hi(p1);
+            (void)r0;
           };
           if (Rp == 32) {
             float v[32];
@@ -460,7 +501,7 @@ __global__ void __launch_bounds__(rm_bound(64 + kRmEpi2), 1)
               float v[16];
               tmem_ld16(col + (uint32_t)r0, v);
 #pragma unroll
-              for (int t = 0; t < 16; ++t) a += fast_exp2(fmaf(v[t], kScoreScale, sh[r0 + t]));
+              for (int t = 0; t < 16; ++t) a += fast_exp2(v[t] * kScoreScale);
             }
           }
           if (tok < n_tok)
@@ -537,9 +578,14 @@ cudaError_t launch_rowmean(const Batch& B, int pi, float2* scratch, int chunks, 
     const bool two = GRp > 256;
     const int NE = two ? ((GRp / 2 + 15) & ~15) : GRp;
     const int qb = ((two ? 2 : 1) * NE * 256 + 1023) & ~1023;
+    const int xb = ((two ? 2 : 1) * rm_xb_bytes(NE) + 1023) & ~1023;
+    const int pre = 1024 + qb + kRmXaBytes + xb;        // before the key stages
     J.nbuf = (two ? 2 * NE : NE) <= 256 ? 2 : 1;
-    J.stages = qb <= 64 * 1024 ? 4 : qb <= 115 * 1024 ? 3 : 2;
-    const size_t smem = 1024 + (size_t)qb + (size_t)J.stages * kRmStageBytes;
+    // key stages: what the 227 KB of shared memory leave (less the static part), at most 4
+    const int st = (232448 - 256 - pre) / kRmStageBytes;
+    J.stages = st < 4 ? st : 4;
+    if (J.stages < 2) return cudaErrorInvalidConfiguration;
+    const size_t smem = (size_t)pre + (size_t)J.stages * kRmStageBytes;
     e = ensure_smem((const void*)k_rm_alpha, (int)smem);
     if (e != cudaSuccess) return e;
     e = launch_pdl(k_rm_alpha, dim3(chunks, n_slabs), dim3(64 + kRmEpi2), smem, s, map, B, J);
