@@ -380,7 +380,6 @@ constexpr int kAtThreads = 192;            // warp 0 TMA, warp 1 MMA, warps 2-5 
 constexpr int kAtTile = 64;                // tokens per tile
 constexpr int kAtTileBytes = kAtTile * kHeadDim * 2;   // 16 KB of keys or values
 constexpr int kAtQBytes = 128 * kHeadDim * 2;          // 32 KB: 128 rows x 128 dims
-constexpr int kAtPBytes = 128 * kAtTile * 2;           // 16 KB: 128 rows x 64 tokens
 constexpr float kAtLazy = 8.0f;            // raise the running max only past this margin
 
 struct AttnJob {
@@ -397,30 +396,33 @@ struct AttnJob {
 // Barriers, at the end of the dynamic shared memory (no static shared memory, so the
 // dynamic region starts on the 1024-byte boundary the swizzled tiles need).
 struct AtBars {
-  unsigned long long kfull[2], kempty[2], vfull[2], vempty[2], sfull[2], sempty[2];
+  unsigned long long kfull[2], kempty[2], vfull[2], vempty[2], sfull[2];
   unsigned long long pfull, pvdone, q_ready, final_mma;
   uint32_t taddr;
   int abort;
 };
 
-constexpr int kAtSmem = kAtQBytes + kAtPBytes + 4 * kAtTileBytes + (int)sizeof(AtBars);
+constexpr int kAtSmem = kAtQBytes + 4 * kAtTileBytes + (int)sizeof(AtBars);
 
 // grid (chunks, halves, Hkv), two CTAs per SM (256 TMEM columns, ~113 KB of shared memory
 // each). Rows rho = h * Rp + r (h < G) of key head g; this CTA takes rho in
 // [128 * half, 128 * half + 128), one thread per row (TMEM lane). Per tile j of 64 tokens:
 //   TMA    K(j), V(j) into two-stage rings
 //   MMA    S(j) = Q K(j)^T into one of two TMEM buffers (64 columns) as soon as K(j) is in
-//          and the buffer is read out; O += P(j) V(j) once P(j) is written (event loop)
-//   rows   S(j) -> m, P(j) = bf16(2^(s - m)) into shared memory, l; the running maximum
-//          raised only past 8 (log2), then O and l rescaled in TMEM
+//          and O += P(j - 2) V(j - 2) has been issued; O += P(j) V(j) once P(j) is written,
+//          its A operand read from TMEM (event loop)
+//   rows   S(j) -> m, P(j) = bf16(2^(s - m)) back into the first 32 columns of S(j)'s
+//          buffer (two weights per column), l; the running maximum raised only past 8
+//          (log2), then O and l rescaled in TMEM
+// P never passes through shared memory: the tensor cores' operand reads there are only Q,
+// K and V (with the TMA writes of K and V, shared-memory bandwidth is this kernel's bound).
 // The second CTA on the SM fills the gaps of each CTA's chain of dependent steps.
 __global__ void __launch_bounds__(256, 2)
     k_fw_attn(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
               const AttnJob J) {
   extern __shared__ __align__(1024) unsigned char sm[];
   unsigned char* qs = sm;                        // A operand of S = Q K^T: 128 rows x 128 dims
-  unsigned char* ps = qs + kAtQBytes;            // A operand of O += P V: 128 rows x 64 tokens
-  unsigned char* kr = ps + kAtPBytes;            // 2 key stages
+  unsigned char* kr = qs + kAtQBytes;            // 2 key stages
   unsigned char* vr = kr + 2 * kAtTileBytes;     // 2 value stages
   AtBars& S = *reinterpret_cast<AtBars*>(vr + 2 * kAtTileBytes);
   const int chunk = blockIdx.x, half = blockIdx.y, g = blockIdx.z;
@@ -441,7 +443,6 @@ __global__ void __launch_bounds__(256, 2)
       mbar_init(smem_u32(&S.vfull[b]), 1);
       mbar_init(smem_u32(&S.vempty[b]), 1);
       mbar_init(smem_u32(&S.sfull[b]), 1);
-      mbar_init(smem_u32(&S.sempty[b]), 128);
     }
     mbar_init(smem_u32(&S.pfull), 128);
     mbar_init(smem_u32(&S.pvdone), 1);
@@ -490,11 +491,12 @@ __global__ void __launch_bounds__(256, 2)
     }
   } else if (warp == 1 && lane == 0) {
     // ---- MMA issuer, an event loop over two queues: S(j1) = Q K(j1)^T as soon as its
-    // keys are in and its TMEM buffer is read out, O += P(j2) V(j2) as soon as its weights
-    // are written (non-blocking tests, so neither queue holds back the other) ----
+    // keys are in and O += P(j1 - 2) V(j1 - 2) (the last reader of its TMEM buffer) has
+    // been issued (the MMAs of one thread run in issue order), O += P(j2) V(j2) as soon as
+    // its weights are written (non-blocking tests, so neither queue holds back the other) ----
     const uint32_t id1 = idesc_bf16_f32(128, kAtTile, false, false);
     const uint32_t id2 = idesc_bf16_f32(128, 128, false, true);
-    const uint32_t qa = smem_u32(qs), pa = smem_u32(ps);
+    const uint32_t qa = smem_u32(qs);
     if (fw_wait(smem_u32(&S.q_ready), 0, abort)) {
       int j1 = 0, j2 = 0;
       uint64_t t_idle = 0;
@@ -503,8 +505,8 @@ __global__ void __launch_bounds__(256, 2)
         bool did = false;
         if (j1 < n) {
           const int st = j1 & 1;
-          bool ready = j1 < 2 || mbar_test_wait(smem_u32(&S.sempty[st]), ((j1 >> 1) - 1) & 1);
-          ready = ready && mbar_test_wait(smem_u32(&S.kfull[st]), (j1 >> 1) & 1);
+          const bool ready =
+              j2 >= j1 - 1 && mbar_test_wait(smem_u32(&S.kfull[st]), (j1 >> 1) & 1);
           if (ready) {
             tc_fence_after();
             const uint32_t ka = smem_u32(kr + st * kAtTileBytes);
@@ -531,11 +533,11 @@ __global__ void __launch_bounds__(256, 2)
             const uint32_t va = smem_u32(vr + st * kAtTileBytes);
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
-              // P: K-major, 64 tokens in one 128-byte row; V: N = dims MN-major (two 64-dim
-              // blocks 8 KB apart), 16 tokens = 2048 bytes per K step
-              umma_bf16(tbase + 128u, sdesc_sw128(pa + k * 32, 16, 1024),
-                        sdesc_sw128(va + k * 2048, kAtTileBytes / 2, 1024), id2,
-                        (j2 > 0 || k > 0) ? 1u : 0u);
+              // P: in TMEM, 16 tokens = 8 columns per K step; V: N = dims MN-major (two
+              // 64-dim blocks 8 KB apart), 16 tokens = 2048 bytes per K step
+              umma_bf16_ts(tbase + 128u, tbase + (uint32_t)(st * 64 + k * 8),
+                           sdesc_sw128(va + k * 2048, kAtTileBytes / 2, 1024), id2,
+                           (j2 > 0 || k > 0) ? 1u : 0u);
             }
             umma_commit(smem_u32(&S.vempty[st]));
             umma_commit(smem_u32(&S.pvdone));
@@ -583,7 +585,6 @@ __global__ void __launch_bounds__(256, 2)
     fw_bar(1, 128);
     if (e == 0) mbar_arrive(smem_u32(&S.q_ready));
     const uint32_t la = tbase + ((uint32_t)(qd * 32) << 16);
-    unsigned char* prow = ps + rl * 128;
     const unsigned long long sc2 = f2pack(kScoreScale, kScoreScale);
     float m = -INFINITY, l = 0.f;
     bool ok = true;
@@ -596,8 +597,6 @@ __global__ void __launch_bounds__(256, 2)
       float s[64];
       tmem_ld32x2(la + st * 64u, la + st * 64u + 32u, *reinterpret_cast<float(*)[32]>(s),
                   *reinterpret_cast<float(*)[32]>(s + 32));
-      tc_fence_before();
-      mbar_arrive(smem_u32(&S.sempty[st]));
       const int nv = min(kAtTile, J.n_tok - (t0 + j) * kAtTile);   // valid tokens
       if (nv < kAtTile) {
 #pragma unroll
@@ -627,8 +626,11 @@ __global__ void __launch_bounds__(256, 2)
         if (c & 1) acc1 = fadd2(acc1, f2pack(p0, p1));
         else acc0 = fadd2(acc0, f2pack(p0, p1));
       }
-      // the P buffer and O are free once O += P(j - 1) V(j - 1) has completed; a raised
-      // maximum then rescales O (and l)
+      // P(j) over S(j) in TMEM (O += P(j - 2) V(j - 2), the buffer's last reader, completed
+      // before S(j) was computed)
+      tmem_st32u(la + st * 64u, pk);
+      // O is free once O += P(j - 1) V(j - 1) has completed; a raised maximum then rescales
+      // O (and l) before P(j) is released
       if (j >= 1) {
         ok = fw_wait(smem_u32(&S.pvdone), (j - 1) & 1, abort);
         ok = __all_sync(0xffffffffu, ok);
@@ -649,13 +651,6 @@ __global__ void __launch_bounds__(256, 2)
       }
       m = m_new;
       l += (f2lo(acc0) + f2hi(acc0)) + (f2lo(acc1) + f2hi(acc1));
-      // the P row: 64 tokens in 128 bytes, 16-byte chunks swizzled
-#pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        const uint4 w = make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
-        *reinterpret_cast<uint4*>(prow + ((c ^ (rl & 7)) << 4)) = w;
-      }
-      fence_proxy_async_smem();
       tc_fence_before();
       mbar_arrive(smem_u32(&S.pfull));
     }
