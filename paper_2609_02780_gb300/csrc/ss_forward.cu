@@ -714,18 +714,32 @@ __global__ void __launch_bounds__(256) k_fw_attn_out(const AttnOutJob J) {
   const uint2 qv = *reinterpret_cast<const uint2*>(J.q + ((int64_t)r * J.Hq + h) * kHeadDim + 4 * lane);
   const float q0 = __uint_as_float(qv.x << 16), q1 = __uint_as_float(qv.x & 0xffff0000u);
   const float q2 = __uint_as_float(qv.y << 16), q3 = __uint_as_float(qv.y & 0xffff0000u);
+  // (eight rows at a time: their loads and butterflies interleaved, each row's sum in
+  // the same order)
   float own0 = -INFINITY, own1 = -INFINITY;     // rows lane and lane + 32
-  for (int jr = 0; jr <= r; ++jr) {
-    const uint2 kv = *reinterpret_cast<const uint2*>(J.k + ((int64_t)jr * J.Hkv + g) * kHeadDim + 4 * lane);
-    float d = q0 * __uint_as_float(kv.x << 16);
-    d = fmaf(q1, __uint_as_float(kv.x & 0xffff0000u), d);
-    d = fmaf(q2, __uint_as_float(kv.y << 16), d);
-    d = fmaf(q3, __uint_as_float(kv.y & 0xffff0000u), d);
+  for (int j0 = 0; j0 <= r; j0 += 8) {
+    float d[8];
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) d += __shfl_xor_sync(0xffffffffu, d, o);
-    if (lane == (jr & 31)) {
-      if (jr < 32) own0 = d * kScoreScale;
-      else own1 = d * kScoreScale;
+    for (int u = 0; u < 8; ++u) {
+      const int jr = min(j0 + u, r);
+      const uint2 kv =
+          *reinterpret_cast<const uint2*>(J.k + ((int64_t)jr * J.Hkv + g) * kHeadDim + 4 * lane);
+      d[u] = q0 * __uint_as_float(kv.x << 16);
+      d[u] = fmaf(q1, __uint_as_float(kv.x & 0xffff0000u), d[u]);
+      d[u] = fmaf(q2, __uint_as_float(kv.y << 16), d[u]);
+      d[u] = fmaf(q3, __uint_as_float(kv.y & 0xffff0000u), d[u]);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+      for (int u = 0; u < 8; ++u) d[u] += __shfl_xor_sync(0xffffffffu, d[u], o);
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int jr = j0 + u;
+      if (jr <= r && lane == (jr & 31)) {
+        if (jr < 32) own0 = d[u] * kScoreScale;
+        else own1 = d[u] * kScoreScale;
+      }
     }
   }
   // chunk statistics: lane c holds chunk c (and c + 32, ...)
@@ -739,17 +753,17 @@ __global__ void __launch_bounds__(256) k_fw_attn_out(const AttnOutJob J) {
   float L = 0.f;
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
   int c = 0;
-  for (; c + 4 <= J.chunks; c += 4) {
-    float2 ml[4];
-    float4 ov[4];
+  for (; c + 8 <= J.chunks; c += 8) {
+    float2 ml[8];
+    float4 ov[8];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 0; u < 8; ++u) {
       const int64_t pr = ((int64_t)g * J.chunks + c + u) * rows + rho;
       ml[u] = J.mlpart[pr];
       ov[u] = reinterpret_cast<const float4*>(J.opart + pr * kHeadDim)[lane];
     }
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 0; u < 8; ++u) {
       if (!(ml[u].y > 0.f)) continue;
       const float wgt = fast_exp2(ml[u].x - M);
       L = fmaf(ml[u].y, wgt, L);
@@ -771,15 +785,25 @@ __global__ void __launch_bounds__(256) k_fw_attn_out(const AttnOutJob J) {
     acc.z = fmaf(ov.z, wgt, acc.z);
     acc.w = fmaf(ov.w, wgt, acc.w);
   }
-  for (int jr = 0; jr <= r; ++jr) {
-    const float s = __shfl_sync(0xffffffffu, jr < 32 ? own0 : own1, jr & 31);
-    const float wgt = fast_exp2(s - M);
-    L += wgt;
-    const uint2 vv = *reinterpret_cast<const uint2*>(J.v + ((int64_t)jr * J.Hkv + g) * kHeadDim + 4 * lane);
-    acc.x = fmaf(__uint_as_float(vv.x << 16), wgt, acc.x);
-    acc.y = fmaf(__uint_as_float(vv.x & 0xffff0000u), wgt, acc.y);
-    acc.z = fmaf(__uint_as_float(vv.y << 16), wgt, acc.z);
-    acc.w = fmaf(__uint_as_float(vv.y & 0xffff0000u), wgt, acc.w);
+  for (int j0 = 0; j0 <= r; j0 += 8) {
+    uint2 vv[8];
+    float sv[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int jr = min(j0 + u, r);
+      vv[u] = *reinterpret_cast<const uint2*>(J.v + ((int64_t)jr * J.Hkv + g) * kHeadDim + 4 * lane);
+      sv[u] = __shfl_sync(0xffffffffu, jr < 32 ? own0 : own1, jr & 31);
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      if (j0 + u > r) break;
+      const float wgt = fast_exp2(sv[u] - M);
+      L += wgt;
+      acc.x = fmaf(__uint_as_float(vv[u].x << 16), wgt, acc.x);
+      acc.y = fmaf(__uint_as_float(vv[u].x & 0xffff0000u), wgt, acc.y);
+      acc.z = fmaf(__uint_as_float(vv[u].y << 16), wgt, acc.z);
+      acc.w = fmaf(__uint_as_float(vv[u].y & 0xffff0000u), wgt, acc.w);
+    }
   }
   const float inv = 1.0f / L;
   reinterpret_cast<__nv_bfloat162*>(dst)[0] = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
