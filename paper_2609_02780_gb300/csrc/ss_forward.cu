@@ -821,9 +821,11 @@ int gemm_stages(int Rp) {
   return s < 2 ? 2 : (s > kGmMaxStages ? kGmMaxStages : s);
 }
 
+// K splits per output tile: as many as keep the grid within one wave of two CTAs per SM
+// (a grid just past the wave leaves a few CTAs running alone at its end)
 int gemm_splits(int n_out, int kblocks, int sm_count) {
   const int tiles = n_out / 128;
-  int s = (2 * sm_count + tiles / 2) / tiles;
+  int s = (2 * sm_count) / tiles;
   if (s < 1) s = 1;
   if (s > kblocks) s = kblocks;
   if (s > 16) s = 16;
