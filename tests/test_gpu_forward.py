@@ -150,14 +150,20 @@ def _attention_layers(layers):
     return out
 
 
-@pytest.mark.parametrize("R,F,Tf", [(32, 21, 64), (5, 13, 50), (1, 3, 64), (64, 2, 200)])
-def test_attention_and_q_of_one_layer(R, F, Tf):
+@pytest.mark.parametrize("R,F,Tf,kscale", [(32, 21, 64, 1), (5, 13, 50, 1), (1, 3, 64, 1),
+                                            (64, 2, 200, 1), (32, 120, 196, 1),
+                                            (32, 60, 196, 6)])
+def test_attention_and_q_of_one_layer(R, F, Tf, kscale):
     """One layer: q (exact up to rounding boundaries) and the attention output over the
     stored tokens plus the question's own rows (bound from the bf16 attention weights).
-    Covers two 128-row halves (R 32, 64), one (R 5, 1), ragged last tiles, several chunks."""
+    Covers two 128-row halves (R 32, 64), one (R 5, 1), ragged last tiles, several chunks,
+    several tiles per chunk (23,520 tokens), and keys scaled by 6 so that a row's maximum
+    keeps rising past the lazy margin, also between the two 64-column steps of a tile."""
     ss = _ss()
     Hkv = 4 if R != 64 else 2          # G * Rp: 224, 112, 112 (G 7), 256 (G 4 with Hq 8)
     w, keys, vals, layers, h_in = _case(1, F, Tf, R, 256, seed=R + F, Hkv=Hkv)
+    if kscale != 1:
+        keys = (keys.float() * kscale).to(torch.bfloat16)
     if R == 64:
         # Hq = 8, Hkv = 2 (G 4): 4 * 64 = 256 rows per key head
         syn = _synth()
