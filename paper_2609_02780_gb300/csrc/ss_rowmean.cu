@@ -254,12 +254,17 @@ __global__ void __launch_bounds__(rm_bound(64 + 128 * NMB * CS), 1)
           float mt = -INFINITY;
           if (nv >= pc + PW) {
             // (a full load needs no per-column test; the max is taken on the raw dot
-            // products and scaled once)
+            // products and scaled once; packed pairs are adjacent columns of one load,
+            // which sit in adjacent registers)
+            auto W = [&](int i) -> float {
+              if constexpr (PW == 64) return i < 32 ? v0[i] : v1[i - 32];
+              else return v0[i];
+            };
             float a0 = -INFINITY, a1 = -INFINITY;
 #pragma unroll
-            for (int c = 0; c < NP; c += 2) {
-              a0 = fmax3(a0, A(c), A(c + 1));
-              a1 = fmax3(a1, Bv(c), Bv(c + 1));
+            for (int c = 0; c < PW; c += 4) {
+              a0 = fmax3(a0, W(c), W(c + 1));
+              a1 = fmax3(a1, W(c + 2), W(c + 3));
             }
             mt = fmaxf(a0, a1) * kScoreScale;
             if (mt > m) {
@@ -270,7 +275,7 @@ __global__ void __launch_bounds__(rm_bound(64 + 128 * NMB * CS), 1)
             unsigned long long p0 = 0ull, p1 = 0ull;
 #pragma unroll
             for (int c = 0; c < NP; ++c) {
-              const unsigned long long x = ffma2(f2pack(A(c), Bv(c)), sc2, nm2);
+              const unsigned long long x = ffma2(f2pack(W(2 * c), W(2 * c + 1)), sc2, nm2);
               const unsigned long long ex = f2pack(fast_exp2(f2lo(x)), fast_exp2(f2hi(x)));
               if (c & 1) p1 = fadd2(p1, ex);
               else p0 = fadd2(p0, ex);
