@@ -228,17 +228,21 @@ __global__ void __launch_bounds__(256) k_fw_norm(const NormJob J) {
       h = reinterpret_cast<const float2*>(J.H + (int64_t)r * D)[x >> 1];
     }
     if (J.part) {
+      // up to 16 splits' partials loaded together (one memory latency), summed in order
       int s = 0;
-      for (; s + 4 <= J.splits; s += 4) {
-        float2 v[4];
+      if (J.splits <= 16) {
+        float2 v[16];
 #pragma unroll
-        for (int u = 0; u < 4; ++u)
-          v[u] = reinterpret_cast<const float2*>(J.part + ((int64_t)(s + u) * J.Rp + r) * D)[x >> 1];
+        for (int u = 0; u < 16; ++u)
+          if (u < J.splits)
+            v[u] = reinterpret_cast<const float2*>(J.part + ((int64_t)u * J.Rp + r) * D)[x >> 1];
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          h.x += v[u].x;
-          h.y += v[u].y;
-        }
+        for (int u = 0; u < 16; ++u)
+          if (u < J.splits) {
+            h.x += v[u].x;
+            h.y += v[u].y;
+          }
+        s = J.splits;
       }
       for (; s < J.splits; ++s) {
         const float2 v = reinterpret_cast<const float2*>(J.part + ((int64_t)s * J.Rp + r) * D)[x >> 1];
@@ -269,6 +273,28 @@ __global__ void __launch_bounds__(256) k_fw_norm(const NormJob J) {
   float tot = 0.f;
   for (int c = 0; c < J.chunks; ++c) tot += __ldcg(J.ssq + (int64_t)r * J.chunks + c);
   const float inv = 1.0f / sqrtf(tot / (float)D + J.eps);
+  // the row's H and weights loaded together (one memory latency) where D <= 16 x 512
+  constexpr int kIt = 16;
+  if (D <= kIt * 512) {
+    float2 hv[kIt];
+    __nv_bfloat162 wv[kIt];
+#pragma unroll
+    for (int it = 0; it < kIt; ++it) {
+      const int y = 2 * t + 512 * it;
+      if (y < D) {
+        hv[it] = __ldcg(reinterpret_cast<const float2*>(J.H + (int64_t)r * D + y));
+        wv[it] = reinterpret_cast<const __nv_bfloat162*>(J.w)[y >> 1];
+      }
+    }
+#pragma unroll
+    for (int it = 0; it < kIt; ++it) {
+      const int y = 2 * t + 512 * it;
+      if (y < D)
+        reinterpret_cast<__nv_bfloat162*>(J.X + (int64_t)r * D)[y >> 1] = __floats2bfloat162_rn(
+            hv[it].x * inv * __low2float(wv[it]), hv[it].y * inv * __high2float(wv[it]));
+    }
+    return;
+  }
   for (int y = 2 * t; y < D; y += 512) {
     const float2 hv = __ldcg(reinterpret_cast<const float2*>(J.H + (int64_t)r * D + y));
     const __nv_bfloat162 wv = reinterpret_cast<const __nv_bfloat162*>(J.w)[y >> 1];
@@ -309,19 +335,23 @@ __global__ void __launch_bounds__(64) k_fw_qkv(const QkvJob J) {
   const int f0 = t * kHeadDim + j, f1 = f0 + 64;
   float y0 = 0.f, y1 = 0.f;
   int s = 0;
-  for (; s + 4 <= J.splits; s += 4) {
-    float a[4], b[4];
+  if (J.splits <= 16) {
+    // every split's partial loaded together (one memory latency), summed in order
+    float a[16], b[16];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const float* p = J.part + ((int64_t)(s + u) * J.Rp + r) * n_out;
-      a[u] = p[f0];
-      b[u] = p[f1];
-    }
+    for (int u = 0; u < 16; ++u)
+      if (u < J.splits) {
+        const float* p = J.part + ((int64_t)u * J.Rp + r) * n_out;
+        a[u] = p[f0];
+        b[u] = p[f1];
+      }
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      y0 += a[u];
-      y1 += b[u];
-    }
+    for (int u = 0; u < 16; ++u)
+      if (u < J.splits) {
+        y0 += a[u];
+        y1 += b[u];
+      }
+    s = J.splits;
   }
   for (; s < J.splits; ++s) {
     const float* p = J.part + ((int64_t)s * J.Rp + r) * n_out;
@@ -714,13 +744,13 @@ __global__ void __launch_bounds__(256) k_fw_attn_out(const AttnOutJob J) {
   const uint2 qv = *reinterpret_cast<const uint2*>(J.q + ((int64_t)r * J.Hq + h) * kHeadDim + 4 * lane);
   const float q0 = __uint_as_float(qv.x << 16), q1 = __uint_as_float(qv.x & 0xffff0000u);
   const float q2 = __uint_as_float(qv.y << 16), q3 = __uint_as_float(qv.y & 0xffff0000u);
-  // (eight rows at a time: their loads and butterflies interleaved, each row's sum in
+  // (sixteen rows at a time: their loads and butterflies interleaved, each row's sum in
   // the same order)
   float own0 = -INFINITY, own1 = -INFINITY;     // rows lane and lane + 32
-  for (int j0 = 0; j0 <= r; j0 += 8) {
-    float d[8];
+  for (int j0 = 0; j0 <= r; j0 += 16) {
+    float d[16];
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
+    for (int u = 0; u < 16; ++u) {
       const int jr = min(j0 + u, r);
       const uint2 kv =
           *reinterpret_cast<const uint2*>(J.k + ((int64_t)jr * J.Hkv + g) * kHeadDim + 4 * lane);
@@ -732,9 +762,9 @@ __global__ void __launch_bounds__(256) k_fw_attn_out(const AttnOutJob J) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1)
 #pragma unroll
-      for (int u = 0; u < 8; ++u) d[u] += __shfl_xor_sync(0xffffffffu, d[u], o);
+      for (int u = 0; u < 16; ++u) d[u] += __shfl_xor_sync(0xffffffffu, d[u], o);
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
+    for (int u = 0; u < 16; ++u) {
       const int jr = j0 + u;
       if (jr <= r && lane == (jr & 31)) {
         if (jr < 32) own0 = d[u] * kScoreScale;
@@ -785,17 +815,17 @@ __global__ void __launch_bounds__(256) k_fw_attn_out(const AttnOutJob J) {
     acc.z = fmaf(ov.z, wgt, acc.z);
     acc.w = fmaf(ov.w, wgt, acc.w);
   }
-  for (int j0 = 0; j0 <= r; j0 += 8) {
-    uint2 vv[8];
-    float sv[8];
+  for (int j0 = 0; j0 <= r; j0 += 16) {
+    uint2 vv[16];
+    float sv[16];
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
+    for (int u = 0; u < 16; ++u) {
       const int jr = min(j0 + u, r);
       vv[u] = *reinterpret_cast<const uint2*>(J.v + ((int64_t)jr * J.Hkv + g) * kHeadDim + 4 * lane);
       sv[u] = __shfl_sync(0xffffffffu, jr < 32 ? own0 : own1, jr & 31);
     }
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
+    for (int u = 0; u < 16; ++u) {
       if (j0 + u > r) break;
       const float wgt = fast_exp2(sv[u] - M);
       L += wgt;
