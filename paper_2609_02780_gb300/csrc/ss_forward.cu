@@ -600,16 +600,28 @@ __global__ void __launch_bounds__(256, 2)
     const bool valid = hl < J.G && r < J.R;
     // (the keys and values stream in meanwhile: they do not depend on the previous kernel)
     pdl_wait();
-    // question rows -> 128-byte swizzled K-major tile (two halves of 64 dims)
-    for (int x = e; x < 128 * 16; x += 128) {
-      const int row = x >> 4, c = x & 15;
-      const int rr = half * 128 + row;
-      const int h2 = rr / J.Rp, r2 = rr - h2 * J.Rp;
-      uint4 v = make_uint4(0u, 0u, 0u, 0u);
-      if (h2 < J.G && r2 < J.R)
-        v = *reinterpret_cast<const uint4*>(J.q + ((int64_t)r2 * J.Hq + g * J.G + h2) * kHeadDim +
-                                            8 * c);
-      *reinterpret_cast<uint4*>(qs + (c >> 3) * 16384 + row * 128 + (((c & 7) ^ (row & 7)) << 4)) = v;
+    // question rows -> 128-byte swizzled K-major tile (two halves of 64 dims); a thread's
+    // 16 chunks loaded together, then stored (one memory latency)
+    {
+      uint4 v[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        const int x = e + 128 * u;
+        const int row = x >> 4, c = x & 15;
+        const int rr = half * 128 + row;
+        const int h2 = rr / J.Rp, r2 = rr - h2 * J.Rp;
+        v[u] = make_uint4(0u, 0u, 0u, 0u);
+        if (h2 < J.G && r2 < J.R)
+          v[u] = *reinterpret_cast<const uint4*>(J.q + ((int64_t)r2 * J.Hq + g * J.G + h2) *
+                                                           kHeadDim + 8 * c);
+      }
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        const int x = e + 128 * u;
+        const int row = x >> 4, c = x & 15;
+        *reinterpret_cast<uint4*>(qs + (c >> 3) * 16384 + row * 128 + (((c & 7) ^ (row & 7)) << 4)) =
+            v[u];
+      }
     }
     fence_proxy_async_smem();
     fw_bar(1, 128);

@@ -49,18 +49,31 @@ __device__ void rm_load_q(const Prob& P, int slab, int Rp, int n_rows, int rows_
                           unsigned char* dst, int t0, int nt) {
   const int i = slab / P.Hkv, g = slab - i * P.Hkv;
   const int64_t row_stride = (int64_t)P.Hq * kHeadDim;
-  for (int e = t0; e < n_rows * 16; e += nt) {
-    const int rho = e >> 4, c = e & 15;
-    const int h = rho / Rp, r = rho - h * Rp;
-    uint4 v = make_uint4(0u, 0u, 0u, 0u);
-    if (h < P.G && r < P.R)
-      v = *reinterpret_cast<const uint4*>(P.q + (int64_t)i * P.R * row_stride +
-                                          (int64_t)r * row_stride +
-                                          (int64_t)(g * P.G + h) * kHeadDim + 8 * c);
-    const int b = rho / rows_per_block, n = rho - b * rows_per_block;
-    unsigned char* blk = dst + (size_t)b * rows_per_block * 256;
-    *reinterpret_cast<uint4*>(blk + (c >> 3) * (rows_per_block * 128) + n * 128 +
-                              ((((c & 7) ^ (n & 7))) << 4)) = v;
+  // eight 16-byte chunks per thread loaded together, then stored (one memory latency
+  // per eight)
+  for (int e0 = t0; e0 < n_rows * 16; e0 += 8 * nt) {
+    uint4 v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int e = e0 + u * nt;
+      const int rho = e >> 4, c = e & 15;
+      const int h = rho / Rp, r = rho - h * Rp;
+      v[u] = make_uint4(0u, 0u, 0u, 0u);
+      if (e < n_rows * 16 && h < P.G && r < P.R)
+        v[u] = *reinterpret_cast<const uint4*>(P.q + (int64_t)i * P.R * row_stride +
+                                               (int64_t)r * row_stride +
+                                               (int64_t)(g * P.G + h) * kHeadDim + 8 * c);
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int e = e0 + u * nt;
+      if (e >= n_rows * 16) break;
+      const int rho = e >> 4, c = e & 15;
+      const int b = rho / rows_per_block, n = rho - b * rows_per_block;
+      unsigned char* blk = dst + (size_t)b * rows_per_block * 256;
+      *reinterpret_cast<uint4*>(blk + (c >> 3) * (rows_per_block * 128) + n * 128 +
+                                ((((c & 7) ^ (n & 7))) << 4)) = v[u];
+    }
   }
 }
 
