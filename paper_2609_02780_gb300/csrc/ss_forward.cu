@@ -305,6 +305,72 @@ __global__ void __launch_bounds__(256) k_fw_norm(const NormJob J) {
 
 // cos and sin of the RoPE angles pos * theta^(-2j/d) of every question row (computed in
 // fp64, stored as fp32): [R][64] pairs.
+// The same in one pass with one CTA per row (D / 4 threads, four columns each; D <= 4096):
+// the row's partials loaded eight splits at a time, its sum of squares reduced in the
+// CTA (warps in order), then normalised; no second kernel phase and no arrival counters.
+__global__ void __launch_bounds__(1024) k_fw_norm_row(const NormJob J) {
+  __shared__ float red[32];
+  __shared__ float s_inv;
+  pdl_wait();
+  pdl_release();
+  const int r = blockIdx.x, t = threadIdx.x, D = J.D;
+  const int x = 4 * t;
+  if (r >= J.R) {
+    if (J.w) {
+      const __nv_bfloat162 z = __floats2bfloat162_rn(0.f, 0.f);
+      reinterpret_cast<__nv_bfloat162*>(J.X + (int64_t)r * D + x)[0] = z;
+      reinterpret_cast<__nv_bfloat162*>(J.X + (int64_t)r * D + x)[1] = z;
+    }
+    return;
+  }
+  float4 h;
+  if (J.h_in) {
+    const uint2 b = *reinterpret_cast<const uint2*>(J.h_in + (int64_t)r * D + x);
+    h = make_float4(__uint_as_float(b.x << 16), __uint_as_float(b.x & 0xffff0000u),
+                    __uint_as_float(b.y << 16), __uint_as_float(b.y & 0xffff0000u));
+  } else {
+    h = *reinterpret_cast<const float4*>(J.H + (int64_t)r * D + x);
+  }
+  if (J.part) {
+    // eight splits' partials at a time, summed in split order
+    for (int s0 = 0; s0 < J.splits; s0 += 8) {
+      float4 v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        if (s0 + u < J.splits)
+          v[u] = *reinterpret_cast<const float4*>(J.part + ((int64_t)(s0 + u) * J.Rp + r) * D + x);
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        if (s0 + u < J.splits) {
+          h.x += v[u].x;
+          h.y += v[u].y;
+          h.z += v[u].z;
+          h.w += v[u].w;
+        }
+    }
+  }
+  *reinterpret_cast<float4*>(J.H + (int64_t)r * D + x) = h;
+  if (!J.w) return;
+  float ss = fmaf(h.w, h.w, fmaf(h.z, h.z, fmaf(h.y, h.y, h.x * h.x)));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  if ((t & 31) == 0) red[t >> 5] = ss;
+  __syncthreads();
+  if (t == 0) {
+    float tot = 0.f;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += red[w];
+    s_inv = 1.0f / sqrtf(tot / (float)D + J.eps);
+  }
+  __syncthreads();
+  const float inv = s_inv;
+  const uint2 wb = *reinterpret_cast<const uint2*>(J.w + x);
+  const float w0 = __uint_as_float(wb.x << 16), w1 = __uint_as_float(wb.x & 0xffff0000u);
+  const float w2 = __uint_as_float(wb.y << 16), w3 = __uint_as_float(wb.y & 0xffff0000u);
+  __nv_bfloat162* dst = reinterpret_cast<__nv_bfloat162*>(J.X + (int64_t)r * D + x);
+  dst[0] = __floats2bfloat162_rn(h.x * inv * w0, h.y * inv * w1);
+  dst[1] = __floats2bfloat162_rn(h.z * inv * w2, h.w * inv * w3);
+}
+
 __global__ void __launch_bounds__(64) k_fw_rope(float2* tab, int64_t pos0, double theta) {
   const int r = blockIdx.x, j = threadIdx.x;
   pdl_wait();     // (an earlier forward's kernels may still read the table)
@@ -1006,6 +1072,12 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
   nj.ticket = ticket;
   nj.chunks = L.nchunks;
   const dim3 ngrid(L.nchunks, L.Rp);
+  // one CTA per row where a row fits one CTA (four columns per thread), else column chunks
+  const bool row_norm = D % 128 == 0 && D / 4 <= 1024;
+  auto norm = [&](const NormJob& J) {
+    return row_norm ? launch_pdl(k_fw_norm_row, dim3(L.Rp), dim3(D / 4), 0, st, J)
+                    : launch_pdl(k_fw_norm, ngrid, dim3(256), 0, st, J);
+  };
   for (int i = 0; i < F.P; ++i) {
     const FwLayerW& W = A.layers[i];
     __nv_bfloat16* q = static_cast<__nv_bfloat16*>(A.q_out) + (int64_t)i * F.R * F.Hq * kHeadDim;
@@ -1016,7 +1088,7 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
     nj.splits = L.sp_d;
     nj.w = static_cast<const __nv_bfloat16*>(W.ln1);
     nj.X = X;
-    if ((e = launch_pdl(k_fw_norm, ngrid, dim3(256), 0, st, nj)) != cudaSuccess) return e;
+    if ((e = norm(nj)) != cudaSuccess) return e;
     if ((e = gemm(W.wqkv, nqkv, D, X, F.R, L.Rp, L.sp_qkv, part, status, st)) != cudaSuccess) return e;
     QkvJob qj;
     qj.part = part;
@@ -1075,7 +1147,7 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
     nj.part = part;
     nj.splits = L.sp_o;
     nj.w = static_cast<const __nv_bfloat16*>(W.ln2);
-    if ((e = launch_pdl(k_fw_norm, ngrid, dim3(256), 0, st, nj)) != cudaSuccess) return e;
+    if ((e = norm(nj)) != cudaSuccess) return e;
     if ((e = gemm(W.wgu, 2 * F.I, D, X, F.R, L.Rp, L.sp_gu, part, status, st)) != cudaSuccess) return e;
     SwigluJob sj;
     sj.part = part;
@@ -1093,7 +1165,7 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
   nj.part = part;
   nj.splits = L.sp_d;
   nj.w = nullptr;
-  if ((e = launch_pdl(k_fw_norm, ngrid, dim3(256), 0, st, nj)) != cudaSuccess) return e;
+  if ((e = norm(nj)) != cudaSuccess) return e;
   if (A.h_out)
     return cudaMemcpyAsync(A.h_out, H, (size_t)F.R * D * sizeof(float), cudaMemcpyDeviceToDevice, st);
   return cudaSuccess;
