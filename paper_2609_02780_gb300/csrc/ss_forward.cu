@@ -55,6 +55,10 @@ __device__ __forceinline__ void fw_bar(int id, int nthreads) {
 
 // ===========================================================================
 // Skinny GEMM: part[split][r][n] = sum over the split's K range of X[r][k] W[n][k].
+// With swiglu_I > 0 (one split), the gate/up projection with the MLP's product fused: CTA b
+// stages gate rows 64 b .. 64 b + 63 of W (TMEM lanes 0-63) and the matching up rows
+// I + 64 b .. (lanes 64-127) as one 128-row operand, and its epilogue writes
+// A[r][f] = bf16(silu(g) * u) directly (no partials, no separate kernel).
 // ===========================================================================
 constexpr int kGmThreads = 192;           // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
 constexpr int kGmMaxStages = 8;
@@ -63,6 +67,8 @@ constexpr int kGmABytes = 128 * 128;      // 128 rows of W x 64 bf16
 struct GemmJob {
   float* part;       // [splits][Rp][n_out]
   int n_out;
+  int swiglu_I;      // > 0: gate/up with SwiGLU in the epilogue (splits 1; see below)
+  __nv_bfloat16* A;  // [Rp][swiglu_I] the SwiGLU product (rows >= R zero)
   int R, Rp;
   int kblocks;       // K / 64
   int splits;
@@ -86,7 +92,7 @@ __global__ void __launch_bounds__(kGmThreads, 1)
   const int stages = J.stages;
   const int b_bytes = J.Rp * 128;
   const int stage_bytes = kGmABytes + b_bytes;   // a multiple of 1024 (Rp % 16 == 0)
-  const int m0 = blockIdx.x * 128, split = blockIdx.y;
+  const int m0 = blockIdx.x * (J.swiglu_I > 0 ? 64 : 128), split = blockIdx.y;
   const int kb0 = (int)((int64_t)J.kblocks * split / J.splits);
   const int kb1 = (int)((int64_t)J.kblocks * (split + 1) / J.splits);
   const int n = kb1 - kb0;
@@ -118,10 +124,19 @@ __global__ void __launch_bounds__(kGmThreads, 1)
     // the weights do not depend on the previous kernel: the first stages' weight tiles
     // are requested before waiting for it, their rows of X after
     const int pre = n < stages ? n : stages;
+    // W rows of a stage: 128 from m0, or 64 gate rows from m0 and 64 up rows from I + m0
+    auto load_w = [&](uint32_t dst, uint32_t bar, int kx) {
+      if (J.swiglu_I > 0) {
+        tma_load_2d(dst, &wmap, bar, kx, m0);
+        tma_load_2d(dst + kGmABytes / 2, &wmap, bar, kx, J.swiglu_I + m0);
+      } else {
+        tma_load_2d(dst, &wmap, bar, kx, m0);
+      }
+    };
     for (int j = 0; j < pre; ++j) {
       const uint32_t bar = smem_u32(&S.full[j]);
       mbar_expect_tx(bar, (uint32_t)stage_bytes);
-      tma_load_2d(smem_u32(sm + j * stage_bytes), &wmap, bar, (kb0 + j) * 64, m0);
+      load_w(smem_u32(sm + j * stage_bytes), bar, (kb0 + j) * 64);
     }
     pdl_wait();
     for (int j = 0; j < pre; ++j) {
@@ -135,7 +150,7 @@ __global__ void __launch_bounds__(kGmThreads, 1)
       const uint32_t bar = smem_u32(&S.full[st]);
       const uint32_t dst = smem_u32(sm + st * stage_bytes);
       mbar_expect_tx(bar, (uint32_t)stage_bytes);
-      tma_load_2d(dst, &wmap, bar, (kb0 + j) * 64, m0);
+      load_w(dst, bar, (kb0 + j) * 64);
       tma_load_2d(dst + kGmABytes, &xmap, bar, (kb0 + j) * 64, 0);
       issued_last[st] = j;
     }
@@ -164,7 +179,36 @@ __global__ void __launch_bounds__(kGmThreads, 1)
     bool ok = fw_wait(smem_u32(&S.d_full), 0, abort) && n > 0;
     ok = __all_sync(0xffffffffu, ok) && !*abort;
     tc_fence_after();
-    if (ok) {
+    if (J.swiglu_I > 0) {
+      // up values (lanes 64-127) through shared memory (the stages are idle now: every
+      // copy was consumed by an MMA that has completed) to the gate lanes' threads
+      float* up = reinterpret_cast<float*>(sm);    // [Rp][64]
+      const uint32_t la = tbase + ((uint32_t)(qd * 32) << 16);
+      if (ok && qd >= 2) {
+        for (int c0 = 0; c0 < J.Rp; c0 += 16) {
+          float v[16];
+          tmem_ld16(la + (uint32_t)c0, v);
+#pragma unroll
+          for (int c = 0; c < 16; ++c) up[(c0 + c) * 64 + (qd - 2) * 32 + lane] = v[c];
+        }
+      }
+      fw_bar(1, 128);
+      if (ok && qd < 2) {
+        const int fl = qd * 32 + lane;             // gate row within the CTA's 64
+        __nv_bfloat16* out = J.A + m0 + fl;
+        for (int c0 = 0; c0 < J.Rp; c0 += 16) {
+          float v[16];
+          tmem_ld16(la + (uint32_t)c0, v);
+#pragma unroll
+          for (int c = 0; c < 16; ++c) {
+            const int r = c0 + c;
+            const float g = v[c], u = up[r * 64 + fl];
+            const float a = r < J.R ? g / (1.0f + expf(-g)) * u : 0.f;
+            out[(int64_t)r * J.swiglu_I] = __float2bfloat16_rn(a);
+          }
+        }
+      }
+    } else if (ok) {
       const uint32_t la = tbase + ((uint32_t)(qd * 32) << 16);
       float* out = J.part + (int64_t)split * J.Rp * J.n_out + f;
       for (int c0 = 0; c0 < J.Rp; c0 += 16) {
@@ -992,10 +1036,11 @@ FwLayout fw_layout(const FwShape& F) {
 }
 
 cudaError_t gemm(const void* W, int n_out, int K, const __nv_bfloat16* X, int R, int Rp,
-                 int splits, float* part, uint32_t* status, cudaStream_t st) {
+                 int splits, float* part, uint32_t* status, cudaStream_t st, int swiglu_I = 0,
+                 __nv_bfloat16* A = nullptr) {
   CUtensorMap wm, xm;
   const uint64_t wd[2] = {(uint64_t)K, (uint64_t)n_out}, ws[1] = {(uint64_t)K * 2};
-  const uint32_t wb[2] = {64, 128};
+  const uint32_t wb[2] = {64, swiglu_I > 0 ? 64u : 128u};
   cudaError_t e = encode_bf16_map(&wm, W, 2, wd, ws, wb);
   if (e != cudaSuccess) return e;
   const uint64_t xd[2] = {(uint64_t)K, (uint64_t)Rp}, xs[1] = {(uint64_t)K * 2};
@@ -1005,6 +1050,8 @@ cudaError_t gemm(const void* W, int n_out, int K, const __nv_bfloat16* X, int R,
   GemmJob J;
   J.part = part;
   J.n_out = n_out;
+  J.swiglu_I = swiglu_I;
+  J.A = A;
   J.R = R;
   J.Rp = Rp;
   J.kblocks = K / 64;
@@ -1014,7 +1061,8 @@ cudaError_t gemm(const void* W, int n_out, int K, const __nv_bfloat16* X, int R,
   const int smem = J.stages * (kGmABytes + Rp * 128) + 1024;
   e = ensure_smem((const void*)k_fw_gemm, smem);
   if (e != cudaSuccess) return e;
-  return launch_pdl(k_fw_gemm, dim3(n_out / 128, splits), dim3(kGmThreads), smem, st, wm, xm, J);
+  return launch_pdl(k_fw_gemm, dim3(swiglu_I > 0 ? swiglu_I / 64 : n_out / 128, splits),
+                    dim3(kGmThreads), smem, st, wm, xm, J);
 }
 
 }  // namespace
@@ -1148,16 +1196,22 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
     nj.splits = L.sp_o;
     nj.w = static_cast<const __nv_bfloat16*>(W.ln2);
     if ((e = norm(nj)) != cudaSuccess) return e;
-    if ((e = gemm(W.wgu, 2 * F.I, D, X, F.R, L.Rp, L.sp_gu, part, status, st)) != cudaSuccess) return e;
-    SwigluJob sj;
-    sj.part = part;
-    sj.splits = L.sp_gu;
-    sj.Rp = L.Rp;
-    sj.R = F.R;
-    sj.I = F.I;
-    sj.A = Ab;
-    if ((e = launch_pdl(k_fw_swiglu, dim3((unsigned)(((int64_t)L.Rp * F.I + 255) / 256)), dim3(256), 0, st, sj)) != cudaSuccess)
-      return e;
+    if (L.sp_gu == 1 && F.I % 64 == 0) {
+      // one split: the SwiGLU product straight from the gate/up GEMM's epilogue
+      if ((e = gemm(W.wgu, 2 * F.I, D, X, F.R, L.Rp, 1, part, status, st, F.I, Ab)) != cudaSuccess)
+        return e;
+    } else {
+      if ((e = gemm(W.wgu, 2 * F.I, D, X, F.R, L.Rp, L.sp_gu, part, status, st)) != cudaSuccess) return e;
+      SwigluJob sj;
+      sj.part = part;
+      sj.splits = L.sp_gu;
+      sj.Rp = L.Rp;
+      sj.R = F.R;
+      sj.I = F.I;
+      sj.A = Ab;
+      if ((e = launch_pdl(k_fw_swiglu, dim3((unsigned)(((int64_t)L.Rp * F.I + 255) / 256)), dim3(256), 0, st, sj)) != cudaSuccess)
+        return e;
+    }
     if ((e = gemm(W.wd, D, F.I, Ab, F.R, L.Rp, L.sp_d, part, status, st)) != cudaSuccess) return e;
   }
   // H += the last down projection

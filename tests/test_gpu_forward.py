@@ -190,17 +190,20 @@ def test_attention_and_q_of_one_layer(R, F, Tf, kscale):
     print(f"q elements at a rounding boundary: {n_q}; o error / bound max {(err / tol).max():.3f}")
 
 
-def test_mlp_of_one_layer_and_no_stored_tokens():
+@pytest.mark.parametrize("I", [384, 9856])
+def test_mlp_of_one_layer_and_no_stored_tokens(I):
     """Wo = 0: H_out = h_in + bf16(silu(x2 Wg^T) (x2 Wu^T)) Wd^T; and an index with no
-    stored frames (the rows attend only to each other)."""
+    stored frames (the rows attend only to each other). MLP width 384 takes the split-K
+    gate/up projection and the separate SwiGLU kernel; 9856 (154 gate/up tiles of 128, one
+    K split on 152 SMs) the projection with the SwiGLU product in its epilogue."""
     ss = _ss()
-    w, keys, vals, layers, h_in = _case(1, 0, 64, 12, 384, seed=7)
+    w, keys, vals, layers, h_in = _case(1, 0, 64, 12, I, seed=7)
     layers = _unit_norm_weights(layers)
     for L in layers:
         L["wo"] = torch.zeros_like(L["wo"])
     h_in = _exact_norm_rows(12, 28 * 128, seed=7)
     idx = ss.Index(1, 28, 4, 64, 8, device=torch.device("cuda"))
-    params = ss.ForwardParams(384, EXACT_EPS, 1e4)
+    params = ss.ForwardParams(I, EXACT_EPS, 1e4)
     qb, h = _run(idx, layers, h_in, params)
     hb = to_bits(h_in)
     npw = _np_weights(layers)[0]
