@@ -843,79 +843,93 @@ struct AttnOutJob {
   const uint32_t* status;
 };
 
-// One warp per (row of Rp, head): the chunks' (m, l, O) and the question's own rows
-// 0..r merged under their common maximum, in a fixed order; lane owns dims 4 lane .. +3.
+// One CTA per (row r of Rp, query head h), eight warps. The row's items are the chunks'
+// partials (m, l, O) and its own rows 0..r (score s, weight 1, value v); warp w takes
+// chunks w, w + 8, ... and own rows w, w + 8, ..., loads them together, and reduces them
+// under its own maximum in item order (lane: dims 4 lane .. 4 lane + 3). The eight warps'
+// results are then merged in warp order under the common maximum.
 __global__ void __launch_bounds__(256) k_fw_attn_out(const AttnOutJob J) {
-  const int wid = (blockIdx.x * 256 + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  __shared__ float4 s_acc[8][32];
+  __shared__ float s_m[8], s_l[8];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x / J.Hq, h = blockIdx.x - r * J.Hq;
   pdl_wait();
   pdl_release();
-  if (wid >= J.Rp * J.Hq) return;
-  const int r = wid / J.Hq, h = wid - r * J.Hq;
   __nv_bfloat16* dst = J.o + (int64_t)r * J.Hq * kHeadDim + h * kHeadDim + 4 * lane;
   if (r >= J.R || (*(volatile const uint32_t*)J.status & kStatusTimeout)) {
-    const __nv_bfloat162 z = __floats2bfloat162_rn(0.f, 0.f);
-    reinterpret_cast<__nv_bfloat162*>(dst)[0] = z;
-    reinterpret_cast<__nv_bfloat162*>(dst)[1] = z;
+    if (warp == 0) {
+      const __nv_bfloat162 z = __floats2bfloat162_rn(0.f, 0.f);
+      reinterpret_cast<__nv_bfloat162*>(dst)[0] = z;
+      reinterpret_cast<__nv_bfloat162*>(dst)[1] = z;
+    }
     return;
   }
   const int g = h / J.G, hl = h - g * J.G;
   const int rho = hl * J.Rp + r;
   const int rows = J.halves * 128;
-  // own rows' scores, lane jr < 32 (and jr + 32) holds row jr's (one dot per row, lanes
-  // summed in a fixed butterfly)
+  constexpr int kC = 8;                         // chunks per warp loaded together (38 / 8 = 5)
+  constexpr int kO = 8;                         // own rows per warp (R <= 64)
+  // own rows jr = warp + 8 u: scores (one dot per row, lanes summed in a fixed butterfly)
   const uint2 qv = *reinterpret_cast<const uint2*>(J.q + ((int64_t)r * J.Hq + h) * kHeadDim + 4 * lane);
   const float q0 = __uint_as_float(qv.x << 16), q1 = __uint_as_float(qv.x & 0xffff0000u);
   const float q2 = __uint_as_float(qv.y << 16), q3 = __uint_as_float(qv.y & 0xffff0000u);
-  // (sixteen rows at a time: their loads and butterflies interleaved, each row's sum in
-  // the same order)
-  float own0 = -INFINITY, own1 = -INFINITY;     // rows lane and lane + 32
-  for (int j0 = 0; j0 <= r; j0 += 16) {
-    float d[16];
+  float so[kO];
+  uint2 vo[kO];
 #pragma unroll
-    for (int u = 0; u < 16; ++u) {
-      const int jr = min(j0 + u, r);
-      const uint2 kv =
-          *reinterpret_cast<const uint2*>(J.k + ((int64_t)jr * J.Hkv + g) * kHeadDim + 4 * lane);
-      d[u] = q0 * __uint_as_float(kv.x << 16);
-      d[u] = fmaf(q1, __uint_as_float(kv.x & 0xffff0000u), d[u]);
-      d[u] = fmaf(q2, __uint_as_float(kv.y << 16), d[u]);
-      d[u] = fmaf(q3, __uint_as_float(kv.y & 0xffff0000u), d[u]);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1)
-#pragma unroll
-      for (int u = 0; u < 16; ++u) d[u] += __shfl_xor_sync(0xffffffffu, d[u], o);
-#pragma unroll
-    for (int u = 0; u < 16; ++u) {
-      const int jr = j0 + u;
-      if (jr <= r && lane == (jr & 31)) {
-        if (jr < 32) own0 = d[u] * kScoreScale;
-        else own1 = d[u] * kScoreScale;
-      }
+  for (int u = 0; u < kO; ++u) {
+    const int jr = warp + 8 * u;
+    so[u] = -INFINITY;
+    vo[u] = make_uint2(0u, 0u);
+    if (jr <= r) {
+      const uint2 kv = *reinterpret_cast<const uint2*>(J.k + ((int64_t)jr * J.Hkv + g) * kHeadDim + 4 * lane);
+      vo[u] = *reinterpret_cast<const uint2*>(J.v + ((int64_t)jr * J.Hkv + g) * kHeadDim + 4 * lane);
+      float d = q0 * __uint_as_float(kv.x << 16);
+      d = fmaf(q1, __uint_as_float(kv.x & 0xffff0000u), d);
+      d = fmaf(q2, __uint_as_float(kv.y << 16), d);
+      d = fmaf(q3, __uint_as_float(kv.y & 0xffff0000u), d);
+      so[u] = d;
     }
   }
-  // chunk statistics: lane c holds chunk c (and c + 32, ...)
-  float M = fmaxf(own0, own1);
-  for (int c = lane; c < J.chunks; c += 32) {
-    const float2 ml = J.mlpart[((int64_t)g * J.chunks + c) * rows + rho];
-    if (ml.y > 0.f) M = fmaxf(M, ml.x);
-  }
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+  for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+    for (int u = 0; u < kO; ++u) so[u] += __shfl_xor_sync(0xffffffffu, so[u], o);
+#pragma unroll
+  for (int u = 0; u < kO; ++u) so[u] = warp + 8 * u <= r ? so[u] * kScoreScale : -INFINITY;
+  // this warp's chunks c = warp + 8 u
+  float M = -INFINITY;
+#pragma unroll
+  for (int u = 0; u < kO; ++u) M = fmaxf(M, so[u]);
   float L = 0.f;
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  int c = 0;
-  for (; c + 8 <= J.chunks; c += 8) {
-    float2 ml[8];
-    float4 ov[8];
+  for (int c0 = warp; c0 < J.chunks; c0 += 8 * kC) {
+    float2 ml[kC];
+    float4 ov[kC];
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
-      const int64_t pr = ((int64_t)g * J.chunks + c + u) * rows + rho;
-      ml[u] = J.mlpart[pr];
-      ov[u] = reinterpret_cast<const float4*>(J.opart + pr * kHeadDim)[lane];
+    for (int u = 0; u < kC; ++u) {
+      const int c = c0 + 8 * u;
+      ml[u] = make_float2(-INFINITY, 0.f);
+      if (c < J.chunks) {
+        const int64_t pr = ((int64_t)g * J.chunks + c) * rows + rho;
+        ml[u] = J.mlpart[pr];
+        ov[u] = reinterpret_cast<const float4*>(J.opart + pr * kHeadDim)[lane];
+      }
+    }
+    float Mb = M;
+#pragma unroll
+    for (int u = 0; u < kC; ++u)
+      if (ml[u].y > 0.f) Mb = fmaxf(Mb, ml[u].x);
+    if (Mb > M) {                               // the batch raised the warp's maximum
+      const float f = M == -INFINITY ? 0.f : fast_exp2(M - Mb);
+      L *= f;
+      acc.x *= f;
+      acc.y *= f;
+      acc.z *= f;
+      acc.w *= f;
+      M = Mb;
     }
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
+    for (int u = 0; u < kC; ++u) {
       if (!(ml[u].y > 0.f)) continue;
       const float wgt = fast_exp2(ml[u].x - M);
       L = fmaf(ml[u].y, wgt, L);
@@ -925,41 +939,42 @@ __global__ void __launch_bounds__(256) k_fw_attn_out(const AttnOutJob J) {
       acc.w = fmaf(ov[u].w, wgt, acc.w);
     }
   }
-  for (; c < J.chunks; ++c) {
-    const int64_t pr = ((int64_t)g * J.chunks + c) * rows + rho;
-    const float2 ml = J.mlpart[pr];
-    if (!(ml.y > 0.f)) continue;
-    const float wgt = fast_exp2(ml.x - M);
-    const float4 ov = reinterpret_cast<const float4*>(J.opart + pr * kHeadDim)[lane];
-    L = fmaf(ml.y, wgt, L);
-    acc.x = fmaf(ov.x, wgt, acc.x);
-    acc.y = fmaf(ov.y, wgt, acc.y);
-    acc.z = fmaf(ov.z, wgt, acc.z);
-    acc.w = fmaf(ov.w, wgt, acc.w);
-  }
-  for (int j0 = 0; j0 <= r; j0 += 16) {
-    uint2 vv[16];
-    float sv[16];
 #pragma unroll
-    for (int u = 0; u < 16; ++u) {
-      const int jr = min(j0 + u, r);
-      vv[u] = *reinterpret_cast<const uint2*>(J.v + ((int64_t)jr * J.Hkv + g) * kHeadDim + 4 * lane);
-      sv[u] = __shfl_sync(0xffffffffu, jr < 32 ? own0 : own1, jr & 31);
-    }
-#pragma unroll
-    for (int u = 0; u < 16; ++u) {
-      if (j0 + u > r) break;
-      const float wgt = fast_exp2(sv[u] - M);
-      L += wgt;
-      acc.x = fmaf(__uint_as_float(vv[u].x << 16), wgt, acc.x);
-      acc.y = fmaf(__uint_as_float(vv[u].x & 0xffff0000u), wgt, acc.y);
-      acc.z = fmaf(__uint_as_float(vv[u].y << 16), wgt, acc.z);
-      acc.w = fmaf(__uint_as_float(vv[u].y & 0xffff0000u), wgt, acc.w);
-    }
+  for (int u = 0; u < kO; ++u) {
+    if (warp + 8 * u > r) break;
+    const float wgt = fast_exp2(so[u] - M);
+    L += wgt;
+    acc.x = fmaf(__uint_as_float(vo[u].x << 16), wgt, acc.x);
+    acc.y = fmaf(__uint_as_float(vo[u].x & 0xffff0000u), wgt, acc.y);
+    acc.z = fmaf(__uint_as_float(vo[u].y << 16), wgt, acc.z);
+    acc.w = fmaf(__uint_as_float(vo[u].y & 0xffff0000u), wgt, acc.w);
   }
-  const float inv = 1.0f / L;
-  reinterpret_cast<__nv_bfloat162*>(dst)[0] = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
-  reinterpret_cast<__nv_bfloat162*>(dst)[1] = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
+  s_acc[warp][lane] = acc;
+  if (lane == 0) {
+    s_m[warp] = M;
+    s_l[warp] = L;
+  }
+  __syncthreads();
+  if (warp != 0) return;
+  float Mt = -INFINITY;
+#pragma unroll
+  for (int w = 0; w < 8; ++w) Mt = fmaxf(Mt, s_m[w]);
+  float Lt = 0.f;
+  float4 at = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+  for (int w = 0; w < 8; ++w) {
+    if (s_m[w] == -INFINITY) continue;
+    const float f = fast_exp2(s_m[w] - Mt);
+    const float4 a = s_acc[w][lane];
+    Lt = fmaf(s_l[w], f, Lt);
+    at.x = fmaf(a.x, f, at.x);
+    at.y = fmaf(a.y, f, at.y);
+    at.z = fmaf(a.z, f, at.z);
+    at.w = fmaf(a.w, f, at.w);
+  }
+  const float inv = 1.0f / Lt;
+  reinterpret_cast<__nv_bfloat162*>(dst)[0] = __floats2bfloat162_rn(at.x * inv, at.y * inv);
+  reinterpret_cast<__nv_bfloat162*>(dst)[1] = __floats2bfloat162_rn(at.z * inv, at.w * inv);
 }
 
 // ===========================================================================
@@ -1186,8 +1201,7 @@ cudaError_t launch_forward(const FwShape& F, const FwArgs& A, cudaStream_t st) {
     oj.mlpart = ml;
     oj.o = X;
     oj.status = status;
-    const int warps = L.Rp * F.Hq;
-    if ((e = launch_pdl(k_fw_attn_out, dim3((warps * 32 + 255) / 256), dim3(256), 0, st, oj)) != cudaSuccess)
+    if ((e = launch_pdl(k_fw_attn_out, dim3(L.Rp * F.Hq), dim3(256), 0, st, oj)) != cudaSuccess)
       return e;
     if ((e = gemm(W.wo, D, D, X, F.R, L.Rp, L.sp_o, part, status, st)) != cudaSuccess) return e;
     // H += o Wo^T; X = bf16(RMSNorm(H) * ln2)
