@@ -526,8 +526,14 @@ def run_ours(args):
         # read once per question
         k1_avg_s = statistics.mean(fw["ms"]) / 1e3
         alg_bytes = fw["bytes"]
-        kernel = "question forward (k_fw_norm, k_fw_gemm, k_fw_qkv, k_fw_attn, k_fw_attn_out, k_fw_swiglu)"
-        launches += 2 + 10 * w.n_layers   # RoPE table, final residual, 10 per layer
+        # per layer: 2 norms, 4 projections, q/k/v, attention, merge, and SwiGLU unless the
+        # gate/up projection runs as one K split (2 I / 128 tiles above two per SM) and
+        # applies it in its epilogue
+        sms = torch.cuda.get_device_properties(dev).multi_processor_count
+        fused = (2 * sms) // (2 * fwd_I // 128) <= 1
+        kernel = ("question forward (k_fw_norm_row, k_fw_gemm, k_fw_qkv, k_fw_attn, "
+                  "k_fw_attn_out" + ("" if fused else ", k_fw_swiglu") + ")")
+        launches += 2 + (9 if fused else 10) * w.n_layers   # RoPE table, final residual
         achieved = alg_bytes / k1_avg_s / 1e9
     traffic = recorded_traffic(w) if not args.frames and n_streams == 1 and fw is None else None
     if roof is None:
