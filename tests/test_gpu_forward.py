@@ -271,6 +271,27 @@ def test_three_layers_and_the_retrieval_of_their_query_rows():
     print(info)
 
 
+def test_wide_model_norm_in_column_chunks():
+    """Hq 42 (D 5376, more columns than one CTA's threads take four at a time): the RMSNorm
+    runs in column chunks with a per-row arrival count instead of one CTA per row."""
+    ss = _ss()
+    P, F, Tf, R, Hkv = 1, 5, 32, 4, 6
+    w, keys, vals, layers, h_in = _case(P, F, Tf, R, 256, seed=17, Hkv=Hkv)
+    Hq = Hkv * 7
+    layers[0]["ln1"] = torch.ones_like(layers[0]["ln1"])
+    h_in = _exact_norm_rows(R, Hq * 128, seed=17)
+    idx = ss.Index(P, Hq, Hkv, Tf, F, device=torch.device("cuda"))
+    idx.append(keys.cuda())
+    idx.append_values(vals.cuda())
+    params = ss.ForwardParams(256, EXACT_EPS)
+    qb, h = _run(idx, layers, h_in, params)
+    ref = FW.forward(to_bits(h_in), _np_weights(layers), to_bits(keys), to_bits(vals),
+                     n_q_heads=Hq, n_kv_heads=Hkv, eps=EXACT_EPS)
+    _check_q(qb[0], ref["layers"][0]["q_pre"],
+             _q_scale(ref["layers"][0], _np_weights(layers)[0], Hq))
+    assert np.linalg.norm(h - ref["h"]) / np.linalg.norm(ref["h"]) <= 2e-2
+
+
 def test_bias_none_explicit_position_and_repeatability():
     ss = _ss()
     w, keys, vals, layers, h_in = _case(2, 9, 64, 7, 256, seed=5)
