@@ -275,6 +275,42 @@ __global__ void __launch_bounds__(256) k_mass_general(const __grid_constant__ Ba
   if (tid == 0) P.mass[u] = acc;
 }
 
+// The same for rows of weights (one list per layer, or the row-averaged lists) when every
+// unit's segment is 16-byte aligned (tokens per unit a multiple of 4; rows start on
+// 64-value boundaries): 16-byte loads, eight per thread in flight, summed in a fixed order.
+__global__ void __launch_bounds__(256) k_mass_rows(const __grid_constant__ Batch B) {
+  __shared__ float sm[32];
+  pdl_wait();
+  pdl_release();
+  const int pi = blockIdx.y;
+  if (pi >= B.n) return;
+  const Prob& P = B.p[pi];
+  const int u = blockIdx.x;
+  if (u >= P.Uh) return;
+  const int Tu = P.Tu, tid = threadIdx.x;
+  const float* rows = B.head_agg == 1 ? P.aval : P.cand_s;
+  const int nL = B.head_agg == 1 ? P.P : P.P * P.Hq;
+  const int n4 = Tu >> 2, items = nL * n4;
+  float acc = 0.f;
+  for (int t0 = tid; t0 < items; t0 += 8 * (int)blockDim.x) {
+    float4 v[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const int t = t0 + q * blockDim.x;
+      v[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (t < items) {
+        const int L = t / n4, g = t - L * n4;
+        v[q] = *reinterpret_cast<const float4*>(rows + (int64_t)L * P.cand_cap +
+                                                (int64_t)u * Tu + 4 * g);
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < 8; ++q) acc += (v[q].x + v[q].y) + (v[q].z + v[q].w);
+  }
+  acc = block_sum(acc, sm);
+  if (tid == 0) P.mass[u] = acc;
+}
+
 cudaError_t launch_general_score(const Batch& B, int max_cand, int max_slabs,
                                  int max_score_lists, cudaStream_t s) {
   cudaError_t e;
@@ -305,7 +341,10 @@ cudaError_t launch_mass_general(const Batch& B, int max_cent, int max_slabs,
     if (e != cudaSuccess) return e;
   }
   if (max_hist_units <= 0) return cudaSuccess;
-  return launch_pdl(k_mass_general, dim3(max_hist_units, B.n), dim3(256), 0, s, B);
+  bool rows = (B.head_agg == 1 || B.q_agg == 2) && !B.use_clusters;
+  for (int j = 0; j < B.n && rows; ++j) rows = B.p[j].Tu % 4 == 0;
+  return rows ? launch_pdl(k_mass_rows, dim3(max_hist_units, B.n), dim3(256), 0, s, B)
+              : launch_pdl(k_mass_general, dim3(max_hist_units, B.n), dim3(256), 0, s, B);
 }
 
 }  // namespace ss

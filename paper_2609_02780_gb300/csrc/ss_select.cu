@@ -316,20 +316,43 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
     if constexpr (kGeneral) return mean ? (int32_t)x : ci[x];
     else return __float_as_int(cp[x].y);
   };
-  // Visits every candidate x < cnt with its value: thread t takes x = t, t + T, ... in
-  // increasing order, loading four values before using them (loads in flight).
+  // Visits every candidate x < cnt with its value. A dense row of weights (16-byte
+  // aligned, its capacity a multiple of 64) is read in 16-byte loads, eight per thread in
+  // flight: thread t takes the groups of four x = 4 g .. 4 g + 3 for g = t, t + T, ...;
+  // other rows and the score kernel's candidate lists one value at a time, four in flight.
   auto each = [&](auto&& f) {
-    for (int x0 = tid; x0 < cnt; x0 += 4 * (int)blockDim.x) {
-      float v[4];
+    if (kGeneral && mean) {
+      const float4* c4 = reinterpret_cast<const float4*>(cs);
+      const int n4 = (cnt + 3) >> 2;
+      for (int g0 = tid; g0 < n4; g0 += 8 * (int)blockDim.x) {
+        float4 v[8];
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int x = x0 + e * blockDim.x;
-        v[e] = x < cnt ? sc_at(x) : 0.f;
+        for (int u = 0; u < 8; ++u) {
+          const int g = g0 + u * blockDim.x;
+          v[u] = g < n4 ? c4[g] : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int x = 4 * (g0 + u * (int)blockDim.x);
+          if (x < cnt) f(x, v[u].x);
+          if (x + 1 < cnt) f(x + 1, v[u].y);
+          if (x + 2 < cnt) f(x + 2, v[u].z);
+          if (x + 3 < cnt) f(x + 3, v[u].w);
+        }
       }
+    } else {
+      for (int x0 = tid; x0 < cnt; x0 += 4 * (int)blockDim.x) {
+        float v[4];
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int x = x0 + e * blockDim.x;
-        if (x < cnt) f(x, v[e]);
+        for (int e = 0; e < 4; ++e) {
+          const int x = x0 + e * blockDim.x;
+          v[e] = x < cnt ? sc_at(x) : 0.f;
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int x = x0 + e * blockDim.x;
+          if (x < cnt) f(x, v[e]);
+        }
       }
     }
   };
