@@ -356,11 +356,30 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
       }
     }
   };
+  // A dense row of weights (values in [0, 1]) also gets its histogram in the same pass:
+  // 32 bins per octave from the value's bits (exactly monotonic in the value), the top bin
+  // holding [2^-1/32 .. 1], bin 0 everything below 2^-64.
+  const bool wbins = kGeneral && mean && cnt > 2 * kThreads;
+  auto wbin = [](float v) -> int {
+    const int b = (int)(__float_as_uint(fmaxf(v, 0.f)) >> 18) - (63 << 5);
+    return min(max(b, 0), kFineBins - 1);
+  };
   if constexpr (kGeneral) {
     // statistics of the dense row in a fixed order: (max, sum 2^(s - max)) of the
     // scores, or (max, sum) of the head-averaged weights; and its minimum (the bound)
     float m = -INFINITY, l = 0.f, mn = INFINITY;
-    if (mean) {
+    if (wbins) {
+      for (int x = tid; x < kFineBins; x += blockDim.x) s_hist[x] = 0;
+      __syncthreads();
+      each([&](int, float v) {
+        m = fmaxf(m, v);
+        l += v;
+        mn = fminf(mn, v);
+        atomicAdd(&s_hist[wbin(v)], 1);
+      });
+      l = block_sum(l, s_l);
+      m = -block_min(-m, s_m);
+    } else if (mean) {
       each([&](int, float v) {
         m = fmaxf(m, v);
         l += v;
@@ -486,19 +505,24 @@ __global__ void __launch_bounds__(kThreads, 1024 / kThreads) k_select_t(const __
   __syncthreads();
   int ns = dense ? kSelCap + 1 : s_n;
   if (ns > kSelCap) {
-    // Too many: a 2048-bin histogram of the candidates over [lo, max] locates the bin
-    // of the n-th best; keep the candidates from that bin up.
+    // Too many: a 2048-bin histogram of the candidates over [lo, max] (linear) locates the
+    // bin of the n-th best; keep the candidates from that bin up.
+    // (a dense row of weights has its histogram from the statistics pass, in the bins
+    // of the value's bits)
     const float hi = M;
     const float scale = (hi > lo) ? (float)kFineBins / (hi - lo) : 0.f;
     auto fbin = [&](float s) -> int {
+      if (wbins) return wbin(s);
       const int b = (int)((s - lo) * scale);
       return min(max(b, 0), kFineBins - 1);
     };
-    for (int x = tid; x < kFineBins; x += blockDim.x) s_hist[x] = 0;
-    __syncthreads();
-    each([&](int, float s) {
-      if (s >= lo) atomicAdd(&s_hist[fbin(s)], 1);
-    });
+    if (!wbins) {
+      for (int x = tid; x < kFineBins; x += blockDim.x) s_hist[x] = 0;
+      __syncthreads();
+      each([&](int, float s) {
+        if (s >= lo) atomicAdd(&s_hist[fbin(s)], 1);
+      });
+    }
     __syncthreads();
     if (tid < 32) {
       constexpr int per = kFineBins / 32;  // lane 0 holds the top bins
