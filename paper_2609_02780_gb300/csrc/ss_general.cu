@@ -251,14 +251,34 @@ __global__ void __launch_bounds__(256) k_mass_general(const __grid_constant__ Ba
       const int x = u - P.win_u0[w];
       const int n_c = P.n_c;
       int vs = 0;
-      for (int t = tid; t < P.P * P.Hkv * n_c; t += blockDim.x) {
-        const int slab = t / n_c, c = t - slab * n_c;
-        const int64_t wc = ((int64_t)slab * P.wcap + w) * n_c + c;
-        const int m = P.mcnt[wc * P.wu + x];
-        if (m) {
-          acc += P.cw[wc] * (float)m / (float)P.msize[wc];
-          vs += P.csel[wc] * m;
+      // four (slab, centroid) items per thread at a time: their member counts, weights,
+      // sizes and selection counts loaded together, then added in item order
+      const int items = P.P * P.Hkv * n_c;
+      for (int t0 = tid; t0 < items; t0 += 4 * (int)blockDim.x) {
+        int m[4], sz[4], cs[4];
+        float cwv[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int t = t0 + q * blockDim.x;
+          m[q] = 0;
+          sz[q] = 1;
+          cs[q] = 0;
+          cwv[q] = 0.f;
+          if (t < items) {
+            const int slab = t / n_c, c = t - slab * n_c;
+            const int64_t wc = ((int64_t)slab * P.wcap + w) * n_c + c;
+            m[q] = P.mcnt[wc * P.wu + x];
+            cwv[q] = P.cw[wc];
+            sz[q] = P.msize[wc];
+            cs[q] = P.csel[wc];
+          }
         }
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          if (m[q]) {
+            acc += cwv[q] * (float)m[q] / (float)sz[q];
+            vs += cs[q] * m[q];
+          }
       }
       // integer block sum (exact in any order)
       __shared__ int svs;
