@@ -196,12 +196,20 @@ __global__ void __launch_bounds__(256) k_centroid_weight(const __grid_constant__
   if (e >= P.n_cand - P.n_raw_tok) return;
   const int i = slab / P.Hkv, gk = slab - i * P.Hkv;
   const int list0 = i * P.Hq + gk * P.G;
+  // the group's (at most kMaxGroup) scores and statistics loaded together, summed in head
+  // order
+  float2 ml[kMaxGroup];
+  float sv[kMaxGroup];
+#pragma unroll
+  for (int h = 0; h < kMaxGroup; ++h)
+    if (h < P.G) {
+      ml[h] = P.list_ml[list0 + h];
+      sv[h] = P.cand_s[(int64_t)(list0 + h) * P.cand_cap + P.n_raw_tok + e];
+    }
   float a = 0.f;
-  for (int h = 0; h < P.G; ++h) {
-    const float2 ml = P.list_ml[list0 + h];
-    a += fast_exp2(P.cand_s[(int64_t)(list0 + h) * P.cand_cap + P.n_raw_tok + e] - ml.x) *
-         (1.0f / ml.y);
-  }
+#pragma unroll
+  for (int h = 0; h < kMaxGroup; ++h)
+    if (h < P.G) a += fast_exp2(sv[h] - ml[h].x) * (1.0f / ml[h].y);
   P.cw[(int64_t)slab * P.wcap * P.n_c + e] = a;
 }
 
