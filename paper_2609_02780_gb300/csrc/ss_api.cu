@@ -174,7 +174,7 @@ Layout layout_of(const ss_index* ix, int R, const ss_retrieve_params* p) {
   l.ladder = take(score_lists * kLadderLevels * 4);
   l.samp_max = take(score_lists * kSampleUnits * 4);
   l.ustats = take(score_lists * ix->ucap * 8);
-  l.next_unit = take((int64_t)c.n_layers * c.n_kv_heads * 4);
+  l.next_unit = take((int64_t)c.n_layers * c.n_kv_heads * kUnitCounterStride * 4);
   l.gram = take(pc * (pc + 1) / 2 * 4 + 4 * kMaxPool);  // + the greedy's reads past the end
   l.topk_tok = take(n_lists * p->k * 4);
   l.topk_w = take(n_lists * p->k * 4);

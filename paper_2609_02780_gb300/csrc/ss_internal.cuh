@@ -61,6 +61,8 @@ constexpr int kSampleUnits = 4;        // history units scored for the ladder an
 // Candidate slots a warp reserves per list at a time (no atomic per append).
 constexpr int kReserve = 64;
 constexpr int kMaxChunksPerSlab = 128;
+// Words between two slabs' unit counters of the score kernel (one 128-byte line each).
+constexpr int kUnitCounterStride = 32;
 
 // Device status word bits (ss_result::status).
 constexpr uint32_t kStatusInternal = 1u;
@@ -97,7 +99,8 @@ struct Prob {
   float* samp_max;             // [n_score_lists][kSampleUnits] maxima of the sampled units
   int n_sample;                // sampled units Z (0..kSampleUnits)
   float2* ustats;              // [n_score_lists][ucap] per-unit (max, sum 2^(s-max))
-  int32_t* next_unit;          // [P*Hkv] next history unit to score in each slab
+  int32_t* next_unit;          // [P*Hkv][kUnitCounterStride] next history unit to score
+                               // in each slab (word 0 of each line)
   float* gram;                 // packed upper triangle of the pool's Gram matrix
   // outputs
   int32_t* topk_tok;           // [n_lists][k]

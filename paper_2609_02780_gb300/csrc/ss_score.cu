@@ -97,7 +97,7 @@ __global__ void __launch_bounds__(256) k_sample(const __grid_constant__ Batch B)
     }
     for (int x = tid; x < G * kLadderLevels; x += blockDim.x)
       P.ladder[(int64_t)list0 * kLadderLevels + x] = 0;
-    if (tid == 0) P.next_unit[slab] = P.chunks * kScoreWarps;  // past the fixed first units
+    if (tid == 0) P.next_unit[slab * kUnitCounterStride] = P.chunks * kScoreWarps;  // past the fixed first units
     for (int v = slab * blockDim.x + tid; v < P.ucap; v += n_slabs * blockDim.x) P.votes[v] = 0;
     if (slab == 0 && tid < 4) P.counts[tid] = 0;
     // a compression whose wait gave up is reported by every later retrieval
@@ -325,9 +325,11 @@ __device__ __noinline__ void threshold_warp(ScoreShared& S, const Prob& P, int l
         const int f = __ffs(hit) - 1;
         const int lv = kLadderLevels - 1 - (32 * qf + f);
         t = S.anchor[c] + (float)(lv - kLadderZero - 1) / kLadderPerUnit;
-        if (lane == 0) atomicMax(P.gthr + list0 + c, float_to_ordered(t));  // not waited for
       }
+      // published only when it raises the bound seen in gthr (the lists' words share a
+      // few cache lines, which every CTA of the grid polls)
       const float other = __shfl_sync(0xffffffffu, pub, c);
+      if (lane == 0 && t > other) atomicMax(P.gthr + list0 + c, float_to_ordered(t));  // not waited for
       t = fmaxf(t, other);
       if (lane == 0 && t > vthr[c]) vthr[c] = t;
     }
@@ -437,7 +439,7 @@ __global__ void __launch_bounds__(kScoreThreads, kScoreCtasPerSm)
   const int c0 = 2 * t4, c1 = 2 * t4 + 1;
   const bool hv0 = c0 < G, hv1 = c1 < G;
   const int L0 = list0 + c0, L1 = list0 + c1;
-  int* next_unit = P.next_unit + slab;
+  int* next_unit = P.next_unit + slab * kUnitCounterStride;
   const int64_t cbase0 = (int64_t)(hv0 ? L0 : list0) * P.cand_cap;
   const int64_t cbase1 = (int64_t)(hv1 ? L1 : list0) * P.cand_cap;
   const volatile float* vthr = S.thr;
