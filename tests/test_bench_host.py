@@ -1,5 +1,6 @@
-"""Host-side pieces of bench.py that need no GPU: the clock record of the timed region
-and the byte count of what the host call's kernels write into host memory."""
+"""Host-side pieces of bench.py that need no GPU: the clock record of the timed region,
+the byte count of what the host call's kernels write into host memory, and the CPU
+baseline's repetitions of its sample."""
 import datetime
 import os
 import sys
@@ -40,3 +41,17 @@ def test_host_copy_bytes_count_what_the_kernels_write_to_host_memory():
     # hour1: K = 64, n_prev = 1, one frame per unit: ids, expansion, frames, counts, status
     assert bench.host_copy_bytes(64, 128, 1) == 256 + 512 + 512 + 16 + 4
     assert bench.host_copy_bytes(1, 2, 2) == 4 + 8 + 16 + 16 + 4
+
+
+def test_cpu_baseline_repeats_its_sample_for_the_set_cpu_time(monkeypatch):
+    import bench
+    from paper_2609_02780_gb300 import synth
+    w = synth.PRESETS["tiny"].replace(n_frames=8, n_planted=1)
+    data = synth.make_workload(w, device="cpu")
+    monkeypatch.setattr(bench, "CPU_BASELINE_SECONDS", 0.2)
+    b = bench.cpu_baseline(w, data["keys"], data["q"], frames=8)
+    keys = w.n_slabs * 8 * w.tokens_per_frame
+    assert b["repetitions"] >= 1 and b["seconds"] >= 0.2
+    # `seconds` is rounded to the millisecond
+    assert abs(b["value"] - keys * b["repetitions"] / b["seconds"]) <= 1e-2 * b["value"]
+    assert f"{b['repetitions']} times" in b["sample"] and b["kind"] == "oracle"
